@@ -1,0 +1,261 @@
+"""Float64 CPU oracle of the GRPO hot path (test infrastructure).
+
+Test infrastructure only: ``tests/``, ``__graft_entry__.smoke()`` and the CPU
+baseline leg of ``bench.py`` may import it; the library never does and shares
+no code with it.
+
+What it computes, in the paper's notation (Section 3.3):
+
+* Eq. 2, the group-relative advantage
+      A_i = (r_i - mean_j r_j) / (std_j r_j + eps)
+  over the G responses of one prompt (readings: the N of Eq. 2 is the group
+  size G; std is the sample std, ddof = 1; eps = 1e-6 keeps a zero-std group
+  at A = 0), broadcast to every token of response i.
+* pi_theta(o_{i,t} | q, o_{i,<t}) inside Eq. 1: the log-softmax of the LM-head
+  logits z_t = H_t W^T (temperature 1), taken at the sampled token y_t.
+* the braces of Eq. 1 per token:  rho = pi_theta / pi_old = exp(logp - old),
+      s = min(rho A, clip(rho, 1-eps_c, 1+eps_c) A)
+      KL = exp(ref - logp) - (ref - logp) - 1     (per-token k3 estimator of
+           D_KL(pi_theta || pi_ref) from the GRPO paper the method cites)
+      l = -(s - beta KL)                          (loss = -J)
+* the aggregation of Eq. 1: agg_mode 1 is Eq. 1 as printed,
+      (1/n_resp) sum_i (1/|o_i|) sum_t l_{i,t};
+  agg_mode 0 (default) is the masked token-mean sum_t mask_t l_t / N_valid.
+* the gradient of that loss to H and W: with g_t = dloss/dlogp_t,
+      dZ_{t,v} = g_t (1[v = y_t] - p_{t,v}),  dH = dZ W,  dW = dZ^T H.
+  At the kink of min() (rho A == clip(rho) A) the unclipped branch is taken.
+
+Rows with mask 0 have logp = 0, weight 0, and zero dH rows.
+Every floating value is float64; bf16 inputs are widened exactly.
+"""
+from __future__ import annotations
+
+import numpy as np
+
+# ---------------------------------------------------------------------------
+# inputs
+# ---------------------------------------------------------------------------
+
+
+def widen_bf16(bits: np.ndarray) -> np.ndarray:
+    """bf16 bit patterns (uint16) -> float64, exactly (a bf16 is the top half of an f32)."""
+    b = np.ascontiguousarray(bits, dtype=np.uint16)
+    return (b.astype(np.uint32) << np.uint32(16)).view(np.float32).astype(np.float64)
+
+
+def as_f64(x) -> np.ndarray:
+    """Float64 view of a float array, or exact widening of bf16 bits given as uint16."""
+    x = np.asarray(x)
+    if x.dtype == np.uint16:
+        return widen_bf16(x)
+    return x.astype(np.float64)
+
+
+# ---------------------------------------------------------------------------
+# Eq. 2: group-relative advantage
+# ---------------------------------------------------------------------------
+
+
+def group_advantages(rewards, G: int, eps: float = 1e-6, ddof: int = 1) -> np.ndarray:
+    """Eq. 2 per group of G consecutive responses; float64 math, rounded once to float32."""
+    r = np.asarray(rewards, dtype=np.float64)
+    if G < 2 or r.size % G:
+        raise ValueError("need G >= 2 and n_resp % G == 0")
+    g = r.reshape(-1, G)
+    mu = g.mean(axis=1, keepdims=True)
+    sd = g.std(axis=1, ddof=ddof, keepdims=True)
+    return ((g - mu) / (sd + eps)).reshape(-1).astype(np.float32)
+
+
+# ---------------------------------------------------------------------------
+# pi_theta(o_t | ...): log-softmax over the vocabulary at the sampled token
+# ---------------------------------------------------------------------------
+
+
+def token_logprobs(H, W, targets, mask, vocab_chunk: int = 8192, row_chunk: int = 4096):
+    """log softmax(H_t W^T)[y_t] for unmasked rows.
+
+    Returns (logp [T], lse [T]) in float64; masked rows are 0.  The logits are
+    formed chunk by chunk over the vocabulary, with a running max and a running
+    sum of exp(z - max) per row, so the [T, V] matrix is never held at once.
+    """
+    H = np.asarray(H)
+    W = as_f64(W)
+    y = np.asarray(targets, dtype=np.int64)
+    m = np.asarray(mask) != 0
+    T, V = H.shape[0], W.shape[0]
+    logp = np.zeros(T, dtype=np.float64)
+    lse = np.zeros(T, dtype=np.float64)
+    idx = np.flatnonzero(m)
+    for r0 in range(0, idx.size, row_chunk):
+        rows = idx[r0:r0 + row_chunk]
+        Hr = as_f64(H[rows])
+        yr = y[rows]
+        run_max = np.full(rows.size, -np.inf)
+        run_sum = np.zeros(rows.size)
+        zy = np.zeros(rows.size)
+        for v0 in range(0, V, vocab_chunk):
+            v1 = min(V, v0 + vocab_chunk)
+            Z = Hr @ W[v0:v1].T
+            new_max = np.maximum(run_max, Z.max(axis=1))
+            run_sum = run_sum * np.exp(run_max - new_max) + np.exp(Z - new_max[:, None]).sum(axis=1)
+            run_max = new_max
+            hit = (yr >= v0) & (yr < v1)
+            zy[hit] = Z[np.flatnonzero(hit), yr[hit] - v0]
+        l = run_max + np.log(run_sum)
+        lse[rows] = l
+        logp[rows] = zy - l
+    return logp, lse
+
+
+# ---------------------------------------------------------------------------
+# Eq. 1: per-token terms, weights, loss and its derivative in logp
+# ---------------------------------------------------------------------------
+
+
+def token_advantages(adv, n_resp: int, L: int) -> np.ndarray:
+    """A_{i,t} = A_i for every padded row of response i (Eq. 2 broadcast)."""
+    a = np.asarray(adv, dtype=np.float64)
+    assert a.size == n_resp
+    return np.repeat(a, L)
+
+
+def token_terms(logp, old_logp, ref_logp, adv_tok, clip_eps: float, beta: float):
+    """The braces of Eq. 1 for every row.
+
+    Returns a dict with rho, the clipped-surrogate value s, the k3 KL, the
+    per-token loss l = -s + beta KL and the 0/1 flag 'unclipped' (the min()
+    picks rho A; ties count as unclipped).
+    """
+    lp = np.asarray(logp, dtype=np.float64)
+    old = np.asarray(old_logp, dtype=np.float64)
+    ref = np.asarray(ref_logp, dtype=np.float64)
+    A = np.asarray(adv_tok, dtype=np.float64)
+    rho = np.exp(lp - old)
+    s1 = rho * A
+    s2 = np.clip(rho, 1.0 - clip_eps, 1.0 + clip_eps) * A
+    unclipped = s1 <= s2
+    s = np.where(unclipped, s1, s2)
+    d = ref - lp
+    kl = np.exp(d) - d - 1.0
+    return {"rho": rho, "s": s, "kl": kl, "ell": -s + beta * kl, "unclipped": unclipped}
+
+
+def token_weights(mask, n_resp: int, L: int, agg_mode: int = 0) -> np.ndarray:
+    """w_t so that loss = sum_t w_t l_t.
+
+    agg_mode 0: mask_t / N_valid (token-mean; 0 when N_valid = 0).
+    agg_mode 1: mask_t / (n_resp |o_i|), Eq. 1's per-response mean then mean
+    over responses (a response with |o_i| = 0 contributes nothing).
+    """
+    m = (np.asarray(mask) != 0).astype(np.float64)
+    if agg_mode == 0:
+        n = m.sum()
+        return m / n if n > 0 else np.zeros_like(m)
+    if agg_mode == 1:
+        lens = m.reshape(n_resp, L).sum(axis=1)
+        inv = np.where(lens > 0, 1.0 / np.maximum(lens, 1.0), 0.0) / n_resp
+        return m * np.repeat(inv, L)
+    raise ValueError(agg_mode)
+
+
+def logp_coef(logp, old_logp, ref_logp, adv_tok, w, clip_eps: float, beta: float) -> np.ndarray:
+    """g_t = dloss/dlogp_t = w_t (-A rho 1[unclipped] + beta (1 - exp(ref - logp)))."""
+    tt = token_terms(logp, old_logp, ref_logp, adv_tok, clip_eps, beta)
+    lp = np.asarray(logp, dtype=np.float64)
+    ref = np.asarray(ref_logp, dtype=np.float64)
+    A = np.asarray(adv_tok, dtype=np.float64)
+    dsurr = np.where(tt["unclipped"], A * tt["rho"], 0.0)
+    dkl = 1.0 - np.exp(ref - lp)
+    return np.asarray(w, dtype=np.float64) * (-dsurr + beta * dkl)
+
+
+def grpo_loss(logp, old_logp, ref_logp, adv, mask, n_resp: int, L: int,
+              clip_eps: float, beta: float, agg_mode: int = 0):
+    """Eq. 1 negated, from per-token log-probs. Returns (loss, g, per-token dict)."""
+    A = token_advantages(adv, n_resp, L)
+    w = token_weights(mask, n_resp, L, agg_mode)
+    tt = token_terms(logp, old_logp, ref_logp, A, clip_eps, beta)
+    m = np.asarray(mask) != 0
+    loss = float(np.sum(w[m] * tt["ell"][m]))
+    g = logp_coef(logp, old_logp, ref_logp, A, w, clip_eps, beta)
+    g[~m] = 0.0
+    tt["w"] = w
+    return loss, g, tt
+
+
+# ---------------------------------------------------------------------------
+# backward through the LM head
+# ---------------------------------------------------------------------------
+
+
+def loss_fwd_bwd(H, W, targets, mask, old_logp, ref_logp, adv, n_resp: int, L: int,
+                 clip_eps: float, beta: float, agg_mode: int = 0, vocab_chunk: int = 8192):
+    """Full forward + backward: returns dict(loss, dH [T,Hd], dW [V,Hd], logp, lse, g)."""
+    Hf = as_f64(H)
+    Wf = as_f64(W)
+    y = np.asarray(targets, dtype=np.int64)
+    m = np.asarray(mask) != 0
+    logp, lse = token_logprobs(Hf, Wf, y, m, vocab_chunk=vocab_chunk)
+    loss, g, tt = grpo_loss(logp, old_logp, ref_logp, adv, m, n_resp, L, clip_eps, beta, agg_mode)
+    T, Hd = Hf.shape
+    V = Wf.shape[0]
+    dH = np.zeros((T, Hd))
+    dW = np.zeros((V, Hd))
+    idx = np.flatnonzero(m)
+    if idx.size:
+        Hv = Hf[idx]
+        gv = g[idx]
+        lv = lse[idx]
+        yv = y[idx]
+        dHv = np.zeros((idx.size, Hd))
+        for v0 in range(0, V, vocab_chunk):
+            v1 = min(V, v0 + vocab_chunk)
+            Z = Hv @ Wf[v0:v1].T
+            dZ = -gv[:, None] * np.exp(Z - lv[:, None])
+            hit = np.flatnonzero((yv >= v0) & (yv < v1))
+            dZ[hit, yv[hit] - v0] += gv[hit]
+            dHv += dZ @ Wf[v0:v1]
+            dW[v0:v1] = dZ.T @ Hv
+        dH[idx] = dHv
+    return {"loss": loss, "dH": dH, "dW": dW, "logp": logp, "lse": lse, "g": g, "terms": tt}
+
+
+def dH_rows(H, W, targets, lse, g, rows, vocab_chunk: int = 8192) -> np.ndarray:
+    """dH_t = g_t (W_{y_t} - sum_v p_{t,v} W_v) for the listed rows (any size)."""
+    rows = np.asarray(rows, dtype=np.int64)
+    Hf = as_f64(np.asarray(H)[rows])
+    Wsrc = np.asarray(W)
+    V = Wsrc.shape[0]
+    y = np.asarray(targets, dtype=np.int64)[rows]
+    l = np.asarray(lse, dtype=np.float64)[rows]
+    gg = np.asarray(g, dtype=np.float64)[rows]
+    acc = np.zeros((rows.size, Hf.shape[1]))
+    for v0 in range(0, V, vocab_chunk):
+        v1 = min(V, v0 + vocab_chunk)
+        Wc = as_f64(Wsrc[v0:v1])
+        P = np.exp(Hf @ Wc.T - l[:, None])
+        acc += P @ Wc
+    Wy = as_f64(Wsrc[y])
+    return gg[:, None] * (Wy - acc)
+
+
+def dW_rows(H, W, targets, mask, lse, g, vrows, row_chunk: int = 8192) -> np.ndarray:
+    """dW_v = sum_t g_t (1[y_t = v] - p_{t,v}) H_t for the listed vocabulary rows (any size)."""
+    vrows = np.asarray(vrows, dtype=np.int64)
+    Wv = as_f64(np.asarray(W)[vrows])
+    m = np.asarray(mask) != 0
+    idx = np.flatnonzero(m)
+    y = np.asarray(targets, dtype=np.int64)
+    out = np.zeros((vrows.size, Wv.shape[1]))
+    for r0 in range(0, idx.size, row_chunk):
+        rows = idx[r0:r0 + row_chunk]
+        Hr = as_f64(np.asarray(H)[rows])
+        gr = np.asarray(g, dtype=np.float64)[rows]
+        lr = np.asarray(lse, dtype=np.float64)[rows]
+        P = np.exp(Hr @ Wv.T - lr[:, None])           # [rows, |vrows|]
+        dZ = -gr[:, None] * P
+        hit = y[rows][:, None] == vrows[None, :]
+        dZ += hit * gr[:, None]
+        out += dZ.T @ Hr
+    return out

@@ -1,0 +1,325 @@
+"""Pins of the float64 oracle against facts that do not come from the oracle itself.
+
+Each pin is a closed form, a brute-force loop, a library routine, an invariant
+or a finite-difference check of Eq. 1 / Eq. 2 (Section 3.3).  The last block
+plants plausible mistakes into a copy of the oracle and checks that a pin
+catches each one.
+"""
+import json
+import math
+import os
+import statistics
+
+import numpy as np
+import pytest
+import scipy.special
+
+import oracle
+from oracle import brute
+from oracle import grpo_oracle as go
+
+HERE = os.path.dirname(os.path.abspath(__file__))
+
+
+def _rand_case(seed, T_resp=3, G=2, L=4, Hd=5, V=7, scale=0.7, ragged=True):
+    """A tiny float64 case with ragged prefix masks and non-degenerate advantages."""
+    rng = np.random.default_rng(seed)
+    n_resp = T_resp * G if T_resp else G
+    T = n_resp * L
+    H = rng.normal(0, 1, (T, Hd))
+    W = rng.normal(0, scale, (V, Hd))
+    y = rng.integers(0, V, T)
+    lens = rng.integers(1, L + 1, n_resp) if ragged else np.full(n_resp, L)
+    mask = (np.arange(L)[None, :] < lens[:, None]).astype(np.uint8).reshape(-1)
+    r = np.tile(np.array([0.0, 1.0] * (G // 2) + [0.5] * (G % 2)), n_resp // G)
+    rng.shuffle(r)
+    return dict(H=H, W=W, y=y, mask=mask, rewards=r, n_resp=n_resp, L=L, G=G, rng=rng)
+
+
+def _old_ref(logp, rng, spread=(-0.6, -0.05, 0.07, 0.5)):
+    """old/ref log-probs at fixed offsets from logp, so rho sits well away from 1 +- eps."""
+    off_old = rng.choice(spread, size=logp.size)
+    off_ref = rng.normal(0, 0.3, size=logp.size)
+    return logp - off_old, logp + off_ref
+
+
+# ---------------------------------------------------------------------------
+# Eq. 2
+# ---------------------------------------------------------------------------
+
+def test_advantage_closed_forms():
+    fx = json.load(open(os.path.join(HERE, "golden", "advantage_closed_forms.json")))
+    for c in fx["cases"]:
+        got = oracle.group_advantages(np.array(c["rewards"], np.float32), c["G"], fx["eps"])
+        np.testing.assert_allclose(got, np.array(c["adv"], np.float32), rtol=0, atol=2e-7)
+        assert statistics.stdev(c["rewards"]) == pytest.approx(c["std"], abs=1e-15)
+        assert statistics.mean(c["rewards"]) == pytest.approx(c["mean"], abs=1e-15)
+
+
+def test_advantages_zero_mean_and_library_std():
+    rng = np.random.default_rng(3)
+    for G in (2, 3, 4, 8, 16, 64):
+        r = rng.random(G * 5).astype(np.float32)
+        a = oracle.group_advantages(r, G, eps=0.0).astype(np.float64).reshape(-1, G)
+        assert np.abs(a.sum(axis=1)).max() < 1e-5
+        # with eps = 0 every group has sample std exactly 1 after normalisation
+        for row in a:
+            assert statistics.stdev(row.tolist()) == pytest.approx(1.0, abs=1e-6)
+        # brute-force loop
+        bf = np.array(brute.advantages(r.tolist(), G), np.float32)
+        np.testing.assert_allclose(oracle.group_advantages(r, G), bf, rtol=0, atol=1e-6)
+
+
+def test_advantages_all_equal_group_is_zero_and_bad_group_rejected():
+    r = np.array([0.5] * 8 + [1, 0, 0, 0, 0, 0, 0, 0], np.float32)
+    a = oracle.group_advantages(r, 8)
+    assert np.all(a[:8] == 0.0)
+    with pytest.raises(ValueError):
+        oracle.group_advantages(r, 1)
+    with pytest.raises(ValueError):
+        oracle.group_advantages(r[:7], 4)
+
+
+# ---------------------------------------------------------------------------
+# pi_theta(o_t): log-softmax at the sampled token
+# ---------------------------------------------------------------------------
+
+def test_uniform_logits_give_minus_log_V():
+    rng = np.random.default_rng(0)
+    for V in (7, 4096, 10001):
+        T, Hd = 9, 16
+        H = rng.normal(size=(T, Hd))
+        y = rng.integers(0, V, T)
+        mask = np.ones(T, np.uint8)
+        logp, lse = oracle.token_logprobs(H, np.zeros((V, Hd)), y, mask, vocab_chunk=1000)
+        assert np.all(logp == -np.log(V)) or np.abs(logp + math.log(V)).max() < 1e-12
+        logp0, _ = oracle.token_logprobs(np.zeros((T, Hd)), rng.normal(size=(V, Hd)), y, mask)
+        assert np.abs(logp0 + math.log(V)).max() < 1e-12
+
+
+def test_logprobs_match_bruteforce_and_scipy():
+    c = _rand_case(1, T_resp=2, G=2, L=5, Hd=6, V=11, scale=1.5)
+    logp, lse = oracle.token_logprobs(c["H"], c["W"], c["y"], c["mask"], vocab_chunk=4)
+    bf = brute.logprobs(c["H"].tolist(), c["W"].tolist(), c["y"].tolist(), c["mask"].tolist())
+    np.testing.assert_allclose(logp, bf, rtol=0, atol=1e-12)
+    Z = c["H"] @ c["W"].T
+    ls = scipy.special.log_softmax(Z, axis=1)[np.arange(len(c["y"])), c["y"]]
+    m = c["mask"] != 0
+    np.testing.assert_allclose(logp[m], ls[m], rtol=0, atol=1e-12)
+    np.testing.assert_allclose(lse[m], scipy.special.logsumexp(Z, axis=1)[m], rtol=0, atol=1e-12)
+    assert np.all(logp[~m] == 0) and np.all(lse[~m] == 0)
+
+
+def test_logprobs_chunking_invariant_and_large_logits():
+    rng = np.random.default_rng(5)
+    H = rng.normal(size=(20, 8))
+    W = rng.normal(0, 30.0, size=(50, 8))   # logits in the hundreds: needs the max shift
+    y = rng.integers(0, 50, 20)
+    mask = np.ones(20, np.uint8)
+    a, _ = oracle.token_logprobs(H, W, y, mask, vocab_chunk=3, row_chunk=7)
+    b, _ = oracle.token_logprobs(H, W, y, mask, vocab_chunk=50)
+    np.testing.assert_allclose(a, b, rtol=0, atol=1e-9)
+    ls = scipy.special.log_softmax(H @ W.T, axis=1)[np.arange(20), y]
+    np.testing.assert_allclose(a, ls, rtol=0, atol=1e-9)
+
+
+def test_bf16_widening_is_exact():
+    bits = np.array([0x3F80, 0xBF80, 0x0000, 0x4049, 0x7F7F, 0x0001], np.uint16)
+    want = np.array([1.0, -1.0, 0.0, 3.140625, 3.3895313892515355e38, 9.183549615799121e-41])
+    np.testing.assert_array_equal(oracle.widen_bf16(bits), want)
+
+
+# ---------------------------------------------------------------------------
+# Eq. 1: ratio, clip, KL, aggregation
+# ---------------------------------------------------------------------------
+
+def test_ratio_one_and_kl_zero_closed_forms():
+    c = _rand_case(2, T_resp=2, G=4, L=6)
+    logp, _ = oracle.token_logprobs(c["H"], c["W"], c["y"], c["mask"])
+    adv = oracle.group_advantages(c["rewards"], c["G"])
+    A = oracle.token_advantages(adv, c["n_resp"], c["L"])
+    m = c["mask"] != 0
+    ref = logp + c["rng"].normal(0, 0.3, logp.size)
+    for agg in (0, 1):
+        w = oracle.token_weights(c["mask"], c["n_resp"], c["L"], agg)
+        # old = policy: rho = 1 -> loss = -sum w A + beta sum w KL
+        loss, _, tt = oracle.grpo_loss(logp, logp, ref, adv, c["mask"], c["n_resp"], c["L"], 0.2, 0.04, agg)
+        assert np.all(tt["rho"][m] == 1.0)
+        d = ref - logp
+        kl = np.exp(d) - d - 1
+        assert loss == pytest.approx(float(np.sum(w[m] * (-A[m] + 0.04 * kl[m]))), abs=1e-14)
+        # ref = policy too: KL = 0 -> loss = -sum w A
+        loss2, _, tt2 = oracle.grpo_loss(logp, logp, logp, adv, c["mask"], c["n_resp"], c["L"], 0.2, 0.04, agg)
+        assert np.all(tt2["kl"][m] == 0.0)
+        assert loss2 == pytest.approx(-float(np.sum(w[m] * A[m])), abs=1e-14)
+
+
+def test_token_mean_of_zero_mean_advantages_is_zero_for_equal_lengths():
+    c = _rand_case(4, T_resp=3, G=4, L=5, ragged=False)
+    logp, _ = oracle.token_logprobs(c["H"], c["W"], c["y"], c["mask"])
+    adv = oracle.group_advantages(c["rewards"], c["G"])
+    for agg in (0, 1):
+        loss, _, _ = oracle.grpo_loss(logp, logp, logp, adv, c["mask"], c["n_resp"], c["L"], 0.2, 0.04, agg)
+        assert abs(loss) < 1e-7  # float32 advantages sum to 0 up to rounding
+    w0 = oracle.token_weights(c["mask"], c["n_resp"], c["L"], 0)
+    w1 = oracle.token_weights(c["mask"], c["n_resp"], c["L"], 1)
+    np.testing.assert_allclose(w0, w1, rtol=1e-15)
+
+
+def test_kl_nonnegative_and_zero_only_at_equality():
+    rng = np.random.default_rng(7)
+    lp = rng.normal(-8, 2, 10000)
+    ref = lp + rng.normal(0, 1, lp.size)
+    tt = oracle.token_terms(lp, lp, ref, np.ones_like(lp), 0.2, 0.04)
+    assert np.all(tt["kl"] >= 0)
+    assert np.all(tt["kl"][np.abs(ref - lp) > 1e-3] > 0)
+    # second-order: KL ~ d^2/2 for small d = ref - logp
+    d = np.array([1e-3, -2e-3, 5e-4])
+    tt = oracle.token_terms(np.zeros(3), np.zeros(3), d, np.ones(3), 0.2, 0.04)
+    np.testing.assert_allclose(tt["kl"], d ** 2 / 2 + d ** 3 / 6, rtol=1e-3)
+
+
+def test_loss_matches_bruteforce_both_aggregations():
+    for seed in (11, 12, 13):
+        c = _rand_case(seed, T_resp=3, G=4, L=5)
+        logp, _ = oracle.token_logprobs(c["H"], c["W"], c["y"], c["mask"])
+        old, ref = _old_ref(logp, c["rng"])
+        adv = oracle.group_advantages(c["rewards"], c["G"])
+        for agg in (0, 1):
+            loss, _, _ = oracle.grpo_loss(logp, old, ref, adv, c["mask"], c["n_resp"], c["L"], 0.2, 0.04, agg)
+            bl = brute.loss(logp.tolist(), old.tolist(), ref.tolist(), adv.astype(float).tolist(),
+                            c["mask"].tolist(), c["n_resp"], c["L"], 0.2, 0.04, agg)
+            assert loss == pytest.approx(bl, rel=1e-12, abs=1e-15)
+
+
+def test_clip_zeroes_surrogate_gradient():
+    lp = np.zeros(4)
+    old = np.array([-0.5, 0.5, -0.5, 0.5])          # rho = e^0.5, e^-0.5, e^0.5, e^-0.5
+    A = np.array([1.0, -1.0, -1.0, 1.0])
+    g = oracle.logp_coef(lp, old, lp, A, np.ones(4), 0.2, 0.0)
+    # A > 0, rho > 1 + eps and A < 0, rho < 1 - eps: clipped, no gradient
+    assert g[0] == 0.0 and g[1] == 0.0
+    # the other two stay on the unclipped branch: g = -A rho
+    np.testing.assert_allclose(g[2:], [math.exp(0.5), -math.exp(-0.5)], rtol=1e-15)
+
+
+def test_textbook_policy_gradient_special_case():
+    c = _rand_case(21, T_resp=2, G=4, L=4)
+    logp, _ = oracle.token_logprobs(c["H"], c["W"], c["y"], c["mask"])
+    old, ref = _old_ref(logp, c["rng"])
+    adv = oracle.group_advantages(c["rewards"], c["G"])
+    A = oracle.token_advantages(adv, c["n_resp"], c["L"])
+    w = oracle.token_weights(c["mask"], c["n_resp"], c["L"], 0)
+    g = oracle.logp_coef(logp, old, ref, A, w, np.inf, 0.0)
+    np.testing.assert_allclose(g, -w * A * np.exp(logp - old), rtol=1e-15)
+
+
+# ---------------------------------------------------------------------------
+# gradients
+# ---------------------------------------------------------------------------
+
+def _loss_of(H, W, c, old, ref, adv, agg, clip=0.2, beta=0.04):
+    logp = brute.logprobs(H.tolist(), W.tolist(), c["y"].tolist(), c["mask"].tolist())
+    return brute.loss(logp, old.tolist(), ref.tolist(), adv.astype(float).tolist(),
+                      c["mask"].tolist(), c["n_resp"], c["L"], clip, beta, agg)
+
+
+@pytest.mark.parametrize("agg", [0, 1])
+def test_gradient_matches_central_differences(agg):
+    c = _rand_case(31, T_resp=2, G=2, L=3, Hd=4, V=6, scale=0.8)
+    logp, _ = oracle.token_logprobs(c["H"], c["W"], c["y"], c["mask"])
+    old, ref = _old_ref(logp, c["rng"])
+    adv = oracle.group_advantages(c["rewards"], c["G"])
+    out = oracle.loss_fwd_bwd(c["H"], c["W"], c["y"], c["mask"], old, ref, adv, c["n_resp"], c["L"],
+                              0.2, 0.04, agg, vocab_chunk=4)
+    h = 1e-6
+    for name, X, dX in (("H", c["H"], out["dH"]), ("W", c["W"], out["dW"])):
+        fd = np.zeros_like(X)
+        for i in range(X.shape[0]):
+            for j in range(X.shape[1]):
+                Xp = X.copy(); Xp[i, j] += h
+                Xm = X.copy(); Xm[i, j] -= h
+                args_p = (Xp, c["W"]) if name == "H" else (c["H"], Xp)
+                args_m = (Xm, c["W"]) if name == "H" else (c["H"], Xm)
+                fd[i, j] = (_loss_of(*args_p, c, old, ref, adv, agg) - _loss_of(*args_m, c, old, ref, adv, agg)) / (2 * h)
+        np.testing.assert_allclose(dX, fd, rtol=1e-5, atol=1e-9, err_msg=name)
+    assert np.all(out["dH"][c["mask"] == 0] == 0.0)
+
+
+def test_dW_column_sums_vanish_and_sampled_rows_match():
+    c = _rand_case(41, T_resp=3, G=4, L=6, Hd=8, V=23)
+    logp, _ = oracle.token_logprobs(c["H"], c["W"], c["y"], c["mask"])
+    old, ref = _old_ref(logp, c["rng"])
+    adv = oracle.group_advantages(c["rewards"], c["G"])
+    out = oracle.loss_fwd_bwd(c["H"], c["W"], c["y"], c["mask"], old, ref, adv, c["n_resp"], c["L"],
+                              0.2, 0.04, 0, vocab_chunk=5)
+    # sum_v dZ_{t,v} = 0 for every t, hence sum_v dW[v, :] = 0
+    assert np.abs(out["dW"].sum(axis=0)).max() < 1e-13
+    rows = np.flatnonzero(c["mask"])[::3]
+    np.testing.assert_allclose(oracle.dH_rows(c["H"], c["W"], c["y"], out["lse"], out["g"], rows, vocab_chunk=4),
+                               out["dH"][rows], rtol=1e-10, atol=1e-14)
+    vrows = np.array([0, 5, 22, int(c["y"][np.flatnonzero(c["mask"])[0]])])
+    np.testing.assert_allclose(oracle.dW_rows(c["H"], c["W"], c["y"], c["mask"], out["lse"], out["g"], vrows, row_chunk=5),
+                               out["dW"][vrows], rtol=1e-10, atol=1e-14)
+    # dH_t = g_t (W_{y_t} - E_p[W])
+    t = rows[0]
+    z = c["W"] @ c["H"][t]
+    p = np.exp(z - scipy.special.logsumexp(z))
+    np.testing.assert_allclose(out["dH"][t], out["g"][t] * (c["W"][c["y"][t]] - p @ c["W"]), rtol=1e-10)
+
+
+def test_all_masked_batch_is_zero():
+    c = _rand_case(51, T_resp=1, G=2, L=3)
+    mask = np.zeros_like(c["mask"])
+    zeros = np.zeros(mask.size)
+    adv = oracle.group_advantages(c["rewards"], c["G"])
+    out = oracle.loss_fwd_bwd(c["H"], c["W"], c["y"], mask, zeros, zeros, adv, c["n_resp"], c["L"], 0.2, 0.04)
+    assert out["loss"] == 0.0 and not out["dH"].any() and not out["dW"].any()
+
+
+# ---------------------------------------------------------------------------
+# planted mistakes: each must trip one of the pins above
+# ---------------------------------------------------------------------------
+
+def test_planted_population_std_is_caught(monkeypatch):
+    real = go.group_advantages
+    monkeypatch.setattr(go, "group_advantages", lambda r, G, eps=1e-6, ddof=1: real(r, G, eps, ddof=0))
+    monkeypatch.setattr(oracle, "group_advantages", go.group_advantages)
+    with pytest.raises(AssertionError):
+        test_advantage_closed_forms()
+
+
+def test_planted_kl_without_minus_one_is_caught(monkeypatch):
+    real = go.token_terms
+
+    def bad(logp, old, ref, A, clip_eps, beta):
+        tt = real(logp, old, ref, A, clip_eps, beta)
+        tt["kl"] = tt["kl"] + 1.0
+        tt["ell"] = -tt["s"] + beta * tt["kl"]
+        return tt
+    monkeypatch.setattr(go, "token_terms", bad)
+    monkeypatch.setattr(oracle, "token_terms", bad)
+    with pytest.raises(AssertionError):
+        test_ratio_one_and_kl_zero_closed_forms()
+
+
+def test_planted_target_off_by_one_is_caught(monkeypatch):
+    real = go.token_logprobs
+    monkeypatch.setattr(oracle, "token_logprobs",
+                        lambda H, W, y, m, **kw: real(H, W, (np.asarray(y) + 1) % np.asarray(W).shape[0], m, **kw))
+    with pytest.raises(AssertionError):
+        test_logprobs_match_bruteforce_and_scipy()
+
+
+def test_planted_gradient_sign_is_caught(monkeypatch):
+    real = go.logp_coef
+
+    def bad(logp, old, ref, A, w, clip_eps, beta):
+        lp = np.asarray(logp, np.float64)
+        tt = go.token_terms(logp, old, ref, A, clip_eps, beta)
+        dsurr = np.where(tt["unclipped"], np.asarray(A) * tt["rho"], 0.0)
+        return np.asarray(w) * (-dsurr - beta * (1.0 - np.exp(np.asarray(ref) - lp)))  # KL sign flipped
+    monkeypatch.setattr(go, "logp_coef", bad)
+    with pytest.raises(AssertionError):
+        test_gradient_matches_central_differences(0)
+    monkeypatch.setattr(go, "logp_coef", real)
