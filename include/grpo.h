@@ -1,0 +1,133 @@
+/*
+ * grpo.h — C ABI of the GB300 (sm_103a) GRPO hot-path library (libgrpo.so).
+ *
+ * The library computes the data-parallel part of a GRPO policy update
+ * (Section 3.3, Eq. 1 and Eq. 2): group-relative advantages, per-token
+ * log-probabilities of sampled tokens through the LM head, the clipped-ratio
+ * objective with a KL penalty, and the backward pass of that loss to the final
+ * hidden states H and the LM-head weight W.
+ *
+ * Conventions shared by every entry point
+ * ---------------------------------------
+ * - Every array pointer is a DEVICE pointer owned by the caller; the library
+ *   never frees or keeps it.  bf16 arrays are passed as their 16-bit patterns
+ *   (uint16_t).  All matrices are row-major and densely packed.
+ * - `stream` is a cudaStream_t (NULL = legacy default stream).  Work is
+ *   enqueued on it; no entry point synchronises the stream except
+ *   grpo_check_device_status.  Nothing is allocated: scratch space comes from
+ *   the caller's workspace `ws` of `ws_bytes` bytes (see grpo_workspace_bytes).
+ * - Errors the host can see (null pointers, bad sizes, misalignment, a
+ *   workspace that is too small) return a status at once and enqueue nothing.
+ *   Data-dependent problems found on the device (a target outside [0, V) on an
+ *   unmasked row, a pipeline wait that timed out, a non-finite log-sum-exp)
+ *   set bits of a status word inside the workspace; the affected rows' outputs
+ *   are 0.  grpo_check_device_status reports that word.
+ * - Outputs are overwritten, never accumulated into.  Results are
+ *   deterministic: no floating-point atomics are used on any output.
+ * - One workspace must not be used by two calls that can run concurrently.
+ */
+#ifndef GRPO_H_
+#define GRPO_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  GRPO_OK = 0,
+  GRPO_ERR_INVALID_ARG = 1,   /* null pointer, bad size or alignment */
+  GRPO_ERR_WORKSPACE = 2,     /* ws missing, misaligned or smaller than grpo_workspace_bytes */
+  GRPO_ERR_CUDA = 3,          /* a CUDA runtime/driver call failed */
+  GRPO_ERR_DEVICE_CHECK = 4,  /* device found a bad target index or a non-finite value */
+  GRPO_ERR_TIMEOUT = 5,       /* a bounded device-side wait gave up; outputs are invalid */
+  GRPO_ERR_UNSUPPORTED = 6    /* device is not sm_103 / sm_100 class, or shape beyond limits */
+} grpo_status;
+
+/* Which call a workspace is sized for (grpo_workspace_bytes `which`). */
+enum { GRPO_WS_LOGPROBS = 0, GRPO_WS_LOSS = 1 };
+
+/* Loss aggregation (grpo_loss_fwd_bwd `agg_mode`). */
+enum {
+  GRPO_AGG_TOKEN_MEAN = 0,    /* sum_t mask_t l_t / N_valid over the whole batch */
+  GRPO_AGG_SEQ_MEAN = 1       /* Eq. 1 as printed: (1/n_resp) sum_i (1/|o_i|) sum_t l_{i,t} */
+};
+
+/*
+ * Group-relative advantage, Eq. 2 (Section 3.3):
+ *   A_i = (r_i - mean_g(r)) / (std_g(r) + eps)
+ * over each group g of G consecutive responses; std is the sample standard
+ * deviation (divisor G - 1).  Computed in fp64, rounded once to fp32.
+ *   rewards  [n_resp] fp32 device, one reward per response
+ *   adv_out  [n_resp] fp32 device
+ * Requires G >= 2, n_resp >= 0 and n_resp % G == 0, else GRPO_ERR_INVALID_ARG.
+ */
+grpo_status grpo_group_advantages(const float* rewards, int64_t n_resp, int32_t G, float eps,
+                                  float* adv_out, void* stream);
+
+/*
+ * Per-token log-probability of the sampled token, the pi_theta(o_{i,t} | q, o_{i,<t})
+ * of Eq. 1 (Section 3.3):  logp_t = z_{t,y_t} - log sum_v exp(z_{t,v}),  z_t = H_t W^T.
+ * The [T x V] logits are never written to memory.
+ *   H        [T x Hd] bf16 device, final hidden states (16-byte aligned)
+ *   W        [V x Hd] bf16 device, LM-head weight (16-byte aligned)
+ *   targets  [T] int32 device, sampled token ids, must lie in [0, V) where mask != 0
+ *   mask     [T] uint8 device, 0 = padding row
+ *   logp_out [T] fp32 device; padding rows get 0
+ *   ws       device workspace of at least grpo_workspace_bytes(T, Hd, V, GRPO_WS_LOGPROBS)
+ *            bytes, 256-byte aligned
+ * Requires Hd % 64 == 0, 0 < V < 2^31, 0 <= T < 2^31.
+ */
+grpo_status grpo_token_logprobs(const uint16_t* H, const uint16_t* W, const int32_t* targets,
+                                const uint8_t* mask, int64_t T, int32_t Hd, int64_t V,
+                                float* logp_out, void* ws, size_t ws_bytes, void* stream);
+
+/*
+ * GRPO loss (the negated objective of Eq. 1, Section 3.3) and its gradient
+ * with respect to H and W.  Per unmasked token t of response i = t / L:
+ *   rho  = exp(logp_t - old_logp_t)
+ *   s    = min(rho A_i, clip(rho, 1 - clip_eps, 1 + clip_eps) A_i)
+ *   KL   = exp(ref_logp_t - logp_t) - (ref_logp_t - logp_t) - 1
+ *   l_t  = -s + beta KL,     loss = sum_t w_t l_t
+ * with w_t from agg_mode.  At the kink of min() the unclipped branch is taken.
+ *   H, W, targets, mask  as for grpo_token_logprobs, with T = n_resp * L
+ *   old_logp, ref_logp   [T] fp32 device: log-probs of the old and reference policies
+ *   adv                  [n_resp] fp32 device (e.g. from grpo_group_advantages)
+ *   loss_out             device pointer to one fp32
+ *   dH                   [T x Hd] fp32 device; padding rows get 0
+ *   dW                   [V x Hd] fp32 device
+ *   ws                   at least grpo_workspace_bytes(T, Hd, V, GRPO_WS_LOSS) bytes
+ * Requires n_resp >= 1, L >= 1, clip_eps >= 0, agg_mode in {0, 1}, dH and dW
+ * 16-byte aligned, and the limits of grpo_token_logprobs.
+ */
+grpo_status grpo_loss_fwd_bwd(const uint16_t* H, const uint16_t* W, const int32_t* targets,
+                              const uint8_t* mask, const float* old_logp, const float* ref_logp,
+                              const float* adv, int64_t n_resp, int64_t L, int32_t Hd, int64_t V,
+                              float clip_eps, float beta, int32_t agg_mode, float* loss_out,
+                              float* dH, float* dW, void* ws, size_t ws_bytes, void* stream);
+
+/*
+ * Bytes of workspace the call `which` (GRPO_WS_LOGPROBS or GRPO_WS_LOSS)
+ * needs for T tokens, hidden size Hd and vocabulary V.  Returns 0 for
+ * arguments the calls would reject.  Sized for the worst case N_valid = T.
+ */
+size_t grpo_workspace_bytes(int64_t T, int32_t Hd, int64_t V, int32_t which);
+
+/*
+ * Synchronises `stream`, reads the device status word of workspace `ws`
+ * (written by the last call that used it) and returns GRPO_OK,
+ * GRPO_ERR_DEVICE_CHECK or GRPO_ERR_TIMEOUT.  The word is cleared at the
+ * start of every compute call.
+ */
+grpo_status grpo_check_device_status(void* ws, void* stream);
+
+/* Static, human-readable name of a status code. */
+const char* grpo_status_string(grpo_status status);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* GRPO_H_ */

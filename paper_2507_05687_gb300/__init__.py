@@ -1,0 +1,12 @@
+"""GB300-native (sm_103a) GRPO hot path: advantages, LM-head log-probs, clipped
+objective with KL penalty, and its backward to H and W (Section 3.3, Eq. 1-2).
+
+The compute lives in libgrpo.so (C ABI in include/grpo.h); this package is
+its ctypes binding plus the in-tree build script.
+"""
+from .binding import (  # noqa: F401
+    GRPO_ERR_CUDA, GRPO_ERR_DEVICE_CHECK, GRPO_ERR_INVALID_ARG, GRPO_ERR_TIMEOUT, GRPO_ERR_UNSUPPORTED,
+    GRPO_ERR_WORKSPACE, GRPO_OK, GRPO_WS_LOGPROBS, GRPO_WS_LOSS, LIB_PATH, SIGNATURES, GrpoError,
+    check_device_status, group_advantages, load, loss_fwd_bwd, status_string, token_logprobs, workspace,
+    workspace_bytes,
+)

@@ -1,0 +1,196 @@
+"""ctypes binding of libgrpo.so (include/grpo.h), same names as the C ABI.
+
+Argument marshalling only: every step of the computation runs in the
+library's CUDA kernels.  PyTorch provides device memory and the current
+stream.  Inputs may be CUDA tensors, or CPU tensors (preferably pinned): CPU
+inputs are copied to the current CUDA device, the call runs there, and the
+results are copied back to CPU tensors.
+
+There is no fallback: if libgrpo.so is missing or the device is not a GB300
+class GPU, the calls raise.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from typing import Optional, Tuple
+
+import torch
+
+_PKG = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_PKG, "libgrpo.so")
+
+GRPO_OK = 0
+GRPO_ERR_INVALID_ARG = 1
+GRPO_ERR_WORKSPACE = 2
+GRPO_ERR_CUDA = 3
+GRPO_ERR_DEVICE_CHECK = 4
+GRPO_ERR_TIMEOUT = 5
+GRPO_ERR_UNSUPPORTED = 6
+GRPO_WS_LOGPROBS = 0
+GRPO_WS_LOSS = 1
+
+# name -> (restype, argtypes); mirrors include/grpo.h
+_P = ctypes.c_void_p
+_I64 = ctypes.c_int64
+_I32 = ctypes.c_int32
+_F = ctypes.c_float
+SIGNATURES = {
+    "grpo_group_advantages": (ctypes.c_int, [_P, _I64, _I32, _F, _P, _P]),
+    "grpo_token_logprobs": (ctypes.c_int, [_P, _P, _P, _P, _I64, _I32, _I64, _P, _P, ctypes.c_size_t, _P]),
+    "grpo_loss_fwd_bwd": (ctypes.c_int, [_P, _P, _P, _P, _P, _P, _P, _I64, _I64, _I32, _I64, _F, _F, _I32,
+                                         _P, _P, _P, _P, ctypes.c_size_t, _P]),
+    "grpo_workspace_bytes": (ctypes.c_size_t, [_I64, _I32, _I64, _I32]),
+    "grpo_check_device_status": (ctypes.c_int, [_P, _P]),
+    "grpo_status_string": (ctypes.c_char_p, [ctypes.c_int]),
+}
+
+_lib: Optional[ctypes.CDLL] = None
+
+
+class GrpoError(RuntimeError):
+    def __init__(self, status: int, where: str):
+        self.status = status
+        super().__init__(f"{where}: {status_string(status)} ({status})")
+
+
+def open_library(path: str) -> ctypes.CDLL:
+    """dlopen the library at `path` and declare its signatures; raises ImportError if absent."""
+    if not os.path.exists(path):
+        raise ImportError(f"{path} is missing: build it with `python -m paper_2507_05687_gb300.build`")
+    lib = ctypes.CDLL(path)
+    for name, (res, args) in SIGNATURES.items():
+        fn = getattr(lib, name)
+        fn.restype = res
+        fn.argtypes = args
+    return lib
+
+
+def load() -> ctypes.CDLL:
+    """The in-tree libgrpo.so (built by build.py), opened once per process."""
+    global _lib
+    if _lib is None:
+        _lib = open_library(LIB_PATH)
+    return _lib
+
+
+def status_string(status: int) -> str:
+    return load().grpo_status_string(int(status)).decode()
+
+
+def _check(st: int, where: str) -> None:
+    if st != GRPO_OK:
+        raise GrpoError(st, where)
+
+
+def _stream(device: torch.device) -> int:
+    return torch.cuda.current_stream(device).cuda_stream
+
+
+def _ptr(t: Optional[torch.Tensor]) -> Optional[int]:
+    return None if t is None else t.data_ptr()
+
+
+def _on_device(t: torch.Tensor, dev: torch.device, dtype: torch.dtype, name: str) -> torch.Tensor:
+    if t.dtype != dtype:
+        raise TypeError(f"{name}: expected {dtype}, got {t.dtype}")
+    if t.device != dev:
+        t = t.to(dev, non_blocking=True)
+    return t.contiguous()
+
+
+def _target_device(*ts: torch.Tensor) -> Tuple[torch.device, bool]:
+    for t in ts:
+        if t.is_cuda:
+            return t.device, False
+    return torch.device("cuda", torch.cuda.current_device()), True
+
+
+def _to_host(*ts: torch.Tensor):
+    """Pinned host copies of device results; returns once they have landed."""
+    outs = []
+    for t in ts:
+        o = torch.empty(t.shape, dtype=t.dtype, pin_memory=True)
+        o.copy_(t, non_blocking=True)
+        outs.append(o)
+    torch.cuda.current_stream(ts[0].device).synchronize()
+    return outs[0] if len(outs) == 1 else tuple(outs)
+
+
+def workspace_bytes(T: int, Hd: int, V: int, which: int) -> int:
+    """grpo_workspace_bytes: scratch bytes the call `which` needs."""
+    return int(load().grpo_workspace_bytes(int(T), int(Hd), int(V), int(which)))
+
+
+def workspace(T: int, Hd: int, V: int, which: int, device=None) -> torch.Tensor:
+    """A device byte tensor large enough for the call `which`."""
+    n = workspace_bytes(T, Hd, V, which)
+    if n == 0:
+        raise GrpoError(GRPO_ERR_INVALID_ARG, "grpo_workspace_bytes")
+    return torch.empty(n, dtype=torch.uint8, device=device or "cuda")
+
+
+def group_advantages(rewards: torch.Tensor, G: int, eps: float = 1e-6,
+                     out: Optional[torch.Tensor] = None) -> torch.Tensor:
+    """grpo_group_advantages: Eq. 2 per group of G consecutive responses."""
+    dev, host = _target_device(rewards)
+    r = _on_device(rewards, dev, torch.float32, "rewards")
+    adv = out if out is not None else torch.empty_like(r)
+    _check(load().grpo_group_advantages(_ptr(r), r.numel(), int(G), float(eps), _ptr(adv), _stream(dev)),
+           "grpo_group_advantages")
+    return _to_host(adv) if host else adv
+
+
+def token_logprobs(H: torch.Tensor, W: torch.Tensor, targets: torch.Tensor, mask: torch.Tensor,
+                   ws: Optional[torch.Tensor] = None, out: Optional[torch.Tensor] = None) -> torch.Tensor:
+    """grpo_token_logprobs: log softmax(H W^T) at the sampled tokens; padding rows give 0."""
+    dev, host = _target_device(H, W)
+    H = _on_device(H, dev, torch.bfloat16, "H")
+    W = _on_device(W, dev, torch.bfloat16, "W")
+    targets = _on_device(targets, dev, torch.int32, "targets")
+    mask = _on_device(mask.view(torch.uint8) if mask.dtype == torch.bool else mask, dev, torch.uint8, "mask")
+    T, Hd = H.shape
+    V = W.shape[0]
+    if ws is None:
+        ws = workspace(T, Hd, V, GRPO_WS_LOGPROBS, dev)
+    logp = out if out is not None else torch.empty(T, dtype=torch.float32, device=dev)
+    _check(load().grpo_token_logprobs(_ptr(H), _ptr(W), _ptr(targets), _ptr(mask), T, Hd, V, _ptr(logp),
+                                      _ptr(ws), ws.numel(), _stream(dev)), "grpo_token_logprobs")
+    return _to_host(logp) if host else logp
+
+
+def loss_fwd_bwd(H: torch.Tensor, W: torch.Tensor, targets: torch.Tensor, mask: torch.Tensor,
+                 old_logp: torch.Tensor, ref_logp: torch.Tensor, adv: torch.Tensor,
+                 n_resp: int, L: int, clip_eps: float = 0.2, beta: float = 0.04, agg_mode: int = 0,
+                 ws: Optional[torch.Tensor] = None,
+                 out: Optional[Tuple[torch.Tensor, torch.Tensor, torch.Tensor]] = None):
+    """grpo_loss_fwd_bwd: returns (loss [1] fp32, dH [T, Hd] fp32, dW [V, Hd] fp32)."""
+    dev, host = _target_device(H, W)
+    H = _on_device(H, dev, torch.bfloat16, "H")
+    W = _on_device(W, dev, torch.bfloat16, "W")
+    targets = _on_device(targets, dev, torch.int32, "targets")
+    mask = _on_device(mask.view(torch.uint8) if mask.dtype == torch.bool else mask, dev, torch.uint8, "mask")
+    old_logp = _on_device(old_logp, dev, torch.float32, "old_logp")
+    ref_logp = _on_device(ref_logp, dev, torch.float32, "ref_logp")
+    adv = _on_device(adv, dev, torch.float32, "adv")
+    T, Hd = H.shape
+    V = W.shape[0]
+    if ws is None:
+        ws = workspace(T, Hd, V, GRPO_WS_LOSS, dev)
+    if out is None:
+        out = (torch.empty(1, dtype=torch.float32, device=dev),
+               torch.empty(T, Hd, dtype=torch.float32, device=dev),
+               torch.empty(V, Hd, dtype=torch.float32, device=dev))
+    loss, dH, dW = out
+    _check(load().grpo_loss_fwd_bwd(_ptr(H), _ptr(W), _ptr(targets), _ptr(mask), _ptr(old_logp), _ptr(ref_logp),
+                                    _ptr(adv), int(n_resp), int(L), Hd, V, float(clip_eps), float(beta),
+                                    int(agg_mode), _ptr(loss), _ptr(dH), _ptr(dW), _ptr(ws), ws.numel(),
+                                    _stream(dev)), "grpo_loss_fwd_bwd")
+    if host:
+        return _to_host(loss, dH, dW)
+    return loss, dH, dW
+
+
+def check_device_status(ws: torch.Tensor) -> int:
+    """grpo_check_device_status: syncs the current stream and returns the status code."""
+    return int(load().grpo_check_device_status(_ptr(ws), _stream(ws.device)))

@@ -1,0 +1,400 @@
+// grpo_api.cu — the C ABI of include/grpo.h: argument checks, workspace
+// layout, TMA tensor maps and the launch sequence of each call.
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <cudaTypedefs.h>
+
+#include <cstdint>
+#include <cstdlib>
+#include <cstring>
+#include <mutex>
+
+#include "../../include/grpo.h"
+#include "gemm_tc.cuh"
+#include "small_kernels.cuh"
+
+using namespace grpo;
+
+namespace {
+
+constexpr int kLseTilesPerUnit = 16;     // vocabulary tiles (of 256) per forward work unit
+constexpr int kLossThreads = 256;
+constexpr int64_t kDefaultVocabChunk = 16384;
+
+int64_t round_up(int64_t x, int64_t m) { return (x + m - 1) / m * m; }
+
+// Vocabulary columns per backward chunk: the dZ chunk buffer holds
+// T x chunk bf16 values.  Multiple of 256; GRPO_VOCAB_CHUNK overrides.
+int64_t vocab_chunk(int64_t V) {
+  int64_t c = kDefaultVocabChunk;
+  if (const char* e = std::getenv("GRPO_VOCAB_CHUNK")) {
+    const long long v = std::atoll(e);
+    if (v >= 256) c = round_up(v, 256);
+  }
+  return std::min<int64_t>(c, round_up(V, 256));
+}
+
+// Workspace layout (byte offsets); every region is 256-byte aligned, the
+// bf16 matrices 1024-byte aligned.
+struct Layout {
+  int64_t T_pad, nsplit, nblk_scan, nblk_loss, vchunk;
+  size_t status, n_valid, counts, offsets, cidx, rank_of, yc, zy, part_m, part_s, lse_c, g_c,
+      block_loss, resp_len, Hc, dz, total;
+};
+
+bool make_layout(int64_t T, int32_t Hd, int64_t V, int32_t which, Layout* L) {
+  if (T < 0 || T >= (int64_t(1) << 31) || Hd <= 0 || Hd % 64 != 0 || V <= 0 ||
+      V >= (int64_t(1) << 31) || (which != GRPO_WS_LOGPROBS && which != GRPO_WS_LOSS))
+    return false;
+  L->T_pad = round_up(std::max<int64_t>(T, 1), kBM);
+  const int64_t vtiles = (V + kBN - 1) / kBN;
+  L->nsplit = (vtiles + kLseTilesPerUnit - 1) / kLseTilesPerUnit;
+  L->nblk_scan = (std::max<int64_t>(T, 1) + kScanChunk - 1) / kScanChunk;
+  L->nblk_loss = (L->T_pad + kLossThreads - 1) / kLossThreads;
+  L->vchunk = which == GRPO_WS_LOSS ? vocab_chunk(V) : 0;
+  size_t off = 0;
+  auto take = [&](size_t bytes, size_t align) {
+    off = (off + align - 1) / align * align;
+    const size_t at = off;
+    off += bytes;
+    return at;
+  };
+  const size_t tp = static_cast<size_t>(L->T_pad);
+  L->status = take(4, 256);
+  L->n_valid = take(4, 4);
+  L->counts = take(4 * L->nblk_scan, 256);
+  L->offsets = take(4 * L->nblk_scan, 256);
+  L->cidx = take(4 * tp, 256);
+  L->rank_of = take(4 * tp, 256);
+  L->yc = take(4 * tp, 256);
+  L->zy = take(4 * tp, 256);
+  L->part_m = take(4 * tp * L->nsplit, 256);
+  L->part_s = take(4 * tp * L->nsplit, 256);
+  L->lse_c = take(4 * tp, 256);
+  L->g_c = take(4 * tp, 256);
+  L->block_loss = take(8 * L->nblk_loss, 256);
+  L->resp_len = take(4 * tp, 256);
+  L->Hc = take(2 * tp * static_cast<size_t>(Hd), 1024);
+  L->dz = which == GRPO_WS_LOSS ? take(2 * tp * static_cast<size_t>(L->vchunk), 1024) : off;
+  L->total = (off + 1023) / 1024 * 1024;
+  return true;
+}
+
+// ---------------------------------------------------------------- driver entry points
+
+PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
+std::once_flag g_encode_once;
+
+bool get_encode() {
+  std::call_once(g_encode_once, [] {
+    void* fn = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      g_encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+  });
+  return g_encode != nullptr;
+}
+
+// 2D bf16 tensor map over a row-major [rows x cols] matrix; the box is
+// box_cols (inner, 64 = 128 bytes) x box_rows with the 128-byte swizzle.
+// Out-of-range elements of a box read as zero.
+bool encode_2d(CUtensorMap* map, const void* base, uint64_t rows, uint64_t cols, uint64_t ld_elems,
+               uint32_t box_cols, uint32_t box_rows) {
+  const cuuint64_t dims[2] = {cols, rows};
+  const cuuint64_t strides[1] = {ld_elems * 2};
+  const cuuint32_t box[2] = {box_cols, box_rows};
+  const cuuint32_t estr[2] = {1, 1};
+  const CUresult r = g_encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims,
+                              strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                              CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
+struct DeviceInfo {
+  int sms = 0;
+  bool ok = false;
+};
+
+// Per-device facts and the one-time opt-in to large dynamic shared memory.
+bool device_info(DeviceInfo* out) {
+  static std::mutex mu;
+  static DeviceInfo cache[64];
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return false;
+  std::lock_guard<std::mutex> lk(mu);
+  if (!cache[dev].ok) {
+    int major = 0, minor = 0, sms = 0;
+    if (cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+      return false;
+    if (major != 10 || minor != 3) return false;
+#define GRPO_SET_SMEM(E, A, B)                                                                   \
+  if (cudaFuncSetAttribute(gemm_tc_kernel<E, A, B>, cudaFuncAttributeMaxDynamicSharedMemorySize, \
+                           kGemmSmemBytes) != cudaSuccess)                                       \
+    return false;
+    GRPO_SET_SMEM(kEpiLse, false, false)
+    GRPO_SET_SMEM(kEpiDz, false, false)
+    GRPO_SET_SMEM(kEpiF32, false, true)
+    GRPO_SET_SMEM(kEpiF32, true, true)
+#undef GRPO_SET_SMEM
+    cache[dev].sms = sms;
+    cache[dev].ok = true;
+  }
+  *out = cache[dev];
+  return true;
+}
+
+template <int E, bool A, bool B>
+cudaError_t launch_gemm(const CUtensorMap& ta, const CUtensorMap& tb, const GemmArgs& a,
+                        int64_t max_units, int sms, cudaStream_t s) {
+  const int grid = static_cast<int>(std::max<int64_t>(1, std::min<int64_t>(sms, max_units)));
+  gemm_tc_kernel<E, A, B><<<grid, kGemmThreads, kGemmSmemBytes, s>>>(ta, tb, a);
+  return cudaGetLastError();
+}
+
+template <typename T>
+T* at(void* ws, size_t off) {
+  return reinterpret_cast<T*>(static_cast<char*>(ws) + off);
+}
+
+bool aligned(const void* p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
+
+// Compaction of unmasked rows + gather of their hidden states and targets.
+cudaError_t run_compaction(const uint16_t* H, const int32_t* targets, const uint8_t* mask, int64_t T,
+                           int32_t Hd, int64_t V, void* ws, const Layout& Ly, int sms,
+                           cudaStream_t s) {
+  unsigned* status = at<unsigned>(ws, Ly.status);
+  int* n_valid = at<int>(ws, Ly.n_valid);
+  cudaError_t e = cudaMemsetAsync(status, 0, 8, s);  // status word and n_valid
+  if (e != cudaSuccess) return e;
+  if (T > 0) {
+    const int nb = static_cast<int>(Ly.nblk_scan);
+    mask_count_kernel<<<nb, kScanThreads, 0, s>>>(mask, T, at<int>(ws, Ly.counts));
+    count_scan_kernel<<<1, 1024, 0, s>>>(at<int>(ws, Ly.counts), nb, at<int>(ws, Ly.offsets), n_valid);
+    mask_scatter_kernel<<<nb, kScanThreads, 0, s>>>(mask, T, at<int>(ws, Ly.offsets),
+                                                      at<int>(ws, Ly.cidx), at<int>(ws, Ly.rank_of));
+  }
+  const int64_t rows = Ly.T_pad;
+  const int gblocks = static_cast<int>(std::max<int64_t>(1, std::min<int64_t>(rows / 8 + 1, sms * 8)));
+  gather_rows_kernel<<<gblocks, 256, 0, s>>>(H, targets, at<int>(ws, Ly.cidx), n_valid, Hd, V,
+                                             at<uint16_t>(ws, Ly.Hc), at<int>(ws, Ly.yc), status);
+  return cudaGetLastError();
+}
+
+// Forward GEMM with the log-softmax epilogue over all V columns.
+cudaError_t run_lse(const uint16_t* W, int32_t Hd, int64_t V, void* ws, const Layout& Ly, int sms,
+                    cudaStream_t s) {
+  CUtensorMap tA, tB;
+  if (!encode_2d(&tA, at<uint16_t>(ws, Ly.Hc), Ly.T_pad, Hd, Hd, kBK, kBM) ||
+      !encode_2d(&tB, W, V, Hd, Hd, kBK, kBN))
+    return cudaErrorInvalidValue;
+  GemmArgs a{};
+  a.n_valid = at<int>(ws, Ly.n_valid);
+  a.M = 0;
+  a.m_dyn = 1;
+  a.N = static_cast<int>(V);
+  a.K = Hd;
+  a.n_per_unit = kLseTilesPerUnit;
+  a.group_m = 8;
+  a.status = at<unsigned>(ws, Ly.status);
+  a.yc = at<int>(ws, Ly.yc);
+  a.part_m = at<float>(ws, Ly.part_m);
+  a.part_s = at<float>(ws, Ly.part_s);
+  a.zy = at<float>(ws, Ly.zy);
+  a.ldp = Ly.T_pad;
+  const int64_t max_units = (Ly.T_pad / kBM) * Ly.nsplit;
+  return launch_gemm<kEpiLse, false, false>(tA, tB, a, max_units, sms, s);
+}
+
+grpo_status from_cuda(cudaError_t e) { return e == cudaSuccess ? GRPO_OK : GRPO_ERR_CUDA; }
+
+}  // namespace
+
+extern "C" {
+
+const char* grpo_status_string(grpo_status st) {
+  switch (st) {
+    case GRPO_OK: return "GRPO_OK";
+    case GRPO_ERR_INVALID_ARG: return "GRPO_ERR_INVALID_ARG";
+    case GRPO_ERR_WORKSPACE: return "GRPO_ERR_WORKSPACE";
+    case GRPO_ERR_CUDA: return "GRPO_ERR_CUDA";
+    case GRPO_ERR_DEVICE_CHECK: return "GRPO_ERR_DEVICE_CHECK";
+    case GRPO_ERR_TIMEOUT: return "GRPO_ERR_TIMEOUT";
+    case GRPO_ERR_UNSUPPORTED: return "GRPO_ERR_UNSUPPORTED";
+  }
+  return "GRPO_ERR_UNKNOWN";
+}
+
+size_t grpo_workspace_bytes(int64_t T, int32_t Hd, int64_t V, int32_t which) {
+  Layout L;
+  return make_layout(T, Hd, V, which, &L) ? L.total : 0;
+}
+
+grpo_status grpo_group_advantages(const float* rewards, int64_t n_resp, int32_t G, float eps,
+                                  float* adv_out, void* stream) {
+  if (G < 2 || n_resp < 0 || n_resp % G != 0) return GRPO_ERR_INVALID_ARG;
+  if (n_resp == 0) return GRPO_OK;
+  if (!rewards || !adv_out) return GRPO_ERR_INVALID_ARG;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if (G <= 32 && (G & (G - 1)) == 0) {
+    const int64_t blocks = (n_resp + 255) / 256;
+    adv_segmented_kernel<<<static_cast<unsigned>(blocks), 256, 0, s>>>(rewards, n_resp, G, eps, adv_out);
+  } else {
+    const int64_t groups = n_resp / G;
+    const int64_t blocks = (groups * 32 + 255) / 256;
+    adv_warp_kernel<<<static_cast<unsigned>(blocks), 256, 0, s>>>(rewards, groups, G, eps, adv_out);
+  }
+  return from_cuda(cudaGetLastError());
+}
+
+grpo_status grpo_token_logprobs(const uint16_t* H, const uint16_t* W, const int32_t* targets,
+                                const uint8_t* mask, int64_t T, int32_t Hd, int64_t V,
+                                float* logp_out, void* ws, size_t ws_bytes, void* stream) {
+  Layout Ly;
+  if (!make_layout(T, Hd, V, GRPO_WS_LOGPROBS, &Ly)) return GRPO_ERR_INVALID_ARG;
+  if (!W) return GRPO_ERR_INVALID_ARG;
+  if (T > 0 && (!H || !targets || !mask || !logp_out)) return GRPO_ERR_INVALID_ARG;
+  if (!aligned(W, 16) || (H && !aligned(H, 16))) return GRPO_ERR_INVALID_ARG;
+  if (!ws || !aligned(ws, 256) || ws_bytes < Ly.total) return GRPO_ERR_WORKSPACE;
+  if (T == 0) return GRPO_OK;
+  DeviceInfo di;
+  if (!device_info(&di)) return GRPO_ERR_UNSUPPORTED;
+  if (!get_encode()) return GRPO_ERR_CUDA;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  cudaError_t e = run_compaction(H, targets, mask, T, Hd, V, ws, Ly, di.sms, s);
+  if (e == cudaSuccess) e = run_lse(W, Hd, V, ws, Ly, di.sms, s);
+  if (e == cudaSuccess) {
+    const int blocks = static_cast<int>(std::min<int64_t>((T + 255) / 256, di.sms * 16));
+    logp_merge_kernel<<<blocks, 256, 0, s>>>(mask, at<int>(ws, Ly.rank_of), T, at<float>(ws, Ly.part_m),
+                                             at<float>(ws, Ly.part_s), static_cast<int>(Ly.nsplit),
+                                             Ly.T_pad, at<float>(ws, Ly.zy), at<int>(ws, Ly.yc),
+                                             logp_out, at<unsigned>(ws, Ly.status));
+    e = cudaGetLastError();
+  }
+  return from_cuda(e);
+}
+
+grpo_status grpo_loss_fwd_bwd(const uint16_t* H, const uint16_t* W, const int32_t* targets,
+                              const uint8_t* mask, const float* old_logp, const float* ref_logp,
+                              const float* adv, int64_t n_resp, int64_t L, int32_t Hd, int64_t V,
+                              float clip_eps, float beta, int32_t agg_mode, float* loss_out,
+                              float* dH, float* dW, void* ws, size_t ws_bytes, void* stream) {
+  if (n_resp < 1 || L < 1 || n_resp > (int64_t(1) << 31) / L) return GRPO_ERR_INVALID_ARG;
+  const int64_t T = n_resp * L;
+  Layout Ly;
+  if (!make_layout(T, Hd, V, GRPO_WS_LOSS, &Ly)) return GRPO_ERR_INVALID_ARG;
+  if (!H || !W || !targets || !mask || !old_logp || !ref_logp || !adv || !loss_out || !dH || !dW)
+    return GRPO_ERR_INVALID_ARG;
+  if (!(clip_eps >= 0.f) || !(beta == beta) || (agg_mode != GRPO_AGG_TOKEN_MEAN && agg_mode != GRPO_AGG_SEQ_MEAN))
+    return GRPO_ERR_INVALID_ARG;
+  if (!aligned(W, 16) || !aligned(H, 16) || !aligned(dH, 16) || !aligned(dW, 16))
+    return GRPO_ERR_INVALID_ARG;
+  if (!ws || !aligned(ws, 256) || ws_bytes < Ly.total) return GRPO_ERR_WORKSPACE;
+  DeviceInfo di;
+  if (!device_info(&di)) return GRPO_ERR_UNSUPPORTED;
+  if (!get_encode()) return GRPO_ERR_CUDA;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const int sms = di.sms;
+  int* n_valid = at<int>(ws, Ly.n_valid);
+  unsigned* status = at<unsigned>(ws, Ly.status);
+
+  cudaError_t e = run_compaction(H, targets, mask, T, Hd, V, ws, Ly, sms, s);
+  if (e == cudaSuccess && agg_mode == GRPO_AGG_SEQ_MEAN) {
+    const int64_t blocks = (n_resp * 32 + 255) / 256;
+    resp_len_kernel<<<static_cast<unsigned>(blocks), 256, 0, s>>>(mask, n_resp, L, at<int>(ws, Ly.resp_len));
+    e = cudaGetLastError();
+  }
+  if (e == cudaSuccess) e = run_lse(W, Hd, V, ws, Ly, sms, s);
+  if (e == cudaSuccess) {
+    loss_terms_kernel<<<static_cast<unsigned>(Ly.nblk_loss), kLossThreads, 0, s>>>(
+        at<int>(ws, Ly.cidx), n_valid, at<float>(ws, Ly.part_m), at<float>(ws, Ly.part_s),
+        static_cast<int>(Ly.nsplit), Ly.T_pad, at<float>(ws, Ly.zy), at<int>(ws, Ly.yc), old_logp,
+        ref_logp, adv, L, at<int>(ws, Ly.resp_len), n_resp, agg_mode, clip_eps, beta,
+        at<float>(ws, Ly.lse_c), at<float>(ws, Ly.g_c), at<double>(ws, Ly.block_loss), status);
+    loss_final_kernel<<<1, 1024, 0, s>>>(at<double>(ws, Ly.block_loss), n_valid, kLossThreads, loss_out);
+    const int zb = static_cast<int>(std::min<int64_t>((T + 7) / 8, sms * 8));
+    zero_masked_rows_kernel<<<zb, 256, 0, s>>>(mask, T, Hd, dH);
+    e = cudaGetLastError();
+  }
+  if (e != cudaSuccess) return from_cuda(e);
+
+  // Backward, one vocabulary chunk at a time.
+  CUtensorMap tHcK, tWK, tDzK, tWMN, tDzMN, tHcMN;
+  uint16_t* Hc = at<uint16_t>(ws, Ly.Hc);
+  uint16_t* dz = at<uint16_t>(ws, Ly.dz);
+  const int64_t vc = Ly.vchunk;
+  if (!encode_2d(&tHcK, Hc, Ly.T_pad, Hd, Hd, kBK, kBM) || !encode_2d(&tWK, W, V, Hd, Hd, kBK, kBN) ||
+      !encode_2d(&tDzK, dz, Ly.T_pad, vc, vc, kBK, kBM) || !encode_2d(&tWMN, W, V, Hd, Hd, 64, 64) ||
+      !encode_2d(&tDzMN, dz, Ly.T_pad, vc, vc, 64, 64) || !encode_2d(&tHcMN, Hc, Ly.T_pad, Hd, Hd, 64, 64))
+    return GRPO_ERR_CUDA;
+  const int64_t mt_max = Ly.T_pad / kBM;
+  const int64_t hd_tiles = (Hd + kBN - 1) / kBN;
+  for (int64_t c0 = 0; c0 < V && e == cudaSuccess; c0 += vc) {
+    const int64_t width = std::min<int64_t>(vc, V - c0);
+    // dZ chunk = g (onehot - softmax) from recomputed logits
+    GemmArgs a{};
+    a.n_valid = n_valid;
+    a.m_dyn = 1;
+    a.N = static_cast<int>(width);
+    a.K = Hd;
+    a.b_off_n = static_cast<int>(c0);
+    a.n_per_unit = 1;
+    a.group_m = 8;
+    a.status = status;
+    a.yc = at<int>(ws, Ly.yc);
+    a.lse = at<float>(ws, Ly.lse_c);
+    a.gcoef = at<float>(ws, Ly.g_c);
+    a.dz = dz;
+    a.ldz = vc;
+    e = launch_gemm<kEpiDz, false, false>(tHcK, tWK, a, mt_max * ((width + kBN - 1) / kBN), sms, s);
+    if (e != cudaSuccess) break;
+    // dH (+)= dZ_c W_c
+    GemmArgs h{};
+    h.n_valid = n_valid;
+    h.m_dyn = 1;
+    h.N = Hd;
+    h.K = static_cast<int>(width);
+    h.b_off_k = static_cast<int>(c0);
+    h.n_per_unit = 1;
+    h.group_m = 8;
+    h.status = status;
+    h.out = dH;
+    h.ldo = Hd;
+    h.accumulate = c0 > 0;
+    h.row_map = at<int>(ws, Ly.cidx);
+    e = launch_gemm<kEpiF32, false, true>(tDzK, tWMN, h, mt_max * hd_tiles, sms, s);
+    if (e != cudaSuccess) break;
+    // dW_c = dZ_c^T Hc
+    GemmArgs w{};
+    w.n_valid = n_valid;
+    w.M = static_cast<int>(width);
+    w.N = Hd;
+    w.k_dyn = 1;
+    w.n_per_unit = 1;
+    w.group_m = 8;
+    w.status = status;
+    w.out = dW + c0 * Hd;
+    w.ldo = Hd;
+    w.accumulate = 0;
+    e = launch_gemm<kEpiF32, true, true>(tDzMN, tHcMN, w, ((width + kBM - 1) / kBM) * hd_tiles, sms, s);
+  }
+  return from_cuda(e);
+}
+
+grpo_status grpo_check_device_status(void* ws, void* stream) {
+  if (!ws) return GRPO_ERR_INVALID_ARG;
+  unsigned word = 0;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if (cudaMemcpyAsync(&word, ws, sizeof(word), cudaMemcpyDeviceToHost, s) != cudaSuccess ||
+      cudaStreamSynchronize(s) != cudaSuccess)
+    return GRPO_ERR_CUDA;
+  if (word & kDevTimeout) return GRPO_ERR_TIMEOUT;
+  if (word) return GRPO_ERR_DEVICE_CHECK;
+  return GRPO_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,312 @@
+// small_kernels.cuh — the O(T) kernels around the LM-head GEMMs:
+// group advantages (Eq. 2), compaction of unmasked rows, the merge of the
+// per-split log-sum-exp partials, the per-token loss terms of Eq. 1 with
+// their derivative in logp, and the deterministic loss reduction.
+#pragma once
+
+#include <stdint.h>
+
+#include "ptx.cuh"
+
+namespace grpo {
+
+constexpr int kScanChunk = 4096;   // tokens per block in the compaction kernels
+constexpr int kScanThreads = 256;  // 16 tokens per thread
+
+// ------------------------------------------------------------------ Eq. 2
+
+// fp64 sum over the lanes of one aligned segment of `width` lanes (power of 2).
+__device__ __forceinline__ double seg_sum(double x, int width) {
+  for (int o = width >> 1; o > 0; o >>= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
+  return x;
+}
+
+// G a power of two <= 32: each warp holds 32/G groups, one reward per lane,
+// and reduces each group with shuffles inside its G-lane segment.
+__global__ void adv_segmented_kernel(const float* __restrict__ r, int64_t n, int G, float eps,
+                                     float* __restrict__ adv) {
+  const int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+  const int64_t base = i - (threadIdx.x & 31);
+  if (base >= n) return;  // whole warp out of range (n % G == 0, groups never straddle warps)
+  const bool in = i < n;
+  const double x = in ? static_cast<double>(r[i]) : 0.0;
+  const double mean = seg_sum(x, G) / G;
+  const double d = in ? x - mean : 0.0;
+  const double var = seg_sum(d * d, G) / (G - 1);
+  const double sd = sqrt(var);
+  if (in) adv[i] = static_cast<float>(d / (sd + static_cast<double>(eps)));
+}
+
+// Any G: one warp per group, lanes stride over its members.
+__global__ void adv_warp_kernel(const float* __restrict__ r, int64_t n_groups, int G, float eps,
+                                float* __restrict__ adv) {
+  const int64_t g = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
+  const int lane = threadIdx.x & 31;
+  if (g >= n_groups) return;
+  const float* rg = r + g * G;
+  double s = 0.0;
+  for (int j = lane; j < G; j += 32) s += static_cast<double>(rg[j]);
+  const double mean = seg_sum(s, 32) / G;
+  double q = 0.0;
+  for (int j = lane; j < G; j += 32) {
+    const double d = static_cast<double>(rg[j]) - mean;
+    q += d * d;
+  }
+  const double sd = sqrt(seg_sum(q, 32) / (G - 1));
+  for (int j = lane; j < G; j += 32)
+    adv[g * G + j] = static_cast<float>((static_cast<double>(rg[j]) - mean) / (sd + static_cast<double>(eps)));
+}
+
+// ------------------------------------------------------------------ compaction
+
+__device__ __forceinline__ int block_exclusive_scan(int v, int* sh /*[32]*/, int* total) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  int x = v;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const int y = __shfl_up_sync(0xffffffffu, x, o);
+    if (lane >= o) x += y;
+  }
+  if (lane == 31) sh[warp] = x;
+  __syncthreads();
+  if (warp == 0) {
+    const int nw = blockDim.x >> 5;
+    int w = lane < nw ? sh[lane] : 0;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int y = __shfl_up_sync(0xffffffffu, w, o);
+      if (lane >= o) w += y;
+    }
+    if (lane < nw) sh[lane] = w;  // inclusive warp totals
+  }
+  __syncthreads();
+  const int before = (warp > 0 ? sh[warp - 1] : 0) + x - v;
+  *total = sh[(blockDim.x >> 5) - 1];
+  __syncthreads();
+  return before;
+}
+
+// counts[b] = number of unmasked rows in chunk b.
+__global__ void mask_count_kernel(const uint8_t* __restrict__ mask, int64_t T, int* __restrict__ counts) {
+  __shared__ int sh[32];
+  const int64_t base = static_cast<int64_t>(blockIdx.x) * kScanChunk + threadIdx.x * 16;
+  int c = 0;
+#pragma unroll
+  for (int j = 0; j < 16; ++j) c += (base + j < T && mask[base + j] != 0) ? 1 : 0;
+  int total;
+  block_exclusive_scan(c, sh, &total);
+  if (threadIdx.x == 0) counts[blockIdx.x] = total;
+}
+
+// Single block: offsets[b] = sum of counts before b; *n_valid = grand total.
+__global__ void count_scan_kernel(const int* __restrict__ counts, int nb, int* __restrict__ offsets,
+                                  int* __restrict__ n_valid) {
+  __shared__ int sh[32];
+  int carry = 0;
+  for (int b0 = 0; b0 < nb; b0 += blockDim.x) {
+    const int b = b0 + threadIdx.x;
+    const int v = b < nb ? counts[b] : 0;
+    int total;
+    const int ex = block_exclusive_scan(v, sh, &total);
+    if (b < nb) offsets[b] = carry + ex;
+    carry += total;
+  }
+  if (threadIdx.x == 0) *n_valid = carry;
+}
+
+// cidx[rank] = t for unmasked rows; rank_of[t] = rank or -1.
+__global__ void mask_scatter_kernel(const uint8_t* __restrict__ mask, int64_t T,
+                                    const int* __restrict__ offsets, int* __restrict__ cidx,
+                                    int* __restrict__ rank_of) {
+  __shared__ int sh[32];
+  const int64_t base = static_cast<int64_t>(blockIdx.x) * kScanChunk + threadIdx.x * 16;
+  uint32_t bits = 0;
+  int c = 0;
+#pragma unroll
+  for (int j = 0; j < 16; ++j) {
+    const bool m = base + j < T && mask[base + j] != 0;
+    bits |= (m ? 1u : 0u) << j;
+    c += m ? 1 : 0;
+  }
+  int total;
+  int pos = offsets[blockIdx.x] + block_exclusive_scan(c, sh, &total);
+#pragma unroll
+  for (int j = 0; j < 16; ++j) {
+    const int64_t t = base + j;
+    if (t < T) {
+      if (bits & (1u << j)) {
+        cidx[pos] = static_cast<int>(t);
+        rank_of[t] = pos;
+        ++pos;
+      } else {
+        rank_of[t] = -1;
+      }
+    }
+  }
+}
+
+// Hc[r] = H[cidx[r]] and yc[r] = targets[cidx[r]] for r < n_valid; rows
+// n_valid .. round_up(n_valid, 128) are zero-filled (they feed K-loops over
+// tokens).  One warp per row, 16-byte vectors.
+__global__ void gather_rows_kernel(const uint16_t* __restrict__ H, const int32_t* __restrict__ targets,
+                                   const int* __restrict__ cidx, const int* __restrict__ n_valid_p,
+                                   int Hd, int64_t V, uint16_t* __restrict__ Hc, int* __restrict__ yc,
+                                   unsigned* status) {
+  const int nv = *n_valid_p;
+  const int rows = (nv + 127) / 128 * 128;
+  const int lane = threadIdx.x & 31;
+  const int vec = Hd / 8;  // uint4 per row
+  for (int r = (blockIdx.x * blockDim.x + threadIdx.x) >> 5; r < rows;
+       r += (gridDim.x * blockDim.x) >> 5) {
+    uint4* dst = reinterpret_cast<uint4*>(Hc + static_cast<int64_t>(r) * Hd);
+    if (r < nv) {
+      const int t = cidx[r];
+      const uint4* src = reinterpret_cast<const uint4*>(H + static_cast<int64_t>(t) * Hd);
+      for (int j = lane; j < vec; j += 32) dst[j] = __ldg(src + j);
+      if (lane == 0) {
+        const int y = targets[t];
+        const bool ok = y >= 0 && static_cast<int64_t>(y) < V;
+        yc[r] = ok ? y : -1;
+        if (!ok) atomicOr(status, kDevBadTarget);
+      }
+    } else {
+      for (int j = lane; j < vec; j += 32) dst[j] = make_uint4(0, 0, 0, 0);
+      if (lane == 0) yc[r] = -1;
+    }
+  }
+}
+
+// |o_i|: unmasked rows of each response (for the Eq. 1 per-response mean).
+__global__ void resp_len_kernel(const uint8_t* __restrict__ mask, int64_t n_resp, int64_t L,
+                                int* __restrict__ len) {
+  const int64_t i = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
+  const int lane = threadIdx.x & 31;
+  if (i >= n_resp) return;
+  int c = 0;
+  for (int64_t j = lane; j < L; j += 32) c += mask[i * L + j] != 0;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) c += __shfl_xor_sync(0xffffffffu, c, o);
+  if (lane == 0) len[i] = c;
+}
+
+// ------------------------------------------------------------------ merge + loss
+
+// log-sum-exp of row r from the per-split partials (log2 units inside).
+__device__ __forceinline__ float merge_lse(const float* __restrict__ pm, const float* __restrict__ ps,
+                                           int nsplit, long ldp, int r) {
+  float m = -INFINITY;
+  for (int j = 0; j < nsplit; ++j) m = fmaxf(m, pm[j * ldp + r]);
+  float s = 0.f;
+  for (int j = 0; j < nsplit; ++j) s += ps[j * ldp + r] * fast_exp2(pm[j * ldp + r] - m);
+  return (m + __log2f(s)) * 0.6931471805599453f;
+}
+
+// logp_out[t] for every row (0 on padding and on rows with a bad target).
+__global__ void logp_merge_kernel(const uint8_t* __restrict__ mask, const int* __restrict__ rank_of,
+                                  int64_t T, const float* __restrict__ pm, const float* __restrict__ ps,
+                                  int nsplit, long ldp, const float* __restrict__ zy,
+                                  const int* __restrict__ yc, float* __restrict__ logp_out,
+                                  unsigned* status) {
+  for (int64_t t = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; t < T;
+       t += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+    float out = 0.f;
+    if (mask[t]) {
+      const int r = rank_of[t];
+      const float lse = merge_lse(pm, ps, nsplit, ldp, r);
+      if (!isfinite(lse)) atomicOr(status, kDevNonFinite);
+      out = yc[r] >= 0 ? zy[r] - lse : 0.f;
+    }
+    logp_out[t] = out;
+  }
+}
+
+// Per-token terms of Eq. 1 over compacted rows: lse_c, g_c (dloss/dlogp) and
+// one fp64 partial sum of w_t l_t per block (fixed order, no atomics).
+__global__ void loss_terms_kernel(const int* __restrict__ cidx, const int* __restrict__ n_valid_p,
+                                  const float* __restrict__ pm, const float* __restrict__ ps,
+                                  int nsplit, long ldp, const float* __restrict__ zy,
+                                  const int* __restrict__ yc, const float* __restrict__ old_logp,
+                                  const float* __restrict__ ref_logp, const float* __restrict__ adv,
+                                  int64_t L, const int* __restrict__ resp_len, int64_t n_resp,
+                                  int agg_mode, float clip_eps, float beta,
+                                  float* __restrict__ lse_c, float* __restrict__ g_c,
+                                  double* __restrict__ block_loss, unsigned* status) {
+  __shared__ double sh[32];
+  const int nv = *n_valid_p;
+  const int r = blockIdx.x * blockDim.x + threadIdx.x;
+  double contrib = 0.0;
+  if (r < nv) {
+    const int t = cidx[r];
+    const int64_t i = t / L;
+    float lse = merge_lse(pm, ps, nsplit, ldp, r);
+    if (!isfinite(lse)) atomicOr(status, kDevNonFinite);
+    const bool yok = yc[r] >= 0;
+    float g = 0.f;
+    if (yok && isfinite(lse)) {
+      const float logp = zy[r] - lse;
+      const float A = adv[i];
+      const float rho = __expf(logp - old_logp[t]);
+      const float s1 = rho * A;
+      const float s2 = fminf(fmaxf(rho, 1.f - clip_eps), 1.f + clip_eps) * A;
+      const bool unclipped = s1 <= s2;
+      const float s = unclipped ? s1 : s2;
+      const float dref = ref_logp[t] - logp;
+      const float e = __expf(dref);
+      const float kl = e - dref - 1.f;
+      const float ell = -s + beta * kl;
+      const float w = agg_mode == 0 ? 1.f / static_cast<float>(nv)
+                                    : 1.f / (static_cast<float>(n_resp) * static_cast<float>(resp_len[i]));
+      g = w * ((unclipped ? -A * rho : 0.f) + beta * (1.f - e));
+      contrib = static_cast<double>(w) * static_cast<double>(ell);
+    } else {
+      lse = 0.f;
+    }
+    lse_c[r] = lse;
+    g_c[r] = g;
+  }
+  // block reduction in a fixed order
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) contrib += __shfl_xor_sync(0xffffffffu, contrib, o);
+  if ((threadIdx.x & 31) == 0) sh[threadIdx.x >> 5] = contrib;
+  __syncthreads();
+  if (threadIdx.x < 32) {
+    double x = threadIdx.x < (blockDim.x >> 5) ? sh[threadIdx.x] : 0.0;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
+    if (threadIdx.x == 0) block_loss[blockIdx.x] = x;
+  }
+}
+
+// Single block: loss = sum of the block partials, in block order.
+__global__ void loss_final_kernel(const double* __restrict__ block_loss, const int* __restrict__ n_valid_p,
+                                  int threads_per_block, float* __restrict__ loss_out) {
+  __shared__ double sh[32];
+  const int nb = (*n_valid_p + threads_per_block - 1) / threads_per_block;
+  double x = 0.0;
+  for (int b = threadIdx.x; b < nb; b += blockDim.x) x += block_loss[b];
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
+  if ((threadIdx.x & 31) == 0) sh[threadIdx.x >> 5] = x;
+  __syncthreads();
+  if (threadIdx.x < 32) {
+    double y = threadIdx.x < (blockDim.x >> 5) ? sh[threadIdx.x] : 0.0;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) y += __shfl_xor_sync(0xffffffffu, y, o);
+    if (threadIdx.x == 0) *loss_out = static_cast<float>(y);
+  }
+}
+
+// dH rows of padding tokens are 0 (the GEMM only writes unmasked rows).
+__global__ void zero_masked_rows_kernel(const uint8_t* __restrict__ mask, int64_t T, int Hd,
+                                        float* __restrict__ dH) {
+  const int lane = threadIdx.x & 31;
+  const int vec = Hd / 4;
+  for (int64_t t = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5; t < T;
+       t += (static_cast<int64_t>(gridDim.x) * blockDim.x) >> 5) {
+    if (mask[t]) continue;
+    float4* row = reinterpret_cast<float4*>(dH + t * Hd);
+    for (int j = lane; j < vec; j += 32) row[j] = make_float4(0.f, 0.f, 0.f, 0.f);
+  }
+}
+
+}  // namespace grpo

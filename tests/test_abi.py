@@ -1,0 +1,97 @@
+"""Host-side checks of the C ABI: the library builds, loads and exports every
+symbol include/grpo.h declares, and host-detectable errors come back as status
+codes without touching a GPU."""
+import ctypes
+import os
+import re
+
+import pytest
+
+import paper_2507_05687_gb300 as grpo
+from paper_2507_05687_gb300 import build as build_mod
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    build_mod.build()
+    return grpo.load()
+
+
+def header_symbols():
+    text = open(os.path.join(ROOT, "include", "grpo.h")).read()
+    return sorted(set(re.findall(r"^\S.*?\b(grpo_\w+)\(", text, flags=re.M)))
+
+
+def test_header_declares_the_boundary():
+    syms = header_symbols()
+    for name in ("grpo_group_advantages", "grpo_token_logprobs", "grpo_loss_fwd_bwd",
+                 "grpo_workspace_bytes", "grpo_check_device_status", "grpo_status_string"):
+        assert name in syms
+    assert set(syms) == set(grpo.SIGNATURES), "binding and header disagree"
+
+
+def test_every_declared_symbol_is_exported(lib):
+    for name in header_symbols():
+        assert hasattr(lib, name), name
+    # exported with C linkage (no mangling)
+    raw = ctypes.CDLL(grpo.LIB_PATH)
+    for name in header_symbols():
+        assert ctypes.cast(getattr(raw, name), ctypes.c_void_p).value
+
+
+def test_status_strings(lib):
+    for code, name in ((0, "GRPO_OK"), (1, "GRPO_ERR_INVALID_ARG"), (2, "GRPO_ERR_WORKSPACE"),
+                       (5, "GRPO_ERR_TIMEOUT"), (6, "GRPO_ERR_UNSUPPORTED")):
+        assert grpo.status_string(code) == name
+
+
+def test_workspace_sizes(lib):
+    f = grpo.workspace_bytes
+    assert f(256, 256, 4096, 0) > 256 * 256 * 2
+    assert f(32768, 4096, 155136, 1) > f(32768, 4096, 155136, 0) > 32768 * 4096 * 2
+    assert f(0, 64, 10, 0) > 0
+    for bad in ((-1, 64, 10, 0), (10, 60, 10, 0), (10, 0, 10, 0), (10, 64, 0, 0), (10, 64, 10, 7),
+                (1 << 31, 64, 10, 0)):
+        assert f(*bad) == 0, bad
+    assert f(1000, 128, 300, 1) % 1024 == 0
+
+
+FAKE = 0x10000  # never dereferenced: every call below is rejected on the host
+
+
+def test_host_rejections(lib):
+    L = lib
+    assert L.grpo_group_advantages(FAKE, 8, 1, 1e-6, FAKE, None) == grpo.GRPO_ERR_INVALID_ARG
+    assert L.grpo_group_advantages(FAKE, 9, 4, 1e-6, FAKE, None) == grpo.GRPO_ERR_INVALID_ARG
+    assert L.grpo_group_advantages(None, 8, 4, 1e-6, FAKE, None) == grpo.GRPO_ERR_INVALID_ARG
+    assert L.grpo_group_advantages(None, 0, 4, 1e-6, None, None) == grpo.GRPO_OK
+    ws_need = grpo.workspace_bytes(100, 64, 1000, 0)
+    args = [FAKE, FAKE, FAKE, FAKE, 100, 64, 1000, FAKE, FAKE, ws_need, None]
+    bad = list(args); bad[4 + 1] = 96 - 1          # Hd not a multiple of 64
+    assert L.grpo_token_logprobs(*bad) == grpo.GRPO_ERR_INVALID_ARG
+    bad = list(args); bad[0] = None               # H missing
+    assert L.grpo_token_logprobs(*bad) == grpo.GRPO_ERR_INVALID_ARG
+    bad = list(args); bad[1] = FAKE + 2           # W not 16-byte aligned
+    assert L.grpo_token_logprobs(*bad) == grpo.GRPO_ERR_INVALID_ARG
+    bad = list(args); bad[9] = ws_need - 1        # workspace too small
+    assert L.grpo_token_logprobs(*bad) == grpo.GRPO_ERR_WORKSPACE
+    bad = list(args); bad[8] = FAKE + 16          # workspace misaligned
+    assert L.grpo_token_logprobs(*bad) == grpo.GRPO_ERR_WORKSPACE
+    ws2 = grpo.workspace_bytes(40, 64, 1000, 1)
+    largs = [FAKE] * 7 + [10, 4, 64, 1000, 0.2, 0.04, 0, FAKE, FAKE, FAKE, FAKE, ws2, None]
+    for i, v in ((7, 0), (8, 0), (11, -0.1), (13, 2), (13, -1)):
+        bad = list(largs); bad[i] = v
+        assert L.grpo_loss_fwd_bwd(*bad) == grpo.GRPO_ERR_INVALID_ARG, i
+    bad = list(largs); bad[16] = FAKE + 4          # dW misaligned
+    assert L.grpo_loss_fwd_bwd(*bad) == grpo.GRPO_ERR_INVALID_ARG
+    bad = list(largs); bad[18] = ws2 - 1024
+    assert L.grpo_loss_fwd_bwd(*bad) == grpo.GRPO_ERR_WORKSPACE
+    assert L.grpo_check_device_status(None, None) == grpo.GRPO_ERR_INVALID_ARG
+
+
+def test_binding_fails_loudly_without_library(tmp_path):
+    from paper_2507_05687_gb300 import binding
+    with pytest.raises(ImportError):
+        binding.open_library(str(tmp_path / "missing.so"))

@@ -1,0 +1,187 @@
+"""GPU parity of the CUDA path against the float64 oracle, element by element,
+at sizes the oracle finishes in seconds: several tiles, ragged tails, several
+vocabulary splits and backward chunks, and the degenerate cases."""
+import numpy as np
+import pytest
+
+import oracle
+import workloads as wl
+from tests._util import GRAD_RTOL, LOGP_ATOL, LOSS_RTOL, dev_tensor, loss_scale, rel_fro
+
+torch = pytest.importorskip("torch")
+pytestmark = pytest.mark.gpu
+
+if not torch.cuda.is_available():  # pragma: no cover
+    pytest.skip("needs a CUDA GPU", allow_module_level=True)
+
+import paper_2507_05687_gb300 as grpo  # noqa: E402
+from paper_2507_05687_gb300 import build as build_mod  # noqa: E402
+
+build_mod.build()
+DEV = torch.device("cuda", 0)
+
+
+def _case(w, agg_mode=0):
+    """Seeded inputs of workload w plus the oracle's outputs on them."""
+    Hb, Wb = wl.gen_hidden(w), wl.gen_weight(w)
+    y, m, r = wl.gen_targets(w), wl.gen_mask(w), wl.gen_rewards(w)
+    W_old, W_ref = wl.gen_weight(w, "old", Wb), wl.gen_weight(w, "ref", Wb)
+    old = oracle.token_logprobs(Hb, W_old, y, m)[0].astype(np.float32)
+    ref = oracle.token_logprobs(Hb, W_ref, y, m)[0].astype(np.float32)
+    adv = oracle.group_advantages(r, w.G, float(np.float32(w.adv_eps)))
+    want = oracle.loss_fwd_bwd(Hb, Wb, y, m, old, ref, adv, w.n_resp, w.L, w.clip_eps, w.beta, agg_mode)
+    return dict(w=w, H=Hb, W=Wb, y=y, m=m, r=r, old=old, ref=ref, adv=adv, want=want)
+
+
+def _dev(c):
+    return dict(H=dev_tensor(c["H"], torch.bfloat16), W=dev_tensor(c["W"], torch.bfloat16),
+                y=dev_tensor(c["y"], torch.int32), m=dev_tensor(c["m"], torch.uint8),
+                old=dev_tensor(c["old"], torch.float32), ref=dev_tensor(c["ref"], torch.float32),
+                adv=dev_tensor(c["adv"], torch.float32), r=dev_tensor(c["r"], torch.float32))
+
+
+def _check_fwd_bwd(c, agg_mode=0):
+    w, d = c["w"], _dev(c)
+    ws = grpo.workspace(w.T, w.Hd, w.V, grpo.GRPO_WS_LOSS, DEV)
+    loss, dH, dW = grpo.loss_fwd_bwd(d["H"], d["W"], d["y"], d["m"], d["old"], d["ref"], d["adv"],
+                                     w.n_resp, w.L, w.clip_eps, w.beta, agg_mode, ws=ws)
+    assert grpo.check_device_status(ws) == grpo.GRPO_OK
+    want = c["want"]
+    scale = loss_scale(want["loss"], want["terms"]["w"], want["terms"]["ell"])
+    assert abs(loss.item() - want["loss"]) <= LOSS_RTOL * scale, (loss.item(), want["loss"], scale)
+    dHn, dWn = dH.double().cpu().numpy(), dW.double().cpu().numpy()
+    assert rel_fro(dHn, want["dH"]) <= GRAD_RTOL, rel_fro(dHn, want["dH"])
+    assert rel_fro(dWn, want["dW"]) <= GRAD_RTOL, rel_fro(dWn, want["dW"])
+    assert np.all(dHn[c["m"] == 0] == 0.0)
+    return loss, dH, dW
+
+
+# ---------------------------------------------------------------- Eq. 2
+
+@pytest.mark.parametrize("G", [2, 3, 4, 5, 8, 16, 32, 48, 64, 100])
+def test_advantages_bit_exact_dyadic(G):
+    rng = np.random.default_rng(G)
+    r = (rng.integers(0, 5, size=G * 37) / 4.0).astype(np.float32)   # {0, .25, .5, .75, 1}
+    r[:G] = 0.5                                                       # a zero-std group
+    got = grpo.group_advantages(dev_tensor(r, torch.float32), G, 1e-6).cpu().numpy()
+    want = oracle.group_advantages(r, G, float(np.float32(1e-6)))
+    assert np.array_equal(got.view(np.uint32), want.view(np.uint32))
+
+
+@pytest.mark.parametrize("G", [2, 7, 8, 32, 33])
+def test_advantages_general_rewards_within_one_ulp(G):
+    rng = np.random.default_rng(100 + G)
+    r = rng.normal(size=G * 50).astype(np.float32)
+    got = grpo.group_advantages(dev_tensor(r, torch.float32), G, 1e-6).cpu().numpy()
+    want = oracle.group_advantages(r, G, float(np.float32(1e-6)))
+    ulp = np.abs(got.view(np.int32).astype(np.int64) - want.view(np.int32).astype(np.int64))
+    assert ulp.max() <= 1
+
+
+@pytest.mark.parametrize("name", list(wl.WORKLOADS))
+def test_advantages_of_every_workload_bit_exact(name):
+    w = wl.WORKLOADS[name]
+    r = wl.gen_rewards(w)
+    got = grpo.group_advantages(dev_tensor(r, torch.float32), w.G, w.adv_eps).cpu().numpy()
+    want = oracle.group_advantages(r, w.G, float(np.float32(w.adv_eps)))
+    assert np.array_equal(got.view(np.uint32), want.view(np.uint32))
+
+
+# ---------------------------------------------------------------- log-probs
+
+LOGP_SHAPES = [
+    # (n_prompts, G, L, Hd, V, lengths)
+    (1, 4, 64, 256, 4096, "full"),            # the tiny workload's shape
+    (2, 3, 150, 192, 1000, "uniform"),        # vocabulary tail (1000 = 3*256 + 232), ragged rows
+    (1, 2, 65, 64, 300, "uniform"),           # one k-block, tail
+    (3, 4, 97, 512, 8292, "uniform"),         # three vocabulary splits, tail of 100
+]
+
+
+@pytest.mark.parametrize("shape", LOGP_SHAPES)
+def test_logprobs_match_oracle(shape):
+    P, G, L, Hd, V, lens = shape
+    w = wl.Workload("t", P, G, L, Hd, V, lens, 1, L, seed=wl.SEED_BASE + 1000 + Hd + V)
+    Hb, Wb, y, m = wl.gen_hidden(w), wl.gen_weight(w), wl.gen_targets(w), wl.gen_mask(w)
+    want, _ = oracle.token_logprobs(Hb, Wb, y, m)
+    got = grpo.token_logprobs(dev_tensor(Hb, torch.bfloat16), dev_tensor(Wb, torch.bfloat16),
+                              dev_tensor(y, torch.int32), dev_tensor(m, torch.uint8)).cpu().numpy()
+    assert np.all(got[m == 0] == 0.0)
+    err = np.abs(got.astype(np.float64) - want)
+    assert err.max() <= LOGP_ATOL, err.max()
+
+
+def test_logprobs_large_logits_and_host_buffers():
+    w = wl.Workload("t", 2, 2, 70, 128, 777, "uniform", 1, 70, seed=wl.SEED_BASE + 77, w_std=0.5)
+    Hb, Wb, y, m = wl.gen_hidden(w), wl.gen_weight(w), wl.gen_targets(w), wl.gen_mask(w)
+    want, _ = oracle.token_logprobs(Hb, Wb, y, m)
+    # CPU tensors in, CPU tensor out (host<->device copies inside the call)
+    got = grpo.token_logprobs(torch.from_numpy(Hb).view(torch.bfloat16), torch.from_numpy(Wb).view(torch.bfloat16),
+                              torch.from_numpy(y), torch.from_numpy(m))
+    assert got.device.type == "cpu"
+    assert np.abs(got.numpy() - want).max() <= LOGP_ATOL * 4  # logits ~ +-100 here
+
+
+# ---------------------------------------------------------------- forward + backward
+
+def test_tiny_workload_fwd_bwd():
+    _check_fwd_bwd(_case(wl.WORKLOADS["tiny_fwdbwd"]))
+
+
+@pytest.mark.parametrize("agg_mode", [0, 1])
+def test_ragged_multi_chunk_fwd_bwd(agg_mode, monkeypatch):
+    monkeypatch.setenv("GRPO_VOCAB_CHUNK", "512")   # several backward chunks + a tail chunk
+    w = wl.Workload("t", 2, 4, 90, 320, 1800, "uniform", 1, 90, rewards="mix", seed=wl.SEED_BASE + 500)
+    _check_fwd_bwd(_case(w, agg_mode), agg_mode)
+
+
+def test_fwd_bwd_is_deterministic():
+    c = _case(wl.Workload("t", 1, 4, 70, 256, 2000, "uniform", 5, 70, seed=wl.SEED_BASE + 600))
+    a = _check_fwd_bwd(c)
+    b = _check_fwd_bwd(c)
+    for x, y in zip(a, b):
+        assert torch.equal(x, y)
+
+
+def test_one_token_per_response_and_zero_std_groups():
+    w = wl.Workload("t", 4, 4, 3, 128, 700, "uniform", 1, 1, rewards="bern", zero_std_every=2,
+                    seed=wl.SEED_BASE + 700)
+    c = _case(w)
+    assert c["m"].reshape(w.n_resp, w.L).sum(1).tolist() == [1] * w.n_resp
+    _check_fwd_bwd(c)
+
+
+def test_all_masked_batch():
+    w = wl.Workload("t", 1, 2, 40, 64, 500, seed=wl.SEED_BASE + 800)
+    c = _case(w)
+    d = _dev(c)
+    m0 = torch.zeros_like(d["m"])
+    loss, dH, dW = grpo.loss_fwd_bwd(d["H"], d["W"], d["y"], m0, d["old"], d["ref"], d["adv"], w.n_resp, w.L)
+    assert loss.item() == 0.0 and not dH.any() and not dW.any()
+    lp = grpo.token_logprobs(d["H"], d["W"], d["y"], m0)
+    assert not lp.any()
+
+
+def test_bad_target_sets_device_status():
+    w = wl.Workload("t", 1, 2, 40, 64, 500, seed=wl.SEED_BASE + 900)
+    c = _case(w)
+    d = _dev(c)
+    y = d["y"].clone()
+    y[3] = w.V + 5
+    ws = grpo.workspace(w.T, w.Hd, w.V, grpo.GRPO_WS_LOGPROBS, DEV)
+    lp = grpo.token_logprobs(d["H"], d["W"], y, d["m"], ws=ws)
+    assert grpo.check_device_status(ws) == grpo.GRPO_ERR_DEVICE_CHECK
+    assert lp[3].item() == 0.0
+    ok = np.flatnonzero(c["m"])
+    ok = ok[ok != 3]
+    want, _ = oracle.token_logprobs(c["H"], c["W"], c["y"], c["m"])
+    assert np.abs(lp.cpu().numpy()[ok] - want[ok]).max() <= LOGP_ATOL
+    # the next good call clears the word
+    grpo.token_logprobs(d["H"], d["W"], d["y"], d["m"], ws=ws)
+    assert grpo.check_device_status(ws) == grpo.GRPO_OK
+
+
+def test_invalid_group_size_rejected():
+    with pytest.raises(grpo.GrpoError) as e:
+        grpo.group_advantages(torch.zeros(8, device=DEV), 1)
+    assert e.value.status == grpo.GRPO_ERR_INVALID_ARG
