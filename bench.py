@@ -1,0 +1,423 @@
+#!/usr/bin/env python
+"""Benchmark of the GRPO hot path on GB300.
+
+One step = the group advantages (Eq. 2) followed by the fused log-prob, loss
+and backward call (Eq. 1 and its gradient to H and W) over one synthetic batch
+shaped like an 8B policy's rollout (workloads.py).  Prints one JSON line.
+
+    python bench.py [--steps K] [--warmup W] [--workload fwdbwd_8b]
+    python bench.py --impl reference ...      # the float64 CPU oracle, bounded sample
+    torchrun --nproc-per-node N bench.py --gpus N ...
+
+value: response (unmasked) tokens per second over all ranks, inputs resident
+in HBM; e2e: the same through the public API with pinned host buffers, the
+host<->device copies inside the timed region.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import workloads as wl  # noqa: E402
+
+METRIC = "response tokens/s for GRPO logprob+loss fwd+bwd; % of dense bf16 peak"
+GOLDEN = {"fwdbwd_8b": "batch8b", "logprob3_8b": "batch8b", "long_8b": "long_8b", "ragged_8b": "ragged_8b"}
+KERNEL_SOURCES = ["paper_2507_05687_gb300/csrc/gemm_tc.cuh", "paper_2507_05687_gb300/csrc/ptx.cuh"]
+KIND_NAMES = ["advantages", "compact", "lse_gemm", "logp_merge", "loss", "dz_gemm", "dh_gemm", "dw_gemm",
+              "zero_rows"]
+KERNELS_PER_SCOPE = {1: 4, 4: 2}  # compaction scope = 4 kernels, loss scope = 2 kernels; others 1
+
+
+def parse():
+    p = argparse.ArgumentParser()
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=10)
+    p.add_argument("--warmup", type=int, default=3)
+    p.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    p.add_argument("--workload", default="fwdbwd_8b", choices=sorted(wl.ALL_WORKLOADS))
+    p.add_argument("--no-e2e", action="store_true")
+    p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--cpu-sample-tokens", type=int, default=1024,
+                   help="tokens of the CPU-baseline sample (the reference arm uses a quarter per step)")
+    return p.parse_args()
+
+
+def peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            d = json.load(f)
+        return d["bf16_tflops"], d["bf16_tflops_sustained"], d["hbm_gbs"], "measured"
+    except (OSError, KeyError, ValueError):
+        return 1900.0, 1700.0, 6800.0, "fallback"
+
+
+def host_cores() -> int:
+    try:
+        return len(os.sched_getaffinity(0))
+    except AttributeError:
+        return os.cpu_count() or 1
+
+
+# ---------------------------------------------------------------- inputs
+
+def make_inputs(w: wl.Workload):
+    """Seeded host arrays of one batch, plus old/ref log-probs and where they came from."""
+    Hb, Wb = wl.gen_hidden(w), wl.gen_weight(w)
+    y, m, r = wl.gen_targets(w), wl.gen_mask(w), wl.gen_rewards(w)
+    old = np.zeros(w.T, np.float32)
+    ref = np.zeros(w.T, np.float32)
+    src = None
+    g = GOLDEN.get(w.name)
+    path = os.path.join(ROOT, "tests", "golden", f"{g}.npz") if g else None
+    if path and os.path.exists(path) and w.seed == wl.ALL_WORKLOADS[w.name].seed:
+        d = np.load(path)
+        idx = wl.valid_index(m)
+        if int(d["n_valid"]) == idx.size:
+            old[idx] = d["old_logp"]
+            ref[idx] = d["ref_logp"]
+            src = "float64 oracle on the perturbed heads (tests/golden)"
+    return dict(H=Hb, W=Wb, y=y, m=m, r=r, old=old, ref=ref, old_src=src)
+
+
+def fill_old_ref_on_gpu(w, inp, grpo, torch, dev):
+    """old/ref log-probs of the perturbed heads from the library's own forward
+    (what a GRPO pipeline does before the update); used when no stored oracle
+    values exist for this batch."""
+    Wold = wl.gen_weight(w, "old", inp["W"])
+    Wref = wl.gen_weight(w, "ref", inp["W"])
+    H = torch.from_numpy(inp["H"]).view(torch.bfloat16).to(dev)
+    y = torch.from_numpy(inp["y"]).to(dev)
+    m = torch.from_numpy(inp["m"]).to(dev)
+    for key, Wx in (("old", Wold), ("ref", Wref)):
+        lp = grpo.token_logprobs(H, torch.from_numpy(Wx).view(torch.bfloat16).to(dev), y, m)
+        inp[key] = lp.cpu().numpy()
+    inp["old_src"] = "library forward on the perturbed heads"
+
+
+# ---------------------------------------------------------------- clocks
+
+class ClockSampler:
+    """nvidia-smi clock / throttle samples while the timed region runs."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.out = tempfile.NamedTemporaryFile("w+", suffix=".csv", delete=False)
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.FIELDS}",
+                                          "--format=csv,noheader,nounits", "-lms", "100"],
+                                         stdout=self.out, stderr=subprocess.DEVNULL)
+        except OSError:
+            self.proc = None
+        time.sleep(0.3)
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        self.proc.wait()
+        self.out.flush()
+        self.out.seek(0)
+        rows = [l.strip().split(", ") for l in self.out if l.strip()]
+        os.unlink(self.out.name)
+        sm, mx, reasons = [], None, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for r in rows:
+            try:
+                sm.append(float(r[1]))
+                mx = float(r[2])
+                for n, v in zip(names, r[5:9]):
+                    if v.strip().lower() == "active":
+                        reasons.add(n)
+            except (ValueError, IndexError):
+                continue
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": mx, "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# ---------------------------------------------------------------- roofline
+
+def kernel_hash() -> str:
+    h = hashlib.sha256()
+    for p in KERNEL_SOURCES:
+        with open(os.path.join(ROOT, p), "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()[:16]
+
+
+def stored_traffic(kind_name: str):
+    """DRAM bytes per launch from the committed ncu summary, if it was taken on
+    the current kernel source (profiles/traffic.txt: '<hash> <kind> <bytes/launch> <cols>')."""
+    path = os.path.join(ROOT, "profiles", "traffic.txt")
+    if not os.path.exists(path):
+        return None
+    kh = kernel_hash()
+    for line in open(path):
+        f = line.split()
+        if len(f) >= 4 and f[0] == kh and f[1] == kind_name:
+            return float(f[2]), int(f[3])
+    return None
+
+
+def roofline(trace, n_valid_total_per_rank, Hd, steps, peak_tf, peak_kind):
+    by = {}
+    for kind, cols, ms in trace:
+        by.setdefault(kind, []).append((cols, ms))
+    gemm_kinds = [2, 5, 6, 7]
+    dom = max(gemm_kinds, key=lambda k: sum(ms for _, ms in by.get(k, [])) if k in by else -1)
+    recs = by[dom]
+    flops = [2.0 * n_valid_total_per_rank * Hd * cols for cols, _ in recs]
+    secs = [ms / 1e3 for _, ms in recs]
+    achieved = (sum(flops) / len(flops)) / (sum(secs) / len(secs)) / 1e12
+    total_ms = sum(ms for v in by.values() for _, ms in v)
+    shares = {KIND_NAMES[k]: round(sum(ms for _, ms in v) / total_ms, 4) for k, v in sorted(by.items())}
+    tr = stored_traffic(KIND_NAMES[dom])
+    traffic = None
+    if tr is not None:
+        bytes_per_launch, cols_ref = tr
+        avg_cols = sum(c for c, _ in recs) / len(recs)
+        traffic = bytes_per_launch * avg_cols / cols_ref
+    return {
+        "bound": "tensor", "kernel": KIND_NAMES[dom], "achieved": round(achieved, 1),
+        "peak": peak_tf, "peak_kind": peak_kind, "unit": "TFLOP/s", "frac": round(achieved / peak_tf, 4),
+        "traffic": traffic, "launches_per_step": len(recs) // max(1, steps),
+        "avg_launch_ms": round(sum(secs) / len(secs) * 1e3, 4), "time_share": shares,
+    }
+
+
+# ---------------------------------------------------------------- CPU oracle
+
+def cpu_oracle_sample(w, inp, n_tokens: int):
+    """Times the float64 oracle's forward + backward on the first n_tokens
+    unmasked tokens of the batch (whole responses from the start of the batch,
+    full vocabulary and hidden size)."""
+    import oracle
+    L = w.L
+    valid = np.flatnonzero(inp["m"])[:n_tokens]
+    k = int(valid[-1] // L) + 1 if valid.size else 1
+    m = np.zeros(k * L, np.uint8)
+    m[valid] = 1
+    adv = oracle.group_advantages(inp["r"], w.G, float(np.float32(w.adv_eps)))[:k]
+    sl = slice(0, k * L)
+    t0 = time.perf_counter()
+    oracle.loss_fwd_bwd(inp["H"][sl], inp["W"], inp["y"][sl], m, inp["old"][sl], inp["ref"][sl], adv, k, L,
+                        w.clip_eps, w.beta)
+    dt = time.perf_counter() - t0
+    return int(m.sum()), dt
+
+
+def run_reference(args):
+    """The float64 oracle on the host cores, one bounded sample per step."""
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    w = wl.ALL_WORKLOADS[args.workload]
+    inp = make_inputs(w)
+    ntok = max(1, args.cpu_sample_tokens // 4)
+    for _ in range(args.warmup):
+        cpu_oracle_sample(w, inp, ntok)
+    toks, secs = 0, 0.0
+    for _ in range(args.steps):
+        n, dt = cpu_oracle_sample(w, inp, ntok)
+        toks += n
+        secs += dt
+    value = toks / secs
+    sample = (f"first {toks // max(1, args.steps)} valid tokens of {w.name} per step: "
+              f"oracle.loss_fwd_bwd in float64, full vocabulary and hidden size")
+    line = {
+        "impl": "reference", "metric": METRIC, "value": round(value, 2), "unit": "tokens/s",
+        "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": round(secs / args.steps * 1e3, 1), "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": w.name, "sample": sample},
+        "cpu_baseline": {"value": round(value, 2), "unit": "tokens/s", "cores": host_cores(), "kind": "oracle",
+                         "sample": sample},
+        "e2e": {"value": round(value, 2), "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+# ---------------------------------------------------------------- GPU arm
+
+def main():
+    args = parse()
+    if args.impl == "reference":
+        run_reference(args)
+        return
+    import torch
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+
+    from paper_2507_05687_gb300 import build as build_mod
+    build_mod.build()
+    import paper_2507_05687_gb300 as grpo
+    lib = grpo.load()
+
+    base = wl.ALL_WORKLOADS[args.workload]
+    w = base if rank == 0 else base.with_(seed=base.seed + 7919 * rank)
+    inp = make_inputs(w)
+    if inp["old_src"] is None:
+        fill_old_ref_on_gpu(w, inp, grpo, torch, dev)
+    n_valid = int(inp["m"].sum())
+
+    def to_dev(a, dt):
+        return torch.from_numpy(np.ascontiguousarray(a)).view(dt).to(dev)
+
+    H, W = to_dev(inp["H"], torch.bfloat16), to_dev(inp["W"], torch.bfloat16)
+    y, m = to_dev(inp["y"], torch.int32), to_dev(inp["m"], torch.uint8)
+    old, ref, r = to_dev(inp["old"], torch.float32), to_dev(inp["ref"], torch.float32), to_dev(inp["r"], torch.float32)
+    ws = grpo.workspace(w.T, w.Hd, w.V, grpo.GRPO_WS_LOSS, dev)
+    adv = torch.empty(w.n_resp, dtype=torch.float32, device=dev)
+    out = (torch.empty(1, dtype=torch.float32, device=dev), torch.empty(w.T, w.Hd, dtype=torch.float32, device=dev),
+           torch.empty(w.V, w.Hd, dtype=torch.float32, device=dev))
+
+    def step():
+        grpo.group_advantages(r, w.G, w.adv_eps, out=adv)
+        grpo.loss_fwd_bwd(H, W, y, m, old, ref, adv, w.n_resp, w.L, w.clip_eps, w.beta, 0, ws=ws, out=out)
+        if dist is not None:
+            dist.all_reduce(out[2])  # data-parallel exchange of the LM-head gradient
+
+    for _ in range(max(3, args.warmup)):
+        step()
+    st = grpo.check_device_status(ws)
+    if st != grpo.GRPO_OK:
+        raise SystemExit(f"device status after warm-up: {grpo.status_string(st)}")
+
+    stream = torch.cuda.current_stream(dev)
+    sampler = ClockSampler(local) if rank == 0 else None
+    if dist is not None:
+        dist.barrier()
+    torch.cuda.synchronize(dev)
+    if sampler:
+        sampler.start()
+    lib.grpo_trace_enable(1)
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    ev0.record(stream)
+    for _ in range(args.steps):
+        step()
+    ev1.record(stream)
+    torch.cuda.synchronize(dev)
+    lib.grpo_trace_enable(0)
+    if dist is not None:
+        dist.barrier()
+    clocks = sampler.stop() if sampler else None
+    ms = ev0.elapsed_time(ev1) / args.steps
+
+    import ctypes
+    nrec = lib.grpo_trace_read(None, None, None, 0)
+    kinds = (ctypes.c_int32 * nrec)()
+    cols = (ctypes.c_int64 * nrec)()
+    kms = (ctypes.c_float * nrec)()
+    lib.grpo_trace_read(kinds, cols, kms, nrec)
+    trace = [(kinds[i], cols[i], kms[i]) for i in range(nrec)]
+    launches = sum(KERNELS_PER_SCOPE.get(k, 1) for k, _, _ in trace)
+    st = grpo.check_device_status(ws)
+    if st != grpo.GRPO_OK:
+        raise SystemExit(f"device status after timing: {grpo.status_string(st)}")
+
+    tot_valid = n_valid
+    if dist is not None:
+        t = torch.tensor([ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = t.item()
+        n = torch.tensor([n_valid], device=dev, dtype=torch.float64)
+        dist.all_reduce(n)
+        tot_valid = int(n.item())
+    value = tot_valid / (ms / 1e3)
+
+    burst, sustained, hbm, peak_src = peaks()
+    rf = roofline(trace, n_valid, w.Hd, args.steps, sustained, f"bf16 sustained, {peak_src}")
+    step_flops8 = 8.0 * n_valid * w.Hd * w.V
+    step_flops6 = 6.0 * n_valid * w.Hd * w.V
+
+    e2e = None
+    if not args.no_e2e and rank == 0:
+        e2e = measure_e2e(grpo, torch, dev, w, inp, steps=min(args.steps, 5))
+
+    cpu = None
+    if not args.no_cpu_baseline and rank == 0 and world == 1:
+        ntok, dt = cpu_oracle_sample(w, inp, args.cpu_sample_tokens)
+        cpu = {"value": round(ntok / dt, 2), "unit": "tokens/s", "cores": host_cores(), "kind": "oracle",
+               "sample": f"first {ntok} valid tokens of {w.name}: oracle.loss_fwd_bwd in "
+                         f"float64 over the full vocabulary and hidden size, {dt:.1f} s"}
+
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": round(value, 1), "unit": "tokens/s", "n_gpus": world,
+            "steps": args.steps, "warmup": max(3, args.warmup), "ms_per_step": round(ms, 3),
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+            "data": "synthetic",
+            "config": {"workload": w.name, "prompts": w.n_prompts, "G": w.G, "L": w.L, "Hd": w.Hd, "V": w.V,
+                       "tokens": w.T, "n_valid": n_valid, "global_valid_tokens": tot_valid,
+                       "parallelism": f"dp{world}",
+                       "l2": "inputs larger than L2 (W %.2f GB, H %.2f GB per rank)" % (w.V * w.Hd * 2 / 1e9,
+                                                                                         w.T * w.Hd * 2 / 1e9),
+                       "old_ref_logp": inp["old_src"]},
+            "step_tflops_8x": round(step_flops8 / (ms / 1e3) / 1e12, 1),
+            "step_frac_8x": round(step_flops8 / (ms / 1e3) / 1e12 / burst, 4),
+            "step_frac_6x": round(step_flops6 / (ms / 1e3) / 1e12 / burst, 4),
+            "roofline": rf, "clocks": clocks, "gpu_launches": launches, "e2e": e2e, "cpu_baseline": cpu,
+        }
+        print(json.dumps(line), flush=True)
+    if dist is not None:
+        dist.destroy_process_group()
+
+
+def measure_e2e(grpo, torch, dev, w, inp, steps: int):
+    """Public API with pinned host buffers: H2D of the batch, the step, D2H of loss, dH, dW."""
+    def pin(a, dt):
+        t = torch.from_numpy(np.ascontiguousarray(a)).view(dt)
+        return t.pin_memory()
+
+    hH, hW = pin(inp["H"], torch.bfloat16), pin(inp["W"], torch.bfloat16)
+    hy, hm = pin(inp["y"], torch.int32), pin(inp["m"], torch.uint8)
+    hold, href, hr = pin(inp["old"], torch.float32), pin(inp["ref"], torch.float32), pin(inp["r"], torch.float32)
+    h2d = sum(t.numel() * t.element_size() for t in (hH, hW, hy, hm, hold, href, hr))
+    d2h = 4 + w.T * w.Hd * 4 + w.V * w.Hd * 4
+
+    def one():
+        adv = grpo.group_advantages(hr.to(dev, non_blocking=True), w.G, w.adv_eps)
+        return grpo.loss_fwd_bwd(hH, hW, hy, hm, hold, href, adv, w.n_resp, w.L, w.clip_eps, w.beta)
+
+    one()
+    torch.cuda.synchronize(dev)
+    t0 = time.perf_counter()
+    for _ in range(steps):
+        loss, dH, dW = one()   # returns pinned host tensors once they have landed
+    dt = (time.perf_counter() - t0) / steps
+    n_valid = int(inp["m"].sum())
+    return {"value": round(n_valid / dt, 1), "unit": "tokens/s", "ms_per_step": round(dt * 1e3, 2),
+            "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h), "steps": steps}
+
+
+if __name__ == "__main__":
+    main()

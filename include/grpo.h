@@ -126,6 +126,41 @@ grpo_status grpo_check_device_status(void* ws, void* stream);
 /* Static, human-readable name of a status code. */
 const char* grpo_status_string(grpo_status status);
 
+/*
+ * Launch tracing (profiling aid; the paper has no counterpart).
+ * Kernel classes reported by grpo_trace_read:
+ */
+enum {
+  GRPO_K_ADVANTAGES = 0,  /* Eq. 2 reduction */
+  GRPO_K_COMPACT = 1,     /* mask scan / scatter and the gather of unmasked rows */
+  GRPO_K_LSE_GEMM = 2,    /* logits GEMM + online log-sum-exp + target gather */
+  GRPO_K_LOGP_MERGE = 3,  /* merge of vocabulary splits -> logp */
+  GRPO_K_LOSS = 4,        /* merge + Eq. 1 terms, dloss/dlogp, loss reduction */
+  GRPO_K_DZ_GEMM = 5,     /* recomputed logits -> dZ chunk (bf16) */
+  GRPO_K_DH_GEMM = 6,     /* dH (+)= dZ_chunk W_chunk */
+  GRPO_K_DW_GEMM = 7,     /* dW_chunk = dZ_chunk^T H */
+  GRPO_K_ZERO_ROWS = 8    /* zero dH rows of padding tokens */
+};
+
+/*
+ * enable != 0: from now on, every kernel launch of the compute calls (from
+ * any host thread) is bracketed by two CUDA events recorded on its stream;
+ * the record is cleared.  enable == 0 stops recording (the record is kept).
+ * Events are created on first use and reused; tracing costs two event
+ * records per launch and nothing when disabled.
+ */
+grpo_status grpo_trace_enable(int32_t enable);
+
+/*
+ * Waits for the traced launches to finish and writes up to max_records of
+ * them, oldest first: kind[i] (GRPO_K_*), cols[i] (vocabulary columns the
+ * launch covered, or 0) and ms[i] (device time between its two events).
+ * Returns the total number of records (may exceed max_records), or -1 if an
+ * event query failed.  Pointers are host memory; any may be NULL when
+ * max_records is 0.
+ */
+int32_t grpo_trace_read(int32_t* kind, int64_t* cols, float* ms, int32_t max_records);
+
 #ifdef __cplusplus
 }
 #endif

@@ -48,7 +48,7 @@ def as_f64(x) -> np.ndarray:
     x = np.asarray(x)
     if x.dtype == np.uint16:
         return widen_bf16(x)
-    return x.astype(np.float64)
+    return np.asarray(x, dtype=np.float64)
 
 
 # ---------------------------------------------------------------------------

@@ -43,6 +43,8 @@ SIGNATURES = {
     "grpo_workspace_bytes": (ctypes.c_size_t, [_I64, _I32, _I64, _I32]),
     "grpo_check_device_status": (ctypes.c_int, [_P, _P]),
     "grpo_status_string": (ctypes.c_char_p, [ctypes.c_int]),
+    "grpo_trace_enable": (ctypes.c_int, [_I32]),
+    "grpo_trace_read": (ctypes.c_int32, [_P, _P, _P, _I32]),
 }
 
 _lib: Optional[ctypes.CDLL] = None

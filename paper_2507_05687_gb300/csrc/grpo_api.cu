@@ -8,6 +8,7 @@
 #include <cstdlib>
 #include <cstring>
 #include <mutex>
+#include <vector>
 
 #include "../../include/grpo.h"
 #include "gemm_tc.cuh"
@@ -148,6 +149,62 @@ bool device_info(DeviceInfo* out) {
   return true;
 }
 
+// ---------------------------------------------------------------- tracing
+
+struct TraceRec {
+  int32_t kind;
+  int64_t cols;
+  cudaEvent_t start, stop;
+};
+
+struct Tracer {
+  std::mutex mu;
+  bool on = false;
+  std::vector<TraceRec> recs;   // recorded launches
+  std::vector<cudaEvent_t> pool;  // created events, reused across records
+  size_t used = 0;
+
+  cudaEvent_t next_event() {
+    if (used == pool.size()) {
+      cudaEvent_t e = nullptr;
+      if (cudaEventCreate(&e) != cudaSuccess) return nullptr;
+      pool.push_back(e);
+    }
+    return pool[used++];
+  }
+};
+
+Tracer& tracer() {
+  static Tracer* t = new Tracer();  // never destroyed: events may outlive static teardown
+  return *t;
+}
+
+// Brackets the launches made in its lifetime with two events when tracing is on.
+class TraceScope {
+ public:
+  TraceScope(int32_t kind, int64_t cols, cudaStream_t s) : s_(s) {
+    Tracer& t = tracer();
+    std::lock_guard<std::mutex> lk(t.mu);
+    if (!t.on) return;
+    rec_.kind = kind;
+    rec_.cols = cols;
+    rec_.start = t.next_event();
+    rec_.stop = t.next_event();
+    if (rec_.start && rec_.stop && cudaEventRecord(rec_.start, s) == cudaSuccess) active_ = true;
+  }
+  ~TraceScope() {
+    if (!active_) return;
+    Tracer& t = tracer();
+    std::lock_guard<std::mutex> lk(t.mu);
+    if (cudaEventRecord(rec_.stop, s_) == cudaSuccess) t.recs.push_back(rec_);
+  }
+
+ private:
+  cudaStream_t s_;
+  TraceRec rec_{};
+  bool active_ = false;
+};
+
 template <int E, bool A, bool B>
 cudaError_t launch_gemm(const CUtensorMap& ta, const CUtensorMap& tb, const GemmArgs& a,
                         int64_t max_units, int sms, cudaStream_t s) {
@@ -171,6 +228,7 @@ cudaError_t run_compaction(const uint16_t* H, const int32_t* targets, const uint
   int* n_valid = at<int>(ws, Ly.n_valid);
   cudaError_t e = cudaMemsetAsync(status, 0, 8, s);  // status word and n_valid
   if (e != cudaSuccess) return e;
+  TraceScope trace(GRPO_K_COMPACT, 0, s);
   if (T > 0) {
     const int nb = static_cast<int>(Ly.nblk_scan);
     mask_count_kernel<<<nb, kScanThreads, 0, s>>>(mask, T, at<int>(ws, Ly.counts));
@@ -207,6 +265,7 @@ cudaError_t run_lse(const uint16_t* W, int32_t Hd, int64_t V, void* ws, const La
   a.zy = at<float>(ws, Ly.zy);
   a.ldp = Ly.T_pad;
   const int64_t max_units = (Ly.T_pad / kBM) * Ly.nsplit;
+  TraceScope trace(GRPO_K_LSE_GEMM, V, s);
   return launch_gemm<kEpiLse, false, false>(tA, tB, a, max_units, sms, s);
 }
 
@@ -240,6 +299,7 @@ grpo_status grpo_group_advantages(const float* rewards, int64_t n_resp, int32_t 
   if (n_resp == 0) return GRPO_OK;
   if (!rewards || !adv_out) return GRPO_ERR_INVALID_ARG;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
+  TraceScope trace(GRPO_K_ADVANTAGES, 0, s);
   if (G <= 32 && (G & (G - 1)) == 0) {
     const int64_t blocks = (n_resp + 255) / 256;
     adv_segmented_kernel<<<static_cast<unsigned>(blocks), 256, 0, s>>>(rewards, n_resp, G, eps, adv_out);
@@ -269,6 +329,7 @@ grpo_status grpo_token_logprobs(const uint16_t* H, const uint16_t* W, const int3
   if (e == cudaSuccess) e = run_lse(W, Hd, V, ws, Ly, di.sms, s);
   if (e == cudaSuccess) {
     const int blocks = static_cast<int>(std::min<int64_t>((T + 255) / 256, di.sms * 16));
+    TraceScope trace(GRPO_K_LOGP_MERGE, 0, s);
     logp_merge_kernel<<<blocks, 256, 0, s>>>(mask, at<int>(ws, Ly.rank_of), T, at<float>(ws, Ly.part_m),
                                              at<float>(ws, Ly.part_s), static_cast<int>(Ly.nsplit),
                                              Ly.T_pad, at<float>(ws, Ly.zy), at<int>(ws, Ly.yc),
@@ -304,18 +365,24 @@ grpo_status grpo_loss_fwd_bwd(const uint16_t* H, const uint16_t* W, const int32_
 
   cudaError_t e = run_compaction(H, targets, mask, T, Hd, V, ws, Ly, sms, s);
   if (e == cudaSuccess && agg_mode == GRPO_AGG_SEQ_MEAN) {
+    TraceScope trace(GRPO_K_COMPACT, 0, s);
     const int64_t blocks = (n_resp * 32 + 255) / 256;
     resp_len_kernel<<<static_cast<unsigned>(blocks), 256, 0, s>>>(mask, n_resp, L, at<int>(ws, Ly.resp_len));
     e = cudaGetLastError();
   }
   if (e == cudaSuccess) e = run_lse(W, Hd, V, ws, Ly, sms, s);
   if (e == cudaSuccess) {
+    TraceScope trace(GRPO_K_LOSS, 0, s);
     loss_terms_kernel<<<static_cast<unsigned>(Ly.nblk_loss), kLossThreads, 0, s>>>(
         at<int>(ws, Ly.cidx), n_valid, at<float>(ws, Ly.part_m), at<float>(ws, Ly.part_s),
         static_cast<int>(Ly.nsplit), Ly.T_pad, at<float>(ws, Ly.zy), at<int>(ws, Ly.yc), old_logp,
         ref_logp, adv, L, at<int>(ws, Ly.resp_len), n_resp, agg_mode, clip_eps, beta,
         at<float>(ws, Ly.lse_c), at<float>(ws, Ly.g_c), at<double>(ws, Ly.block_loss), status);
     loss_final_kernel<<<1, 1024, 0, s>>>(at<double>(ws, Ly.block_loss), n_valid, kLossThreads, loss_out);
+    e = cudaGetLastError();
+  }
+  if (e == cudaSuccess) {
+    TraceScope trace(GRPO_K_ZERO_ROWS, 0, s);
     const int zb = static_cast<int>(std::min<int64_t>((T + 7) / 8, sms * 8));
     zero_masked_rows_kernel<<<zb, 256, 0, s>>>(mask, T, Hd, dH);
     e = cudaGetLastError();
@@ -350,7 +417,10 @@ grpo_status grpo_loss_fwd_bwd(const uint16_t* H, const uint16_t* W, const int32_
     a.gcoef = at<float>(ws, Ly.g_c);
     a.dz = dz;
     a.ldz = vc;
-    e = launch_gemm<kEpiDz, false, false>(tHcK, tWK, a, mt_max * ((width + kBN - 1) / kBN), sms, s);
+    {
+      TraceScope trace(GRPO_K_DZ_GEMM, width, s);
+      e = launch_gemm<kEpiDz, false, false>(tHcK, tWK, a, mt_max * ((width + kBN - 1) / kBN), sms, s);
+    }
     if (e != cudaSuccess) break;
     // dH (+)= dZ_c W_c
     GemmArgs h{};
@@ -366,7 +436,10 @@ grpo_status grpo_loss_fwd_bwd(const uint16_t* H, const uint16_t* W, const int32_
     h.ldo = Hd;
     h.accumulate = c0 > 0;
     h.row_map = at<int>(ws, Ly.cidx);
-    e = launch_gemm<kEpiF32, false, true>(tDzK, tWMN, h, mt_max * hd_tiles, sms, s);
+    {
+      TraceScope trace(GRPO_K_DH_GEMM, width, s);
+      e = launch_gemm<kEpiF32, false, true>(tDzK, tWMN, h, mt_max * hd_tiles, sms, s);
+    }
     if (e != cudaSuccess) break;
     // dW_c = dZ_c^T Hc
     GemmArgs w{};
@@ -380,9 +453,44 @@ grpo_status grpo_loss_fwd_bwd(const uint16_t* H, const uint16_t* W, const int32_
     w.out = dW + c0 * Hd;
     w.ldo = Hd;
     w.accumulate = 0;
+    TraceScope trace(GRPO_K_DW_GEMM, width, s);
     e = launch_gemm<kEpiF32, true, true>(tDzMN, tHcMN, w, ((width + kBM - 1) / kBM) * hd_tiles, sms, s);
   }
   return from_cuda(e);
+}
+
+grpo_status grpo_trace_enable(int32_t enable) {
+  Tracer& t = tracer();
+  std::lock_guard<std::mutex> lk(t.mu);
+  if (enable) {
+    t.recs.clear();
+    t.used = 0;
+    // create events up front so the first traced launches do not pay for it
+    while (t.pool.size() < 1024) {
+      cudaEvent_t e = nullptr;
+      if (cudaEventCreate(&e) != cudaSuccess) break;
+      t.pool.push_back(e);
+    }
+  }
+  t.on = enable != 0;
+  return GRPO_OK;
+}
+
+int32_t grpo_trace_read(int32_t* kind, int64_t* cols, float* ms, int32_t max_records) {
+  Tracer& t = tracer();
+  std::lock_guard<std::mutex> lk(t.mu);
+  const int32_t n = static_cast<int32_t>(t.recs.size());
+  for (int32_t i = 0; i < n && i < max_records; ++i) {
+    const TraceRec& r = t.recs[i];
+    float dt = 0.f;
+    if (cudaEventSynchronize(r.stop) != cudaSuccess ||
+        cudaEventElapsedTime(&dt, r.start, r.stop) != cudaSuccess)
+      return -1;
+    if (kind) kind[i] = r.kind;
+    if (cols) cols[i] = r.cols;
+    if (ms) ms[i] = dt;
+  }
+  return n;
 }
 
 grpo_status grpo_check_device_status(void* ws, void* stream) {

@@ -1,0 +1,152 @@
+"""GPU parity at the full 8B-shaped sizes (hidden 4096, vocabulary 155136),
+in the launch configuration bench.py times.
+
+The float64 oracle's log-sum-exp of every unmasked token (and the old /
+reference log-probs, which are inputs of the loss) were written once by
+tests/golden/make_golden.py, which calls only oracle/.  From them:
+
+* logp: every token, |dlogp| <= 2e-3;
+* loss: exact oracle loss over all tokens (O(T) from the stored values);
+* dH: sampled rows the oracle computes one by one (full vocabulary sweep);
+* dW: sampled vocabulary rows (a sum over all tokens), plus the invariant
+  sum_v dW[v, :] = 0 on the whole GPU output.
+"""
+import os
+
+import numpy as np
+import pytest
+
+import oracle
+import workloads as wl
+from tests._util import GRAD_RTOL, LOGP_ATOL, LOSS_RTOL, dev_tensor, loss_scale, rel_fro
+
+torch = pytest.importorskip("torch")
+pytestmark = pytest.mark.gpu
+
+if not torch.cuda.is_available():  # pragma: no cover
+    pytest.skip("needs a CUDA GPU", allow_module_level=True)
+
+import paper_2507_05687_gb300 as grpo  # noqa: E402
+from paper_2507_05687_gb300 import build as build_mod  # noqa: E402
+
+build_mod.build()
+DEV = torch.device("cuda", 0)
+GOLDEN_DIR = os.path.join(os.path.dirname(os.path.abspath(__file__)), "golden")
+BATCH = {"logprob3_8b": "batch8b", "fwdbwd_8b": "batch8b", "long_8b": "long_8b", "ragged_8b": "ragged_8b"}
+
+
+def _load(name):
+    path = os.path.join(GOLDEN_DIR, BATCH[name] + ".npz")
+    if not os.path.exists(path):
+        pytest.skip(f"stored oracle values {path} not generated")
+    return np.load(path)
+
+
+def _inputs(w, gold):
+    Hb, Wb, y, m = wl.gen_hidden(w), wl.gen_weight(w), wl.gen_targets(w), wl.gen_mask(w)
+    idx = wl.valid_index(m)
+    # the regenerated inputs must be the ones the stored values were computed on
+    assert idx.size == int(gold["n_valid"])
+    assert np.uint64(Hb[idx].astype(np.uint64).sum()) == gold["ck_h"]
+    assert np.uint64(Wb.astype(np.uint64).sum()) == gold["ck_w"]
+    assert np.uint64(y[idx].astype(np.uint64).sum()) == gold["ck_y"]
+    return Hb, Wb, y, m, idx
+
+
+def _target_logits(Hb, Wb, y, idx, chunk=16384):
+    """z_{t, y_t} = H_t . W_{y_t} in float64 for the listed rows."""
+    out = np.empty(idx.size)
+    for a in range(0, idx.size, chunk):
+        rows = idx[a:a + chunk]
+        out[a:a + chunk] = np.einsum("ij,ij->i", oracle.widen_bf16(Hb[rows]), oracle.widen_bf16(Wb[y[rows]]))
+    return out
+
+
+def _oracle_logp(Hb, Wb, y, idx, lse):
+    return _target_logits(Hb, Wb, y, idx) - lse
+
+
+def test_logprob_three_heads_full_size():
+    """Config: 8 prompts x G=8 x 512 tokens, policy / old / reference heads."""
+    w = wl.WORKLOADS["logprob3_8b"]
+    gold = _load(w.name)
+    Hb, Wb, y, m, idx = _inputs(w, gold)
+    H, yd, md = dev_tensor(Hb, torch.bfloat16), dev_tensor(y, torch.int32), dev_tensor(m, torch.uint8)
+    ws = grpo.workspace(w.T, w.Hd, w.V, grpo.GRPO_WS_LOGPROBS, DEV)
+    want = {"policy": _oracle_logp(Hb, Wb, y, idx, gold["lse_policy"]),
+            "old": gold["old_logp"].astype(np.float64), "ref": gold["ref_logp"].astype(np.float64)}
+    for which in ("policy", "old", "ref"):
+        Wx = Wb if which == "policy" else wl.gen_weight(w, which, Wb)
+        lp = grpo.token_logprobs(H, dev_tensor(Wx, torch.bfloat16), yd, md, ws=ws)
+        assert grpo.check_device_status(ws) == grpo.GRPO_OK
+        got = lp.cpu().numpy()
+        assert np.all(got[m == 0] == 0.0)
+        err = np.abs(got[idx].astype(np.float64) - want[which])
+        assert err.max() <= LOGP_ATOL, (which, err.max())
+        del Wx
+
+
+def _sample_rows(w, m, idx, r, k=96):
+    """Sampled compacted positions: first/last tokens, shortest and longest
+    responses, zero-std groups, plus a seeded random draw."""
+    lens = m.reshape(w.n_resp, w.L).sum(1)
+    must = [idx[0], idx[-1]]
+    for i in (int(np.argmin(lens)), int(np.argmax(lens))):
+        must += [i * w.L, i * w.L + lens[i] - 1]
+    zs = np.flatnonzero(r.reshape(w.n_prompts, w.G).std(1) == 0)
+    for g in zs[:2]:
+        must.append(g * w.G * w.L)
+    pos = wl.sample_rows(idx.size, k, w.seed)
+    rows = np.unique(np.concatenate([idx[pos], np.array(must, dtype=np.int64)]))
+    return rows[m[rows] != 0]
+
+
+@pytest.mark.parametrize("name", ["fwdbwd_8b", "long_8b", "ragged_8b"])
+def test_fwd_bwd_full_size(name):
+    w = wl.WORKLOADS[name]
+    gold = _load(name)
+    Hb, Wb, y, m, idx = _inputs(w, gold)
+    r = wl.gen_rewards(w)
+    old = np.zeros(w.T, np.float32)
+    ref = np.zeros(w.T, np.float32)
+    old[idx], ref[idx] = gold["old_logp"], gold["ref_logp"]
+    adv = oracle.group_advantages(r, w.G, float(np.float32(w.adv_eps)))
+
+    H, W = dev_tensor(Hb, torch.bfloat16), dev_tensor(Wb, torch.bfloat16)
+    ws = grpo.workspace(w.T, w.Hd, w.V, grpo.GRPO_WS_LOSS, DEV)
+    adv_d = grpo.group_advantages(dev_tensor(r, torch.float32), w.G, w.adv_eps)
+    assert np.array_equal(adv_d.cpu().numpy().view(np.uint32), adv.view(np.uint32))
+    loss, dH, dW = grpo.loss_fwd_bwd(H, W, dev_tensor(y, torch.int32), dev_tensor(m, torch.uint8),
+                                     dev_tensor(old, torch.float32), dev_tensor(ref, torch.float32), adv_d,
+                                     w.n_resp, w.L, w.clip_eps, w.beta, 0, ws=ws)
+    assert grpo.check_device_status(ws) == grpo.GRPO_OK
+
+    # loss over every token, from the stored oracle log-sum-exp
+    lse = np.zeros(w.T)
+    lse[idx] = gold["lse_policy"]
+    logp = np.zeros(w.T)
+    logp[idx] = _oracle_logp(Hb, Wb, y, idx, gold["lse_policy"])
+    want_loss, g, tt = oracle.grpo_loss(logp, old, ref, adv, m, w.n_resp, w.L, w.clip_eps, w.beta, 0)
+    scale = loss_scale(want_loss, tt["w"], tt["ell"])
+    assert abs(loss.item() - want_loss) <= LOSS_RTOL * scale, (loss.item(), want_loss, scale)
+
+    # dH on sampled rows; padding rows exactly zero
+    rows = _sample_rows(w, m, idx, r)
+    want_dH = oracle.dH_rows(Hb, Wb, y, lse, g, rows)
+    got_dH = dH[torch.from_numpy(rows).to(DEV)].double().cpu().numpy()
+    assert rel_fro(got_dH, want_dH) <= GRAD_RTOL, rel_fro(got_dH, want_dH)
+    pad = np.flatnonzero(m == 0)
+    if pad.size:
+        pr = pad[wl.sample_rows(pad.size, 256, w.seed + 1)]
+        assert not dH[torch.from_numpy(pr).to(DEV)].any()
+
+    # dW on sampled vocabulary rows (target hits included)
+    vrows = wl.sample_rows(w.V, 48, w.seed + 2, must=np.concatenate([[0, w.V - 1], y[idx[:16]]]))
+    want_dW = oracle.dW_rows(Hb, Wb, y, m, lse, g, vrows)
+    got_dW = dW[torch.from_numpy(vrows).to(DEV)].double().cpu().numpy()
+    assert rel_fro(got_dW, want_dW) <= GRAD_RTOL, rel_fro(got_dW, want_dW)
+
+    # sum_v dZ_{t,v} = 0 for every token, hence the columns of dW sum to ~0
+    colsum = dW.double().sum(0)
+    colabs = dW.double().abs().sum(0)
+    assert (colsum.norm() / colabs.norm()).item() <= 1e-2

@@ -95,6 +95,14 @@ WORKLOADS = {
                           rewards="mix", zero_std_every=4, seed=SEED_BASE + 5),
 }
 
+# Smaller cases of the same kernels, for profiler captures that must stay a
+# few GB on the device (inputs still larger than the 129 MB L2).
+PROFILE_WORKLOADS = {
+    "fwdbwd_small": Workload("fwdbwd_small", 2, 8, 512, 4096, 32768, "uniform", 128, 512,
+                             rewards="mix", seed=SEED_BASE + 6),
+}
+ALL_WORKLOADS = {**WORKLOADS, **PROFILE_WORKLOADS}
+
 
 def _rng(seed: int, stream: int, chunk: int = 0) -> np.random.Generator:
     return np.random.Generator(np.random.PCG64(np.random.SeedSequence([seed, stream, chunk])))
