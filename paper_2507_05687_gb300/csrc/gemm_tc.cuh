@@ -3,13 +3,15 @@
 //
 //   D[M x N] = A[M x K] * B[N x K]^T      (bf16 in, fp32 accumulate in TMEM)
 //
-// Roles (192 threads, one CTA per SM):
-//   warp 0      TMA producer: streams 128x64 A and 256x64 B k-blocks into a
-//               4-stage shared-memory ring (128-byte swizzle).
-//   warp 1      allocates 512 TMEM columns; one lane issues tcgen05.mma
-//               (128x256x16 per instruction) into one of two 256-column
-//               accumulators, so the epilogue of tile i overlaps the MMAs of
-//               tile i + 1.
+// Tile 128 x 256 per CTA (kPair = 1) or 256 x 256 per CTA pair (kPair = 2,
+// tcgen05 cta_group::2: each CTA stages its own 128 rows of A and half of B's
+// 256 columns, the even CTA issues the MMAs for both, and each CTA's TMEM
+// holds its 128 accumulator rows).  Roles per CTA (192 threads):
+//   warp 0      TMA producer: 64-wide k-blocks (128-byte swizzle) into a ring
+//               of shared-memory stages.
+//   warp 1      owns 512 TMEM columns (two 256-column accumulators, so the
+//               epilogue of tile i overlaps the MMAs of tile i + 1); one lane
+//               of the issuing CTA issues the 128x256x16 / 256x256x16 MMAs.
 //   warps 2..5  epilogue: one thread per accumulator row (TMEM lane), reading
 //               32 columns per tcgen05.ld.
 //
@@ -34,16 +36,23 @@
 
 namespace grpo {
 
-constexpr int kBM = 128;                 // accumulator rows (TMEM lanes)
-constexpr int kBN = 256;                 // accumulator columns per buffer
-constexpr int kBK = 64;                  // bf16 elements per 128-byte swizzle row
-constexpr int kStages = 4;
-constexpr int kABytes = kBM * kBK * 2;   // 16 KB
-constexpr int kBBytes = kBN * kBK * 2;   // 32 KB
-constexpr int kStageBytes = kABytes + kBBytes;
+constexpr int kBK = 64;            // bf16 elements per 128-byte swizzle row
+constexpr int kTileN = 256;        // accumulator columns per TMEM buffer
+constexpr int kRowsCta = 128;      // accumulator rows per CTA (TMEM lanes)
 constexpr int kGemmThreads = 192;
 constexpr int kTmemCols = 512;
-constexpr int kGemmSmemBytes = kStages * kStageBytes + 1024 /*align*/ + 256 /*barriers*/;
+constexpr int kRowAlign = 256;     // row padding of every token-indexed buffer
+
+template <int kPair>
+struct TileCfg {
+  static constexpr int kTileM = kRowsCta * kPair;       // rows of one tile
+  static constexpr int kBRows = kTileN / kPair;         // B rows (N) staged per CTA
+  static constexpr int kABytes = kRowsCta * kBK * 2;    // 16 KB
+  static constexpr int kBBytes = kBRows * kBK * 2;      // 32 KB (single) / 16 KB (pair)
+  static constexpr int kStageBytes = kABytes + kBBytes;
+  static constexpr int kStages = kPair == 2 ? 6 : 4;
+  static constexpr int kSmemBytes = kStages * kStageBytes + 1024 /*align*/ + 256 /*barriers*/;
+};
 
 enum { kEpiLse = 0, kEpiDz = 1, kEpiF32 = 2 };
 
@@ -53,7 +62,7 @@ struct GemmArgs {
   int m_dyn, k_dyn;
   int a_off_m, a_off_k; // coordinate offsets into A's tensor map
   int b_off_n, b_off_k; // coordinate offsets into B's tensor map
-  int n_per_unit;       // consecutive N tiles one CTA walks as one work unit
+  int n_per_unit;       // consecutive N tiles one CTA (pair) walks as one work unit
   int group_m;          // raster: M tiles per group sharing the same N sweep
   unsigned* status;     // device status word
 
@@ -78,16 +87,16 @@ struct GemmArgs {
 };
 
 struct TileSched {
-  int m_tiles, n_tiles, units_n, total, k_blocks;
+  int m_tiles, n_tiles, units_n, total, k_blocks, m_rows;
 };
 
-__device__ __forceinline__ TileSched make_sched(const GemmArgs& a) {
+__device__ __forceinline__ TileSched make_sched(const GemmArgs& a, int tile_m) {
   TileSched s;
   const int nv = *a.n_valid;
-  const int M = a.m_dyn ? nv : a.M;
+  s.m_rows = a.m_dyn ? nv : a.M;
   const int K = a.k_dyn ? nv : a.K;
-  s.m_tiles = (M + kBM - 1) / kBM;
-  s.n_tiles = (a.N + kBN - 1) / kBN;
+  s.m_tiles = (s.m_rows + tile_m - 1) / tile_m;
+  s.n_tiles = (a.N + kTileN - 1) / kTileN;
   s.units_n = (s.n_tiles + a.n_per_unit - 1) / a.n_per_unit;
   s.total = s.m_tiles * s.units_n;
   s.k_blocks = (K + kBK - 1) / kBK;
@@ -108,62 +117,213 @@ __device__ __forceinline__ void unit_coords(const GemmArgs& a, const TileSched& 
   un = w / gm;
 }
 
-template <int kEpi, bool kAmn, bool kBmn>
-__global__ void __launch_bounds__(kGemmThreads, 1)
-    gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
-                   const GemmArgs args) {
+// ---------------------------------------------------------------- epilogue
+
+// Per-row state of the epilogue for one work unit.
+struct EpiRow {
+  int r;          // accumulator row (compacted token / vocabulary row)
+  bool rv;        // row inside M
+  float run_m, run_s, zy_val;  // kEpiLse
+  bool found;
+  int y;
+  float lse2, gr;  // kEpiDz
+  int orow;        // kEpiF32
+};
+
+template <int kEpi>
+__device__ __forceinline__ void epi_begin(EpiRow& e, const GemmArgs& a, int r, int m_rows) {
+  const float kLog2e = 1.4426950408889634f;
+  e.r = r;
+  e.rv = r < m_rows;
+  e.run_m = -INFINITY;
+  e.run_s = 0.f;
+  e.zy_val = 0.f;
+  e.found = false;
+  e.y = -1;
+  e.lse2 = 0.f;
+  e.gr = 0.f;
+  e.orow = -1;
+  if (kEpi == kEpiLse) {
+    e.y = e.rv ? a.yc[r] : -1;
+  } else if (kEpi == kEpiDz) {
+    if (e.rv) {
+      e.y = a.yc[r];
+      e.lse2 = a.lse[r] * kLog2e;
+      e.gr = a.gcoef[r];
+    }
+  } else {
+    if (e.rv) e.orow = a.row_map ? a.row_map[r] : r;
+  }
+}
+
+// One 256-column accumulator tile of this thread's row; `tbase` is the TMEM
+// address of column 0 of the tile in this warp's lane quarter.
+template <int kEpi>
+__device__ __forceinline__ void epi_tile(EpiRow& e, const GemmArgs& a, uint32_t tbase, int col0,
+                                         bool have_acc) {
+  const float kLog2e = 1.4426950408889634f;
+#pragma unroll 1
+  for (int c = 0; c < kTileN / 32; ++c) {
+    float v[32];
+    if (have_acc) {
+      tmem_ld32(tbase + c * 32, v);
+    } else {
+#pragma unroll
+      for (int j = 0; j < 32; ++j) v[j] = 0.f;
+    }
+    const int cb = col0 + c * 32;
+    if (kEpi == kEpiLse) {
+      if (cb + 32 > a.N) {
+#pragma unroll
+        for (int j = 0; j < 32; ++j)
+          if (cb + j >= a.N) v[j] = -INFINITY;
+      }
+      const unsigned off = static_cast<unsigned>(e.y - cb);
+      if (off < 32u) {
+        float t = v[0];
+#pragma unroll
+        for (int j = 1; j < 32; ++j) t = (off == static_cast<unsigned>(j)) ? v[j] : t;
+        e.zy_val = t;
+        e.found = true;
+      }
+      float cm = v[0];
+#pragma unroll
+      for (int j = 1; j < 32; ++j) cm = fmaxf(cm, v[j]);
+      const float nm = fmaxf(e.run_m, cm * kLog2e);
+      float acc = 0.f;
+#pragma unroll
+      for (int j = 0; j < 32; ++j) acc += fast_exp2(fmaf(v[j], kLog2e, -nm));
+      e.run_s = e.run_s * fast_exp2(e.run_m - nm) + acc;
+      e.run_m = nm;
+    } else if (kEpi == kEpiDz) {
+      const int gc = a.b_off_n + cb;  // vocabulary id of column 0 of this group
+      uint32_t packed[16];
+#pragma unroll
+      for (int j = 0; j < 32; j += 2) {
+        float d0 = -e.gr * fast_exp2(fmaf(v[j], kLog2e, -e.lse2));
+        float d1 = -e.gr * fast_exp2(fmaf(v[j + 1], kLog2e, -e.lse2));
+        if (gc + j == e.y) d0 += e.gr;
+        if (gc + j + 1 == e.y) d1 += e.gr;
+        if (cb + j >= a.N || !e.rv) d0 = 0.f;
+        if (cb + j + 1 >= a.N || !e.rv) d1 = 0.f;
+        packed[j / 2] = pack_bf16x2(d0, d1);
+      }
+      uint4* dst = reinterpret_cast<uint4*>(a.dz + static_cast<long>(e.r) * a.ldz + cb);
+#pragma unroll
+      for (int q = 0; q < 4; ++q)
+        dst[q] = make_uint4(packed[4 * q], packed[4 * q + 1], packed[4 * q + 2], packed[4 * q + 3]);
+    } else {
+      if (e.rv) {
+        float* dst = a.out + static_cast<long>(e.orow) * a.ldo + cb;
+        if (cb + 32 <= a.N) {
+          float4* d4 = reinterpret_cast<float4*>(dst);
+#pragma unroll
+          for (int q = 0; q < 8; ++q) {
+            float4 o = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+            if (a.accumulate) {
+              const float4 p = d4[q];
+              o.x += p.x;
+              o.y += p.y;
+              o.z += p.z;
+              o.w += p.w;
+            }
+            d4[q] = o;
+          }
+        } else {
+#pragma unroll
+          for (int j = 0; j < 32; ++j)
+            if (cb + j < a.N) dst[j] = a.accumulate ? dst[j] + v[j] : v[j];
+        }
+      }
+    }
+  }
+}
+
+template <int kEpi>
+__device__ __forceinline__ void epi_end(const EpiRow& e, const GemmArgs& a, int un) {
+  if (kEpi == kEpiLse && e.rv) {
+    a.part_m[static_cast<long>(un) * a.ldp + e.r] = e.run_m;
+    a.part_s[static_cast<long>(un) * a.ldp + e.r] = e.run_s;
+    if (e.found) a.zy[e.r] = e.zy_val;
+  }
+}
+
+// ---------------------------------------------------------------- kernel body
+
+template <int kPair, int kEpi, bool kAmn, bool kBmn>
+__device__ __forceinline__ void gemm_body(const CUtensorMap* tmA, const CUtensorMap* tmB,
+                                          const GemmArgs& args) {
+  using C = TileCfg<kPair>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
-  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + kStages * kStageBytes);
-  uint64_t* full_bar = bars;                  // [kStages] TMA -> MMA
-  uint64_t* empty_bar = bars + kStages;       // [kStages] MMA -> TMA
-  uint64_t* tfull_bar = bars + 2 * kStages;   // [2] MMA -> epilogue
-  uint64_t* tempty_bar = bars + 2 * kStages + 2;  // [2] epilogue -> MMA
-  uint64_t* done_bar = bars + 2 * kStages + 4;    // [1] all MMAs retired
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * kStages + 5);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + C::kStages * C::kStageBytes);
+  uint64_t* full_bar = bars;                          // [kStages] TMA -> MMA (issuing CTA)
+  uint64_t* empty_bar = bars + C::kStages;            // [kStages] MMA -> TMA (each CTA)
+  uint64_t* tfull_bar = bars + 2 * C::kStages;        // [2] MMA -> epilogue (each CTA)
+  uint64_t* tempty_bar = bars + 2 * C::kStages + 2;   // [2] epilogue -> MMA (issuing CTA)
+  uint64_t* done_bar = bars + 2 * C::kStages + 4;     // [1] all MMAs retired (issuing CTA)
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * C::kStages + 5);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
+  const uint32_t rank = kPair == 2 ? cluster_ctarank() : 0u;
+  const bool issuer = rank == 0;
+  const int unit0 = blockIdx.x / kPair;
+  const int unit_stride = gridDim.x / kPair;
 
   if (threadIdx.x == 0) {
-    for (int i = 0; i < kStages; ++i) {
+    for (int i = 0; i < C::kStages; ++i) {
       mbar_init(smem_addr(&full_bar[i]), 1);
       mbar_init(smem_addr(&empty_bar[i]), 1);
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(smem_addr(&tfull_bar[i]), 1);
-      mbar_init(smem_addr(&tempty_bar[i]), 4 * 32);
+      mbar_init(smem_addr(&tempty_bar[i]), 4 * kPair);  // one arrival per epilogue warp
     }
     mbar_init(smem_addr(done_bar), 1);
     *abort_flag = 0;
     fence_mbar_init();
   }
   if (warp == 0 && lane == 0) {
-    tma_prefetch_desc(&tmA);
-    tma_prefetch_desc(&tmB);
+    tma_prefetch_desc(tmA);
+    tma_prefetch_desc(tmB);
   }
   if (warp == 1) {
-    tmem_alloc(smem_addr(tmem_slot), kTmemCols);
-    tmem_relinquish();
+    if (kPair == 2) {
+      tmem_alloc_pair(smem_addr(tmem_slot), kTmemCols);
+      tmem_relinquish_pair();
+    } else {
+      tmem_alloc(smem_addr(tmem_slot), kTmemCols);
+      tmem_relinquish();
+    }
   }
   tc_fence_before();
-  __syncthreads();
+  if (kPair == 2) cluster_sync(); else __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
 
-  const TileSched sch = make_sched(args);
+  const TileSched sch = make_sched(args, C::kTileM);
   const int KB = sch.k_blocks;
+
+  // Raises the abort flag of this CTA and of its peer.
+  auto raise_abort = [&]() {
+    *abort_flag = 1;
+    if (kPair == 2) st_shared_cluster(mapa_shared(smem_addr(const_cast<int*>(abort_flag)), rank ^ 1u), 1u);
+    atomicOr(args.status, kDevTimeout);
+  };
 
   if (warp == 0) {
     // ------------------------------------------------------------ producer
     if (lane == 0) {
       int stage = 0;
       uint32_t phase = 0;
-      int uses[kStages] = {0, 0, 0, 0};
+      int uses[C::kStages];
+#pragma unroll
+      for (int s = 0; s < C::kStages; ++s) uses[s] = 0;
       bool ok = true;
-      for (int u = blockIdx.x; u < sch.total && ok; u += gridDim.x) {
+      for (int u = unit0; u < sch.total && ok; u += unit_stride) {
         int mt, un;
         unit_coords(args, sch, u, mt, un);
         const int nt0 = un * args.n_per_unit;
@@ -174,53 +334,56 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
               ok = false;
               break;
             }
-            const uint32_t fb = smem_addr(&full_bar[stage]);
-            mbar_arrive_expect_tx(fb, kStageBytes);
-            const uint32_t sa = smem_addr(smem + stage * kStageBytes);
-            const uint32_t sb = sa + kABytes;
+            const uint32_t fb_local = smem_addr(&full_bar[stage]);
+            const uint32_t fb = kPair == 2 ? mapa_shared(fb_local, 0) : fb_local;
+            if (issuer) mbar_arrive_expect_tx(fb_local, kPair * C::kStageBytes);
+            const uint32_t sa = smem_addr(smem + stage * C::kStageBytes);
+            const uint32_t sb = sa + C::kABytes;
             const int k0 = kb * kBK;
-            const int m0 = mt * kBM;
-            const int n0 = nt * kBN;
+            const int m0 = mt * C::kTileM + static_cast<int>(rank) * kRowsCta;
+            const int n0 = nt * kTileN + static_cast<int>(rank) * C::kBRows;
+            auto load = [&](uint32_t dst, const CUtensorMap* map, int c0, int c1) {
+              if (kPair == 2) tma_load_2d_pair(dst, map, fb, c0, c1);
+              else tma_load_2d(dst, map, fb, c0, c1);
+            };
             if (!kAmn) {
-              tma_load_2d(sa, &tmA, fb, k0 + args.a_off_k, m0 + args.a_off_m);
+              load(sa, tmA, k0 + args.a_off_k, m0 + args.a_off_m);
             } else {
 #pragma unroll
-              for (int j = 0; j < kBM / 64; ++j)
-                tma_load_2d(sa + j * 8192, &tmA, fb, m0 + args.a_off_m + 64 * j, k0 + args.a_off_k);
+              for (int j = 0; j < kRowsCta / 64; ++j)
+                load(sa + j * 8192, tmA, m0 + args.a_off_m + 64 * j, k0 + args.a_off_k);
             }
             if (!kBmn) {
-              tma_load_2d(sb, &tmB, fb, k0 + args.b_off_k, n0 + args.b_off_n);
+              load(sb, tmB, k0 + args.b_off_k, n0 + args.b_off_n);
             } else {
 #pragma unroll
-              for (int j = 0; j < kBN / 64; ++j)
-                tma_load_2d(sb + j * 8192, &tmB, fb, n0 + args.b_off_n + 64 * j, k0 + args.b_off_k);
+              for (int j = 0; j < C::kBRows / 64; ++j)
+                load(sb + j * 8192, tmB, n0 + args.b_off_n + 64 * j, k0 + args.b_off_k);
             }
             ++uses[stage];
-            if (++stage == kStages) {
+            if (++stage == C::kStages) {
               stage = 0;
               phase ^= 1u;
             }
           }
         }
       }
-      if (!ok) {
-        *abort_flag = 1;
-        atomicOr(args.status, kDevTimeout);
-      }
-      // Let every copy this thread started land before the CTA can exit.
-      for (int s = 0; s < kStages; ++s)
+      if (!ok) raise_abort();
+      // Every stage this CTA filled must have been consumed (so its copies
+      // have landed) before the CTA can exit.
+      for (int s = 0; s < C::kStages; ++s)
         if (uses[s] > 0)
-          mbar_wait(smem_addr(&full_bar[s]), static_cast<uint32_t>(uses[s] - 1) & 1u, abort_flag);
+          mbar_wait(smem_addr(&empty_bar[s]), static_cast<uint32_t>(uses[s] - 1) & 1u, abort_flag);
     }
   } else if (warp == 1) {
     // ------------------------------------------------------------ MMA issuer
-    if (lane == 0) {
-      constexpr uint32_t idesc = idesc_bf16_f32(kBM, kBN, kAmn, kBmn);
+    if (lane == 0 && issuer) {
+      constexpr uint32_t idesc = idesc_bf16_f32(C::kTileM, kTileN, kAmn, kBmn);
       int stage = 0;
       uint32_t phase = 0;
       int tile = 0;
       bool ok = true;
-      for (int u = blockIdx.x; u < sch.total && ok; u += gridDim.x) {
+      for (int u = unit0; u < sch.total && ok; u += unit_stride) {
         int mt, un;
         unit_coords(args, sch, u, mt, un);
         const int nt0 = un * args.n_per_unit;
@@ -234,78 +397,62 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             break;
           }
           tc_fence_after();
-          const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(buf * kBN);
+          const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(buf * kTileN);
           for (int kb = 0; kb < KB; ++kb) {
             if (!mbar_wait(smem_addr(&full_bar[stage]), phase, abort_flag)) {
               ok = false;
               break;
             }
             tc_fence_after();
-            const uint32_t sa = smem_addr(smem + stage * kStageBytes);
-            const uint32_t sb = sa + kABytes;
+            const uint32_t sa = smem_addr(smem + stage * C::kStageBytes);
+            const uint32_t sb = sa + C::kABytes;
 #pragma unroll
             for (int kk = 0; kk < kBK / 16; ++kk) {
               const uint64_t ad = kAmn ? sdesc_sw128(sa + kk * 2048, 8192, 1024)
                                        : sdesc_sw128(sa + kk * 32, 16, 1024);
               const uint64_t bd = kBmn ? sdesc_sw128(sb + kk * 2048, 8192, 1024)
                                        : sdesc_sw128(sb + kk * 32, 16, 1024);
-              tc_mma_bf16(d_tmem, ad, bd, idesc, (kb | kk) != 0 ? 1u : 0u);
+              const uint32_t acc = (kb | kk) != 0 ? 1u : 0u;
+              if (kPair == 2) tc_mma_bf16_pair(d_tmem, ad, bd, idesc, acc);
+              else tc_mma_bf16(d_tmem, ad, bd, idesc, acc);
             }
-            tc_commit(smem_addr(&empty_bar[stage]));
-            if (++stage == kStages) {
+            if (kPair == 2) tc_commit_pair_mc(smem_addr(&empty_bar[stage]), 0x3);
+            else tc_commit(smem_addr(&empty_bar[stage]));
+            if (++stage == C::kStages) {
               stage = 0;
               phase ^= 1u;
             }
           }
           if (!ok) break;
-          tc_commit(smem_addr(&tfull_bar[buf]));
+          if (kPair == 2) tc_commit_pair_mc(smem_addr(&tfull_bar[buf]), 0x3);
+          else tc_commit(smem_addr(&tfull_bar[buf]));
           ++tile;
         }
       }
-      if (!ok) {
-        *abort_flag = 1;
-        atomicOr(args.status, kDevTimeout);
-      }
+      if (!ok) raise_abort();
       // Retire every MMA before TMEM is released.
-      tc_commit(smem_addr(done_bar));
+      if (kPair == 2) tc_commit_pair_mc(smem_addr(done_bar), 0x1);
+      else tc_commit(smem_addr(done_bar));
       mbar_wait(smem_addr(done_bar), 0, abort_flag);
     }
   } else {
     // ------------------------------------------------------------ epilogue
-    const int quad = warp & 3;             // TMEM lanes quad*32 .. quad*32+31
-    const int row = quad * 32 + lane;      // accumulator row of this thread
+    const int quad = warp & 3;  // TMEM lanes quad*32 .. quad*32+31
+    const int row = static_cast<int>(rank) * kRowsCta + quad * 32 + lane;  // row within the tile
     const uint32_t lane_addr = tmem_base + (static_cast<uint32_t>(quad * 32) << 16);
-    const int nv = *args.n_valid;
-    const int Mrows = args.m_dyn ? nv : args.M;
-    const float kLog2e = 1.4426950408889634f;
+    const uint32_t tempty0 = smem_addr(&tempty_bar[0]);
+    const uint32_t tempty1 = smem_addr(&tempty_bar[1]);
+    const uint32_t tempty_c0 = kPair == 2 ? mapa_shared(tempty0, 0) : tempty0;
+    const uint32_t tempty_c1 = kPair == 2 ? mapa_shared(tempty1, 0) : tempty1;
     int tile = 0;
     bool ok = true;
-    for (int u = blockIdx.x; u < sch.total && ok; u += gridDim.x) {
+    for (int u = unit0; u < sch.total && ok; u += unit_stride) {
       int mt, un;
       unit_coords(args, sch, u, mt, un);
       const int nt0 = un * args.n_per_unit;
       const int nt1 = min(sch.n_tiles, nt0 + args.n_per_unit);
-      const int r = mt * kBM + row;
-      const bool rv = r < Mrows;
-
-      // per-unit state of the log-softmax epilogue
-      float run_m = -INFINITY, run_s = 0.f, zy_val = 0.f;
-      bool found = false;
-      int y = -1;
-      float lse2 = 0.f, gr = 0.f;
-      int orow = -1;
-      if (kEpi == kEpiLse) {
-        y = rv ? args.yc[r] : -1;
-      } else if (kEpi == kEpiDz) {
-        if (rv) {
-          y = args.yc[r];
-          lse2 = args.lse[r] * kLog2e;
-          gr = args.gcoef[r];
-        }
-      } else {
-        if (rv) orow = args.row_map ? args.row_map[r] : r;
-      }
-
+      EpiRow e;
+      epi_begin<kEpi>(e, args, mt * C::kTileM + row, sch.m_rows);
       for (int nt = nt0; nt < nt1; ++nt) {
         const int buf = tile & 1;
         const uint32_t use = static_cast<uint32_t>(tile >> 1);
@@ -317,105 +464,47 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
           }
           tc_fence_after();
         }
-        const uint32_t tbase = lane_addr + static_cast<uint32_t>(buf * kBN);
-        const int col0 = nt * kBN;
-#pragma unroll 1
-        for (int c = 0; c < kBN / 32; ++c) {
-          float v[32];
-          if (have_acc) {
-            tmem_ld32(tbase + c * 32, v);
-          } else {
-#pragma unroll
-            for (int j = 0; j < 32; ++j) v[j] = 0.f;
-          }
-          const int cb = col0 + c * 32;
-          if (kEpi == kEpiLse) {
-            if (cb + 32 > args.N) {
-#pragma unroll
-              for (int j = 0; j < 32; ++j)
-                if (cb + j >= args.N) v[j] = -INFINITY;
-            }
-            const unsigned off = static_cast<unsigned>(y - cb);
-            if (off < 32u) {
-              float t = v[0];
-#pragma unroll
-              for (int j = 1; j < 32; ++j) t = (off == static_cast<unsigned>(j)) ? v[j] : t;
-              zy_val = t;
-              found = true;
-            }
-            float cm = v[0];
-#pragma unroll
-            for (int j = 1; j < 32; ++j) cm = fmaxf(cm, v[j]);
-            const float nm = fmaxf(run_m, cm * kLog2e);
-            float acc = 0.f;
-#pragma unroll
-            for (int j = 0; j < 32; ++j) acc += fast_exp2(fmaf(v[j], kLog2e, -nm));
-            run_s = run_s * fast_exp2(run_m - nm) + acc;
-            run_m = nm;
-          } else if (kEpi == kEpiDz) {
-            const int gc = args.b_off_n + cb;  // vocabulary id of column 0 of this group
-            uint32_t packed[16];
-#pragma unroll
-            for (int j = 0; j < 32; j += 2) {
-              float d0 = -gr * fast_exp2(fmaf(v[j], kLog2e, -lse2));
-              float d1 = -gr * fast_exp2(fmaf(v[j + 1], kLog2e, -lse2));
-              if (gc + j == y) d0 += gr;
-              if (gc + j + 1 == y) d1 += gr;
-              if (cb + j >= args.N || !rv) d0 = 0.f;
-              if (cb + j + 1 >= args.N || !rv) d1 = 0.f;
-              packed[j / 2] = pack_bf16x2(d0, d1);
-            }
-            uint4* dst = reinterpret_cast<uint4*>(args.dz + static_cast<long>(r) * args.ldz + cb);
-#pragma unroll
-            for (int q = 0; q < 4; ++q)
-              dst[q] = make_uint4(packed[4 * q], packed[4 * q + 1], packed[4 * q + 2], packed[4 * q + 3]);
-          } else {
-            if (rv) {
-              float* dst = args.out + static_cast<long>(orow) * args.ldo + cb;
-              if (cb + 32 <= args.N) {
-                float4* d4 = reinterpret_cast<float4*>(dst);
-#pragma unroll
-                for (int q = 0; q < 8; ++q) {
-                  float4 o = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
-                  if (args.accumulate) {
-                    const float4 p = d4[q];
-                    o.x += p.x; o.y += p.y; o.z += p.z; o.w += p.w;
-                  }
-                  d4[q] = o;
-                }
-              } else {
-#pragma unroll
-                for (int j = 0; j < 32; ++j)
-                  if (cb + j < args.N) dst[j] = args.accumulate ? dst[j] + v[j] : v[j];
-              }
-            }
-          }
-        }
+        epi_tile<kEpi>(e, args, lane_addr + static_cast<uint32_t>(buf * kTileN), nt * kTileN, have_acc);
         if (have_acc) {
           tc_fence_before();
-          mbar_arrive(smem_addr(&tempty_bar[buf]));
+          __syncwarp();
+          if (lane == 0) {
+            const uint32_t tb = buf ? tempty_c1 : tempty_c0;
+            if (kPair == 2) mbar_arrive_cluster(tb); else mbar_arrive(tb);
+          }
           ++tile;
         }
       }
       if (!ok) break;
-      if (kEpi == kEpiLse && rv) {
-        args.part_m[static_cast<long>(un) * args.ldp + r] = run_m;
-        args.part_s[static_cast<long>(un) * args.ldp + r] = run_s;
-        if (found) args.zy[r] = zy_val;
-      }
+      epi_end<kEpi>(e, args, un);
     }
-    if (!ok) {
-      *abort_flag = 1;
-      atomicOr(args.status, kDevTimeout);
-    }
+    if (!ok) raise_abort();
   }
 
+  // After a timeout, give copies that may still be in flight time to land
+  // before the shared memory they target is released.
+  if (*abort_flag) __nanosleep(200000);
   tc_fence_before();
-  __syncthreads();
+  if (kPair == 2) cluster_sync(); else __syncthreads();
   if (warp == 1) {
     tc_fence_after();
-    tmem_dealloc(tmem_base, kTmemCols);
+    if (kPair == 2) tmem_dealloc_pair(tmem_base, kTmemCols);
+    else tmem_dealloc(tmem_base, kTmemCols);
   }
+}
+
+template <int kEpi, bool kAmn, bool kBmn>
+__global__ void __launch_bounds__(kGemmThreads, 1)
+    gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+                   const GemmArgs args) {
+  gemm_body<1, kEpi, kAmn, kBmn>(&tmA, &tmB, args);
+}
+
+template <int kEpi, bool kAmn, bool kBmn>
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
+    gemm_tc_pair_kernel(const __grid_constant__ CUtensorMap tmA,
+                        const __grid_constant__ CUtensorMap tmB, const GemmArgs args) {
+  gemm_body<2, kEpi, kAmn, kBmn>(&tmA, &tmB, args);
 }
 
 }  // namespace grpo

@@ -47,8 +47,8 @@ bool make_layout(int64_t T, int32_t Hd, int64_t V, int32_t which, Layout* L) {
   if (T < 0 || T >= (int64_t(1) << 31) || Hd <= 0 || Hd % 64 != 0 || V <= 0 ||
       V >= (int64_t(1) << 31) || (which != GRPO_WS_LOGPROBS && which != GRPO_WS_LOSS))
     return false;
-  L->T_pad = round_up(std::max<int64_t>(T, 1), kBM);
-  const int64_t vtiles = (V + kBN - 1) / kBN;
+  L->T_pad = round_up(std::max<int64_t>(T, 1), kRowAlign);
+  const int64_t vtiles = (V + kTileN - 1) / kTileN;
   L->nsplit = (vtiles + kLseTilesPerUnit - 1) / kLseTilesPerUnit;
   L->nblk_scan = (std::max<int64_t>(T, 1) + kScanChunk - 1) / kScanChunk;
   L->nblk_loss = (L->T_pad + kLossThreads - 1) / kLossThreads;
@@ -116,8 +116,29 @@ bool encode_2d(CUtensorMap* map, const void* base, uint64_t rows, uint64_t cols,
 
 struct DeviceInfo {
   int sms = 0;
+  int pairs = 0;  // CTA pairs of the pair kernels that can be resident at once
   bool ok = false;
 };
+
+template <int E, bool A, bool B>
+bool prepare_kernels(int* pairs) {
+  if (cudaFuncSetAttribute(gemm_tc_kernel<E, A, B>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           TileCfg<1>::kSmemBytes) != cudaSuccess ||
+      cudaFuncSetAttribute(gemm_tc_pair_kernel<E, A, B>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           TileCfg<2>::kSmemBytes) != cudaSuccess)
+    return false;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(2 * 1024, 1, 1);
+  cfg.blockDim = dim3(kGemmThreads, 1, 1);
+  cfg.dynamicSmemBytes = TileCfg<2>::kSmemBytes;
+  int n = 0;
+  if (cudaOccupancyMaxActiveClusters(&n, gemm_tc_pair_kernel<E, A, B>, &cfg) != cudaSuccess) {
+    cudaGetLastError();  // clear: without the query the single-CTA tiles are used
+    n = 0;
+  }
+  *pairs = *pairs < 0 ? n : std::min(*pairs, n);
+  return true;
+}
 
 // Per-device facts and the one-time opt-in to large dynamic shared memory.
 bool device_info(DeviceInfo* out) {
@@ -127,26 +148,27 @@ bool device_info(DeviceInfo* out) {
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return false;
   std::lock_guard<std::mutex> lk(mu);
   if (!cache[dev].ok) {
-    int major = 0, minor = 0, sms = 0;
+    int major = 0, minor = 0, sms = 0, pairs = -1;
     if (cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev) != cudaSuccess ||
         cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev) != cudaSuccess ||
         cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
       return false;
     if (major != 10 || minor != 3) return false;
-#define GRPO_SET_SMEM(E, A, B)                                                                   \
-  if (cudaFuncSetAttribute(gemm_tc_kernel<E, A, B>, cudaFuncAttributeMaxDynamicSharedMemorySize, \
-                           kGemmSmemBytes) != cudaSuccess)                                       \
-    return false;
-    GRPO_SET_SMEM(kEpiLse, false, false)
-    GRPO_SET_SMEM(kEpiDz, false, false)
-    GRPO_SET_SMEM(kEpiF32, false, true)
-    GRPO_SET_SMEM(kEpiF32, true, true)
-#undef GRPO_SET_SMEM
+    if (!prepare_kernels<kEpiLse, false, false>(&pairs) || !prepare_kernels<kEpiDz, false, false>(&pairs) ||
+        !prepare_kernels<kEpiF32, false, true>(&pairs) || !prepare_kernels<kEpiF32, true, true>(&pairs))
+      return false;
     cache[dev].sms = sms;
+    cache[dev].pairs = std::max(pairs, 0);
     cache[dev].ok = true;
   }
   *out = cache[dev];
   return true;
+}
+
+// 2-CTA (cta_group::2) tiles unless GRPO_CTA_PAIR=0.
+bool use_pairs() {
+  const char* e = std::getenv("GRPO_CTA_PAIR");
+  return !(e && e[0] == '0');
 }
 
 // ---------------------------------------------------------------- tracing
@@ -205,12 +227,39 @@ class TraceScope {
   bool active_ = false;
 };
 
-template <int E, bool A, bool B>
-cudaError_t launch_gemm(const CUtensorMap& ta, const CUtensorMap& tb, const GemmArgs& a,
-                        int64_t max_units, int sms, cudaStream_t s) {
-  const int grid = static_cast<int>(std::max<int64_t>(1, std::min<int64_t>(sms, max_units)));
-  gemm_tc_kernel<E, A, B><<<grid, kGemmThreads, kGemmSmemBytes, s>>>(ta, tb, a);
+// A bf16 row-major matrix [rows x cols] with leading dimension ld (elements).
+struct Operand {
+  const void* base;
+  uint64_t rows, cols, ld;
+};
+
+// Builds the tensor maps of A and B for the tile shape of kPair and launches
+// the persistent GEMM with at most one CTA (pair) per work unit.
+template <int kPair, int E, bool AMN, bool BMN>
+cudaError_t launch_gemm_cfg(const Operand& A, const Operand& B, const GemmArgs& a, int64_t max_m_rows,
+                            const DeviceInfo& di, cudaStream_t s) {
+  using C = TileCfg<kPair>;
+  CUtensorMap ta, tb;
+  if (!encode_2d(&ta, A.base, A.rows, A.cols, A.ld, kBK, AMN ? 64 : kRowsCta) ||
+      !encode_2d(&tb, B.base, B.rows, B.cols, B.ld, kBK, BMN ? 64 : C::kBRows))
+    return cudaErrorInvalidValue;
+  const int64_t n_tiles = (a.N + kTileN - 1) / kTileN;
+  const int64_t units = ((max_m_rows + C::kTileM - 1) / C::kTileM) * ((n_tiles + a.n_per_unit - 1) / a.n_per_unit);
+  if (kPair == 2) {
+    const int64_t pairs = std::max<int64_t>(1, std::min<int64_t>(di.pairs, units));
+    gemm_tc_pair_kernel<E, AMN, BMN><<<static_cast<unsigned>(2 * pairs), kGemmThreads, C::kSmemBytes, s>>>(ta, tb, a);
+  } else {
+    const int64_t grid = std::max<int64_t>(1, std::min<int64_t>(di.sms, units));
+    gemm_tc_kernel<E, AMN, BMN><<<static_cast<unsigned>(grid), kGemmThreads, C::kSmemBytes, s>>>(ta, tb, a);
+  }
   return cudaGetLastError();
+}
+
+template <int E, bool AMN, bool BMN>
+cudaError_t launch_gemm(const Operand& A, const Operand& B, const GemmArgs& a, int64_t max_m_rows,
+                        const DeviceInfo& di, cudaStream_t s) {
+  return use_pairs() && di.pairs > 0 ? launch_gemm_cfg<2, E, AMN, BMN>(A, B, a, max_m_rows, di, s)
+                                     : launch_gemm_cfg<1, E, AMN, BMN>(A, B, a, max_m_rows, di, s);
 }
 
 template <typename T>
@@ -244,12 +293,8 @@ cudaError_t run_compaction(const uint16_t* H, const int32_t* targets, const uint
 }
 
 // Forward GEMM with the log-softmax epilogue over all V columns.
-cudaError_t run_lse(const uint16_t* W, int32_t Hd, int64_t V, void* ws, const Layout& Ly, int sms,
-                    cudaStream_t s) {
-  CUtensorMap tA, tB;
-  if (!encode_2d(&tA, at<uint16_t>(ws, Ly.Hc), Ly.T_pad, Hd, Hd, kBK, kBM) ||
-      !encode_2d(&tB, W, V, Hd, Hd, kBK, kBN))
-    return cudaErrorInvalidValue;
+cudaError_t run_lse(const uint16_t* W, int32_t Hd, int64_t V, void* ws, const Layout& Ly,
+                    const DeviceInfo& di, cudaStream_t s) {
   GemmArgs a{};
   a.n_valid = at<int>(ws, Ly.n_valid);
   a.M = 0;
@@ -264,9 +309,11 @@ cudaError_t run_lse(const uint16_t* W, int32_t Hd, int64_t V, void* ws, const La
   a.part_s = at<float>(ws, Ly.part_s);
   a.zy = at<float>(ws, Ly.zy);
   a.ldp = Ly.T_pad;
-  const int64_t max_units = (Ly.T_pad / kBM) * Ly.nsplit;
+  const Operand A{at<uint16_t>(ws, Ly.Hc), static_cast<uint64_t>(Ly.T_pad), static_cast<uint64_t>(Hd),
+                  static_cast<uint64_t>(Hd)};
+  const Operand B{W, static_cast<uint64_t>(V), static_cast<uint64_t>(Hd), static_cast<uint64_t>(Hd)};
   TraceScope trace(GRPO_K_LSE_GEMM, V, s);
-  return launch_gemm<kEpiLse, false, false>(tA, tB, a, max_units, sms, s);
+  return launch_gemm<kEpiLse, false, false>(A, B, a, Ly.T_pad, di, s);
 }
 
 grpo_status from_cuda(cudaError_t e) { return e == cudaSuccess ? GRPO_OK : GRPO_ERR_CUDA; }
@@ -326,7 +373,7 @@ grpo_status grpo_token_logprobs(const uint16_t* H, const uint16_t* W, const int3
   if (!get_encode()) return GRPO_ERR_CUDA;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   cudaError_t e = run_compaction(H, targets, mask, T, Hd, V, ws, Ly, di.sms, s);
-  if (e == cudaSuccess) e = run_lse(W, Hd, V, ws, Ly, di.sms, s);
+  if (e == cudaSuccess) e = run_lse(W, Hd, V, ws, Ly, di, s);
   if (e == cudaSuccess) {
     const int blocks = static_cast<int>(std::min<int64_t>((T + 255) / 256, di.sms * 16));
     TraceScope trace(GRPO_K_LOGP_MERGE, 0, s);
@@ -370,7 +417,7 @@ grpo_status grpo_loss_fwd_bwd(const uint16_t* H, const uint16_t* W, const int32_
     resp_len_kernel<<<static_cast<unsigned>(blocks), 256, 0, s>>>(mask, n_resp, L, at<int>(ws, Ly.resp_len));
     e = cudaGetLastError();
   }
-  if (e == cudaSuccess) e = run_lse(W, Hd, V, ws, Ly, sms, s);
+  if (e == cudaSuccess) e = run_lse(W, Hd, V, ws, Ly, di, s);
   if (e == cudaSuccess) {
     TraceScope trace(GRPO_K_LOSS, 0, s);
     loss_terms_kernel<<<static_cast<unsigned>(Ly.nblk_loss), kLossThreads, 0, s>>>(
@@ -390,71 +437,67 @@ grpo_status grpo_loss_fwd_bwd(const uint16_t* H, const uint16_t* W, const int32_
   if (e != cudaSuccess) return from_cuda(e);
 
   // Backward, one vocabulary chunk at a time.
-  CUtensorMap tHcK, tWK, tDzK, tWMN, tDzMN, tHcMN;
   uint16_t* Hc = at<uint16_t>(ws, Ly.Hc);
   uint16_t* dz = at<uint16_t>(ws, Ly.dz);
   const int64_t vc = Ly.vchunk;
-  if (!encode_2d(&tHcK, Hc, Ly.T_pad, Hd, Hd, kBK, kBM) || !encode_2d(&tWK, W, V, Hd, Hd, kBK, kBN) ||
-      !encode_2d(&tDzK, dz, Ly.T_pad, vc, vc, kBK, kBM) || !encode_2d(&tWMN, W, V, Hd, Hd, 64, 64) ||
-      !encode_2d(&tDzMN, dz, Ly.T_pad, vc, vc, 64, 64) || !encode_2d(&tHcMN, Hc, Ly.T_pad, Hd, Hd, 64, 64))
-    return GRPO_ERR_CUDA;
-  const int64_t mt_max = Ly.T_pad / kBM;
-  const int64_t hd_tiles = (Hd + kBN - 1) / kBN;
+  const uint64_t tp = static_cast<uint64_t>(Ly.T_pad), hd = static_cast<uint64_t>(Hd);
+  const Operand opHc{Hc, tp, hd, hd};
+  const Operand opW{W, static_cast<uint64_t>(V), hd, hd};
+  const Operand opDz{dz, tp, static_cast<uint64_t>(vc), static_cast<uint64_t>(vc)};
   for (int64_t c0 = 0; c0 < V && e == cudaSuccess; c0 += vc) {
     const int64_t width = std::min<int64_t>(vc, V - c0);
-    // dZ chunk = g (onehot - softmax) from recomputed logits
-    GemmArgs a{};
-    a.n_valid = n_valid;
-    a.m_dyn = 1;
-    a.N = static_cast<int>(width);
-    a.K = Hd;
-    a.b_off_n = static_cast<int>(c0);
-    a.n_per_unit = 1;
-    a.group_m = 8;
-    a.status = status;
-    a.yc = at<int>(ws, Ly.yc);
-    a.lse = at<float>(ws, Ly.lse_c);
-    a.gcoef = at<float>(ws, Ly.g_c);
-    a.dz = dz;
-    a.ldz = vc;
-    {
+    {  // dZ chunk = g (onehot - softmax) from recomputed logits
+      GemmArgs a{};
+      a.n_valid = n_valid;
+      a.m_dyn = 1;
+      a.N = static_cast<int>(width);
+      a.K = Hd;
+      a.b_off_n = static_cast<int>(c0);
+      a.n_per_unit = 1;
+      a.group_m = 8;
+      a.status = status;
+      a.yc = at<int>(ws, Ly.yc);
+      a.lse = at<float>(ws, Ly.lse_c);
+      a.gcoef = at<float>(ws, Ly.g_c);
+      a.dz = dz;
+      a.ldz = vc;
       TraceScope trace(GRPO_K_DZ_GEMM, width, s);
-      e = launch_gemm<kEpiDz, false, false>(tHcK, tWK, a, mt_max * ((width + kBN - 1) / kBN), sms, s);
+      e = launch_gemm<kEpiDz, false, false>(opHc, opW, a, Ly.T_pad, di, s);
     }
     if (e != cudaSuccess) break;
-    // dH (+)= dZ_c W_c
-    GemmArgs h{};
-    h.n_valid = n_valid;
-    h.m_dyn = 1;
-    h.N = Hd;
-    h.K = static_cast<int>(width);
-    h.b_off_k = static_cast<int>(c0);
-    h.n_per_unit = 1;
-    h.group_m = 8;
-    h.status = status;
-    h.out = dH;
-    h.ldo = Hd;
-    h.accumulate = c0 > 0;
-    h.row_map = at<int>(ws, Ly.cidx);
-    {
+    {  // dH (+)= dZ_c W_c
+      GemmArgs h{};
+      h.n_valid = n_valid;
+      h.m_dyn = 1;
+      h.N = Hd;
+      h.K = static_cast<int>(width);
+      h.b_off_k = static_cast<int>(c0);
+      h.n_per_unit = 1;
+      h.group_m = 8;
+      h.status = status;
+      h.out = dH;
+      h.ldo = Hd;
+      h.accumulate = c0 > 0;
+      h.row_map = at<int>(ws, Ly.cidx);
       TraceScope trace(GRPO_K_DH_GEMM, width, s);
-      e = launch_gemm<kEpiF32, false, true>(tDzK, tWMN, h, mt_max * hd_tiles, sms, s);
+      e = launch_gemm<kEpiF32, false, true>(opDz, opW, h, Ly.T_pad, di, s);
     }
     if (e != cudaSuccess) break;
-    // dW_c = dZ_c^T Hc
-    GemmArgs w{};
-    w.n_valid = n_valid;
-    w.M = static_cast<int>(width);
-    w.N = Hd;
-    w.k_dyn = 1;
-    w.n_per_unit = 1;
-    w.group_m = 8;
-    w.status = status;
-    w.out = dW + c0 * Hd;
-    w.ldo = Hd;
-    w.accumulate = 0;
-    TraceScope trace(GRPO_K_DW_GEMM, width, s);
-    e = launch_gemm<kEpiF32, true, true>(tDzMN, tHcMN, w, ((width + kBM - 1) / kBM) * hd_tiles, sms, s);
+    {  // dW_c = dZ_c^T Hc
+      GemmArgs w{};
+      w.n_valid = n_valid;
+      w.M = static_cast<int>(width);
+      w.N = Hd;
+      w.k_dyn = 1;
+      w.n_per_unit = 1;
+      w.group_m = 8;
+      w.status = status;
+      w.out = dW + c0 * Hd;
+      w.ldo = Hd;
+      w.accumulate = 0;
+      TraceScope trace(GRPO_K_DW_GEMM, width, s);
+      e = launch_gemm<kEpiF32, true, true>(opDz, opHc, w, width, di, s);
+    }
   }
   return from_cuda(e);
 }

@@ -146,14 +146,14 @@ __global__ void mask_scatter_kernel(const uint8_t* __restrict__ mask, int64_t T,
 }
 
 // Hc[r] = H[cidx[r]] and yc[r] = targets[cidx[r]] for r < n_valid; rows
-// n_valid .. round_up(n_valid, 128) are zero-filled (they feed K-loops over
-// tokens).  One warp per row, 16-byte vectors.
+// n_valid .. round_up(n_valid, 256) are zero-filled (they feed K-loops over
+// tokens and the last row tile).  One warp per row, 16-byte vectors.
 __global__ void gather_rows_kernel(const uint16_t* __restrict__ H, const int32_t* __restrict__ targets,
                                    const int* __restrict__ cidx, const int* __restrict__ n_valid_p,
                                    int Hd, int64_t V, uint16_t* __restrict__ Hc, int* __restrict__ yc,
                                    unsigned* status) {
   const int nv = *n_valid_p;
-  const int rows = (nv + 127) / 128 * 128;
+  const int rows = (nv + 255) / 256 * 256;
   const int lane = threadIdx.x & 31;
   const int vec = Hd / 8;  // uint4 per row
   for (int r = (blockIdx.x * blockDim.x + threadIdx.x) >> 5; r < rows;

@@ -135,6 +135,15 @@ def test_ragged_multi_chunk_fwd_bwd(agg_mode, monkeypatch):
     _check_fwd_bwd(_case(w, agg_mode), agg_mode)
 
 
+@pytest.mark.parametrize("pair", ["0", "1"])
+def test_single_and_paired_tiles_agree(pair, monkeypatch):
+    """The 128x256 single-CTA tile and the 256x256 CTA-pair tile both meet the bar."""
+    monkeypatch.setenv("GRPO_CTA_PAIR", pair)
+    monkeypatch.setenv("GRPO_VOCAB_CHUNK", "768")
+    w = wl.Workload("t", 3, 4, 60, 192, 2100, "uniform", 1, 60, rewards="mix", seed=wl.SEED_BASE + 550)
+    _check_fwd_bwd(_case(w))
+
+
 def test_fwd_bwd_is_deterministic():
     c = _case(wl.Workload("t", 1, 4, 70, 256, 2000, "uniform", 5, 70, seed=wl.SEED_BASE + 600))
     a = _check_fwd_bwd(c)
