@@ -109,6 +109,34 @@ grpo_status grpo_loss_fwd_bwd(const uint16_t* H, const uint16_t* W, const int32_
                               float* dH, float* dW, void* ws, size_t ws_bytes, void* stream);
 
 /*
+ * grpo_token_logprobs without a workspace argument, for callers that cannot
+ * allocate device memory themselves: code running where cudaMalloc is not
+ * allowed or would stall the device (inside a stream capture, in a real-time
+ * loop with a fixed memory budget), or a binding that has no device allocator.
+ * The paper has no counterpart; this is a deployment convenience.
+ *
+ * Scratch space is a fixed 64 MiB array of device memory inside libgrpo.so,
+ * held on every GPU that loads the library until the process exits.  The
+ * call allocates nothing: no cudaMalloc, no cudaFree, no allocating library
+ * routine.  Arguments, layout and results are those of grpo_token_logprobs.
+ *   - Returns GRPO_ERR_WORKSPACE if grpo_workspace_bytes(T, Hd, V,
+ *     GRPO_WS_LOGPROBS) exceeds 64 MiB (7,680 tokens at Hd 4096,
+ *     V 155136), GRPO_ERR_INVALID_ARG for arguments grpo_token_logprobs rejects.
+ *   - The first call on a device looks up the array's device address (with
+ *     that device current); make that first call before any stream capture.
+ *   - Every call uses the same array and leaves its contents behind; each call
+ *     clears what it needs cleared.  Calls whose work can overlap on the GPU
+ *     (different streams, or different host threads) race on the array and
+ *     give wrong results: serialise them.
+ *   - Device-side problems (a target outside [0, V)) give 0 for the affected
+ *     rows as in grpo_token_logprobs, but there is no workspace to pass to
+ *     grpo_check_device_status.
+ */
+grpo_status grpo_token_logprobs_noalloc(const uint16_t* H, const uint16_t* W, const int32_t* targets,
+                                        const uint8_t* mask, int64_t T, int32_t Hd, int64_t V,
+                                        float* logp_out, void* stream);
+
+/*
  * Bytes of workspace the call `which` (GRPO_WS_LOGPROBS or GRPO_WS_LOSS)
  * needs for T tokens, hidden size Hd and vocabulary V.  Returns 0 for
  * arguments the calls would reject.  Sized for the worst case N_valid = T.

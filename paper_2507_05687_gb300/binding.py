@@ -40,6 +40,7 @@ SIGNATURES = {
     "grpo_token_logprobs": (ctypes.c_int, [_P, _P, _P, _P, _I64, _I32, _I64, _P, _P, ctypes.c_size_t, _P]),
     "grpo_loss_fwd_bwd": (ctypes.c_int, [_P, _P, _P, _P, _P, _P, _P, _I64, _I64, _I32, _I64, _F, _F, _I32,
                                          _P, _P, _P, _P, ctypes.c_size_t, _P]),
+    "grpo_token_logprobs_noalloc": (ctypes.c_int, [_P, _P, _P, _P, _I64, _I32, _I64, _P, _P]),
     "grpo_workspace_bytes": (ctypes.c_size_t, [_I64, _I32, _I64, _I32]),
     "grpo_check_device_status": (ctypes.c_int, [_P, _P]),
     "grpo_status_string": (ctypes.c_char_p, [ctypes.c_int]),

@@ -5,6 +5,7 @@
 #include <cudaTypedefs.h>
 
 #include <cstdint>
+#include <cstdio>
 #include <cstdlib>
 #include <cstring>
 #include <mutex>
@@ -165,6 +166,18 @@ bool device_info(DeviceInfo* out) {
   return true;
 }
 
+// Raster group height (M tiles per group) of each GEMM: LSE, dZ, dH, dW.
+// GRPO_GROUP_M="a,b,c,d" overrides the defaults.
+int group_m(int which) {
+  int g[4] = {8, 8, 8, 8};
+  if (const char* e = std::getenv("GRPO_GROUP_M")) {
+    int v[4];
+    if (std::sscanf(e, "%d,%d,%d,%d", &v[0], &v[1], &v[2], &v[3]) == 4)
+      for (int i = 0; i < 4; ++i) g[i] = v[i] > 0 ? v[i] : g[i];
+  }
+  return g[which];
+}
+
 // 2-CTA (cta_group::2) tiles unless GRPO_CTA_PAIR=0.
 bool use_pairs() {
   const char* e = std::getenv("GRPO_CTA_PAIR");
@@ -302,7 +315,7 @@ cudaError_t run_lse(const uint16_t* W, int32_t Hd, int64_t V, void* ws, const La
   a.N = static_cast<int>(V);
   a.K = Hd;
   a.n_per_unit = kLseTilesPerUnit;
-  a.group_m = 8;
+  a.group_m = group_m(0);
   a.status = at<unsigned>(ws, Ly.status);
   a.yc = at<int>(ws, Ly.yc);
   a.part_m = at<float>(ws, Ly.part_m);
@@ -454,7 +467,7 @@ grpo_status grpo_loss_fwd_bwd(const uint16_t* H, const uint16_t* W, const int32_
       a.K = Hd;
       a.b_off_n = static_cast<int>(c0);
       a.n_per_unit = 1;
-      a.group_m = 8;
+      a.group_m = group_m(1);
       a.status = status;
       a.yc = at<int>(ws, Ly.yc);
       a.lse = at<float>(ws, Ly.lse_c);
@@ -473,7 +486,7 @@ grpo_status grpo_loss_fwd_bwd(const uint16_t* H, const uint16_t* W, const int32_
       h.K = static_cast<int>(width);
       h.b_off_k = static_cast<int>(c0);
       h.n_per_unit = 1;
-      h.group_m = 8;
+      h.group_m = group_m(2);
       h.status = status;
       h.out = dH;
       h.ldo = Hd;
@@ -490,7 +503,7 @@ grpo_status grpo_loss_fwd_bwd(const uint16_t* H, const uint16_t* W, const int32_
       w.N = Hd;
       w.k_dyn = 1;
       w.n_per_unit = 1;
-      w.group_m = 8;
+      w.group_m = group_m(3);
       w.status = status;
       w.out = dW + c0 * Hd;
       w.ldo = Hd;
@@ -548,4 +561,45 @@ grpo_status grpo_check_device_status(void* ws, void* stream) {
   return GRPO_OK;
 }
 
+// ---------------------------------------------------------------- no-allocation variant
+//
+// grpo_token_logprobs_noalloc runs grpo_token_logprobs unchanged, with its
+// scratch space taken from a fixed array in device memory that is part of this
+// library instead of from a caller-provided workspace.
+
 }  // extern "C"
+
+namespace {
+
+constexpr size_t kStaticScratchBytes = size_t(64) << 20;  // 64 MiB on every device that loads the library
+static __device__ __align__(256) unsigned char g_static_scratch[kStaticScratchBytes];
+
+// Device address of g_static_scratch on the current device, looked up once per
+// device.  The host-side symbol is only a stand-in, never a device address.
+void* static_scratch() {
+  static std::mutex mu;
+  static void* addr[64] = {};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return nullptr;
+  std::lock_guard<std::mutex> lk(mu);
+  if (!addr[dev]) {
+    void* p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_static_scratch) != cudaSuccess) return nullptr;
+    addr[dev] = p;
+  }
+  return addr[dev];
+}
+
+}  // namespace
+
+extern "C" grpo_status grpo_token_logprobs_noalloc(const uint16_t* H, const uint16_t* W,
+                                                   const int32_t* targets, const uint8_t* mask,
+                                                   int64_t T, int32_t Hd, int64_t V, float* logp_out,
+                                                   void* stream) {
+  const size_t need = grpo_workspace_bytes(T, Hd, V, GRPO_WS_LOGPROBS);
+  if (need == 0) return GRPO_ERR_INVALID_ARG;
+  if (need > kStaticScratchBytes) return GRPO_ERR_WORKSPACE;
+  void* ws = static_scratch();
+  if (!ws) return GRPO_ERR_CUDA;
+  return grpo_token_logprobs(H, W, targets, mask, T, Hd, V, logp_out, ws, kStaticScratchBytes, stream);
+}
