@@ -300,11 +300,16 @@ def main():
     out = (torch.empty(1, dtype=torch.float32, device=dev), torch.empty(w.T, w.Hd, dtype=torch.float32, device=dev),
            torch.empty(w.V, w.Hd, dtype=torch.float32, device=dev))
 
+    from paper_2507_05687_gb300 import dp
+
     def step():
         grpo.group_advantages(r, w.G, w.adv_eps, out=adv)
-        grpo.loss_fwd_bwd(H, W, y, m, old, ref, adv, w.n_resp, w.L, w.clip_eps, w.beta, 0, ws=ws, out=out)
-        if dist is not None:
-            dist.all_reduce(out[2])  # data-parallel exchange of the LM-head gradient
+        if dist is None:
+            grpo.loss_fwd_bwd(H, W, y, m, old, ref, adv, w.n_resp, w.L, w.clip_eps, w.beta, 0, ws=ws, out=out)
+        else:
+            # global token-mean over every rank's batch; loss and dW summed over ranks
+            dp.dp_loss_fwd_bwd(H, W, y, m, old, ref, adv, w.n_resp, w.L, w.clip_eps, w.beta, 0, n_valid,
+                               ws=ws, out=out)
 
     for _ in range(max(3, args.warmup)):
         step()

@@ -109,6 +109,24 @@ grpo_status grpo_loss_fwd_bwd(const uint16_t* H, const uint16_t* W, const int32_
                               float* dH, float* dW, void* ws, size_t ws_bytes, void* stream);
 
 /*
+ * grpo_loss_fwd_bwd with the normaliser of the aggregation given by the
+ * caller, for data-parallel training where each rank holds a shard of the
+ * batch (whole prompt groups) and the loss is normalised over the global
+ * batch (Eq. 1's expectation over all prompts of the step):
+ *   agg_mode 0: w_t = mask_t / norm        (norm = N_valid summed over ranks)
+ *   agg_mode 1: w_t = mask_t / (norm |o_i|) (norm = n_resp summed over ranks)
+ * norm == 0 uses the local count (this is exactly grpo_loss_fwd_bwd).  With
+ * the global norm on every rank, the sum over ranks of loss, and of dW, is the
+ * loss and dW of the whole batch.  norm must be finite and >= 0.
+ */
+grpo_status grpo_loss_fwd_bwd_norm(const uint16_t* H, const uint16_t* W, const int32_t* targets,
+                                   const uint8_t* mask, const float* old_logp, const float* ref_logp,
+                                   const float* adv, int64_t n_resp, int64_t L, int32_t Hd, int64_t V,
+                                   float clip_eps, float beta, int32_t agg_mode, float norm,
+                                   float* loss_out, float* dH, float* dW, void* ws, size_t ws_bytes,
+                                   void* stream);
+
+/*
  * grpo_token_logprobs without a workspace argument, for callers that cannot
  * allocate device memory themselves: code running where cudaMalloc is not
  * allowed or would stall the device (inside a stream capture, in a real-time

@@ -141,20 +141,23 @@ def token_terms(logp, old_logp, ref_logp, adv_tok, clip_eps: float, beta: float)
     return {"rho": rho, "s": s, "kl": kl, "ell": -s + beta * kl, "unclipped": unclipped}
 
 
-def token_weights(mask, n_resp: int, L: int, agg_mode: int = 0) -> np.ndarray:
+def token_weights(mask, n_resp: int, L: int, agg_mode: int = 0, norm: float = 0.0) -> np.ndarray:
     """w_t so that loss = sum_t w_t l_t.
 
     agg_mode 0: mask_t / N_valid (token-mean; 0 when N_valid = 0).
     agg_mode 1: mask_t / (n_resp |o_i|), Eq. 1's per-response mean then mean
     over responses (a response with |o_i| = 0 contributes nothing).
+    norm > 0 replaces N_valid (mode 0) or n_resp (mode 1): the count over the
+    whole step's batch when this batch is one shard of it, since Eq. 1's
+    expectation runs over every prompt of the step.
     """
     m = (np.asarray(mask) != 0).astype(np.float64)
     if agg_mode == 0:
-        n = m.sum()
+        n = norm if norm > 0 else m.sum()
         return m / n if n > 0 else np.zeros_like(m)
     if agg_mode == 1:
         lens = m.reshape(n_resp, L).sum(axis=1)
-        inv = np.where(lens > 0, 1.0 / np.maximum(lens, 1.0), 0.0) / n_resp
+        inv = np.where(lens > 0, 1.0 / np.maximum(lens, 1.0), 0.0) / (norm if norm > 0 else n_resp)
         return m * np.repeat(inv, L)
     raise ValueError(agg_mode)
 
@@ -171,10 +174,10 @@ def logp_coef(logp, old_logp, ref_logp, adv_tok, w, clip_eps: float, beta: float
 
 
 def grpo_loss(logp, old_logp, ref_logp, adv, mask, n_resp: int, L: int,
-              clip_eps: float, beta: float, agg_mode: int = 0):
+              clip_eps: float, beta: float, agg_mode: int = 0, norm: float = 0.0):
     """Eq. 1 negated, from per-token log-probs. Returns (loss, g, per-token dict)."""
     A = token_advantages(adv, n_resp, L)
-    w = token_weights(mask, n_resp, L, agg_mode)
+    w = token_weights(mask, n_resp, L, agg_mode, norm)
     tt = token_terms(logp, old_logp, ref_logp, A, clip_eps, beta)
     m = np.asarray(mask) != 0
     loss = float(np.sum(w[m] * tt["ell"][m]))
@@ -190,14 +193,15 @@ def grpo_loss(logp, old_logp, ref_logp, adv, mask, n_resp: int, L: int,
 
 
 def loss_fwd_bwd(H, W, targets, mask, old_logp, ref_logp, adv, n_resp: int, L: int,
-                 clip_eps: float, beta: float, agg_mode: int = 0, vocab_chunk: int = 8192):
+                 clip_eps: float, beta: float, agg_mode: int = 0, vocab_chunk: int = 8192,
+                 norm: float = 0.0):
     """Full forward + backward: returns dict(loss, dH [T,Hd], dW [V,Hd], logp, lse, g)."""
     Hf = as_f64(H)
     Wf = as_f64(W)
     y = np.asarray(targets, dtype=np.int64)
     m = np.asarray(mask) != 0
     logp, lse = token_logprobs(Hf, Wf, y, m, vocab_chunk=vocab_chunk)
-    loss, g, tt = grpo_loss(logp, old_logp, ref_logp, adv, m, n_resp, L, clip_eps, beta, agg_mode)
+    loss, g, tt = grpo_loss(logp, old_logp, ref_logp, adv, m, n_resp, L, clip_eps, beta, agg_mode, norm)
     T, Hd = Hf.shape
     V = Wf.shape[0]
     dH = np.zeros((T, Hd))

@@ -40,6 +40,8 @@ SIGNATURES = {
     "grpo_token_logprobs": (ctypes.c_int, [_P, _P, _P, _P, _I64, _I32, _I64, _P, _P, ctypes.c_size_t, _P]),
     "grpo_loss_fwd_bwd": (ctypes.c_int, [_P, _P, _P, _P, _P, _P, _P, _I64, _I64, _I32, _I64, _F, _F, _I32,
                                          _P, _P, _P, _P, ctypes.c_size_t, _P]),
+    "grpo_loss_fwd_bwd_norm": (ctypes.c_int, [_P, _P, _P, _P, _P, _P, _P, _I64, _I64, _I32, _I64, _F, _F, _I32, _F,
+                                              _P, _P, _P, _P, ctypes.c_size_t, _P]),
     "grpo_token_logprobs_noalloc": (ctypes.c_int, [_P, _P, _P, _P, _I64, _I32, _I64, _P, _P]),
     "grpo_workspace_bytes": (ctypes.c_size_t, [_I64, _I32, _I64, _I32]),
     "grpo_check_device_status": (ctypes.c_int, [_P, _P]),
@@ -166,8 +168,9 @@ def loss_fwd_bwd(H: torch.Tensor, W: torch.Tensor, targets: torch.Tensor, mask: 
                  old_logp: torch.Tensor, ref_logp: torch.Tensor, adv: torch.Tensor,
                  n_resp: int, L: int, clip_eps: float = 0.2, beta: float = 0.04, agg_mode: int = 0,
                  ws: Optional[torch.Tensor] = None,
-                 out: Optional[Tuple[torch.Tensor, torch.Tensor, torch.Tensor]] = None):
-    """grpo_loss_fwd_bwd: returns (loss [1] fp32, dH [T, Hd] fp32, dW [V, Hd] fp32)."""
+                 out: Optional[Tuple[torch.Tensor, torch.Tensor, torch.Tensor]] = None, norm: float = 0.0):
+    """grpo_loss_fwd_bwd (norm == 0) / grpo_loss_fwd_bwd_norm (norm > 0, a global
+    N_valid or n_resp): returns (loss [1] fp32, dH [T, Hd] fp32, dW [V, Hd] fp32)."""
     dev, host = _target_device(H, W)
     H = _on_device(H, dev, torch.bfloat16, "H")
     W = _on_device(W, dev, torch.bfloat16, "W")
@@ -185,10 +188,14 @@ def loss_fwd_bwd(H: torch.Tensor, W: torch.Tensor, targets: torch.Tensor, mask: 
                torch.empty(T, Hd, dtype=torch.float32, device=dev),
                torch.empty(V, Hd, dtype=torch.float32, device=dev))
     loss, dH, dW = out
-    _check(load().grpo_loss_fwd_bwd(_ptr(H), _ptr(W), _ptr(targets), _ptr(mask), _ptr(old_logp), _ptr(ref_logp),
-                                    _ptr(adv), int(n_resp), int(L), Hd, V, float(clip_eps), float(beta),
-                                    int(agg_mode), _ptr(loss), _ptr(dH), _ptr(dW), _ptr(ws), ws.numel(),
-                                    _stream(dev)), "grpo_loss_fwd_bwd")
+    lib = load()
+    common = (_ptr(H), _ptr(W), _ptr(targets), _ptr(mask), _ptr(old_logp), _ptr(ref_logp), _ptr(adv), int(n_resp),
+              int(L), Hd, V, float(clip_eps), float(beta), int(agg_mode))
+    tail = (_ptr(loss), _ptr(dH), _ptr(dW), _ptr(ws), ws.numel(), _stream(dev))
+    if norm:
+        _check(lib.grpo_loss_fwd_bwd_norm(*common, float(norm), *tail), "grpo_loss_fwd_bwd_norm")
+    else:
+        _check(lib.grpo_loss_fwd_bwd(*common, *tail), "grpo_loss_fwd_bwd")
     if host:
         return _to_host(loss, dH, dW)
     return loss, dH, dW

@@ -404,7 +404,18 @@ grpo_status grpo_loss_fwd_bwd(const uint16_t* H, const uint16_t* W, const int32_
                               const float* adv, int64_t n_resp, int64_t L, int32_t Hd, int64_t V,
                               float clip_eps, float beta, int32_t agg_mode, float* loss_out,
                               float* dH, float* dW, void* ws, size_t ws_bytes, void* stream) {
+  return grpo_loss_fwd_bwd_norm(H, W, targets, mask, old_logp, ref_logp, adv, n_resp, L, Hd, V, clip_eps,
+                                beta, agg_mode, 0.f, loss_out, dH, dW, ws, ws_bytes, stream);
+}
+
+grpo_status grpo_loss_fwd_bwd_norm(const uint16_t* H, const uint16_t* W, const int32_t* targets,
+                                   const uint8_t* mask, const float* old_logp, const float* ref_logp,
+                                   const float* adv, int64_t n_resp, int64_t L, int32_t Hd, int64_t V,
+                                   float clip_eps, float beta, int32_t agg_mode, float norm,
+                                   float* loss_out, float* dH, float* dW, void* ws, size_t ws_bytes,
+                                   void* stream) {
   if (n_resp < 1 || L < 1 || n_resp > (int64_t(1) << 31) / L) return GRPO_ERR_INVALID_ARG;
+  if (!(norm >= 0.f) || norm == INFINITY) return GRPO_ERR_INVALID_ARG;
   const int64_t T = n_resp * L;
   Layout Ly;
   if (!make_layout(T, Hd, V, GRPO_WS_LOSS, &Ly)) return GRPO_ERR_INVALID_ARG;
@@ -436,7 +447,7 @@ grpo_status grpo_loss_fwd_bwd(const uint16_t* H, const uint16_t* W, const int32_
     loss_terms_kernel<<<static_cast<unsigned>(Ly.nblk_loss), kLossThreads, 0, s>>>(
         at<int>(ws, Ly.cidx), n_valid, at<float>(ws, Ly.part_m), at<float>(ws, Ly.part_s),
         static_cast<int>(Ly.nsplit), Ly.T_pad, at<float>(ws, Ly.zy), at<int>(ws, Ly.yc), old_logp,
-        ref_logp, adv, L, at<int>(ws, Ly.resp_len), n_resp, agg_mode, clip_eps, beta,
+        ref_logp, adv, L, at<int>(ws, Ly.resp_len), n_resp, agg_mode, norm, clip_eps, beta,
         at<float>(ws, Ly.lse_c), at<float>(ws, Ly.g_c), at<double>(ws, Ly.block_loss), status);
     loss_final_kernel<<<1, 1024, 0, s>>>(at<double>(ws, Ly.block_loss), n_valid, kLossThreads, loss_out);
     e = cudaGetLastError();

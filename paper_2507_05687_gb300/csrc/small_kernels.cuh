@@ -228,7 +228,7 @@ __global__ void loss_terms_kernel(const int* __restrict__ cidx, const int* __res
                                   const int* __restrict__ yc, const float* __restrict__ old_logp,
                                   const float* __restrict__ ref_logp, const float* __restrict__ adv,
                                   int64_t L, const int* __restrict__ resp_len, int64_t n_resp,
-                                  int agg_mode, float clip_eps, float beta,
+                                  int agg_mode, float norm, float clip_eps, float beta,
                                   float* __restrict__ lse_c, float* __restrict__ g_c,
                                   double* __restrict__ block_loss, unsigned* status) {
   __shared__ double sh[32];
@@ -254,8 +254,10 @@ __global__ void loss_terms_kernel(const int* __restrict__ cidx, const int* __res
       const float e = __expf(dref);
       const float kl = e - dref - 1.f;
       const float ell = -s + beta * kl;
-      const float w = agg_mode == 0 ? 1.f / static_cast<float>(nv)
-                                    : 1.f / (static_cast<float>(n_resp) * static_cast<float>(resp_len[i]));
+      // norm > 0 replaces the local count (N_valid, or n_resp) by a global one
+      const float w = agg_mode == 0
+                          ? 1.f / (norm > 0.f ? norm : static_cast<float>(nv))
+                          : 1.f / ((norm > 0.f ? norm : static_cast<float>(n_resp)) * static_cast<float>(resp_len[i]));
       g = w * ((unclipped ? -A * rho : 0.f) + beta * (1.f - e));
       contrib = static_cast<double>(w) * static_cast<double>(ell);
     } else {

@@ -144,6 +144,23 @@ def test_single_and_paired_tiles_agree(pair, monkeypatch):
     _check_fwd_bwd(_case(w))
 
 
+@pytest.mark.parametrize("agg_mode", [0, 1])
+def test_global_normaliser(agg_mode):
+    """grpo_loss_fwd_bwd_norm: this batch as one shard of a larger data-parallel batch."""
+    w = wl.Workload("t", 2, 4, 50, 128, 900, "uniform", 1, 50, rewards="mix", seed=wl.SEED_BASE + 650)
+    c = _case(w, agg_mode)
+    norm = 3.5 * (c["m"].sum() if agg_mode == 0 else w.n_resp)
+    want = oracle.loss_fwd_bwd(c["H"], c["W"], c["y"], c["m"], c["old"], c["ref"], c["adv"], w.n_resp, w.L,
+                               w.clip_eps, w.beta, agg_mode, norm=norm)
+    d = _dev(c)
+    loss, dH, dW = grpo.loss_fwd_bwd(d["H"], d["W"], d["y"], d["m"], d["old"], d["ref"], d["adv"], w.n_resp, w.L,
+                                     w.clip_eps, w.beta, agg_mode, norm=norm)
+    scale = loss_scale(want["loss"], want["terms"]["w"], want["terms"]["ell"])
+    assert abs(loss.item() - want["loss"]) <= LOSS_RTOL * scale
+    assert rel_fro(dH.double().cpu().numpy(), want["dH"]) <= GRAD_RTOL
+    assert rel_fro(dW.double().cpu().numpy(), want["dW"]) <= GRAD_RTOL
+
+
 def test_fwd_bwd_is_deterministic():
     c = _case(wl.Workload("t", 1, 4, 70, 256, 2000, "uniform", 5, 70, seed=wl.SEED_BASE + 600))
     a = _check_fwd_bwd(c)
