@@ -64,6 +64,7 @@ struct GemmArgs {
   int b_off_n, b_off_k; // coordinate offsets into B's tensor map
   int n_per_unit;       // consecutive N tiles one CTA (pair) walks as one work unit
   int group_m;          // raster: M tiles per group sharing the same N sweep
+  int a_hint, b_hint;   // L2 eviction policy of A / B loads (kHint*)
   unsigned* status;     // device status word
 
   // kEpiLse
@@ -317,6 +318,8 @@ __device__ __forceinline__ void gemm_body(const CUtensorMap* tmA, const CUtensor
   if (warp == 0) {
     // ------------------------------------------------------------ producer
     if (lane == 0) {
+      const uint64_t pol_a = l2_policy(args.a_hint);
+      const uint64_t pol_b = l2_policy(args.b_hint);
       int stage = 0;
       uint32_t phase = 0;
       int uses[C::kStages];
@@ -342,23 +345,23 @@ __device__ __forceinline__ void gemm_body(const CUtensorMap* tmA, const CUtensor
             const int k0 = kb * kBK;
             const int m0 = mt * C::kTileM + static_cast<int>(rank) * kRowsCta;
             const int n0 = nt * kTileN + static_cast<int>(rank) * C::kBRows;
-            auto load = [&](uint32_t dst, const CUtensorMap* map, int c0, int c1) {
-              if (kPair == 2) tma_load_2d_pair(dst, map, fb, c0, c1);
-              else tma_load_2d(dst, map, fb, c0, c1);
+            auto load = [&](uint32_t dst, const CUtensorMap* map, int c0, int c1, uint64_t pol) {
+              if (kPair == 2) tma_load_2d_pair_hint(dst, map, fb, c0, c1, pol);
+              else tma_load_2d_hint(dst, map, fb, c0, c1, pol);
             };
             if (!kAmn) {
-              load(sa, tmA, k0 + args.a_off_k, m0 + args.a_off_m);
+              load(sa, tmA, k0 + args.a_off_k, m0 + args.a_off_m, pol_a);
             } else {
 #pragma unroll
               for (int j = 0; j < kRowsCta / 64; ++j)
-                load(sa + j * 8192, tmA, m0 + args.a_off_m + 64 * j, k0 + args.a_off_k);
+                load(sa + j * 8192, tmA, m0 + args.a_off_m + 64 * j, k0 + args.a_off_k, pol_a);
             }
             if (!kBmn) {
-              load(sb, tmB, k0 + args.b_off_k, n0 + args.b_off_n);
+              load(sb, tmB, k0 + args.b_off_k, n0 + args.b_off_n, pol_b);
             } else {
 #pragma unroll
               for (int j = 0; j < C::kBRows / 64; ++j)
-                load(sb + j * 8192, tmB, n0 + args.b_off_n + 64 * j, k0 + args.b_off_k);
+                load(sb + j * 8192, tmB, n0 + args.b_off_n + 64 * j, k0 + args.b_off_k, pol_b);
             }
             ++uses[stage];
             if (++stage == C::kStages) {

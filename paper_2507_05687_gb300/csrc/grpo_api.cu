@@ -166,10 +166,40 @@ bool device_info(DeviceInfo* out) {
   return true;
 }
 
+// L2 policy of the A and B loads of GEMM `which` (LSE, dZ, dH, dW) as
+// kHint* values; GRPO_L2_HINTS="aL,bL,aZ,bZ,aH,bH,aW,bW" overrides them.
+void l2_hints(int which, int* a_hint, int* b_hint) {
+  // Forward: keep A, stream W.  The backward GEMMs measured best without hints.
+  int h[8] = {kHintEvictLast, kHintEvictFirst, kHintNone, kHintNone,
+              kHintNone, kHintNone, kHintNone, kHintNone};
+  if (const char* e = std::getenv("GRPO_L2_HINTS")) {
+    int v[8];
+    if (std::sscanf(e, "%d,%d,%d,%d,%d,%d,%d,%d", &v[0], &v[1], &v[2], &v[3], &v[4], &v[5], &v[6], &v[7]) == 8)
+      for (int i = 0; i < 8; ++i) h[i] = (v[i] >= 0 && v[i] <= 2) ? v[i] : h[i];
+  }
+  *a_hint = h[2 * which];
+  *b_hint = h[2 * which + 1];
+}
+
+// 2-CTA (cta_group::2) tiles unless GRPO_CTA_PAIR=0.
+bool use_pairs() {
+  const char* e = std::getenv("GRPO_CTA_PAIR");
+  return !(e && e[0] == '0');
+}
+
 // Raster group height (M tiles per group) of each GEMM: LSE, dZ, dH, dW.
+// The forward GEMM re-reads A (the gathered hidden states) for every one of
+// its ~600 vocabulary tiles: a group of a quarter as many M tiles as there
+// are CTAs (pairs) makes every round of the persistent grid cover whole
+// groups (each W tile read by that many CTAs at once) while the group's A
+// tiles (38 MB on GB300) stay in L2; measured DRAM reads per launch at
+// 19,572 tokens x 155,136: 62.7 GB with 8 M tiles, 34.8 GB with pairs / 2,
+// 26.7 GB with pairs / 4.  The backward GEMMs measured best at 8.
 // GRPO_GROUP_M="a,b,c,d" overrides the defaults.
-int group_m(int which) {
-  int g[4] = {8, 8, 8, 8};
+int group_m(int which, const DeviceInfo& di) {
+  const int workers = use_pairs() && di.pairs > 0 ? di.pairs : di.sms;
+  const int quarter = std::max(1, workers / 4);
+  int g[4] = {quarter, 8, 8, 8};
   if (const char* e = std::getenv("GRPO_GROUP_M")) {
     int v[4];
     if (std::sscanf(e, "%d,%d,%d,%d", &v[0], &v[1], &v[2], &v[3]) == 4)
@@ -178,11 +208,6 @@ int group_m(int which) {
   return g[which];
 }
 
-// 2-CTA (cta_group::2) tiles unless GRPO_CTA_PAIR=0.
-bool use_pairs() {
-  const char* e = std::getenv("GRPO_CTA_PAIR");
-  return !(e && e[0] == '0');
-}
 
 // ---------------------------------------------------------------- tracing
 
@@ -315,7 +340,10 @@ cudaError_t run_lse(const uint16_t* W, int32_t Hd, int64_t V, void* ws, const La
   a.N = static_cast<int>(V);
   a.K = Hd;
   a.n_per_unit = kLseTilesPerUnit;
-  a.group_m = group_m(0);
+  a.group_m = group_m(0, di);
+  // gathered hidden states: re-read for every vocabulary tile (evict last);
+  // W: streamed, shared by the CTAs of one round (evict first)
+  l2_hints(0, &a.a_hint, &a.b_hint);
   a.status = at<unsigned>(ws, Ly.status);
   a.yc = at<int>(ws, Ly.yc);
   a.part_m = at<float>(ws, Ly.part_m);
@@ -478,7 +506,8 @@ grpo_status grpo_loss_fwd_bwd_norm(const uint16_t* H, const uint16_t* W, const i
       a.K = Hd;
       a.b_off_n = static_cast<int>(c0);
       a.n_per_unit = 1;
-      a.group_m = group_m(1);
+      a.group_m = group_m(1, di);
+      l2_hints(1, &a.a_hint, &a.b_hint);
       a.status = status;
       a.yc = at<int>(ws, Ly.yc);
       a.lse = at<float>(ws, Ly.lse_c);
@@ -497,7 +526,8 @@ grpo_status grpo_loss_fwd_bwd_norm(const uint16_t* H, const uint16_t* W, const i
       h.K = static_cast<int>(width);
       h.b_off_k = static_cast<int>(c0);
       h.n_per_unit = 1;
-      h.group_m = group_m(2);
+      h.group_m = group_m(2, di);
+      l2_hints(2, &h.a_hint, &h.b_hint);
       h.status = status;
       h.out = dH;
       h.ldo = Hd;
@@ -514,7 +544,8 @@ grpo_status grpo_loss_fwd_bwd_norm(const uint16_t* H, const uint16_t* W, const i
       w.N = Hd;
       w.k_dyn = 1;
       w.n_per_unit = 1;
-      w.group_m = group_m(3);
+      w.group_m = group_m(3, di);
+      l2_hints(3, &w.a_hint, &w.b_hint);
       w.status = status;
       w.out = dW + c0 * Hd;
       w.ldo = Hd;
