@@ -228,6 +228,21 @@ def cpu_oracle_sample(w, inp, n_tokens: int):
     return int(m.sum()), dt
 
 
+def cpu_oracle_scoring_sample(w, inp, n_tokens: int):
+    """Times the float64 oracle's log-probs of the first n_tokens unmasked tokens
+    under the policy, old and reference heads (full vocabulary and hidden size)."""
+    import oracle
+    valid = np.flatnonzero(inp["m"])[:n_tokens]
+    m = np.zeros(w.T, np.uint8)
+    m[valid] = 1
+    sl = slice(0, int(valid[-1]) + 1 if valid.size else 1)
+    heads = [inp["W"], wl.gen_weight(w, "old", inp["W"]), wl.gen_weight(w, "ref", inp["W"])]
+    t0 = time.perf_counter()
+    for Wx in heads:
+        oracle.token_logprobs(inp["H"][sl], Wx, inp["y"][sl], m[sl])
+    return int(m.sum()), time.perf_counter() - t0
+
+
 def run_reference(args):
     """The float64 oracle on the host cores, one bounded sample per step."""
     rank = int(os.environ.get("RANK", "0"))
@@ -236,11 +251,12 @@ def run_reference(args):
     w = wl.ALL_WORKLOADS[args.workload]
     inp = make_inputs(w)
     ntok = max(1, args.cpu_sample_tokens // 4)
+    sample_fn = cpu_oracle_scoring_sample if w.name.startswith("logprob") else cpu_oracle_sample
     for _ in range(args.warmup):
-        cpu_oracle_sample(w, inp, ntok)
+        sample_fn(w, inp, ntok)
     toks, secs = 0, 0.0
     for _ in range(args.steps):
-        n, dt = cpu_oracle_sample(w, inp, ntok)
+        n, dt = sample_fn(w, inp, ntok)
         toks += n
         secs += dt
     value = toks / secs
@@ -286,8 +302,9 @@ def main():
 
     base = wl.ALL_WORKLOADS[args.workload]
     w = base if rank == 0 else base.with_(seed=base.seed + 7919 * rank)
+    scoring = w.name.startswith("logprob")  # log-probs of three heads, no loss / backward
     inp = make_inputs(w)
-    if inp["old_src"] is None:
+    if inp["old_src"] is None and not scoring:
         fill_old_ref_on_gpu(w, inp, grpo, torch, dev)
     n_valid = int(inp["m"].sum())
 
@@ -297,21 +314,32 @@ def main():
     H, W = to_dev(inp["H"], torch.bfloat16), to_dev(inp["W"], torch.bfloat16)
     y, m = to_dev(inp["y"], torch.int32), to_dev(inp["m"], torch.uint8)
     old, ref, r = to_dev(inp["old"], torch.float32), to_dev(inp["ref"], torch.float32), to_dev(inp["r"], torch.float32)
-    ws = grpo.workspace(w.T, w.Hd, w.V, grpo.GRPO_WS_LOSS, dev)
-    adv = torch.empty(w.n_resp, dtype=torch.float32, device=dev)
-    out = (torch.empty(1, dtype=torch.float32, device=dev), torch.empty(w.T, w.Hd, dtype=torch.float32, device=dev),
-           torch.empty(w.V, w.Hd, dtype=torch.float32, device=dev))
-
     from paper_2507_05687_gb300 import dp
 
-    def step():
-        grpo.group_advantages(r, w.G, w.adv_eps, out=adv)
-        if dist is None:
-            grpo.loss_fwd_bwd(H, W, y, m, old, ref, adv, w.n_resp, w.L, w.clip_eps, w.beta, 0, ws=ws, out=out)
-        else:
-            # global token-mean over every rank's batch; loss and dW summed over ranks
-            dp.dp_loss_fwd_bwd(H, W, y, m, old, ref, adv, w.n_resp, w.L, w.clip_eps, w.beta, 0, n_valid,
-                               ws=ws, out=out)
+    if scoring:
+        heads = [W, to_dev(wl.gen_weight(w, "old", inp["W"]), torch.bfloat16),
+                 to_dev(wl.gen_weight(w, "ref", inp["W"]), torch.bfloat16)]
+        ws = grpo.workspace(w.T, w.Hd, w.V, grpo.GRPO_WS_LOGPROBS_HEADS, dev)
+        logp3 = torch.empty(len(heads), w.T, dtype=torch.float32, device=dev)
+
+        def step():
+            # policy / old / reference log-probs of one rollout batch; ranks score independently
+            grpo.token_logprobs_heads(H, heads, y, m, ws=ws, out=logp3)
+    else:
+        ws = grpo.workspace(w.T, w.Hd, w.V, grpo.GRPO_WS_LOSS, dev)
+        adv = torch.empty(w.n_resp, dtype=torch.float32, device=dev)
+        out = (torch.empty(1, dtype=torch.float32, device=dev),
+               torch.empty(w.T, w.Hd, dtype=torch.float32, device=dev),
+               torch.empty(w.V, w.Hd, dtype=torch.float32, device=dev))
+
+        def step():
+            grpo.group_advantages(r, w.G, w.adv_eps, out=adv)
+            if dist is None:
+                grpo.loss_fwd_bwd(H, W, y, m, old, ref, adv, w.n_resp, w.L, w.clip_eps, w.beta, 0, ws=ws, out=out)
+            else:
+                # global token-mean over every rank's batch; loss and dW summed over ranks
+                dp.dp_loss_fwd_bwd(H, W, y, m, old, ref, adv, w.n_resp, w.L, w.clip_eps, w.beta, 0, n_valid,
+                                   ws=ws, out=out)
 
     for _ in range(max(3, args.warmup)):
         step()
@@ -363,18 +391,25 @@ def main():
 
     burst, sustained, hbm, peak_src = peaks()
     rf = roofline(trace, n_valid, w.Hd, args.steps, sustained, f"bf16 sustained, {peak_src}")
-    step_flops8 = 8.0 * n_valid * w.Hd * w.V
-    step_flops6 = 6.0 * n_valid * w.Hd * w.V
+    if scoring:
+        step_flops8 = step_flops6 = 2.0 * 3 * n_valid * w.Hd * w.V  # three forward passes, nothing recomputed
+    else:
+        step_flops8 = 8.0 * n_valid * w.Hd * w.V
+        step_flops6 = 6.0 * n_valid * w.Hd * w.V
 
     e2e = None
     if not args.no_e2e and rank == 0:
-        e2e = measure_e2e(grpo, torch, dev, w, inp, steps=min(args.steps, 5))
+        if scoring:
+            e2e = measure_e2e_scoring(grpo, torch, dev, w, inp, heads, steps=min(args.steps, 5))
+        else:
+            e2e = measure_e2e(grpo, torch, dev, w, inp, steps=min(args.steps, 5))
 
     cpu = None
     if not args.no_cpu_baseline and rank == 0 and world == 1:
-        ntok, dt = cpu_oracle_sample(w, inp, args.cpu_sample_tokens)
+        ntok, dt = (cpu_oracle_scoring_sample if scoring else cpu_oracle_sample)(w, inp, args.cpu_sample_tokens)
         cpu = {"value": round(ntok / dt, 2), "unit": "tokens/s", "cores": host_cores(), "kind": "oracle",
-               "sample": f"first {ntok} valid tokens of {w.name}: oracle.loss_fwd_bwd in "
+               "sample": f"first {ntok} valid tokens of {w.name}: "
+                         f"{'oracle.token_logprobs under 3 heads' if scoring else 'oracle.loss_fwd_bwd'} in "
                          f"float64 over the full vocabulary and hidden size, {dt:.1f} s"}
 
     if rank == 0:
@@ -397,6 +432,25 @@ def main():
         print(json.dumps(line), flush=True)
     if dist is not None:
         dist.destroy_process_group()
+
+
+def measure_e2e_scoring(grpo, torch, dev, w, inp, heads, steps: int):
+    """Public API with pinned host buffers: H2D of H and the three heads, the call, D2H of the log-probs."""
+    def pin(a, dt):
+        return torch.from_numpy(np.ascontiguousarray(a)).view(dt).pin_memory()
+
+    hH, hy, hm = pin(inp["H"], torch.bfloat16), pin(inp["y"], torch.int32), pin(inp["m"], torch.uint8)
+    hheads = [h.cpu().pin_memory() for h in heads]
+    h2d = sum(t.numel() * t.element_size() for t in [hH, hy, hm, *hheads])
+    d2h = len(heads) * w.T * 4
+    grpo.token_logprobs_heads(hH, hheads, hy, hm)
+    t0 = time.perf_counter()
+    for _ in range(steps):
+        grpo.token_logprobs_heads(hH, hheads, hy, hm)  # returns a pinned host tensor once it has landed
+    dt = (time.perf_counter() - t0) / steps
+    n_valid = int(inp["m"].sum())
+    return {"value": round(n_valid / dt, 1), "unit": "tokens/s", "ms_per_step": round(dt * 1e3, 2),
+            "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h), "steps": steps}
 
 
 def measure_e2e(grpo, torch, dev, w, inp, steps: int):

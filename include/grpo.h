@@ -47,7 +47,10 @@ typedef enum {
 } grpo_status;
 
 /* Which call a workspace is sized for (grpo_workspace_bytes `which`). */
-enum { GRPO_WS_LOGPROBS = 0, GRPO_WS_LOSS = 1 };
+enum { GRPO_WS_LOGPROBS = 0, GRPO_WS_LOSS = 1, GRPO_WS_LOGPROBS_HEADS = 2 };
+
+/* Most LM heads grpo_token_logprobs_heads sweeps in one call. */
+enum { GRPO_MAX_HEADS = 4 };
 
 /* Loss aggregation (grpo_loss_fwd_bwd `agg_mode`). */
 enum {
@@ -83,6 +86,23 @@ grpo_status grpo_group_advantages(const float* rewards, int64_t n_resp, int32_t 
 grpo_status grpo_token_logprobs(const uint16_t* H, const uint16_t* W, const int32_t* targets,
                                 const uint8_t* mask, int64_t T, int32_t Hd, int64_t V,
                                 float* logp_out, void* ws, size_t ws_bytes, void* stream);
+
+/*
+ * grpo_token_logprobs for n_heads LM heads at once: the log-probs of the same
+ * sampled tokens under the current policy, the old policy (the pi_theta_old
+ * of Eq. 1's ratio) and the reference policy (the pi_ref of Eq. 1's KL term),
+ * as the rollout-scoring step of GRPO needs them.  The unmasked rows are
+ * gathered once and every head is swept in one launch.
+ *   W_heads   HOST array of n_heads device pointers, each a [V x Hd] bf16 head
+ *             (16-byte aligned); 1 <= n_heads <= GRPO_MAX_HEADS
+ *   logp_out  [n_heads x T] fp32 device: row h holds head h's log-probs,
+ *             0 on padding rows
+ *   ws        at least grpo_workspace_bytes(T, Hd, V, GRPO_WS_LOGPROBS_HEADS) bytes
+ * Other arguments and limits as grpo_token_logprobs.
+ */
+grpo_status grpo_token_logprobs_heads(const uint16_t* H, const uint16_t* const* W_heads, int32_t n_heads,
+                                      const int32_t* targets, const uint8_t* mask, int64_t T, int32_t Hd,
+                                      int64_t V, float* logp_out, void* ws, size_t ws_bytes, void* stream);
 
 /*
  * GRPO loss (the negated objective of Eq. 1, Section 3.3) and its gradient
@@ -155,8 +175,8 @@ grpo_status grpo_token_logprobs_noalloc(const uint16_t* H, const uint16_t* W, co
                                         float* logp_out, void* stream);
 
 /*
- * Bytes of workspace the call `which` (GRPO_WS_LOGPROBS or GRPO_WS_LOSS)
- * needs for T tokens, hidden size Hd and vocabulary V.  Returns 0 for
+ * Bytes of workspace the call `which` (GRPO_WS_LOGPROBS, GRPO_WS_LOSS or
+ * GRPO_WS_LOGPROBS_HEADS) needs for T tokens, hidden size Hd and vocabulary V.  Returns 0 for
  * arguments the calls would reject.  Sized for the worst case N_valid = T.
  */
 size_t grpo_workspace_bytes(int64_t T, int32_t Hd, int64_t V, int32_t which);

@@ -29,6 +29,8 @@ GRPO_ERR_TIMEOUT = 5
 GRPO_ERR_UNSUPPORTED = 6
 GRPO_WS_LOGPROBS = 0
 GRPO_WS_LOSS = 1
+GRPO_WS_LOGPROBS_HEADS = 2
+GRPO_MAX_HEADS = 4
 
 # name -> (restype, argtypes); mirrors include/grpo.h
 _P = ctypes.c_void_p
@@ -40,6 +42,8 @@ SIGNATURES = {
     "grpo_token_logprobs": (ctypes.c_int, [_P, _P, _P, _P, _I64, _I32, _I64, _P, _P, ctypes.c_size_t, _P]),
     "grpo_loss_fwd_bwd": (ctypes.c_int, [_P, _P, _P, _P, _P, _P, _P, _I64, _I64, _I32, _I64, _F, _F, _I32,
                                          _P, _P, _P, _P, ctypes.c_size_t, _P]),
+    "grpo_token_logprobs_heads": (ctypes.c_int, [_P, _P, _I32, _P, _P, _I64, _I32, _I64, _P, _P, ctypes.c_size_t,
+                                                 _P]),
     "grpo_loss_fwd_bwd_norm": (ctypes.c_int, [_P, _P, _P, _P, _P, _P, _P, _I64, _I64, _I32, _I64, _F, _F, _I32, _F,
                                               _P, _P, _P, _P, ctypes.c_size_t, _P]),
     "grpo_token_logprobs_noalloc": (ctypes.c_int, [_P, _P, _P, _P, _I64, _I32, _I64, _P, _P]),
@@ -161,6 +165,30 @@ def token_logprobs(H: torch.Tensor, W: torch.Tensor, targets: torch.Tensor, mask
     logp = out if out is not None else torch.empty(T, dtype=torch.float32, device=dev)
     _check(load().grpo_token_logprobs(_ptr(H), _ptr(W), _ptr(targets), _ptr(mask), T, Hd, V, _ptr(logp),
                                       _ptr(ws), ws.numel(), _stream(dev)), "grpo_token_logprobs")
+    return _to_host(logp) if host else logp
+
+
+def token_logprobs_heads(H: torch.Tensor, W_heads, targets: torch.Tensor, mask: torch.Tensor,
+                         ws: Optional[torch.Tensor] = None, out: Optional[torch.Tensor] = None) -> torch.Tensor:
+    """grpo_token_logprobs_heads: log-probs under each head in W_heads (policy,
+    old, reference ...); returns [n_heads, T] fp32, 0 on padding rows."""
+    W_heads = list(W_heads)
+    dev, host = _target_device(H, *W_heads)
+    H = _on_device(H, dev, torch.bfloat16, "H")
+    W_heads = [_on_device(w, dev, torch.bfloat16, f"W_heads[{i}]") for i, w in enumerate(W_heads)]
+    targets = _on_device(targets, dev, torch.int32, "targets")
+    mask = _on_device(mask.view(torch.uint8) if mask.dtype == torch.bool else mask, dev, torch.uint8, "mask")
+    T, Hd = H.shape
+    V = W_heads[0].shape[0]
+    if any(w.shape != W_heads[0].shape for w in W_heads):
+        raise ValueError("all heads must have the same [V, Hd] shape")
+    if ws is None:
+        ws = workspace(T, Hd, V, GRPO_WS_LOGPROBS_HEADS, dev)
+    logp = out if out is not None else torch.empty(len(W_heads), T, dtype=torch.float32, device=dev)
+    ptrs = (ctypes.c_void_p * len(W_heads))(*[w.data_ptr() for w in W_heads])
+    _check(load().grpo_token_logprobs_heads(_ptr(H), ptrs, len(W_heads), _ptr(targets), _ptr(mask), T, Hd, V,
+                                            _ptr(logp), _ptr(ws), ws.numel(), _stream(dev)),
+           "grpo_token_logprobs_heads")
     return _to_host(logp) if host else logp
 
 

@@ -42,6 +42,7 @@ constexpr int kRowsCta = 128;      // accumulator rows per CTA (TMEM lanes)
 constexpr int kGemmThreads = 192;
 constexpr int kTmemCols = 512;
 constexpr int kRowAlign = 256;     // row padding of every token-indexed buffer
+constexpr int kMaxHeads = 4;       // LM heads one forward launch can sweep
 
 template <int kPair>
 struct TileCfg {
@@ -63,6 +64,7 @@ struct GemmArgs {
   int a_off_m, a_off_k; // coordinate offsets into A's tensor map
   int b_off_n, b_off_k; // coordinate offsets into B's tensor map
   int n_per_unit;       // consecutive N tiles one CTA (pair) walks as one work unit
+  int n_heads;          // B matrices (LM heads) swept against the same A, 1..kMaxHeads
   int group_m;          // raster: M tiles per group sharing the same N sweep
   int a_hint, b_hint;   // L2 eviction policy of A / B loads (kHint*)
   unsigned* status;     // device status word
@@ -71,7 +73,7 @@ struct GemmArgs {
   const int* yc;        // [M] target of each compacted row (-1: none)
   float* part_m;        // [units_n x ldp] running max (log2 units)
   float* part_s;        // [units_n x ldp] running sum of 2^(z log2e - max)
-  float* zy;            // [M] logit of the target
+  float* zy;            // [n_heads x ldp] logit of the target
   long ldp;
 
   // kEpiDz
@@ -88,7 +90,7 @@ struct GemmArgs {
 };
 
 struct TileSched {
-  int m_tiles, n_tiles, units_n, total, k_blocks, m_rows;
+  int m_tiles, n_tiles, units_head, units_n, total, k_blocks, m_rows;
 };
 
 __device__ __forceinline__ TileSched make_sched(const GemmArgs& a, int tile_m) {
@@ -97,8 +99,9 @@ __device__ __forceinline__ TileSched make_sched(const GemmArgs& a, int tile_m) {
   s.m_rows = a.m_dyn ? nv : a.M;
   const int K = a.k_dyn ? nv : a.K;
   s.m_tiles = (s.m_rows + tile_m - 1) / tile_m;
-  s.n_tiles = (a.N + kTileN - 1) / kTileN;
-  s.units_n = (s.n_tiles + a.n_per_unit - 1) / a.n_per_unit;
+  s.n_tiles = (a.N + kTileN - 1) / kTileN;  // per head
+  s.units_head = (s.n_tiles + a.n_per_unit - 1) / a.n_per_unit;
+  s.units_n = s.units_head * max(1, a.n_heads);
   s.total = s.m_tiles * s.units_n;
   s.k_blocks = (K + kBK - 1) / kBK;
   return s;
@@ -241,18 +244,18 @@ __device__ __forceinline__ void epi_tile(EpiRow& e, const GemmArgs& a, uint32_t 
 }
 
 template <int kEpi>
-__device__ __forceinline__ void epi_end(const EpiRow& e, const GemmArgs& a, int un) {
+__device__ __forceinline__ void epi_end(const EpiRow& e, const GemmArgs& a, int un, int head) {
   if (kEpi == kEpiLse && e.rv) {
     a.part_m[static_cast<long>(un) * a.ldp + e.r] = e.run_m;
     a.part_s[static_cast<long>(un) * a.ldp + e.r] = e.run_s;
-    if (e.found) a.zy[e.r] = e.zy_val;
+    if (e.found) a.zy[static_cast<long>(head) * a.ldp + e.r] = e.zy_val;
   }
 }
 
 // ---------------------------------------------------------------- kernel body
 
 template <int kPair, int kEpi, bool kAmn, bool kBmn>
-__device__ __forceinline__ void gemm_body(const CUtensorMap* tmA, const CUtensorMap* tmB,
+__device__ __forceinline__ void gemm_body(const CUtensorMap* tmA, const CUtensorMap* const* tmBs,
                                           const GemmArgs& args) {
   using C = TileCfg<kPair>;
   extern __shared__ uint8_t smem_raw[];
@@ -289,7 +292,7 @@ __device__ __forceinline__ void gemm_body(const CUtensorMap* tmA, const CUtensor
   }
   if (warp == 0 && lane == 0) {
     tma_prefetch_desc(tmA);
-    tma_prefetch_desc(tmB);
+    for (int h = 0; h < args.n_heads; ++h) tma_prefetch_desc(tmBs[h]);
   }
   if (warp == 1) {
     if (kPair == 2) {
@@ -329,7 +332,8 @@ __device__ __forceinline__ void gemm_body(const CUtensorMap* tmA, const CUtensor
       for (int u = unit0; u < sch.total && ok; u += unit_stride) {
         int mt, un;
         unit_coords(args, sch, u, mt, un);
-        const int nt0 = un * args.n_per_unit;
+        const int head = un / sch.units_head;
+        const int nt0 = (un - head * sch.units_head) * args.n_per_unit;
         const int nt1 = min(sch.n_tiles, nt0 + args.n_per_unit);
         for (int nt = nt0; nt < nt1 && ok; ++nt) {
           for (int kb = 0; kb < KB; ++kb) {
@@ -357,11 +361,11 @@ __device__ __forceinline__ void gemm_body(const CUtensorMap* tmA, const CUtensor
                 load(sa + j * 8192, tmA, m0 + args.a_off_m + 64 * j, k0 + args.a_off_k, pol_a);
             }
             if (!kBmn) {
-              load(sb, tmB, k0 + args.b_off_k, n0 + args.b_off_n, pol_b);
+              load(sb, tmBs[head], k0 + args.b_off_k, n0 + args.b_off_n, pol_b);
             } else {
 #pragma unroll
               for (int j = 0; j < C::kBRows / 64; ++j)
-                load(sb + j * 8192, tmB, n0 + args.b_off_n + 64 * j, k0 + args.b_off_k, pol_b);
+                load(sb + j * 8192, tmBs[head], n0 + args.b_off_n + 64 * j, k0 + args.b_off_k, pol_b);
             }
             ++uses[stage];
             if (++stage == C::kStages) {
@@ -389,7 +393,8 @@ __device__ __forceinline__ void gemm_body(const CUtensorMap* tmA, const CUtensor
       for (int u = unit0; u < sch.total && ok; u += unit_stride) {
         int mt, un;
         unit_coords(args, sch, u, mt, un);
-        const int nt0 = un * args.n_per_unit;
+        const int head = un / sch.units_head;
+        const int nt0 = (un - head * sch.units_head) * args.n_per_unit;
         const int nt1 = min(sch.n_tiles, nt0 + args.n_per_unit);
         for (int nt = nt0; nt < nt1 && ok; ++nt) {
           if (KB == 0) continue;
@@ -452,7 +457,8 @@ __device__ __forceinline__ void gemm_body(const CUtensorMap* tmA, const CUtensor
     for (int u = unit0; u < sch.total && ok; u += unit_stride) {
       int mt, un;
       unit_coords(args, sch, u, mt, un);
-      const int nt0 = un * args.n_per_unit;
+      const int head = un / sch.units_head;
+      const int nt0 = (un - head * sch.units_head) * args.n_per_unit;
       const int nt1 = min(sch.n_tiles, nt0 + args.n_per_unit);
       EpiRow e;
       epi_begin<kEpi>(e, args, mt * C::kTileM + row, sch.m_rows);
@@ -479,7 +485,7 @@ __device__ __forceinline__ void gemm_body(const CUtensorMap* tmA, const CUtensor
         }
       }
       if (!ok) break;
-      epi_end<kEpi>(e, args, un);
+      epi_end<kEpi>(e, args, un, head);
     }
     if (!ok) raise_abort();
   }
@@ -496,18 +502,23 @@ __device__ __forceinline__ void gemm_body(const CUtensorMap* tmA, const CUtensor
   }
 }
 
+// One tensor map per B matrix; B1..B3 are read only when args.n_heads > 1.
 template <int kEpi, bool kAmn, bool kBmn>
 __global__ void __launch_bounds__(kGemmThreads, 1)
-    gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
-                   const GemmArgs args) {
-  gemm_body<1, kEpi, kAmn, kBmn>(&tmA, &tmB, args);
+    gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB0,
+                   const __grid_constant__ CUtensorMap tmB1, const __grid_constant__ CUtensorMap tmB2,
+                   const __grid_constant__ CUtensorMap tmB3, const GemmArgs args) {
+  const CUtensorMap* tmBs[kMaxHeads] = {&tmB0, &tmB1, &tmB2, &tmB3};
+  gemm_body<1, kEpi, kAmn, kBmn>(&tmA, tmBs, args);
 }
 
 template <int kEpi, bool kAmn, bool kBmn>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
-    gemm_tc_pair_kernel(const __grid_constant__ CUtensorMap tmA,
-                        const __grid_constant__ CUtensorMap tmB, const GemmArgs args) {
-  gemm_body<2, kEpi, kAmn, kBmn>(&tmA, &tmB, args);
+    gemm_tc_pair_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB0,
+                        const __grid_constant__ CUtensorMap tmB1, const __grid_constant__ CUtensorMap tmB2,
+                        const __grid_constant__ CUtensorMap tmB3, const GemmArgs args) {
+  const CUtensorMap* tmBs[kMaxHeads] = {&tmB0, &tmB1, &tmB2, &tmB3};
+  gemm_body<2, kEpi, kAmn, kBmn>(&tmA, tmBs, args);
 }
 
 }  // namespace grpo

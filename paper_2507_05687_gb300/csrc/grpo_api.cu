@@ -46,8 +46,10 @@ struct Layout {
 
 bool make_layout(int64_t T, int32_t Hd, int64_t V, int32_t which, Layout* L) {
   if (T < 0 || T >= (int64_t(1) << 31) || Hd <= 0 || Hd % 64 != 0 || V <= 0 ||
-      V >= (int64_t(1) << 31) || (which != GRPO_WS_LOGPROBS && which != GRPO_WS_LOSS))
+      V >= (int64_t(1) << 31) ||
+      (which != GRPO_WS_LOGPROBS && which != GRPO_WS_LOSS && which != GRPO_WS_LOGPROBS_HEADS))
     return false;
+  const size_t heads = which == GRPO_WS_LOGPROBS_HEADS ? kMaxHeads : 1;
   L->T_pad = round_up(std::max<int64_t>(T, 1), kRowAlign);
   const int64_t vtiles = (V + kTileN - 1) / kTileN;
   L->nsplit = (vtiles + kLseTilesPerUnit - 1) / kLseTilesPerUnit;
@@ -69,9 +71,9 @@ bool make_layout(int64_t T, int32_t Hd, int64_t V, int32_t which, Layout* L) {
   L->cidx = take(4 * tp, 256);
   L->rank_of = take(4 * tp, 256);
   L->yc = take(4 * tp, 256);
-  L->zy = take(4 * tp, 256);
-  L->part_m = take(4 * tp * L->nsplit, 256);
-  L->part_s = take(4 * tp * L->nsplit, 256);
+  L->zy = take(4 * tp * heads, 256);
+  L->part_m = take(4 * tp * L->nsplit * heads, 256);
+  L->part_s = take(4 * tp * L->nsplit * heads, 256);
   L->lse_c = take(4 * tp, 256);
   L->g_c = take(4 * tp, 256);
   L->block_loss = take(8 * L->nblk_loss, 256);
@@ -164,6 +166,18 @@ bool device_info(DeviceInfo* out) {
   }
   *out = cache[dev];
   return true;
+}
+
+// N tiles one CTA (pair) walks per work unit in the backward GEMMs (dZ, dH,
+// dW): consecutive tiles of a unit share the A tile.  GRPO_UNIT_N="z,h,w".
+int units_n(int which) {
+  int u[3] = {1, 1, 1};
+  if (const char* e = std::getenv("GRPO_UNIT_N")) {
+    int v[3];
+    if (std::sscanf(e, "%d,%d,%d", &v[0], &v[1], &v[2]) == 3)
+      for (int i = 0; i < 3; ++i) u[i] = v[i] > 0 ? v[i] : u[i];
+  }
+  return u[which];
 }
 
 // L2 policy of the A and B loads of GEMM `which` (LSE, dZ, dH, dW) as
@@ -271,33 +285,51 @@ struct Operand {
   uint64_t rows, cols, ld;
 };
 
-// Builds the tensor maps of A and B for the tile shape of kPair and launches
-// the persistent GEMM with at most one CTA (pair) per work unit.
+// Builds the tensor maps of A and of each B (one per LM head; a.n_heads of
+// them) for the tile shape of kPair and launches the persistent GEMM with at
+// most one CTA (pair) per work unit.
 template <int kPair, int E, bool AMN, bool BMN>
-cudaError_t launch_gemm_cfg(const Operand& A, const Operand& B, const GemmArgs& a, int64_t max_m_rows,
+cudaError_t launch_gemm_cfg(const Operand& A, const Operand* B, const GemmArgs& args, int64_t max_m_rows,
                             const DeviceInfo& di, cudaStream_t s) {
   using C = TileCfg<kPair>;
-  CUtensorMap ta, tb;
-  if (!encode_2d(&ta, A.base, A.rows, A.cols, A.ld, kBK, AMN ? 64 : kRowsCta) ||
-      !encode_2d(&tb, B.base, B.rows, B.cols, B.ld, kBK, BMN ? 64 : C::kBRows))
-    return cudaErrorInvalidValue;
+  GemmArgs a = args;
+  a.n_heads = std::max(1, std::min(a.n_heads, kMaxHeads));
+  CUtensorMap ta, tb[kMaxHeads];
+  if (!encode_2d(&ta, A.base, A.rows, A.cols, A.ld, kBK, AMN ? 64 : kRowsCta)) return cudaErrorInvalidValue;
+  for (int h = 0; h < kMaxHeads; ++h) {
+    if (h >= a.n_heads) {
+      tb[h] = tb[0];
+      continue;
+    }
+    if (!encode_2d(&tb[h], B[h].base, B[h].rows, B[h].cols, B[h].ld, kBK, BMN ? 64 : C::kBRows))
+      return cudaErrorInvalidValue;
+  }
   const int64_t n_tiles = (a.N + kTileN - 1) / kTileN;
-  const int64_t units = ((max_m_rows + C::kTileM - 1) / C::kTileM) * ((n_tiles + a.n_per_unit - 1) / a.n_per_unit);
+  const int64_t units = ((max_m_rows + C::kTileM - 1) / C::kTileM) *
+                        ((n_tiles + a.n_per_unit - 1) / a.n_per_unit) * a.n_heads;
   if (kPair == 2) {
     const int64_t pairs = std::max<int64_t>(1, std::min<int64_t>(di.pairs, units));
-    gemm_tc_pair_kernel<E, AMN, BMN><<<static_cast<unsigned>(2 * pairs), kGemmThreads, C::kSmemBytes, s>>>(ta, tb, a);
+    gemm_tc_pair_kernel<E, AMN, BMN><<<static_cast<unsigned>(2 * pairs), kGemmThreads, C::kSmemBytes, s>>>(
+        ta, tb[0], tb[1], tb[2], tb[3], a);
   } else {
     const int64_t grid = std::max<int64_t>(1, std::min<int64_t>(di.sms, units));
-    gemm_tc_kernel<E, AMN, BMN><<<static_cast<unsigned>(grid), kGemmThreads, C::kSmemBytes, s>>>(ta, tb, a);
+    gemm_tc_kernel<E, AMN, BMN><<<static_cast<unsigned>(grid), kGemmThreads, C::kSmemBytes, s>>>(
+        ta, tb[0], tb[1], tb[2], tb[3], a);
   }
   return cudaGetLastError();
 }
 
 template <int E, bool AMN, bool BMN>
-cudaError_t launch_gemm(const Operand& A, const Operand& B, const GemmArgs& a, int64_t max_m_rows,
+cudaError_t launch_gemm(const Operand& A, const Operand* B, const GemmArgs& a, int64_t max_m_rows,
                         const DeviceInfo& di, cudaStream_t s) {
   return use_pairs() && di.pairs > 0 ? launch_gemm_cfg<2, E, AMN, BMN>(A, B, a, max_m_rows, di, s)
                                      : launch_gemm_cfg<1, E, AMN, BMN>(A, B, a, max_m_rows, di, s);
+}
+
+template <int E, bool AMN, bool BMN>
+cudaError_t launch_gemm(const Operand& A, const Operand& B, const GemmArgs& a, int64_t max_m_rows,
+                        const DeviceInfo& di, cudaStream_t s) {
+  return launch_gemm<E, AMN, BMN>(A, &B, a, max_m_rows, di, s);
 }
 
 template <typename T>
@@ -330,8 +362,9 @@ cudaError_t run_compaction(const uint16_t* H, const int32_t* targets, const uint
   return cudaGetLastError();
 }
 
-// Forward GEMM with the log-softmax epilogue over all V columns.
-cudaError_t run_lse(const uint16_t* W, int32_t Hd, int64_t V, void* ws, const Layout& Ly,
+// Forward GEMM with the log-softmax epilogue over all V columns of each of
+// the n_heads LM heads (one launch; the heads share the gathered hidden states).
+cudaError_t run_lse(const uint16_t* const* W, int n_heads, int32_t Hd, int64_t V, void* ws, const Layout& Ly,
                     const DeviceInfo& di, cudaStream_t s) {
   GemmArgs a{};
   a.n_valid = at<int>(ws, Ly.n_valid);
@@ -340,6 +373,7 @@ cudaError_t run_lse(const uint16_t* W, int32_t Hd, int64_t V, void* ws, const La
   a.N = static_cast<int>(V);
   a.K = Hd;
   a.n_per_unit = kLseTilesPerUnit;
+  a.n_heads = n_heads;
   a.group_m = group_m(0, di);
   // gathered hidden states: re-read for every vocabulary tile (evict last);
   // W: streamed, shared by the CTAs of one round (evict first)
@@ -352,8 +386,10 @@ cudaError_t run_lse(const uint16_t* W, int32_t Hd, int64_t V, void* ws, const La
   a.ldp = Ly.T_pad;
   const Operand A{at<uint16_t>(ws, Ly.Hc), static_cast<uint64_t>(Ly.T_pad), static_cast<uint64_t>(Hd),
                   static_cast<uint64_t>(Hd)};
-  const Operand B{W, static_cast<uint64_t>(V), static_cast<uint64_t>(Hd), static_cast<uint64_t>(Hd)};
-  TraceScope trace(GRPO_K_LSE_GEMM, V, s);
+  Operand B[kMaxHeads];
+  for (int h = 0; h < n_heads; ++h)
+    B[h] = Operand{W[h], static_cast<uint64_t>(V), static_cast<uint64_t>(Hd), static_cast<uint64_t>(Hd)};
+  TraceScope trace(GRPO_K_LSE_GEMM, V * n_heads, s);
   return launch_gemm<kEpiLse, false, false>(A, B, a, Ly.T_pad, di, s);
 }
 
@@ -414,7 +450,7 @@ grpo_status grpo_token_logprobs(const uint16_t* H, const uint16_t* W, const int3
   if (!get_encode()) return GRPO_ERR_CUDA;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   cudaError_t e = run_compaction(H, targets, mask, T, Hd, V, ws, Ly, di.sms, s);
-  if (e == cudaSuccess) e = run_lse(W, Hd, V, ws, Ly, di, s);
+  if (e == cudaSuccess) e = run_lse(&W, 1, Hd, V, ws, Ly, di, s);
   if (e == cudaSuccess) {
     const int blocks = static_cast<int>(std::min<int64_t>((T + 255) / 256, di.sms * 16));
     TraceScope trace(GRPO_K_LOGP_MERGE, 0, s);
@@ -423,6 +459,40 @@ grpo_status grpo_token_logprobs(const uint16_t* H, const uint16_t* W, const int3
                                              Ly.T_pad, at<float>(ws, Ly.zy), at<int>(ws, Ly.yc),
                                              logp_out, at<unsigned>(ws, Ly.status));
     e = cudaGetLastError();
+  }
+  return from_cuda(e);
+}
+
+grpo_status grpo_token_logprobs_heads(const uint16_t* H, const uint16_t* const* W_heads, int32_t n_heads,
+                                      const int32_t* targets, const uint8_t* mask, int64_t T, int32_t Hd,
+                                      int64_t V, float* logp_out, void* ws, size_t ws_bytes, void* stream) {
+  Layout Ly;
+  if (!make_layout(T, Hd, V, GRPO_WS_LOGPROBS_HEADS, &Ly)) return GRPO_ERR_INVALID_ARG;
+  if (n_heads < 1 || n_heads > kMaxHeads || !W_heads) return GRPO_ERR_INVALID_ARG;
+  for (int h = 0; h < n_heads; ++h)
+    if (!W_heads[h] || !aligned(W_heads[h], 16)) return GRPO_ERR_INVALID_ARG;
+  if (T > 0 && (!H || !targets || !mask || !logp_out)) return GRPO_ERR_INVALID_ARG;
+  if (H && !aligned(H, 16)) return GRPO_ERR_INVALID_ARG;
+  if (!ws || !aligned(ws, 256) || ws_bytes < Ly.total) return GRPO_ERR_WORKSPACE;
+  if (T == 0) return GRPO_OK;
+  DeviceInfo di;
+  if (!device_info(&di)) return GRPO_ERR_UNSUPPORTED;
+  if (!get_encode()) return GRPO_ERR_CUDA;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  cudaError_t e = run_compaction(H, targets, mask, T, Hd, V, ws, Ly, di.sms, s);
+  if (e == cudaSuccess) e = run_lse(W_heads, n_heads, Hd, V, ws, Ly, di, s);
+  if (e == cudaSuccess) {
+    const int blocks = static_cast<int>(std::min<int64_t>((T + 255) / 256, di.sms * 16));
+    TraceScope trace(GRPO_K_LOGP_MERGE, 0, s);
+    for (int h = 0; h < n_heads && e == cudaSuccess; ++h) {
+      const size_t head_parts = static_cast<size_t>(h) * Ly.nsplit * Ly.T_pad;
+      logp_merge_kernel<<<blocks, 256, 0, s>>>(mask, at<int>(ws, Ly.rank_of), T, at<float>(ws, Ly.part_m) + head_parts,
+                                               at<float>(ws, Ly.part_s) + head_parts, static_cast<int>(Ly.nsplit),
+                                               Ly.T_pad, at<float>(ws, Ly.zy) + static_cast<size_t>(h) * Ly.T_pad,
+                                               at<int>(ws, Ly.yc), logp_out + static_cast<size_t>(h) * T,
+                                               at<unsigned>(ws, Ly.status));
+      e = cudaGetLastError();
+    }
   }
   return from_cuda(e);
 }
@@ -469,7 +539,7 @@ grpo_status grpo_loss_fwd_bwd_norm(const uint16_t* H, const uint16_t* W, const i
     resp_len_kernel<<<static_cast<unsigned>(blocks), 256, 0, s>>>(mask, n_resp, L, at<int>(ws, Ly.resp_len));
     e = cudaGetLastError();
   }
-  if (e == cudaSuccess) e = run_lse(W, Hd, V, ws, Ly, di, s);
+  if (e == cudaSuccess) e = run_lse(&W, 1, Hd, V, ws, Ly, di, s);
   if (e == cudaSuccess) {
     TraceScope trace(GRPO_K_LOSS, 0, s);
     loss_terms_kernel<<<static_cast<unsigned>(Ly.nblk_loss), kLossThreads, 0, s>>>(
@@ -505,7 +575,7 @@ grpo_status grpo_loss_fwd_bwd_norm(const uint16_t* H, const uint16_t* W, const i
       a.N = static_cast<int>(width);
       a.K = Hd;
       a.b_off_n = static_cast<int>(c0);
-      a.n_per_unit = 1;
+      a.n_per_unit = units_n(0);
       a.group_m = group_m(1, di);
       l2_hints(1, &a.a_hint, &a.b_hint);
       a.status = status;
@@ -525,7 +595,7 @@ grpo_status grpo_loss_fwd_bwd_norm(const uint16_t* H, const uint16_t* W, const i
       h.N = Hd;
       h.K = static_cast<int>(width);
       h.b_off_k = static_cast<int>(c0);
-      h.n_per_unit = 1;
+      h.n_per_unit = units_n(1);
       h.group_m = group_m(2, di);
       l2_hints(2, &h.a_hint, &h.b_hint);
       h.status = status;
@@ -543,7 +613,7 @@ grpo_status grpo_loss_fwd_bwd_norm(const uint16_t* H, const uint16_t* W, const i
       w.M = static_cast<int>(width);
       w.N = Hd;
       w.k_dyn = 1;
-      w.n_per_unit = 1;
+      w.n_per_unit = units_n(2);
       w.group_m = group_m(3, di);
       l2_hints(3, &w.a_hint, &w.b_hint);
       w.status = status;

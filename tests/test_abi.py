@@ -89,6 +89,18 @@ def test_host_rejections(lib):
     bad = list(largs); bad[18] = ws2 - 1024
     assert L.grpo_loss_fwd_bwd(*bad) == grpo.GRPO_ERR_WORKSPACE
     assert L.grpo_check_device_status(None, None) == grpo.GRPO_ERR_INVALID_ARG
+    ws3 = grpo.workspace_bytes(100, 64, 1000, grpo.GRPO_WS_LOGPROBS_HEADS)
+    assert ws3 > grpo.workspace_bytes(100, 64, 1000, grpo.GRPO_WS_LOGPROBS)
+    heads = (ctypes.c_void_p * 5)(*([FAKE] * 5))
+    hargs = [FAKE, heads, 3, FAKE, FAKE, 100, 64, 1000, FAKE, FAKE, ws3, None]
+    for n in (0, 5):
+        bad = list(hargs); bad[2] = n
+        assert L.grpo_token_logprobs_heads(*bad) == grpo.GRPO_ERR_INVALID_ARG
+    nulls = (ctypes.c_void_p * 3)(FAKE, None, FAKE)
+    bad = list(hargs); bad[1] = nulls
+    assert L.grpo_token_logprobs_heads(*bad) == grpo.GRPO_ERR_INVALID_ARG
+    bad = list(hargs); bad[10] = ws3 - 1
+    assert L.grpo_token_logprobs_heads(*bad) == grpo.GRPO_ERR_WORKSPACE
 
 
 def test_binding_fails_loudly_without_library(tmp_path):

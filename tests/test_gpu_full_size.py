@@ -75,15 +75,23 @@ def test_logprob_three_heads_full_size():
     ws = grpo.workspace(w.T, w.Hd, w.V, grpo.GRPO_WS_LOGPROBS, DEV)
     want = {"policy": _oracle_logp(Hb, Wb, y, idx, gold["lse_policy"]),
             "old": gold["old_logp"].astype(np.float64), "ref": gold["ref_logp"].astype(np.float64)}
+    heads = []
     for which in ("policy", "old", "ref"):
-        Wx = Wb if which == "policy" else wl.gen_weight(w, which, Wb)
-        lp = grpo.token_logprobs(H, dev_tensor(Wx, torch.bfloat16), yd, md, ws=ws)
+        Wx = dev_tensor(Wb if which == "policy" else wl.gen_weight(w, which, Wb), torch.bfloat16)
+        heads.append(Wx)
+        lp = grpo.token_logprobs(H, Wx, yd, md, ws=ws)
         assert grpo.check_device_status(ws) == grpo.GRPO_OK
         got = lp.cpu().numpy()
         assert np.all(got[m == 0] == 0.0)
         err = np.abs(got[idx].astype(np.float64) - want[which])
         assert err.max() <= LOGP_ATOL, (which, err.max())
-        del Wx
+    # the three heads in one call (the configuration bench.py times for this workload)
+    ws3 = grpo.workspace(w.T, w.Hd, w.V, grpo.GRPO_WS_LOGPROBS_HEADS, DEV)
+    lp3 = grpo.token_logprobs_heads(H, heads, yd, md, ws=ws3)
+    assert grpo.check_device_status(ws3) == grpo.GRPO_OK
+    for h, which in enumerate(("policy", "old", "ref")):
+        err = np.abs(lp3[h].cpu().numpy()[idx].astype(np.float64) - want[which])
+        assert err.max() <= LOGP_ATOL, (which, err.max())
 
 
 def _sample_rows(w, m, idx, r, k=96):

@@ -111,6 +111,25 @@ def test_logprobs_match_oracle(shape):
     assert err.max() <= LOGP_ATOL, err.max()
 
 
+@pytest.mark.parametrize("n_heads", [1, 2, 3, 4])
+def test_logprobs_heads_match_oracle_and_single_calls(n_heads):
+    """Policy / old / reference (and a fourth) heads in one call: each row matches
+    the oracle, and the single-head call bit for bit."""
+    w = wl.Workload("t", 2, 3, 120, 256, 4400, "uniform", 1, 120, seed=wl.SEED_BASE + 1500 + n_heads)
+    Hb, Wb, y, m = wl.gen_hidden(w), wl.gen_weight(w), wl.gen_targets(w), wl.gen_mask(w)
+    heads = [Wb, wl.gen_weight(w, "old", Wb), wl.gen_weight(w, "ref", Wb), wl.gen_weight(w.with_(w_std=0.05))][:n_heads]
+    H, yd, md = dev_tensor(Hb, torch.bfloat16), dev_tensor(y, torch.int32), dev_tensor(m, torch.uint8)
+    Wd = [dev_tensor(x, torch.bfloat16) for x in heads]
+    got = grpo.token_logprobs_heads(H, Wd, yd, md)
+    assert got.shape == (n_heads, w.T)
+    for h in range(n_heads):
+        want, _ = oracle.token_logprobs(Hb, heads[h], y, m)
+        g = got[h].cpu().numpy()
+        assert np.all(g[m == 0] == 0.0)
+        assert np.abs(g - want).max() <= LOGP_ATOL
+        assert torch.equal(got[h], grpo.token_logprobs(H, Wd[h], yd, md))
+
+
 def test_logprobs_large_logits_and_host_buffers():
     w = wl.Workload("t", 2, 2, 70, 128, 777, "uniform", 1, 70, seed=wl.SEED_BASE + 77, w_std=0.5)
     Hb, Wb, y, m = wl.gen_hidden(w), wl.gen_weight(w), wl.gen_targets(w), wl.gen_mask(w)
