@@ -465,9 +465,14 @@ def measure_e2e(grpo, torch, dev, w, inp, steps: int):
     h2d = sum(t.numel() * t.element_size() for t in (hH, hW, hy, hm, hold, href, hr))
     d2h = 4 + w.T * w.Hd * 4 + w.V * w.Hd * 4
 
+    # the caller's own buffers, allocated once: pinned host outputs and a device workspace
+    hout = (torch.empty(1, dtype=torch.float32).pin_memory(), torch.empty(w.T, w.Hd, dtype=torch.float32).pin_memory(),
+            torch.empty(w.V, w.Hd, dtype=torch.float32).pin_memory())
+    ws = grpo.workspace(w.T, w.Hd, w.V, grpo.GRPO_WS_LOSS, dev)
+
     def one():
         adv = grpo.group_advantages(hr.to(dev, non_blocking=True), w.G, w.adv_eps)
-        return grpo.loss_fwd_bwd(hH, hW, hy, hm, hold, href, adv, w.n_resp, w.L, w.clip_eps, w.beta)
+        return grpo.loss_fwd_bwd(hH, hW, hy, hm, hold, href, adv, w.n_resp, w.L, w.clip_eps, w.beta, ws=ws, out=hout)
 
     one()
     torch.cuda.synchronize(dev)

@@ -115,11 +115,12 @@ def _target_device(*ts: torch.Tensor) -> Tuple[torch.device, bool]:
     return torch.device("cuda", torch.cuda.current_device()), True
 
 
-def _to_host(*ts: torch.Tensor):
-    """Pinned host copies of device results; returns once they have landed."""
+def _to_host(*ts: torch.Tensor, dst=None):
+    """Host copies of device results (into `dst` host tensors when given,
+    else new pinned ones); returns once they have landed."""
     outs = []
-    for t in ts:
-        o = torch.empty(t.shape, dtype=t.dtype, pin_memory=True)
+    for i, t in enumerate(ts):
+        o = dst[i] if dst is not None else torch.empty(t.shape, dtype=t.dtype, pin_memory=True)
         o.copy_(t, non_blocking=True)
         outs.append(o)
     torch.cuda.current_stream(ts[0].device).synchronize()
@@ -198,7 +199,9 @@ def loss_fwd_bwd(H: torch.Tensor, W: torch.Tensor, targets: torch.Tensor, mask: 
                  ws: Optional[torch.Tensor] = None,
                  out: Optional[Tuple[torch.Tensor, torch.Tensor, torch.Tensor]] = None, norm: float = 0.0):
     """grpo_loss_fwd_bwd (norm == 0) / grpo_loss_fwd_bwd_norm (norm > 0, a global
-    N_valid or n_resp): returns (loss [1] fp32, dH [T, Hd] fp32, dW [V, Hd] fp32)."""
+    N_valid or n_resp): returns (loss [1] fp32, dH [T, Hd] fp32, dW [V, Hd] fp32).
+    `out` may be device tensors (written in place) or host tensors, preferably
+    pinned (the results are copied there before the call returns)."""
     dev, host = _target_device(H, W)
     H = _on_device(H, dev, torch.bfloat16, "H")
     W = _on_device(W, dev, torch.bfloat16, "W")
@@ -211,6 +214,9 @@ def loss_fwd_bwd(H: torch.Tensor, W: torch.Tensor, targets: torch.Tensor, mask: 
     V = W.shape[0]
     if ws is None:
         ws = workspace(T, Hd, V, GRPO_WS_LOSS, dev)
+    host_out = None
+    if out is not None and not out[0].is_cuda:
+        host_out, out = out, None  # results land in the caller's host buffers
     if out is None:
         out = (torch.empty(1, dtype=torch.float32, device=dev),
                torch.empty(T, Hd, dtype=torch.float32, device=dev),
@@ -224,8 +230,8 @@ def loss_fwd_bwd(H: torch.Tensor, W: torch.Tensor, targets: torch.Tensor, mask: 
         _check(lib.grpo_loss_fwd_bwd_norm(*common, float(norm), *tail), "grpo_loss_fwd_bwd_norm")
     else:
         _check(lib.grpo_loss_fwd_bwd(*common, *tail), "grpo_loss_fwd_bwd")
-    if host:
-        return _to_host(loss, dH, dW)
+    if host or host_out is not None:
+        return _to_host(loss, dH, dW, dst=host_out)
     return loss, dH, dW
 
 
