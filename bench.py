@@ -38,7 +38,7 @@ GOLDEN = {"fwdbwd_8b": "batch8b", "logprob3_8b": "batch8b", "long_8b": "long_8b"
 KERNEL_SOURCES = ["paper_2507_05687_gb300/csrc/gemm_tc.cuh", "paper_2507_05687_gb300/csrc/ptx.cuh",
                   "paper_2507_05687_gb300/csrc/grpo_api.cu"]
 KIND_NAMES = ["advantages", "compact", "lse_gemm", "logp_merge", "loss", "dz_gemm", "dh_gemm", "dw_gemm",
-              "zero_rows"]
+              "zero_rows", "adamw"]
 KERNELS_PER_SCOPE = {1: 4, 4: 2}  # compaction scope = 4 kernels, loss scope = 2 kernels; others 1
 
 
@@ -49,6 +49,9 @@ def parse():
     p.add_argument("--warmup", type=int, default=3)
     p.add_argument("--impl", choices=["ours", "reference"], default="ours")
     p.add_argument("--workload", default="fwdbwd_8b", choices=sorted(wl.ALL_WORKLOADS))
+    p.add_argument("--adamw", choices=["none", "fused", "separate"], default="none",
+                   help="fwd+bwd workloads: add the AdamW step of the LM head, fused into the dW GEMM "
+                        "or as a separate pass over the stored dW")
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--cpu-sample-tokens", type=int, default=1024,
@@ -332,9 +335,27 @@ def main():
                torch.empty(w.T, w.Hd, dtype=torch.float32, device=dev),
                torch.empty(w.V, w.Hd, dtype=torch.float32, device=dev))
 
+        if args.adamw != "none":
+            master = W.float()
+            exp_avg, exp_avg_sq = torch.zeros_like(master), torch.zeros_like(master)
+            adam_step = [0]
+
         def step():
             grpo.group_advantages(r, w.G, w.adv_eps, out=adv)
-            if dist is None:
+            if args.adamw == "separate":
+                adam_step[0] += 1
+                grpo.loss_fwd_bwd(H, W, y, m, old, ref, adv, w.n_resp, w.L, w.clip_eps, w.beta, 0, ws=ws, out=out)
+                grpo.adamw_step(master, exp_avg, exp_avg_sq, out[2], W, adam_step[0], lr=1e-6)
+            elif args.adamw == "fused":
+                # loss, dH and the actor's AdamW step on the LM head (lr 1e-6) in one call; dW is never stored
+                adam_step[0] += 1
+                norm = 0.0
+                if dist is not None:
+                    norm = dp.global_count(n_valid, dev)
+                grpo.loss_fwd_bwd_adamw(H, W, y, m, old, ref, adv, w.n_resp, w.L, master, exp_avg, exp_avg_sq,
+                                        adam_step[0], lr=1e-6, clip_eps=w.clip_eps, beta=w.beta, norm=norm, ws=ws,
+                                        out=out[:2])
+            elif dist is None:
                 grpo.loss_fwd_bwd(H, W, y, m, old, ref, adv, w.n_resp, w.L, w.clip_eps, w.beta, 0, ws=ws, out=out)
             else:
                 # global token-mean over every rank's batch; loss and dW summed over ranks
@@ -423,7 +444,7 @@ def main():
                        "parallelism": f"dp{world}",
                        "l2": "inputs larger than L2 (W %.2f GB, H %.2f GB per rank)" % (w.V * w.Hd * 2 / 1e9,
                                                                                          w.T * w.Hd * 2 / 1e9),
-                       "old_ref_logp": inp["old_src"]},
+                       "old_ref_logp": inp["old_src"], "adamw": args.adamw},
             "step_tflops_8x": round(step_flops8 / (ms / 1e3) / 1e12, 1),
             "step_frac_8x": round(step_flops8 / (ms / 1e3) / 1e12 / burst, 4),
             "step_frac_6x": round(step_flops6 / (ms / 1e3) / 1e12 / burst, 4),

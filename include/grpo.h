@@ -147,6 +147,41 @@ grpo_status grpo_loss_fwd_bwd_norm(const uint16_t* H, const uint16_t* W, const i
                                    void* stream);
 
 /*
+ * grpo_loss_fwd_bwd_norm followed by the actor's optimiser step on the LM
+ * head, with the step fused into the dW GEMM: each dW tile is consumed in
+ * place by one AdamW step (Adam with decoupled weight decay) and dW itself is
+ * never written.  The paper sets the actor learning rate (1e-6, Section 4.1)
+ * but not the optimiser; AdamW is the reading taken:
+ *   m <- beta1 m + (1 - beta1) g,  v <- beta2 v + (1 - beta2) g^2,
+ *   W_master <- W_master (1 - lr wd) - lr (m / (1 - beta1^step)) / (sqrt(v / (1 - beta2^step)) + eps)
+ *   W_master, exp_avg, exp_avg_sq   [V x Hd] fp32 device, updated in place
+ *   W_out                           [V x Hd] bf16 device, receives bf16(W_master);
+ *                                   may be W itself (the rows of a vocabulary chunk are
+ *                                   no longer read when its update runs)
+ *   step >= 1 (bias correction), 0 <= beta1, beta2 < 1, eps > 0, lr >= 0, weight_decay >= 0.
+ * Everything else as grpo_loss_fwd_bwd_norm (loss_out and dH are written).
+ */
+grpo_status grpo_loss_fwd_bwd_adamw(const uint16_t* H, const uint16_t* W, const int32_t* targets,
+                                    const uint8_t* mask, const float* old_logp, const float* ref_logp,
+                                    const float* adv, int64_t n_resp, int64_t L, int32_t Hd, int64_t V,
+                                    float clip_eps, float beta, int32_t agg_mode, float norm, float lr,
+                                    float beta1, float beta2, float eps, float weight_decay, int64_t step,
+                                    float* W_master, float* exp_avg, float* exp_avg_sq, uint16_t* W_out,
+                                    float* loss_out, float* dH, void* ws, size_t ws_bytes, void* stream);
+
+/*
+ * One AdamW step over n fp32 elements (the same update as
+ * grpo_loss_fwd_bwd_adamw, as a separate bandwidth-bound pass over a stored
+ * gradient, e.g. the dW of grpo_loss_fwd_bwd).  W_master, exp_avg,
+ * exp_avg_sq are updated in place; W_out receives bf16(W_master).  All
+ * pointers are device memory, 16-byte aligned; n % 4 == 0.  Hyper-parameter
+ * limits as grpo_loss_fwd_bwd_adamw.
+ */
+grpo_status grpo_adamw_step(float* W_master, float* exp_avg, float* exp_avg_sq, const float* grad,
+                            uint16_t* W_out, int64_t n, float lr, float beta1, float beta2, float eps,
+                            float weight_decay, int64_t step, void* stream);
+
+/*
  * grpo_token_logprobs without a workspace argument, for callers that cannot
  * allocate device memory themselves: code running where cudaMalloc is not
  * allowed or would stall the device (inside a stream capture, in a real-time
@@ -205,7 +240,8 @@ enum {
   GRPO_K_DZ_GEMM = 5,     /* recomputed logits -> dZ chunk (bf16) */
   GRPO_K_DH_GEMM = 6,     /* dH (+)= dZ_chunk W_chunk */
   GRPO_K_DW_GEMM = 7,     /* dW_chunk = dZ_chunk^T H */
-  GRPO_K_ZERO_ROWS = 8    /* zero dH rows of padding tokens */
+  GRPO_K_ZERO_ROWS = 8,   /* zero dH rows of padding tokens */
+  GRPO_K_ADAMW = 9        /* standalone AdamW step (grpo_adamw_step) */
 };
 
 /*

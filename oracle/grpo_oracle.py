@@ -263,3 +263,28 @@ def dW_rows(H, W, targets, mask, lse, g, vrows, row_chunk: int = 8192) -> np.nda
         dZ += hit * gr[:, None]
         out += dZ.T @ Hr
     return out
+
+
+# ---------------------------------------------------------------------------
+# the update that consumes dW: the actor's optimiser step
+# ---------------------------------------------------------------------------
+
+
+def adamw_step(theta, m, v, g, lr: float, beta1: float, beta2: float, eps: float,
+               weight_decay: float, step: int):
+    """One AdamW step (Adam with decoupled weight decay), float64.
+
+    The paper fixes only the actor learning rate (1e-6, Section 4.1); the
+    optimiser is read as AdamW:
+        m <- beta1 m + (1 - beta1) g
+        v <- beta2 v + (1 - beta2) g^2
+        theta <- theta (1 - lr wd) - lr (m / (1 - beta1^t)) / (sqrt(v / (1 - beta2^t)) + eps)
+    Returns (theta, m, v) as new arrays.
+    """
+    th = np.asarray(theta, dtype=np.float64)
+    m1 = beta1 * np.asarray(m, dtype=np.float64) + (1.0 - beta1) * np.asarray(g, dtype=np.float64)
+    v1 = beta2 * np.asarray(v, dtype=np.float64) + (1.0 - beta2) * np.asarray(g, dtype=np.float64) ** 2
+    mhat = m1 / (1.0 - beta1 ** step)
+    vhat = v1 / (1.0 - beta2 ** step)
+    th1 = th * (1.0 - lr * weight_decay) - lr * mhat / (np.sqrt(vhat) + eps)
+    return th1, m1, v1

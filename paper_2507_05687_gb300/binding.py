@@ -46,6 +46,10 @@ SIGNATURES = {
                                                  _P]),
     "grpo_loss_fwd_bwd_norm": (ctypes.c_int, [_P, _P, _P, _P, _P, _P, _P, _I64, _I64, _I32, _I64, _F, _F, _I32, _F,
                                               _P, _P, _P, _P, ctypes.c_size_t, _P]),
+    "grpo_loss_fwd_bwd_adamw": (ctypes.c_int, [_P, _P, _P, _P, _P, _P, _P, _I64, _I64, _I32, _I64, _F, _F, _I32, _F,
+                                               _F, _F, _F, _F, _F, _I64, _P, _P, _P, _P, _P, _P, _P,
+                                               ctypes.c_size_t, _P]),
+    "grpo_adamw_step": (ctypes.c_int, [_P, _P, _P, _P, _P, _I64, _F, _F, _F, _F, _F, _I64, _P]),
     "grpo_token_logprobs_noalloc": (ctypes.c_int, [_P, _P, _P, _P, _I64, _I32, _I64, _P, _P]),
     "grpo_workspace_bytes": (ctypes.c_size_t, [_I64, _I32, _I64, _I32]),
     "grpo_check_device_status": (ctypes.c_int, [_P, _P]),
@@ -233,6 +237,59 @@ def loss_fwd_bwd(H: torch.Tensor, W: torch.Tensor, targets: torch.Tensor, mask: 
     if host or host_out is not None:
         return _to_host(loss, dH, dW, dst=host_out)
     return loss, dH, dW
+
+
+def loss_fwd_bwd_adamw(H: torch.Tensor, W: torch.Tensor, targets: torch.Tensor, mask: torch.Tensor,
+                       old_logp: torch.Tensor, ref_logp: torch.Tensor, adv: torch.Tensor, n_resp: int, L: int,
+                       W_master: torch.Tensor, exp_avg: torch.Tensor, exp_avg_sq: torch.Tensor, step: int,
+                       lr: float = 1e-6, betas=(0.9, 0.999), eps: float = 1e-8, weight_decay: float = 0.01,
+                       clip_eps: float = 0.2, beta: float = 0.04, agg_mode: int = 0, norm: float = 0.0,
+                       W_out: Optional[torch.Tensor] = None, ws: Optional[torch.Tensor] = None,
+                       out: Optional[Tuple[torch.Tensor, torch.Tensor]] = None):
+    """grpo_loss_fwd_bwd_adamw: loss and dH as loss_fwd_bwd; the LM-head gradient
+    is consumed by an AdamW step on W_master / exp_avg / exp_avg_sq (device fp32,
+    in place) and W_out (bf16, default W itself).  Returns (loss, dH)."""
+    dev = W.device
+    if not (H.is_cuda and W.is_cuda and W_master.is_cuda and exp_avg.is_cuda and exp_avg_sq.is_cuda):
+        raise ValueError("loss_fwd_bwd_adamw takes device tensors")
+    H = _on_device(H, dev, torch.bfloat16, "H")
+    targets = _on_device(targets, dev, torch.int32, "targets")
+    mask = _on_device(mask.view(torch.uint8) if mask.dtype == torch.bool else mask, dev, torch.uint8, "mask")
+    old_logp = _on_device(old_logp, dev, torch.float32, "old_logp")
+    ref_logp = _on_device(ref_logp, dev, torch.float32, "ref_logp")
+    adv = _on_device(adv, dev, torch.float32, "adv")
+    for name, t in (("W_master", W_master), ("exp_avg", exp_avg), ("exp_avg_sq", exp_avg_sq)):
+        if t.dtype != torch.float32 or not t.is_contiguous() or t.shape != W.shape:
+            raise ValueError(f"{name}: contiguous fp32 [V, Hd] expected")
+    W_out = W if W_out is None else W_out
+    T, Hd = H.shape
+    V = W.shape[0]
+    if ws is None:
+        ws = workspace(T, Hd, V, GRPO_WS_LOSS, dev)
+    if out is None:
+        out = (torch.empty(1, dtype=torch.float32, device=dev), torch.empty(T, Hd, dtype=torch.float32, device=dev))
+    loss, dH = out
+    _check(load().grpo_loss_fwd_bwd_adamw(
+        _ptr(H), _ptr(W), _ptr(targets), _ptr(mask), _ptr(old_logp), _ptr(ref_logp), _ptr(adv), int(n_resp), int(L),
+        Hd, V, float(clip_eps), float(beta), int(agg_mode), float(norm), float(lr), float(betas[0]), float(betas[1]),
+        float(eps), float(weight_decay), int(step), _ptr(W_master), _ptr(exp_avg), _ptr(exp_avg_sq), _ptr(W_out),
+        _ptr(loss), _ptr(dH), _ptr(ws), ws.numel(), _stream(dev)), "grpo_loss_fwd_bwd_adamw")
+    return loss, dH
+
+
+def adamw_step(W_master: torch.Tensor, exp_avg: torch.Tensor, exp_avg_sq: torch.Tensor, grad: torch.Tensor,
+               W_out: torch.Tensor, step: int, lr: float = 1e-6, betas=(0.9, 0.999), eps: float = 1e-8,
+               weight_decay: float = 0.01) -> None:
+    """grpo_adamw_step: one AdamW step in place over contiguous fp32 device tensors."""
+    n = W_master.numel()
+    for name, t in (("exp_avg", exp_avg), ("exp_avg_sq", exp_avg_sq), ("grad", grad)):
+        if t.numel() != n or t.dtype != torch.float32 or not t.is_contiguous():
+            raise ValueError(f"{name}: contiguous fp32 with W_master's size expected")
+    if W_out.numel() != n or W_out.dtype != torch.bfloat16:
+        raise ValueError("W_out: bf16 with W_master's size expected")
+    _check(load().grpo_adamw_step(_ptr(W_master), _ptr(exp_avg), _ptr(exp_avg_sq), _ptr(grad), _ptr(W_out), n,
+                                  float(lr), float(betas[0]), float(betas[1]), float(eps), float(weight_decay),
+                                  int(step), _stream(W_master.device)), "grpo_adamw_step")
 
 
 def check_device_status(ws: torch.Tensor) -> int:

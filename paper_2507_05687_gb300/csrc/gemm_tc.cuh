@@ -23,6 +23,9 @@
 //            writes dZ = g (onehot(y) - softmax) as bf16.
 //   kEpiF32  plain fp32 store (optionally added to the existing values) with
 //            an optional row map: dH += dZ W and dW = dZ^T H.
+//   kEpiAdam dW = dZ^T H consumed in place by an AdamW step on the matching
+//            LM-head rows (fp32 master, both moments, bf16 weights out), so
+//            dW itself is never stored.
 //
 // Operands may be K-major (rows of the matrix run along K) or MN-major (rows
 // run along M or N); the MN-major forms let dH and dW read W, H and dZ in the
@@ -55,7 +58,7 @@ struct TileCfg {
   static constexpr int kSmemBytes = kStages * kStageBytes + 1024 /*align*/ + 256 /*barriers*/;
 };
 
-enum { kEpiLse = 0, kEpiDz = 1, kEpiF32 = 2 };
+enum { kEpiLse = 0, kEpiDz = 1, kEpiF32 = 2, kEpiAdam = 3 };
 
 struct GemmArgs {
   const int* n_valid;   // device: number of compacted rows
@@ -87,6 +90,17 @@ struct GemmArgs {
   long ldo;
   int accumulate;       // 1: out += acc, 0: out = acc
   const int* row_map;   // optional: output row of accumulator row r
+
+  // kEpiAdam: the accumulator is a dW tile; an AdamW step is applied to the
+  // matching weights in place (row stride ldo) instead of storing dW.
+  float* master;        // fp32 weights
+  float* exp_avg;       // first moment
+  float* exp_avg_sq;    // second moment
+  uint16_t* w_out;      // bf16 copy of the updated weights
+  float adam_b1, adam_b2, adam_eps, adam_lr;
+  float adam_decay;     // 1 - lr * weight_decay
+  float adam_bc1;       // 1 / (1 - beta1^step)
+  float adam_bc2;       // 1 / (1 - beta2^step)
 };
 
 struct TileSched {
@@ -160,8 +174,17 @@ __device__ __forceinline__ void epi_begin(EpiRow& e, const GemmArgs& a, int r, i
   }
 }
 
+// One AdamW step of one weight element from its gradient g (fp32).
+__device__ __forceinline__ void adam_update(float g, float& theta, float& m, float& v, const GemmArgs& a) {
+  m = a.adam_b1 * m + (1.f - a.adam_b1) * g;
+  v = a.adam_b2 * v + (1.f - a.adam_b2) * g * g;
+  theta = theta * a.adam_decay - a.adam_lr * (m * a.adam_bc1) / (sqrtf(v * a.adam_bc2) + a.adam_eps);
+}
+
 // One 256-column accumulator tile of this thread's row; `tbase` is the TMEM
-// address of column 0 of the tile in this warp's lane quarter.
+// address of column 0 of the tile in this warp's lane quarter.  Each thread
+// moves its own row with 16-byte vectors (measured faster than transposing
+// 32x32 blocks through shared memory for warp-contiguous scalar accesses).
 template <int kEpi>
 __device__ __forceinline__ void epi_tile(EpiRow& e, const GemmArgs& a, uint32_t tbase, int col0,
                                          bool have_acc) {
@@ -216,6 +239,50 @@ __device__ __forceinline__ void epi_tile(EpiRow& e, const GemmArgs& a, uint32_t 
 #pragma unroll
       for (int q = 0; q < 4; ++q)
         dst[q] = make_uint4(packed[4 * q], packed[4 * q + 1], packed[4 * q + 2], packed[4 * q + 3]);
+    } else if (kEpi == kEpiAdam) {
+      if (e.rv) {
+        const long base = static_cast<long>(e.r) * a.ldo + cb;
+        if (cb + 32 <= a.N) {
+          float4* __restrict__ P = reinterpret_cast<float4*>(a.master + base);
+          float4* __restrict__ M = reinterpret_cast<float4*>(a.exp_avg + base);
+          float4* __restrict__ S = reinterpret_cast<float4*>(a.exp_avg_sq + base);
+          uint2* __restrict__ O = reinterpret_cast<uint2*>(a.w_out + base);
+          // all 24 loads of the 32 columns in flight at once, then the math, then the stores
+          float4 p[8], m[8], sq[8];
+#pragma unroll
+          for (int q = 0; q < 8; ++q) {
+            p[q] = __ldcs(P + q);
+            m[q] = __ldcs(M + q);
+            sq[q] = __ldcs(S + q);
+          }
+#pragma unroll
+          for (int q = 0; q < 8; ++q) {
+            adam_update(v[4 * q + 0], p[q].x, m[q].x, sq[q].x, a);
+            adam_update(v[4 * q + 1], p[q].y, m[q].y, sq[q].y, a);
+            adam_update(v[4 * q + 2], p[q].z, m[q].z, sq[q].z, a);
+            adam_update(v[4 * q + 3], p[q].w, m[q].w, sq[q].w, a);
+          }
+#pragma unroll
+          for (int q = 0; q < 8; ++q) {
+            __stcs(P + q, p[q]);
+            __stcs(M + q, m[q]);
+            __stcs(S + q, sq[q]);
+            O[q] = make_uint2(pack_bf16x2(p[q].x, p[q].y), pack_bf16x2(p[q].z, p[q].w));
+          }
+        } else {
+#pragma unroll
+          for (int j = 0; j < 32; ++j) {
+            if (cb + j < a.N) {
+              float p = a.master[base + j], m = a.exp_avg[base + j], sq = a.exp_avg_sq[base + j];
+              adam_update(v[j], p, m, sq, a);
+              a.master[base + j] = p;
+              a.exp_avg[base + j] = m;
+              a.exp_avg_sq[base + j] = sq;
+              a.w_out[base + j] = static_cast<uint16_t>(pack_bf16x2(p, 0.f) & 0xFFFFu);
+            }
+          }
+        }
+      }
     } else {
       if (e.rv) {
         float* dst = a.out + static_cast<long>(e.orow) * a.ldo + cb;

@@ -4,6 +4,7 @@
 #include <cuda_runtime.h>
 #include <cudaTypedefs.h>
 
+#include <cmath>
 #include <cstdint>
 #include <cstdio>
 #include <cstdlib>
@@ -158,7 +159,8 @@ bool device_info(DeviceInfo* out) {
       return false;
     if (major != 10 || minor != 3) return false;
     if (!prepare_kernels<kEpiLse, false, false>(&pairs) || !prepare_kernels<kEpiDz, false, false>(&pairs) ||
-        !prepare_kernels<kEpiF32, false, true>(&pairs) || !prepare_kernels<kEpiF32, true, true>(&pairs))
+        !prepare_kernels<kEpiF32, false, true>(&pairs) || !prepare_kernels<kEpiF32, true, true>(&pairs) ||
+        !prepare_kernels<kEpiAdam, true, true>(&pairs))
       return false;
     cache[dev].sms = sms;
     cache[dev].pairs = std::max(pairs, 0);
@@ -395,6 +397,21 @@ cudaError_t run_lse(const uint16_t* const* W, int n_heads, int32_t Hd, int64_t V
 
 grpo_status from_cuda(cudaError_t e) { return e == cudaSuccess ? GRPO_OK : GRPO_ERR_CUDA; }
 
+// AdamW step fused into the dW GEMM (grpo_loss_fwd_bwd_adamw).
+struct AdamParams {
+  float* master;
+  float* exp_avg;
+  float* exp_avg_sq;
+  uint16_t* w_out;
+  float b1, b2, eps, lr, decay, bc1, bc2;
+};
+
+grpo_status loss_impl(const uint16_t* H, const uint16_t* W, const int32_t* targets, const uint8_t* mask,
+                      const float* old_logp, const float* ref_logp, const float* adv, int64_t n_resp,
+                      int64_t L, int32_t Hd, int64_t V, float clip_eps, float beta, int32_t agg_mode,
+                      float norm, float* loss_out, float* dH, float* dW, const AdamParams* adam, void* ws,
+                      size_t ws_bytes, void* stream);
+
 }  // namespace
 
 extern "C" {
@@ -512,6 +529,49 @@ grpo_status grpo_loss_fwd_bwd_norm(const uint16_t* H, const uint16_t* W, const i
                                    float clip_eps, float beta, int32_t agg_mode, float norm,
                                    float* loss_out, float* dH, float* dW, void* ws, size_t ws_bytes,
                                    void* stream) {
+  return loss_impl(H, W, targets, mask, old_logp, ref_logp, adv, n_resp, L, Hd, V, clip_eps, beta, agg_mode,
+                   norm, loss_out, dH, dW, nullptr, ws, ws_bytes, stream);
+}
+
+grpo_status grpo_loss_fwd_bwd_adamw(const uint16_t* H, const uint16_t* W, const int32_t* targets,
+                                    const uint8_t* mask, const float* old_logp, const float* ref_logp,
+                                    const float* adv, int64_t n_resp, int64_t L, int32_t Hd, int64_t V,
+                                    float clip_eps, float beta, int32_t agg_mode, float norm, float lr,
+                                    float beta1, float beta2, float eps, float weight_decay, int64_t step,
+                                    float* W_master, float* exp_avg, float* exp_avg_sq, uint16_t* W_out,
+                                    float* loss_out, float* dH, void* ws, size_t ws_bytes, void* stream) {
+  if (!W_master || !exp_avg || !exp_avg_sq || !W_out || !aligned(W_master, 16) || !aligned(exp_avg, 16) ||
+      !aligned(exp_avg_sq, 16) || !aligned(W_out, 16))
+    return GRPO_ERR_INVALID_ARG;
+  if (step < 1 || !(lr >= 0.f) || !(beta1 >= 0.f && beta1 < 1.f) || !(beta2 >= 0.f && beta2 < 1.f) ||
+      !(eps > 0.f) || !(weight_decay >= 0.f))
+    return GRPO_ERR_INVALID_ARG;
+  AdamParams ap{};
+  ap.master = W_master;
+  ap.exp_avg = exp_avg;
+  ap.exp_avg_sq = exp_avg_sq;
+  ap.w_out = W_out;
+  ap.b1 = beta1;
+  ap.b2 = beta2;
+  ap.eps = eps;
+  ap.lr = lr;
+  ap.decay = static_cast<float>(1.0 - static_cast<double>(lr) * weight_decay);
+  ap.bc1 = static_cast<float>(1.0 / (1.0 - std::pow(static_cast<double>(beta1), static_cast<double>(step))));
+  ap.bc2 = static_cast<float>(1.0 / (1.0 - std::pow(static_cast<double>(beta2), static_cast<double>(step))));
+  // dW is not stored: pass the master weights as a placeholder output pointer
+  return loss_impl(H, W, targets, mask, old_logp, ref_logp, adv, n_resp, L, Hd, V, clip_eps, beta, agg_mode,
+                   norm, loss_out, dH, W_master, &ap, ws, ws_bytes, stream);
+}
+
+}  // extern "C"
+
+namespace {
+
+grpo_status loss_impl(const uint16_t* H, const uint16_t* W, const int32_t* targets, const uint8_t* mask,
+                      const float* old_logp, const float* ref_logp, const float* adv, int64_t n_resp,
+                      int64_t L, int32_t Hd, int64_t V, float clip_eps, float beta, int32_t agg_mode,
+                      float norm, float* loss_out, float* dH, float* dW, const AdamParams* adam, void* ws,
+                      size_t ws_bytes, void* stream) {
   if (n_resp < 1 || L < 1 || n_resp > (int64_t(1) << 31) / L) return GRPO_ERR_INVALID_ARG;
   if (!(norm >= 0.f) || norm == INFINITY) return GRPO_ERR_INVALID_ARG;
   const int64_t T = n_resp * L;
@@ -607,7 +667,7 @@ grpo_status grpo_loss_fwd_bwd_norm(const uint16_t* H, const uint16_t* W, const i
       e = launch_gemm<kEpiF32, false, true>(opDz, opW, h, Ly.T_pad, di, s);
     }
     if (e != cudaSuccess) break;
-    {  // dW_c = dZ_c^T Hc
+    {  // dW_c = dZ_c^T Hc (stored, or consumed by the AdamW step)
       GemmArgs w{};
       w.n_valid = n_valid;
       w.M = static_cast<int>(width);
@@ -621,10 +681,55 @@ grpo_status grpo_loss_fwd_bwd_norm(const uint16_t* H, const uint16_t* W, const i
       w.ldo = Hd;
       w.accumulate = 0;
       TraceScope trace(GRPO_K_DW_GEMM, width, s);
-      e = launch_gemm<kEpiF32, true, true>(opDz, opHc, w, width, di, s);
+      if (adam) {
+        const int64_t off = c0 * Hd;
+        w.master = adam->master + off;
+        w.exp_avg = adam->exp_avg + off;
+        w.exp_avg_sq = adam->exp_avg_sq + off;
+        w.w_out = adam->w_out + off;
+        w.adam_b1 = adam->b1;
+        w.adam_b2 = adam->b2;
+        w.adam_eps = adam->eps;
+        w.adam_lr = adam->lr;
+        w.adam_decay = adam->decay;
+        w.adam_bc1 = adam->bc1;
+        w.adam_bc2 = adam->bc2;
+        e = launch_gemm<kEpiAdam, true, true>(opDz, opHc, w, width, di, s);
+      } else {
+        e = launch_gemm<kEpiF32, true, true>(opDz, opHc, w, width, di, s);
+      }
     }
   }
   return from_cuda(e);
+}
+
+}  // namespace
+
+extern "C" {
+
+grpo_status grpo_adamw_step(float* W_master, float* exp_avg, float* exp_avg_sq, const float* grad,
+                            uint16_t* W_out, int64_t n, float lr, float beta1, float beta2, float eps,
+                            float weight_decay, int64_t step, void* stream) {
+  if (n < 0 || n % 4 != 0) return GRPO_ERR_INVALID_ARG;
+  if (n == 0) return GRPO_OK;
+  if (!W_master || !exp_avg || !exp_avg_sq || !grad || !W_out || !aligned(W_master, 16) ||
+      !aligned(exp_avg, 16) || !aligned(exp_avg_sq, 16) || !aligned(grad, 16) || !aligned(W_out, 16))
+    return GRPO_ERR_INVALID_ARG;
+  if (step < 1 || !(lr >= 0.f) || !(beta1 >= 0.f && beta1 < 1.f) || !(beta2 >= 0.f && beta2 < 1.f) ||
+      !(eps > 0.f) || !(weight_decay >= 0.f))
+    return GRPO_ERR_INVALID_ARG;
+  DeviceInfo di;
+  if (!device_info(&di)) return GRPO_ERR_UNSUPPORTED;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const float decay = static_cast<float>(1.0 - static_cast<double>(lr) * weight_decay);
+  const float bc1 = static_cast<float>(1.0 / (1.0 - std::pow(static_cast<double>(beta1), static_cast<double>(step))));
+  const float bc2 = static_cast<float>(1.0 / (1.0 - std::pow(static_cast<double>(beta2), static_cast<double>(step))));
+  const int64_t n4 = n / 4;
+  const int blocks = static_cast<int>(std::min<int64_t>((n4 + 255) / 256, static_cast<int64_t>(di.sms) * 8));
+  TraceScope trace(GRPO_K_ADAMW, 0, s);
+  adamw_kernel<<<blocks, 256, 0, s>>>(W_master, exp_avg, exp_avg_sq, grad, W_out, n4, beta1, beta2, eps, lr,
+                                      decay, bc1, bc2);
+  return from_cuda(cudaGetLastError());
 }
 
 grpo_status grpo_trace_enable(int32_t enable) {

@@ -298,6 +298,34 @@ __global__ void loss_final_kernel(const double* __restrict__ block_loss, const i
   }
 }
 
+// One AdamW step over n contiguous fp32 elements (n % 4 == 0), 16-byte vectors,
+// grid-stride: theta, m, v updated in place from the gradient g, bf16 copy out.
+__global__ void adamw_kernel(float* __restrict__ theta, float* __restrict__ m, float* __restrict__ v,
+                             const float* __restrict__ g, uint16_t* __restrict__ w_out, int64_t n4, float b1,
+                             float b2, float eps, float lr, float decay, float bc1, float bc2) {
+  for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < n4;
+       i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+    float4 t = __ldcs(reinterpret_cast<float4*>(theta) + i);
+    float4 mm = __ldcs(reinterpret_cast<float4*>(m) + i);
+    float4 vv = __ldcs(reinterpret_cast<float4*>(v) + i);
+    const float4 gg = __ldcs(reinterpret_cast<const float4*>(g) + i);
+    float* tp = &t.x;
+    float* mp = &mm.x;
+    float* vp = &vv.x;
+    const float* gp = &gg.x;
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      mp[k] = b1 * mp[k] + (1.f - b1) * gp[k];
+      vp[k] = b2 * vp[k] + (1.f - b2) * gp[k] * gp[k];
+      tp[k] = tp[k] * decay - lr * (mp[k] * bc1) / (sqrtf(vp[k] * bc2) + eps);
+    }
+    __stcs(reinterpret_cast<float4*>(theta) + i, t);
+    __stcs(reinterpret_cast<float4*>(m) + i, mm);
+    __stcs(reinterpret_cast<float4*>(v) + i, vv);
+    reinterpret_cast<uint2*>(w_out)[i] = make_uint2(pack_bf16x2(t.x, t.y), pack_bf16x2(t.z, t.w));
+  }
+}
+
 // dH rows of padding tokens are 0 (the GEMM only writes unmasked rows).
 __global__ void zero_masked_rows_kernel(const uint8_t* __restrict__ mask, int64_t T, int Hd,
                                         float* __restrict__ dH) {

@@ -278,6 +278,39 @@ def test_all_masked_batch_is_zero():
 
 
 # ---------------------------------------------------------------------------
+# the optimiser step that consumes dW
+# ---------------------------------------------------------------------------
+
+def test_adamw_first_step_closed_form():
+    g = np.array([3.0, -2e-3, 0.5, 0.0])
+    th = np.array([1.0, -1.0, 0.25, 2.0])
+    lr, wd, eps = 1e-3, 0.01, 1e-8
+    t1, m1, v1 = oracle.adamw_step(th, np.zeros(4), np.zeros(4), g, lr, 0.9, 0.999, eps, wd, 1)
+    # step 1 from zero moments: m_hat = g, v_hat = g^2
+    np.testing.assert_allclose(m1, 0.1 * g, rtol=1e-15)
+    np.testing.assert_allclose(v1, 0.001 * g * g, rtol=1e-15)
+    np.testing.assert_allclose(t1, th * (1 - lr * wd) - lr * g / (np.abs(g) + eps), rtol=1e-12)
+
+
+def test_adamw_matches_torch_optimizer():
+    torch = pytest.importorskip("torch")
+    rng = np.random.default_rng(9)
+    th0 = rng.normal(size=(5, 7))
+    grads = [rng.normal(size=(5, 7)) * s for s in (1.0, 0.3, 2.0)]
+    p = torch.nn.Parameter(torch.from_numpy(th0.copy()))
+    opt = torch.optim.AdamW([p], lr=1e-3, betas=(0.9, 0.95), eps=1e-8, weight_decay=0.1)
+    th, m, v = th0, np.zeros_like(th0), np.zeros_like(th0)
+    for t, g in enumerate(grads, start=1):
+        p.grad = torch.from_numpy(g.copy())
+        opt.step()
+        th, m, v = oracle.adamw_step(th, m, v, g, 1e-3, 0.9, 0.95, 1e-8, 0.1, t)
+    np.testing.assert_allclose(th, p.detach().numpy(), rtol=0, atol=1e-13)
+    st = opt.state[p]
+    np.testing.assert_allclose(m, st["exp_avg"].numpy(), rtol=1e-13)
+    np.testing.assert_allclose(v, st["exp_avg_sq"].numpy(), rtol=1e-13)
+
+
+# ---------------------------------------------------------------------------
 # planted mistakes: each must trip one of the pins above
 # ---------------------------------------------------------------------------
 
@@ -323,3 +356,13 @@ def test_planted_gradient_sign_is_caught(monkeypatch):
     with pytest.raises(AssertionError):
         test_gradient_matches_central_differences(0)
     monkeypatch.setattr(go, "logp_coef", real)
+
+
+def test_planted_adam_bias_correction_is_caught(monkeypatch):
+    def bad(theta, m, v, g, lr, beta1, beta2, eps, weight_decay, step):
+        m1 = beta1 * m + (1 - beta1) * g
+        v1 = beta2 * v + (1 - beta2) * g * g
+        return theta * (1 - lr * weight_decay) - lr * m1 / (np.sqrt(v1) + eps), m1, v1  # no bias correction
+    monkeypatch.setattr(oracle, "adamw_step", bad)
+    with pytest.raises(AssertionError):
+        test_adamw_first_step_closed_form()
