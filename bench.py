@@ -38,7 +38,7 @@ GOLDEN = {"fwdbwd_8b": "batch8b", "logprob3_8b": "batch8b", "long_8b": "long_8b"
 KERNEL_SOURCES = ["paper_2507_05687_gb300/csrc/gemm_tc.cuh", "paper_2507_05687_gb300/csrc/ptx.cuh",
                   "paper_2507_05687_gb300/csrc/grpo_api.cu"]
 KIND_NAMES = ["advantages", "compact", "lse_gemm", "logp_merge", "loss", "dz_gemm", "dh_gemm", "dw_gemm",
-              "zero_rows", "adamw"]
+              "zero_rows", "adamw", "sample_gemm"]
 KERNELS_PER_SCOPE = {1: 4, 4: 2}  # compaction scope = 4 kernels, loss scope = 2 kernels; others 1
 
 
@@ -52,6 +52,8 @@ def parse():
     p.add_argument("--adamw", choices=["none", "fused", "separate"], default="none",
                    help="fwd+bwd workloads: add the AdamW step of the LM head, fused into the dW GEMM "
                         "or as a separate pass over the stored dW")
+    p.add_argument("--sample", action="store_true",
+                   help="time the rollout draw (grpo_sample_tokens) over the workload's rows instead")
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--cpu-sample-tokens", type=int, default=1024,
@@ -188,7 +190,7 @@ def roofline(trace, n_valid_total_per_rank, Hd, steps, peak_tf, peak_kind):
     by = {}
     for kind, cols, ms in trace:
         by.setdefault(kind, []).append((cols, ms))
-    gemm_kinds = [2, 5, 6, 7]
+    gemm_kinds = [2, 5, 6, 7, 10]
     dom = max(gemm_kinds, key=lambda k: sum(ms for _, ms in by.get(k, [])) if k in by else -1)
     recs = by[dom]
     flops = [2.0 * n_valid_total_per_rank * Hd * cols for cols, _ in recs]
@@ -305,9 +307,10 @@ def main():
 
     base = wl.ALL_WORKLOADS[args.workload]
     w = base if rank == 0 else base.with_(seed=base.seed + 7919 * rank)
-    scoring = w.name.startswith("logprob")  # log-probs of three heads, no loss / backward
+    sampling = args.sample  # the rollout draw over every unmasked row
+    scoring = w.name.startswith("logprob") and not sampling  # log-probs of three heads, no loss / backward
     inp = make_inputs(w)
-    if inp["old_src"] is None and not scoring:
+    if inp["old_src"] is None and not scoring and not sampling:
         fill_old_ref_on_gpu(w, inp, grpo, torch, dev)
     n_valid = int(inp["m"].sum())
 
@@ -319,7 +322,15 @@ def main():
     old, ref, r = to_dev(inp["old"], torch.float32), to_dev(inp["ref"], torch.float32), to_dev(inp["r"], torch.float32)
     from paper_2507_05687_gb300 import dp
 
-    if scoring:
+    if sampling:
+        ws = grpo.workspace(w.T, w.Hd, w.V, grpo.GRPO_WS_SAMPLE, dev)
+        tok_out = (torch.empty(w.T, dtype=torch.int32, device=dev), torch.empty(w.T, dtype=torch.float32, device=dev))
+        draw = [0]
+
+        def step():
+            draw[0] += 1  # a new offset per step: a fresh draw
+            grpo.sample_tokens(H, W, m, 1.0, seed=w.seed, offset=draw[0], ws=ws, out=tok_out)
+    elif scoring:
         heads = [W, to_dev(wl.gen_weight(w, "old", inp["W"]), torch.bfloat16),
                  to_dev(wl.gen_weight(w, "ref", inp["W"]), torch.bfloat16)]
         ws = grpo.workspace(w.T, w.Hd, w.V, grpo.GRPO_WS_LOGPROBS_HEADS, dev)
@@ -412,21 +423,23 @@ def main():
 
     burst, sustained, hbm, peak_src = peaks()
     rf = roofline(trace, n_valid, w.Hd, args.steps, sustained, f"bf16 sustained, {peak_src}")
-    if scoring:
+    if sampling:
+        step_flops8 = step_flops6 = 2.0 * n_valid * w.Hd * w.V
+    elif scoring:
         step_flops8 = step_flops6 = 2.0 * 3 * n_valid * w.Hd * w.V  # three forward passes, nothing recomputed
     else:
         step_flops8 = 8.0 * n_valid * w.Hd * w.V
         step_flops6 = 6.0 * n_valid * w.Hd * w.V
 
     e2e = None
-    if not args.no_e2e and rank == 0:
+    if not args.no_e2e and rank == 0 and not sampling:
         if scoring:
             e2e = measure_e2e_scoring(grpo, torch, dev, w, inp, heads, steps=min(args.steps, 5))
         else:
             e2e = measure_e2e(grpo, torch, dev, w, inp, steps=min(args.steps, 5))
 
     cpu = None
-    if not args.no_cpu_baseline and rank == 0 and world == 1:
+    if not args.no_cpu_baseline and rank == 0 and world == 1 and not sampling:
         ntok, dt = (cpu_oracle_scoring_sample if scoring else cpu_oracle_sample)(w, inp, args.cpu_sample_tokens)
         cpu = {"value": round(ntok / dt, 2), "unit": "tokens/s", "cores": host_cores(), "kind": "oracle",
                "sample": f"first {ntok} valid tokens of {w.name}: "
@@ -444,7 +457,8 @@ def main():
                        "parallelism": f"dp{world}",
                        "l2": "inputs larger than L2 (W %.2f GB, H %.2f GB per rank)" % (w.V * w.Hd * 2 / 1e9,
                                                                                          w.T * w.Hd * 2 / 1e9),
-                       "old_ref_logp": inp["old_src"], "adamw": args.adamw},
+                       "old_ref_logp": inp["old_src"], "adamw": args.adamw,
+                       "step": "sample" if sampling else ("score3" if scoring else "fwdbwd")},
             "step_tflops_8x": round(step_flops8 / (ms / 1e3) / 1e12, 1),
             "step_frac_8x": round(step_flops8 / (ms / 1e3) / 1e12 / burst, 4),
             "step_frac_6x": round(step_flops6 / (ms / 1e3) / 1e12 / burst, 4),

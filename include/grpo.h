@@ -47,7 +47,7 @@ typedef enum {
 } grpo_status;
 
 /* Which call a workspace is sized for (grpo_workspace_bytes `which`). */
-enum { GRPO_WS_LOGPROBS = 0, GRPO_WS_LOSS = 1, GRPO_WS_LOGPROBS_HEADS = 2 };
+enum { GRPO_WS_LOGPROBS = 0, GRPO_WS_LOSS = 1, GRPO_WS_LOGPROBS_HEADS = 2, GRPO_WS_SAMPLE = 3 };
 
 /* Most LM heads grpo_token_logprobs_heads sweeps in one call. */
 enum { GRPO_MAX_HEADS = 4 };
@@ -103,6 +103,24 @@ grpo_status grpo_token_logprobs(const uint16_t* H, const uint16_t* W, const int3
 grpo_status grpo_token_logprobs_heads(const uint16_t* H, const uint16_t* const* W_heads, int32_t n_heads,
                                       const int32_t* targets, const uint8_t* mask, int64_t T, int32_t Hd,
                                       int64_t V, float* logp_out, void* ws, size_t ws_bytes, void* stream);
+
+/*
+ * The rollout draw of Eq. 1, {o_i} ~ pi_theta_old: for every unmasked row t,
+ * sample o_t from softmax(H_t W^T / temperature) by the Gumbel-max rule
+ *   o_t = argmax_v  z_{t,v} / temperature + G_{t,v}   (lowest v on a tie)
+ * with G = -log(-log U) and U = ((w >> 9) + 1/2) / 2^23, w = word (v mod 4) of
+ * Philox4x32-10 at counter (v / 4, t, offset mod 2^32, offset / 2^32) and key
+ * (seed mod 2^32, seed / 2^32).  The logits never reach memory.
+ *   mask        [T] uint8 device: rows to sample (0: token -1, log-prob 0)
+ *   tokens_out  [T] int32 device, the sampled token ids
+ *   logp_out    [T] fp32 device, log softmax(z_t / temperature) at the sampled token
+ *   ws          at least grpo_workspace_bytes(T, Hd, V, GRPO_WS_SAMPLE) bytes
+ * temperature must be finite and > 0; the same (seed, offset) gives the same draw.
+ * Other arguments and limits as grpo_token_logprobs.
+ */
+grpo_status grpo_sample_tokens(const uint16_t* H, const uint16_t* W, const uint8_t* mask, int64_t T, int32_t Hd,
+                               int64_t V, float temperature, uint64_t seed, uint64_t offset, int32_t* tokens_out,
+                               float* logp_out, void* ws, size_t ws_bytes, void* stream);
 
 /*
  * GRPO loss (the negated objective of Eq. 1, Section 3.3) and its gradient
@@ -210,8 +228,8 @@ grpo_status grpo_token_logprobs_noalloc(const uint16_t* H, const uint16_t* W, co
                                         float* logp_out, void* stream);
 
 /*
- * Bytes of workspace the call `which` (GRPO_WS_LOGPROBS, GRPO_WS_LOSS or
- * GRPO_WS_LOGPROBS_HEADS) needs for T tokens, hidden size Hd and vocabulary V.  Returns 0 for
+ * Bytes of workspace the call `which` (GRPO_WS_LOGPROBS, GRPO_WS_LOSS,
+ * GRPO_WS_LOGPROBS_HEADS or GRPO_WS_SAMPLE) needs for T tokens, hidden size Hd and vocabulary V.  Returns 0 for
  * arguments the calls would reject.  Sized for the worst case N_valid = T.
  */
 size_t grpo_workspace_bytes(int64_t T, int32_t Hd, int64_t V, int32_t which);
@@ -241,7 +259,8 @@ enum {
   GRPO_K_DH_GEMM = 6,     /* dH (+)= dZ_chunk W_chunk */
   GRPO_K_DW_GEMM = 7,     /* dW_chunk = dZ_chunk^T H */
   GRPO_K_ZERO_ROWS = 8,   /* zero dH rows of padding tokens */
-  GRPO_K_ADAMW = 9        /* standalone AdamW step (grpo_adamw_step) */
+  GRPO_K_ADAMW = 9,       /* standalone AdamW step (grpo_adamw_step) */
+  GRPO_K_SAMPLE_GEMM = 10 /* logits GEMM + log-sum-exp + Gumbel-max draw */
 };
 
 /*

@@ -288,3 +288,72 @@ def adamw_step(theta, m, v, g, lr: float, beta1: float, beta2: float, eps: float
     vhat = v1 / (1.0 - beta2 ** step)
     th1 = th * (1.0 - lr * weight_decay) - lr * mhat / (np.sqrt(vhat) + eps)
     return th1, m1, v1
+
+
+# ---------------------------------------------------------------------------
+# the rollout side: sampling o_{i,t} ~ pi_theta_old (Eq. 1's {o_i} ~ pi_old)
+# ---------------------------------------------------------------------------
+
+
+def gumbel_noise(seed: int, offset: int, rows, V: int, cols=None) -> np.ndarray:
+    """G[t, v] = -log(-log U) with U the uniform of Philox4x32-10 word (v mod 4) at
+    counter (v div 4, t, offset mod 2^32, offset div 2^32), key (seed mod 2^32, seed div 2^32).
+    `rows` are token positions t; returns float64 [len(rows), V] (or [len(rows), len(cols)])."""
+    from .philox import philox4x32_10, uniform_open
+    t = np.asarray(rows, dtype=np.uint64)[:, None]
+    v = np.arange(V, dtype=np.uint64) if cols is None else np.asarray(cols, dtype=np.uint64)
+    words = philox4x32_10(v[None, :] >> np.uint64(2), t, offset & 0xFFFFFFFF, (offset >> 32) & 0xFFFFFFFF,
+                          seed & 0xFFFFFFFF, (seed >> 32) & 0xFFFFFFFF)
+    sel = (v & np.uint64(3))[None, :]
+    w = np.where(sel == 0, words[0], np.where(sel == 1, words[1], np.where(sel == 2, words[2], words[3])))
+    return -np.log(-np.log(uniform_open(w)))
+
+
+def sample_tokens(H, W, mask, temperature: float, seed: int, offset: int, rows=None, vocab_chunk: int = 8192):
+    """Gumbel-max sampling from softmax(H_t W^T / temperature) at the listed
+    (or all unmasked) rows: y_t = argmax_v (z_{t,v} / temperature + G[t, v]),
+    the lowest v on ties.  Returns (tokens int64 [-1 on masked], logp of the
+    sampled token under softmax(z / temperature), gap between the best and
+    second-best perturbed score) for every row (masked rows: -1, 0, inf)."""
+    Hf = np.asarray(H)
+    Wf = as_f64(W)
+    T, V = Hf.shape[0], Wf.shape[0]
+    m = np.asarray(mask) != 0
+    idx = np.flatnonzero(m) if rows is None else np.asarray(rows, dtype=np.int64)
+    tokens = np.full(T, -1, dtype=np.int64)
+    logp = np.zeros(T)
+    gap = np.full(T, np.inf)
+    inv_t = 1.0 / temperature
+    for r0 in range(0, idx.size, 256):
+        rr = idx[r0:r0 + 256]
+        rr = rr[m[rr]]
+        if rr.size == 0:
+            continue
+        Hr = as_f64(Hf[rr])
+        best = np.full(rr.size, -np.inf)
+        second = np.full(rr.size, -np.inf)
+        arg = np.zeros(rr.size, dtype=np.int64)
+        zbest = np.zeros(rr.size)
+        run_max = np.full(rr.size, -np.inf)
+        run_sum = np.zeros(rr.size)
+        for v0 in range(0, V, vocab_chunk):
+            v1 = min(V, v0 + vocab_chunk)
+            Z = (Hr @ Wf[v0:v1].T) * inv_t
+            S = Z + gumbel_noise(seed, offset, rr, V, cols=np.arange(v0, v1))
+            j = np.argmax(S, axis=1)
+            sj = S[np.arange(rr.size), j]
+            S2 = S.copy()
+            S2[np.arange(rr.size), j] = -np.inf
+            s2 = S2.max(axis=1)
+            better = sj > best
+            second = np.where(better, np.maximum(best, s2), np.maximum(second, sj))
+            zbest = np.where(better, Z[np.arange(rr.size), j], zbest)
+            arg = np.where(better, v0 + j, arg)
+            best = np.where(better, sj, best)
+            nm = np.maximum(run_max, Z.max(axis=1))
+            run_sum = run_sum * np.exp(run_max - nm) + np.exp(Z - nm[:, None]).sum(axis=1)
+            run_max = nm
+        tokens[rr] = arg
+        logp[rr] = zbest - (run_max + np.log(run_sum))
+        gap[rr] = best - second
+    return tokens, logp, gap

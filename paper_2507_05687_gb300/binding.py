@@ -30,6 +30,7 @@ GRPO_ERR_UNSUPPORTED = 6
 GRPO_WS_LOGPROBS = 0
 GRPO_WS_LOSS = 1
 GRPO_WS_LOGPROBS_HEADS = 2
+GRPO_WS_SAMPLE = 3
 GRPO_MAX_HEADS = 4
 
 # name -> (restype, argtypes); mirrors include/grpo.h
@@ -49,6 +50,8 @@ SIGNATURES = {
     "grpo_loss_fwd_bwd_adamw": (ctypes.c_int, [_P, _P, _P, _P, _P, _P, _P, _I64, _I64, _I32, _I64, _F, _F, _I32, _F,
                                                _F, _F, _F, _F, _F, _I64, _P, _P, _P, _P, _P, _P, _P,
                                                ctypes.c_size_t, _P]),
+    "grpo_sample_tokens": (ctypes.c_int, [_P, _P, _P, _I64, _I32, _I64, _F, ctypes.c_uint64, ctypes.c_uint64, _P, _P,
+                                          _P, ctypes.c_size_t, _P]),
     "grpo_adamw_step": (ctypes.c_int, [_P, _P, _P, _P, _P, _I64, _F, _F, _F, _F, _F, _I64, _P]),
     "grpo_token_logprobs_noalloc": (ctypes.c_int, [_P, _P, _P, _P, _I64, _I32, _I64, _P, _P]),
     "grpo_workspace_bytes": (ctypes.c_size_t, [_I64, _I32, _I64, _I32]),
@@ -195,6 +198,27 @@ def token_logprobs_heads(H: torch.Tensor, W_heads, targets: torch.Tensor, mask: 
                                             _ptr(logp), _ptr(ws), ws.numel(), _stream(dev)),
            "grpo_token_logprobs_heads")
     return _to_host(logp) if host else logp
+
+
+def sample_tokens(H: torch.Tensor, W: torch.Tensor, mask: torch.Tensor, temperature: float = 1.0, seed: int = 0,
+                  offset: int = 0, ws: Optional[torch.Tensor] = None, out=None):
+    """grpo_sample_tokens: Gumbel-max draw from softmax(H W^T / temperature) at
+    the unmasked rows; returns (tokens int32 [T] (-1 masked), logp fp32 [T])."""
+    dev, host = _target_device(H, W)
+    H = _on_device(H, dev, torch.bfloat16, "H")
+    W = _on_device(W, dev, torch.bfloat16, "W")
+    mask = _on_device(mask.view(torch.uint8) if mask.dtype == torch.bool else mask, dev, torch.uint8, "mask")
+    T, Hd = H.shape
+    V = W.shape[0]
+    if ws is None:
+        ws = workspace(T, Hd, V, GRPO_WS_SAMPLE, dev)
+    if out is None:
+        out = (torch.empty(T, dtype=torch.int32, device=dev), torch.empty(T, dtype=torch.float32, device=dev))
+    tok, logp = out
+    _check(load().grpo_sample_tokens(_ptr(H), _ptr(W), _ptr(mask), T, Hd, V, float(temperature),
+                                     int(seed) & (2 ** 64 - 1), int(offset) & (2 ** 64 - 1), _ptr(tok), _ptr(logp),
+                                     _ptr(ws), ws.numel(), _stream(dev)), "grpo_sample_tokens")
+    return _to_host(tok, logp) if host else (tok, logp)
 
 
 def loss_fwd_bwd(H: torch.Tensor, W: torch.Tensor, targets: torch.Tensor, mask: torch.Tensor,

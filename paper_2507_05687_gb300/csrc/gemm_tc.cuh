@@ -23,6 +23,10 @@
 //            writes dZ = g (onehot(y) - softmax) as bf16.
 //   kEpiF32  plain fp32 store (optionally added to the existing values) with
 //            an optional row map: dH += dZ W and dW = dZ^T H.
+//   kEpiSample  the rollout draw o_t ~ softmax(z_t / temperature): per row the
+//            running log-sum-exp of z / temperature and the running argmax of
+//            z / temperature + Gumbel noise (Philox4x32-10, counter = (v / 4, t,
+//            offset), key = seed); the logits never leave the SM.
 //   kEpiAdam dW = dZ^T H consumed in place by an AdamW step on the matching
 //            LM-head rows (fp32 master, both moments, bf16 weights out), so
 //            dW itself is never stored.
@@ -58,7 +62,7 @@ struct TileCfg {
   static constexpr int kSmemBytes = kStages * kStageBytes + 1024 /*align*/ + 256 /*barriers*/;
 };
 
-enum { kEpiLse = 0, kEpiDz = 1, kEpiF32 = 2, kEpiAdam = 3 };
+enum { kEpiLse = 0, kEpiDz = 1, kEpiF32 = 2, kEpiAdam = 3, kEpiSample = 4 };
 
 struct GemmArgs {
   const int* n_valid;   // device: number of compacted rows
@@ -101,6 +105,13 @@ struct GemmArgs {
   float adam_decay;     // 1 - lr * weight_decay
   float adam_bc1;       // 1 / (1 - beta1^step)
   float adam_bc2;       // 1 / (1 - beta2^step)
+
+  // kEpiSample (row_map gives the token position t of each compacted row)
+  float inv_temp;       // 1 / temperature
+  uint32_t seed_lo, seed_hi, off_lo, off_hi;
+  float* best_s;        // [units_n x ldp] best perturbed score of the split
+  int* best_c;          // [units_n x ldp] its vocabulary column
+  float* best_z;        // [units_n x ldp] its z / temperature
 };
 
 struct TileSched {
@@ -145,7 +156,9 @@ struct EpiRow {
   bool found;
   int y;
   float lse2, gr;  // kEpiDz
-  int orow;        // kEpiF32
+  int orow;        // kEpiF32; kEpiSample: token position t
+  float best_s, best_z;  // kEpiSample
+  int best_c;
 };
 
 template <int kEpi>
@@ -161,7 +174,12 @@ __device__ __forceinline__ void epi_begin(EpiRow& e, const GemmArgs& a, int r, i
   e.lse2 = 0.f;
   e.gr = 0.f;
   e.orow = -1;
-  if (kEpi == kEpiLse) {
+  e.best_s = -INFINITY;
+  e.best_z = -INFINITY;
+  e.best_c = -1;
+  if (kEpi == kEpiSample) {
+    if (e.rv) e.orow = a.row_map[r];
+  } else if (kEpi == kEpiLse) {
     e.y = e.rv ? a.yc[r] : -1;
   } else if (kEpi == kEpiDz) {
     if (e.rv) {
@@ -212,6 +230,38 @@ __device__ __forceinline__ void epi_tile(EpiRow& e, const GemmArgs& a, uint32_t 
         for (int j = 1; j < 32; ++j) t = (off == static_cast<unsigned>(j)) ? v[j] : t;
         e.zy_val = t;
         e.found = true;
+      }
+      float cm = v[0];
+#pragma unroll
+      for (int j = 1; j < 32; ++j) cm = fmaxf(cm, v[j]);
+      const float nm = fmaxf(e.run_m, cm * kLog2e);
+      float acc = 0.f;
+#pragma unroll
+      for (int j = 0; j < 32; ++j) acc += fast_exp2(fmaf(v[j], kLog2e, -nm));
+      e.run_s = e.run_s * fast_exp2(e.run_m - nm) + acc;
+      e.run_m = nm;
+    } else if (kEpi == kEpiSample) {
+      // scaled logits (cols >= N: -inf) -> running LSE and running argmax of z + noise
+#pragma unroll
+      for (int j = 0; j < 32; ++j) v[j] = (cb + j < a.N) ? v[j] * a.inv_temp : -INFINITY;
+      if (e.rv) {
+#pragma unroll
+        for (int q = 0; q < 8; ++q) {
+          const uint4 w = philox4x32_10(
+              make_uint4(static_cast<uint32_t>((cb >> 2) + q), static_cast<uint32_t>(e.orow), a.off_lo, a.off_hi),
+              a.seed_lo, a.seed_hi);
+          const uint32_t ws[4] = {w.x, w.y, w.z, w.w};
+#pragma unroll
+          for (int k = 0; k < 4; ++k) {
+            const int j = 4 * q + k;
+            const float sc = v[j] + gumbel_of(ws[k]);
+            if (sc > e.best_s) {  // strict: the lowest column wins a tie
+              e.best_s = sc;
+              e.best_c = cb + j;
+              e.best_z = v[j];
+            }
+          }
+        }
       }
       float cm = v[0];
 #pragma unroll
@@ -312,6 +362,14 @@ __device__ __forceinline__ void epi_tile(EpiRow& e, const GemmArgs& a, uint32_t 
 
 template <int kEpi>
 __device__ __forceinline__ void epi_end(const EpiRow& e, const GemmArgs& a, int un, int head) {
+  if (kEpi == kEpiSample && e.rv) {
+    const long at = static_cast<long>(un) * a.ldp + e.r;
+    a.part_m[at] = e.run_m;
+    a.part_s[at] = e.run_s;
+    a.best_s[at] = e.best_s;
+    a.best_c[at] = e.best_c;
+    a.best_z[at] = e.best_z;
+  }
   if (kEpi == kEpiLse && e.rv) {
     a.part_m[static_cast<long>(un) * a.ldp + e.r] = e.run_m;
     a.part_s[static_cast<long>(un) * a.ldp + e.r] = e.run_s;

@@ -42,13 +42,14 @@ int64_t vocab_chunk(int64_t V) {
 struct Layout {
   int64_t T_pad, nsplit, nblk_scan, nblk_loss, vchunk;
   size_t status, n_valid, counts, offsets, cidx, rank_of, yc, zy, part_m, part_s, lse_c, g_c,
-      block_loss, resp_len, Hc, dz, total;
+      block_loss, resp_len, best_s, best_c, best_z, Hc, dz, total;
 };
 
 bool make_layout(int64_t T, int32_t Hd, int64_t V, int32_t which, Layout* L) {
   if (T < 0 || T >= (int64_t(1) << 31) || Hd <= 0 || Hd % 64 != 0 || V <= 0 ||
       V >= (int64_t(1) << 31) ||
-      (which != GRPO_WS_LOGPROBS && which != GRPO_WS_LOSS && which != GRPO_WS_LOGPROBS_HEADS))
+      (which != GRPO_WS_LOGPROBS && which != GRPO_WS_LOSS && which != GRPO_WS_LOGPROBS_HEADS &&
+       which != GRPO_WS_SAMPLE))
     return false;
   const size_t heads = which == GRPO_WS_LOGPROBS_HEADS ? kMaxHeads : 1;
   L->T_pad = round_up(std::max<int64_t>(T, 1), kRowAlign);
@@ -79,6 +80,10 @@ bool make_layout(int64_t T, int32_t Hd, int64_t V, int32_t which, Layout* L) {
   L->g_c = take(4 * tp, 256);
   L->block_loss = take(8 * L->nblk_loss, 256);
   L->resp_len = take(4 * tp, 256);
+  const size_t best = which == GRPO_WS_SAMPLE ? 4 * tp * L->nsplit : 0;
+  L->best_s = take(best, 256);
+  L->best_c = take(best, 256);
+  L->best_z = take(best, 256);
   L->Hc = take(2 * tp * static_cast<size_t>(Hd), 1024);
   L->dz = which == GRPO_WS_LOSS ? take(2 * tp * static_cast<size_t>(L->vchunk), 1024) : off;
   L->total = (off + 1023) / 1024 * 1024;
@@ -160,7 +165,7 @@ bool device_info(DeviceInfo* out) {
     if (major != 10 || minor != 3) return false;
     if (!prepare_kernels<kEpiLse, false, false>(&pairs) || !prepare_kernels<kEpiDz, false, false>(&pairs) ||
         !prepare_kernels<kEpiF32, false, true>(&pairs) || !prepare_kernels<kEpiF32, true, true>(&pairs) ||
-        !prepare_kernels<kEpiAdam, true, true>(&pairs))
+        !prepare_kernels<kEpiAdam, true, true>(&pairs) || !prepare_kernels<kEpiSample, false, false>(&pairs))
       return false;
     cache[dev].sms = sms;
     cache[dev].pairs = std::max(pairs, 0);
@@ -510,6 +515,64 @@ grpo_status grpo_token_logprobs_heads(const uint16_t* H, const uint16_t* const* 
                                                at<unsigned>(ws, Ly.status));
       e = cudaGetLastError();
     }
+  }
+  return from_cuda(e);
+}
+
+grpo_status grpo_sample_tokens(const uint16_t* H, const uint16_t* W, const uint8_t* mask, int64_t T, int32_t Hd,
+                               int64_t V, float temperature, uint64_t seed, uint64_t offset, int32_t* tokens_out,
+                               float* logp_out, void* ws, size_t ws_bytes, void* stream) {
+  Layout Ly;
+  if (!make_layout(T, Hd, V, GRPO_WS_SAMPLE, &Ly)) return GRPO_ERR_INVALID_ARG;
+  if (!W || !aligned(W, 16)) return GRPO_ERR_INVALID_ARG;
+  if (T > 0 && (!H || !mask || !tokens_out || !logp_out)) return GRPO_ERR_INVALID_ARG;
+  if (H && !aligned(H, 16)) return GRPO_ERR_INVALID_ARG;
+  if (!(temperature > 0.f) || !(temperature < INFINITY)) return GRPO_ERR_INVALID_ARG;
+  if (!ws || !aligned(ws, 256) || ws_bytes < Ly.total) return GRPO_ERR_WORKSPACE;
+  if (T == 0) return GRPO_OK;
+  DeviceInfo di;
+  if (!device_info(&di)) return GRPO_ERR_UNSUPPORTED;
+  if (!get_encode()) return GRPO_ERR_CUDA;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  cudaError_t e = run_compaction(H, nullptr, mask, T, Hd, V, ws, Ly, di.sms, s);
+  if (e == cudaSuccess) {
+    GemmArgs a{};
+    a.n_valid = at<int>(ws, Ly.n_valid);
+    a.m_dyn = 1;
+    a.N = static_cast<int>(V);
+    a.K = Hd;
+    a.n_per_unit = kLseTilesPerUnit;
+    a.n_heads = 1;
+    a.group_m = group_m(0, di);
+    l2_hints(0, &a.a_hint, &a.b_hint);
+    a.status = at<unsigned>(ws, Ly.status);
+    a.row_map = at<int>(ws, Ly.cidx);
+    a.part_m = at<float>(ws, Ly.part_m);
+    a.part_s = at<float>(ws, Ly.part_s);
+    a.best_s = at<float>(ws, Ly.best_s);
+    a.best_c = at<int>(ws, Ly.best_c);
+    a.best_z = at<float>(ws, Ly.best_z);
+    a.ldp = Ly.T_pad;
+    a.inv_temp = 1.f / temperature;
+    a.seed_lo = static_cast<uint32_t>(seed);
+    a.seed_hi = static_cast<uint32_t>(seed >> 32);
+    a.off_lo = static_cast<uint32_t>(offset);
+    a.off_hi = static_cast<uint32_t>(offset >> 32);
+    const Operand A{at<uint16_t>(ws, Ly.Hc), static_cast<uint64_t>(Ly.T_pad), static_cast<uint64_t>(Hd),
+                    static_cast<uint64_t>(Hd)};
+    const Operand B{W, static_cast<uint64_t>(V), static_cast<uint64_t>(Hd), static_cast<uint64_t>(Hd)};
+    TraceScope trace(GRPO_K_SAMPLE_GEMM, V, s);
+    e = launch_gemm<kEpiSample, false, false>(A, B, a, Ly.T_pad, di, s);
+  }
+  if (e == cudaSuccess) {
+    const int blocks = static_cast<int>(std::min<int64_t>((T + 255) / 256, di.sms * 16));
+    TraceScope trace(GRPO_K_LOGP_MERGE, 0, s);
+    sample_merge_kernel<<<blocks, 256, 0, s>>>(mask, at<int>(ws, Ly.rank_of), T, at<float>(ws, Ly.part_m),
+                                               at<float>(ws, Ly.part_s), at<float>(ws, Ly.best_s),
+                                               at<int>(ws, Ly.best_c), at<float>(ws, Ly.best_z),
+                                               static_cast<int>(Ly.nsplit), Ly.T_pad, tokens_out, logp_out,
+                                               at<unsigned>(ws, Ly.status));
+    e = cudaGetLastError();
   }
   return from_cuda(e);
 }

@@ -303,6 +303,31 @@ __device__ __forceinline__ float fast_exp2(float x) {
   return y;
 }
 
+// Philox4x32-10 (Salmon et al., SC 2011): ten rounds of two 32 x 32 -> 64-bit
+// multiplies on a 4-word counter, the 2-word key advanced by the Weyl
+// constants between rounds.
+__device__ __forceinline__ uint4 philox4x32_10(uint4 c, uint32_t k0, uint32_t k1) {
+#pragma unroll
+  for (int r = 0; r < 10; ++r) {
+    if (r) {
+      k0 += 0x9E3779B9u;
+      k1 += 0xBB67AE85u;
+    }
+    const uint32_t lo0 = 0xD2511F53u * c.x, hi0 = __umulhi(0xD2511F53u, c.x);
+    const uint32_t lo1 = 0xCD9E8D57u * c.z, hi1 = __umulhi(0xCD9E8D57u, c.z);
+    c = make_uint4(hi1 ^ c.y ^ k0, lo1, hi0 ^ c.w ^ k1, lo0);
+  }
+  return c;
+}
+
+// Gumbel noise -log(-log U) of the uniform U = ((w >> 9) + 1/2) / 2^23 in (0, 1).
+// The inner logarithm uses the accurate logf: near U = 1 it is a tiny
+// negative number whose relative accuracy decides the outer one.
+__device__ __forceinline__ float gumbel_of(uint32_t w) {
+  const float u = (static_cast<float>(w >> 9) + 0.5f) * (1.f / 8388608.f);
+  return -__logf(-logf(u));
+}
+
 __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
   uint32_t r;
   asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(hi), "f"(lo));

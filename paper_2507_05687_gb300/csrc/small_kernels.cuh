@@ -164,10 +164,14 @@ __global__ void gather_rows_kernel(const uint16_t* __restrict__ H, const int32_t
       const uint4* src = reinterpret_cast<const uint4*>(H + static_cast<int64_t>(t) * Hd);
       for (int j = lane; j < vec; j += 32) dst[j] = __ldg(src + j);
       if (lane == 0) {
-        const int y = targets[t];
-        const bool ok = y >= 0 && static_cast<int64_t>(y) < V;
-        yc[r] = ok ? y : -1;
-        if (!ok) atomicOr(status, kDevBadTarget);
+        if (targets) {
+          const int y = targets[t];
+          const bool ok = y >= 0 && static_cast<int64_t>(y) < V;
+          yc[r] = ok ? y : -1;
+          if (!ok) atomicOr(status, kDevBadTarget);
+        } else {
+          yc[r] = -1;  // no targets (sampling)
+        }
       }
     } else {
       for (int j = lane; j < vec; j += 32) dst[j] = make_uint4(0, 0, 0, 0);
@@ -217,6 +221,38 @@ __global__ void logp_merge_kernel(const uint8_t* __restrict__ mask, const int* _
       out = yc[r] >= 0 ? zy[r] - lse : 0.f;
     }
     logp_out[t] = out;
+  }
+}
+
+// The sampled token of every row: the split with the best perturbed score
+// (the lowest split on a tie, i.e. the lowest column), and its log-prob under
+// softmax(z / temperature).  Masked rows: token -1, log-prob 0.
+__global__ void sample_merge_kernel(const uint8_t* __restrict__ mask, const int* __restrict__ rank_of, int64_t T,
+                                    const float* __restrict__ pm, const float* __restrict__ ps,
+                                    const float* __restrict__ bs, const int* __restrict__ bc,
+                                    const float* __restrict__ bz, int nsplit, long ldp,
+                                    int32_t* __restrict__ tokens, float* __restrict__ logp, unsigned* status) {
+  for (int64_t t = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; t < T;
+       t += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+    int tok = -1;
+    float lp = 0.f;
+    if (mask[t]) {
+      const int r = rank_of[t];
+      float best = -INFINITY, z = 0.f;
+      for (int j = 0; j < nsplit; ++j) {
+        const float sc = bs[j * ldp + r];
+        if (sc > best) {
+          best = sc;
+          tok = bc[j * ldp + r];
+          z = bz[j * ldp + r];
+        }
+      }
+      const float lse = merge_lse(pm, ps, nsplit, ldp, r);
+      if (!isfinite(lse) || tok < 0) atomicOr(status, kDevNonFinite);
+      lp = z - lse;
+    }
+    tokens[t] = tok;
+    logp[t] = lp;
   }
 }
 

@@ -101,6 +101,16 @@ def test_host_rejections(lib):
     assert L.grpo_token_logprobs_heads(*bad) == grpo.GRPO_ERR_INVALID_ARG
     bad = list(hargs); bad[10] = ws3 - 1
     assert L.grpo_token_logprobs_heads(*bad) == grpo.GRPO_ERR_WORKSPACE
+    wss = grpo.workspace_bytes(100, 64, 1000, grpo.GRPO_WS_SAMPLE)
+    assert wss > grpo.workspace_bytes(100, 64, 1000, grpo.GRPO_WS_LOGPROBS)
+    sargs = [FAKE, FAKE, FAKE, 100, 64, 1000, 1.0, 1, 2, FAKE, FAKE, FAKE, wss, None]
+    for tau in (0.0, -2.0, float("inf"), float("nan")):
+        bad = list(sargs); bad[6] = tau
+        assert L.grpo_sample_tokens(*bad) == grpo.GRPO_ERR_INVALID_ARG
+    bad = list(sargs); bad[12] = wss - 1
+    assert L.grpo_sample_tokens(*bad) == grpo.GRPO_ERR_WORKSPACE
+    bad = list(sargs); bad[2] = None
+    assert L.grpo_sample_tokens(*bad) == grpo.GRPO_ERR_INVALID_ARG
 
 
 def test_binding_fails_loudly_without_library(tmp_path):

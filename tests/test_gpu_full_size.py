@@ -158,3 +158,21 @@ def test_fwd_bwd_full_size(name):
     colsum = dW.double().sum(0)
     colabs = dW.double().abs().sum(0)
     assert (colsum.norm() / colabs.norm()).item() <= 1e-2
+
+
+def test_sampling_full_size():
+    """The rollout draw over the 32768-row batch at 4096 x 155136, checked on sampled rows."""
+    w = wl.WORKLOADS["logprob3_8b"]
+    Hb, Wb, m = wl.gen_hidden(w), wl.gen_weight(w), wl.gen_mask(w)
+    tok, lp = grpo.sample_tokens(dev_tensor(Hb, torch.bfloat16), dev_tensor(Wb, torch.bfloat16),
+                                 dev_tensor(m, torch.uint8), 1.0, seed=20250705, offset=687)
+    tok, lp = tok.cpu().numpy(), lp.cpu().numpy()
+    assert np.all(tok[m == 0] == -1)
+    idx = wl.valid_index(m)
+    assert tok[idx].min() >= 0 and tok[idx].max() < w.V
+    rows = idx[wl.sample_rows(idx.size, 96, w.seed + 5)]
+    want_tok, want_lp, gap = oracle.sample_tokens(Hb, Wb, m, 1.0, 20250705, 687, rows=rows)
+    clear = rows[gap[rows] > 1e-3]
+    assert clear.size >= 0.9 * rows.size
+    assert np.array_equal(tok[clear], want_tok[clear])
+    assert np.abs(lp[clear] - want_lp[clear]).max() <= LOGP_ATOL

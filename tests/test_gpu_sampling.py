@@ -1,0 +1,91 @@
+"""The rollout draw o_t ~ softmax(z_t / temperature) (grpo_sample_tokens)
+against the oracle's Gumbel-max sampler on the same Philox noise.
+
+The argmax is decided in the kernel's fp32 on tensor-core logits and in the
+oracle's fp64: the draws must agree wherever the oracle's best perturbed score
+beats the second by more than 1e-3; within that margin the GPU's token must be
+one of the near-best candidates.
+"""
+import numpy as np
+import pytest
+import scipy.special
+
+import oracle
+import workloads as wl
+from tests._util import LOGP_ATOL, dev_tensor
+
+torch = pytest.importorskip("torch")
+pytestmark = pytest.mark.gpu
+
+if not torch.cuda.is_available():  # pragma: no cover
+    pytest.skip("needs a CUDA GPU", allow_module_level=True)
+
+import paper_2507_05687_gb300 as grpo  # noqa: E402
+from paper_2507_05687_gb300 import build as build_mod  # noqa: E402
+
+build_mod.build()
+DEV = torch.device("cuda", 0)
+TIE = 1e-3
+
+
+def _compare(Hb, Wb, m, tau, seed, offset, tok, logp, rows=None):
+    want_tok, want_lp, gap = oracle.sample_tokens(Hb, Wb, m, tau, seed, offset, rows=rows)
+    idx = np.flatnonzero(m) if rows is None else np.asarray(rows)
+    clear = idx[gap[idx] > TIE]
+    assert clear.size >= 0.9 * idx.size
+    assert np.array_equal(tok[clear], want_tok[clear])
+    assert np.abs(logp[clear] - want_lp[clear]).max() <= LOGP_ATOL
+    for t in idx[gap[idx] <= TIE]:   # near-ties: the GPU's pick must be within the margin of the best
+        z = oracle.as_f64(Hb[t]) @ oracle.as_f64(Wb).T / tau
+        s = z + oracle.gumbel_noise(seed, offset, [t], Wb.shape[0])[0]
+        assert s.max() - s[tok[t]] <= 2 * TIE
+    return idx
+
+
+@pytest.mark.parametrize("tau", [1.0, 0.7, 1.6])
+def test_sampling_matches_oracle(tau):
+    w = wl.Workload("s", 2, 3, 90, 192, 5000, "uniform", 1, 90, seed=wl.SEED_BASE + 2100, w_std=0.08)
+    Hb, Wb, m = wl.gen_hidden(w), wl.gen_weight(w), wl.gen_mask(w)
+    tok, lp = grpo.sample_tokens(dev_tensor(Hb, torch.bfloat16), dev_tensor(Wb, torch.bfloat16),
+                                 dev_tensor(m, torch.uint8), tau, seed=2507, offset=11)
+    tok, lp = tok.cpu().numpy(), lp.cpu().numpy()
+    assert np.all(tok[m == 0] == -1) and np.all(lp[m == 0] == 0.0)
+    _compare(Hb, Wb, m, tau, 2507, 11, tok, lp)
+
+
+def test_sampling_is_reproducible_and_keyed():
+    w = wl.Workload("s", 1, 4, 64, 128, 3000, seed=wl.SEED_BASE + 2200, w_std=0.05)
+    H, W = dev_tensor(wl.gen_hidden(w), torch.bfloat16), dev_tensor(wl.gen_weight(w), torch.bfloat16)
+    m = torch.ones(w.T, dtype=torch.uint8, device=DEV)
+    a = grpo.sample_tokens(H, W, m, 1.0, seed=1, offset=0)[0]
+    b = grpo.sample_tokens(H, W, m, 1.0, seed=1, offset=0)[0]
+    c = grpo.sample_tokens(H, W, m, 1.0, seed=1, offset=1)[0]
+    d = grpo.sample_tokens(H, W, m, 1.0, seed=2, offset=0)[0]
+    assert torch.equal(a, b)
+    assert (a != c).float().mean() > 0.5 and (a != d).float().mean() > 0.5
+
+
+def test_sampled_frequencies_follow_the_softmax():
+    """20000 rows with the same logits over 7 tokens: frequencies ~ softmax(z / tau)."""
+    from scipy.stats import chisquare
+    Hd, V, T = 64, 7, 20000
+    rng = np.random.default_rng(3)
+    Wf = rng.normal(0, 0.15, (V, Hd)).astype(np.float32)
+    hf = rng.normal(0, 1, Hd).astype(np.float32)
+    Wb, hb = wl.f32_to_bf16_bits(Wf), wl.f32_to_bf16_bits(hf)
+    z = oracle.as_f64(Wb) @ oracle.as_f64(hb)
+    H = dev_tensor(np.tile(hb, (T, 1)), torch.bfloat16)
+    m = torch.ones(T, dtype=torch.uint8, device=DEV)
+    for tau in (1.0, 0.5):
+        tok = grpo.sample_tokens(H, dev_tensor(Wb, torch.bfloat16), m, tau, seed=77, offset=3)[0].cpu().numpy()
+        p = scipy.special.softmax(z / tau)
+        assert chisquare(np.bincount(tok, minlength=V), p * T).pvalue > 1e-4
+
+
+def test_sampling_rejects_bad_temperature():
+    H = torch.zeros(4, 64, dtype=torch.bfloat16, device=DEV)
+    W = torch.zeros(10, 64, dtype=torch.bfloat16, device=DEV)
+    m = torch.ones(4, dtype=torch.uint8, device=DEV)
+    for tau in (0.0, -1.0, float("inf")):
+        with pytest.raises(grpo.GrpoError):
+            grpo.sample_tokens(H, W, m, tau)

@@ -311,6 +311,51 @@ def test_adamw_matches_torch_optimizer():
 
 
 # ---------------------------------------------------------------------------
+# sampling: Philox4x32-10 and the Gumbel-max draw
+# ---------------------------------------------------------------------------
+
+def test_philox_known_answer_vectors():
+    """The known-answer vectors published with the generator's reference implementation."""
+    from oracle import philox
+    cases = [((0, 0, 0, 0), (0, 0), (0x6627E8D5, 0xE169C58D, 0xBC57AC4C, 0x9B00DBD8)),
+             ((0xFFFFFFFF,) * 4, (0xFFFFFFFF,) * 2, (0x408F276D, 0x41C83B0E, 0xA20BC7C6, 0x6D5451FD)),
+             ((0x243F6A88, 0x85A308D3, 0x13198A2E, 0x03707344), (0xA4093822, 0x299F31D0),
+              (0xD16CFE09, 0x94FDCCEB, 0x5001E420, 0x24126EA1))]
+    for ctr, key, want in cases:
+        assert [int(x) for x in philox.philox4x32_10(*ctr, *key)] == list(want)
+    u = philox.uniform_open(np.array([0, 511, 512, 0xFFFFFFFF], dtype=np.uint64))
+    np.testing.assert_array_equal(u, [0.5 / 2 ** 23, 0.5 / 2 ** 23, 1.5 / 2 ** 23, 1 - 0.5 / 2 ** 23])
+
+
+def test_gumbel_max_samples_follow_the_softmax():
+    """Many rows with the same logits: the sampled tokens' frequencies follow softmax(z / tau)."""
+    from scipy.stats import chisquare
+    V, T, Hd = 6, 30000, 3
+    W = np.array([[1.0, 0, 0], [0.5, 0, 0], [0, 1, 0], [0, 0, 1], [-1.0, 0, 0], [0.2, 0.2, 0.2]])
+    H = np.tile(np.array([[0.9, -0.4, 0.3]]), (T, 1))
+    z = W @ H[0]
+    for tau in (1.0, 0.5, 2.0):
+        tok, logp, _ = oracle.sample_tokens(H, W, np.ones(T, np.uint8), tau, seed=1234, offset=7)
+        p = scipy.special.softmax(z / tau)
+        counts = np.bincount(tok, minlength=V)
+        assert chisquare(counts, p * T).pvalue > 1e-4
+        np.testing.assert_allclose(logp, np.log(p)[tok], rtol=0, atol=1e-12)
+    tok, _, _ = oracle.sample_tokens(H[:50], W, np.ones(50, np.uint8), 1e-3, seed=5, offset=0)
+    assert np.all(tok == np.argmax(z))  # tau -> 0: greedy
+
+
+def test_sampling_counter_layout():
+    """Rows, offsets and seeds index disjoint noise; word v mod 4 of counter v div 4."""
+    from oracle import philox
+    g = oracle.gumbel_noise(99, 5, [3, 4], 9)
+    w = philox.philox4x32_10(2, 3, 5, 0, 99, 0)
+    assert g[0, 9 - 1] == -np.log(-np.log(philox.uniform_open(w[0])))   # v = 8 -> counter 2, word 0
+    assert not np.array_equal(g[0], g[1])
+    assert not np.array_equal(g, oracle.gumbel_noise(99, 6, [3, 4], 9))
+    assert not np.array_equal(g, oracle.gumbel_noise(98, 5, [3, 4], 9))
+
+
+# ---------------------------------------------------------------------------
 # planted mistakes: each must trip one of the pins above
 # ---------------------------------------------------------------------------
 
@@ -366,3 +411,10 @@ def test_planted_adam_bias_correction_is_caught(monkeypatch):
     monkeypatch.setattr(oracle, "adamw_step", bad)
     with pytest.raises(AssertionError):
         test_adamw_first_step_closed_form()
+
+
+def test_planted_gumbel_sign_is_caught(monkeypatch):
+    real = go.gumbel_noise
+    monkeypatch.setattr(go, "gumbel_noise", lambda *a, **k: -real(*a, **k))
+    with pytest.raises(AssertionError):
+        test_gumbel_max_samples_follow_the_softmax()
