@@ -75,6 +75,9 @@ struct GemmArgs {
   int group_m;          // raster: M tiles per group sharing the same N sweep
   int a_hint, b_hint;   // L2 eviction policy of A / B loads (kHint*)
   unsigned* status;     // device status word
+  unsigned long long wait_ns;  // bound of every pipeline wait (0: kWaitLimitNs)
+  int drop_kblock1;     // fault-injection test hook: CTA 0 skips the copies of its
+                        // k-block number drop_kblock1 - 1 (0: never), so a wait runs out
 
   // kEpiLse
   const int* yc;        // [M] target of each compacted row (-1: none)
@@ -435,6 +438,7 @@ __device__ __forceinline__ void gemm_body(const CUtensorMap* tmA, const CUtensor
 
   const TileSched sch = make_sched(args, C::kTileM);
   const int KB = sch.k_blocks;
+  const unsigned long long wlim = args.wait_ns ? args.wait_ns : kWaitLimitNs;
 
   // Raises the abort flag of this CTA and of its peer.
   auto raise_abort = [&]() {
@@ -454,6 +458,7 @@ __device__ __forceinline__ void gemm_body(const CUtensorMap* tmA, const CUtensor
 #pragma unroll
       for (int s = 0; s < C::kStages; ++s) uses[s] = 0;
       bool ok = true;
+      int kblock_count = 0;  // k-blocks this CTA has staged (fault-injection hook)
       for (int u = unit0; u < sch.total && ok; u += unit_stride) {
         int mt, un;
         unit_coords(args, sch, u, mt, un);
@@ -462,7 +467,7 @@ __device__ __forceinline__ void gemm_body(const CUtensorMap* tmA, const CUtensor
         const int nt1 = min(sch.n_tiles, nt0 + args.n_per_unit);
         for (int nt = nt0; nt < nt1 && ok; ++nt) {
           for (int kb = 0; kb < KB; ++kb) {
-            if (!mbar_wait(smem_addr(&empty_bar[stage]), phase ^ 1u, abort_flag)) {
+            if (!mbar_wait(smem_addr(&empty_bar[stage]), phase ^ 1u, abort_flag, wlim)) {
               ok = false;
               break;
             }
@@ -474,7 +479,9 @@ __device__ __forceinline__ void gemm_body(const CUtensorMap* tmA, const CUtensor
             const int k0 = kb * kBK;
             const int m0 = mt * C::kTileM + static_cast<int>(rank) * kRowsCta;
             const int n0 = nt * kTileN + static_cast<int>(rank) * C::kBRows;
+            const bool drop = blockIdx.x == 0 && ++kblock_count == args.drop_kblock1;
             auto load = [&](uint32_t dst, const CUtensorMap* map, int c0, int c1, uint64_t pol) {
+              if (drop) return;  // the test hook: these bytes never arrive
               if (kPair == 2) tma_load_2d_pair_hint(dst, map, fb, c0, c1, pol);
               else tma_load_2d_hint(dst, map, fb, c0, c1, pol);
             };
@@ -505,7 +512,7 @@ __device__ __forceinline__ void gemm_body(const CUtensorMap* tmA, const CUtensor
       // have landed) before the CTA can exit.
       for (int s = 0; s < C::kStages; ++s)
         if (uses[s] > 0)
-          mbar_wait(smem_addr(&empty_bar[s]), static_cast<uint32_t>(uses[s] - 1) & 1u, abort_flag);
+          mbar_wait(smem_addr(&empty_bar[s]), static_cast<uint32_t>(uses[s] - 1) & 1u, abort_flag, wlim);
     }
   } else if (warp == 1) {
     // ------------------------------------------------------------ MMA issuer
@@ -525,14 +532,14 @@ __device__ __forceinline__ void gemm_body(const CUtensorMap* tmA, const CUtensor
           if (KB == 0) continue;
           const int buf = tile & 1;
           const uint32_t use = static_cast<uint32_t>(tile >> 1);
-          if (!mbar_wait(smem_addr(&tempty_bar[buf]), (use & 1u) ^ 1u, abort_flag)) {
+          if (!mbar_wait(smem_addr(&tempty_bar[buf]), (use & 1u) ^ 1u, abort_flag, wlim)) {
             ok = false;
             break;
           }
           tc_fence_after();
           const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(buf * kTileN);
           for (int kb = 0; kb < KB; ++kb) {
-            if (!mbar_wait(smem_addr(&full_bar[stage]), phase, abort_flag)) {
+            if (!mbar_wait(smem_addr(&full_bar[stage]), phase, abort_flag, wlim)) {
               ok = false;
               break;
             }
@@ -563,10 +570,12 @@ __device__ __forceinline__ void gemm_body(const CUtensorMap* tmA, const CUtensor
         }
       }
       if (!ok) raise_abort();
-      // Retire every MMA before TMEM is released.
+      // Retire every MMA before TMEM is released (not cut short by the abort flag:
+      // issued MMAs always finish).
       if (kPair == 2) tc_commit_pair_mc(smem_addr(done_bar), 0x1);
       else tc_commit(smem_addr(done_bar));
-      mbar_wait(smem_addr(done_bar), 0, abort_flag);
+      volatile int never = 0;
+      mbar_wait(smem_addr(done_bar), 0, &never, wlim);
     }
   } else {
     // ------------------------------------------------------------ epilogue
@@ -592,7 +601,10 @@ __device__ __forceinline__ void gemm_body(const CUtensorMap* tmA, const CUtensor
         const uint32_t use = static_cast<uint32_t>(tile >> 1);
         const bool have_acc = KB > 0;
         if (have_acc) {
-          if (!mbar_wait(smem_addr(&tfull_bar[buf]), use & 1u, abort_flag)) {
+          // all lanes must agree before the warp-wide tcgen05.ld: a lane that gave up
+          // (abort) while another saw the phase complete makes the whole warp give up
+          const bool got = mbar_wait(smem_addr(&tfull_bar[buf]), use & 1u, abort_flag, wlim);
+          if (!__all_sync(0xffffffffu, got)) {
             ok = false;
             break;
           }

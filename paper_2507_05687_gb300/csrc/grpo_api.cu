@@ -382,6 +382,13 @@ cudaError_t run_lse(const uint16_t* const* W, int n_heads, int32_t Hd, int64_t V
   a.n_per_unit = kLseTilesPerUnit;
   a.n_heads = n_heads;
   a.group_m = group_m(0, di);
+  // Fault-injection test hook (failure-detection tests): GRPO_TEST_DROP_KBLOCK=k
+  // makes CTA 0 skip the copies of its k-th k-block (1-based) so its pipeline
+  // wait runs out after 0.2 s and the call reports GRPO_ERR_TIMEOUT.
+  if (const char* d = std::getenv("GRPO_TEST_DROP_KBLOCK")) {
+    a.drop_kblock1 = std::atoi(d);
+    if (a.drop_kblock1 > 0) a.wait_ns = 200000000ull;
+  }
   // gathered hidden states: re-read for every vocabulary tile (evict last);
   // W: streamed, shared by the CTAs of one round (evict first)
   l2_hints(0, &a.a_hint, &a.b_hint);

@@ -230,3 +230,36 @@ def test_invalid_group_size_rejected():
     with pytest.raises(grpo.GrpoError) as e:
         grpo.group_advantages(torch.zeros(8, device=DEV), 1)
     assert e.value.status == grpo.GRPO_ERR_INVALID_ARG
+
+
+# ---------------------------------------------------------------- tile and split boundaries
+
+@pytest.mark.parametrize("n_valid,V", [(1, 100), (255, 256), (256, 4096), (257, 4097), (512, 8191),
+                                       (511, 65), (1000, 12288)])
+def test_logprobs_at_tile_and_split_boundaries(n_valid, V):
+    """Valid-row counts around the 256-row tile, vocabularies around the 256-column tile
+    and the 4096-column split, down to a single token and a single partial tile."""
+    Hd = 64
+    w = wl.Workload("b", 1, 2, (n_valid + 1) // 2 + 3, Hd, V, seed=wl.SEED_BASE + 4000 + n_valid + V)
+    Hb, Wb, y = wl.gen_hidden(w), wl.gen_weight(w.with_(w_std=0.3)), wl.gen_targets(w)
+    m = np.zeros(w.T, np.uint8)
+    m[np.random.default_rng(n_valid).choice(w.T, n_valid, replace=False)] = 1
+    want, _ = oracle.token_logprobs(Hb, Wb, y, m)
+    got = grpo.token_logprobs(dev_tensor(Hb, torch.bfloat16), dev_tensor(Wb, torch.bfloat16),
+                              dev_tensor(y, torch.int32), dev_tensor(m, torch.uint8)).cpu().numpy()
+    assert np.all(got[m == 0] == 0.0)
+    assert np.abs(got - want).max() <= LOGP_ATOL
+
+
+@pytest.mark.parametrize("n_valid,V,Hd", [(1, 100, 64), (257, 300, 128), (300, 4097, 64)])
+def test_fwd_bwd_at_boundaries(n_valid, V, Hd, monkeypatch):
+    monkeypatch.setenv("GRPO_VOCAB_CHUNK", "256")
+    G, L = 2, (n_valid + 1) // 2 + 2
+    w = wl.Workload("b", 1, G, L, Hd, V, rewards="mix", seed=wl.SEED_BASE + 4500 + n_valid)
+    c = _case(w)
+    m = np.zeros(w.T, np.uint8)
+    m[:n_valid] = 1                                   # response 0 full, response 1 partly (or empty)
+    c["m"] = m
+    c["want"] = oracle.loss_fwd_bwd(c["H"], c["W"], c["y"], m, c["old"], c["ref"], c["adv"], w.n_resp, w.L,
+                                    w.clip_eps, w.beta)
+    _check_fwd_bwd(c)
