@@ -6,14 +6,16 @@
 // Tile 128 x 256 per CTA (kPair = 1) or 256 x 256 per CTA pair (kPair = 2,
 // tcgen05 cta_group::2: each CTA stages its own 128 rows of A and half of B's
 // 256 columns, the even CTA issues the MMAs for both, and each CTA's TMEM
-// holds its 128 accumulator rows).  Roles per CTA (192 threads):
+// holds its 128 accumulator rows).  Roles per CTA (64 + 32 kEpiWarps threads):
 //   warp 0      TMA producer: 64-wide k-blocks (128-byte swizzle) into a ring
 //               of shared-memory stages.
 //   warp 1      owns 512 TMEM columns (two 256-column accumulators, so the
 //               epilogue of tile i overlaps the MMAs of tile i + 1); one lane
 //               of the issuing CTA issues the 128x256x16 / 256x256x16 MMAs.
-//   warps 2..5  epilogue: one thread per accumulator row (TMEM lane), reading
-//               32 columns per tcgen05.ld.
+//   warps 2..   epilogue (kEpiWarps of them): one thread per accumulator row
+//               (TMEM lane), 32 columns per tcgen05.ld; with 8 warps two share a
+//               lane quarter and split the columns, their per-row log-softmax /
+//               sampling state written as separate split entries.
 //
 // Epilogues:
 //   kEpiLse  forward of the log-softmax (pi_theta in Eq. 1): per row a running
@@ -46,7 +48,13 @@ namespace grpo {
 constexpr int kBK = 64;            // bf16 elements per 128-byte swizzle row
 constexpr int kTileN = 256;        // accumulator columns per TMEM buffer
 constexpr int kRowsCta = 128;      // accumulator rows per CTA (TMEM lanes)
-constexpr int kGemmThreads = 192;
+// Epilogue warps: 4 = one per TMEM lane quarter (each thread walks its row's
+// 256 columns); 8 = two per quarter, each taking half the columns.  Measured
+// on the 8B batch: 8 warps slowed the dW GEMM (15.7 -> 16.7 ms per step) and
+// did not speed up the sampling epilogue (its integer / MUFU pipes are busy).
+constexpr int kEpiWarps = 4;
+constexpr int kEpiHalves = kEpiWarps / 4;        // column halves of a tile, one per warp of a quarter
+constexpr int kGemmThreads = 64 + 32 * kEpiWarps;
 constexpr int kTmemCols = 512;
 constexpr int kRowAlign = 256;     // row padding of every token-indexed buffer
 constexpr int kMaxHeads = 4;       // LM heads one forward launch can sweep
@@ -81,8 +89,8 @@ struct GemmArgs {
 
   // kEpiLse
   const int* yc;        // [M] target of each compacted row (-1: none)
-  float* part_m;        // [units_n x ldp] running max (log2 units)
-  float* part_s;        // [units_n x ldp] running sum of 2^(z log2e - max)
+  float* part_m;        // [units_n x kEpiHalves x ldp] running max (log2 units)
+  float* part_s;        // [units_n x kEpiHalves x ldp] running sum of 2^(z log2e - max)
   float* zy;            // [n_heads x ldp] logit of the target
   long ldp;
 
@@ -112,9 +120,9 @@ struct GemmArgs {
   // kEpiSample (row_map gives the token position t of each compacted row)
   float inv_temp;       // 1 / temperature
   uint32_t seed_lo, seed_hi, off_lo, off_hi;
-  float* best_s;        // [units_n x ldp] best perturbed score of the split
-  int* best_c;          // [units_n x ldp] its vocabulary column
-  float* best_z;        // [units_n x ldp] its z / temperature
+  float* best_s;        // [units_n x kEpiHalves x ldp] best perturbed score of the split entry
+  int* best_c;          // [units_n x kEpiHalves x ldp] its vocabulary column
+  float* best_z;        // [units_n x kEpiHalves x ldp] its z / temperature
 };
 
 struct TileSched {
@@ -208,10 +216,11 @@ __device__ __forceinline__ void adam_update(float g, float& theta, float& m, flo
 // 32x32 blocks through shared memory for warp-contiguous scalar accesses).
 template <int kEpi>
 __device__ __forceinline__ void epi_tile(EpiRow& e, const GemmArgs& a, uint32_t tbase, int col0,
-                                         bool have_acc) {
+                                         bool have_acc, int half) {
   const float kLog2e = 1.4426950408889634f;
+  constexpr int kChunks = kTileN / 32 / kEpiHalves;
 #pragma unroll 1
-  for (int c = 0; c < kTileN / 32; ++c) {
+  for (int c = half * kChunks; c < (half + 1) * kChunks; ++c) {
     float v[32];
     if (have_acc) {
       tmem_ld32(tbase + c * 32, v);
@@ -238,11 +247,13 @@ __device__ __forceinline__ void epi_tile(EpiRow& e, const GemmArgs& a, uint32_t 
 #pragma unroll
       for (int j = 1; j < 32; ++j) cm = fmaxf(cm, v[j]);
       const float nm = fmaxf(e.run_m, cm * kLog2e);
-      float acc = 0.f;
+      if (nm != -INFINITY) {  // a half-tile past V is all -inf: nothing to add
+        float acc = 0.f;
 #pragma unroll
-      for (int j = 0; j < 32; ++j) acc += fast_exp2(fmaf(v[j], kLog2e, -nm));
-      e.run_s = e.run_s * fast_exp2(e.run_m - nm) + acc;
-      e.run_m = nm;
+        for (int j = 0; j < 32; ++j) acc += fast_exp2(fmaf(v[j], kLog2e, -nm));
+        e.run_s = e.run_s * fast_exp2(e.run_m - nm) + acc;
+        e.run_m = nm;
+      }
     } else if (kEpi == kEpiSample) {
       // scaled logits (cols >= N: -inf) -> running LSE and running argmax of z + noise
 #pragma unroll
@@ -270,11 +281,13 @@ __device__ __forceinline__ void epi_tile(EpiRow& e, const GemmArgs& a, uint32_t 
 #pragma unroll
       for (int j = 1; j < 32; ++j) cm = fmaxf(cm, v[j]);
       const float nm = fmaxf(e.run_m, cm * kLog2e);
-      float acc = 0.f;
+      if (nm != -INFINITY) {  // a half-tile past V is all -inf: nothing to add
+        float acc = 0.f;
 #pragma unroll
-      for (int j = 0; j < 32; ++j) acc += fast_exp2(fmaf(v[j], kLog2e, -nm));
-      e.run_s = e.run_s * fast_exp2(e.run_m - nm) + acc;
-      e.run_m = nm;
+        for (int j = 0; j < 32; ++j) acc += fast_exp2(fmaf(v[j], kLog2e, -nm));
+        e.run_s = e.run_s * fast_exp2(e.run_m - nm) + acc;
+        e.run_m = nm;
+      }
     } else if (kEpi == kEpiDz) {
       const int gc = a.b_off_n + cb;  // vocabulary id of column 0 of this group
       uint32_t packed[16];
@@ -364,9 +377,10 @@ __device__ __forceinline__ void epi_tile(EpiRow& e, const GemmArgs& a, uint32_t 
 }
 
 template <int kEpi>
-__device__ __forceinline__ void epi_end(const EpiRow& e, const GemmArgs& a, int un, int head) {
+__device__ __forceinline__ void epi_end(const EpiRow& e, const GemmArgs& a, int un, int head, int half) {
+  const long entry = static_cast<long>(un) * kEpiHalves + half;  // split entry of this column half
   if (kEpi == kEpiSample && e.rv) {
-    const long at = static_cast<long>(un) * a.ldp + e.r;
+    const long at = entry * a.ldp + e.r;
     a.part_m[at] = e.run_m;
     a.part_s[at] = e.run_s;
     a.best_s[at] = e.best_s;
@@ -374,8 +388,8 @@ __device__ __forceinline__ void epi_end(const EpiRow& e, const GemmArgs& a, int 
     a.best_z[at] = e.best_z;
   }
   if (kEpi == kEpiLse && e.rv) {
-    a.part_m[static_cast<long>(un) * a.ldp + e.r] = e.run_m;
-    a.part_s[static_cast<long>(un) * a.ldp + e.r] = e.run_s;
+    a.part_m[entry * a.ldp + e.r] = e.run_m;
+    a.part_s[entry * a.ldp + e.r] = e.run_s;
     if (e.found) a.zy[static_cast<long>(head) * a.ldp + e.r] = e.zy_val;
   }
 }
@@ -412,7 +426,7 @@ __device__ __forceinline__ void gemm_body(const CUtensorMap* tmA, const CUtensor
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(smem_addr(&tfull_bar[i]), 1);
-      mbar_init(smem_addr(&tempty_bar[i]), 4 * kPair);  // one arrival per epilogue warp
+      mbar_init(smem_addr(&tempty_bar[i]), kEpiWarps * kPair);  // one arrival per epilogue warp
     }
     mbar_init(smem_addr(done_bar), 1);
     *abort_flag = 0;
@@ -579,7 +593,8 @@ __device__ __forceinline__ void gemm_body(const CUtensorMap* tmA, const CUtensor
     }
   } else {
     // ------------------------------------------------------------ epilogue
-    const int quad = warp & 3;  // TMEM lanes quad*32 .. quad*32+31
+    const int quad = warp & 3;              // TMEM lanes quad*32 .. quad*32+31
+    const int half = (warp - 2) / 4;         // which 128 of the tile's 256 columns
     const int row = static_cast<int>(rank) * kRowsCta + quad * 32 + lane;  // row within the tile
     const uint32_t lane_addr = tmem_base + (static_cast<uint32_t>(quad * 32) << 16);
     const uint32_t tempty0 = smem_addr(&tempty_bar[0]);
@@ -610,7 +625,7 @@ __device__ __forceinline__ void gemm_body(const CUtensorMap* tmA, const CUtensor
           }
           tc_fence_after();
         }
-        epi_tile<kEpi>(e, args, lane_addr + static_cast<uint32_t>(buf * kTileN), nt * kTileN, have_acc);
+        epi_tile<kEpi>(e, args, lane_addr + static_cast<uint32_t>(buf * kTileN), nt * kTileN, have_acc, half);
         if (have_acc) {
           tc_fence_before();
           __syncwarp();
@@ -622,7 +637,7 @@ __device__ __forceinline__ void gemm_body(const CUtensorMap* tmA, const CUtensor
         }
       }
       if (!ok) break;
-      epi_end<kEpi>(e, args, un, head);
+      epi_end<kEpi>(e, args, un, head, half);
     }
     if (!ok) raise_abort();
   }

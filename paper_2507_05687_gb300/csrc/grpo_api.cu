@@ -54,7 +54,8 @@ bool make_layout(int64_t T, int32_t Hd, int64_t V, int32_t which, Layout* L) {
   const size_t heads = which == GRPO_WS_LOGPROBS_HEADS ? kMaxHeads : 1;
   L->T_pad = round_up(std::max<int64_t>(T, 1), kRowAlign);
   const int64_t vtiles = (V + kTileN - 1) / kTileN;
-  L->nsplit = (vtiles + kLseTilesPerUnit - 1) / kLseTilesPerUnit;
+  // partial (max, sum) entries per row: one per vocabulary split and column half
+  L->nsplit = (vtiles + kLseTilesPerUnit - 1) / kLseTilesPerUnit * kEpiHalves;
   L->nblk_scan = (std::max<int64_t>(T, 1) + kScanChunk - 1) / kScanChunk;
   L->nblk_loss = (L->T_pad + kLossThreads - 1) / kLossThreads;
   L->vchunk = which == GRPO_WS_LOSS ? vocab_chunk(V) : 0;
