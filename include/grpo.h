@@ -165,6 +165,23 @@ grpo_status grpo_loss_fwd_bwd_norm(const uint16_t* H, const uint16_t* W, const i
                                    void* stream);
 
 /*
+ * grpo_loss_fwd_bwd_norm for a caller that wants dW in host memory: each
+ * vocabulary chunk of dW is copied to dW_host as soon as it is computed, on
+ * an internal copy stream (created once per device), so the copy of the
+ * 2.5 GB gradient of an 8B head overlaps the rest of the backward instead of
+ * following it.  dW (device) is still written.  When `stream` reaches the end
+ * of the call's work, dW_host holds dW.
+ *   dW_host  [V x Hd] fp32 HOST memory, page-locked (cudaHostAlloc /
+ *            cudaHostRegister), 16-byte aligned; must stay valid until then
+ */
+grpo_status grpo_loss_fwd_bwd_to_host(const uint16_t* H, const uint16_t* W, const int32_t* targets,
+                                      const uint8_t* mask, const float* old_logp, const float* ref_logp,
+                                      const float* adv, int64_t n_resp, int64_t L, int32_t Hd, int64_t V,
+                                      float clip_eps, float beta, int32_t agg_mode, float norm, float* loss_out,
+                                      float* dH, float* dW, float* dW_host, void* ws, size_t ws_bytes,
+                                      void* stream);
+
+/*
  * grpo_loss_fwd_bwd_norm followed by the actor's optimiser step on the LM
  * head, with the step fused into the dW GEMM: each dW tile is consumed in
  * place by one AdamW step (Adam with decoupled weight decay) and dW itself is

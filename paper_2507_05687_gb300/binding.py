@@ -47,6 +47,8 @@ SIGNATURES = {
                                                  _P]),
     "grpo_loss_fwd_bwd_norm": (ctypes.c_int, [_P, _P, _P, _P, _P, _P, _P, _I64, _I64, _I32, _I64, _F, _F, _I32, _F,
                                               _P, _P, _P, _P, ctypes.c_size_t, _P]),
+    "grpo_loss_fwd_bwd_to_host": (ctypes.c_int, [_P, _P, _P, _P, _P, _P, _P, _I64, _I64, _I32, _I64, _F, _F, _I32,
+                                                 _F, _P, _P, _P, _P, _P, ctypes.c_size_t, _P]),
     "grpo_loss_fwd_bwd_adamw": (ctypes.c_int, [_P, _P, _P, _P, _P, _P, _P, _I64, _I64, _I32, _I64, _F, _F, _I32, _F,
                                                _F, _F, _F, _F, _F, _I64, _P, _P, _P, _P, _P, _P, _P,
                                                ctypes.c_size_t, _P]),
@@ -254,6 +256,13 @@ def loss_fwd_bwd(H: torch.Tensor, W: torch.Tensor, targets: torch.Tensor, mask: 
     common = (_ptr(H), _ptr(W), _ptr(targets), _ptr(mask), _ptr(old_logp), _ptr(ref_logp), _ptr(adv), int(n_resp),
               int(L), Hd, V, float(clip_eps), float(beta), int(agg_mode))
     tail = (_ptr(loss), _ptr(dH), _ptr(dW), _ptr(ws), ws.numel(), _stream(dev))
+    if host_out is not None and host_out[2].is_pinned():
+        # dW streams to the caller's pinned buffer chunk by chunk while the backward runs
+        _check(lib.grpo_loss_fwd_bwd_to_host(*common, float(norm), _ptr(loss), _ptr(dH), _ptr(dW),
+                                             _ptr(host_out[2]), _ptr(ws), ws.numel(), _stream(dev)),
+               "grpo_loss_fwd_bwd_to_host")
+        lh, dHh = _to_host(loss, dH, dst=host_out[:2])
+        return lh, dHh, host_out[2]
     if norm:
         _check(lib.grpo_loss_fwd_bwd_norm(*common, float(norm), *tail), "grpo_loss_fwd_bwd_norm")
     else:

@@ -287,6 +287,36 @@ class TraceScope {
   bool active_ = false;
 };
 
+// Copy-out stream of grpo_loss_fwd_bwd_to_host: one per device, created on
+// first use (a driver object, not device memory) and shared by calls, which
+// enqueue under `mu` so a ring event is never re-recorded before its wait.
+struct CopyOut {
+  std::mutex mu;
+  cudaStream_t stream = nullptr;
+  static constexpr int kRing = 4;
+  cudaEvent_t ready[kRing] = {};
+  cudaEvent_t done = nullptr;
+  bool ok = false;
+};
+
+CopyOut* copy_out_for_device() {
+  static std::mutex mu;
+  static CopyOut* per_dev[64] = {};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return nullptr;
+  std::lock_guard<std::mutex> lk(mu);
+  if (!per_dev[dev]) {
+    CopyOut* c = new CopyOut();
+    bool ok = cudaStreamCreateWithFlags(&c->stream, cudaStreamNonBlocking) == cudaSuccess &&
+              cudaEventCreateWithFlags(&c->done, cudaEventDisableTiming) == cudaSuccess;
+    for (int i = 0; ok && i < CopyOut::kRing; ++i)
+      ok = cudaEventCreateWithFlags(&c->ready[i], cudaEventDisableTiming) == cudaSuccess;
+    c->ok = ok;
+    per_dev[dev] = c;
+  }
+  return per_dev[dev]->ok ? per_dev[dev] : nullptr;
+}
+
 // A bf16 row-major matrix [rows x cols] with leading dimension ld (elements).
 struct Operand {
   const void* base;
@@ -423,7 +453,7 @@ grpo_status loss_impl(const uint16_t* H, const uint16_t* W, const int32_t* targe
                       const float* old_logp, const float* ref_logp, const float* adv, int64_t n_resp,
                       int64_t L, int32_t Hd, int64_t V, float clip_eps, float beta, int32_t agg_mode,
                       float norm, float* loss_out, float* dH, float* dW, const AdamParams* adam, void* ws,
-                      size_t ws_bytes, void* stream);
+                      size_t ws_bytes, void* stream, float* dW_host = nullptr);
 
 }  // namespace
 
@@ -604,6 +634,17 @@ grpo_status grpo_loss_fwd_bwd_norm(const uint16_t* H, const uint16_t* W, const i
                    norm, loss_out, dH, dW, nullptr, ws, ws_bytes, stream);
 }
 
+grpo_status grpo_loss_fwd_bwd_to_host(const uint16_t* H, const uint16_t* W, const int32_t* targets,
+                                      const uint8_t* mask, const float* old_logp, const float* ref_logp,
+                                      const float* adv, int64_t n_resp, int64_t L, int32_t Hd, int64_t V,
+                                      float clip_eps, float beta, int32_t agg_mode, float norm, float* loss_out,
+                                      float* dH, float* dW, float* dW_host, void* ws, size_t ws_bytes,
+                                      void* stream) {
+  if (!dW_host || !aligned(dW_host, 16)) return GRPO_ERR_INVALID_ARG;
+  return loss_impl(H, W, targets, mask, old_logp, ref_logp, adv, n_resp, L, Hd, V, clip_eps, beta, agg_mode,
+                   norm, loss_out, dH, dW, nullptr, ws, ws_bytes, stream, dW_host);
+}
+
 grpo_status grpo_loss_fwd_bwd_adamw(const uint16_t* H, const uint16_t* W, const int32_t* targets,
                                     const uint8_t* mask, const float* old_logp, const float* ref_logp,
                                     const float* adv, int64_t n_resp, int64_t L, int32_t Hd, int64_t V,
@@ -642,7 +683,7 @@ grpo_status loss_impl(const uint16_t* H, const uint16_t* W, const int32_t* targe
                       const float* old_logp, const float* ref_logp, const float* adv, int64_t n_resp,
                       int64_t L, int32_t Hd, int64_t V, float clip_eps, float beta, int32_t agg_mode,
                       float norm, float* loss_out, float* dH, float* dW, const AdamParams* adam, void* ws,
-                      size_t ws_bytes, void* stream) {
+                      size_t ws_bytes, void* stream, float* dW_host) {
   if (n_resp < 1 || L < 1 || n_resp > (int64_t(1) << 31) / L) return GRPO_ERR_INVALID_ARG;
   if (!(norm >= 0.f) || norm == INFINITY) return GRPO_ERR_INVALID_ARG;
   const int64_t T = n_resp * L;
@@ -689,7 +730,17 @@ grpo_status loss_impl(const uint16_t* H, const uint16_t* W, const int32_t* targe
   }
   if (e != cudaSuccess) return from_cuda(e);
 
-  // Backward, one vocabulary chunk at a time.
+  // Backward, one vocabulary chunk at a time.  With dW_host, each finished dW
+  // chunk is copied to the host on the copy-out stream while the next chunks
+  // compute; `s` waits for the last copy at the end.
+  CopyOut* co = nullptr;
+  std::unique_lock<std::mutex> co_lock;
+  if (dW_host && !adam) {
+    co = copy_out_for_device();
+    if (!co) return GRPO_ERR_CUDA;
+    co_lock = std::unique_lock<std::mutex>(co->mu);
+  }
+  int chunk = 0;
   uint16_t* Hc = at<uint16_t>(ws, Ly.Hc);
   uint16_t* dz = at<uint16_t>(ws, Ly.dz);
   const int64_t vc = Ly.vchunk;
@@ -770,6 +821,19 @@ grpo_status loss_impl(const uint16_t* H, const uint16_t* W, const int32_t* targe
         e = launch_gemm<kEpiF32, true, true>(opDz, opHc, w, width, di, s);
       }
     }
+    if (e == cudaSuccess && co) {
+      cudaEvent_t ready = co->ready[chunk % CopyOut::kRing];
+      e = cudaEventRecord(ready, s);
+      if (e == cudaSuccess) e = cudaStreamWaitEvent(co->stream, ready, 0);
+      if (e == cudaSuccess)
+        e = cudaMemcpyAsync(dW_host + c0 * Hd, dW + c0 * Hd, static_cast<size_t>(width) * Hd * sizeof(float),
+                            cudaMemcpyDeviceToHost, co->stream);
+    }
+    ++chunk;
+  }
+  if (co && e == cudaSuccess) {
+    e = cudaEventRecord(co->done, co->stream);
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(s, co->done, 0);
   }
   return from_cuda(e);
 }

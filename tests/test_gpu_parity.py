@@ -263,3 +263,17 @@ def test_fwd_bwd_at_boundaries(n_valid, V, Hd, monkeypatch):
     c["want"] = oracle.loss_fwd_bwd(c["H"], c["W"], c["y"], m, c["old"], c["ref"], c["adv"], w.n_resp, w.L,
                                     w.clip_eps, w.beta)
     _check_fwd_bwd(c)
+
+
+def test_host_output_buffers_stream_dw(monkeypatch):
+    """Pinned host outputs: dW arrives chunk by chunk through grpo_loss_fwd_bwd_to_host
+    and equals the device-output call bit for bit."""
+    monkeypatch.setenv("GRPO_VOCAB_CHUNK", "512")
+    c = _case(wl.Workload("t", 2, 4, 48, 128, 1800, "uniform", 1, 48, rewards="mix", seed=wl.SEED_BASE + 660))
+    w, d = c["w"], _dev(c)
+    dev_out = grpo.loss_fwd_bwd(d["H"], d["W"], d["y"], d["m"], d["old"], d["ref"], d["adv"], w.n_resp, w.L)
+    host = (torch.empty(1).pin_memory(), torch.empty(w.T, w.Hd).pin_memory(), torch.empty(w.V, w.Hd).pin_memory())
+    got = grpo.loss_fwd_bwd(d["H"], d["W"], d["y"], d["m"], d["old"], d["ref"], d["adv"], w.n_resp, w.L, out=host)
+    assert all(g is h for g, h in zip(got, host))
+    for g, x in zip(got, dev_out):
+        assert torch.equal(g, x.cpu())
