@@ -165,6 +165,24 @@ grpo_status grpo_loss_fwd_bwd_norm(const uint16_t* H, const uint16_t* W, const i
                                    void* stream);
 
 /*
+ * grpo_loss_fwd_bwd_norm with a cap on the per-token KL value (Eq. 1's
+ * D_KL term; the paper leaves the estimator open):
+ *   KL_t = min(k3_t, kl_clamp),  k3_t = exp(ref_logp_t - logp_t) - (ref_logp_t - logp_t) - 1
+ * A token whose k3 lies above the cap adds beta * kl_clamp to its loss term and
+ * nothing to the gradient through the KL; a tie counts as below the cap.  This
+ * bounds the penalty of the few tokens on which the reference and the policy
+ * disagree by many nats.  kl_clamp must be >= 0 (not NaN); +infinity is
+ * exactly grpo_loss_fwd_bwd_norm, and 0 removes the KL term (k3 >= 0).
+ * Every other argument as grpo_loss_fwd_bwd_norm.
+ */
+grpo_status grpo_loss_fwd_bwd_kl_clamp(const uint16_t* H, const uint16_t* W, const int32_t* targets,
+                                       const uint8_t* mask, const float* old_logp, const float* ref_logp,
+                                       const float* adv, int64_t n_resp, int64_t L, int32_t Hd, int64_t V,
+                                       float clip_eps, float beta, int32_t agg_mode, float norm, float kl_clamp,
+                                       float* loss_out, float* dH, float* dW, void* ws, size_t ws_bytes,
+                                       void* stream);
+
+/*
  * grpo_loss_fwd_bwd_norm for a caller that wants dW in host memory: each
  * vocabulary chunk of dW is copied to dW_host as soon as it is computed, on
  * an internal copy stream (created once per device), so the copy of the

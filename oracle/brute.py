@@ -35,8 +35,9 @@ def logprobs(H, W, targets, mask):
     return out
 
 
-def loss(logp, old, ref, adv, mask, n_resp, L, clip_eps, beta, agg_mode=0):
-    """Negated Eq. 1; agg_mode 0 = masked token-mean, 1 = per-response mean then mean."""
+def loss(logp, old, ref, adv, mask, n_resp, L, clip_eps, beta, agg_mode=0, kl_clamp=math.inf):
+    """Negated Eq. 1; agg_mode 0 = masked token-mean, 1 = per-response mean then mean.
+    kl_clamp caps each token's KL value (no cap by default)."""
     total_tok = sum(1 for t in range(n_resp * L) if mask[t])
     acc = 0.0
     for i in range(n_resp):
@@ -50,6 +51,8 @@ def loss(logp, old, ref, adv, mask, n_resp, L, clip_eps, beta, agg_mode=0):
             clipped = min(max(rho, 1.0 - clip_eps), 1.0 + clip_eps)
             s = min(rho * A, clipped * A)
             kl = math.exp(ref[t] - logp[t]) - (ref[t] - logp[t]) - 1.0
+            if kl > kl_clamp:
+                kl = kl_clamp
             ell = -(s - beta * kl)
             if agg_mode == 0:
                 acc += ell / total_tok

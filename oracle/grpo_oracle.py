@@ -18,6 +18,9 @@ What it computes, in the paper's notation (Section 3.3):
       KL = exp(ref - logp) - (ref - logp) - 1     (per-token k3 estimator of
            D_KL(pi_theta || pi_ref) from the GRPO paper the method cites)
       l = -(s - beta KL)                          (loss = -J)
+  Optionally the KL value is capped, KL = min(k3, kl_clamp) (the paper does
+  not fix the estimator; a cap bounds one token's penalty when the reference
+  and the policy disagree strongly).  A capped token has no KL gradient.
 * the aggregation of Eq. 1: agg_mode 1 is Eq. 1 as printed,
       (1/n_resp) sum_i (1/|o_i|) sum_t l_{i,t};
   agg_mode 0 (default) is the masked token-mean sum_t mask_t l_t / N_valid.
@@ -120,12 +123,17 @@ def token_advantages(adv, n_resp: int, L: int) -> np.ndarray:
     return np.repeat(a, L)
 
 
-def token_terms(logp, old_logp, ref_logp, adv_tok, clip_eps: float, beta: float):
+def token_terms(logp, old_logp, ref_logp, adv_tok, clip_eps: float, beta: float, kl_clamp: float = np.inf):
     """The braces of Eq. 1 for every row.
 
     Returns a dict with rho, the clipped-surrogate value s, the k3 KL, the
     per-token loss l = -s + beta KL and the 0/1 flag 'unclipped' (the min()
     picks rho A; ties count as unclipped).
+
+    kl_clamp caps the per-token KL value: KL = min(k3, kl_clamp), and a token
+    whose k3 lies above the cap contributes a constant (no KL gradient); a tie
+    counts as inside.  The default (infinity) is the plain k3 estimator.  The
+    flag 'kl_inside' marks the tokens whose KL is not capped.
     """
     lp = np.asarray(logp, dtype=np.float64)
     old = np.asarray(old_logp, dtype=np.float64)
@@ -137,8 +145,10 @@ def token_terms(logp, old_logp, ref_logp, adv_tok, clip_eps: float, beta: float)
     unclipped = s1 <= s2
     s = np.where(unclipped, s1, s2)
     d = ref - lp
-    kl = np.exp(d) - d - 1.0
-    return {"rho": rho, "s": s, "kl": kl, "ell": -s + beta * kl, "unclipped": unclipped}
+    k3 = np.exp(d) - d - 1.0
+    inside = ~(k3 > kl_clamp)
+    kl = np.where(inside, k3, kl_clamp)
+    return {"rho": rho, "s": s, "kl": kl, "ell": -s + beta * kl, "unclipped": unclipped, "kl_inside": inside}
 
 
 def token_weights(mask, n_resp: int, L: int, agg_mode: int = 0, norm: float = 0.0) -> np.ndarray:
@@ -162,26 +172,27 @@ def token_weights(mask, n_resp: int, L: int, agg_mode: int = 0, norm: float = 0.
     raise ValueError(agg_mode)
 
 
-def logp_coef(logp, old_logp, ref_logp, adv_tok, w, clip_eps: float, beta: float) -> np.ndarray:
-    """g_t = dloss/dlogp_t = w_t (-A rho 1[unclipped] + beta (1 - exp(ref - logp)))."""
-    tt = token_terms(logp, old_logp, ref_logp, adv_tok, clip_eps, beta)
+def logp_coef(logp, old_logp, ref_logp, adv_tok, w, clip_eps: float, beta: float,
+              kl_clamp: float = np.inf) -> np.ndarray:
+    """g_t = dloss/dlogp_t = w_t (-A rho 1[unclipped] + beta (1 - exp(ref - logp)) 1[kl inside])."""
+    tt = token_terms(logp, old_logp, ref_logp, adv_tok, clip_eps, beta, kl_clamp)
     lp = np.asarray(logp, dtype=np.float64)
     ref = np.asarray(ref_logp, dtype=np.float64)
     A = np.asarray(adv_tok, dtype=np.float64)
     dsurr = np.where(tt["unclipped"], A * tt["rho"], 0.0)
-    dkl = 1.0 - np.exp(ref - lp)
+    dkl = np.where(tt["kl_inside"], 1.0 - np.exp(ref - lp), 0.0)
     return np.asarray(w, dtype=np.float64) * (-dsurr + beta * dkl)
 
 
 def grpo_loss(logp, old_logp, ref_logp, adv, mask, n_resp: int, L: int,
-              clip_eps: float, beta: float, agg_mode: int = 0, norm: float = 0.0):
+              clip_eps: float, beta: float, agg_mode: int = 0, norm: float = 0.0, kl_clamp: float = np.inf):
     """Eq. 1 negated, from per-token log-probs. Returns (loss, g, per-token dict)."""
     A = token_advantages(adv, n_resp, L)
     w = token_weights(mask, n_resp, L, agg_mode, norm)
-    tt = token_terms(logp, old_logp, ref_logp, A, clip_eps, beta)
+    tt = token_terms(logp, old_logp, ref_logp, A, clip_eps, beta, kl_clamp)
     m = np.asarray(mask) != 0
     loss = float(np.sum(w[m] * tt["ell"][m]))
-    g = logp_coef(logp, old_logp, ref_logp, A, w, clip_eps, beta)
+    g = logp_coef(logp, old_logp, ref_logp, A, w, clip_eps, beta, kl_clamp)
     g[~m] = 0.0
     tt["w"] = w
     return loss, g, tt
@@ -194,14 +205,15 @@ def grpo_loss(logp, old_logp, ref_logp, adv, mask, n_resp: int, L: int,
 
 def loss_fwd_bwd(H, W, targets, mask, old_logp, ref_logp, adv, n_resp: int, L: int,
                  clip_eps: float, beta: float, agg_mode: int = 0, vocab_chunk: int = 8192,
-                 norm: float = 0.0):
+                 norm: float = 0.0, kl_clamp: float = np.inf):
     """Full forward + backward: returns dict(loss, dH [T,Hd], dW [V,Hd], logp, lse, g)."""
     Hf = as_f64(H)
     Wf = as_f64(W)
     y = np.asarray(targets, dtype=np.int64)
     m = np.asarray(mask) != 0
     logp, lse = token_logprobs(Hf, Wf, y, m, vocab_chunk=vocab_chunk)
-    loss, g, tt = grpo_loss(logp, old_logp, ref_logp, adv, m, n_resp, L, clip_eps, beta, agg_mode, norm)
+    loss, g, tt = grpo_loss(logp, old_logp, ref_logp, adv, m, n_resp, L, clip_eps, beta, agg_mode, norm,
+                            kl_clamp)
     T, Hd = Hf.shape
     V = Wf.shape[0]
     dH = np.zeros((T, Hd))

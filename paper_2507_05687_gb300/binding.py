@@ -47,6 +47,8 @@ SIGNATURES = {
                                                  _P]),
     "grpo_loss_fwd_bwd_norm": (ctypes.c_int, [_P, _P, _P, _P, _P, _P, _P, _I64, _I64, _I32, _I64, _F, _F, _I32, _F,
                                               _P, _P, _P, _P, ctypes.c_size_t, _P]),
+    "grpo_loss_fwd_bwd_kl_clamp": (ctypes.c_int, [_P, _P, _P, _P, _P, _P, _P, _I64, _I64, _I32, _I64, _F, _F, _I32,
+                                                  _F, _F, _P, _P, _P, _P, ctypes.c_size_t, _P]),
     "grpo_loss_fwd_bwd_to_host": (ctypes.c_int, [_P, _P, _P, _P, _P, _P, _P, _I64, _I64, _I32, _I64, _F, _F, _I32,
                                                  _F, _P, _P, _P, _P, _P, ctypes.c_size_t, _P]),
     "grpo_loss_fwd_bwd_adamw": (ctypes.c_int, [_P, _P, _P, _P, _P, _P, _P, _I64, _I64, _I32, _I64, _F, _F, _I32, _F,
@@ -227,9 +229,11 @@ def loss_fwd_bwd(H: torch.Tensor, W: torch.Tensor, targets: torch.Tensor, mask: 
                  old_logp: torch.Tensor, ref_logp: torch.Tensor, adv: torch.Tensor,
                  n_resp: int, L: int, clip_eps: float = 0.2, beta: float = 0.04, agg_mode: int = 0,
                  ws: Optional[torch.Tensor] = None,
-                 out: Optional[Tuple[torch.Tensor, torch.Tensor, torch.Tensor]] = None, norm: float = 0.0):
+                 out: Optional[Tuple[torch.Tensor, torch.Tensor, torch.Tensor]] = None, norm: float = 0.0,
+                 kl_clamp: Optional[float] = None):
     """grpo_loss_fwd_bwd (norm == 0) / grpo_loss_fwd_bwd_norm (norm > 0, a global
-    N_valid or n_resp): returns (loss [1] fp32, dH [T, Hd] fp32, dW [V, Hd] fp32).
+    N_valid or n_resp) / grpo_loss_fwd_bwd_kl_clamp (kl_clamp given, a cap on the
+    per-token KL value): returns (loss [1] fp32, dH [T, Hd] fp32, dW [V, Hd] fp32).
     `out` may be device tensors (written in place) or host tensors, preferably
     pinned (the results are copied there before the call returns)."""
     dev, host = _target_device(H, W)
@@ -256,14 +260,17 @@ def loss_fwd_bwd(H: torch.Tensor, W: torch.Tensor, targets: torch.Tensor, mask: 
     common = (_ptr(H), _ptr(W), _ptr(targets), _ptr(mask), _ptr(old_logp), _ptr(ref_logp), _ptr(adv), int(n_resp),
               int(L), Hd, V, float(clip_eps), float(beta), int(agg_mode))
     tail = (_ptr(loss), _ptr(dH), _ptr(dW), _ptr(ws), ws.numel(), _stream(dev))
-    if host_out is not None and host_out[2].is_pinned():
+    if host_out is not None and host_out[2].is_pinned() and kl_clamp is None:
         # dW streams to the caller's pinned buffer chunk by chunk while the backward runs
         _check(lib.grpo_loss_fwd_bwd_to_host(*common, float(norm), _ptr(loss), _ptr(dH), _ptr(dW),
                                              _ptr(host_out[2]), _ptr(ws), ws.numel(), _stream(dev)),
                "grpo_loss_fwd_bwd_to_host")
         lh, dHh = _to_host(loss, dH, dst=host_out[:2])
         return lh, dHh, host_out[2]
-    if norm:
+    if kl_clamp is not None:
+        _check(lib.grpo_loss_fwd_bwd_kl_clamp(*common, float(norm), float(kl_clamp), *tail),
+               "grpo_loss_fwd_bwd_kl_clamp")
+    elif norm:
         _check(lib.grpo_loss_fwd_bwd_norm(*common, float(norm), *tail), "grpo_loss_fwd_bwd_norm")
     else:
         _check(lib.grpo_loss_fwd_bwd(*common, *tail), "grpo_loss_fwd_bwd")

@@ -453,7 +453,7 @@ grpo_status loss_impl(const uint16_t* H, const uint16_t* W, const int32_t* targe
                       const float* old_logp, const float* ref_logp, const float* adv, int64_t n_resp,
                       int64_t L, int32_t Hd, int64_t V, float clip_eps, float beta, int32_t agg_mode,
                       float norm, float* loss_out, float* dH, float* dW, const AdamParams* adam, void* ws,
-                      size_t ws_bytes, void* stream, float* dW_host = nullptr);
+                      size_t ws_bytes, void* stream, float* dW_host = nullptr, float kl_clamp = INFINITY);
 
 }  // namespace
 
@@ -634,6 +634,16 @@ grpo_status grpo_loss_fwd_bwd_norm(const uint16_t* H, const uint16_t* W, const i
                    norm, loss_out, dH, dW, nullptr, ws, ws_bytes, stream);
 }
 
+grpo_status grpo_loss_fwd_bwd_kl_clamp(const uint16_t* H, const uint16_t* W, const int32_t* targets,
+                                       const uint8_t* mask, const float* old_logp, const float* ref_logp,
+                                       const float* adv, int64_t n_resp, int64_t L, int32_t Hd, int64_t V,
+                                       float clip_eps, float beta, int32_t agg_mode, float norm, float kl_clamp,
+                                       float* loss_out, float* dH, float* dW, void* ws, size_t ws_bytes,
+                                       void* stream) {
+  return loss_impl(H, W, targets, mask, old_logp, ref_logp, adv, n_resp, L, Hd, V, clip_eps, beta, agg_mode,
+                   norm, loss_out, dH, dW, nullptr, ws, ws_bytes, stream, nullptr, kl_clamp);
+}
+
 grpo_status grpo_loss_fwd_bwd_to_host(const uint16_t* H, const uint16_t* W, const int32_t* targets,
                                       const uint8_t* mask, const float* old_logp, const float* ref_logp,
                                       const float* adv, int64_t n_resp, int64_t L, int32_t Hd, int64_t V,
@@ -683,9 +693,10 @@ grpo_status loss_impl(const uint16_t* H, const uint16_t* W, const int32_t* targe
                       const float* old_logp, const float* ref_logp, const float* adv, int64_t n_resp,
                       int64_t L, int32_t Hd, int64_t V, float clip_eps, float beta, int32_t agg_mode,
                       float norm, float* loss_out, float* dH, float* dW, const AdamParams* adam, void* ws,
-                      size_t ws_bytes, void* stream, float* dW_host) {
+                      size_t ws_bytes, void* stream, float* dW_host, float kl_clamp) {
   if (n_resp < 1 || L < 1 || n_resp > (int64_t(1) << 31) / L) return GRPO_ERR_INVALID_ARG;
   if (!(norm >= 0.f) || norm == INFINITY) return GRPO_ERR_INVALID_ARG;
+  if (!(kl_clamp >= 0.f)) return GRPO_ERR_INVALID_ARG;
   const int64_t T = n_resp * L;
   Layout Ly;
   if (!make_layout(T, Hd, V, GRPO_WS_LOSS, &Ly)) return GRPO_ERR_INVALID_ARG;
@@ -717,7 +728,7 @@ grpo_status loss_impl(const uint16_t* H, const uint16_t* W, const int32_t* targe
     loss_terms_kernel<<<static_cast<unsigned>(Ly.nblk_loss), kLossThreads, 0, s>>>(
         at<int>(ws, Ly.cidx), n_valid, at<float>(ws, Ly.part_m), at<float>(ws, Ly.part_s),
         static_cast<int>(Ly.nsplit), Ly.T_pad, at<float>(ws, Ly.zy), at<int>(ws, Ly.yc), old_logp,
-        ref_logp, adv, L, at<int>(ws, Ly.resp_len), n_resp, agg_mode, norm, clip_eps, beta,
+        ref_logp, adv, L, at<int>(ws, Ly.resp_len), n_resp, agg_mode, norm, clip_eps, beta, kl_clamp,
         at<float>(ws, Ly.lse_c), at<float>(ws, Ly.g_c), at<double>(ws, Ly.block_loss), status);
     loss_final_kernel<<<1, 1024, 0, s>>>(at<double>(ws, Ly.block_loss), n_valid, kLossThreads, loss_out);
     e = cudaGetLastError();

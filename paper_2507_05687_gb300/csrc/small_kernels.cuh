@@ -264,7 +264,7 @@ __global__ void loss_terms_kernel(const int* __restrict__ cidx, const int* __res
                                   const int* __restrict__ yc, const float* __restrict__ old_logp,
                                   const float* __restrict__ ref_logp, const float* __restrict__ adv,
                                   int64_t L, const int* __restrict__ resp_len, int64_t n_resp,
-                                  int agg_mode, float norm, float clip_eps, float beta,
+                                  int agg_mode, float norm, float clip_eps, float beta, float kl_clamp,
                                   float* __restrict__ lse_c, float* __restrict__ g_c,
                                   double* __restrict__ block_loss, unsigned* status) {
   __shared__ double sh[32];
@@ -288,13 +288,17 @@ __global__ void loss_terms_kernel(const int* __restrict__ cidx, const int* __res
       const float s = unclipped ? s1 : s2;
       const float dref = ref_logp[t] - logp;
       const float e = __expf(dref);
-      const float kl = e - dref - 1.f;
+      const float k3 = e - dref - 1.f;
+      // capped KL: above the cap the value is the cap and the slope 0 (a tie is inside;
+      // an infinite cap leaves every value, NaN included, as it is)
+      const bool kl_in = !(k3 > kl_clamp);
+      const float kl = kl_in ? k3 : kl_clamp;
       const float ell = -s + beta * kl;
       // norm > 0 replaces the local count (N_valid, or n_resp) by a global one
       const float w = agg_mode == 0
                           ? 1.f / (norm > 0.f ? norm : static_cast<float>(nv))
                           : 1.f / ((norm > 0.f ? norm : static_cast<float>(n_resp)) * static_cast<float>(resp_len[i]));
-      g = w * ((unclipped ? -A * rho : 0.f) + beta * (1.f - e));
+      g = w * ((unclipped ? -A * rho : 0.f) + (kl_in ? beta * (1.f - e) : 0.f));
       contrib = static_cast<double>(w) * static_cast<double>(ell);
     } else {
       lse = 0.f;

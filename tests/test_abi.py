@@ -88,6 +88,12 @@ def test_host_rejections(lib):
     assert L.grpo_loss_fwd_bwd(*bad) == grpo.GRPO_ERR_INVALID_ARG
     bad = list(largs); bad[18] = ws2 - 1024
     assert L.grpo_loss_fwd_bwd(*bad) == grpo.GRPO_ERR_WORKSPACE
+    kargs = largs[:14] + [0.0, 1.0] + largs[14:]
+    for kappa in (-1.0, float("nan"), float("-inf")):
+        bad = list(kargs); bad[15] = kappa
+        assert L.grpo_loss_fwd_bwd_kl_clamp(*bad) == grpo.GRPO_ERR_INVALID_ARG, kappa
+    bad = list(kargs); bad[7] = 0                 # n_resp 0
+    assert L.grpo_loss_fwd_bwd_kl_clamp(*bad) == grpo.GRPO_ERR_INVALID_ARG
     assert L.grpo_check_device_status(None, None) == grpo.GRPO_ERR_INVALID_ARG
     ws3 = grpo.workspace_bytes(100, 64, 1000, grpo.GRPO_WS_LOGPROBS_HEADS)
     assert ws3 > grpo.workspace_bytes(100, 64, 1000, grpo.GRPO_WS_LOGPROBS)

@@ -180,6 +180,41 @@ def test_global_normaliser(agg_mode):
     assert rel_fro(dW.double().cpu().numpy(), want["dW"]) <= GRAD_RTOL
 
 
+@pytest.mark.parametrize("agg_mode", [0, 1])
+def test_clamped_kl(agg_mode):
+    """grpo_loss_fwd_bwd_kl_clamp: reference log-probs at fixed offsets d from the
+    policy's, so that k3(d) lies on both sides of the cap, each value at least
+    0.29 from it (the GPU's log-prob error moves k3 by < 0.01)."""
+    w = wl.Workload("t", 2, 4, 60, 128, 1500, "uniform", 1, 60, rewards="mix", seed=wl.SEED_BASE + 660)
+    c = _case(w, agg_mode)
+    kappa, beta = 0.4, 0.5
+    rng = np.random.default_rng(w.seed + 9)
+    d = rng.choice([-1.5, -0.5, 0.3, 1.0, 1.5], size=w.T)     # k3 = 0.72, 0.11, 0.05, 0.72, 2.98
+    ref = (c["want"]["logp"] + d).astype(np.float32)
+    args = (c["H"], c["W"], c["y"], c["m"], c["old"], ref, c["adv"], w.n_resp, w.L, w.clip_eps, beta, agg_mode)
+    want = oracle.loss_fwd_bwd(*args, kl_clamp=kappa)
+    plain = oracle.loss_fwd_bwd(*args)
+    capped = ~want["terms"]["kl_inside"] & (c["m"] != 0)
+    assert 0.2 < capped.mean() / (c["m"] != 0).mean() < 0.8
+    assert rel_fro(want["dW"], plain["dW"]) > 5 * GRAD_RTOL      # the cap changes the gradient visibly
+    dd = _dev(c)
+    ws = grpo.workspace(w.T, w.Hd, w.V, grpo.GRPO_WS_LOSS, DEV)
+    loss, dH, dW = grpo.loss_fwd_bwd(dd["H"], dd["W"], dd["y"], dd["m"], dd["old"], dev_tensor(ref, torch.float32),
+                                     dd["adv"], w.n_resp, w.L, w.clip_eps, beta, agg_mode, ws=ws, kl_clamp=kappa)
+    assert grpo.check_device_status(ws) == grpo.GRPO_OK
+    scale = loss_scale(want["loss"], want["terms"]["w"], want["terms"]["ell"])
+    assert abs(loss.item() - want["loss"]) <= LOSS_RTOL * scale, (loss.item(), want["loss"])
+    assert rel_fro(dH.double().cpu().numpy(), want["dH"]) <= GRAD_RTOL
+    assert rel_fro(dW.double().cpu().numpy(), want["dW"]) <= GRAD_RTOL
+    # an infinite cap is the plain entry point, bit for bit
+    a = grpo.loss_fwd_bwd(dd["H"], dd["W"], dd["y"], dd["m"], dd["old"], dev_tensor(ref, torch.float32), dd["adv"],
+                          w.n_resp, w.L, w.clip_eps, beta, agg_mode, kl_clamp=float("inf"))
+    b = grpo.loss_fwd_bwd(dd["H"], dd["W"], dd["y"], dd["m"], dd["old"], dev_tensor(ref, torch.float32), dd["adv"],
+                          w.n_resp, w.L, w.clip_eps, beta, agg_mode)
+    for x, y in zip(a, b):
+        assert torch.equal(x, y)
+
+
 def test_fwd_bwd_is_deterministic():
     c = _case(wl.Workload("t", 1, 4, 70, 256, 2000, "uniform", 5, 70, seed=wl.SEED_BASE + 600))
     a = _check_fwd_bwd(c)

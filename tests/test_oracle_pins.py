@@ -246,6 +246,72 @@ def test_gradient_matches_central_differences(agg):
     assert np.all(out["dH"][c["mask"] == 0] == 0.0)
 
 
+def _clamp_case(seed=33, kl_clamp=0.15):
+    """A tiny case whose per-token k3 values lie on both sides of kl_clamp, each
+    at least 0.02 away from it (finite differences stay on one side)."""
+    c = _rand_case(seed, T_resp=2, G=2, L=3, Hd=4, V=6, scale=0.8)
+    logp, _ = oracle.token_logprobs(c["H"], c["W"], c["y"], c["mask"])
+    old, _ = _old_ref(logp, c["rng"])
+    d = np.tile([-1.2, -0.2, 0.9, 0.1, 1.6, -0.5], logp.size // 6 + 1)[:logp.size]
+    ref = logp + d
+    k3 = np.exp(d) - d - 1.0
+    m = c["mask"] != 0
+    assert np.any(k3[m] > kl_clamp + 0.02) and np.any(k3[m] < kl_clamp - 0.02)
+    assert np.all(np.abs(k3 - kl_clamp) > 0.02)
+    return c, old, ref
+
+
+def test_clamped_kl_gradient_matches_central_differences():
+    kappa, beta = 0.15, 0.3
+    c, old, ref = _clamp_case(kl_clamp=kappa)
+    adv = oracle.group_advantages(c["rewards"], c["G"])
+    out = oracle.loss_fwd_bwd(c["H"], c["W"], c["y"], c["mask"], old, ref, adv, c["n_resp"], c["L"],
+                              0.2, beta, 0, vocab_chunk=4, kl_clamp=kappa)
+    logp = oracle.token_logprobs(c["H"], c["W"], c["y"], c["mask"])[0]
+    bl = brute.loss(logp.tolist(), old.tolist(), ref.tolist(), adv.astype(float).tolist(), c["mask"].tolist(),
+                    c["n_resp"], c["L"], 0.2, beta, 0, kl_clamp=kappa)
+    assert out["loss"] == pytest.approx(bl, rel=1e-12, abs=1e-15)
+    h = 1e-6
+
+    def f(H, W):
+        lp = brute.logprobs(H.tolist(), W.tolist(), c["y"].tolist(), c["mask"].tolist())
+        return brute.loss(lp, old.tolist(), ref.tolist(), adv.astype(float).tolist(), c["mask"].tolist(),
+                          c["n_resp"], c["L"], 0.2, beta, 0, kl_clamp=kappa)
+    for name, X, dX in (("H", c["H"], out["dH"]), ("W", c["W"], out["dW"])):
+        fd = np.zeros_like(X)
+        for i in range(X.shape[0]):
+            for j in range(X.shape[1]):
+                Xp = X.copy(); Xp[i, j] += h
+                Xm = X.copy(); Xm[i, j] -= h
+                fp = f(Xp, c["W"]) if name == "H" else f(c["H"], Xp)
+                fm = f(Xm, c["W"]) if name == "H" else f(c["H"], Xm)
+                fd[i, j] = (fp - fm) / (2 * h)
+        np.testing.assert_allclose(dX, fd, rtol=1e-5, atol=1e-9, err_msg=name)
+
+
+def test_kl_clamp_special_cases():
+    """A cap of 0 removes the KL term (k3 >= 0), so the result is that of beta = 0;
+    a cap above every k3 is the plain estimator, bit for bit."""
+    c, old, ref = _clamp_case()
+    adv = oracle.group_advantages(c["rewards"], c["G"])
+    args = (c["H"], c["W"], c["y"], c["mask"], old, ref, adv, c["n_resp"], c["L"], 0.2)
+    zero = oracle.loss_fwd_bwd(*args, 0.3, 0, vocab_chunk=4, kl_clamp=0.0)
+    nokl = oracle.loss_fwd_bwd(*args, 0.0, 0, vocab_chunk=4)
+    assert zero["loss"] == pytest.approx(nokl["loss"], rel=1e-12, abs=1e-15)
+    np.testing.assert_allclose(zero["dH"], nokl["dH"], rtol=1e-12, atol=1e-15)
+    np.testing.assert_allclose(zero["dW"], nokl["dW"], rtol=1e-12, atol=1e-15)
+    big = oracle.loss_fwd_bwd(*args, 0.3, 0, vocab_chunk=4, kl_clamp=1e30)
+    plain = oracle.loss_fwd_bwd(*args, 0.3, 0, vocab_chunk=4)
+    assert big["loss"] == plain["loss"]
+    assert np.array_equal(big["dH"], plain["dH"]) and np.array_equal(big["dW"], plain["dW"])
+    # capped tokens carry exactly the cap as their KL value
+    tt = plain["terms"]
+    kt = oracle.token_terms(plain["logp"], old, ref, np.zeros_like(old), 0.2, 0.3, 0.15)
+    capped = ~kt["kl_inside"]
+    assert capped.any() and np.all(kt["kl"][capped] == 0.15)
+    assert np.array_equal(kt["kl"][~capped], tt["kl"][~capped])
+
+
 def test_dW_column_sums_vanish_and_sampled_rows_match():
     c = _rand_case(41, T_resp=3, G=4, L=6, Hd=8, V=23)
     logp, _ = oracle.token_logprobs(c["H"], c["W"], c["y"], c["mask"])
@@ -370,8 +436,8 @@ def test_planted_population_std_is_caught(monkeypatch):
 def test_planted_kl_without_minus_one_is_caught(monkeypatch):
     real = go.token_terms
 
-    def bad(logp, old, ref, A, clip_eps, beta):
-        tt = real(logp, old, ref, A, clip_eps, beta)
+    def bad(logp, old, ref, A, clip_eps, beta, *rest):
+        tt = real(logp, old, ref, A, clip_eps, beta, *rest)
         tt["kl"] = tt["kl"] + 1.0
         tt["ell"] = -tt["s"] + beta * tt["kl"]
         return tt
@@ -392,7 +458,7 @@ def test_planted_target_off_by_one_is_caught(monkeypatch):
 def test_planted_gradient_sign_is_caught(monkeypatch):
     real = go.logp_coef
 
-    def bad(logp, old, ref, A, w, clip_eps, beta):
+    def bad(logp, old, ref, A, w, clip_eps, beta, *rest):
         lp = np.asarray(logp, np.float64)
         tt = go.token_terms(logp, old, ref, A, clip_eps, beta)
         dsurr = np.where(tt["unclipped"], np.asarray(A) * tt["rho"], 0.0)
@@ -400,6 +466,15 @@ def test_planted_gradient_sign_is_caught(monkeypatch):
     monkeypatch.setattr(go, "logp_coef", bad)
     with pytest.raises(AssertionError):
         test_gradient_matches_central_differences(0)
+    monkeypatch.setattr(go, "logp_coef", real)
+
+
+def test_planted_clamp_without_gradient_cut_is_caught(monkeypatch):
+    real = go.logp_coef
+    # the capped tokens keep their KL gradient: the value is capped, the slope is not
+    monkeypatch.setattr(go, "logp_coef", lambda *a: real(*a[:7]))
+    with pytest.raises(AssertionError):
+        test_clamped_kl_gradient_matches_central_differences()
     monkeypatch.setattr(go, "logp_coef", real)
 
 
