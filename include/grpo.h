@@ -123,6 +123,18 @@ grpo_status grpo_sample_tokens(const uint16_t* H, const uint16_t* W, const uint8
                                float* logp_out, void* ws, size_t ws_bytes, void* stream);
 
 /*
+ * The noise grpo_sample_tokens adds, written out for checking the generator
+ * and the logarithms (the draw of Eq. 1 has no other observable):
+ *   out[(t - row0) * cols + v] = G_{t,v}  for row0 <= t < row0 + rows, 0 <= v < cols
+ * with G, U and the Philox counter exactly as grpo_sample_tokens defines them
+ * (t is the token position).  out is [rows x cols] fp32 device memory (4-byte
+ * aligned); row0 >= 0, row0 + rows <= 2^32, cols < 2^31, rows * cols <= 2^40.
+ * Asynchronous on `stream`.
+ */
+grpo_status grpo_gumbel_noise(uint64_t seed, uint64_t offset, int64_t row0, int64_t rows, int64_t cols,
+                              float* out, void* stream);
+
+/*
  * GRPO loss (the negated objective of Eq. 1, Section 3.3) and its gradient
  * with respect to H and W.  Per unmasked token t of response i = t / L:
  *   rho  = exp(logp_t - old_logp_t)

@@ -56,6 +56,7 @@ SIGNATURES = {
                                                ctypes.c_size_t, _P]),
     "grpo_sample_tokens": (ctypes.c_int, [_P, _P, _P, _I64, _I32, _I64, _F, ctypes.c_uint64, ctypes.c_uint64, _P, _P,
                                           _P, ctypes.c_size_t, _P]),
+    "grpo_gumbel_noise": (ctypes.c_int, [ctypes.c_uint64, ctypes.c_uint64, _I64, _I64, _I64, _P, _P]),
     "grpo_adamw_step": (ctypes.c_int, [_P, _P, _P, _P, _P, _I64, _F, _F, _F, _F, _F, _I64, _P]),
     "grpo_token_logprobs_noalloc": (ctypes.c_int, [_P, _P, _P, _P, _I64, _I32, _I64, _P, _P]),
     "grpo_workspace_bytes": (ctypes.c_size_t, [_I64, _I32, _I64, _I32]),
@@ -330,6 +331,16 @@ def adamw_step(W_master: torch.Tensor, exp_avg: torch.Tensor, exp_avg_sq: torch.
     _check(load().grpo_adamw_step(_ptr(W_master), _ptr(exp_avg), _ptr(exp_avg_sq), _ptr(grad), _ptr(W_out), n,
                                   float(lr), float(betas[0]), float(betas[1]), float(eps), float(weight_decay),
                                   int(step), _stream(W_master.device)), "grpo_adamw_step")
+
+
+def gumbel_noise(row0: int, rows: int, cols: int, seed: int, offset: int = 0, device=None) -> torch.Tensor:
+    """grpo_gumbel_noise: the fp32 noise grpo_sample_tokens adds to z / temperature at
+    token positions row0 .. row0 + rows - 1 and vocabulary ids 0 .. cols - 1."""
+    dev = torch.device("cuda", torch.cuda.current_device()) if device is None else torch.device(device)
+    out = torch.empty(rows, cols, dtype=torch.float32, device=dev)
+    _check(load().grpo_gumbel_noise(int(seed) & (2**64 - 1), int(offset) & (2**64 - 1), int(row0), int(rows),
+                                    int(cols), _ptr(out), _stream(dev)), "grpo_gumbel_noise")
+    return out
 
 
 def check_device_status(ws: torch.Tensor) -> int:

@@ -6,13 +6,13 @@
 // Tile 128 x 256 per CTA (kPair = 1) or 256 x 256 per CTA pair (kPair = 2,
 // tcgen05 cta_group::2: each CTA stages its own 128 rows of A and half of B's
 // 256 columns, the even CTA issues the MMAs for both, and each CTA's TMEM
-// holds its 128 accumulator rows).  Roles per CTA (64 + 32 kEpiWarps threads):
+// holds its 128 accumulator rows).  Roles per CTA (64 + 32 EpiShape::kWarps threads):
 //   warp 0      TMA producer: 64-wide k-blocks (128-byte swizzle) into a ring
 //               of shared-memory stages.
 //   warp 1      owns 512 TMEM columns (two 256-column accumulators, so the
 //               epilogue of tile i overlaps the MMAs of tile i + 1); one lane
 //               of the issuing CTA issues the 128x256x16 / 256x256x16 MMAs.
-//   warps 2..   epilogue (kEpiWarps of them): one thread per accumulator row
+//   warps 2..   epilogue (EpiShape::kWarps of them): one thread per accumulator row
 //               (TMEM lane), 32 columns per tcgen05.ld; with 8 warps two share a
 //               lane quarter and split the columns, their per-row log-softmax /
 //               sampling state written as separate split entries.
@@ -48,13 +48,6 @@ namespace grpo {
 constexpr int kBK = 64;            // bf16 elements per 128-byte swizzle row
 constexpr int kTileN = 256;        // accumulator columns per TMEM buffer
 constexpr int kRowsCta = 128;      // accumulator rows per CTA (TMEM lanes)
-// Epilogue warps: 4 = one per TMEM lane quarter (each thread walks its row's
-// 256 columns); 8 = two per quarter, each taking half the columns.  Measured
-// on the 8B batch: 8 warps slowed the dW GEMM (15.7 -> 16.7 ms per step) and
-// did not speed up the sampling epilogue (its integer / MUFU pipes are busy).
-constexpr int kEpiWarps = 4;
-constexpr int kEpiHalves = kEpiWarps / 4;        // column halves of a tile, one per warp of a quarter
-constexpr int kGemmThreads = 64 + 32 * kEpiWarps;
 constexpr int kTmemCols = 512;
 constexpr int kRowAlign = 256;     // row padding of every token-indexed buffer
 constexpr int kMaxHeads = 4;       // LM heads one forward launch can sweep
@@ -71,6 +64,18 @@ struct TileCfg {
 };
 
 enum { kEpiLse = 0, kEpiDz = 1, kEpiF32 = 2, kEpiAdam = 3, kEpiSample = 4 };
+
+// Epilogue warps per CTA: 4 = one per TMEM lane quarter (each thread walks its
+// row's 256 columns); 8 = two per quarter, each taking half the columns.  The
+// sampling epilogue (Philox and two logarithms per element) uses 8: measured
+// on the 8B batch, 17.6 -> 16.7 ms.  The others keep 4: with 8, the dW GEMM
+// of the same batch went from 15.7 to 16.7 ms per step.
+template <int kEpi>
+struct EpiShape {
+  static constexpr int kWarps = kEpi == kEpiSample ? 8 : 4;
+  static constexpr int kHalves = kWarps / 4;    // column halves of a tile, one per warp of a quarter
+  static constexpr int kThreads = 64 + 32 * kWarps;
+};
 
 struct GemmArgs {
   const int* n_valid;   // device: number of compacted rows
@@ -89,8 +94,8 @@ struct GemmArgs {
 
   // kEpiLse
   const int* yc;        // [M] target of each compacted row (-1: none)
-  float* part_m;        // [units_n x kEpiHalves x ldp] running max (log2 units)
-  float* part_s;        // [units_n x kEpiHalves x ldp] running sum of 2^(z log2e - max)
+  float* part_m;        // [units_n x halves x ldp] running max (log2 units); halves = EpiShape::kHalves
+  float* part_s;        // [units_n x halves x ldp] running sum of 2^(z log2e - max)
   float* zy;            // [n_heads x ldp] logit of the target
   long ldp;
 
@@ -120,9 +125,9 @@ struct GemmArgs {
   // kEpiSample (row_map gives the token position t of each compacted row)
   float inv_temp;       // 1 / temperature
   uint32_t seed_lo, seed_hi, off_lo, off_hi;
-  float* best_s;        // [units_n x kEpiHalves x ldp] best perturbed score of the split entry
-  int* best_c;          // [units_n x kEpiHalves x ldp] its vocabulary column
-  float* best_z;        // [units_n x kEpiHalves x ldp] its z / temperature
+  float* best_s;        // [units_n x halves x ldp] best perturbed score of the split entry
+  int* best_c;          // [units_n x halves x ldp] its vocabulary column
+  float* best_z;        // [units_n x halves x ldp] its z / temperature
 };
 
 struct TileSched {
@@ -218,7 +223,7 @@ template <int kEpi>
 __device__ __forceinline__ void epi_tile(EpiRow& e, const GemmArgs& a, uint32_t tbase, int col0,
                                          bool have_acc, int half) {
   const float kLog2e = 1.4426950408889634f;
-  constexpr int kChunks = kTileN / 32 / kEpiHalves;
+  constexpr int kChunks = kTileN / 32 / EpiShape<kEpi>::kHalves;
 #pragma unroll 1
   for (int c = half * kChunks; c < (half + 1) * kChunks; ++c) {
     float v[32];
@@ -378,7 +383,7 @@ __device__ __forceinline__ void epi_tile(EpiRow& e, const GemmArgs& a, uint32_t 
 
 template <int kEpi>
 __device__ __forceinline__ void epi_end(const EpiRow& e, const GemmArgs& a, int un, int head, int half) {
-  const long entry = static_cast<long>(un) * kEpiHalves + half;  // split entry of this column half
+  const long entry = static_cast<long>(un) * EpiShape<kEpi>::kHalves + half;  // split entry of this column half
   if (kEpi == kEpiSample && e.rv) {
     const long at = entry * a.ldp + e.r;
     a.part_m[at] = e.run_m;
@@ -426,7 +431,7 @@ __device__ __forceinline__ void gemm_body(const CUtensorMap* tmA, const CUtensor
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(smem_addr(&tfull_bar[i]), 1);
-      mbar_init(smem_addr(&tempty_bar[i]), kEpiWarps * kPair);  // one arrival per epilogue warp
+      mbar_init(smem_addr(&tempty_bar[i]), EpiShape<kEpi>::kWarps * kPair);  // one arrival per epilogue warp
     }
     mbar_init(smem_addr(done_bar), 1);
     *abort_flag = 0;
@@ -656,7 +661,7 @@ __device__ __forceinline__ void gemm_body(const CUtensorMap* tmA, const CUtensor
 
 // One tensor map per B matrix; B1..B3 are read only when args.n_heads > 1.
 template <int kEpi, bool kAmn, bool kBmn>
-__global__ void __launch_bounds__(kGemmThreads, 1)
+__global__ void __launch_bounds__(EpiShape<kEpi>::kThreads, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB0,
                    const __grid_constant__ CUtensorMap tmB1, const __grid_constant__ CUtensorMap tmB2,
                    const __grid_constant__ CUtensorMap tmB3, const GemmArgs args) {
@@ -665,7 +670,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
 }
 
 template <int kEpi, bool kAmn, bool kBmn>
-__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(EpiShape<kEpi>::kThreads, 1)
     gemm_tc_pair_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB0,
                         const __grid_constant__ CUtensorMap tmB1, const __grid_constant__ CUtensorMap tmB2,
                         const __grid_constant__ CUtensorMap tmB3, const GemmArgs args) {

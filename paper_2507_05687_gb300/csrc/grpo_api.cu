@@ -55,7 +55,8 @@ bool make_layout(int64_t T, int32_t Hd, int64_t V, int32_t which, Layout* L) {
   L->T_pad = round_up(std::max<int64_t>(T, 1), kRowAlign);
   const int64_t vtiles = (V + kTileN - 1) / kTileN;
   // partial (max, sum) entries per row: one per vocabulary split and column half
-  L->nsplit = (vtiles + kLseTilesPerUnit - 1) / kLseTilesPerUnit * kEpiHalves;
+  L->nsplit = (vtiles + kLseTilesPerUnit - 1) / kLseTilesPerUnit *
+              (which == GRPO_WS_SAMPLE ? EpiShape<kEpiSample>::kHalves : EpiShape<kEpiLse>::kHalves);
   L->nblk_scan = (std::max<int64_t>(T, 1) + kScanChunk - 1) / kScanChunk;
   L->nblk_loss = (L->T_pad + kLossThreads - 1) / kLossThreads;
   L->vchunk = which == GRPO_WS_LOSS ? vocab_chunk(V) : 0;
@@ -139,7 +140,7 @@ bool prepare_kernels(int* pairs) {
     return false;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(2 * 1024, 1, 1);
-  cfg.blockDim = dim3(kGemmThreads, 1, 1);
+  cfg.blockDim = dim3(EpiShape<E>::kThreads, 1, 1);
   cfg.dynamicSmemBytes = TileCfg<2>::kSmemBytes;
   int n = 0;
   if (cudaOccupancyMaxActiveClusters(&n, gemm_tc_pair_kernel<E, A, B>, &cfg) != cudaSuccess) {
@@ -347,11 +348,12 @@ cudaError_t launch_gemm_cfg(const Operand& A, const Operand* B, const GemmArgs& 
                         ((n_tiles + a.n_per_unit - 1) / a.n_per_unit) * a.n_heads;
   if (kPair == 2) {
     const int64_t pairs = std::max<int64_t>(1, std::min<int64_t>(di.pairs, units));
-    gemm_tc_pair_kernel<E, AMN, BMN><<<static_cast<unsigned>(2 * pairs), kGemmThreads, C::kSmemBytes, s>>>(
+    gemm_tc_pair_kernel<E, AMN, BMN><<<static_cast<unsigned>(2 * pairs), EpiShape<E>::kThreads, C::kSmemBytes,
+                                       s>>>(
         ta, tb[0], tb[1], tb[2], tb[3], a);
   } else {
     const int64_t grid = std::max<int64_t>(1, std::min<int64_t>(di.sms, units));
-    gemm_tc_kernel<E, AMN, BMN><<<static_cast<unsigned>(grid), kGemmThreads, C::kSmemBytes, s>>>(
+    gemm_tc_kernel<E, AMN, BMN><<<static_cast<unsigned>(grid), EpiShape<E>::kThreads, C::kSmemBytes, s>>>(
         ta, tb[0], tb[1], tb[2], tb[3], a);
   }
   return cudaGetLastError();
@@ -613,6 +615,23 @@ grpo_status grpo_sample_tokens(const uint16_t* H, const uint16_t* W, const uint8
     e = cudaGetLastError();
   }
   return from_cuda(e);
+}
+
+grpo_status grpo_gumbel_noise(uint64_t seed, uint64_t offset, int64_t row0, int64_t rows, int64_t cols,
+                              float* out, void* stream) {
+  if (row0 < 0 || rows < 0 || cols < 0 || row0 > (int64_t(1) << 32) - rows || cols >= (int64_t(1) << 31))
+    return GRPO_ERR_INVALID_ARG;
+  if (rows > 0 && cols > 0 && rows > (int64_t(1) << 40) / cols) return GRPO_ERR_INVALID_ARG;
+  if (rows == 0 || cols == 0) return GRPO_OK;
+  if (!out || !aligned(out, 4)) return GRPO_ERR_INVALID_ARG;
+  DeviceInfo di;
+  if (!device_info(&di)) return GRPO_ERR_UNSUPPORTED;
+  const int64_t work = rows * ((cols + 3) / 4);
+  const int blocks = static_cast<int>(std::min<int64_t>((work + 255) / 256, int64_t(di.sms) * 16));
+  gumbel_noise_kernel<<<blocks, 256, 0, static_cast<cudaStream_t>(stream)>>>(
+      static_cast<uint32_t>(seed), static_cast<uint32_t>(seed >> 32), static_cast<uint32_t>(offset),
+      static_cast<uint32_t>(offset >> 32), row0, rows, cols, out);
+  return from_cuda(cudaGetLastError());
 }
 
 grpo_status grpo_loss_fwd_bwd(const uint16_t* H, const uint16_t* W, const int32_t* targets,

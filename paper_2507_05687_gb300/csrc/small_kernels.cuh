@@ -227,6 +227,26 @@ __global__ void logp_merge_kernel(const uint8_t* __restrict__ mask, const int* _
 // The sampled token of every row: the split with the best perturbed score
 // (the lowest split on a tie, i.e. the lowest column), and its log-prob under
 // softmax(z / temperature).  Masked rows: token -1, log-prob 0.
+// The sampler's noise G_{t,v} for a [rows x cols] block: one thread per group
+// of 4 columns (one Philox call), grid-stride over the block.
+__global__ void gumbel_noise_kernel(uint32_t seed_lo, uint32_t seed_hi, uint32_t off_lo, uint32_t off_hi,
+                                    int64_t row0, int64_t rows, int64_t cols, float* __restrict__ out) {
+  const int64_t groups = (cols + 3) / 4;
+  for (int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; i < rows * groups;
+       i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+    const int64_t t = i / groups;
+    const int64_t g = i - t * groups;
+    const uint4 w = philox4x32_10(
+        make_uint4(static_cast<uint32_t>(g), static_cast<uint32_t>(row0 + t), off_lo, off_hi), seed_lo, seed_hi);
+    const uint32_t ws[4] = {w.x, w.y, w.z, w.w};
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      const int64_t v = 4 * g + k;
+      if (v < cols) out[t * cols + v] = gumbel_of(ws[k]);
+    }
+  }
+}
+
 __global__ void sample_merge_kernel(const uint8_t* __restrict__ mask, const int* __restrict__ rank_of, int64_t T,
                                     const float* __restrict__ pm, const float* __restrict__ ps,
                                     const float* __restrict__ bs, const int* __restrict__ bc,

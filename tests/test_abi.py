@@ -94,6 +94,12 @@ def test_host_rejections(lib):
         assert L.grpo_loss_fwd_bwd_kl_clamp(*bad) == grpo.GRPO_ERR_INVALID_ARG, kappa
     bad = list(kargs); bad[7] = 0                 # n_resp 0
     assert L.grpo_loss_fwd_bwd_kl_clamp(*bad) == grpo.GRPO_ERR_INVALID_ARG
+    for row0, rows, cols in ((0, -1, 4), (0, 4, -1), (-1, 4, 4), (0, 2**32 + 1, 4), (2**32 - 3, 4, 4),
+                             (0, 4, 2**31), (0, 2**21, 2**20)):
+        assert L.grpo_gumbel_noise(1, 2, row0, rows, cols, FAKE, None) == grpo.GRPO_ERR_INVALID_ARG, (row0, rows)
+    assert L.grpo_gumbel_noise(1, 2, 0, 4, 4, None, None) == grpo.GRPO_ERR_INVALID_ARG
+    assert L.grpo_gumbel_noise(1, 2, 0, 4, 4, FAKE + 2, None) == grpo.GRPO_ERR_INVALID_ARG
+    assert L.grpo_gumbel_noise(1, 2, 2**32, 0, 4, None, None) == grpo.GRPO_OK
     assert L.grpo_check_device_status(None, None) == grpo.GRPO_ERR_INVALID_ARG
     ws3 = grpo.workspace_bytes(100, 64, 1000, grpo.GRPO_WS_LOGPROBS_HEADS)
     assert ws3 > grpo.workspace_bytes(100, 64, 1000, grpo.GRPO_WS_LOGPROBS)

@@ -89,3 +89,23 @@ def test_sampling_rejects_bad_temperature():
     for tau in (0.0, -1.0, float("inf")):
         with pytest.raises(grpo.GrpoError):
             grpo.sample_tokens(H, W, m, tau)
+
+
+
+def test_noise_matches_float64():
+    """The kernel's Gumbel noise (exact uniforms, a series for -ln U near U = 1,
+    the hardware log2 elsewhere) against float64 -log(-log U) on 20 x 155136
+    draws, at token positions up to 2^32 - 1 and an offset above 2^32 so every
+    counter word is exercised.  The large values, which decide the argmax, must
+    be accurate to a few fp32 ulps; every value to far below the 1e-3 tie margin."""
+    V, seed, offset = 155136, 20250705, (7 << 32) + 12345
+    starts = [0, 65534, 2**31 - 2, 2**32 - 2]
+    rows = np.concatenate([np.arange(r, r + 6) if r + 6 <= 2**32 else np.arange(r, 2**32) for r in starts])
+    got = np.concatenate([grpo.gumbel_noise(r, min(6, 2**32 - r), V, seed, offset).double().cpu().numpy()
+                          for r in starts])
+    want = oracle.gumbel_noise(seed, offset, rows, V)
+    err = np.abs(got - want)
+    tail = want > 4.2                      # U > 0.985: the series branch
+    assert tail.sum() > 1000 and (want > 11.0).sum() > 5
+    assert err.max() <= 5e-5, err.max()
+    assert (err[tail] / want[tail]).max() <= 1e-6, (err[tail] / want[tail]).max()
