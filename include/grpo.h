@@ -305,7 +305,7 @@ enum {
   GRPO_K_DZ_GEMM = 5,     /* recomputed logits -> dZ chunk (bf16) */
   GRPO_K_DH_GEMM = 6,     /* dH (+)= dZ_chunk W_chunk */
   GRPO_K_DW_GEMM = 7,     /* dW_chunk = dZ_chunk^T H */
-  GRPO_K_ZERO_ROWS = 8,   /* zero dH rows of padding tokens */
+  GRPO_K_DH_ROWS = 8,     /* dH rows from the compacted order to the padded one (padding rows 0) */
   GRPO_K_ADAMW = 9,       /* standalone AdamW step (grpo_adamw_step) */
   GRPO_K_SAMPLE_GEMM = 10 /* logits GEMM + log-sum-exp + Gumbel-max draw */
 };

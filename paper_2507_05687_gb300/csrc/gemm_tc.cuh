@@ -23,8 +23,12 @@
 //            the logit of the target token; the logits never leave the SM.
 //   kEpiDz   backward: recomputes the logits of one vocabulary chunk and
 //            writes dZ = g (onehot(y) - softmax) as bf16.
-//   kEpiF32  plain fp32 store (optionally added to the existing values) with
-//            an optional row map: dH += dZ W and dW = dZ^T H.
+//   kEpiF32  fp32 tile written as is or added to the existing values:
+//            dW = dZ^T H, and dH += dZ W over the compacted rows.
+//   Both write through a tensor map: each epilogue warp stages its 32 rows x
+//   32 columns in shared memory and one lane issues a TMA store (or an L2
+//   reduce-add), so the output leaves the SM as whole 32-row boxes instead of
+//   32 scattered row segments per store instruction.
 //   kEpiSample  the rollout draw o_t ~ softmax(z_t / temperature): per row the
 //            running log-sum-exp of z / temperature and the running argmax of
 //            z / temperature + Gumbel noise (Philox4x32-10, counter = (v / 4, t,
@@ -60,7 +64,6 @@ struct TileCfg {
   static constexpr int kBBytes = kBRows * kBK * 2;      // 32 KB (single) / 16 KB (pair)
   static constexpr int kStageBytes = kABytes + kBBytes;
   static constexpr int kStages = kPair == 2 ? 6 : 4;
-  static constexpr int kSmemBytes = kStages * kStageBytes + 1024 /*align*/ + 256 /*barriers*/;
 };
 
 enum { kEpiLse = 0, kEpiDz = 1, kEpiF32 = 2, kEpiAdam = 3, kEpiSample = 4 };
@@ -75,7 +78,19 @@ struct EpiShape {
   static constexpr int kWarps = kEpi == kEpiSample ? 8 : 4;
   static constexpr int kHalves = kWarps / 4;    // column halves of a tile, one per warp of a quarter
   static constexpr int kThreads = 64 + 32 * kWarps;
+  static constexpr bool kTmaOut = kEpi == kEpiDz || kEpi == kEpiF32;
+  // one warp's 32 x 32 output block in shared memory (bf16 dZ / fp32), two per warp
+  static constexpr int kBlockBytes = kEpi == kEpiDz ? 32 * 32 * 2 : kEpi == kEpiF32 ? 32 * 32 * 4 : 0;
+  static constexpr int kOutBytes = 2 * kBlockBytes * kWarps;
 };
+
+// Dynamic shared memory of one CTA: the operand ring, the output staging
+// blocks (1024-byte aligned, as the output swizzle needs), the barriers.
+template <int kPair, int kEpi>
+constexpr int smem_bytes() {
+  return TileCfg<kPair>::kStages * TileCfg<kPair>::kStageBytes + EpiShape<kEpi>::kOutBytes + 1024 /*align*/ +
+         256 /*barriers*/;
+}
 
 struct GemmArgs {
   const int* n_valid;   // device: number of compacted rows
@@ -99,17 +114,15 @@ struct GemmArgs {
   float* zy;            // [n_heads x ldp] logit of the target
   long ldp;
 
-  // kEpiDz
+  // kEpiDz (output: bf16 through the output tensor map)
   const float* lse;     // [M] natural log-sum-exp of each row
   const float* gcoef;   // [M] dloss/dlogp of each row
-  uint16_t* dz;         // [rows x ldz] bf16 output
-  long ldz;
 
-  // kEpiF32
-  float* out;           // fp32 output
-  long ldo;
-  int accumulate;       // 1: out += acc, 0: out = acc
-  const int* row_map;   // optional: output row of accumulator row r
+  // kEpiF32 (output: fp32 through the output tensor map)
+  int accumulate;       // 1: out += acc (L2 reduce-add), 0: out = acc
+
+  long ldo;             // kEpiAdam: row stride of the weights
+  const int* row_map;   // kEpiSample: token position of each compacted row
 
   // kEpiAdam: the accumulator is a dW tile; an AdamW step is applied to the
   // matching weights in place (row stride ldo) instead of storing dW.
@@ -172,7 +185,7 @@ struct EpiRow {
   bool found;
   int y;
   float lse2, gr;  // kEpiDz
-  int orow;        // kEpiF32; kEpiSample: token position t
+  int orow;        // kEpiSample: token position t
   float best_s, best_z;  // kEpiSample
   int best_c;
 };
@@ -203,8 +216,6 @@ __device__ __forceinline__ void epi_begin(EpiRow& e, const GemmArgs& a, int r, i
       e.lse2 = a.lse[r] * kLog2e;
       e.gr = a.gcoef[r];
     }
-  } else {
-    if (e.rv) e.orow = a.row_map ? a.row_map[r] : r;
   }
 }
 
@@ -215,13 +226,52 @@ __device__ __forceinline__ void adam_update(float g, float& theta, float& m, flo
   theta = theta * a.adam_decay - a.adam_lr * (m * a.adam_bc1) / (sqrtf(v * a.adam_bc2) + a.adam_eps);
 }
 
+// Output staging of one epilogue warp: two 32 x 32 blocks in shared memory,
+// used in turn, and the tensor map of the output.
+struct OutStage {
+  uint32_t smem;             // first block (shared address); the second follows it
+  int count;                 // blocks written so far by this warp
+  const CUtensorMap* map;
+  int lane;
+};
+
+// Writes this warp's 32 x 32 output block (lane = row, `words` = the row's 64
+// bytes of bf16 pairs or 128 bytes of fp32) to global memory at (x, y): the
+// rows go into a shared block in the swizzle the output map declares (64-byte
+// rows in the 64-byte swizzle, 128-byte rows in the 128-byte one: the 16-byte
+// chunk index is XORed with bits 7.. of the offset, which also puts the writes
+// of any 8 consecutive lanes on distinct bank groups), then lane 0 issues a
+// TMA store, or an element-wise add at L2 when `reduce`.
+template <int kWords>
+__device__ __forceinline__ void out_block(OutStage& o, const uint32_t* words, int x, int y, bool reduce) {
+  constexpr int kRowBytes = kWords * 4;
+  const uint32_t buf = o.smem + static_cast<uint32_t>(o.count & 1) * (32 * kRowBytes);
+  // the store issued from this block two blocks ago must have read it
+  if (o.lane == 0) bulk_wait_read_1();
+  __syncwarp();
+  const uint32_t row = buf + static_cast<uint32_t>(o.lane * kRowBytes);
+  const uint32_t sw = kRowBytes == 64 ? (o.lane >> 1) & 3 : o.lane & 7;
+#pragma unroll
+  for (int j = 0; j < kWords / 4; ++j)
+    st_shared_v4(row + 16u * (static_cast<uint32_t>(j) ^ sw), words[4 * j], words[4 * j + 1], words[4 * j + 2],
+                 words[4 * j + 3]);
+  fence_proxy_async_smem();
+  __syncwarp();
+  if (o.lane == 0) {
+    if (reduce) tma_reduce_add_2d(o.map, buf, x, y);
+    else tma_store_2d(o.map, buf, x, y);
+    bulk_commit();
+  }
+  ++o.count;
+}
+
 // One 256-column accumulator tile of this thread's row; `tbase` is the TMEM
-// address of column 0 of the tile in this warp's lane quarter.  Each thread
-// moves its own row with 16-byte vectors (measured faster than transposing
-// 32x32 blocks through shared memory for warp-contiguous scalar accesses).
+// address of column 0 of the tile in this warp's lane quarter; `row0` is the
+// accumulator row of lane 0 (the TMA row coordinate of the warp's block) and
+// m_rows the rows of the output (M).
 template <int kEpi>
 __device__ __forceinline__ void epi_tile(EpiRow& e, const GemmArgs& a, uint32_t tbase, int col0,
-                                         bool have_acc, int half) {
+                                         bool have_acc, int half, OutStage& os, int row0, int m_rows) {
   const float kLog2e = 1.4426950408889634f;
   constexpr int kChunks = kTileN / 32 / EpiShape<kEpi>::kHalves;
 #pragma unroll 1
@@ -306,10 +356,7 @@ __device__ __forceinline__ void epi_tile(EpiRow& e, const GemmArgs& a, uint32_t 
         if (cb + j + 1 >= a.N || !e.rv) d1 = 0.f;
         packed[j / 2] = pack_bf16x2(d0, d1);
       }
-      uint4* dst = reinterpret_cast<uint4*>(a.dz + static_cast<long>(e.r) * a.ldz + cb);
-#pragma unroll
-      for (int q = 0; q < 4; ++q)
-        dst[q] = make_uint4(packed[4 * q], packed[4 * q + 1], packed[4 * q + 2], packed[4 * q + 3]);
+      out_block<16>(os, packed, cb, row0, false);
     } else if (kEpi == kEpiAdam) {
       if (e.rv) {
         const long base = static_cast<long>(e.r) * a.ldo + cb;
@@ -355,27 +402,13 @@ __device__ __forceinline__ void epi_tile(EpiRow& e, const GemmArgs& a, uint32_t 
         }
       }
     } else {
-      if (e.rv) {
-        float* dst = a.out + static_cast<long>(e.orow) * a.ldo + cb;
-        if (cb + 32 <= a.N) {
-          float4* d4 = reinterpret_cast<float4*>(dst);
+      // kEpiF32: a block wholly past M or N is skipped; the tensor map clips
+      // the rest (its rows are the output's M, its columns N)
+      if (row0 < m_rows && cb < a.N) {
+        uint32_t bits[32];
 #pragma unroll
-          for (int q = 0; q < 8; ++q) {
-            float4 o = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
-            if (a.accumulate) {
-              const float4 p = d4[q];
-              o.x += p.x;
-              o.y += p.y;
-              o.z += p.z;
-              o.w += p.w;
-            }
-            d4[q] = o;
-          }
-        } else {
-#pragma unroll
-          for (int j = 0; j < 32; ++j)
-            if (cb + j < a.N) dst[j] = a.accumulate ? dst[j] + v[j] : v[j];
-        }
+        for (int j = 0; j < 32; ++j) bits[j] = __float_as_uint(v[j]);
+        out_block<32>(os, bits, cb, row0, a.accumulate != 0);
       }
     }
   }
@@ -403,12 +436,14 @@ __device__ __forceinline__ void epi_end(const EpiRow& e, const GemmArgs& a, int 
 
 template <int kPair, int kEpi, bool kAmn, bool kBmn>
 __device__ __forceinline__ void gemm_body(const CUtensorMap* tmA, const CUtensorMap* const* tmBs,
-                                          const GemmArgs& args) {
+                                          const CUtensorMap* tmD, const GemmArgs& args) {
   using C = TileCfg<kPair>;
+  using ES = EpiShape<kEpi>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
-  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + C::kStages * C::kStageBytes);
+  uint8_t* out_stage = smem + C::kStages * C::kStageBytes;  // [warps][2] output blocks
+  uint64_t* bars = reinterpret_cast<uint64_t*>(out_stage + ES::kOutBytes);
   uint64_t* full_bar = bars;                          // [kStages] TMA -> MMA (issuing CTA)
   uint64_t* empty_bar = bars + C::kStages;            // [kStages] MMA -> TMA (each CTA)
   uint64_t* tfull_bar = bars + 2 * C::kStages;        // [2] MMA -> epilogue (each CTA)
@@ -440,6 +475,7 @@ __device__ __forceinline__ void gemm_body(const CUtensorMap* tmA, const CUtensor
   if (warp == 0 && lane == 0) {
     tma_prefetch_desc(tmA);
     for (int h = 0; h < args.n_heads; ++h) tma_prefetch_desc(tmBs[h]);
+    if (ES::kTmaOut) tma_prefetch_desc(tmD);
   }
   if (warp == 1) {
     if (kPair == 2) {
@@ -606,6 +642,7 @@ __device__ __forceinline__ void gemm_body(const CUtensorMap* tmA, const CUtensor
     const uint32_t tempty1 = smem_addr(&tempty_bar[1]);
     const uint32_t tempty_c0 = kPair == 2 ? mapa_shared(tempty0, 0) : tempty0;
     const uint32_t tempty_c1 = kPair == 2 ? mapa_shared(tempty1, 0) : tempty1;
+    OutStage os{smem_addr(out_stage) + static_cast<uint32_t>((warp - 2) * 2 * ES::kBlockBytes), 0, tmD, lane};
     int tile = 0;
     bool ok = true;
     for (int u = unit0; u < sch.total && ok; u += unit_stride) {
@@ -616,6 +653,7 @@ __device__ __forceinline__ void gemm_body(const CUtensorMap* tmA, const CUtensor
       const int nt1 = min(sch.n_tiles, nt0 + args.n_per_unit);
       EpiRow e;
       epi_begin<kEpi>(e, args, mt * C::kTileM + row, sch.m_rows);
+      const int row0 = mt * C::kTileM + row - lane;  // accumulator row of lane 0
       for (int nt = nt0; nt < nt1; ++nt) {
         const int buf = tile & 1;
         const uint32_t use = static_cast<uint32_t>(tile >> 1);
@@ -630,7 +668,8 @@ __device__ __forceinline__ void gemm_body(const CUtensorMap* tmA, const CUtensor
           }
           tc_fence_after();
         }
-        epi_tile<kEpi>(e, args, lane_addr + static_cast<uint32_t>(buf * kTileN), nt * kTileN, have_acc, half);
+        epi_tile<kEpi>(e, args, lane_addr + static_cast<uint32_t>(buf * kTileN), nt * kTileN, have_acc, half, os,
+                       row0, sch.m_rows);
         if (have_acc) {
           tc_fence_before();
           __syncwarp();
@@ -645,6 +684,8 @@ __device__ __forceinline__ void gemm_body(const CUtensorMap* tmA, const CUtensor
       epi_end<kEpi>(e, args, un, head, half);
     }
     if (!ok) raise_abort();
+    // the output boxes in flight read shared memory and must land before exit
+    if (ES::kTmaOut && lane == 0) bulk_wait_all();
   }
 
   // After a timeout, give copies that may still be in flight time to land
@@ -664,18 +705,20 @@ template <int kEpi, bool kAmn, bool kBmn>
 __global__ void __launch_bounds__(EpiShape<kEpi>::kThreads, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB0,
                    const __grid_constant__ CUtensorMap tmB1, const __grid_constant__ CUtensorMap tmB2,
-                   const __grid_constant__ CUtensorMap tmB3, const GemmArgs args) {
+                   const __grid_constant__ CUtensorMap tmB3, const __grid_constant__ CUtensorMap tmD,
+                   const GemmArgs args) {
   const CUtensorMap* tmBs[kMaxHeads] = {&tmB0, &tmB1, &tmB2, &tmB3};
-  gemm_body<1, kEpi, kAmn, kBmn>(&tmA, tmBs, args);
+  gemm_body<1, kEpi, kAmn, kBmn>(&tmA, tmBs, &tmD, args);
 }
 
 template <int kEpi, bool kAmn, bool kBmn>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(EpiShape<kEpi>::kThreads, 1)
     gemm_tc_pair_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB0,
                         const __grid_constant__ CUtensorMap tmB1, const __grid_constant__ CUtensorMap tmB2,
-                        const __grid_constant__ CUtensorMap tmB3, const GemmArgs args) {
+                        const __grid_constant__ CUtensorMap tmB3, const __grid_constant__ CUtensorMap tmD,
+                        const GemmArgs args) {
   const CUtensorMap* tmBs[kMaxHeads] = {&tmB0, &tmB1, &tmB2, &tmB3};
-  gemm_body<2, kEpi, kAmn, kBmn>(&tmA, tmBs, args);
+  gemm_body<2, kEpi, kAmn, kBmn>(&tmA, tmBs, &tmD, args);
 }
 
 }  // namespace grpo

@@ -42,7 +42,7 @@ int64_t vocab_chunk(int64_t V) {
 struct Layout {
   int64_t T_pad, nsplit, nblk_scan, nblk_loss, vchunk;
   size_t status, n_valid, counts, offsets, cidx, rank_of, yc, zy, part_m, part_s, lse_c, g_c,
-      block_loss, resp_len, best_s, best_c, best_z, Hc, dz, total;
+      block_loss, resp_len, best_s, best_c, best_z, Hc, dz, dhc, total;
 };
 
 bool make_layout(int64_t T, int32_t Hd, int64_t V, int32_t which, Layout* L) {
@@ -88,6 +88,8 @@ bool make_layout(int64_t T, int32_t Hd, int64_t V, int32_t which, Layout* L) {
   L->best_z = take(best, 256);
   L->Hc = take(2 * tp * static_cast<size_t>(Hd), 1024);
   L->dz = which == GRPO_WS_LOSS ? take(2 * tp * static_cast<size_t>(L->vchunk), 1024) : off;
+  // dH over the compacted rows, accumulated across vocabulary chunks
+  L->dhc = which == GRPO_WS_LOSS ? take(4 * tp * static_cast<size_t>(Hd), 1024) : off;
   L->total = (off + 1023) / 1024 * 1024;
   return true;
 }
@@ -112,16 +114,19 @@ bool get_encode() {
 // 2D bf16 tensor map over a row-major [rows x cols] matrix; the box is
 // box_cols (inner, 64 = 128 bytes) x box_rows with the 128-byte swizzle.
 // Out-of-range elements of a box read as zero.
+// A 2-D tensor map over a row-major matrix [rows x cols] (leading dimension
+// ld elements): bf16 operands in the 128-byte swizzle by default; the output
+// maps of the epilogue use fp32 / the 64-byte swizzle as their boxes need.
 bool encode_2d(CUtensorMap* map, const void* base, uint64_t rows, uint64_t cols, uint64_t ld_elems,
-               uint32_t box_cols, uint32_t box_rows) {
+               uint32_t box_cols, uint32_t box_rows, bool f32 = false,
+               CUtensorMapSwizzle swizzle = CU_TENSOR_MAP_SWIZZLE_128B) {
   const cuuint64_t dims[2] = {cols, rows};
-  const cuuint64_t strides[1] = {ld_elems * 2};
+  const cuuint64_t strides[1] = {ld_elems * (f32 ? 4 : 2)};
   const cuuint32_t box[2] = {box_cols, box_rows};
   const cuuint32_t estr[2] = {1, 1};
-  const CUresult r = g_encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims,
-                              strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
-                              CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-                              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  const CUresult r = g_encode(map, f32 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2,
+                              const_cast<void*>(base), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                              swizzle, CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   return r == CUDA_SUCCESS;
 }
 
@@ -134,14 +139,14 @@ struct DeviceInfo {
 template <int E, bool A, bool B>
 bool prepare_kernels(int* pairs) {
   if (cudaFuncSetAttribute(gemm_tc_kernel<E, A, B>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                           TileCfg<1>::kSmemBytes) != cudaSuccess ||
+                           smem_bytes<1, E>()) != cudaSuccess ||
       cudaFuncSetAttribute(gemm_tc_pair_kernel<E, A, B>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                           TileCfg<2>::kSmemBytes) != cudaSuccess)
+                           smem_bytes<2, E>()) != cudaSuccess)
     return false;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(2 * 1024, 1, 1);
   cfg.blockDim = dim3(EpiShape<E>::kThreads, 1, 1);
-  cfg.dynamicSmemBytes = TileCfg<2>::kSmemBytes;
+  cfg.dynamicSmemBytes = smem_bytes<2, E>();
   int n = 0;
   if (cudaOccupancyMaxActiveClusters(&n, gemm_tc_pair_kernel<E, A, B>, &cfg) != cudaSuccess) {
     cudaGetLastError();  // clear: without the query the single-CTA tiles are used
@@ -318,23 +323,43 @@ CopyOut* copy_out_for_device() {
   return per_dev[dev]->ok ? per_dev[dev] : nullptr;
 }
 
+bool aligned(const void* p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
+
 // A bf16 row-major matrix [rows x cols] with leading dimension ld (elements).
 struct Operand {
   const void* base;
   uint64_t rows, cols, ld;
 };
 
-// Builds the tensor maps of A and of each B (one per LM head; a.n_heads of
-// them) for the tile shape of kPair and launches the persistent GEMM with at
-// most one CTA (pair) per work unit.
+// The output of a kEpiDz (bf16) or kEpiF32 (fp32) GEMM: a row-major matrix
+// [rows x cols], leading dimension ld elements; accumulator row r, column n
+// lands at (r, n), and what lies outside rows x cols is not written.
+struct OutMat {
+  void* base;
+  uint64_t rows, cols, ld;
+};
+
+// Builds the tensor maps of A, of each B (one per LM head; a.n_heads of them)
+// and of the output D for the tile shape of kPair and launches the persistent
+// GEMM with at most one CTA (pair) per work unit.
 template <int kPair, int E, bool AMN, bool BMN>
 cudaError_t launch_gemm_cfg(const Operand& A, const Operand* B, const GemmArgs& args, int64_t max_m_rows,
-                            const DeviceInfo& di, cudaStream_t s) {
+                            const DeviceInfo& di, cudaStream_t s, const OutMat* D) {
   using C = TileCfg<kPair>;
   GemmArgs a = args;
   a.n_heads = std::max(1, std::min(a.n_heads, kMaxHeads));
-  CUtensorMap ta, tb[kMaxHeads];
+  CUtensorMap ta, tb[kMaxHeads], td;
   if (!encode_2d(&ta, A.base, A.rows, A.cols, A.ld, kBK, AMN ? 64 : kRowsCta)) return cudaErrorInvalidValue;
+  if (EpiShape<E>::kTmaOut) {
+    // 32 x 32 boxes: 64-byte bf16 rows in the 64-byte swizzle, 128-byte fp32 rows in the 128-byte one
+    const bool f32 = E == kEpiF32;
+    if (!D || !aligned(D->base, 16) ||
+        !encode_2d(&td, D->base, D->rows, D->cols, D->ld, 32, 32, f32,
+                   f32 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_64B))
+      return cudaErrorInvalidValue;
+  } else {
+    td = ta;  // not read
+  }
   for (int h = 0; h < kMaxHeads; ++h) {
     if (h >= a.n_heads) {
       tb[h] = tb[0];
@@ -348,28 +373,27 @@ cudaError_t launch_gemm_cfg(const Operand& A, const Operand* B, const GemmArgs& 
                         ((n_tiles + a.n_per_unit - 1) / a.n_per_unit) * a.n_heads;
   if (kPair == 2) {
     const int64_t pairs = std::max<int64_t>(1, std::min<int64_t>(di.pairs, units));
-    gemm_tc_pair_kernel<E, AMN, BMN><<<static_cast<unsigned>(2 * pairs), EpiShape<E>::kThreads, C::kSmemBytes,
-                                       s>>>(
-        ta, tb[0], tb[1], tb[2], tb[3], a);
+    gemm_tc_pair_kernel<E, AMN, BMN><<<static_cast<unsigned>(2 * pairs), EpiShape<E>::kThreads,
+                                       smem_bytes<2, E>(), s>>>(ta, tb[0], tb[1], tb[2], tb[3], td, a);
   } else {
     const int64_t grid = std::max<int64_t>(1, std::min<int64_t>(di.sms, units));
-    gemm_tc_kernel<E, AMN, BMN><<<static_cast<unsigned>(grid), EpiShape<E>::kThreads, C::kSmemBytes, s>>>(
-        ta, tb[0], tb[1], tb[2], tb[3], a);
+    gemm_tc_kernel<E, AMN, BMN><<<static_cast<unsigned>(grid), EpiShape<E>::kThreads, smem_bytes<1, E>(), s>>>(
+        ta, tb[0], tb[1], tb[2], tb[3], td, a);
   }
   return cudaGetLastError();
 }
 
 template <int E, bool AMN, bool BMN>
 cudaError_t launch_gemm(const Operand& A, const Operand* B, const GemmArgs& a, int64_t max_m_rows,
-                        const DeviceInfo& di, cudaStream_t s) {
-  return use_pairs() && di.pairs > 0 ? launch_gemm_cfg<2, E, AMN, BMN>(A, B, a, max_m_rows, di, s)
-                                     : launch_gemm_cfg<1, E, AMN, BMN>(A, B, a, max_m_rows, di, s);
+                        const DeviceInfo& di, cudaStream_t s, const OutMat* D = nullptr) {
+  return use_pairs() && di.pairs > 0 ? launch_gemm_cfg<2, E, AMN, BMN>(A, B, a, max_m_rows, di, s, D)
+                                     : launch_gemm_cfg<1, E, AMN, BMN>(A, B, a, max_m_rows, di, s, D);
 }
 
 template <int E, bool AMN, bool BMN>
 cudaError_t launch_gemm(const Operand& A, const Operand& B, const GemmArgs& a, int64_t max_m_rows,
-                        const DeviceInfo& di, cudaStream_t s) {
-  return launch_gemm<E, AMN, BMN>(A, &B, a, max_m_rows, di, s);
+                        const DeviceInfo& di, cudaStream_t s, const OutMat* D = nullptr) {
+  return launch_gemm<E, AMN, BMN>(A, &B, a, max_m_rows, di, s, D);
 }
 
 template <typename T>
@@ -377,7 +401,6 @@ T* at(void* ws, size_t off) {
   return reinterpret_cast<T*>(static_cast<char*>(ws) + off);
 }
 
-bool aligned(const void* p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
 
 // Compaction of unmasked rows + gather of their hidden states and targets.
 cudaError_t run_compaction(const uint16_t* H, const int32_t* targets, const uint8_t* mask, int64_t T,
@@ -752,12 +775,6 @@ grpo_status loss_impl(const uint16_t* H, const uint16_t* W, const int32_t* targe
     loss_final_kernel<<<1, 1024, 0, s>>>(at<double>(ws, Ly.block_loss), n_valid, kLossThreads, loss_out);
     e = cudaGetLastError();
   }
-  if (e == cudaSuccess) {
-    TraceScope trace(GRPO_K_ZERO_ROWS, 0, s);
-    const int zb = static_cast<int>(std::min<int64_t>((T + 7) / 8, sms * 8));
-    zero_masked_rows_kernel<<<zb, 256, 0, s>>>(mask, T, Hd, dH);
-    e = cudaGetLastError();
-  }
   if (e != cudaSuccess) return from_cuda(e);
 
   // Backward, one vocabulary chunk at a time.  With dW_host, each finished dW
@@ -773,11 +790,14 @@ grpo_status loss_impl(const uint16_t* H, const uint16_t* W, const int32_t* targe
   int chunk = 0;
   uint16_t* Hc = at<uint16_t>(ws, Ly.Hc);
   uint16_t* dz = at<uint16_t>(ws, Ly.dz);
+  float* dHc = at<float>(ws, Ly.dhc);
   const int64_t vc = Ly.vchunk;
   const uint64_t tp = static_cast<uint64_t>(Ly.T_pad), hd = static_cast<uint64_t>(Hd);
   const Operand opHc{Hc, tp, hd, hd};
   const Operand opW{W, static_cast<uint64_t>(V), hd, hd};
   const Operand opDz{dz, tp, static_cast<uint64_t>(vc), static_cast<uint64_t>(vc)};
+  const OutMat outDz{dz, tp, static_cast<uint64_t>(vc), static_cast<uint64_t>(vc)};
+  const OutMat outDh{dHc, tp, hd, hd};
   for (int64_t c0 = 0; c0 < V && e == cudaSuccess; c0 += vc) {
     const int64_t width = std::min<int64_t>(vc, V - c0);
     {  // dZ chunk = g (onehot - softmax) from recomputed logits
@@ -794,13 +814,11 @@ grpo_status loss_impl(const uint16_t* H, const uint16_t* W, const int32_t* targe
       a.yc = at<int>(ws, Ly.yc);
       a.lse = at<float>(ws, Ly.lse_c);
       a.gcoef = at<float>(ws, Ly.g_c);
-      a.dz = dz;
-      a.ldz = vc;
       TraceScope trace(GRPO_K_DZ_GEMM, width, s);
-      e = launch_gemm<kEpiDz, false, false>(opHc, opW, a, Ly.T_pad, di, s);
+      e = launch_gemm<kEpiDz, false, false>(opHc, opW, a, Ly.T_pad, di, s, &outDz);
     }
     if (e != cudaSuccess) break;
-    {  // dH (+)= dZ_c W_c
+    {  // dHc (+)= dZ_c W_c: stored by the first chunk, added at L2 by the others
       GemmArgs h{};
       h.n_valid = n_valid;
       h.m_dyn = 1;
@@ -811,12 +829,9 @@ grpo_status loss_impl(const uint16_t* H, const uint16_t* W, const int32_t* targe
       h.group_m = group_m(2, di);
       l2_hints(2, &h.a_hint, &h.b_hint);
       h.status = status;
-      h.out = dH;
-      h.ldo = Hd;
       h.accumulate = c0 > 0;
-      h.row_map = at<int>(ws, Ly.cidx);
       TraceScope trace(GRPO_K_DH_GEMM, width, s);
-      e = launch_gemm<kEpiF32, false, true>(opDz, opW, h, Ly.T_pad, di, s);
+      e = launch_gemm<kEpiF32, false, true>(opDz, opW, h, Ly.T_pad, di, s, &outDh);
     }
     if (e != cudaSuccess) break;
     {  // dW_c = dZ_c^T Hc (stored, or consumed by the AdamW step)
@@ -829,9 +844,9 @@ grpo_status loss_impl(const uint16_t* H, const uint16_t* W, const int32_t* targe
       w.group_m = group_m(3, di);
       l2_hints(3, &w.a_hint, &w.b_hint);
       w.status = status;
-      w.out = dW + c0 * Hd;
       w.ldo = Hd;
       w.accumulate = 0;
+      const OutMat outDw{dW + c0 * Hd, static_cast<uint64_t>(width), hd, hd};
       TraceScope trace(GRPO_K_DW_GEMM, width, s);
       if (adam) {
         const int64_t off = c0 * Hd;
@@ -848,7 +863,7 @@ grpo_status loss_impl(const uint16_t* H, const uint16_t* W, const int32_t* targe
         w.adam_bc2 = adam->bc2;
         e = launch_gemm<kEpiAdam, true, true>(opDz, opHc, w, width, di, s);
       } else {
-        e = launch_gemm<kEpiF32, true, true>(opDz, opHc, w, width, di, s);
+        e = launch_gemm<kEpiF32, true, true>(opDz, opHc, w, width, di, s, &outDw);
       }
     }
     if (e == cudaSuccess && co) {
@@ -860,6 +875,12 @@ grpo_status loss_impl(const uint16_t* H, const uint16_t* W, const int32_t* targe
                             cudaMemcpyDeviceToHost, co->stream);
     }
     ++chunk;
+  }
+  if (e == cudaSuccess) {  // dH rows to their padded positions, padding rows 0
+    TraceScope trace(GRPO_K_DH_ROWS, 0, s);
+    const int rb = static_cast<int>(std::min<int64_t>((T + 7) / 8, sms * 8));
+    dh_rows_kernel<<<rb, 256, 0, s>>>(at<int>(ws, Ly.rank_of), T, Hd, dHc, dH);
+    e = cudaGetLastError();
   }
   if (co && e == cudaSuccess) {
     e = cudaEventRecord(co->done, co->stream);

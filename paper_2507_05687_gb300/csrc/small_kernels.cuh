@@ -386,16 +386,22 @@ __global__ void adamw_kernel(float* __restrict__ theta, float* __restrict__ m, f
   }
 }
 
-// dH rows of padding tokens are 0 (the GEMM only writes unmasked rows).
-__global__ void zero_masked_rows_kernel(const uint8_t* __restrict__ mask, int64_t T, int Hd,
-                                        float* __restrict__ dH) {
+// dH[t] = dHc[rank_of[t]] for unmasked rows, 0 for padding rows: one warp per
+// row, 16-byte accesses (the compacted rows are read once).
+__global__ void dh_rows_kernel(const int* __restrict__ rank_of, int64_t T, int Hd, const float* __restrict__ dHc,
+                               float* __restrict__ dH) {
   const int lane = threadIdx.x & 31;
   const int vec = Hd / 4;
   for (int64_t t = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5; t < T;
        t += (static_cast<int64_t>(gridDim.x) * blockDim.x) >> 5) {
-    if (mask[t]) continue;
+    const int r = rank_of[t];
     float4* row = reinterpret_cast<float4*>(dH + t * Hd);
-    for (int j = lane; j < vec; j += 32) row[j] = make_float4(0.f, 0.f, 0.f, 0.f);
+    if (r < 0) {
+      for (int j = lane; j < vec; j += 32) row[j] = make_float4(0.f, 0.f, 0.f, 0.f);
+    } else {
+      const float4* src = reinterpret_cast<const float4*>(dHc + static_cast<int64_t>(r) * Hd);
+      for (int j = lane; j < vec; j += 32) row[j] = __ldcs(src + j);
+    }
   }
 }
 
