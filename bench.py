@@ -38,7 +38,7 @@ GOLDEN = {"fwdbwd_8b": "batch8b", "logprob3_8b": "batch8b", "long_8b": "long_8b"
 KERNEL_SOURCES = ["paper_2507_05687_gb300/csrc/gemm_tc.cuh", "paper_2507_05687_gb300/csrc/ptx.cuh",
                   "paper_2507_05687_gb300/csrc/grpo_api.cu"]
 KIND_NAMES = ["advantages", "compact", "lse_gemm", "logp_merge", "loss", "dz_gemm", "dh_gemm", "dw_gemm",
-              "dh_rows", "adamw", "sample_gemm"]
+              "dh_rows", "adamw", "sample_gemm", "transpose"]
 KERNELS_PER_SCOPE = {1: 4, 4: 2}  # compaction scope = 4 kernels, loss scope = 2 kernels; others 1
 
 

@@ -307,7 +307,8 @@ enum {
   GRPO_K_DW_GEMM = 7,     /* dW_chunk = dZ_chunk^T H */
   GRPO_K_DH_ROWS = 8,     /* dH rows from the compacted order to the padded one (padding rows 0) */
   GRPO_K_ADAMW = 9,       /* standalone AdamW step (grpo_adamw_step) */
-  GRPO_K_SAMPLE_GEMM = 10 /* logits GEMM + log-sum-exp + Gumbel-max draw */
+  GRPO_K_SAMPLE_GEMM = 10, /* logits GEMM + log-sum-exp + Gumbel-max draw */
+  GRPO_K_TRANSPOSE = 11   /* K-major (transposed) copy of the gathered hidden states for dW */
 };
 
 /*

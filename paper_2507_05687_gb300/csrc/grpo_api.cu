@@ -42,7 +42,7 @@ int64_t vocab_chunk(int64_t V) {
 struct Layout {
   int64_t T_pad, nsplit, nblk_scan, nblk_loss, vchunk;
   size_t status, n_valid, counts, offsets, cidx, rank_of, yc, zy, part_m, part_s, lse_c, g_c,
-      block_loss, resp_len, best_s, best_c, best_z, Hc, dz, dhc, total;
+      block_loss, resp_len, best_s, best_c, best_z, Hc, HcT, dz, dhc, total;
 };
 
 bool make_layout(int64_t T, int32_t Hd, int64_t V, int32_t which, Layout* L) {
@@ -87,6 +87,8 @@ bool make_layout(int64_t T, int32_t Hd, int64_t V, int32_t which, Layout* L) {
   L->best_c = take(best, 256);
   L->best_z = take(best, 256);
   L->Hc = take(2 * tp * static_cast<size_t>(Hd), 1024);
+  // H_c transposed [Hd x T_pad]: the K-major B operand of the dW GEMM
+  L->HcT = which == GRPO_WS_LOSS ? take(2 * tp * static_cast<size_t>(Hd), 1024) : off;
   L->dz = which == GRPO_WS_LOSS ? take(2 * tp * static_cast<size_t>(L->vchunk), 1024) : off;
   // dH over the compacted rows, accumulated across vocabulary chunks
   L->dhc = which == GRPO_WS_LOSS ? take(4 * tp * static_cast<size_t>(Hd), 1024) : off;
@@ -171,7 +173,7 @@ bool device_info(DeviceInfo* out) {
       return false;
     if (major != 10 || minor != 3) return false;
     if (!prepare_kernels<kEpiLse, false, false>(&pairs) || !prepare_kernels<kEpiDz, false, false>(&pairs) ||
-        !prepare_kernels<kEpiF32, false, true>(&pairs) || !prepare_kernels<kEpiF32, true, true>(&pairs) ||
+        !prepare_kernels<kEpiF32, false, true>(&pairs) || !prepare_kernels<kEpiF32, true, false>(&pairs) ||
         !prepare_kernels<kEpiAdam, true, true>(&pairs) || !prepare_kernels<kEpiSample, false, false>(&pairs))
       return false;
     cache[dev].sms = sms;
@@ -764,6 +766,13 @@ grpo_status loss_impl(const uint16_t* H, const uint16_t* W, const int32_t* targe
     resp_len_kernel<<<static_cast<unsigned>(blocks), 256, 0, s>>>(mask, n_resp, L, at<int>(ws, Ly.resp_len));
     e = cudaGetLastError();
   }
+  if (e == cudaSuccess && !adam) {
+    TraceScope trace(GRPO_K_TRANSPOSE, 0, s);
+    const int tb = static_cast<int>(std::min<int64_t>(Ly.T_pad / 64 * (Hd / 64), int64_t(sms) * 8));
+    transpose_rows_kernel<<<tb, 256, 0, s>>>(at<uint16_t>(ws, Ly.Hc), n_valid, Hd, Ly.T_pad,
+                                             at<uint16_t>(ws, Ly.HcT));
+    e = cudaGetLastError();
+  }
   if (e == cudaSuccess) e = run_lse(&W, 1, Hd, V, ws, Ly, di, s);
   if (e == cudaSuccess) {
     TraceScope trace(GRPO_K_LOSS, 0, s);
@@ -794,6 +803,7 @@ grpo_status loss_impl(const uint16_t* H, const uint16_t* W, const int32_t* targe
   const int64_t vc = Ly.vchunk;
   const uint64_t tp = static_cast<uint64_t>(Ly.T_pad), hd = static_cast<uint64_t>(Hd);
   const Operand opHc{Hc, tp, hd, hd};
+  const Operand opHcT{at<uint16_t>(ws, Ly.HcT), hd, tp, tp};
   const Operand opW{W, static_cast<uint64_t>(V), hd, hd};
   const Operand opDz{dz, tp, static_cast<uint64_t>(vc), static_cast<uint64_t>(vc)};
   const OutMat outDz{dz, tp, static_cast<uint64_t>(vc), static_cast<uint64_t>(vc)};
@@ -863,7 +873,7 @@ grpo_status loss_impl(const uint16_t* H, const uint16_t* W, const int32_t* targe
         w.adam_bc2 = adam->bc2;
         e = launch_gemm<kEpiAdam, true, true>(opDz, opHc, w, width, di, s);
       } else {
-        e = launch_gemm<kEpiF32, true, true>(opDz, opHc, w, width, di, s, &outDw);
+        e = launch_gemm<kEpiF32, true, false>(opDz, opHcT, w, width, di, s, &outDw);
       }
     }
     if (e == cudaSuccess && co) {

@@ -386,6 +386,40 @@ __global__ void adamw_kernel(float* __restrict__ theta, float* __restrict__ m, f
   }
 }
 
+// HcT[k][r] = Hc[r][k] for r < round_up(n_valid, 256) (the rows the token
+// K-loop of the dW GEMM can reach, zero past n_valid): the K-major copy of the
+// gathered hidden states.  64 x 64 tiles through shared memory, 32-bit words
+// (two bf16) on both the read and the write side.
+__global__ void transpose_rows_kernel(const uint16_t* __restrict__ Hc, const int* __restrict__ n_valid_p, int Hd,
+                                      int64_t ld_t, uint16_t* __restrict__ HcT) {
+  __shared__ uint16_t tile[64][66];
+  const int nv = *n_valid_p;
+  const int rows = (nv + 255) / 256 * 256;
+  const int col_tiles = Hd / 64;
+  const int64_t tiles = static_cast<int64_t>(rows / 64) * col_tiles;
+  const int w = threadIdx.x & 31;
+  const int q = threadIdx.x >> 5;  // 0..7
+  for (int64_t i = blockIdx.x; i < tiles; i += gridDim.x) {
+    const int r0 = static_cast<int>(i / col_tiles) * 64;
+    const int c0 = static_cast<int>(i % col_tiles) * 64;
+#pragma unroll
+    for (int k = 0; k < 8; ++k) {  // rows r0 + q + 8k, columns c0 + 2w, 2w + 1
+      const int r = q + 8 * k;
+      const uint32_t v = *reinterpret_cast<const uint32_t*>(Hc + static_cast<int64_t>(r0 + r) * Hd + c0 + 2 * w);
+      tile[r][2 * w] = static_cast<uint16_t>(v & 0xFFFFu);
+      tile[r][2 * w + 1] = static_cast<uint16_t>(v >> 16);
+    }
+    __syncthreads();
+#pragma unroll
+    for (int k = 0; k < 8; ++k) {  // output rows c0 + q + 8k, columns r0 + 2w, 2w + 1
+      const int c = q + 8 * k;
+      const uint32_t v = static_cast<uint32_t>(tile[2 * w][c]) | (static_cast<uint32_t>(tile[2 * w + 1][c]) << 16);
+      *reinterpret_cast<uint32_t*>(HcT + static_cast<int64_t>(c0 + c) * ld_t + r0 + 2 * w) = v;
+    }
+    __syncthreads();
+  }
+}
+
 // dH[t] = dHc[rank_of[t]] for unmasked rows, 0 for padding rows: one warp per
 // row, 16-byte accesses (the compacted rows are read once).
 __global__ void dh_rows_kernel(const int* __restrict__ rank_of, int64_t T, int Hd, const float* __restrict__ dHc,
