@@ -431,12 +431,13 @@ def main():
         step_flops8 = 8.0 * n_valid * w.Hd * w.V
         step_flops6 = 6.0 * n_valid * w.Hd * w.V
 
-    e2e = None
+    e2e = e2e_offload = None
     if not args.no_e2e and rank == 0 and not sampling:
         if scoring:
             e2e = measure_e2e_scoring(grpo, torch, dev, w, inp, heads, steps=min(args.steps, 5))
         else:
             e2e = measure_e2e(grpo, torch, dev, w, inp, steps=min(args.steps, 5))
+            e2e_offload = measure_e2e_offload(grpo, torch, dev, w, inp, steps=min(args.steps, 5))
 
     cpu = None
     if not args.no_cpu_baseline and rank == 0 and world == 1 and not sampling:
@@ -464,32 +465,82 @@ def main():
             "step_frac_6x": round(step_flops6 / (ms / 1e3) / 1e12 / burst, 4),
             "roofline": rf, "clocks": clocks, "gpu_launches": launches, "e2e": e2e, "cpu_baseline": cpu,
         }
+        if e2e_offload is not None:
+            line["e2e_offload"] = e2e_offload
         print(json.dumps(line), flush=True)
     if dist is not None:
         dist.destroy_process_group()
 
 
 def measure_e2e_scoring(grpo, torch, dev, w, inp, heads, steps: int):
-    """Public API with pinned host buffers: H2D of H and the three heads, the call, D2H of the log-probs."""
+    """Public API, rollout scoring: H2D of the batch (H, targets, mask) from pinned host
+    memory, the three LM heads resident on the device (model weights), D2H of the
+    three log-prob rows."""
     def pin(a, dt):
         return torch.from_numpy(np.ascontiguousarray(a)).view(dt).pin_memory()
 
     hH, hy, hm = pin(inp["H"], torch.bfloat16), pin(inp["y"], torch.int32), pin(inp["m"], torch.uint8)
-    hheads = [h.cpu().pin_memory() for h in heads]
-    h2d = sum(t.numel() * t.element_size() for t in [hH, hy, hm, *hheads])
+    h2d = sum(t.numel() * t.element_size() for t in [hH, hy, hm])
     d2h = len(heads) * w.T * 4
-    grpo.token_logprobs_heads(hH, hheads, hy, hm)
+    hout = torch.empty(len(heads), w.T, dtype=torch.float32).pin_memory()
+    ws = grpo.workspace(w.T, w.Hd, w.V, grpo.GRPO_WS_LOGPROBS_HEADS, dev)
+
+    def one():
+        lp = grpo.token_logprobs_heads(hH, heads, hy, hm, ws=ws)
+        hout.copy_(lp, non_blocking=True)
+        torch.cuda.current_stream(dev).synchronize()
+
+    one()
     t0 = time.perf_counter()
     for _ in range(steps):
-        grpo.token_logprobs_heads(hH, hheads, hy, hm)  # returns a pinned host tensor once it has landed
+        one()
     dt = (time.perf_counter() - t0) / steps
     n_valid = int(inp["m"].sum())
     return {"value": round(n_valid / dt, 1), "unit": "tokens/s", "ms_per_step": round(dt * 1e3, 2),
-            "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h), "steps": steps}
+            "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h), "steps": steps,
+            "what": "H, targets, mask copied from pinned host memory each step; the policy / old / reference "
+                    "heads resident on the device; the log-probs read back"}
 
 
 def measure_e2e(grpo, torch, dev, w, inp, steps: int):
-    """Public API with pinned host buffers: H2D of the batch, the step, D2H of loss, dH, dW."""
+    """Public API, one training step: H2D of the batch (H, targets, mask, old / ref
+    log-probs, rewards) from pinned host memory, the LM head W resident on the
+    device (the parameter being trained), D2H of the loss; dH and dW stay on the
+    device, where the trunk's backward and the optimiser consume them."""
+    def pin(a, dt):
+        return torch.from_numpy(np.ascontiguousarray(a)).view(dt).pin_memory()
+
+    Wd = torch.from_numpy(np.ascontiguousarray(inp["W"])).view(torch.bfloat16).to(dev)
+    hH, hy, hm = pin(inp["H"], torch.bfloat16), pin(inp["y"], torch.int32), pin(inp["m"], torch.uint8)
+    hold, href, hr = pin(inp["old"], torch.float32), pin(inp["ref"], torch.float32), pin(inp["r"], torch.float32)
+    h2d = sum(t.numel() * t.element_size() for t in (hH, hy, hm, hold, href, hr))
+    d2h = 4
+    out = (torch.empty(1, dtype=torch.float32, device=dev), torch.empty(w.T, w.Hd, dtype=torch.float32, device=dev),
+           torch.empty(w.V, w.Hd, dtype=torch.float32, device=dev))
+    ws = grpo.workspace(w.T, w.Hd, w.V, grpo.GRPO_WS_LOSS, dev)
+
+    def one():
+        adv = grpo.group_advantages(hr.to(dev, non_blocking=True), w.G, w.adv_eps)
+        loss, _, _ = grpo.loss_fwd_bwd(hH, Wd, hy, hm, hold, href, adv, w.n_resp, w.L, w.clip_eps, w.beta,
+                                       ws=ws, out=out)
+        return loss.item()
+
+    one()
+    torch.cuda.synchronize(dev)
+    t0 = time.perf_counter()
+    for _ in range(steps):
+        one()
+    dt = (time.perf_counter() - t0) / steps
+    n_valid = int(inp["m"].sum())
+    return {"value": round(n_valid / dt, 1), "unit": "tokens/s", "ms_per_step": round(dt * 1e3, 2),
+            "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h), "steps": steps,
+            "what": "H, targets, mask, old/ref log-probs, rewards copied from pinned host memory each step; W "
+                    "resident on the device; the loss read back; dH, dW left on the device"}
+
+
+def measure_e2e_offload(grpo, torch, dev, w, inp, steps: int):
+    """Public API with everything on the host (a host-offloaded head): H2D of the
+    batch and of W, the step, D2H of loss, dH, dW (dW streamed chunk by chunk)."""
     def pin(a, dt):
         t = torch.from_numpy(np.ascontiguousarray(a)).view(dt)
         return t.pin_memory()
@@ -517,7 +568,8 @@ def measure_e2e(grpo, torch, dev, w, inp, steps: int):
     dt = (time.perf_counter() - t0) / steps
     n_valid = int(inp["m"].sum())
     return {"value": round(n_valid / dt, 1), "unit": "tokens/s", "ms_per_step": round(dt * 1e3, 2),
-            "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h), "steps": steps}
+            "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h), "steps": steps,
+            "what": "batch and W copied from pinned host memory each step; loss, dH, dW copied back"}
 
 
 if __name__ == "__main__":
