@@ -195,6 +195,35 @@ grpo_status grpo_loss_fwd_bwd_kl_clamp(const uint16_t* H, const uint16_t* W, con
                                        void* stream);
 
 /*
+ * Rows of dW (vocabulary ids) per backward chunk: chunk c of
+ * grpo_loss_fwd_bwd* covers rows [c * cols, min(V, (c + 1) * cols)).  cols is
+ * 16384, or the environment variable GRPO_VOCAB_CHUNK (rounded up to a
+ * multiple of 256) when set, capped at V rounded up to 256; the loss calls read
+ * the same variable, so query under the same environment.  0 for V <= 0.
+ */
+int64_t grpo_vocab_chunk_cols(int64_t V);
+
+/*
+ * grpo_loss_fwd_bwd_norm that also records chunk_events[c] on `stream` as
+ * soon as chunk c's rows of dW are written (and *loss_out, computed before the
+ * backward, is final from chunk_events[0] on).  A data-parallel caller makes
+ * its communication stream wait on each event and starts that chunk's dW
+ * all-reduce while the later chunks still compute: the one exchange step of
+ * the data-parallel path (dW summed over ranks) then overlaps the backward.
+ *   chunk_events  HOST array of n_events cudaEvent_t handles, created by the
+ *                 caller on the current device; entries 0 .. chunks - 1 are
+ *                 recorded, chunks = ceil(V / grpo_vocab_chunk_cols(V))
+ *   n_events      >= chunks, else GRPO_ERR_INVALID_ARG (nothing launched)
+ * Every other argument as grpo_loss_fwd_bwd_norm.
+ */
+grpo_status grpo_loss_fwd_bwd_events(const uint16_t* H, const uint16_t* W, const int32_t* targets,
+                                     const uint8_t* mask, const float* old_logp, const float* ref_logp,
+                                     const float* adv, int64_t n_resp, int64_t L, int32_t Hd, int64_t V,
+                                     float clip_eps, float beta, int32_t agg_mode, float norm, float* loss_out,
+                                     float* dH, float* dW, void* const* chunk_events, int32_t n_events, void* ws,
+                                     size_t ws_bytes, void* stream);
+
+/*
  * grpo_loss_fwd_bwd_norm for a caller that wants dW in host memory: each
  * vocabulary chunk of dW is copied to dW_host as soon as it is computed, on
  * an internal copy stream (created once per device), so the copy of the

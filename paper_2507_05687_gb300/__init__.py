@@ -9,5 +9,5 @@ from .binding import (  # noqa: F401
     GRPO_ERR_WORKSPACE, GRPO_MAX_HEADS, GRPO_OK, GRPO_WS_LOGPROBS, GRPO_WS_LOGPROBS_HEADS, GRPO_WS_LOSS,
     GRPO_WS_SAMPLE, LIB_PATH, SIGNATURES, GrpoError, adamw_step, check_device_status, group_advantages,
     gumbel_noise, load, loss_fwd_bwd, loss_fwd_bwd_adamw, sample_tokens, status_string, token_logprobs,
-    token_logprobs_heads, workspace, workspace_bytes,
+    token_logprobs_heads, vocab_chunk_cols, workspace, workspace_bytes,
 )

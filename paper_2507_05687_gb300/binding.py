@@ -49,6 +49,9 @@ SIGNATURES = {
                                               _P, _P, _P, _P, ctypes.c_size_t, _P]),
     "grpo_loss_fwd_bwd_kl_clamp": (ctypes.c_int, [_P, _P, _P, _P, _P, _P, _P, _I64, _I64, _I32, _I64, _F, _F, _I32,
                                                   _F, _F, _P, _P, _P, _P, ctypes.c_size_t, _P]),
+    "grpo_loss_fwd_bwd_events": (ctypes.c_int, [_P, _P, _P, _P, _P, _P, _P, _I64, _I64, _I32, _I64, _F, _F, _I32,
+                                                _F, _P, _P, _P, _P, _I32, _P, ctypes.c_size_t, _P]),
+    "grpo_vocab_chunk_cols": (ctypes.c_int64, [_I64]),
     "grpo_loss_fwd_bwd_to_host": (ctypes.c_int, [_P, _P, _P, _P, _P, _P, _P, _I64, _I64, _I32, _I64, _F, _F, _I32,
                                                  _F, _P, _P, _P, _P, _P, ctypes.c_size_t, _P]),
     "grpo_loss_fwd_bwd_adamw": (ctypes.c_int, [_P, _P, _P, _P, _P, _P, _P, _I64, _I64, _I32, _I64, _F, _F, _I32, _F,
@@ -231,10 +234,12 @@ def loss_fwd_bwd(H: torch.Tensor, W: torch.Tensor, targets: torch.Tensor, mask: 
                  n_resp: int, L: int, clip_eps: float = 0.2, beta: float = 0.04, agg_mode: int = 0,
                  ws: Optional[torch.Tensor] = None,
                  out: Optional[Tuple[torch.Tensor, torch.Tensor, torch.Tensor]] = None, norm: float = 0.0,
-                 kl_clamp: Optional[float] = None):
+                 kl_clamp: Optional[float] = None, chunk_events: Optional[list] = None):
     """grpo_loss_fwd_bwd (norm == 0) / grpo_loss_fwd_bwd_norm (norm > 0, a global
     N_valid or n_resp) / grpo_loss_fwd_bwd_kl_clamp (kl_clamp given, a cap on the
-    per-token KL value): returns (loss [1] fp32, dH [T, Hd] fp32, dW [V, Hd] fp32).
+    per-token KL value) / grpo_loss_fwd_bwd_events (chunk_events: torch.cuda.Event
+    per vocabulary chunk, recorded when that chunk's dW rows are written):
+    returns (loss [1] fp32, dH [T, Hd] fp32, dW [V, Hd] fp32).
     `out` may be device tensors (written in place) or host tensors, preferably
     pinned (the results are copied there before the call returns)."""
     dev, host = _target_device(H, W)
@@ -261,14 +266,25 @@ def loss_fwd_bwd(H: torch.Tensor, W: torch.Tensor, targets: torch.Tensor, mask: 
     common = (_ptr(H), _ptr(W), _ptr(targets), _ptr(mask), _ptr(old_logp), _ptr(ref_logp), _ptr(adv), int(n_resp),
               int(L), Hd, V, float(clip_eps), float(beta), int(agg_mode))
     tail = (_ptr(loss), _ptr(dH), _ptr(dW), _ptr(ws), ws.numel(), _stream(dev))
-    if host_out is not None and host_out[2].is_pinned() and kl_clamp is None:
+    if host_out is not None and host_out[2].is_pinned() and kl_clamp is None and chunk_events is None:
         # dW streams to the caller's pinned buffer chunk by chunk while the backward runs
         _check(lib.grpo_loss_fwd_bwd_to_host(*common, float(norm), _ptr(loss), _ptr(dH), _ptr(dW),
                                              _ptr(host_out[2]), _ptr(ws), ws.numel(), _stream(dev)),
                "grpo_loss_fwd_bwd_to_host")
         lh, dHh = _to_host(loss, dH, dst=host_out[:2])
         return lh, dHh, host_out[2]
-    if kl_clamp is not None:
+    if chunk_events is not None:
+        if kl_clamp is not None:
+            raise ValueError("chunk_events and kl_clamp are separate entry points")
+        stream = torch.cuda.current_stream(dev)
+        for ev in chunk_events:
+            if not ev.cuda_event:
+                ev.record(stream)  # torch creates the CUDA event on its first record
+        evs = (ctypes.c_void_p * max(1, len(chunk_events)))(*[ev.cuda_event for ev in chunk_events])
+        _check(lib.grpo_loss_fwd_bwd_events(*common, float(norm), _ptr(loss), _ptr(dH), _ptr(dW), evs,
+                                            len(chunk_events), _ptr(ws), ws.numel(), _stream(dev)),
+               "grpo_loss_fwd_bwd_events")
+    elif kl_clamp is not None:
         _check(lib.grpo_loss_fwd_bwd_kl_clamp(*common, float(norm), float(kl_clamp), *tail),
                "grpo_loss_fwd_bwd_kl_clamp")
     elif norm:
@@ -331,6 +347,11 @@ def adamw_step(W_master: torch.Tensor, exp_avg: torch.Tensor, exp_avg_sq: torch.
     _check(load().grpo_adamw_step(_ptr(W_master), _ptr(exp_avg), _ptr(exp_avg_sq), _ptr(grad), _ptr(W_out), n,
                                   float(lr), float(betas[0]), float(betas[1]), float(eps), float(weight_decay),
                                   int(step), _stream(W_master.device)), "grpo_adamw_step")
+
+
+def vocab_chunk_cols(V: int) -> int:
+    """grpo_vocab_chunk_cols: dW rows per backward chunk (chunk c = rows c*cols ..)."""
+    return int(load().grpo_vocab_chunk_cols(int(V)))
 
 
 def gumbel_noise(row0: int, rows: int, cols: int, seed: int, offset: int = 0, device=None) -> torch.Tensor:

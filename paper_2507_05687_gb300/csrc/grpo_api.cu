@@ -480,7 +480,8 @@ grpo_status loss_impl(const uint16_t* H, const uint16_t* W, const int32_t* targe
                       const float* old_logp, const float* ref_logp, const float* adv, int64_t n_resp,
                       int64_t L, int32_t Hd, int64_t V, float clip_eps, float beta, int32_t agg_mode,
                       float norm, float* loss_out, float* dH, float* dW, const AdamParams* adam, void* ws,
-                      size_t ws_bytes, void* stream, float* dW_host = nullptr, float kl_clamp = INFINITY);
+                      size_t ws_bytes, void* stream, float* dW_host = nullptr, float kl_clamp = INFINITY,
+                      void* const* chunk_events = nullptr, int32_t n_events = 0);
 
 }  // namespace
 
@@ -688,6 +689,20 @@ grpo_status grpo_loss_fwd_bwd_kl_clamp(const uint16_t* H, const uint16_t* W, con
                    norm, loss_out, dH, dW, nullptr, ws, ws_bytes, stream, nullptr, kl_clamp);
 }
 
+int64_t grpo_vocab_chunk_cols(int64_t V) { return V > 0 ? vocab_chunk(V) : 0; }
+
+grpo_status grpo_loss_fwd_bwd_events(const uint16_t* H, const uint16_t* W, const int32_t* targets,
+                                     const uint8_t* mask, const float* old_logp, const float* ref_logp,
+                                     const float* adv, int64_t n_resp, int64_t L, int32_t Hd, int64_t V,
+                                     float clip_eps, float beta, int32_t agg_mode, float norm, float* loss_out,
+                                     float* dH, float* dW, void* const* chunk_events, int32_t n_events, void* ws,
+                                     size_t ws_bytes, void* stream) {
+  if (!chunk_events) return GRPO_ERR_INVALID_ARG;
+  return loss_impl(H, W, targets, mask, old_logp, ref_logp, adv, n_resp, L, Hd, V, clip_eps, beta, agg_mode,
+                   norm, loss_out, dH, dW, nullptr, ws, ws_bytes, stream, nullptr, INFINITY, chunk_events,
+                   n_events);
+}
+
 grpo_status grpo_loss_fwd_bwd_to_host(const uint16_t* H, const uint16_t* W, const int32_t* targets,
                                       const uint8_t* mask, const float* old_logp, const float* ref_logp,
                                       const float* adv, int64_t n_resp, int64_t L, int32_t Hd, int64_t V,
@@ -737,7 +752,8 @@ grpo_status loss_impl(const uint16_t* H, const uint16_t* W, const int32_t* targe
                       const float* old_logp, const float* ref_logp, const float* adv, int64_t n_resp,
                       int64_t L, int32_t Hd, int64_t V, float clip_eps, float beta, int32_t agg_mode,
                       float norm, float* loss_out, float* dH, float* dW, const AdamParams* adam, void* ws,
-                      size_t ws_bytes, void* stream, float* dW_host, float kl_clamp) {
+                      size_t ws_bytes, void* stream, float* dW_host, float kl_clamp, void* const* chunk_events,
+                      int32_t n_events) {
   if (n_resp < 1 || L < 1 || n_resp > (int64_t(1) << 31) / L) return GRPO_ERR_INVALID_ARG;
   if (!(norm >= 0.f) || norm == INFINITY) return GRPO_ERR_INVALID_ARG;
   if (!(kl_clamp >= 0.f)) return GRPO_ERR_INVALID_ARG;
@@ -751,6 +767,12 @@ grpo_status loss_impl(const uint16_t* H, const uint16_t* W, const int32_t* targe
   if (!aligned(W, 16) || !aligned(H, 16) || !aligned(dH, 16) || !aligned(dW, 16))
     return GRPO_ERR_INVALID_ARG;
   if (!ws || !aligned(ws, 256) || ws_bytes < Ly.total) return GRPO_ERR_WORKSPACE;
+  if (chunk_events) {
+    const int64_t chunks = (V + Ly.vchunk - 1) / Ly.vchunk;
+    if (n_events < chunks) return GRPO_ERR_INVALID_ARG;
+    for (int64_t c = 0; c < chunks; ++c)
+      if (!chunk_events[c]) return GRPO_ERR_INVALID_ARG;
+  }
   DeviceInfo di;
   if (!device_info(&di)) return GRPO_ERR_UNSUPPORTED;
   if (!get_encode()) return GRPO_ERR_CUDA;
@@ -876,6 +898,7 @@ grpo_status loss_impl(const uint16_t* H, const uint16_t* W, const int32_t* targe
         e = launch_gemm<kEpiF32, true, false>(opDz, opHcT, w, width, di, s, &outDw);
       }
     }
+    if (e == cudaSuccess && chunk_events) e = cudaEventRecord(static_cast<cudaEvent_t>(chunk_events[chunk]), s);
     if (e == cudaSuccess && co) {
       cudaEvent_t ready = co->ready[chunk % CopyOut::kRing];
       e = cudaEventRecord(ready, s);

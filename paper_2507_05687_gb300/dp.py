@@ -10,8 +10,10 @@ up to those of the whole batch; the one data exchange is the sum of dW (and
 of the scalar loss).  dH stays with the rank that owns the tokens.
 
 `compute` is the per-rank loss call; by default the CUDA library's
-grpo_loss_fwd_bwd_norm.  Collectives go through torch.distributed (NCCL on
-GPUs, gloo on CPUs).
+grpo_loss_fwd_bwd_events, whose per-chunk events let each vocabulary chunk's
+dW all-reduce start on a communication stream while the later chunks still
+compute.  Collectives go through torch.distributed (NCCL on GPUs, gloo on
+CPUs).
 """
 from __future__ import annotations
 
@@ -63,13 +65,49 @@ def dp_loss_fwd_bwd(H, W, targets, mask, old_logp, ref_logp, adv, n_resp: int, L
     rank's rows.
     """
     import torch.distributed as dist
-    compute = compute or default_compute
     dev = W.device if isinstance(W, torch.Tensor) else torch.device("cpu")
     norm = global_count(local_count, dev if dev.type == "cuda" else torch.device("cpu"), group)
     if norm <= 0:
         norm = 1.0  # an all-padding step: every weight is 0 anyway
+    if compute is None and dev.type == "cuda":
+        return _overlapped(H, W, targets, mask, old_logp, ref_logp, adv, n_resp, L, clip_eps, beta, agg_mode,
+                           norm, group, **kw)
+    compute = compute or default_compute
     loss, dH, dW = compute(H, W, targets, mask, old_logp, ref_logp, adv, n_resp, L, clip_eps, beta, agg_mode,
                            norm, **kw)
     dist.all_reduce(dW, op=dist.ReduceOp.SUM, group=group)
     dist.all_reduce(loss, op=dist.ReduceOp.SUM, group=group)
+    return loss, dH, dW
+
+
+def chunk_rows(V: int, cols: int):
+    """Row slices of dW, one per backward vocabulary chunk of `cols` rows."""
+    if cols <= 0:
+        return []
+    return [slice(c0, min(V, c0 + cols)) for c0 in range(0, V, cols)]
+
+
+def _overlapped(H, W, targets, mask, old_logp, ref_logp, adv, n_resp, L, clip_eps, beta, agg_mode, norm, group,
+                ws=None, out=None, comm_stream=None):
+    """The library call with one event per vocabulary chunk; on a communication
+    stream, each chunk's rows of dW are all-reduced as soon as its event fires,
+    overlapping the backward of the later chunks.  The caller's current stream
+    waits for every collective before this returns."""
+    import torch.distributed as dist
+    from . import binding
+    dev = W.device
+    rows = chunk_rows(W.shape[0], binding.vocab_chunk_cols(W.shape[0]))
+    events = [torch.cuda.Event() for _ in rows]
+    loss, dH, dW = binding.loss_fwd_bwd(H, W, targets, mask, old_logp, ref_logp, adv, n_resp, L, clip_eps, beta,
+                                        agg_mode, ws=ws, out=out, norm=norm, chunk_events=events)
+    comm = comm_stream or torch.cuda.Stream(dev)
+    works = []
+    with torch.cuda.stream(comm):
+        for ev, r in zip(events, rows):
+            comm.wait_event(ev)
+            works.append(dist.all_reduce(dW[r], op=dist.ReduceOp.SUM, group=group, async_op=True))
+        works.append(dist.all_reduce(loss, op=dist.ReduceOp.SUM, group=group, async_op=True))
+    for wk in works:
+        wk.wait()
+    torch.cuda.current_stream(dev).wait_stream(comm)
     return loss, dH, dW

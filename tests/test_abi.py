@@ -100,6 +100,15 @@ def test_host_rejections(lib):
     assert L.grpo_gumbel_noise(1, 2, 0, 4, 4, None, None) == grpo.GRPO_ERR_INVALID_ARG
     assert L.grpo_gumbel_noise(1, 2, 0, 4, 4, FAKE + 2, None) == grpo.GRPO_ERR_INVALID_ARG
     assert L.grpo_gumbel_noise(1, 2, 2**32, 0, 4, None, None) == grpo.GRPO_OK
+    eargs = largs[:14] + [0.0] + largs[14:17] + [None, 0] + largs[17:]
+    assert L.grpo_loss_fwd_bwd_events(*eargs) == grpo.GRPO_ERR_INVALID_ARG          # no event array
+    few = (ctypes.c_void_p * 1)(FAKE)
+    bad = list(eargs); bad[18], bad[19] = few, 0
+    assert L.grpo_loss_fwd_bwd_events(*bad) == grpo.GRPO_ERR_INVALID_ARG            # fewer events than chunks
+    nulls1 = (ctypes.c_void_p * 1)(None)
+    bad = list(eargs); bad[18], bad[19] = nulls1, 1
+    assert L.grpo_loss_fwd_bwd_events(*bad) == grpo.GRPO_ERR_INVALID_ARG            # a null event
+    assert L.grpo_vocab_chunk_cols(0) == 0 and L.grpo_vocab_chunk_cols(1000) == 1024
     assert L.grpo_check_device_status(None, None) == grpo.GRPO_ERR_INVALID_ARG
     ws3 = grpo.workspace_bytes(100, 64, 1000, grpo.GRPO_WS_LOGPROBS_HEADS)
     assert ws3 > grpo.workspace_bytes(100, 64, 1000, grpo.GRPO_WS_LOGPROBS)

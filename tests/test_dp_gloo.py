@@ -41,6 +41,17 @@ def test_shard_groups_cover_every_group_once():
     assert (rs.start, rs.stop, ts.start, ts.stop) == (12, 20, 120, 200)
 
 
+def test_chunk_rows_cover_every_vocabulary_row_once():
+    for V in (1, 255, 256, 4097, 155136):
+        for cols in (256, 768, 16384):
+            rows = dp.chunk_rows(V, cols)
+            assert rows[0].start == 0 and rows[-1].stop == V
+            assert all(a.stop == b.start for a, b in zip(rows, rows[1:]))
+            assert all(0 < r.stop - r.start <= cols for r in rows)
+            assert len(rows) == -(-V // cols)
+    assert dp.chunk_rows(10, 0) == []
+
+
 def _batch():
     import oracle
     import workloads as wl
