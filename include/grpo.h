@@ -23,7 +23,10 @@
  *   set bits of a status word inside the workspace; the affected rows' outputs
  *   are 0.  grpo_check_device_status reports that word.
  * - Outputs are overwritten, never accumulated into.  Results are
- *   deterministic: no floating-point atomics are used on any output.
+ *   deterministic: the one floating-point accumulation across launches (dH
+ *   over vocabulary chunks, in the workspace) adds each chunk's value to each
+ *   element once, in stream order, so the rounding order is fixed; nothing
+ *   else uses atomics on floating-point values.
  * - One workspace must not be used by two calls that can run concurrently.
  */
 #ifndef GRPO_H_
