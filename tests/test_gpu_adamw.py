@@ -5,7 +5,7 @@ import pytest
 
 import oracle
 import workloads as wl
-from tests._util import GRAD_RTOL, dev_tensor, rel_fro
+from tests._util import GRAD_RTOL, clear_of_clip_kink, dev_tensor, rel_fro
 
 torch = pytest.importorskip("torch")
 pytestmark = pytest.mark.gpu
@@ -27,6 +27,7 @@ def _case(monkeypatch, chunk="768"):
     Hb, Wb = wl.gen_hidden(w), wl.gen_weight(w)
     y, m, r = wl.gen_targets(w), wl.gen_mask(w), wl.gen_rewards(w)
     old = oracle.token_logprobs(Hb, wl.gen_weight(w, "old", Wb), y, m)[0].astype(np.float32)
+    old = clear_of_clip_kink(oracle.token_logprobs(Hb, Wb, y, m)[0], old, w.clip_eps)
     ref = oracle.token_logprobs(Hb, wl.gen_weight(w, "ref", Wb), y, m)[0].astype(np.float32)
     adv = oracle.group_advantages(r, w.G, float(np.float32(w.adv_eps)))
     want = oracle.loss_fwd_bwd(Hb, Wb, y, m, old, ref, adv, w.n_resp, w.L, w.clip_eps, w.beta)

@@ -6,7 +6,7 @@ import pytest
 
 import oracle
 import workloads as wl
-from tests._util import GRAD_RTOL, LOGP_ATOL, LOSS_RTOL, dev_tensor, loss_scale, rel_fro
+from tests._util import GRAD_RTOL, LOGP_ATOL, LOSS_RTOL, clear_of_clip_kink, dev_tensor, loss_scale, rel_fro
 
 torch = pytest.importorskip("torch")
 pytestmark = pytest.mark.gpu
@@ -27,6 +27,7 @@ def _case(w, agg_mode=0):
     y, m, r = wl.gen_targets(w), wl.gen_mask(w), wl.gen_rewards(w)
     W_old, W_ref = wl.gen_weight(w, "old", Wb), wl.gen_weight(w, "ref", Wb)
     old = oracle.token_logprobs(Hb, W_old, y, m)[0].astype(np.float32)
+    old = clear_of_clip_kink(oracle.token_logprobs(Hb, Wb, y, m)[0], old, w.clip_eps)
     ref = oracle.token_logprobs(Hb, W_ref, y, m)[0].astype(np.float32)
     adv = oracle.group_advantages(r, w.G, float(np.float32(w.adv_eps)))
     want = oracle.loss_fwd_bwd(Hb, Wb, y, m, old, ref, adv, w.n_resp, w.L, w.clip_eps, w.beta, agg_mode)
@@ -312,3 +313,18 @@ def test_host_output_buffers_stream_dw(monkeypatch):
     assert all(g is h for g, h in zip(got, host))
     for g, x in zip(got, dev_out):
         assert torch.equal(g, x.cpu())
+
+
+def test_larger_hidden_and_vocabulary():
+    """Beyond the 8B shape: a 262147-entry vocabulary (65 forward splits, odd tail)
+    for the log-probs, and hidden 8192 (128 k-blocks per tile) with a
+    40000-entry vocabulary through the whole loss forward + backward."""
+    w = wl.Workload("t", 1, 2, 70, 2048, 262147, "uniform", 40, 70, seed=wl.SEED_BASE + 1700)
+    Hb, Wb, y, m = wl.gen_hidden(w), wl.gen_weight(w), wl.gen_targets(w), wl.gen_mask(w)
+    want, _ = oracle.token_logprobs(Hb, Wb, y, m)
+    got = grpo.token_logprobs(dev_tensor(Hb, torch.bfloat16), dev_tensor(Wb, torch.bfloat16),
+                              dev_tensor(y, torch.int32), dev_tensor(m, torch.uint8)).cpu().numpy()
+    assert np.all(got[m == 0] == 0.0)
+    assert np.abs(got.astype(np.float64) - want).max() <= LOGP_ATOL
+    w2 = wl.Workload("t", 1, 4, 60, 8192, 40000, "uniform", 20, 60, rewards="mix", seed=wl.SEED_BASE + 1701)
+    _check_fwd_bwd(_case(w2))
