@@ -172,21 +172,22 @@ def kernel_hash() -> str:
     return h.hexdigest()[:16]
 
 
-def stored_traffic(kind_name: str):
+def stored_traffic(workload: str, kind_name: str):
     """DRAM bytes per launch from the committed ncu summary, if it was taken on
-    the current kernel source (profiles/traffic.txt: '<hash> <kind> <bytes/launch> <cols>')."""
+    the current kernel source and this workload (profiles/traffic.txt:
+    '<hash> <workload> <kind> <bytes/launch> <cols>')."""
     path = os.path.join(ROOT, "profiles", "traffic.txt")
     if not os.path.exists(path):
         return None
     kh = kernel_hash()
     for line in open(path):
         f = line.split()
-        if len(f) >= 4 and f[0] == kh and f[1] == kind_name:
-            return float(f[2]), int(f[3])
+        if len(f) >= 5 and f[0] == kh and f[1] == workload and f[2] == kind_name:
+            return float(f[3]), int(f[4])
     return None
 
 
-def roofline(trace, n_valid_total_per_rank, Hd, steps, peak_tf, peak_kind):
+def roofline(trace, n_valid_total_per_rank, Hd, steps, peak_tf, peak_kind, workload_key):
     by = {}
     for kind, cols, ms in trace:
         by.setdefault(kind, []).append((cols, ms))
@@ -198,7 +199,7 @@ def roofline(trace, n_valid_total_per_rank, Hd, steps, peak_tf, peak_kind):
     achieved = (sum(flops) / len(flops)) / (sum(secs) / len(secs)) / 1e12
     total_ms = sum(ms for v in by.values() for _, ms in v)
     shares = {KIND_NAMES[k]: round(sum(ms for _, ms in v) / total_ms, 4) for k, v in sorted(by.items())}
-    tr = stored_traffic(KIND_NAMES[dom])
+    tr = stored_traffic(workload_key, KIND_NAMES[dom])
     traffic = None
     if tr is not None:
         bytes_per_launch, cols_ref = tr
@@ -422,7 +423,8 @@ def main():
     value = tot_valid / (ms / 1e3)
 
     burst, sustained, hbm, peak_src = peaks()
-    rf = roofline(trace, n_valid, w.Hd, args.steps, sustained, f"bf16 sustained, {peak_src}")
+    rkey = w.name + ("+sample" if sampling else "") + ("" if args.adamw == "none" else "+adamw_" + args.adamw)
+    rf = roofline(trace, n_valid, w.Hd, args.steps, sustained, f"bf16 sustained, {peak_src}", rkey)
     if sampling:
         step_flops8 = step_flops6 = 2.0 * n_valid * w.Hd * w.V
     elif scoring:
