@@ -63,7 +63,6 @@ struct TileCfg {
   static constexpr int kABytes = kRowsCta * kBK * 2;    // 16 KB
   static constexpr int kBBytes = kBRows * kBK * 2;      // 32 KB (single) / 16 KB (pair)
   static constexpr int kStageBytes = kABytes + kBBytes;
-  static constexpr int kStages = kPair == 2 ? 6 : 4;
 };
 
 enum { kEpiLse = 0, kEpiDz = 1, kEpiF32 = 2, kEpiAdam = 3, kEpiSample = 4 };
@@ -78,17 +77,28 @@ struct EpiShape {
   static constexpr int kWarps = kEpi == kEpiSample ? 8 : 4;
   static constexpr int kHalves = kWarps / 4;    // column halves of a tile, one per warp of a quarter
   static constexpr int kThreads = 64 + 32 * kWarps;
-  static constexpr bool kTmaOut = kEpi == kEpiDz || kEpi == kEpiF32;
-  // one warp's 32 x 32 output block in shared memory (bf16 dZ / fp32), two per warp
-  static constexpr int kBlockBytes = kEpi == kEpiDz ? 32 * 32 * 2 : kEpi == kEpiF32 ? 32 * 32 * 4 : 0;
-  static constexpr int kOutBytes = 2 * kBlockBytes * kWarps;
+  static constexpr bool kTmaOut = kEpi == kEpiDz || kEpi == kEpiF32 || kEpi == kEpiAdam;
+  // one warp's 32 x 32 block in shared memory: bf16 dZ / fp32 output, two per
+  // warp; kEpiAdam: fp32 weights, first and second moments (4 KB each) and the
+  // bf16 weights (2 KB), one per warp (the dW K-loop is long enough to hide it)
+  static constexpr int kBlockBytes =
+      kEpi == kEpiDz ? 32 * 32 * 2 : kEpi == kEpiF32 ? 32 * 32 * 4 : kEpi == kEpiAdam ? 3 * 4096 + 2048 : 0;
+  static constexpr int kBlocks = kEpi == kEpiAdam ? 1 : 2;
+  static constexpr int kOutBytes = kBlocks * kBlockBytes * kWarps;
 };
+
+// Operand-ring depth: 6 stages of 32 KB (pair) / 4 of 48 KB (single), one
+// fewer for kEpiAdam (6 / 3), whose staging blocks take the room.
+template <int kPair, int kEpi>
+__host__ __device__ constexpr int ring_stages() {
+  return kEpi == kEpiAdam ? (kPair == 2 ? 5 : 3) : (kPair == 2 ? 6 : 4);
+}
 
 // Dynamic shared memory of one CTA: the operand ring, the output staging
 // blocks (1024-byte aligned, as the output swizzle needs), the barriers.
 template <int kPair, int kEpi>
-constexpr int smem_bytes() {
-  return TileCfg<kPair>::kStages * TileCfg<kPair>::kStageBytes + EpiShape<kEpi>::kOutBytes + 1024 /*align*/ +
+__host__ __device__ constexpr int smem_bytes() {
+  return ring_stages<kPair, kEpi>() * TileCfg<kPair>::kStageBytes + EpiShape<kEpi>::kOutBytes + 1024 /*align*/ +
          256 /*barriers*/;
 }
 
@@ -121,15 +131,12 @@ struct GemmArgs {
   // kEpiF32 (output: fp32 through the output tensor map)
   int accumulate;       // 1: out += acc (L2 reduce-add), 0: out = acc
 
-  long ldo;             // kEpiAdam: row stride of the weights
   const int* row_map;   // kEpiSample: token position of each compacted row
 
   // kEpiAdam: the accumulator is a dW tile; an AdamW step is applied to the
-  // matching weights in place (row stride ldo) instead of storing dW.
-  float* master;        // fp32 weights
-  float* exp_avg;       // first moment
-  float* exp_avg_sq;    // second moment
-  uint16_t* w_out;      // bf16 copy of the updated weights
+  // matching weights instead of storing dW.  The fp32 weights, both moments
+  // and the bf16 weights are reached through tensor maps (the output map and
+  // B maps 1..3, which a one-head launch does not otherwise use).
   float adam_b1, adam_b2, adam_eps, adam_lr;
   float adam_decay;     // 1 - lr * weight_decay
   float adam_bc1;       // 1 / (1 - beta1^step)
@@ -233,6 +240,14 @@ struct OutStage {
   int count;                 // blocks written so far by this warp
   const CUtensorMap* map;
   int lane;
+  // kEpiAdam: the moments' and bf16 weights' maps, the block's load barrier
+  const CUtensorMap* m_map;
+  const CUtensorMap* v_map;
+  const CUtensorMap* w_map;
+  uint32_t ld_bar;
+  uint32_t ld_phase;
+  volatile int* abort;
+  unsigned long long wlim;
 };
 
 // Writes this warp's 32 x 32 output block (lane = row, `words` = the row's 64
@@ -265,12 +280,68 @@ __device__ __forceinline__ void out_block(OutStage& o, const uint32_t* words, in
   ++o.count;
 }
 
+// One AdamW step on this warp's 32 x 32 block of LM-head weights at (x, y),
+// whose gradient rows are in `g` (lane = row): lane 0 loads the fp32 weights
+// and both moments with TMA (128-byte swizzle, zero-filled past the matrix),
+// every lane updates its row in shared memory, and lane 0 stores the three
+// blocks and the bf16 weights back (clipped at the matrix).  False if the load
+// wait gave up (abort or time limit).
+__device__ __forceinline__ bool adam_block(OutStage& o, const float* g, int x, int y, const GemmArgs& a) {
+  const uint32_t th = o.smem, mo = o.smem + 4096, ve = o.smem + 8192, wb = o.smem + 12288;
+  if (o.lane == 0) {
+    bulk_wait_read_0();  // the previous block's stores have read the buffer
+    mbar_arrive_expect_tx(o.ld_bar, 3 * 4096);
+    tma_load_2d(th, o.map, o.ld_bar, x, y);
+    tma_load_2d(mo, o.m_map, o.ld_bar, x, y);
+    tma_load_2d(ve, o.v_map, o.ld_bar, x, y);
+  }
+  const bool got = mbar_wait(o.ld_bar, o.ld_phase, o.abort, o.wlim);
+  o.ld_phase ^= 1u;
+  if (!__all_sync(0xffffffffu, got)) return false;
+  const uint32_t row = static_cast<uint32_t>(o.lane * 128);
+  const uint32_t sw = o.lane & 7;
+  uint32_t wpk[16];
+#pragma unroll
+  for (int q = 0; q < 8; ++q) {
+    const uint32_t off = row + 16u * (static_cast<uint32_t>(q) ^ sw);
+    float4 p, m, v;
+    ld_shared_v4(th + off, p);
+    ld_shared_v4(mo + off, m);
+    ld_shared_v4(ve + off, v);
+    adam_update(g[4 * q + 0], p.x, m.x, v.x, a);
+    adam_update(g[4 * q + 1], p.y, m.y, v.y, a);
+    adam_update(g[4 * q + 2], p.z, m.z, v.z, a);
+    adam_update(g[4 * q + 3], p.w, m.w, v.w, a);
+    st_shared_v4(th + off, __float_as_uint(p.x), __float_as_uint(p.y), __float_as_uint(p.z), __float_as_uint(p.w));
+    st_shared_v4(mo + off, __float_as_uint(m.x), __float_as_uint(m.y), __float_as_uint(m.z), __float_as_uint(m.w));
+    st_shared_v4(ve + off, __float_as_uint(v.x), __float_as_uint(v.y), __float_as_uint(v.z), __float_as_uint(v.w));
+    wpk[2 * q] = pack_bf16x2(p.x, p.y);
+    wpk[2 * q + 1] = pack_bf16x2(p.z, p.w);
+  }
+  const uint32_t wrow = wb + static_cast<uint32_t>(o.lane * 64);
+  const uint32_t wsw = (o.lane >> 1) & 3;
+#pragma unroll
+  for (int j = 0; j < 4; ++j)
+    st_shared_v4(wrow + 16u * (static_cast<uint32_t>(j) ^ wsw), wpk[4 * j], wpk[4 * j + 1], wpk[4 * j + 2],
+                 wpk[4 * j + 3]);
+  fence_proxy_async_smem();
+  __syncwarp();
+  if (o.lane == 0) {
+    tma_store_2d(o.map, th, x, y);
+    tma_store_2d(o.m_map, mo, x, y);
+    tma_store_2d(o.v_map, ve, x, y);
+    tma_store_2d(o.w_map, wb, x, y);
+    bulk_commit();
+  }
+  return true;
+}
+
 // One 256-column accumulator tile of this thread's row; `tbase` is the TMEM
 // address of column 0 of the tile in this warp's lane quarter; `row0` is the
 // accumulator row of lane 0 (the TMA row coordinate of the warp's block) and
 // m_rows the rows of the output (M).
 template <int kEpi>
-__device__ __forceinline__ void epi_tile(EpiRow& e, const GemmArgs& a, uint32_t tbase, int col0,
+__device__ __forceinline__ bool epi_tile(EpiRow& e, const GemmArgs& a, uint32_t tbase, int col0,
                                          bool have_acc, int half, OutStage& os, int row0, int m_rows) {
   const float kLog2e = 1.4426950408889634f;
   constexpr int kChunks = kTileN / 32 / EpiShape<kEpi>::kHalves;
@@ -358,49 +429,8 @@ __device__ __forceinline__ void epi_tile(EpiRow& e, const GemmArgs& a, uint32_t 
       }
       out_block<16>(os, packed, cb, row0, false);
     } else if (kEpi == kEpiAdam) {
-      if (e.rv) {
-        const long base = static_cast<long>(e.r) * a.ldo + cb;
-        if (cb + 32 <= a.N) {
-          float4* __restrict__ P = reinterpret_cast<float4*>(a.master + base);
-          float4* __restrict__ M = reinterpret_cast<float4*>(a.exp_avg + base);
-          float4* __restrict__ S = reinterpret_cast<float4*>(a.exp_avg_sq + base);
-          uint2* __restrict__ O = reinterpret_cast<uint2*>(a.w_out + base);
-          // all 24 loads of the 32 columns in flight at once, then the math, then the stores
-          float4 p[8], m[8], sq[8];
-#pragma unroll
-          for (int q = 0; q < 8; ++q) {
-            p[q] = __ldcs(P + q);
-            m[q] = __ldcs(M + q);
-            sq[q] = __ldcs(S + q);
-          }
-#pragma unroll
-          for (int q = 0; q < 8; ++q) {
-            adam_update(v[4 * q + 0], p[q].x, m[q].x, sq[q].x, a);
-            adam_update(v[4 * q + 1], p[q].y, m[q].y, sq[q].y, a);
-            adam_update(v[4 * q + 2], p[q].z, m[q].z, sq[q].z, a);
-            adam_update(v[4 * q + 3], p[q].w, m[q].w, sq[q].w, a);
-          }
-#pragma unroll
-          for (int q = 0; q < 8; ++q) {
-            __stcs(P + q, p[q]);
-            __stcs(M + q, m[q]);
-            __stcs(S + q, sq[q]);
-            O[q] = make_uint2(pack_bf16x2(p[q].x, p[q].y), pack_bf16x2(p[q].z, p[q].w));
-          }
-        } else {
-#pragma unroll
-          for (int j = 0; j < 32; ++j) {
-            if (cb + j < a.N) {
-              float p = a.master[base + j], m = a.exp_avg[base + j], sq = a.exp_avg_sq[base + j];
-              adam_update(v[j], p, m, sq, a);
-              a.master[base + j] = p;
-              a.exp_avg[base + j] = m;
-              a.exp_avg_sq[base + j] = sq;
-              a.w_out[base + j] = static_cast<uint16_t>(pack_bf16x2(p, 0.f) & 0xFFFFu);
-            }
-          }
-        }
-      }
+      // a block wholly past M or N is skipped; the tensor maps clip the rest
+      if (row0 < m_rows && cb < a.N && !adam_block(os, v, cb, row0, a)) return false;
     } else {
       // kEpiF32: a block wholly past M or N is skipped; the tensor map clips
       // the rest (its rows are the output's M, its columns N)
@@ -412,6 +442,7 @@ __device__ __forceinline__ void epi_tile(EpiRow& e, const GemmArgs& a, uint32_t 
       }
     }
   }
+  return true;
 }
 
 template <int kEpi>
@@ -439,17 +470,19 @@ __device__ __forceinline__ void gemm_body(const CUtensorMap* tmA, const CUtensor
                                           const CUtensorMap* tmD, const GemmArgs& args) {
   using C = TileCfg<kPair>;
   using ES = EpiShape<kEpi>;
+  constexpr int kStages = ring_stages<kPair, kEpi>();
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
-  uint8_t* out_stage = smem + C::kStages * C::kStageBytes;  // [warps][2] output blocks
+  uint8_t* out_stage = smem + kStages * C::kStageBytes;  // [warps][blocks] output staging
   uint64_t* bars = reinterpret_cast<uint64_t*>(out_stage + ES::kOutBytes);
   uint64_t* full_bar = bars;                          // [kStages] TMA -> MMA (issuing CTA)
-  uint64_t* empty_bar = bars + C::kStages;            // [kStages] MMA -> TMA (each CTA)
-  uint64_t* tfull_bar = bars + 2 * C::kStages;        // [2] MMA -> epilogue (each CTA)
-  uint64_t* tempty_bar = bars + 2 * C::kStages + 2;   // [2] epilogue -> MMA (issuing CTA)
-  uint64_t* done_bar = bars + 2 * C::kStages + 4;     // [1] all MMAs retired (issuing CTA)
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * C::kStages + 5);
+  uint64_t* empty_bar = bars + kStages;               // [kStages] MMA -> TMA (each CTA)
+  uint64_t* tfull_bar = bars + 2 * kStages;           // [2] MMA -> epilogue (each CTA)
+  uint64_t* tempty_bar = bars + 2 * kStages + 2;      // [2] epilogue -> MMA (issuing CTA)
+  uint64_t* done_bar = bars + 2 * kStages + 4;        // [1] all MMAs retired (issuing CTA)
+  uint64_t* ld_bar = bars + 2 * kStages + 5;          // [4] kEpiAdam block loads (one per epilogue warp)
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * kStages + 9);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5;
@@ -460,7 +493,7 @@ __device__ __forceinline__ void gemm_body(const CUtensorMap* tmA, const CUtensor
   const int unit_stride = gridDim.x / kPair;
 
   if (threadIdx.x == 0) {
-    for (int i = 0; i < C::kStages; ++i) {
+    for (int i = 0; i < kStages; ++i) {
       mbar_init(smem_addr(&full_bar[i]), 1);
       mbar_init(smem_addr(&empty_bar[i]), 1);
     }
@@ -469,6 +502,8 @@ __device__ __forceinline__ void gemm_body(const CUtensorMap* tmA, const CUtensor
       mbar_init(smem_addr(&tempty_bar[i]), EpiShape<kEpi>::kWarps * kPair);  // one arrival per epilogue warp
     }
     mbar_init(smem_addr(done_bar), 1);
+    if (kEpi == kEpiAdam)
+      for (int i = 0; i < ES::kWarps; ++i) mbar_init(smem_addr(&ld_bar[i]), 1);
     *abort_flag = 0;
     fence_mbar_init();
   }
@@ -509,9 +544,9 @@ __device__ __forceinline__ void gemm_body(const CUtensorMap* tmA, const CUtensor
       const uint64_t pol_b = l2_policy(args.b_hint);
       int stage = 0;
       uint32_t phase = 0;
-      int uses[C::kStages];
+      int uses[kStages];
 #pragma unroll
-      for (int s = 0; s < C::kStages; ++s) uses[s] = 0;
+      for (int s = 0; s < kStages; ++s) uses[s] = 0;
       bool ok = true;
       int kblock_count = 0;  // k-blocks this CTA has staged (fault-injection hook)
       for (int u = unit0; u < sch.total && ok; u += unit_stride) {
@@ -555,7 +590,7 @@ __device__ __forceinline__ void gemm_body(const CUtensorMap* tmA, const CUtensor
                 load(sb + j * 8192, tmBs[head], n0 + args.b_off_n + 64 * j, k0 + args.b_off_k, pol_b);
             }
             ++uses[stage];
-            if (++stage == C::kStages) {
+            if (++stage == kStages) {
               stage = 0;
               phase ^= 1u;
             }
@@ -565,7 +600,7 @@ __device__ __forceinline__ void gemm_body(const CUtensorMap* tmA, const CUtensor
       if (!ok) raise_abort();
       // Every stage this CTA filled must have been consumed (so its copies
       // have landed) before the CTA can exit.
-      for (int s = 0; s < C::kStages; ++s)
+      for (int s = 0; s < kStages; ++s)
         if (uses[s] > 0)
           mbar_wait(smem_addr(&empty_bar[s]), static_cast<uint32_t>(uses[s] - 1) & 1u, abort_flag, wlim);
     }
@@ -613,7 +648,7 @@ __device__ __forceinline__ void gemm_body(const CUtensorMap* tmA, const CUtensor
             }
             if (kPair == 2) tc_commit_pair_mc(smem_addr(&empty_bar[stage]), 0x3);
             else tc_commit(smem_addr(&empty_bar[stage]));
-            if (++stage == C::kStages) {
+            if (++stage == kStages) {
               stage = 0;
               phase ^= 1u;
             }
@@ -642,7 +677,17 @@ __device__ __forceinline__ void gemm_body(const CUtensorMap* tmA, const CUtensor
     const uint32_t tempty1 = smem_addr(&tempty_bar[1]);
     const uint32_t tempty_c0 = kPair == 2 ? mapa_shared(tempty0, 0) : tempty0;
     const uint32_t tempty_c1 = kPair == 2 ? mapa_shared(tempty1, 0) : tempty1;
-    OutStage os{smem_addr(out_stage) + static_cast<uint32_t>((warp - 2) * 2 * ES::kBlockBytes), 0, tmD, lane};
+    OutStage os{smem_addr(out_stage) + static_cast<uint32_t>((warp - 2) * ES::kBlocks * ES::kBlockBytes),
+                0,
+                tmD,
+                lane,
+                tmBs[1],
+                tmBs[2],
+                tmBs[3],
+                smem_addr(&ld_bar[kEpi == kEpiAdam ? warp - 2 : 0]),
+                0u,
+                abort_flag,
+                wlim};
     int tile = 0;
     bool ok = true;
     for (int u = unit0; u < sch.total && ok; u += unit_stride) {
@@ -668,8 +713,8 @@ __device__ __forceinline__ void gemm_body(const CUtensorMap* tmA, const CUtensor
           }
           tc_fence_after();
         }
-        epi_tile<kEpi>(e, args, lane_addr + static_cast<uint32_t>(buf * kTileN), nt * kTileN, have_acc, half, os,
-                       row0, sch.m_rows);
+        const bool done = epi_tile<kEpi>(e, args, lane_addr + static_cast<uint32_t>(buf * kTileN), nt * kTileN,
+                                         have_acc, half, os, row0, sch.m_rows);
         if (have_acc) {
           tc_fence_before();
           __syncwarp();
@@ -678,6 +723,10 @@ __device__ __forceinline__ void gemm_body(const CUtensorMap* tmA, const CUtensor
             if (kPair == 2) mbar_arrive_cluster(tb); else mbar_arrive(tb);
           }
           ++tile;
+        }
+        if (!done) {  // a kEpiAdam block load gave up
+          ok = false;
+          break;
         }
       }
       if (!ok) break;

@@ -174,7 +174,7 @@ bool device_info(DeviceInfo* out) {
     if (major != 10 || minor != 3) return false;
     if (!prepare_kernels<kEpiLse, false, false>(&pairs) || !prepare_kernels<kEpiDz, false, false>(&pairs) ||
         !prepare_kernels<kEpiF32, false, true>(&pairs) || !prepare_kernels<kEpiF32, true, false>(&pairs) ||
-        !prepare_kernels<kEpiAdam, true, true>(&pairs) || !prepare_kernels<kEpiSample, false, false>(&pairs))
+        !prepare_kernels<kEpiAdam, true, false>(&pairs) || !prepare_kernels<kEpiSample, false, false>(&pairs))
       return false;
     cache[dev].sms = sms;
     cache[dev].pairs = std::max(pairs, 0);
@@ -352,16 +352,6 @@ cudaError_t launch_gemm_cfg(const Operand& A, const Operand* B, const GemmArgs& 
   a.n_heads = std::max(1, std::min(a.n_heads, kMaxHeads));
   CUtensorMap ta, tb[kMaxHeads], td;
   if (!encode_2d(&ta, A.base, A.rows, A.cols, A.ld, kBK, AMN ? 64 : kRowsCta)) return cudaErrorInvalidValue;
-  if (EpiShape<E>::kTmaOut) {
-    // 32 x 32 boxes: 64-byte bf16 rows in the 64-byte swizzle, 128-byte fp32 rows in the 128-byte one
-    const bool f32 = E == kEpiF32;
-    if (!D || !aligned(D->base, 16) ||
-        !encode_2d(&td, D->base, D->rows, D->cols, D->ld, 32, 32, f32,
-                   f32 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_64B))
-      return cudaErrorInvalidValue;
-  } else {
-    td = ta;  // not read
-  }
   for (int h = 0; h < kMaxHeads; ++h) {
     if (h >= a.n_heads) {
       tb[h] = tb[0];
@@ -369,6 +359,23 @@ cudaError_t launch_gemm_cfg(const Operand& A, const Operand* B, const GemmArgs& 
     }
     if (!encode_2d(&tb[h], B[h].base, B[h].rows, B[h].cols, B[h].ld, kBK, BMN ? 64 : C::kBRows))
       return cudaErrorInvalidValue;
+  }
+  // 32 x 32 boxes: 64-byte bf16 rows in the 64-byte swizzle, 128-byte fp32 rows in the 128-byte one
+  auto out_map = [](CUtensorMap* m, const OutMat* o, bool f32) {
+    return o && aligned(o->base, 16) &&
+           encode_2d(m, o->base, o->rows, o->cols, o->ld, 32, 32, f32,
+                     f32 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_64B);
+  };
+  if (E == kEpiAdam) {
+    // D[0..3]: fp32 weights (the output map), first and second moments, bf16
+    // weights; the moments and the bf16 weights ride in the unused B slots 1..3
+    if (a.n_heads != 1 || !D || !out_map(&td, &D[0], true) || !out_map(&tb[1], &D[1], true) ||
+        !out_map(&tb[2], &D[2], true) || !out_map(&tb[3], &D[3], false))
+      return cudaErrorInvalidValue;
+  } else if (EpiShape<E>::kTmaOut) {
+    if (!out_map(&td, D, E == kEpiF32)) return cudaErrorInvalidValue;
+  } else {
+    td = ta;  // not read
   }
   const int64_t n_tiles = (a.N + kTileN - 1) / kTileN;
   const int64_t units = ((max_m_rows + C::kTileM - 1) / C::kTileM) *
@@ -788,7 +795,7 @@ grpo_status loss_impl(const uint16_t* H, const uint16_t* W, const int32_t* targe
     resp_len_kernel<<<static_cast<unsigned>(blocks), 256, 0, s>>>(mask, n_resp, L, at<int>(ws, Ly.resp_len));
     e = cudaGetLastError();
   }
-  if (e == cudaSuccess && !adam) {
+  if (e == cudaSuccess) {
     TraceScope trace(GRPO_K_TRANSPOSE, 0, s);
     const int tb = static_cast<int>(std::min<int64_t>(Ly.T_pad / 64 * (Hd / 64), int64_t(sms) * 8));
     transpose_rows_kernel<<<tb, 256, 0, s>>>(at<uint16_t>(ws, Ly.Hc), n_valid, Hd, Ly.T_pad,
@@ -876,16 +883,16 @@ grpo_status loss_impl(const uint16_t* H, const uint16_t* W, const int32_t* targe
       w.group_m = group_m(3, di);
       l2_hints(3, &w.a_hint, &w.b_hint);
       w.status = status;
-      w.ldo = Hd;
       w.accumulate = 0;
       const OutMat outDw{dW + c0 * Hd, static_cast<uint64_t>(width), hd, hd};
       TraceScope trace(GRPO_K_DW_GEMM, width, s);
       if (adam) {
         const int64_t off = c0 * Hd;
-        w.master = adam->master + off;
-        w.exp_avg = adam->exp_avg + off;
-        w.exp_avg_sq = adam->exp_avg_sq + off;
-        w.w_out = adam->w_out + off;
+        const uint64_t wd = static_cast<uint64_t>(width);
+        const OutMat adam_maps[4] = {{adam->master + off, wd, hd, hd},
+                                     {adam->exp_avg + off, wd, hd, hd},
+                                     {adam->exp_avg_sq + off, wd, hd, hd},
+                                     {adam->w_out + off, wd, hd, hd}};
         w.adam_b1 = adam->b1;
         w.adam_b2 = adam->b2;
         w.adam_eps = adam->eps;
@@ -893,7 +900,7 @@ grpo_status loss_impl(const uint16_t* H, const uint16_t* W, const int32_t* targe
         w.adam_decay = adam->decay;
         w.adam_bc1 = adam->bc1;
         w.adam_bc2 = adam->bc2;
-        e = launch_gemm<kEpiAdam, true, true>(opDz, opHc, w, width, di, s);
+        e = launch_gemm<kEpiAdam, true, false>(opDz, opHcT, w, width, di, s, adam_maps);
       } else {
         e = launch_gemm<kEpiF32, true, false>(opDz, opHcT, w, width, di, s, &outDw);
       }

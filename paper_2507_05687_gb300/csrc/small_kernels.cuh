@@ -431,10 +431,19 @@ __global__ void dh_rows_kernel(const int* __restrict__ rank_of, int64_t T, int H
     const int r = rank_of[t];
     float4* row = reinterpret_cast<float4*>(dH + t * Hd);
     if (r < 0) {
-      for (int j = lane; j < vec; j += 32) row[j] = make_float4(0.f, 0.f, 0.f, 0.f);
+      for (int j = lane; j < vec; j += 32) __stcs(row + j, make_float4(0.f, 0.f, 0.f, 0.f));
     } else {
       const float4* src = reinterpret_cast<const float4*>(dHc + static_cast<int64_t>(r) * Hd);
-      for (int j = lane; j < vec; j += 32) row[j] = __ldcs(src + j);
+      int j = lane;
+      for (; j + 96 < vec; j += 128) {  // four 16-byte loads in flight per lane
+        const float4 a = __ldcs(src + j), b = __ldcs(src + j + 32), c = __ldcs(src + j + 64),
+                     d = __ldcs(src + j + 96);
+        __stcs(row + j, a);
+        __stcs(row + j + 32, b);
+        __stcs(row + j + 64, c);
+        __stcs(row + j + 96, d);
+      }
+      for (; j < vec; j += 32) __stcs(row + j, __ldcs(src + j));
     }
   }
 }
