@@ -35,11 +35,14 @@
 //            offset), key = seed); the logits never leave the SM.
 //   kEpiAdam dW = dZ^T H consumed in place by an AdamW step on the matching
 //            LM-head rows (fp32 master, both moments, bf16 weights out), so
-//            dW itself is never stored.
+//            dW itself is never stored; the weights and moments move through
+//            shared memory with TMA loads and stores, 32 x 32 blocks per warp.
 //
 // Operands may be K-major (rows of the matrix run along K) or MN-major (rows
-// run along M or N); the MN-major forms let dH and dW read W, H and dZ in the
-// layout they already have, with no transposed copies.
+// run along M or N); the MN-major forms let dH read W and dW read dZ in the
+// layout they already have.  dW's other operand is a transposed copy of the
+// gathered hidden states (K-major), which measured faster than reading them
+// MN-major.
 #pragma once
 
 #include <cuda.h>
