@@ -113,12 +113,11 @@ bool get_encode() {
   return g_encode != nullptr;
 }
 
-// 2D bf16 tensor map over a row-major [rows x cols] matrix; the box is
-// box_cols (inner, 64 = 128 bytes) x box_rows with the 128-byte swizzle.
-// Out-of-range elements of a box read as zero.
 // A 2-D tensor map over a row-major matrix [rows x cols] (leading dimension
-// ld elements): bf16 operands in the 128-byte swizzle by default; the output
-// maps of the epilogue use fp32 / the 64-byte swizzle as their boxes need.
+// ld elements) with boxes of box_cols (inner) x box_rows: bf16 operands in the
+// 128-byte swizzle by default (box_cols 64 = 128 bytes); the output maps of
+// the epilogues use fp32 / the 64-byte swizzle as their boxes need.
+// Out-of-range elements of a box read as zero and are not written.
 bool encode_2d(CUtensorMap* map, const void* base, uint64_t rows, uint64_t cols, uint64_t ld_elems,
                uint32_t box_cols, uint32_t box_rows, bool f32 = false,
                CUtensorMapSwizzle swizzle = CU_TENSOR_MAP_SWIZZLE_128B) {

@@ -52,7 +52,11 @@ def _run(w, Hb, Wb, y, m, old, ref, adv, theta0, m0, v0, in_place):
     return loss, dH, master, ea, eas, W_out
 
 
-def test_fused_adamw_matches_oracle(monkeypatch):
+@pytest.mark.parametrize("pair", ["1", "0"])
+def test_fused_adamw_matches_oracle(pair, monkeypatch):
+    """Both tile shapes (their operand rings differ: 5 stages of the pair tile,
+    3 of the single-CTA tile, to make room for the weight / moment blocks)."""
+    monkeypatch.setenv("GRPO_CTA_PAIR", pair)
     w, Hb, Wb, y, m, old, ref, adv, want, theta0, m0, v0 = _case(monkeypatch)
     loss, dH, master, ea, eas, W_out = _run(w, Hb, Wb, y, m, old, ref, adv, theta0, m0, v0, in_place=False)
     th_o, m_o, v_o = oracle.adamw_step(theta0, m0, v0, want["dW"], LR, B1, B2, EPS, WD, STEP)

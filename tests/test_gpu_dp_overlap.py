@@ -2,7 +2,7 @@
 and the data-parallel call that overlaps each chunk's dW all-reduce with the
 later chunks (paper_2507_05687_gb300.dp).
 
-The box has one GPU, so the collective runs in a one-rank NCCL group: the
+With one GPU, the collective runs in a one-rank NCCL group: the
 events, the communication stream and the NCCL calls are the real ones, and a
 one-rank sum must leave every bit of loss and dW unchanged.  The sharding and
 the global normaliser are covered by the two-rank gloo tests.
