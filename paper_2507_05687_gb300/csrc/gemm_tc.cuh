@@ -468,7 +468,9 @@ __device__ __forceinline__ void epi_end(const EpiRow& e, const GemmArgs& a, int 
 
 // ---------------------------------------------------------------- kernel body
 
-template <int kPair, int kEpi, bool kAmn, bool kBmn>
+// kBblk: B is K-major and stored in k-blocks [K / 64][N][64] (a 3-D tensor
+// map), so that one stage of B is a single contiguous run however long K is.
+template <int kPair, int kEpi, bool kAmn, bool kBmn, bool kBblk>
 __device__ __forceinline__ void gemm_body(const CUtensorMap* tmA, const CUtensorMap* const* tmBs,
                                           const CUtensorMap* tmD, const GemmArgs& args) {
   using C = TileCfg<kPair>;
@@ -578,6 +580,11 @@ __device__ __forceinline__ void gemm_body(const CUtensorMap* tmA, const CUtensor
               if (kPair == 2) tma_load_2d_pair_hint(dst, map, fb, c0, c1, pol);
               else tma_load_2d_hint(dst, map, fb, c0, c1, pol);
             };
+            auto load_blk = [&](uint32_t dst, const CUtensorMap* map, int row, int kblk, uint64_t pol) {
+              if (drop) return;
+              if (kPair == 2) tma_load_3d_pair_hint(dst, map, fb, 0, row, kblk, pol);
+              else tma_load_3d_hint(dst, map, fb, 0, row, kblk, pol);
+            };
             if (!kAmn) {
               load(sa, tmA, k0 + args.a_off_k, m0 + args.a_off_m, pol_a);
             } else {
@@ -585,7 +592,9 @@ __device__ __forceinline__ void gemm_body(const CUtensorMap* tmA, const CUtensor
               for (int j = 0; j < kRowsCta / 64; ++j)
                 load(sa + j * 8192, tmA, m0 + args.a_off_m + 64 * j, k0 + args.a_off_k, pol_a);
             }
-            if (!kBmn) {
+            if (!kBmn && kBblk) {
+              load_blk(sb, tmBs[head], n0 + args.b_off_n, (k0 + args.b_off_k) >> 6, pol_b);
+            } else if (!kBmn) {
               load(sb, tmBs[head], k0 + args.b_off_k, n0 + args.b_off_n, pol_b);
             } else {
 #pragma unroll
@@ -753,24 +762,24 @@ __device__ __forceinline__ void gemm_body(const CUtensorMap* tmA, const CUtensor
 }
 
 // One tensor map per B matrix; B1..B3 are read only when args.n_heads > 1.
-template <int kEpi, bool kAmn, bool kBmn>
+template <int kEpi, bool kAmn, bool kBmn, bool kBblk = false>
 __global__ void __launch_bounds__(EpiShape<kEpi>::kThreads, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB0,
                    const __grid_constant__ CUtensorMap tmB1, const __grid_constant__ CUtensorMap tmB2,
                    const __grid_constant__ CUtensorMap tmB3, const __grid_constant__ CUtensorMap tmD,
                    const GemmArgs args) {
   const CUtensorMap* tmBs[kMaxHeads] = {&tmB0, &tmB1, &tmB2, &tmB3};
-  gemm_body<1, kEpi, kAmn, kBmn>(&tmA, tmBs, &tmD, args);
+  gemm_body<1, kEpi, kAmn, kBmn, kBblk>(&tmA, tmBs, &tmD, args);
 }
 
-template <int kEpi, bool kAmn, bool kBmn>
+template <int kEpi, bool kAmn, bool kBmn, bool kBblk = false>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(EpiShape<kEpi>::kThreads, 1)
     gemm_tc_pair_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB0,
                         const __grid_constant__ CUtensorMap tmB1, const __grid_constant__ CUtensorMap tmB2,
                         const __grid_constant__ CUtensorMap tmB3, const __grid_constant__ CUtensorMap tmD,
                         const GemmArgs args) {
   const CUtensorMap* tmBs[kMaxHeads] = {&tmB0, &tmB1, &tmB2, &tmB3};
-  gemm_body<2, kEpi, kAmn, kBmn>(&tmA, tmBs, &tmD, args);
+  gemm_body<2, kEpi, kAmn, kBmn, kBblk>(&tmA, tmBs, &tmD, args);
 }
 
 }  // namespace grpo

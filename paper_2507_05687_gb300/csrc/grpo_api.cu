@@ -10,6 +10,7 @@
 #include <cstdlib>
 #include <cstring>
 #include <mutex>
+#include <type_traits>
 #include <vector>
 
 #include "../../include/grpo.h"
@@ -20,7 +21,13 @@ using namespace grpo;
 
 namespace {
 
-constexpr int kLseTilesPerUnit = 16;     // vocabulary tiles (of 256) per forward work unit
+constexpr int kLseTilesPerUnit = 16;
+// Longest row of the transposed hidden states kept as plain rows.  Past it a
+// GEMM stage (128 rows of 128 bytes) would touch one 2 MB page per row; the
+// k-block layout keeps a stage contiguous.  Measured on the dW GEMM: plain rows
+// faster at 64 KB and 512 KB rows (14.6 vs 15.7 ms and 128.7 vs 140.6 ms per
+// step), k-blocks faster at 2 MB rows (147.6 vs 190.4 ms).
+constexpr int64_t kMaxTransposedRowBytes = int64_t(1) << 20;     // vocabulary tiles (of 256) per forward work unit
 constexpr int kLossThreads = 256;
 constexpr int64_t kDefaultVocabChunk = 16384;
 
@@ -87,7 +94,8 @@ bool make_layout(int64_t T, int32_t Hd, int64_t V, int32_t which, Layout* L) {
   L->best_c = take(best, 256);
   L->best_z = take(best, 256);
   L->Hc = take(2 * tp * static_cast<size_t>(Hd), 1024);
-  // H_c transposed [Hd x T_pad]: the K-major B operand of the dW GEMM
+  // H_c transposed (rows [Hd x T_pad], or k-blocks [T_pad / 64][Hd][64] when a
+  // row would exceed kMaxTransposedRowBytes): the K-major B operand of the dW GEMM
   L->HcT = which == GRPO_WS_LOSS ? take(2 * tp * static_cast<size_t>(Hd), 1024) : off;
   L->dz = which == GRPO_WS_LOSS ? take(2 * tp * static_cast<size_t>(L->vchunk), 1024) : off;
   // dH over the compacted rows, accumulated across vocabulary chunks
@@ -131,17 +139,31 @@ bool encode_2d(CUtensorMap* map, const void* base, uint64_t rows, uint64_t cols,
   return r == CUDA_SUCCESS;
 }
 
+// A 3-D tensor map over a bf16 operand stored in k-blocks [K / 64][rows][64]
+// (64 contiguous K elements per row of a block): the box is 64 x box_rows x 1
+// in the 128-byte swizzle, the same shared-memory tile as the 2-D K-major box.
+bool encode_blk(CUtensorMap* map, const void* base, uint64_t rows, uint64_t k, uint32_t box_rows) {
+  const cuuint64_t dims[3] = {64, rows, k / 64};
+  const cuuint64_t strides[2] = {64 * 2, rows * 64 * 2};
+  const cuuint32_t box[3] = {64, box_rows, 1};
+  const cuuint32_t estr[3] = {1, 1, 1};
+  const CUresult r = g_encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides, box,
+                              estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
 struct DeviceInfo {
   int sms = 0;
   int pairs = 0;  // CTA pairs of the pair kernels that can be resident at once
   bool ok = false;
 };
 
-template <int E, bool A, bool B>
+template <int E, bool A, bool B, bool BLK = false>
 bool prepare_kernels(int* pairs) {
-  if (cudaFuncSetAttribute(gemm_tc_kernel<E, A, B>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+  if (cudaFuncSetAttribute(gemm_tc_kernel<E, A, B, BLK>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                            smem_bytes<1, E>()) != cudaSuccess ||
-      cudaFuncSetAttribute(gemm_tc_pair_kernel<E, A, B>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+      cudaFuncSetAttribute(gemm_tc_pair_kernel<E, A, B, BLK>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                            smem_bytes<2, E>()) != cudaSuccess)
     return false;
   cudaLaunchConfig_t cfg = {};
@@ -149,7 +171,7 @@ bool prepare_kernels(int* pairs) {
   cfg.blockDim = dim3(EpiShape<E>::kThreads, 1, 1);
   cfg.dynamicSmemBytes = smem_bytes<2, E>();
   int n = 0;
-  if (cudaOccupancyMaxActiveClusters(&n, gemm_tc_pair_kernel<E, A, B>, &cfg) != cudaSuccess) {
+  if (cudaOccupancyMaxActiveClusters(&n, gemm_tc_pair_kernel<E, A, B, BLK>, &cfg) != cudaSuccess) {
     cudaGetLastError();  // clear: without the query the single-CTA tiles are used
     n = 0;
   }
@@ -173,6 +195,7 @@ bool device_info(DeviceInfo* out) {
     if (major != 10 || minor != 3) return false;
     if (!prepare_kernels<kEpiLse, false, false>(&pairs) || !prepare_kernels<kEpiDz, false, false>(&pairs) ||
         !prepare_kernels<kEpiF32, false, true>(&pairs) || !prepare_kernels<kEpiF32, true, false>(&pairs) ||
+        !prepare_kernels<kEpiF32, true, false, true>(&pairs) || !prepare_kernels<kEpiAdam, true, false, true>(&pairs) ||
         !prepare_kernels<kEpiAdam, true, false>(&pairs) || !prepare_kernels<kEpiSample, false, false>(&pairs))
       return false;
     cache[dev].sms = sms;
@@ -208,6 +231,17 @@ void l2_hints(int which, int* a_hint, int* b_hint) {
   }
   *a_hint = h[2 * which];
   *b_hint = h[2 * which + 1];
+}
+
+// Layout of the transposed hidden states for T_pad tokens: k-blocks when a
+// plain row would be longer than kMaxTransposedRowBytes;
+// GRPO_HCT_LAYOUT=rows|blocks forces one (the tests cover both on small sizes).
+bool hct_blocks(int64_t T_pad) {
+  if (const char* e = std::getenv("GRPO_HCT_LAYOUT")) {
+    if (std::strcmp(e, "rows") == 0) return false;
+    if (std::strcmp(e, "blocks") == 0) return true;
+  }
+  return T_pad * 2 > kMaxTransposedRowBytes;
 }
 
 // 2-CTA (cta_group::2) tiles unless GRPO_CTA_PAIR=0.
@@ -326,10 +360,13 @@ CopyOut* copy_out_for_device() {
 
 bool aligned(const void* p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
 
-// A bf16 row-major matrix [rows x cols] with leading dimension ld (elements).
+// A bf16 row-major matrix [rows x cols] with leading dimension ld (elements),
+// or, with blk, a K-major operand of `rows` rows and `cols` = K stored in
+// k-blocks [cols / 64][rows][64] (ld unused; cols a multiple of 64).
 struct Operand {
   const void* base;
   uint64_t rows, cols, ld;
+  bool blk = false;
 };
 
 // The output of a kEpiDz (bf16) or kEpiF32 (fp32) GEMM: a row-major matrix
@@ -349,6 +386,10 @@ cudaError_t launch_gemm_cfg(const Operand& A, const Operand* B, const GemmArgs& 
   using C = TileCfg<kPair>;
   GemmArgs a = args;
   a.n_heads = std::max(1, std::min(a.n_heads, kMaxHeads));
+  // the k-block form of B exists only for the dW GEMMs (fp32 output or the AdamW step)
+  constexpr bool kBlkOk = !BMN && (E == kEpiF32 || E == kEpiAdam);
+  const bool blk = B[0].blk;
+  if (blk && !kBlkOk) return cudaErrorInvalidValue;
   CUtensorMap ta, tb[kMaxHeads], td;
   if (!encode_2d(&ta, A.base, A.rows, A.cols, A.ld, kBK, AMN ? 64 : kRowsCta)) return cudaErrorInvalidValue;
   for (int h = 0; h < kMaxHeads; ++h) {
@@ -356,8 +397,9 @@ cudaError_t launch_gemm_cfg(const Operand& A, const Operand* B, const GemmArgs& 
       tb[h] = tb[0];
       continue;
     }
-    if (!encode_2d(&tb[h], B[h].base, B[h].rows, B[h].cols, B[h].ld, kBK, BMN ? 64 : C::kBRows))
-      return cudaErrorInvalidValue;
+    const bool ok = B[h].blk ? !BMN && encode_blk(&tb[h], B[h].base, B[h].rows, B[h].cols, C::kBRows)
+                             : encode_2d(&tb[h], B[h].base, B[h].rows, B[h].cols, B[h].ld, kBK, BMN ? 64 : C::kBRows);
+    if (!ok) return cudaErrorInvalidValue;
   }
   // 32 x 32 boxes: 64-byte bf16 rows in the 64-byte swizzle, 128-byte fp32 rows in the 128-byte one
   auto out_map = [](CUtensorMap* m, const OutMat* o, bool f32) {
@@ -379,14 +421,23 @@ cudaError_t launch_gemm_cfg(const Operand& A, const Operand* B, const GemmArgs& 
   const int64_t n_tiles = (a.N + kTileN - 1) / kTileN;
   const int64_t units = ((max_m_rows + C::kTileM - 1) / C::kTileM) *
                         ((n_tiles + a.n_per_unit - 1) / a.n_per_unit) * a.n_heads;
-  if (kPair == 2) {
-    const int64_t pairs = std::max<int64_t>(1, std::min<int64_t>(di.pairs, units));
-    gemm_tc_pair_kernel<E, AMN, BMN><<<static_cast<unsigned>(2 * pairs), EpiShape<E>::kThreads,
-                                       smem_bytes<2, E>(), s>>>(ta, tb[0], tb[1], tb[2], tb[3], td, a);
+  const unsigned grid = static_cast<unsigned>(
+      kPair == 2 ? 2 * std::max<int64_t>(1, std::min<int64_t>(di.pairs, units))
+                 : std::max<int64_t>(1, std::min<int64_t>(di.sms, units)));
+  auto go = [&](auto blk_tag) {
+    constexpr bool BLK = decltype(blk_tag)::value;
+    if (kPair == 2)
+      gemm_tc_pair_kernel<E, AMN, BMN, BLK><<<grid, EpiShape<E>::kThreads, smem_bytes<2, E>(), s>>>(
+          ta, tb[0], tb[1], tb[2], tb[3], td, a);
+    else
+      gemm_tc_kernel<E, AMN, BMN, BLK><<<grid, EpiShape<E>::kThreads, smem_bytes<1, E>(), s>>>(
+          ta, tb[0], tb[1], tb[2], tb[3], td, a);
+  };
+  if constexpr (kBlkOk) {
+    if (blk) go(std::true_type{});
+    else go(std::false_type{});
   } else {
-    const int64_t grid = std::max<int64_t>(1, std::min<int64_t>(di.sms, units));
-    gemm_tc_kernel<E, AMN, BMN><<<static_cast<unsigned>(grid), EpiShape<E>::kThreads, smem_bytes<1, E>(), s>>>(
-        ta, tb[0], tb[1], tb[2], tb[3], td, a);
+    go(std::false_type{});
   }
   return cudaGetLastError();
 }
@@ -794,10 +845,11 @@ grpo_status loss_impl(const uint16_t* H, const uint16_t* W, const int32_t* targe
     resp_len_kernel<<<static_cast<unsigned>(blocks), 256, 0, s>>>(mask, n_resp, L, at<int>(ws, Ly.resp_len));
     e = cudaGetLastError();
   }
+  const bool hct_blk = hct_blocks(Ly.T_pad);
   if (e == cudaSuccess) {
     TraceScope trace(GRPO_K_TRANSPOSE, 0, s);
     const int tb = static_cast<int>(std::min<int64_t>(Ly.T_pad / 64 * (Hd / 64), int64_t(sms) * 8));
-    transpose_rows_kernel<<<tb, 256, 0, s>>>(at<uint16_t>(ws, Ly.Hc), n_valid, Hd, Ly.T_pad,
+    transpose_rows_kernel<<<tb, 256, 0, s>>>(at<uint16_t>(ws, Ly.Hc), n_valid, Hd, hct_blk ? 0 : Ly.T_pad,
                                              at<uint16_t>(ws, Ly.HcT));
     e = cudaGetLastError();
   }
@@ -831,7 +883,7 @@ grpo_status loss_impl(const uint16_t* H, const uint16_t* W, const int32_t* targe
   const int64_t vc = Ly.vchunk;
   const uint64_t tp = static_cast<uint64_t>(Ly.T_pad), hd = static_cast<uint64_t>(Hd);
   const Operand opHc{Hc, tp, hd, hd};
-  const Operand opHcT{at<uint16_t>(ws, Ly.HcT), hd, tp, tp};
+  const Operand opHcT{at<uint16_t>(ws, Ly.HcT), hd, tp, tp, hct_blk};
   const Operand opW{W, static_cast<uint64_t>(V), hd, hd};
   const Operand opDz{dz, tp, static_cast<uint64_t>(vc), static_cast<uint64_t>(vc)};
   const OutMat outDz{dz, tp, static_cast<uint64_t>(vc), static_cast<uint64_t>(vc)};

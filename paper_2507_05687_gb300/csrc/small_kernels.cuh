@@ -386,10 +386,12 @@ __global__ void adamw_kernel(float* __restrict__ theta, float* __restrict__ m, f
   }
 }
 
-// HcT[k][r] = Hc[r][k] for r < round_up(n_valid, 256) (the rows the token
-// K-loop of the dW GEMM can reach, zero past n_valid): the K-major copy of the
-// gathered hidden states.  64 x 64 tiles through shared memory, 32-bit words
-// (two bf16) on both the read and the write side.
+// The K-major copy of the gathered hidden states for the dW GEMM, for the
+// rows r < round_up(n_valid, 256) that the token K-loop can reach (zero past
+// n_valid): with ld_t > 0 plain rows, HcT[k][r] = Hc[r][k] (row stride ld_t);
+// with ld_t == 0 k-blocks of 64 tokens, HcT[r / 64][k][r % 64] = Hc[r][k], where
+// a GEMM stage is one contiguous run however long the rows are.  64 x 64 tiles
+// through shared memory, 32-bit words (two bf16) on both sides.
 __global__ void transpose_rows_kernel(const uint16_t* __restrict__ Hc, const int* __restrict__ n_valid_p, int Hd,
                                       int64_t ld_t, uint16_t* __restrict__ HcT) {
   __shared__ uint16_t tile[64][66];
@@ -411,10 +413,12 @@ __global__ void transpose_rows_kernel(const uint16_t* __restrict__ Hc, const int
     }
     __syncthreads();
 #pragma unroll
-    for (int k = 0; k < 8; ++k) {  // output rows c0 + q + 8k, columns r0 + 2w, 2w + 1
+    for (int k = 0; k < 8; ++k) {  // rows c0 + q + 8k, tokens r0 + 2w, 2w + 1
       const int c = q + 8 * k;
       const uint32_t v = static_cast<uint32_t>(tile[2 * w][c]) | (static_cast<uint32_t>(tile[2 * w + 1][c]) << 16);
-      *reinterpret_cast<uint32_t*>(HcT + static_cast<int64_t>(c0 + c) * ld_t + r0 + 2 * w) = v;
+      const int64_t at = ld_t > 0 ? static_cast<int64_t>(c0 + c) * ld_t + r0 + 2 * w
+                                  : static_cast<int64_t>(r0) * Hd + static_cast<int64_t>(c0 + c) * 64 + 2 * w;
+      *reinterpret_cast<uint32_t*>(HcT + at) = v;
     }
     __syncthreads();
   }

@@ -155,6 +155,16 @@ def test_ragged_multi_chunk_fwd_bwd(agg_mode, monkeypatch):
     _check_fwd_bwd(_case(w, agg_mode), agg_mode)
 
 
+@pytest.mark.parametrize("layout", ["rows", "blocks"])
+def test_transposed_hidden_state_layouts(layout, monkeypatch):
+    """dW reads the gathered hidden states transposed, as plain rows or in
+    64-token k-blocks (chosen by length; forced here on a small ragged case)."""
+    monkeypatch.setenv("GRPO_HCT_LAYOUT", layout)
+    monkeypatch.setenv("GRPO_VOCAB_CHUNK", "768")
+    w = wl.Workload("t", 3, 4, 60, 192, 2100, "uniform", 1, 60, rewards="mix", seed=wl.SEED_BASE + 560)
+    _check_fwd_bwd(_case(w))
+
+
 @pytest.mark.parametrize("pair", ["0", "1"])
 def test_single_and_paired_tiles_agree(pair, monkeypatch):
     """The 128x256 single-CTA tile and the 256x256 CTA-pair tile both meet the bar."""
