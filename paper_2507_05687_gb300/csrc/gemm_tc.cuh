@@ -119,6 +119,8 @@ struct GemmArgs {
   unsigned long long wait_ns;  // bound of every pipeline wait (0: kWaitLimitNs)
   int drop_kblock1;     // fault-injection test hook: CTA 0 skips the copies of its
                         // k-block number drop_kblock1 - 1 (0: never), so a wait runs out
+  int drop_adam1;       // the same for kEpiAdam: CTA 0's epilogue warp 0 skips the loads of
+                        // its weight block number drop_adam1 - 1 (0: never)
 
   // kEpiLse
   const int* yc;        // [M] target of each compacted row (-1: none)
@@ -251,6 +253,8 @@ struct OutStage {
   uint32_t ld_phase;
   volatile int* abort;
   unsigned long long wlim;
+  int blocks_loaded;         // kEpiAdam blocks this warp has loaded (fault-injection hook)
+  bool first_warp;           // epilogue warp 0 of CTA 0 (fault-injection hook)
 };
 
 // Writes this warp's 32 x 32 output block (lane = row, `words` = the row's 64
@@ -294,9 +298,13 @@ __device__ __forceinline__ bool adam_block(OutStage& o, const float* g, int x, i
   if (o.lane == 0) {
     bulk_wait_read_0();  // the previous block's stores have read the buffer
     mbar_arrive_expect_tx(o.ld_bar, 3 * 4096);
-    tma_load_2d(th, o.map, o.ld_bar, x, y);
-    tma_load_2d(mo, o.m_map, o.ld_bar, x, y);
-    tma_load_2d(ve, o.v_map, o.ld_bar, x, y);
+    // the test hook: these bytes never arrive, so the wait below runs out
+    const bool drop = o.first_warp && ++o.blocks_loaded == a.drop_adam1;
+    if (!drop) {
+      tma_load_2d(th, o.map, o.ld_bar, x, y);
+      tma_load_2d(mo, o.m_map, o.ld_bar, x, y);
+      tma_load_2d(ve, o.v_map, o.ld_bar, x, y);
+    }
   }
   const bool got = mbar_wait(o.ld_bar, o.ld_phase, o.abort, o.wlim);
   o.ld_phase ^= 1u;
@@ -699,7 +707,9 @@ __device__ __forceinline__ void gemm_body(const CUtensorMap* tmA, const CUtensor
                 smem_addr(&ld_bar[kEpi == kEpiAdam ? warp - 2 : 0]),
                 0u,
                 abort_flag,
-                wlim};
+                wlim,
+                0,
+                blockIdx.x == 0 && warp == 2};
     int tile = 0;
     bool ok = true;
     for (int u = unit0; u < sch.total && ok; u += unit_stride) {

@@ -944,6 +944,13 @@ grpo_status loss_impl(const uint16_t* H, const uint16_t* W, const int32_t* targe
                                      {adam->exp_avg + off, wd, hd, hd},
                                      {adam->exp_avg_sq + off, wd, hd, hd},
                                      {adam->w_out + off, wd, hd, hd}};
+        // fault-injection test hook: GRPO_TEST_DROP_ADAM=n makes CTA 0 skip the
+        // loads of its n-th weight block, so that wait runs out after 0.2 s and
+        // the call reports GRPO_ERR_TIMEOUT
+        if (const char* d = std::getenv("GRPO_TEST_DROP_ADAM")) {
+          w.drop_adam1 = std::atoi(d);
+          if (w.drop_adam1 > 0) w.wait_ns = 200000000ull;
+        }
         w.adam_b1 = adam->b1;
         w.adam_b2 = adam->b2;
         w.adam_eps = adam->eps;

@@ -39,7 +39,7 @@ def _case(monkeypatch, chunk="768"):
     return w, Hb, Wb, y, m, old, ref, adv, want, theta0, m0, v0
 
 
-def _run(w, Hb, Wb, y, m, old, ref, adv, theta0, m0, v0, in_place):
+def _run(w, Hb, Wb, y, m, old, ref, adv, theta0, m0, v0, in_place, ws=None):
     W = dev_tensor(Wb, torch.bfloat16)
     master, ea, eas = (torch.from_numpy(x.copy()).to(DEV) for x in (theta0, m0, v0))
     W_out = W if in_place else torch.empty_like(W)
@@ -47,7 +47,7 @@ def _run(w, Hb, Wb, y, m, old, ref, adv, theta0, m0, v0, in_place):
                                        dev_tensor(m, torch.uint8), dev_tensor(old, torch.float32),
                                        dev_tensor(ref, torch.float32), dev_tensor(adv, torch.float32), w.n_resp,
                                        w.L, master, ea, eas, STEP, lr=LR, betas=(B1, B2), eps=EPS,
-                                       weight_decay=WD, W_out=W_out)
+                                       weight_decay=WD, W_out=W_out, ws=ws)
     torch.cuda.synchronize()
     return loss, dH, master, ea, eas, W_out
 
@@ -130,3 +130,22 @@ def test_fused_equals_stored_dw_plus_separate_step(monkeypatch):
     grpo.adamw_step(master, ea, eas, dW, wout, STEP, lr=LR, betas=(B1, B2), eps=EPS, weight_decay=WD)
     for a, b in ((master_f, master), (ea_f, ea), (eas_f, eas)):
         torch.testing.assert_close(a, b, rtol=1e-6, atol=1e-9)
+
+
+@pytest.mark.parametrize("pair", ["1", "0"])
+def test_weight_block_wait_that_runs_out_reports_timeout(pair, monkeypatch):
+    """Failure detection of the fused step's own wait, without a fault: a test
+    hook (GRPO_TEST_DROP_ADAM) makes CTA 0 skip the loads of one weight block,
+    the bounded wait for them gives up (0.2 s), the call reports
+    GRPO_ERR_TIMEOUT, and the next call on the same context is correct."""
+    monkeypatch.setenv("GRPO_CTA_PAIR", pair)
+    w, Hb, Wb, y, m, old, ref, adv, want, theta0, m0, v0 = _case(monkeypatch)
+    ws = grpo.workspace(w.T, w.Hd, w.V, grpo.GRPO_WS_LOSS, DEV)
+    monkeypatch.setenv("GRPO_TEST_DROP_ADAM", "2")
+    _run(w, Hb, Wb, y, m, old, ref, adv, theta0, m0, v0, in_place=False, ws=ws)
+    assert grpo.check_device_status(ws) == grpo.GRPO_ERR_TIMEOUT
+    monkeypatch.delenv("GRPO_TEST_DROP_ADAM")
+    loss, dH, master, ea, eas, W_out = _run(w, Hb, Wb, y, m, old, ref, adv, theta0, m0, v0, in_place=False, ws=ws)
+    assert grpo.check_device_status(ws) == grpo.GRPO_OK
+    th_o, _, _ = oracle.adamw_step(theta0, m0, v0, want["dW"], LR, B1, B2, EPS, WD, STEP)
+    assert rel_fro(master.double().cpu().numpy() - theta0, th_o - theta0) <= GRAD_RTOL
