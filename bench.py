@@ -324,7 +324,7 @@ def main():
     from paper_2507_05687_gb300 import dp
 
     if sampling:
-        ws = grpo.workspace(w.T, w.Hd, w.V, grpo.GRPO_WS_SAMPLE, dev)
+        ws = grpo.workspace(w.T, w.Hd, w.V, grpo.GRPO_WS_SAMPLE, dev, max_valid=n_valid)
         tok_out = (torch.empty(w.T, dtype=torch.int32, device=dev), torch.empty(w.T, dtype=torch.float32, device=dev))
         draw = [0]
 
@@ -334,14 +334,14 @@ def main():
     elif scoring:
         heads = [W, to_dev(wl.gen_weight(w, "old", inp["W"]), torch.bfloat16),
                  to_dev(wl.gen_weight(w, "ref", inp["W"]), torch.bfloat16)]
-        ws = grpo.workspace(w.T, w.Hd, w.V, grpo.GRPO_WS_LOGPROBS_HEADS, dev)
+        ws = grpo.workspace(w.T, w.Hd, w.V, grpo.GRPO_WS_LOGPROBS_HEADS, dev, max_valid=n_valid)
         logp3 = torch.empty(len(heads), w.T, dtype=torch.float32, device=dev)
 
         def step():
             # policy / old / reference log-probs of one rollout batch; ranks score independently
             grpo.token_logprobs_heads(H, heads, y, m, ws=ws, out=logp3)
     else:
-        ws = grpo.workspace(w.T, w.Hd, w.V, grpo.GRPO_WS_LOSS, dev)
+        ws = grpo.workspace(w.T, w.Hd, w.V, grpo.GRPO_WS_LOSS, dev, max_valid=n_valid)
         adv = torch.empty(w.n_resp, dtype=torch.float32, device=dev)
         out = (torch.empty(1, dtype=torch.float32, device=dev),
                torch.empty(w.T, w.Hd, dtype=torch.float32, device=dev),
@@ -478,6 +478,8 @@ def measure_e2e_scoring(grpo, torch, dev, w, inp, heads, steps: int):
     """Public API, rollout scoring: H2D of the batch (H, targets, mask) from pinned host
     memory, the three LM heads resident on the device (model weights), D2H of the
     three log-prob rows."""
+    n_valid = int(inp["m"].sum())
+
     def pin(a, dt):
         return torch.from_numpy(np.ascontiguousarray(a)).view(dt).pin_memory()
 
@@ -485,7 +487,7 @@ def measure_e2e_scoring(grpo, torch, dev, w, inp, heads, steps: int):
     h2d = sum(t.numel() * t.element_size() for t in [hH, hy, hm])
     d2h = len(heads) * w.T * 4
     hout = torch.empty(len(heads), w.T, dtype=torch.float32).pin_memory()
-    ws = grpo.workspace(w.T, w.Hd, w.V, grpo.GRPO_WS_LOGPROBS_HEADS, dev)
+    ws = grpo.workspace(w.T, w.Hd, w.V, grpo.GRPO_WS_LOGPROBS_HEADS, dev, max_valid=n_valid)
 
     def one():
         lp = grpo.token_logprobs_heads(hH, heads, hy, hm, ws=ws)
@@ -509,6 +511,8 @@ def measure_e2e(grpo, torch, dev, w, inp, steps: int):
     log-probs, rewards) from pinned host memory, the LM head W resident on the
     device (the parameter being trained), D2H of the loss; dH and dW stay on the
     device, where the trunk's backward and the optimiser consume them."""
+    n_valid = int(inp["m"].sum())
+
     def pin(a, dt):
         return torch.from_numpy(np.ascontiguousarray(a)).view(dt).pin_memory()
 
@@ -519,7 +523,7 @@ def measure_e2e(grpo, torch, dev, w, inp, steps: int):
     d2h = 4
     out = (torch.empty(1, dtype=torch.float32, device=dev), torch.empty(w.T, w.Hd, dtype=torch.float32, device=dev),
            torch.empty(w.V, w.Hd, dtype=torch.float32, device=dev))
-    ws = grpo.workspace(w.T, w.Hd, w.V, grpo.GRPO_WS_LOSS, dev)
+    ws = grpo.workspace(w.T, w.Hd, w.V, grpo.GRPO_WS_LOSS, dev, max_valid=n_valid)
 
     def one():
         adv = grpo.group_advantages(hr.to(dev, non_blocking=True), w.G, w.adv_eps)
@@ -543,6 +547,8 @@ def measure_e2e(grpo, torch, dev, w, inp, steps: int):
 def measure_e2e_offload(grpo, torch, dev, w, inp, steps: int):
     """Public API with everything on the host (a host-offloaded head): H2D of the
     batch and of W, the step, D2H of loss, dH, dW (dW streamed chunk by chunk)."""
+    n_valid = int(inp["m"].sum())
+
     def pin(a, dt):
         t = torch.from_numpy(np.ascontiguousarray(a)).view(dt)
         return t.pin_memory()
@@ -556,7 +562,7 @@ def measure_e2e_offload(grpo, torch, dev, w, inp, steps: int):
     # the caller's own buffers, allocated once: pinned host outputs and a device workspace
     hout = (torch.empty(1, dtype=torch.float32).pin_memory(), torch.empty(w.T, w.Hd, dtype=torch.float32).pin_memory(),
             torch.empty(w.V, w.Hd, dtype=torch.float32).pin_memory())
-    ws = grpo.workspace(w.T, w.Hd, w.V, grpo.GRPO_WS_LOSS, dev)
+    ws = grpo.workspace(w.T, w.Hd, w.V, grpo.GRPO_WS_LOSS, dev, max_valid=n_valid)
 
     def one():
         adv = grpo.group_advantages(hr.to(dev, non_blocking=True), w.G, w.adv_eps)

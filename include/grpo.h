@@ -46,7 +46,9 @@ typedef enum {
   GRPO_ERR_CUDA = 3,          /* a CUDA runtime/driver call failed */
   GRPO_ERR_DEVICE_CHECK = 4,  /* device found a bad target index or a non-finite value */
   GRPO_ERR_TIMEOUT = 5,       /* a bounded device-side wait gave up; outputs are invalid */
-  GRPO_ERR_UNSUPPORTED = 6    /* device is not sm_103 / sm_100 class, or shape beyond limits */
+  GRPO_ERR_UNSUPPORTED = 6,   /* device is not sm_103 / sm_100 class, or shape beyond limits */
+  GRPO_ERR_CAPACITY = 7       /* more unmasked rows than the workspace was sized for
+                                 (grpo_workspace_bytes_rows); outputs are invalid */
 } grpo_status;
 
 /* Which call a workspace is sized for (grpo_workspace_bytes `which`). */
@@ -312,6 +314,23 @@ grpo_status grpo_token_logprobs_noalloc(const uint16_t* H, const uint16_t* W, co
  * arguments the calls would reject.  Sized for the worst case N_valid = T.
  */
 size_t grpo_workspace_bytes(int64_t T, int32_t Hd, int64_t V, int32_t which);
+
+/*
+ * Bytes of workspace for the call `which` on batches of T padded tokens of
+ * which at most max_valid are unmasked (e.g. a ragged rollout batch where most
+ * rows are padding): the regions that hold one row per unmasked token (the
+ * gathered hidden states and, for the loss, its transposed copy, the dZ chunk
+ * and the compacted dH) are sized for max_valid rounded up to 256 rows instead
+ * of T.  At the 1M-row ragged 8B batch (168k unmasked) the loss workspace
+ * shrinks from 69 GB to about 11 GB.  Every call accepts such a smaller
+ * workspace: it derives the row capacity from ws_bytes.  A batch with more
+ * unmasked rows than the capacity is not an error the host can see (the count
+ * is only known on the device): the device status becomes GRPO_ERR_CAPACITY,
+ * rows past the capacity get no output (0 / token -1), and every other output
+ * of that call is invalid.  Returns 0 for arguments the calls would reject
+ * or a negative max_valid; max_valid >= T gives grpo_workspace_bytes.
+ */
+size_t grpo_workspace_bytes_rows(int64_t T, int64_t max_valid, int32_t Hd, int64_t V, int32_t which);
 
 /*
  * Synchronises `stream`, reads the device status word of workspace `ws`

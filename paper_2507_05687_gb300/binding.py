@@ -27,6 +27,7 @@ GRPO_ERR_CUDA = 3
 GRPO_ERR_DEVICE_CHECK = 4
 GRPO_ERR_TIMEOUT = 5
 GRPO_ERR_UNSUPPORTED = 6
+GRPO_ERR_CAPACITY = 7
 GRPO_WS_LOGPROBS = 0
 GRPO_WS_LOSS = 1
 GRPO_WS_LOGPROBS_HEADS = 2
@@ -63,6 +64,7 @@ SIGNATURES = {
     "grpo_adamw_step": (ctypes.c_int, [_P, _P, _P, _P, _P, _I64, _F, _F, _F, _F, _F, _I64, _P]),
     "grpo_token_logprobs_noalloc": (ctypes.c_int, [_P, _P, _P, _P, _I64, _I32, _I64, _P, _P]),
     "grpo_workspace_bytes": (ctypes.c_size_t, [_I64, _I32, _I64, _I32]),
+    "grpo_workspace_bytes_rows": (ctypes.c_size_t, [_I64, _I64, _I32, _I64, _I32]),
     "grpo_check_device_status": (ctypes.c_int, [_P, _P]),
     "grpo_status_string": (ctypes.c_char_p, [ctypes.c_int]),
     "grpo_trace_enable": (ctypes.c_int, [_I32]),
@@ -147,9 +149,15 @@ def workspace_bytes(T: int, Hd: int, V: int, which: int) -> int:
     return int(load().grpo_workspace_bytes(int(T), int(Hd), int(V), int(which)))
 
 
-def workspace(T: int, Hd: int, V: int, which: int, device=None) -> torch.Tensor:
-    """A device byte tensor large enough for the call `which`."""
-    n = workspace_bytes(T, Hd, V, which)
+def workspace_bytes_rows(T: int, max_valid: int, Hd: int, V: int, which: int) -> int:
+    """grpo_workspace_bytes_rows: scratch bytes for batches with at most max_valid unmasked rows."""
+    return int(load().grpo_workspace_bytes_rows(int(T), int(max_valid), int(Hd), int(V), int(which)))
+
+
+def workspace(T: int, Hd: int, V: int, which: int, device=None, max_valid: Optional[int] = None) -> torch.Tensor:
+    """A device byte tensor large enough for the call `which` (for batches with at
+    most max_valid unmasked rows when given)."""
+    n = workspace_bytes(T, Hd, V, which) if max_valid is None else workspace_bytes_rows(T, max_valid, Hd, V, which)
     if n == 0:
         raise GrpoError(GRPO_ERR_INVALID_ARG, "grpo_workspace_bytes")
     return torch.empty(n, dtype=torch.uint8, device=device or "cuda")

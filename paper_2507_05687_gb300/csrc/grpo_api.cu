@@ -45,14 +45,17 @@ int64_t vocab_chunk(int64_t V) {
 }
 
 // Workspace layout (byte offsets); every region is 256-byte aligned, the
-// bf16 matrices 1024-byte aligned.
+// bf16 matrices 1024-byte aligned.  Regions indexed by token position hold
+// T_pad rows; regions indexed by compacted (unmasked) row hold `rows`, the
+// row capacity: T_pad for a full workspace, less for one sized by
+// grpo_workspace_bytes_rows for batches with few unmasked rows.
 struct Layout {
-  int64_t T_pad, nsplit, nblk_scan, nblk_loss, vchunk;
+  int64_t T_pad, rows, nsplit, nblk_scan, nblk_loss, vchunk;
   size_t status, n_valid, counts, offsets, cidx, rank_of, yc, zy, part_m, part_s, lse_c, g_c,
       block_loss, resp_len, best_s, best_c, best_z, Hc, HcT, dz, dhc, total;
 };
 
-bool make_layout(int64_t T, int32_t Hd, int64_t V, int32_t which, Layout* L) {
+bool make_layout(int64_t T, int32_t Hd, int64_t V, int32_t which, Layout* L, int64_t rows_cap = -1) {
   if (T < 0 || T >= (int64_t(1) << 31) || Hd <= 0 || Hd % 64 != 0 || V <= 0 ||
       V >= (int64_t(1) << 31) ||
       (which != GRPO_WS_LOGPROBS && which != GRPO_WS_LOSS && which != GRPO_WS_LOGPROBS_HEADS &&
@@ -64,8 +67,9 @@ bool make_layout(int64_t T, int32_t Hd, int64_t V, int32_t which, Layout* L) {
   // partial (max, sum) entries per row: one per vocabulary split and column half
   L->nsplit = (vtiles + kLseTilesPerUnit - 1) / kLseTilesPerUnit *
               (which == GRPO_WS_SAMPLE ? EpiShape<kEpiSample>::kHalves : EpiShape<kEpiLse>::kHalves);
+  L->rows = rows_cap < 0 ? L->T_pad : std::min(L->T_pad, round_up(std::max<int64_t>(rows_cap, 1), kRowAlign));
   L->nblk_scan = (std::max<int64_t>(T, 1) + kScanChunk - 1) / kScanChunk;
-  L->nblk_loss = (L->T_pad + kLossThreads - 1) / kLossThreads;
+  L->nblk_loss = (L->rows + kLossThreads - 1) / kLossThreads;
   L->vchunk = which == GRPO_WS_LOSS ? vocab_chunk(V) : 0;
   size_t off = 0;
   auto take = [&](size_t bytes, size_t align) {
@@ -74,34 +78,57 @@ bool make_layout(int64_t T, int32_t Hd, int64_t V, int32_t which, Layout* L) {
     off += bytes;
     return at;
   };
-  const size_t tp = static_cast<size_t>(L->T_pad);
+  const size_t tp = static_cast<size_t>(L->T_pad);  // token rows
+  const size_t cr = static_cast<size_t>(L->rows);   // compacted rows
   L->status = take(4, 256);
   L->n_valid = take(4, 4);
   L->counts = take(4 * L->nblk_scan, 256);
   L->offsets = take(4 * L->nblk_scan, 256);
-  L->cidx = take(4 * tp, 256);
+  L->cidx = take(4 * cr, 256);
   L->rank_of = take(4 * tp, 256);
-  L->yc = take(4 * tp, 256);
-  L->zy = take(4 * tp * heads, 256);
-  L->part_m = take(4 * tp * L->nsplit * heads, 256);
-  L->part_s = take(4 * tp * L->nsplit * heads, 256);
-  L->lse_c = take(4 * tp, 256);
-  L->g_c = take(4 * tp, 256);
+  L->yc = take(4 * cr, 256);
+  L->zy = take(4 * cr * heads, 256);
+  L->part_m = take(4 * cr * L->nsplit * heads, 256);
+  L->part_s = take(4 * cr * L->nsplit * heads, 256);
+  L->lse_c = take(4 * cr, 256);
+  L->g_c = take(4 * cr, 256);
   L->block_loss = take(8 * L->nblk_loss, 256);
   L->resp_len = take(4 * tp, 256);
-  const size_t best = which == GRPO_WS_SAMPLE ? 4 * tp * L->nsplit : 0;
+  const size_t best = which == GRPO_WS_SAMPLE ? 4 * cr * L->nsplit : 0;
   L->best_s = take(best, 256);
   L->best_c = take(best, 256);
   L->best_z = take(best, 256);
-  L->Hc = take(2 * tp * static_cast<size_t>(Hd), 1024);
-  // H_c transposed (rows [Hd x T_pad], or k-blocks [T_pad / 64][Hd][64] when a
+  L->Hc = take(2 * cr * static_cast<size_t>(Hd), 1024);
+  // H_c transposed (rows [Hd x rows], or k-blocks [rows / 64][Hd][64] when a
   // row would exceed kMaxTransposedRowBytes): the K-major B operand of the dW GEMM
-  L->HcT = which == GRPO_WS_LOSS ? take(2 * tp * static_cast<size_t>(Hd), 1024) : off;
-  L->dz = which == GRPO_WS_LOSS ? take(2 * tp * static_cast<size_t>(L->vchunk), 1024) : off;
+  L->HcT = which == GRPO_WS_LOSS ? take(2 * cr * static_cast<size_t>(Hd), 1024) : off;
+  L->dz = which == GRPO_WS_LOSS ? take(2 * cr * static_cast<size_t>(L->vchunk), 1024) : off;
   // dH over the compacted rows, accumulated across vocabulary chunks
-  L->dhc = which == GRPO_WS_LOSS ? take(4 * tp * static_cast<size_t>(Hd), 1024) : off;
+  L->dhc = which == GRPO_WS_LOSS ? take(4 * cr * static_cast<size_t>(Hd), 1024) : off;
   L->total = (off + 1023) / 1024 * 1024;
   return true;
+}
+
+// The layout a call uses with a workspace of ws_bytes: the full one when it
+// fits, else the largest row capacity (a multiple of 256) that fits.  False
+// when the arguments are invalid or not even 256 rows fit.
+bool fit_layout(int64_t T, int32_t Hd, int64_t V, int32_t which, size_t ws_bytes, Layout* L) {
+  if (!make_layout(T, Hd, V, which, L)) return false;
+  if (ws_bytes >= L->total) return true;
+  int64_t lo = 0, hi = L->T_pad / kRowAlign;  // lo fits (0 = none found), hi does not
+  Layout t;
+  while (hi - lo > 1) {
+    const int64_t mid = (lo + hi) / 2;
+    make_layout(T, Hd, V, which, &t, mid * kRowAlign);
+    if (t.total <= ws_bytes) lo = mid;
+    else hi = mid;
+  }
+  if (lo == 0) {
+    make_layout(T, Hd, V, which, &t, kRowAlign);
+    if (t.total > ws_bytes) return false;
+    lo = 1;
+  }
+  return make_layout(T, Hd, V, which, L, lo * kRowAlign);
 }
 
 // ---------------------------------------------------------------- driver entry points
@@ -473,11 +500,12 @@ cudaError_t run_compaction(const uint16_t* H, const int32_t* targets, const uint
   if (T > 0) {
     const int nb = static_cast<int>(Ly.nblk_scan);
     mask_count_kernel<<<nb, kScanThreads, 0, s>>>(mask, T, at<int>(ws, Ly.counts));
-    count_scan_kernel<<<1, 1024, 0, s>>>(at<int>(ws, Ly.counts), nb, at<int>(ws, Ly.offsets), n_valid);
-    mask_scatter_kernel<<<nb, kScanThreads, 0, s>>>(mask, T, at<int>(ws, Ly.offsets),
+    count_scan_kernel<<<1, 1024, 0, s>>>(at<int>(ws, Ly.counts), nb, at<int>(ws, Ly.offsets), n_valid,
+                                         static_cast<int>(Ly.rows), status);
+    mask_scatter_kernel<<<nb, kScanThreads, 0, s>>>(mask, T, at<int>(ws, Ly.offsets), static_cast<int>(Ly.rows),
                                                       at<int>(ws, Ly.cidx), at<int>(ws, Ly.rank_of));
   }
-  const int64_t rows = Ly.T_pad;
+  const int64_t rows = Ly.rows;
   const int gblocks = static_cast<int>(std::max<int64_t>(1, std::min<int64_t>(rows / 8 + 1, sms * 8)));
   gather_rows_kernel<<<gblocks, 256, 0, s>>>(H, targets, at<int>(ws, Ly.cidx), n_valid, Hd, V,
                                              at<uint16_t>(ws, Ly.Hc), at<int>(ws, Ly.yc), status);
@@ -512,14 +540,14 @@ cudaError_t run_lse(const uint16_t* const* W, int n_heads, int32_t Hd, int64_t V
   a.part_m = at<float>(ws, Ly.part_m);
   a.part_s = at<float>(ws, Ly.part_s);
   a.zy = at<float>(ws, Ly.zy);
-  a.ldp = Ly.T_pad;
-  const Operand A{at<uint16_t>(ws, Ly.Hc), static_cast<uint64_t>(Ly.T_pad), static_cast<uint64_t>(Hd),
+  a.ldp = Ly.rows;
+  const Operand A{at<uint16_t>(ws, Ly.Hc), static_cast<uint64_t>(Ly.rows), static_cast<uint64_t>(Hd),
                   static_cast<uint64_t>(Hd)};
   Operand B[kMaxHeads];
   for (int h = 0; h < n_heads; ++h)
     B[h] = Operand{W[h], static_cast<uint64_t>(V), static_cast<uint64_t>(Hd), static_cast<uint64_t>(Hd)};
   TraceScope trace(GRPO_K_LSE_GEMM, V * n_heads, s);
-  return launch_gemm<kEpiLse, false, false>(A, B, a, Ly.T_pad, di, s);
+  return launch_gemm<kEpiLse, false, false>(A, B, a, Ly.rows, di, s);
 }
 
 grpo_status from_cuda(cudaError_t e) { return e == cudaSuccess ? GRPO_OK : GRPO_ERR_CUDA; }
@@ -553,8 +581,15 @@ const char* grpo_status_string(grpo_status st) {
     case GRPO_ERR_DEVICE_CHECK: return "GRPO_ERR_DEVICE_CHECK";
     case GRPO_ERR_TIMEOUT: return "GRPO_ERR_TIMEOUT";
     case GRPO_ERR_UNSUPPORTED: return "GRPO_ERR_UNSUPPORTED";
+    case GRPO_ERR_CAPACITY: return "GRPO_ERR_CAPACITY";
   }
   return "GRPO_ERR_UNKNOWN";
+}
+
+size_t grpo_workspace_bytes_rows(int64_t T, int64_t max_valid, int32_t Hd, int64_t V, int32_t which) {
+  Layout L;
+  if (max_valid < 0) return 0;
+  return make_layout(T, Hd, V, which, &L, max_valid) ? L.total : 0;
 }
 
 size_t grpo_workspace_bytes(int64_t T, int32_t Hd, int64_t V, int32_t which) {
@@ -588,7 +623,8 @@ grpo_status grpo_token_logprobs(const uint16_t* H, const uint16_t* W, const int3
   if (!W) return GRPO_ERR_INVALID_ARG;
   if (T > 0 && (!H || !targets || !mask || !logp_out)) return GRPO_ERR_INVALID_ARG;
   if (!aligned(W, 16) || (H && !aligned(H, 16))) return GRPO_ERR_INVALID_ARG;
-  if (!ws || !aligned(ws, 256) || ws_bytes < Ly.total) return GRPO_ERR_WORKSPACE;
+  if (!ws || !aligned(ws, 256) || !fit_layout(T, Hd, V, GRPO_WS_LOGPROBS, ws_bytes, &Ly))
+    return GRPO_ERR_WORKSPACE;
   if (T == 0) return GRPO_OK;
   DeviceInfo di;
   if (!device_info(&di)) return GRPO_ERR_UNSUPPORTED;
@@ -601,7 +637,7 @@ grpo_status grpo_token_logprobs(const uint16_t* H, const uint16_t* W, const int3
     TraceScope trace(GRPO_K_LOGP_MERGE, 0, s);
     logp_merge_kernel<<<blocks, 256, 0, s>>>(mask, at<int>(ws, Ly.rank_of), T, at<float>(ws, Ly.part_m),
                                              at<float>(ws, Ly.part_s), static_cast<int>(Ly.nsplit),
-                                             Ly.T_pad, at<float>(ws, Ly.zy), at<int>(ws, Ly.yc),
+                                             Ly.rows, at<float>(ws, Ly.zy), at<int>(ws, Ly.yc),
                                              logp_out, at<unsigned>(ws, Ly.status));
     e = cudaGetLastError();
   }
@@ -618,7 +654,8 @@ grpo_status grpo_token_logprobs_heads(const uint16_t* H, const uint16_t* const* 
     if (!W_heads[h] || !aligned(W_heads[h], 16)) return GRPO_ERR_INVALID_ARG;
   if (T > 0 && (!H || !targets || !mask || !logp_out)) return GRPO_ERR_INVALID_ARG;
   if (H && !aligned(H, 16)) return GRPO_ERR_INVALID_ARG;
-  if (!ws || !aligned(ws, 256) || ws_bytes < Ly.total) return GRPO_ERR_WORKSPACE;
+  if (!ws || !aligned(ws, 256) || !fit_layout(T, Hd, V, GRPO_WS_LOGPROBS_HEADS, ws_bytes, &Ly))
+    return GRPO_ERR_WORKSPACE;
   if (T == 0) return GRPO_OK;
   DeviceInfo di;
   if (!device_info(&di)) return GRPO_ERR_UNSUPPORTED;
@@ -630,10 +667,10 @@ grpo_status grpo_token_logprobs_heads(const uint16_t* H, const uint16_t* const* 
     const int blocks = static_cast<int>(std::min<int64_t>((T + 255) / 256, di.sms * 16));
     TraceScope trace(GRPO_K_LOGP_MERGE, 0, s);
     for (int h = 0; h < n_heads && e == cudaSuccess; ++h) {
-      const size_t head_parts = static_cast<size_t>(h) * Ly.nsplit * Ly.T_pad;
+      const size_t head_parts = static_cast<size_t>(h) * Ly.nsplit * Ly.rows;
       logp_merge_kernel<<<blocks, 256, 0, s>>>(mask, at<int>(ws, Ly.rank_of), T, at<float>(ws, Ly.part_m) + head_parts,
                                                at<float>(ws, Ly.part_s) + head_parts, static_cast<int>(Ly.nsplit),
-                                               Ly.T_pad, at<float>(ws, Ly.zy) + static_cast<size_t>(h) * Ly.T_pad,
+                                               Ly.rows, at<float>(ws, Ly.zy) + static_cast<size_t>(h) * Ly.rows,
                                                at<int>(ws, Ly.yc), logp_out + static_cast<size_t>(h) * T,
                                                at<unsigned>(ws, Ly.status));
       e = cudaGetLastError();
@@ -651,7 +688,8 @@ grpo_status grpo_sample_tokens(const uint16_t* H, const uint16_t* W, const uint8
   if (T > 0 && (!H || !mask || !tokens_out || !logp_out)) return GRPO_ERR_INVALID_ARG;
   if (H && !aligned(H, 16)) return GRPO_ERR_INVALID_ARG;
   if (!(temperature > 0.f) || !(temperature < INFINITY)) return GRPO_ERR_INVALID_ARG;
-  if (!ws || !aligned(ws, 256) || ws_bytes < Ly.total) return GRPO_ERR_WORKSPACE;
+  if (!ws || !aligned(ws, 256) || !fit_layout(T, Hd, V, GRPO_WS_SAMPLE, ws_bytes, &Ly))
+    return GRPO_ERR_WORKSPACE;
   if (T == 0) return GRPO_OK;
   DeviceInfo di;
   if (!device_info(&di)) return GRPO_ERR_UNSUPPORTED;
@@ -675,17 +713,17 @@ grpo_status grpo_sample_tokens(const uint16_t* H, const uint16_t* W, const uint8
     a.best_s = at<float>(ws, Ly.best_s);
     a.best_c = at<int>(ws, Ly.best_c);
     a.best_z = at<float>(ws, Ly.best_z);
-    a.ldp = Ly.T_pad;
+    a.ldp = Ly.rows;
     a.inv_temp = 1.f / temperature;
     a.seed_lo = static_cast<uint32_t>(seed);
     a.seed_hi = static_cast<uint32_t>(seed >> 32);
     a.off_lo = static_cast<uint32_t>(offset);
     a.off_hi = static_cast<uint32_t>(offset >> 32);
-    const Operand A{at<uint16_t>(ws, Ly.Hc), static_cast<uint64_t>(Ly.T_pad), static_cast<uint64_t>(Hd),
+    const Operand A{at<uint16_t>(ws, Ly.Hc), static_cast<uint64_t>(Ly.rows), static_cast<uint64_t>(Hd),
                     static_cast<uint64_t>(Hd)};
     const Operand B{W, static_cast<uint64_t>(V), static_cast<uint64_t>(Hd), static_cast<uint64_t>(Hd)};
     TraceScope trace(GRPO_K_SAMPLE_GEMM, V, s);
-    e = launch_gemm<kEpiSample, false, false>(A, B, a, Ly.T_pad, di, s);
+    e = launch_gemm<kEpiSample, false, false>(A, B, a, Ly.rows, di, s);
   }
   if (e == cudaSuccess) {
     const int blocks = static_cast<int>(std::min<int64_t>((T + 255) / 256, di.sms * 16));
@@ -693,7 +731,7 @@ grpo_status grpo_sample_tokens(const uint16_t* H, const uint16_t* W, const uint8
     sample_merge_kernel<<<blocks, 256, 0, s>>>(mask, at<int>(ws, Ly.rank_of), T, at<float>(ws, Ly.part_m),
                                                at<float>(ws, Ly.part_s), at<float>(ws, Ly.best_s),
                                                at<int>(ws, Ly.best_c), at<float>(ws, Ly.best_z),
-                                               static_cast<int>(Ly.nsplit), Ly.T_pad, tokens_out, logp_out,
+                                               static_cast<int>(Ly.nsplit), Ly.rows, tokens_out, logp_out,
                                                at<unsigned>(ws, Ly.status));
     e = cudaGetLastError();
   }
@@ -823,7 +861,8 @@ grpo_status loss_impl(const uint16_t* H, const uint16_t* W, const int32_t* targe
     return GRPO_ERR_INVALID_ARG;
   if (!aligned(W, 16) || !aligned(H, 16) || !aligned(dH, 16) || !aligned(dW, 16))
     return GRPO_ERR_INVALID_ARG;
-  if (!ws || !aligned(ws, 256) || ws_bytes < Ly.total) return GRPO_ERR_WORKSPACE;
+  if (!ws || !aligned(ws, 256) || !fit_layout(T, Hd, V, GRPO_WS_LOSS, ws_bytes, &Ly))
+    return GRPO_ERR_WORKSPACE;
   if (chunk_events) {
     const int64_t chunks = (V + Ly.vchunk - 1) / Ly.vchunk;
     if (n_events < chunks) return GRPO_ERR_INVALID_ARG;
@@ -845,11 +884,11 @@ grpo_status loss_impl(const uint16_t* H, const uint16_t* W, const int32_t* targe
     resp_len_kernel<<<static_cast<unsigned>(blocks), 256, 0, s>>>(mask, n_resp, L, at<int>(ws, Ly.resp_len));
     e = cudaGetLastError();
   }
-  const bool hct_blk = hct_blocks(Ly.T_pad);
+  const bool hct_blk = hct_blocks(Ly.rows);
   if (e == cudaSuccess) {
     TraceScope trace(GRPO_K_TRANSPOSE, 0, s);
-    const int tb = static_cast<int>(std::min<int64_t>(Ly.T_pad / 64 * (Hd / 64), int64_t(sms) * 8));
-    transpose_rows_kernel<<<tb, 256, 0, s>>>(at<uint16_t>(ws, Ly.Hc), n_valid, Hd, hct_blk ? 0 : Ly.T_pad,
+    const int tb = static_cast<int>(std::min<int64_t>(Ly.rows / 64 * (Hd / 64), int64_t(sms) * 8));
+    transpose_rows_kernel<<<tb, 256, 0, s>>>(at<uint16_t>(ws, Ly.Hc), n_valid, Hd, hct_blk ? 0 : Ly.rows,
                                              at<uint16_t>(ws, Ly.HcT));
     e = cudaGetLastError();
   }
@@ -858,7 +897,7 @@ grpo_status loss_impl(const uint16_t* H, const uint16_t* W, const int32_t* targe
     TraceScope trace(GRPO_K_LOSS, 0, s);
     loss_terms_kernel<<<static_cast<unsigned>(Ly.nblk_loss), kLossThreads, 0, s>>>(
         at<int>(ws, Ly.cidx), n_valid, at<float>(ws, Ly.part_m), at<float>(ws, Ly.part_s),
-        static_cast<int>(Ly.nsplit), Ly.T_pad, at<float>(ws, Ly.zy), at<int>(ws, Ly.yc), old_logp,
+        static_cast<int>(Ly.nsplit), Ly.rows, at<float>(ws, Ly.zy), at<int>(ws, Ly.yc), old_logp,
         ref_logp, adv, L, at<int>(ws, Ly.resp_len), n_resp, agg_mode, norm, clip_eps, beta, kl_clamp,
         at<float>(ws, Ly.lse_c), at<float>(ws, Ly.g_c), at<double>(ws, Ly.block_loss), status);
     loss_final_kernel<<<1, 1024, 0, s>>>(at<double>(ws, Ly.block_loss), n_valid, kLossThreads, loss_out);
@@ -881,7 +920,7 @@ grpo_status loss_impl(const uint16_t* H, const uint16_t* W, const int32_t* targe
   uint16_t* dz = at<uint16_t>(ws, Ly.dz);
   float* dHc = at<float>(ws, Ly.dhc);
   const int64_t vc = Ly.vchunk;
-  const uint64_t tp = static_cast<uint64_t>(Ly.T_pad), hd = static_cast<uint64_t>(Hd);
+  const uint64_t tp = static_cast<uint64_t>(Ly.rows), hd = static_cast<uint64_t>(Hd);  // compacted rows
   const Operand opHc{Hc, tp, hd, hd};
   const Operand opHcT{at<uint16_t>(ws, Ly.HcT), hd, tp, tp, hct_blk};
   const Operand opW{W, static_cast<uint64_t>(V), hd, hd};
@@ -905,7 +944,7 @@ grpo_status loss_impl(const uint16_t* H, const uint16_t* W, const int32_t* targe
       a.lse = at<float>(ws, Ly.lse_c);
       a.gcoef = at<float>(ws, Ly.g_c);
       TraceScope trace(GRPO_K_DZ_GEMM, width, s);
-      e = launch_gemm<kEpiDz, false, false>(opHc, opW, a, Ly.T_pad, di, s, &outDz);
+      e = launch_gemm<kEpiDz, false, false>(opHc, opW, a, Ly.rows, di, s, &outDz);
     }
     if (e != cudaSuccess) break;
     {  // dHc (+)= dZ_c W_c: stored by the first chunk, added at L2 by the others
@@ -921,7 +960,7 @@ grpo_status loss_impl(const uint16_t* H, const uint16_t* W, const int32_t* targe
       h.status = status;
       h.accumulate = c0 > 0;
       TraceScope trace(GRPO_K_DH_GEMM, width, s);
-      e = launch_gemm<kEpiF32, false, true>(opDz, opW, h, Ly.T_pad, di, s, &outDh);
+      e = launch_gemm<kEpiF32, false, true>(opDz, opW, h, Ly.rows, di, s, &outDh);
     }
     if (e != cudaSuccess) break;
     {  // dW_c = dZ_c^T Hc (stored, or consumed by the AdamW step)
@@ -1058,6 +1097,7 @@ grpo_status grpo_check_device_status(void* ws, void* stream) {
       cudaStreamSynchronize(s) != cudaSuccess)
     return GRPO_ERR_CUDA;
   if (word & kDevTimeout) return GRPO_ERR_TIMEOUT;
+  if (word & kDevCapacity) return GRPO_ERR_CAPACITY;
   if (word) return GRPO_ERR_DEVICE_CHECK;
   return GRPO_OK;
 }

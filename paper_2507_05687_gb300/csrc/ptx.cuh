@@ -13,6 +13,7 @@ enum : unsigned {
   kDevBadTarget = 1u,   // a target index outside [0, V) on an unmasked row
   kDevTimeout = 2u,     // a pipeline wait exceeded kWaitLimitNs
   kDevNonFinite = 4u,   // a log-sum-exp came out inf / nan
+  kDevCapacity = 8u,    // more unmasked rows than the workspace's row capacity
 };
 
 // A wait longer than this is treated as a hang: the kernel records kDevTimeout

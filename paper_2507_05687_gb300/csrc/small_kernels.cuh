@@ -99,8 +99,10 @@ __global__ void mask_count_kernel(const uint8_t* __restrict__ mask, int64_t T, i
 }
 
 // Single block: offsets[b] = sum of counts before b; *n_valid = grand total.
+// n_valid = the number of unmasked rows, clamped to the workspace's row
+// capacity `cap` (kDevCapacity is set when it had to be clamped).
 __global__ void count_scan_kernel(const int* __restrict__ counts, int nb, int* __restrict__ offsets,
-                                  int* __restrict__ n_valid) {
+                                  int* __restrict__ n_valid, int cap, unsigned* status) {
   __shared__ int sh[32];
   int carry = 0;
   for (int b0 = 0; b0 < nb; b0 += blockDim.x) {
@@ -111,12 +113,15 @@ __global__ void count_scan_kernel(const int* __restrict__ counts, int nb, int* _
     if (b < nb) offsets[b] = carry + ex;
     carry += total;
   }
-  if (threadIdx.x == 0) *n_valid = carry;
+  if (threadIdx.x == 0) {
+    *n_valid = min(carry, cap);
+    if (carry > cap) atomicOr(status, kDevCapacity);
+  }
 }
 
 // cidx[rank] = t for unmasked rows; rank_of[t] = rank or -1.
 __global__ void mask_scatter_kernel(const uint8_t* __restrict__ mask, int64_t T,
-                                    const int* __restrict__ offsets, int* __restrict__ cidx,
+                                    const int* __restrict__ offsets, int cap, int* __restrict__ cidx,
                                     int* __restrict__ rank_of) {
   __shared__ int sh[32];
   const int64_t base = static_cast<int64_t>(blockIdx.x) * kScanChunk + threadIdx.x * 16;
@@ -135,8 +140,10 @@ __global__ void mask_scatter_kernel(const uint8_t* __restrict__ mask, int64_t T,
     const int64_t t = base + j;
     if (t < T) {
       if (bits & (1u << j)) {
-        cidx[pos] = static_cast<int>(t);
-        rank_of[t] = pos;
+        // rows past the capacity get no compacted row (their outputs are 0
+        // and the status word carries kDevCapacity)
+        if (pos < cap) cidx[pos] = static_cast<int>(t);
+        rank_of[t] = pos < cap ? pos : -1;
         ++pos;
       } else {
         rank_of[t] = -1;
@@ -214,8 +221,8 @@ __global__ void logp_merge_kernel(const uint8_t* __restrict__ mask, const int* _
   for (int64_t t = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; t < T;
        t += static_cast<int64_t>(gridDim.x) * blockDim.x) {
     float out = 0.f;
-    if (mask[t]) {
-      const int r = rank_of[t];
+    const int r = mask[t] ? rank_of[t] : -1;
+    if (r >= 0) {
       const float lse = merge_lse(pm, ps, nsplit, ldp, r);
       if (!isfinite(lse)) atomicOr(status, kDevNonFinite);
       out = yc[r] >= 0 ? zy[r] - lse : 0.f;
@@ -256,8 +263,8 @@ __global__ void sample_merge_kernel(const uint8_t* __restrict__ mask, const int*
        t += static_cast<int64_t>(gridDim.x) * blockDim.x) {
     int tok = -1;
     float lp = 0.f;
-    if (mask[t]) {
-      const int r = rank_of[t];
+    const int r = mask[t] ? rank_of[t] : -1;
+    if (r >= 0) {
       float best = -INFINITY, z = 0.f;
       for (int j = 0; j < nsplit; ++j) {
         const float sc = bs[j * ldp + r];

@@ -61,6 +61,18 @@ def test_workspace_sizes(lib):
 FAKE = 0x10000  # never dereferenced: every call below is rejected on the host
 
 
+def test_workspace_sized_for_fewer_rows(lib):
+    f, g = grpo.workspace_bytes, grpo.workspace_bytes_rows
+    for which in (0, 1, 2, 3):
+        full = f(32768, 4096, 155136, which)
+        assert g(32768, 32768, 4096, 155136, which) == full == g(32768, 10**9, 4096, 155136, which)
+        sizes = [g(32768, n, 4096, 155136, which) for n in (1, 256, 257, 5000, 20000)]
+        assert sizes[0] == sizes[1] < sizes[2] <= sizes[3] <= sizes[4] < full   # 256-row granularity
+        assert g(32768, -1, 4096, 155136, which) == 0
+    # a ragged batch: 1M padded rows, 168k unmasked
+    assert g(1 << 20, 168251, 4096, 155136, 1) < 0.2 * f(1 << 20, 4096, 155136, 1)
+
+
 def test_host_rejections(lib):
     L = lib
     assert L.grpo_group_advantages(FAKE, 8, 1, 1e-6, FAKE, None) == grpo.GRPO_ERR_INVALID_ARG
@@ -86,7 +98,7 @@ def test_host_rejections(lib):
         assert L.grpo_loss_fwd_bwd(*bad) == grpo.GRPO_ERR_INVALID_ARG, i
     bad = list(largs); bad[16] = FAKE + 4          # dW misaligned
     assert L.grpo_loss_fwd_bwd(*bad) == grpo.GRPO_ERR_INVALID_ARG
-    bad = list(largs); bad[18] = ws2 - 1024
+    bad = list(largs); bad[18] = grpo.workspace_bytes_rows(40, 1, 64, 1000, 1) - 256   # not even 256 rows fit
     assert L.grpo_loss_fwd_bwd(*bad) == grpo.GRPO_ERR_WORKSPACE
     kargs = largs[:14] + [0.0, 1.0] + largs[14:]
     for kappa in (-1.0, float("nan"), float("-inf")):

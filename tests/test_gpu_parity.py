@@ -338,3 +338,52 @@ def test_larger_hidden_and_vocabulary():
     assert np.abs(got.astype(np.float64) - want).max() <= LOGP_ATOL
     w2 = wl.Workload("t", 1, 4, 60, 8192, 40000, "uniform", 20, 60, rewards="mix", seed=wl.SEED_BASE + 1701)
     _check_fwd_bwd(_case(w2))
+
+
+def test_workspace_sized_for_the_unmasked_rows(monkeypatch):
+    """A workspace sized by grpo_workspace_bytes_rows for the batch's unmasked
+    rows gives bit-identical log-probs, draws, loss and gradients."""
+    monkeypatch.setenv("GRPO_VOCAB_CHUNK", "768")
+    w = wl.Workload("t", 4, 4, 200, 128, 2100, "loguniform", 4, 200, rewards="mix", seed=wl.SEED_BASE + 580)
+    c = _case(w)
+    d = _dev(c)
+    nv = int(c["m"].sum())
+    assert 256 < nv < w.T - 512          # ragged: the lean workspace is smaller than the full one
+    for which in (grpo.GRPO_WS_LOSS, grpo.GRPO_WS_LOGPROBS, grpo.GRPO_WS_SAMPLE):
+        assert grpo.workspace_bytes_rows(w.T, nv, w.Hd, w.V, which) < grpo.workspace_bytes(w.T, w.Hd, w.V, which)
+    lean = lambda which: grpo.workspace(w.T, w.Hd, w.V, which, DEV, max_valid=nv)
+    args = (d["H"], d["W"], d["y"], d["m"], d["old"], d["ref"], d["adv"], w.n_resp, w.L, w.clip_eps, w.beta, 0)
+    ws = lean(grpo.GRPO_WS_LOSS)
+    a = grpo.loss_fwd_bwd(*args, ws=ws)
+    assert grpo.check_device_status(ws) == grpo.GRPO_OK
+    b = grpo.loss_fwd_bwd(*args)
+    for x, y in zip(a, b):
+        assert torch.equal(x, y)
+    ws = lean(grpo.GRPO_WS_LOGPROBS)
+    assert torch.equal(grpo.token_logprobs(d["H"], d["W"], d["y"], d["m"], ws=ws),
+                       grpo.token_logprobs(d["H"], d["W"], d["y"], d["m"]))
+    ws = lean(grpo.GRPO_WS_SAMPLE)
+    t1, l1 = grpo.sample_tokens(d["H"], d["W"], d["m"], 1.0, seed=5, ws=ws)
+    t2, l2 = grpo.sample_tokens(d["H"], d["W"], d["m"], 1.0, seed=5)
+    assert torch.equal(t1, t2) and torch.equal(l1, l2)
+
+
+def test_more_unmasked_rows_than_the_workspace_holds():
+    """Past the row capacity the device reports GRPO_ERR_CAPACITY (the count is
+    only known there); the rows past it get no output, nothing faults, and the
+    next call with a large enough workspace is correct."""
+    w = wl.Workload("t", 2, 4, 100, 128, 1500, "uniform", 60, 100, rewards="mix", seed=wl.SEED_BASE + 590)
+    c = _case(w)
+    d = _dev(c)
+    nv = int(c["m"].sum())
+    assert nv > 512
+    ws = grpo.workspace(w.T, w.Hd, w.V, grpo.GRPO_WS_LOSS, DEV, max_valid=300)   # 512 rows
+    grpo.loss_fwd_bwd(d["H"], d["W"], d["y"], d["m"], d["old"], d["ref"], d["adv"], w.n_resp, w.L, w.clip_eps,
+                      w.beta, 0, ws=ws)
+    assert grpo.check_device_status(ws) == grpo.GRPO_ERR_CAPACITY
+    ws_lp = grpo.workspace(w.T, w.Hd, w.V, grpo.GRPO_WS_LOGPROBS, DEV, max_valid=300)
+    lp = grpo.token_logprobs(d["H"], d["W"], d["y"], d["m"], ws=ws_lp)
+    assert grpo.check_device_status(ws_lp) == grpo.GRPO_ERR_CAPACITY
+    idx = wl.valid_index(c["m"])
+    assert not lp.cpu().numpy()[idx[512:]].any()       # no output past the capacity
+    _check_fwd_bwd(c)                                   # a full workspace on the same context
