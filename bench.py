@@ -187,7 +187,7 @@ def stored_traffic(workload: str, kind_name: str):
     return None
 
 
-def roofline(trace, n_valid_total_per_rank, Hd, steps, peak_tf, peak_kind, workload_key):
+def roofline(trace, n_valid_total_per_rank, Hd, steps, peak_tf, peak_kind, workload_key, hbm_gbs=None):
     by = {}
     for kind, cols, ms in trace:
         by.setdefault(kind, []).append((cols, ms))
@@ -201,15 +201,27 @@ def roofline(trace, n_valid_total_per_rank, Hd, steps, peak_tf, peak_kind, workl
     shares = {KIND_NAMES[k]: round(sum(ms for _, ms in v) / total_ms, 4) for k, v in sorted(by.items())}
     tr = stored_traffic(workload_key, KIND_NAMES[dom])
     traffic = None
+    avg_cols = sum(c for c, _ in recs) / len(recs)
     if tr is not None:
         bytes_per_launch, cols_ref = tr
-        avg_cols = sum(c for c, _ in recs) / len(recs)
         traffic = bytes_per_launch * avg_cols / cols_ref
+    common = {"kernel": KIND_NAMES[dom], "traffic": traffic, "launches_per_step": len(recs) // max(1, steps),
+              "avg_launch_ms": round(sum(secs) / len(secs) * 1e3, 4), "time_share": shares}
+    # A forward launch over few rows (a decode step) reads all of W for little
+    # work: below the ridge point (peak flop/s / peak B/s) its bound is HBM, and
+    # its algorithmic bytes are W's columns plus the gathered rows.
+    if hbm_gbs and dom in (2, 10):
+        alg_bytes = 2.0 * Hd * avg_cols + 2.0 * Hd * n_valid_total_per_rank
+        alg_flops = 2.0 * n_valid_total_per_rank * Hd * avg_cols
+        if alg_flops / alg_bytes < peak_tf * 1e12 / (hbm_gbs * 1e9):
+            gbs = alg_bytes / (sum(secs) / len(secs)) / 1e9
+            return {"bound": "hbm", "achieved": round(gbs, 1), "peak": hbm_gbs,
+                    "peak_kind": "HBM copy, measured", "unit": "GB/s", "frac": round(gbs / hbm_gbs, 4),
+                    "bytes_per_launch": alg_bytes, **common}
     return {
-        "bound": "tensor", "kernel": KIND_NAMES[dom], "achieved": round(achieved, 1),
+        "bound": "tensor", "achieved": round(achieved, 1),
         "peak": peak_tf, "peak_kind": peak_kind, "unit": "TFLOP/s", "frac": round(achieved / peak_tf, 4),
-        "traffic": traffic, "launches_per_step": len(recs) // max(1, steps),
-        "avg_launch_ms": round(sum(secs) / len(secs) * 1e3, 4), "time_share": shares,
+        **common,
     }
 
 
@@ -424,7 +436,7 @@ def main():
 
     burst, sustained, hbm, peak_src = peaks()
     rkey = w.name + ("+sample" if sampling else "") + ("" if args.adamw == "none" else "+adamw_" + args.adamw)
-    rf = roofline(trace, n_valid, w.Hd, args.steps, sustained, f"bf16 sustained, {peak_src}", rkey)
+    rf = roofline(trace, n_valid, w.Hd, args.steps, sustained, f"bf16 sustained, {peak_src}", rkey, hbm)
     if sampling:
         step_flops8 = step_flops6 = 2.0 * n_valid * w.Hd * w.V
     elif scoring:

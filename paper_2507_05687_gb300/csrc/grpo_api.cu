@@ -21,13 +21,18 @@ using namespace grpo;
 
 namespace {
 
-constexpr int kLseTilesPerUnit = 16;
+constexpr int kLseTilesPerUnit = 16;  // vocabulary tiles (of 256) per forward work unit
+// Forward work units are narrowed (16 -> 8 -> 4 vocabulary tiles) while a batch
+// has too few 256-row tiles to give every CTA pair of a GB300 (76) a unit: a
+// decode step of 256 rows would otherwise leave half the pairs idle (measured:
+// 0.36 ms and 52% of HBM bandwidth for the 1.27 GB head with 16-tile units).
+constexpr int kNominalPairs = 76;
 // Longest row of the transposed hidden states kept as plain rows.  Past it a
 // GEMM stage (128 rows of 128 bytes) would touch one 2 MB page per row; the
 // k-block layout keeps a stage contiguous.  Measured on the dW GEMM: plain rows
 // faster at 64 KB and 512 KB rows (14.6 vs 15.7 ms and 128.7 vs 140.6 ms per
 // step), k-blocks faster at 2 MB rows (147.6 vs 190.4 ms).
-constexpr int64_t kMaxTransposedRowBytes = int64_t(1) << 20;     // vocabulary tiles (of 256) per forward work unit
+constexpr int64_t kMaxTransposedRowBytes = int64_t(1) << 20;
 constexpr int kLossThreads = 256;
 constexpr int64_t kDefaultVocabChunk = 16384;
 
@@ -51,6 +56,7 @@ int64_t vocab_chunk(int64_t V) {
 // grpo_workspace_bytes_rows for batches with few unmasked rows.
 struct Layout {
   int64_t T_pad, rows, nsplit, nblk_scan, nblk_loss, vchunk;
+  int lse_tiles;  // vocabulary tiles (of 256) per forward work unit
   size_t status, n_valid, counts, offsets, cidx, rank_of, yc, zy, part_m, part_s, lse_c, g_c,
       block_loss, resp_len, best_s, best_c, best_z, Hc, HcT, dz, dhc, total;
 };
@@ -65,7 +71,11 @@ bool make_layout(int64_t T, int32_t Hd, int64_t V, int32_t which, Layout* L, int
   L->T_pad = round_up(std::max<int64_t>(T, 1), kRowAlign);
   const int64_t vtiles = (V + kTileN - 1) / kTileN;
   // partial (max, sum) entries per row: one per vocabulary split and column half
-  L->nsplit = (vtiles + kLseTilesPerUnit - 1) / kLseTilesPerUnit *
+  L->lse_tiles = kLseTilesPerUnit;
+  const int64_t m_tiles = (std::max<int64_t>(T, 1) + 2 * kRowsCta - 1) / (2 * kRowsCta);
+  while (L->lse_tiles > 4 && m_tiles * ((vtiles + L->lse_tiles - 1) / L->lse_tiles) < kNominalPairs)
+    L->lse_tiles /= 2;
+  L->nsplit = (vtiles + L->lse_tiles - 1) / L->lse_tiles *
               (which == GRPO_WS_SAMPLE ? EpiShape<kEpiSample>::kHalves : EpiShape<kEpiLse>::kHalves);
   L->rows = rows_cap < 0 ? L->T_pad : std::min(L->T_pad, round_up(std::max<int64_t>(rows_cap, 1), kRowAlign));
   L->nblk_scan = (std::max<int64_t>(T, 1) + kScanChunk - 1) / kScanChunk;
@@ -522,7 +532,7 @@ cudaError_t run_lse(const uint16_t* const* W, int n_heads, int32_t Hd, int64_t V
   a.m_dyn = 1;
   a.N = static_cast<int>(V);
   a.K = Hd;
-  a.n_per_unit = kLseTilesPerUnit;
+  a.n_per_unit = Ly.lse_tiles;
   a.n_heads = n_heads;
   a.group_m = group_m(0, di);
   // Fault-injection test hook (failure-detection tests): GRPO_TEST_DROP_KBLOCK=k
@@ -702,7 +712,7 @@ grpo_status grpo_sample_tokens(const uint16_t* H, const uint16_t* W, const uint8
     a.m_dyn = 1;
     a.N = static_cast<int>(V);
     a.K = Hd;
-    a.n_per_unit = kLseTilesPerUnit;
+    a.n_per_unit = Ly.lse_tiles;
     a.n_heads = 1;
     a.group_m = group_m(0, di);
     l2_hints(0, &a.a_hint, &a.b_hint);

@@ -101,7 +101,15 @@ PROFILE_WORKLOADS = {
     "fwdbwd_small": Workload("fwdbwd_small", 2, 8, 512, 4096, 32768, "uniform", 128, 512,
                              rewards="mix", seed=SEED_BASE + 6),
 }
-ALL_WORKLOADS = {**WORKLOADS, **PROFILE_WORKLOADS}
+# One decode step of rollout generation: every active sequence samples its next
+# token, so the LM-head GEMM sees a few hundred to a few thousand rows (here
+# 64 prompts x G=8 sequences = 512 rows, and 256 / 2048 rows), one per sequence.
+DECODE_WORKLOADS = {
+    "decode256_8b": Workload("decode256_8b", 32, 8, 1, 4096, 155136, seed=SEED_BASE + 7),
+    "decode512_8b": Workload("decode512_8b", 64, 8, 1, 4096, 155136, seed=SEED_BASE + 7),
+    "decode2048_8b": Workload("decode2048_8b", 256, 8, 1, 4096, 155136, seed=SEED_BASE + 7),
+}
+ALL_WORKLOADS = {**WORKLOADS, **PROFILE_WORKLOADS, **DECODE_WORKLOADS}
 
 
 def _rng(seed: int, stream: int, chunk: int = 0) -> np.random.Generator:
