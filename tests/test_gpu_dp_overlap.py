@@ -7,7 +7,6 @@ events, the communication stream and the NCCL calls are the real ones, and a
 one-rank sum must leave every bit of loss and dW unchanged.  The sharding and
 the global normaliser are covered by the two-rank gloo tests.
 """
-import os
 import socket
 
 import numpy as np
