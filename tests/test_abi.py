@@ -11,6 +11,7 @@ import paper_2507_05687_gb300 as grpo
 from paper_2507_05687_gb300 import build as build_mod
 
 ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HERE = os.path.dirname(os.path.abspath(__file__))
 
 
 @pytest.fixture(scope="module")
@@ -150,3 +151,29 @@ def test_binding_fails_loudly_without_library(tmp_path):
     from paper_2507_05687_gb300 import binding
     with pytest.raises(ImportError):
         binding.open_library(str(tmp_path / "missing.so"))
+
+
+def _build_c_check(tmp_path):
+    """gcc -std=c11 against include/grpo.h, linked to the in-tree libgrpo.so."""
+    import shutil
+    import subprocess
+    gcc = shutil.which("gcc")
+    if gcc is None:
+        pytest.skip("gcc not available")
+    cuda = os.environ.get("CUDA_HOME", "/usr/local/cuda")
+    lib_dir = os.path.dirname(grpo.LIB_PATH)
+    exe = str(tmp_path / "c_abi_check")
+    cmd = [gcc, "-std=c11", "-Wall", "-Wextra", "-Werror", os.path.join(HERE, "c_abi_check.c"),
+           "-I", os.path.join(ROOT, "include"), "-I", os.path.join(cuda, "include"), "-o", exe,
+           "-L", lib_dir, "-lgrpo", "-Wl,-rpath," + lib_dir, "-L", os.path.join(cuda, "lib64"), "-lcudart",
+           "-Wl,-rpath," + os.path.join(cuda, "lib64"), "-lm"]
+    subprocess.run(cmd, check=True, capture_output=True, text=True)
+    return exe
+
+
+def test_c_program_compiles_links_and_runs_host_checks(lib, tmp_path):
+    """The boundary is a C ABI: a C11 program uses it with no Python involved."""
+    import subprocess
+    exe = _build_c_check(tmp_path)
+    out = subprocess.run([exe, "host"], capture_output=True, text=True, timeout=60)
+    assert out.returncode == 0 and out.stdout.strip() == "ok", out.stdout + out.stderr
