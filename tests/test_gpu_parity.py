@@ -387,3 +387,20 @@ def test_more_unmasked_rows_than_the_workspace_holds():
     idx = wl.valid_index(c["m"])
     assert not lp.cpu().numpy()[idx[512:]].any()       # no output past the capacity
     _check_fwd_bwd(c)                                   # a full workspace on the same context
+
+
+def test_empty_batches():
+    """T = 0: every call accepts it and returns empty outputs (nothing launched
+    that reads the inputs); a zero-row noise block is a no-op."""
+    Hd, V = 128, 500
+    H = torch.empty(0, Hd, dtype=torch.bfloat16, device=DEV)
+    W = dev_tensor(wl.gen_weight(wl.Workload("t", 1, 2, 1, Hd, V, seed=wl.SEED_BASE + 1)), torch.bfloat16)
+    y = torch.empty(0, dtype=torch.int32, device=DEV)
+    m = torch.empty(0, dtype=torch.uint8, device=DEV)
+    assert grpo.token_logprobs(H, W, y, m).numel() == 0
+    assert grpo.token_logprobs_heads(H, [W, W], y, m).shape == (2, 0)
+    tok, lp = grpo.sample_tokens(H, W, m, 1.0, seed=3)
+    assert tok.numel() == 0 and lp.numel() == 0
+    assert grpo.gumbel_noise(5, 0, V, seed=1).shape == (0, V)
+    adv = grpo.group_advantages(torch.empty(0, dtype=torch.float32, device=DEV), 4)
+    assert adv.numel() == 0
