@@ -1,5 +1,6 @@
 """GPU parity at the full 8B-shaped sizes (hidden 4096, vocabulary 155136),
-in the launch configuration bench.py times.
+in the launch configuration bench.py times (workspaces sized for the
+unmasked rows).
 
 The float64 oracle's log-sum-exp of every unmasked token (and the old /
 reference log-probs, which are inputs of the loss) were written once by
@@ -72,7 +73,7 @@ def test_logprob_three_heads_full_size():
     gold = _load(w.name)
     Hb, Wb, y, m, idx = _inputs(w, gold)
     H, yd, md = dev_tensor(Hb, torch.bfloat16), dev_tensor(y, torch.int32), dev_tensor(m, torch.uint8)
-    ws = grpo.workspace(w.T, w.Hd, w.V, grpo.GRPO_WS_LOGPROBS, DEV)
+    ws = grpo.workspace(w.T, w.Hd, w.V, grpo.GRPO_WS_LOGPROBS, DEV, max_valid=idx.size)
     want = {"policy": _oracle_logp(Hb, Wb, y, idx, gold["lse_policy"]),
             "old": gold["old_logp"].astype(np.float64), "ref": gold["ref_logp"].astype(np.float64)}
     heads = []
@@ -86,7 +87,7 @@ def test_logprob_three_heads_full_size():
         err = np.abs(got[idx].astype(np.float64) - want[which])
         assert err.max() <= LOGP_ATOL, (which, err.max())
     # the three heads in one call (the configuration bench.py times for this workload)
-    ws3 = grpo.workspace(w.T, w.Hd, w.V, grpo.GRPO_WS_LOGPROBS_HEADS, DEV)
+    ws3 = grpo.workspace(w.T, w.Hd, w.V, grpo.GRPO_WS_LOGPROBS_HEADS, DEV, max_valid=idx.size)
     lp3 = grpo.token_logprobs_heads(H, heads, yd, md, ws=ws3)
     assert grpo.check_device_status(ws3) == grpo.GRPO_OK
     for h, which in enumerate(("policy", "old", "ref")):
@@ -123,7 +124,7 @@ def test_fwd_bwd_full_size(name):
     adv = oracle.group_advantages(r, w.G, float(np.float32(w.adv_eps)))
 
     H, W = dev_tensor(Hb, torch.bfloat16), dev_tensor(Wb, torch.bfloat16)
-    ws = grpo.workspace(w.T, w.Hd, w.V, grpo.GRPO_WS_LOSS, DEV)
+    ws = grpo.workspace(w.T, w.Hd, w.V, grpo.GRPO_WS_LOSS, DEV, max_valid=idx.size)  # as bench.py sizes it
     adv_d = grpo.group_advantages(dev_tensor(r, torch.float32), w.G, w.adv_eps)
     assert np.array_equal(adv_d.cpu().numpy().view(np.uint32), adv.view(np.uint32))
     loss, dH, dW = grpo.loss_fwd_bwd(H, W, dev_tensor(y, torch.int32), dev_tensor(m, torch.uint8),
@@ -166,8 +167,9 @@ def test_sampling_full_size():
     """The rollout draw over the 32768-row batch at 4096 x 155136, checked on sampled rows."""
     w = wl.WORKLOADS["logprob3_8b"]
     Hb, Wb, m = wl.gen_hidden(w), wl.gen_weight(w), wl.gen_mask(w)
+    ws = grpo.workspace(w.T, w.Hd, w.V, grpo.GRPO_WS_SAMPLE, DEV, max_valid=int(m.sum()))
     tok, lp = grpo.sample_tokens(dev_tensor(Hb, torch.bfloat16), dev_tensor(Wb, torch.bfloat16),
-                                 dev_tensor(m, torch.uint8), 1.0, seed=20250705, offset=687)
+                                 dev_tensor(m, torch.uint8), 1.0, seed=20250705, offset=687, ws=ws)
     tok, lp = tok.cpu().numpy(), lp.cpu().numpy()
     assert np.all(tok[m == 0] == -1)
     idx = wl.valid_index(m)
