@@ -180,3 +180,22 @@ def test_sampling_full_size():
     assert clear.size >= 0.9 * rows.size
     assert np.array_equal(tok[clear], want_tok[clear])
     assert np.abs(lp[clear] - want_lp[clear]).max() <= LOGP_ATOL
+
+
+def test_decode_step_full_vocabulary():
+    """One decode step of 256 sequences at 4096 x 155136 (forward units narrowed
+    to 8 vocabulary tiles, 76 splits): every row's log-prob against the oracle's
+    float64 log-sum-exp, and every row's draw against the oracle's Gumbel-max."""
+    w = wl.DECODE_WORKLOADS["decode256_8b"]
+    Hb, Wb, y, m = wl.gen_hidden(w), wl.gen_weight(w), wl.gen_targets(w), wl.gen_mask(w)
+    H, W = dev_tensor(Hb, torch.bfloat16), dev_tensor(Wb, torch.bfloat16)
+    got = grpo.token_logprobs(H, W, dev_tensor(y, torch.int32), dev_tensor(m, torch.uint8)).cpu().numpy()
+    want, _ = oracle.token_logprobs(Hb, Wb, y, m)
+    assert np.abs(got.astype(np.float64) - want).max() <= LOGP_ATOL
+    tok, lp = grpo.sample_tokens(H, W, dev_tensor(m, torch.uint8), 0.7, seed=9, offset=2**33 + 5)
+    tok, lp = tok.cpu().numpy(), lp.cpu().numpy()
+    want_tok, want_lp, gap = oracle.sample_tokens(Hb, Wb, m, 0.7, 9, 2**33 + 5)
+    clear = np.flatnonzero(gap > 1e-3)
+    assert clear.size >= 0.9 * w.T
+    assert np.array_equal(tok[clear], want_tok[clear])
+    assert np.abs(lp[clear] - want_lp[clear]).max() <= LOGP_ATOL
