@@ -75,3 +75,33 @@ def test_decode_step_draw_replays_from_a_graph():
     g.replay()
     torch.cuda.synchronize()
     assert torch.equal(out[0], eager[0]) and torch.equal(out[1], eager[1])
+
+
+def test_calls_on_two_streams_with_their_own_workspaces():
+    """Two loss calls in flight at once on different streams (each with its own
+    workspace) give what they give one after the other: the library's shared
+    state (device properties, tensor-map encoder) is read-only after set-up and
+    its kernels never wait on one another across launches."""
+    cases = []
+    for seed in (960, 961):
+        w = wl.Workload("s", 2, 4, 50, 128, 1700, "uniform", 1, 50, rewards="mix", seed=wl.SEED_BASE + seed)
+        Hb, Wb, y, m, r = wl.gen_hidden(w), wl.gen_weight(w), wl.gen_targets(w), wl.gen_mask(w), wl.gen_rewards(w)
+        lp = oracle.token_logprobs(Hb, Wb, y, m)[0]
+        d = [dev_tensor(Hb, torch.bfloat16), dev_tensor(Wb, torch.bfloat16), dev_tensor(y, torch.int32),
+             dev_tensor(m, torch.uint8), dev_tensor((lp - 0.05).astype(np.float32), torch.float32),
+             dev_tensor((lp + 0.1).astype(np.float32), torch.float32),
+             dev_tensor(oracle.group_advantages(r, w.G, float(np.float32(w.adv_eps))), torch.float32)]
+        cases.append((w, d))
+    seq = [grpo.loss_fwd_bwd(*d, w.n_resp, w.L, w.clip_eps, w.beta, 0) for w, d in cases]
+    torch.cuda.synchronize()
+    streams = [torch.cuda.Stream(DEV) for _ in cases]
+    outs = []
+    for (w, d), st in zip(cases, streams):
+        st.wait_stream(torch.cuda.current_stream(DEV))
+        with torch.cuda.stream(st):
+            ws = grpo.workspace(w.T, w.Hd, w.V, grpo.GRPO_WS_LOSS, DEV)
+            outs.append(grpo.loss_fwd_bwd(*d, w.n_resp, w.L, w.clip_eps, w.beta, 0, ws=ws))
+    torch.cuda.synchronize()
+    for a, b in zip(outs, seq):
+        for x, y in zip(a, b):
+            assert torch.equal(x, y)
