@@ -125,6 +125,28 @@ def _on_device(t: torch.Tensor, dev: torch.device, dtype: torch.dtype, name: str
     return t.contiguous()
 
 
+def _shape(t: torch.Tensor, shape, name: str) -> None:
+    """The C ABI sees only pointers and sizes: a tensor of the wrong shape would
+    be read or written past its end, so every shape is checked here."""
+    if tuple(t.shape) != tuple(shape):
+        raise ValueError(f"{name}: expected shape {tuple(shape)}, got {tuple(t.shape)}")
+
+
+def _output(t: torch.Tensor, shape, dtype: torch.dtype, dev: torch.device, name: str) -> torch.Tensor:
+    """A caller-given output is written in place: it must already be a dense
+    tensor of the right shape, type and device (a copy would be written instead)."""
+    if t.dtype != dtype or t.device != dev or not t.is_contiguous():
+        raise ValueError(f"{name}: contiguous {dtype} on {dev} expected")
+    _shape(t, shape, name)
+    return t
+
+
+def _workspace(ws: torch.Tensor, dev: torch.device) -> torch.Tensor:
+    if ws.dtype != torch.uint8 or ws.device != dev or not ws.is_contiguous():
+        raise ValueError(f"ws: contiguous uint8 on {dev} expected (see workspace())")
+    return ws
+
+
 def _target_device(*ts: torch.Tensor) -> Tuple[torch.device, bool]:
     for t in ts:
         if t.is_cuda:
@@ -167,8 +189,8 @@ def group_advantages(rewards: torch.Tensor, G: int, eps: float = 1e-6,
                      out: Optional[torch.Tensor] = None) -> torch.Tensor:
     """grpo_group_advantages: Eq. 2 per group of G consecutive responses."""
     dev, host = _target_device(rewards)
-    r = _on_device(rewards, dev, torch.float32, "rewards")
-    adv = out if out is not None else torch.empty_like(r)
+    r = _on_device(rewards, dev, torch.float32, "rewards").reshape(-1)
+    adv = _output(out, r.shape, torch.float32, dev, "out") if out is not None else torch.empty_like(r)
     _check(load().grpo_group_advantages(_ptr(r), r.numel(), int(G), float(eps), _ptr(adv), _stream(dev)),
            "grpo_group_advantages")
     return _to_host(adv) if host else adv
@@ -184,9 +206,12 @@ def token_logprobs(H: torch.Tensor, W: torch.Tensor, targets: torch.Tensor, mask
     mask = _on_device(mask.view(torch.uint8) if mask.dtype == torch.bool else mask, dev, torch.uint8, "mask")
     T, Hd = H.shape
     V = W.shape[0]
-    if ws is None:
-        ws = workspace(T, Hd, V, GRPO_WS_LOGPROBS, dev)
-    logp = out if out is not None else torch.empty(T, dtype=torch.float32, device=dev)
+    _shape(W, (V, Hd), "W")
+    _shape(targets, (T,), "targets")
+    _shape(mask, (T,), "mask")
+    ws = workspace(T, Hd, V, GRPO_WS_LOGPROBS, dev) if ws is None else _workspace(ws, dev)
+    logp = _output(out, (T,), torch.float32, dev, "out") if out is not None else \
+        torch.empty(T, dtype=torch.float32, device=dev)
     _check(load().grpo_token_logprobs(_ptr(H), _ptr(W), _ptr(targets), _ptr(mask), T, Hd, V, _ptr(logp),
                                       _ptr(ws), ws.numel(), _stream(dev)), "grpo_token_logprobs")
     return _to_host(logp) if host else logp
@@ -204,11 +229,13 @@ def token_logprobs_heads(H: torch.Tensor, W_heads, targets: torch.Tensor, mask: 
     mask = _on_device(mask.view(torch.uint8) if mask.dtype == torch.bool else mask, dev, torch.uint8, "mask")
     T, Hd = H.shape
     V = W_heads[0].shape[0]
-    if any(w.shape != W_heads[0].shape for w in W_heads):
-        raise ValueError("all heads must have the same [V, Hd] shape")
-    if ws is None:
-        ws = workspace(T, Hd, V, GRPO_WS_LOGPROBS_HEADS, dev)
-    logp = out if out is not None else torch.empty(len(W_heads), T, dtype=torch.float32, device=dev)
+    for i, w in enumerate(W_heads):
+        _shape(w, (V, Hd), f"W_heads[{i}]")
+    _shape(targets, (T,), "targets")
+    _shape(mask, (T,), "mask")
+    ws = workspace(T, Hd, V, GRPO_WS_LOGPROBS_HEADS, dev) if ws is None else _workspace(ws, dev)
+    logp = _output(out, (len(W_heads), T), torch.float32, dev, "out") if out is not None else \
+        torch.empty(len(W_heads), T, dtype=torch.float32, device=dev)
     ptrs = (ctypes.c_void_p * len(W_heads))(*[w.data_ptr() for w in W_heads])
     _check(load().grpo_token_logprobs_heads(_ptr(H), ptrs, len(W_heads), _ptr(targets), _ptr(mask), T, Hd, V,
                                             _ptr(logp), _ptr(ws), ws.numel(), _stream(dev)),
@@ -226,11 +253,13 @@ def sample_tokens(H: torch.Tensor, W: torch.Tensor, mask: torch.Tensor, temperat
     mask = _on_device(mask.view(torch.uint8) if mask.dtype == torch.bool else mask, dev, torch.uint8, "mask")
     T, Hd = H.shape
     V = W.shape[0]
-    if ws is None:
-        ws = workspace(T, Hd, V, GRPO_WS_SAMPLE, dev)
+    _shape(W, (V, Hd), "W")
+    _shape(mask, (T,), "mask")
+    ws = workspace(T, Hd, V, GRPO_WS_SAMPLE, dev) if ws is None else _workspace(ws, dev)
     if out is None:
         out = (torch.empty(T, dtype=torch.int32, device=dev), torch.empty(T, dtype=torch.float32, device=dev))
-    tok, logp = out
+    tok = _output(out[0], (T,), torch.int32, dev, "out[0]")
+    logp = _output(out[1], (T,), torch.float32, dev, "out[1]")
     _check(load().grpo_sample_tokens(_ptr(H), _ptr(W), _ptr(mask), T, Hd, V, float(temperature),
                                      int(seed) & (2 ** 64 - 1), int(offset) & (2 ** 64 - 1), _ptr(tok), _ptr(logp),
                                      _ptr(ws), ws.numel(), _stream(dev)), "grpo_sample_tokens")
@@ -260,16 +289,28 @@ def loss_fwd_bwd(H: torch.Tensor, W: torch.Tensor, targets: torch.Tensor, mask: 
     adv = _on_device(adv, dev, torch.float32, "adv")
     T, Hd = H.shape
     V = W.shape[0]
-    if ws is None:
-        ws = workspace(T, Hd, V, GRPO_WS_LOSS, dev)
+    if T != int(n_resp) * int(L):
+        raise ValueError(f"H has {T} rows, n_resp * L = {int(n_resp) * int(L)}")
+    _shape(W, (V, Hd), "W")
+    for name, t in (("targets", targets), ("mask", mask), ("old_logp", old_logp), ("ref_logp", ref_logp)):
+        _shape(t, (T,), name)
+    _shape(adv, (int(n_resp),), "adv")
+    ws = workspace(T, Hd, V, GRPO_WS_LOSS, dev) if ws is None else _workspace(ws, dev)
     host_out = None
     if out is not None and not out[0].is_cuda:
         host_out, out = out, None  # results land in the caller's host buffers
+        for name, t, shp in (("out[0]", host_out[0], (1,)), ("out[1]", host_out[1], (T, Hd)),
+                             ("out[2]", host_out[2], (V, Hd))):
+            if t.dtype != torch.float32 or t.is_cuda or not t.is_contiguous():
+                raise ValueError(f"{name}: contiguous fp32 host tensor expected")
+            _shape(t, shp, name)
     if out is None:
         out = (torch.empty(1, dtype=torch.float32, device=dev),
                torch.empty(T, Hd, dtype=torch.float32, device=dev),
                torch.empty(V, Hd, dtype=torch.float32, device=dev))
-    loss, dH, dW = out
+    loss = _output(out[0], (1,), torch.float32, dev, "out[0]")
+    dH = _output(out[1], (T, Hd), torch.float32, dev, "out[1]")
+    dW = _output(out[2], (V, Hd), torch.float32, dev, "out[2]")
     lib = load()
     common = (_ptr(H), _ptr(W), _ptr(targets), _ptr(mask), _ptr(old_logp), _ptr(ref_logp), _ptr(adv), int(n_resp),
               int(L), Hd, V, float(clip_eps), float(beta), int(agg_mode))
@@ -329,11 +370,20 @@ def loss_fwd_bwd_adamw(H: torch.Tensor, W: torch.Tensor, targets: torch.Tensor, 
     W_out = W if W_out is None else W_out
     T, Hd = H.shape
     V = W.shape[0]
-    if ws is None:
-        ws = workspace(T, Hd, V, GRPO_WS_LOSS, dev)
+    if T != int(n_resp) * int(L):
+        raise ValueError(f"H has {T} rows, n_resp * L = {int(n_resp) * int(L)}")
+    if W.dtype != torch.bfloat16 or not W.is_contiguous():
+        raise ValueError("W: contiguous bf16 expected")
+    _shape(W, (V, Hd), "W")
+    _output(W_out, (V, Hd), torch.bfloat16, dev, "W_out")
+    for name, t in (("targets", targets), ("mask", mask), ("old_logp", old_logp), ("ref_logp", ref_logp)):
+        _shape(t, (T,), name)
+    _shape(adv, (int(n_resp),), "adv")
+    ws = workspace(T, Hd, V, GRPO_WS_LOSS, dev) if ws is None else _workspace(ws, dev)
     if out is None:
         out = (torch.empty(1, dtype=torch.float32, device=dev), torch.empty(T, Hd, dtype=torch.float32, device=dev))
-    loss, dH = out
+    loss = _output(out[0], (1,), torch.float32, dev, "out[0]")
+    dH = _output(out[1], (T, Hd), torch.float32, dev, "out[1]")
     _check(load().grpo_loss_fwd_bwd_adamw(
         _ptr(H), _ptr(W), _ptr(targets), _ptr(mask), _ptr(old_logp), _ptr(ref_logp), _ptr(adv), int(n_resp), int(L),
         Hd, V, float(clip_eps), float(beta), int(agg_mode), float(norm), float(lr), float(betas[0]), float(betas[1]),
@@ -347,11 +397,12 @@ def adamw_step(W_master: torch.Tensor, exp_avg: torch.Tensor, exp_avg_sq: torch.
                weight_decay: float = 0.01) -> None:
     """grpo_adamw_step: one AdamW step in place over contiguous fp32 device tensors."""
     n = W_master.numel()
-    for name, t in (("exp_avg", exp_avg), ("exp_avg_sq", exp_avg_sq), ("grad", grad)):
-        if t.numel() != n or t.dtype != torch.float32 or not t.is_contiguous():
-            raise ValueError(f"{name}: contiguous fp32 with W_master's size expected")
-    if W_out.numel() != n or W_out.dtype != torch.bfloat16:
-        raise ValueError("W_out: bf16 with W_master's size expected")
+    dev = W_master.device
+    for name, t in (("W_master", W_master), ("exp_avg", exp_avg), ("exp_avg_sq", exp_avg_sq), ("grad", grad)):
+        if t.numel() != n or t.dtype != torch.float32 or not t.is_contiguous() or t.device != dev or not t.is_cuda:
+            raise ValueError(f"{name}: contiguous fp32 device tensor with W_master's size expected")
+    if W_out.numel() != n or W_out.dtype != torch.bfloat16 or not W_out.is_contiguous() or W_out.device != dev:
+        raise ValueError("W_out: contiguous bf16 with W_master's size expected")
     _check(load().grpo_adamw_step(_ptr(W_master), _ptr(exp_avg), _ptr(exp_avg_sq), _ptr(grad), _ptr(W_out), n,
                                   float(lr), float(betas[0]), float(betas[1]), float(eps), float(weight_decay),
                                   int(step), _stream(W_master.device)), "grpo_adamw_step")

@@ -404,3 +404,37 @@ def test_empty_batches():
     assert grpo.gumbel_noise(5, 0, V, seed=1).shape == (0, V)
     adv = grpo.group_advantages(torch.empty(0, dtype=torch.float32, device=DEV), 4)
     assert adv.numel() == 0
+
+
+def test_binding_rejects_mismatched_shapes():
+    """The C ABI takes pointers and sizes only; the binding checks every shape,
+    output and workspace first, so a mismatch raises instead of reading past a
+    buffer."""
+    w = wl.Workload("t", 1, 2, 40, 64, 300, "uniform", 1, 40, seed=wl.SEED_BASE + 970)
+    c = _case(w)
+    d = _dev(c)
+    args = [d["H"], d["W"], d["y"], d["m"], d["old"], d["ref"], d["adv"], w.n_resp, w.L]
+    bad_cases = [
+        (1, d["W"][:, :32]),            # hidden size differs from H
+        (2, d["y"][:-1]),               # one target short
+        (3, d["m"][:-1]),               # mask short
+        (4, d["old"][:-1]),
+        (6, d["adv"][:-1]),             # advantages for fewer responses
+        (8, w.L + 1),                   # n_resp * L != rows of H
+    ]
+    for i, v in bad_cases:
+        a = list(args)
+        a[i] = v
+        with pytest.raises(ValueError):
+            grpo.loss_fwd_bwd(*a)
+    with pytest.raises(ValueError):
+        grpo.token_logprobs(d["H"], d["W"], d["y"][:-1], d["m"])
+    with pytest.raises(ValueError):
+        grpo.loss_fwd_bwd(*args, out=(torch.empty(1, device=DEV), torch.empty(w.T, w.Hd, device=DEV),
+                                      torch.empty(w.V - 1, w.Hd, device=DEV)))
+    with pytest.raises(ValueError):
+        grpo.token_logprobs(d["H"], d["W"], d["y"], d["m"], ws=torch.empty(10, dtype=torch.float32, device=DEV))
+    with pytest.raises(ValueError):
+        grpo.sample_tokens(d["H"], d["W"], d["m"][:-1])
+    # and the well-formed call still works
+    grpo.loss_fwd_bwd(*args)
