@@ -36,9 +36,9 @@ METRIC = "response tokens/s for GRPO logprob+loss fwd+bwd; % of dense bf16 peak"
 GOLDEN = {"fwdbwd_8b": "batch8b", "logprob3_8b": "batch8b", "long_8b": "long_8b", "ragged_8b": "ragged_8b"}
 # the GEMM kernels and the launch parameters (raster, cache hints) that set their DRAM traffic
 KERNEL_SOURCES = ["paper_2507_05687_gb300/csrc/gemm_tc.cuh", "paper_2507_05687_gb300/csrc/ptx.cuh",
-                  "paper_2507_05687_gb300/csrc/grpo_api.cu"]
+                  "paper_2507_05687_gb300/csrc/grpo_api.cu", "paper_2507_05687_gb300/csrc/small_kernels.cuh"]
 KIND_NAMES = ["advantages", "compact", "lse_gemm", "logp_merge", "loss", "dz_gemm", "dh_gemm", "dw_gemm",
-              "dh_rows", "adamw", "sample_gemm", "transpose"]
+              "dh_rows", "adamw", "sample_gemm", "transpose", "dz_logits"]
 KERNELS_PER_SCOPE = {1: 4, 4: 2}  # compaction scope = 4 kernels, loss scope = 2 kernels; others 1
 
 
@@ -52,6 +52,9 @@ def parse():
     p.add_argument("--adamw", choices=["none", "fused", "separate"], default="none",
                    help="fwd+bwd workloads: add the AdamW step of the LM head, fused into the dW GEMM "
                         "or as a separate pass over the stored dW")
+    p.add_argument("--logits", choices=["keep", "recompute"], default="keep",
+                   help="fwd+bwd workloads: keep the forward's fp32 logits for the backward (a GRPO_WS_LOSS_LOGITS "
+                        "workspace) or recompute them in the backward with a second logits GEMM (GRPO_WS_LOSS)")
     p.add_argument("--sample", action="store_true",
                    help="time the rollout draw (grpo_sample_tokens) over the workload's rows instead")
     p.add_argument("--no-e2e", action="store_true")
@@ -207,6 +210,17 @@ def roofline(trace, n_valid_total_per_rank, Hd, steps, peak_tf, peak_kind, workl
         traffic = bytes_per_launch * avg_cols / cols_ref
     common = {"kernel": KIND_NAMES[dom], "traffic": traffic, "launches_per_step": len(recs) // max(1, steps),
               "avg_launch_ms": round(sum(secs) / len(secs) * 1e3, 4), "time_share": shares}
+    if 12 in by and hbm_gbs:
+        # dZ from the kept logits, HBM-bound: per launch it reads N_valid x cols
+        # fp32 logits and writes N_valid x cols bf16 dZ (algorithmic bytes)
+        zr = by[12]
+        zb = sum(6.0 * n_valid_total_per_rank * c for c, _ in zr) / len(zr)
+        zs = sum(ms for _, ms in zr) / len(zr) / 1e3
+        ztr = stored_traffic(workload_key, "dz_logits")
+        common["dz_logits_hbm"] = {
+            "achieved": round(zb / zs / 1e9, 1), "peak": hbm_gbs, "unit": "GB/s",
+            "frac": round(zb / zs / 1e9 / hbm_gbs, 4), "bytes_per_launch": zb, "avg_launch_ms": round(zs * 1e3, 4),
+            "traffic": None if ztr is None else ztr[0] * (sum(c for c, _ in zr) / len(zr)) / ztr[1]}
     # A forward launch over few rows (a decode step) reads all of W for little
     # work: below the ridge point (peak flop/s / peak B/s) its bound is HBM, and
     # its algorithmic bytes are W's columns plus the gathered rows.
@@ -353,7 +367,10 @@ def main():
             # policy / old / reference log-probs of one rollout batch; ranks score independently
             grpo.token_logprobs_heads(H, heads, y, m, ws=ws, out=logp3)
     else:
-        ws = grpo.workspace(w.T, w.Hd, w.V, grpo.GRPO_WS_LOSS, dev, max_valid=n_valid)
+        ws_kind = grpo.GRPO_WS_LOSS_LOGITS if args.logits == "keep" else grpo.GRPO_WS_LOSS
+        ws = grpo.workspace(w.T, w.Hd, w.V, ws_kind, dev, max_valid=n_valid)
+        if grpo.loss_plan(w.T, w.Hd, w.V, ws.numel())[0] != (args.logits == "keep"):
+            raise SystemExit("the workspace does not give the requested logits handling")
         adv = torch.empty(w.n_resp, dtype=torch.float32, device=dev)
         out = (torch.empty(1, dtype=torch.float32, device=dev),
                torch.empty(w.T, w.Hd, dtype=torch.float32, device=dev),
@@ -435,7 +452,8 @@ def main():
     value = tot_valid / (ms / 1e3)
 
     burst, sustained, hbm, peak_src = peaks()
-    rkey = w.name + ("+sample" if sampling else "") + ("" if args.adamw == "none" else "+adamw_" + args.adamw)
+    rkey = w.name + ("+sample" if sampling else "") + ("" if args.adamw == "none" else "+adamw_" + args.adamw) + \
+        ("+recompute" if args.logits == "recompute" and not (sampling or scoring) else "")
     rf = roofline(trace, n_valid, w.Hd, args.steps, sustained, f"bf16 sustained, {peak_src}", rkey, hbm)
     if sampling:
         step_flops8 = step_flops6 = 2.0 * n_valid * w.Hd * w.V
@@ -446,12 +464,14 @@ def main():
         step_flops6 = 6.0 * n_valid * w.Hd * w.V
 
     e2e = e2e_offload = None
-    if not args.no_e2e and rank == 0 and not sampling:
+    if not args.no_e2e and not sampling:
         if scoring:
-            e2e = measure_e2e_scoring(grpo, torch, dev, w, inp, heads, steps=min(args.steps, 5))
+            e2e = measure_e2e_scoring(grpo, torch, dev, w, inp, heads, steps=min(args.steps, 5), dist=dist)
         else:
-            e2e = measure_e2e(grpo, torch, dev, w, inp, steps=min(args.steps, 5))
-            e2e_offload = measure_e2e_offload(grpo, torch, dev, w, inp, steps=min(args.steps, 5))
+            # the step's own workspace: a second one of the same size may not fit beside it
+            e2e = measure_e2e(grpo, torch, dev, w, inp, steps=min(args.steps, 5), dist=dist, ws=ws)
+            if world == 1:
+                e2e_offload = measure_e2e_offload(grpo, torch, dev, w, inp, steps=min(args.steps, 5), ws=ws)
 
     cpu = None
     if not args.no_cpu_baseline and rank == 0 and world == 1 and not sampling:
@@ -473,6 +493,8 @@ def main():
                        "l2": "inputs larger than L2 (W %.2f GB, H %.2f GB per rank)" % (w.V * w.Hd * 2 / 1e9,
                                                                                          w.T * w.Hd * 2 / 1e9),
                        "old_ref_logp": inp["old_src"], "adamw": args.adamw,
+                       "logits": None if sampling or scoring else
+                       ("kept from the forward" if args.logits == "keep" else "recomputed in the backward"),
                        "step": "sample" if sampling else ("score3" if scoring else "fwdbwd")},
             "step_tflops_8x": round(step_flops8 / (ms / 1e3) / 1e12, 1),
             "step_frac_8x": round(step_flops8 / (ms / 1e3) / 1e12 / burst, 4),
@@ -486,10 +508,21 @@ def main():
         dist.destroy_process_group()
 
 
-def measure_e2e_scoring(grpo, torch, dev, w, inp, heads, steps: int):
+def across_ranks(torch, dev, dist, dt: float, n_tok: int):
+    """(slowest rank's seconds per step, tokens summed over ranks)."""
+    if dist is None:
+        return dt, n_tok
+    t = torch.tensor([dt, float(n_tok)], dtype=torch.float64, device=dev)
+    dist.all_reduce(t[:1], op=dist.ReduceOp.MAX)
+    dist.all_reduce(t[1:], op=dist.ReduceOp.SUM)
+    return float(t[0].item()), int(t[1].item())
+
+
+def measure_e2e_scoring(grpo, torch, dev, w, inp, heads, steps: int, dist=None):
     """Public API, rollout scoring: H2D of the batch (H, targets, mask) from pinned host
     memory, the three LM heads resident on the device (model weights), D2H of the
-    three log-prob rows."""
+    three log-prob rows.  Across ranks each scores its own batch (no exchange);
+    the time is the slowest rank's and the tokens are summed."""
     n_valid = int(inp["m"].sum())
 
     def pin(a, dt):
@@ -507,22 +540,26 @@ def measure_e2e_scoring(grpo, torch, dev, w, inp, heads, steps: int):
         torch.cuda.current_stream(dev).synchronize()
 
     one()
+    if dist is not None:
+        dist.barrier()
     t0 = time.perf_counter()
     for _ in range(steps):
         one()
-    dt = (time.perf_counter() - t0) / steps
-    n_valid = int(inp["m"].sum())
-    return {"value": round(n_valid / dt, 1), "unit": "tokens/s", "ms_per_step": round(dt * 1e3, 2),
+    dt, n_tok = across_ranks(torch, dev, dist, (time.perf_counter() - t0) / steps, n_valid)
+    return {"value": round(n_tok / dt, 1), "unit": "tokens/s", "ms_per_step": round(dt * 1e3, 2),
             "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h), "steps": steps,
             "what": "H, targets, mask copied from pinned host memory each step; the policy / old / reference "
                     "heads resident on the device; the log-probs read back"}
 
 
-def measure_e2e(grpo, torch, dev, w, inp, steps: int):
+def measure_e2e(grpo, torch, dev, w, inp, steps: int, dist=None, ws=None):
     """Public API, one training step: H2D of the batch (H, targets, mask, old / ref
     log-probs, rewards) from pinned host memory, the LM head W resident on the
     device (the parameter being trained), D2H of the loss; dH and dW stay on the
-    device, where the trunk's backward and the optimiser consume them."""
+    device, where the trunk's backward and the optimiser consume them.  Across
+    ranks every rank runs the data-parallel call on its own batch; the time is
+    the slowest rank's and the tokens are summed, like the device-timed value."""
+    from paper_2507_05687_gb300 import dp
     n_valid = int(inp["m"].sum())
 
     def pin(a, dt):
@@ -535,28 +572,34 @@ def measure_e2e(grpo, torch, dev, w, inp, steps: int):
     d2h = 4
     out = (torch.empty(1, dtype=torch.float32, device=dev), torch.empty(w.T, w.Hd, dtype=torch.float32, device=dev),
            torch.empty(w.V, w.Hd, dtype=torch.float32, device=dev))
-    ws = grpo.workspace(w.T, w.Hd, w.V, grpo.GRPO_WS_LOSS, dev, max_valid=n_valid)
+    if ws is None:
+        ws = grpo.loss_workspace(w.T, w.Hd, w.V, dev, max_valid=n_valid)
 
     def one():
         adv = grpo.group_advantages(hr.to(dev, non_blocking=True), w.G, w.adv_eps)
-        loss, _, _ = grpo.loss_fwd_bwd(hH, Wd, hy, hm, hold, href, adv, w.n_resp, w.L, w.clip_eps, w.beta,
-                                       ws=ws, out=out)
+        if dist is None:
+            loss, _, _ = grpo.loss_fwd_bwd(hH, Wd, hy, hm, hold, href, adv, w.n_resp, w.L, w.clip_eps, w.beta,
+                                           ws=ws, out=out)
+        else:
+            loss, _, _ = dp.dp_loss_fwd_bwd(hH, Wd, hy, hm, hold, href, adv, w.n_resp, w.L, w.clip_eps, w.beta, 0,
+                                            n_valid, ws=ws, out=out)
         return loss.item()
 
     one()
     torch.cuda.synchronize(dev)
+    if dist is not None:
+        dist.barrier()
     t0 = time.perf_counter()
     for _ in range(steps):
         one()
-    dt = (time.perf_counter() - t0) / steps
-    n_valid = int(inp["m"].sum())
-    return {"value": round(n_valid / dt, 1), "unit": "tokens/s", "ms_per_step": round(dt * 1e3, 2),
+    dt, n_tok = across_ranks(torch, dev, dist, (time.perf_counter() - t0) / steps, n_valid)
+    return {"value": round(n_tok / dt, 1), "unit": "tokens/s", "ms_per_step": round(dt * 1e3, 2),
             "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h), "steps": steps,
             "what": "H, targets, mask, old/ref log-probs, rewards copied from pinned host memory each step; W "
                     "resident on the device; the loss read back; dH, dW left on the device"}
 
 
-def measure_e2e_offload(grpo, torch, dev, w, inp, steps: int):
+def measure_e2e_offload(grpo, torch, dev, w, inp, steps: int, ws=None):
     """Public API with everything on the host (a host-offloaded head): H2D of the
     batch and of W, the step, D2H of loss, dH, dW (dW streamed chunk by chunk)."""
     n_valid = int(inp["m"].sum())
@@ -574,7 +617,8 @@ def measure_e2e_offload(grpo, torch, dev, w, inp, steps: int):
     # the caller's own buffers, allocated once: pinned host outputs and a device workspace
     hout = (torch.empty(1, dtype=torch.float32).pin_memory(), torch.empty(w.T, w.Hd, dtype=torch.float32).pin_memory(),
             torch.empty(w.V, w.Hd, dtype=torch.float32).pin_memory())
-    ws = grpo.workspace(w.T, w.Hd, w.V, grpo.GRPO_WS_LOSS, dev, max_valid=n_valid)
+    if ws is None:
+        ws = grpo.loss_workspace(w.T, w.Hd, w.V, dev, max_valid=n_valid)
 
     def one():
         adv = grpo.group_advantages(hr.to(dev, non_blocking=True), w.G, w.adv_eps)

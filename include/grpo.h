@@ -51,8 +51,20 @@ typedef enum {
                                  (grpo_workspace_bytes_rows); outputs are invalid */
 } grpo_status;
 
-/* Which call a workspace is sized for (grpo_workspace_bytes `which`). */
-enum { GRPO_WS_LOGPROBS = 0, GRPO_WS_LOSS = 1, GRPO_WS_LOGPROBS_HEADS = 2, GRPO_WS_SAMPLE = 3 };
+/*
+ * Which call a workspace is sized for (grpo_workspace_bytes `which`).
+ * GRPO_WS_LOSS_LOGITS sizes a loss workspace that also keeps the fp32 logits
+ * of the forward ([rows x V], 4 bytes each: 12.2 GB for 19,572 unmasked rows
+ * at V 155136) so that the backward forms dZ from them with an HBM-bound
+ * pass instead of recomputing the logits GEMM; see grpo_loss_plan.
+ */
+enum {
+  GRPO_WS_LOGPROBS = 0,
+  GRPO_WS_LOSS = 1,
+  GRPO_WS_LOGPROBS_HEADS = 2,
+  GRPO_WS_SAMPLE = 3,
+  GRPO_WS_LOSS_LOGITS = 4
+};
 
 /* Most LM heads grpo_token_logprobs_heads sweeps in one call. */
 enum { GRPO_MAX_HEADS = 4 };
@@ -153,7 +165,10 @@ grpo_status grpo_gumbel_noise(uint64_t seed, uint64_t offset, int64_t row0, int6
  *   loss_out             device pointer to one fp32
  *   dH                   [T x Hd] fp32 device; padding rows get 0
  *   dW                   [V x Hd] fp32 device
- *   ws                   at least grpo_workspace_bytes(T, Hd, V, GRPO_WS_LOSS) bytes
+ *   ws                   at least grpo_workspace_bytes(T, Hd, V, GRPO_WS_LOSS) bytes;
+ *                        with grpo_workspace_bytes(T, Hd, V, GRPO_WS_LOSS_LOGITS)
+ *                        the logits are kept from the forward for the backward
+ *                        (faster; bit-identical results, see grpo_loss_plan)
  * Requires n_resp >= 1, L >= 1, clip_eps >= 0, agg_mode in {0, 1}, dH and dW
  * 16-byte aligned, and the limits of grpo_token_logprobs.
  */
@@ -310,8 +325,9 @@ grpo_status grpo_token_logprobs_noalloc(const uint16_t* H, const uint16_t* W, co
 
 /*
  * Bytes of workspace the call `which` (GRPO_WS_LOGPROBS, GRPO_WS_LOSS,
- * GRPO_WS_LOGPROBS_HEADS or GRPO_WS_SAMPLE) needs for T tokens, hidden size Hd and vocabulary V.  Returns 0 for
- * arguments the calls would reject.  Sized for the worst case N_valid = T.
+ * GRPO_WS_LOGPROBS_HEADS, GRPO_WS_SAMPLE or GRPO_WS_LOSS_LOGITS) needs for T
+ * tokens, hidden size Hd and vocabulary V.  Returns 0 for arguments the calls
+ * would reject.  Sized for the worst case N_valid = T.
  */
 size_t grpo_workspace_bytes(int64_t T, int32_t Hd, int64_t V, int32_t which);
 
@@ -331,6 +347,25 @@ size_t grpo_workspace_bytes(int64_t T, int32_t Hd, int64_t V, int32_t which);
  * or a negative max_valid; max_valid >= T gives grpo_workspace_bytes.
  */
 size_t grpo_workspace_bytes_rows(int64_t T, int64_t max_valid, int32_t Hd, int64_t V, int32_t which);
+
+/*
+ * How the loss calls (grpo_loss_fwd_bwd and its variants) use a workspace of
+ * ws_bytes for T tokens, hidden size Hd and vocabulary V (no device work; the
+ * paper has no counterpart).  Returns 1 when the forward keeps the fp32
+ * logits for the backward, 0 when the backward recomputes them with a second
+ * logits GEMM, -1 for arguments or a workspace the calls would reject; *rows
+ * (if not null) gets the row capacity (unmasked rows the call can hold).
+ * The logits are kept when the workspace holds them at the row capacity the
+ * plain loss layout gives (so a plain workspace never loses capacity to
+ * them), or when ws_bytes is exactly what grpo_workspace_bytes or
+ * grpo_workspace_bytes_rows returns for GRPO_WS_LOSS_LOGITS, in which case the
+ * capacity is the one it was sized for (max_valid rounded up to 256 rows).
+ * A workspace of another size (e.g. rounded up) that does not hold the logits
+ * at the plain capacity runs the recomputing backward.
+ * Both ways give bit-identical loss, dH and dW: the two GEMMs accumulate the
+ * same logits in the same order, and both form dZ with the same arithmetic.
+ */
+int32_t grpo_loss_plan(int64_t T, int32_t Hd, int64_t V, size_t ws_bytes, int64_t* rows);
 
 /*
  * Synchronises `stream`, reads the device status word of workspace `ws`
@@ -359,7 +394,8 @@ enum {
   GRPO_K_DH_ROWS = 8,     /* dH rows from the compacted order to the padded one (padding rows 0) */
   GRPO_K_ADAMW = 9,       /* standalone AdamW step (grpo_adamw_step) */
   GRPO_K_SAMPLE_GEMM = 10, /* logits GEMM + log-sum-exp + Gumbel-max draw */
-  GRPO_K_TRANSPOSE = 11   /* K-major (transposed) copy of the gathered hidden states for dW */
+  GRPO_K_TRANSPOSE = 11,  /* K-major (transposed) copy of the gathered hidden states for dW */
+  GRPO_K_DZ_LOGITS = 12   /* kept logits -> dZ chunk (bf16), element-wise */
 };
 
 /*

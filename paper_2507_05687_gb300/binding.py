@@ -32,6 +32,7 @@ GRPO_WS_LOGPROBS = 0
 GRPO_WS_LOSS = 1
 GRPO_WS_LOGPROBS_HEADS = 2
 GRPO_WS_SAMPLE = 3
+GRPO_WS_LOSS_LOGITS = 4
 GRPO_MAX_HEADS = 4
 
 # name -> (restype, argtypes); mirrors include/grpo.h
@@ -65,6 +66,7 @@ SIGNATURES = {
     "grpo_token_logprobs_noalloc": (ctypes.c_int, [_P, _P, _P, _P, _I64, _I32, _I64, _P, _P]),
     "grpo_workspace_bytes": (ctypes.c_size_t, [_I64, _I32, _I64, _I32]),
     "grpo_workspace_bytes_rows": (ctypes.c_size_t, [_I64, _I64, _I32, _I64, _I32]),
+    "grpo_loss_plan": (ctypes.c_int32, [_I64, _I32, _I64, ctypes.c_size_t, _P]),
     "grpo_check_device_status": (ctypes.c_int, [_P, _P]),
     "grpo_status_string": (ctypes.c_char_p, [ctypes.c_int]),
     "grpo_trace_enable": (ctypes.c_int, [_I32]),
@@ -174,6 +176,29 @@ def workspace_bytes(T: int, Hd: int, V: int, which: int) -> int:
 def workspace_bytes_rows(T: int, max_valid: int, Hd: int, V: int, which: int) -> int:
     """grpo_workspace_bytes_rows: scratch bytes for batches with at most max_valid unmasked rows."""
     return int(load().grpo_workspace_bytes_rows(int(T), int(max_valid), int(Hd), int(V), int(which)))
+
+
+def loss_plan(T: int, Hd: int, V: int, ws_bytes: int) -> Tuple[int, int]:
+    """grpo_loss_plan: (1 if the loss calls keep the logits for the backward
+    with a workspace of ws_bytes, else 0; the row capacity)."""
+    rows = ctypes.c_int64(0)
+    kept = int(load().grpo_loss_plan(int(T), int(Hd), int(V), int(ws_bytes), ctypes.byref(rows)))
+    if kept < 0:
+        raise GrpoError(GRPO_ERR_WORKSPACE, "grpo_loss_plan")
+    return kept, int(rows.value)
+
+
+def loss_workspace(T: int, Hd: int, V: int, device=None, max_valid: Optional[int] = None) -> torch.Tensor:
+    """A workspace for the loss calls: one that keeps the logits from the
+    forward for the backward (GRPO_WS_LOSS_LOGITS) when that fits in half of
+    the device's free memory, else the plain one (GRPO_WS_LOSS).  Both give
+    the same results; the first skips the backward's logits GEMM."""
+    dev = torch.device(device or "cuda")
+    kept = workspace_bytes(T, Hd, V, GRPO_WS_LOSS_LOGITS) if max_valid is None else \
+        workspace_bytes_rows(T, max_valid, Hd, V, GRPO_WS_LOSS_LOGITS)
+    free = torch.cuda.mem_get_info(dev)[0] if dev.type == "cuda" else 0
+    which = GRPO_WS_LOSS_LOGITS if 0 < kept <= free // 2 else GRPO_WS_LOSS
+    return workspace(T, Hd, V, which, dev, max_valid=max_valid)
 
 
 def workspace(T: int, Hd: int, V: int, which: int, device=None, max_valid: Optional[int] = None) -> torch.Tensor:
@@ -295,7 +320,7 @@ def loss_fwd_bwd(H: torch.Tensor, W: torch.Tensor, targets: torch.Tensor, mask: 
     for name, t in (("targets", targets), ("mask", mask), ("old_logp", old_logp), ("ref_logp", ref_logp)):
         _shape(t, (T,), name)
     _shape(adv, (int(n_resp),), "adv")
-    ws = workspace(T, Hd, V, GRPO_WS_LOSS, dev) if ws is None else _workspace(ws, dev)
+    ws = loss_workspace(T, Hd, V, dev) if ws is None else _workspace(ws, dev)
     host_out = None
     if out is not None and not out[0].is_cuda:
         host_out, out = out, None  # results land in the caller's host buffers
@@ -379,7 +404,7 @@ def loss_fwd_bwd_adamw(H: torch.Tensor, W: torch.Tensor, targets: torch.Tensor, 
     for name, t in (("targets", targets), ("mask", mask), ("old_logp", old_logp), ("ref_logp", ref_logp)):
         _shape(t, (T,), name)
     _shape(adv, (int(n_resp),), "adv")
-    ws = workspace(T, Hd, V, GRPO_WS_LOSS, dev) if ws is None else _workspace(ws, dev)
+    ws = loss_workspace(T, Hd, V, dev) if ws is None else _workspace(ws, dev)
     if out is None:
         out = (torch.empty(1, dtype=torch.float32, device=dev), torch.empty(T, Hd, dtype=torch.float32, device=dev))
     loss = _output(out[0], (1,), torch.float32, dev, "out[0]")

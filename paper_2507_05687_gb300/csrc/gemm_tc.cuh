@@ -21,6 +21,9 @@
 //   kEpiLse  forward of the log-softmax (pi_theta in Eq. 1): per row a running
 //            max and sum of exp over the tiles of one vocabulary split, plus
 //            the logit of the target token; the logits never leave the SM.
+//   kEpiLseZ the same, and the fp32 logits themselves are stored (through the
+//            output tensor map, like kEpiF32), so that the backward forms dZ
+//            from them instead of recomputing the GEMM.
 //   kEpiDz   backward: recomputes the logits of one vocabulary chunk and
 //            writes dZ = g (onehot(y) - softmax) as bf16.
 //   kEpiF32  fp32 tile written as is or added to the existing values:
@@ -68,7 +71,7 @@ struct TileCfg {
   static constexpr int kStageBytes = kABytes + kBBytes;
 };
 
-enum { kEpiLse = 0, kEpiDz = 1, kEpiF32 = 2, kEpiAdam = 3, kEpiSample = 4 };
+enum { kEpiLse = 0, kEpiDz = 1, kEpiF32 = 2, kEpiAdam = 3, kEpiSample = 4, kEpiLseZ = 5 };
 
 // Epilogue warps per CTA: 4 = one per TMEM lane quarter (each thread walks its
 // row's 256 columns); 8 = two per quarter, each taking half the columns.  The
@@ -80,12 +83,18 @@ struct EpiShape {
   static constexpr int kWarps = kEpi == kEpiSample ? 8 : 4;
   static constexpr int kHalves = kWarps / 4;    // column halves of a tile, one per warp of a quarter
   static constexpr int kThreads = 64 + 32 * kWarps;
-  static constexpr bool kTmaOut = kEpi == kEpiDz || kEpi == kEpiF32 || kEpi == kEpiAdam;
-  // one warp's 32 x 32 block in shared memory: bf16 dZ / fp32 output, two per
-  // warp; kEpiAdam: fp32 weights, first and second moments (4 KB each) and the
+  static constexpr bool kTmaOut = kEpi == kEpiDz || kEpi == kEpiF32 || kEpi == kEpiAdam || kEpi == kEpiLseZ;
+  // element type of the output tensor map: fp32 (128-byte rows of 32, 128-byte
+  // swizzle) or bf16 (kEpiDz: 64-byte rows, 64-byte swizzle)
+  static constexpr bool kOutF32 = kEpi == kEpiF32 || kEpi == kEpiLseZ || kEpi == kEpiAdam;
+  // one warp's 32 x 32 block in shared memory: bf16 dZ / fp32 output or
+  // logits, two per warp; kEpiAdam: fp32 weights, first and second moments (4 KB each) and the
   // bf16 weights (2 KB), one per warp (the dW K-loop is long enough to hide it)
   static constexpr int kBlockBytes =
-      kEpi == kEpiDz ? 32 * 32 * 2 : kEpi == kEpiF32 ? 32 * 32 * 4 : kEpi == kEpiAdam ? 3 * 4096 + 2048 : 0;
+      kEpi == kEpiDz                        ? 32 * 32 * 2
+      : kEpi == kEpiF32 || kEpi == kEpiLseZ ? 32 * 32 * 4
+      : kEpi == kEpiAdam                    ? 3 * 4096 + 2048
+                                            : 0;
   static constexpr int kBlocks = kEpi == kEpiAdam ? 1 : 2;
   static constexpr int kOutBytes = kBlocks * kBlockBytes * kWarps;
 };
@@ -220,7 +229,7 @@ __device__ __forceinline__ void epi_begin(EpiRow& e, const GemmArgs& a, int r, i
   e.best_c = -1;
   if (kEpi == kEpiSample) {
     if (e.rv) e.orow = a.row_map[r];
-  } else if (kEpi == kEpiLse) {
+  } else if (kEpi == kEpiLse || kEpi == kEpiLseZ) {
     e.y = e.rv ? a.yc[r] : -1;
   } else if (kEpi == kEpiDz) {
     if (e.rv) {
@@ -366,7 +375,15 @@ __device__ __forceinline__ bool epi_tile(EpiRow& e, const GemmArgs& a, uint32_t 
       for (int j = 0; j < 32; ++j) v[j] = 0.f;
     }
     const int cb = col0 + c * 32;
-    if (kEpi == kEpiLse) {
+    if (kEpi == kEpiLse || kEpi == kEpiLseZ) {
+      // kEpiLseZ: the raw logits first (blocks wholly past M or N skipped, the
+      // tensor map clips the rest)
+      if (kEpi == kEpiLseZ && row0 < m_rows && cb < a.N) {
+        uint32_t bits[32];
+#pragma unroll
+        for (int j = 0; j < 32; ++j) bits[j] = __float_as_uint(v[j]);
+        out_block<32>(os, bits, cb, row0, false);
+      }
       if (cb + 32 > a.N) {
 #pragma unroll
         for (int j = 0; j < 32; ++j)
@@ -430,10 +447,8 @@ __device__ __forceinline__ bool epi_tile(EpiRow& e, const GemmArgs& a, uint32_t 
       uint32_t packed[16];
 #pragma unroll
       for (int j = 0; j < 32; j += 2) {
-        float d0 = -e.gr * fast_exp2(fmaf(v[j], kLog2e, -e.lse2));
-        float d1 = -e.gr * fast_exp2(fmaf(v[j + 1], kLog2e, -e.lse2));
-        if (gc + j == e.y) d0 += e.gr;
-        if (gc + j + 1 == e.y) d1 += e.gr;
+        float d0 = dz_value(v[j], e.lse2, e.gr, gc + j == e.y);
+        float d1 = dz_value(v[j + 1], e.lse2, e.gr, gc + j + 1 == e.y);
         if (cb + j >= a.N || !e.rv) d0 = 0.f;
         if (cb + j + 1 >= a.N || !e.rv) d1 = 0.f;
         packed[j / 2] = pack_bf16x2(d0, d1);
@@ -467,7 +482,7 @@ __device__ __forceinline__ void epi_end(const EpiRow& e, const GemmArgs& a, int 
     a.best_c[at] = e.best_c;
     a.best_z[at] = e.best_z;
   }
-  if (kEpi == kEpiLse && e.rv) {
+  if ((kEpi == kEpiLse || kEpi == kEpiLseZ) && e.rv) {
     a.part_m[entry * a.ldp + e.r] = e.run_m;
     a.part_s[entry * a.ldp + e.r] = e.run_s;
     if (e.found) a.zy[static_cast<long>(head) * a.ldp + e.r] = e.zy_val;

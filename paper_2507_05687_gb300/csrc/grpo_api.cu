@@ -56,17 +56,19 @@ int64_t vocab_chunk(int64_t V) {
 // grpo_workspace_bytes_rows for batches with few unmasked rows.
 struct Layout {
   int64_t T_pad, rows, nsplit, nblk_scan, nblk_loss, vchunk;
+  int64_t ldz;    // leading dimension (fp32 elements) of the stored logits; 0: not stored
   int lse_tiles;  // vocabulary tiles (of 256) per forward work unit
   size_t status, n_valid, counts, offsets, cidx, rank_of, yc, zy, part_m, part_s, lse_c, g_c,
-      block_loss, resp_len, best_s, best_c, best_z, Hc, HcT, dz, dhc, total;
+      block_loss, resp_len, best_s, best_c, best_z, Hc, HcT, dz, dhc, z, total;
 };
 
 bool make_layout(int64_t T, int32_t Hd, int64_t V, int32_t which, Layout* L, int64_t rows_cap = -1) {
   if (T < 0 || T >= (int64_t(1) << 31) || Hd <= 0 || Hd % 64 != 0 || V <= 0 ||
       V >= (int64_t(1) << 31) ||
       (which != GRPO_WS_LOGPROBS && which != GRPO_WS_LOSS && which != GRPO_WS_LOGPROBS_HEADS &&
-       which != GRPO_WS_SAMPLE))
+       which != GRPO_WS_SAMPLE && which != GRPO_WS_LOSS_LOGITS))
     return false;
+  const bool loss = which == GRPO_WS_LOSS || which == GRPO_WS_LOSS_LOGITS;
   const size_t heads = which == GRPO_WS_LOGPROBS_HEADS ? kMaxHeads : 1;
   L->T_pad = round_up(std::max<int64_t>(T, 1), kRowAlign);
   const int64_t vtiles = (V + kTileN - 1) / kTileN;
@@ -80,7 +82,8 @@ bool make_layout(int64_t T, int32_t Hd, int64_t V, int32_t which, Layout* L, int
   L->rows = rows_cap < 0 ? L->T_pad : std::min(L->T_pad, round_up(std::max<int64_t>(rows_cap, 1), kRowAlign));
   L->nblk_scan = (std::max<int64_t>(T, 1) + kScanChunk - 1) / kScanChunk;
   L->nblk_loss = (L->rows + kLossThreads - 1) / kLossThreads;
-  L->vchunk = which == GRPO_WS_LOSS ? vocab_chunk(V) : 0;
+  L->vchunk = loss ? vocab_chunk(V) : 0;
+  L->ldz = which == GRPO_WS_LOSS_LOGITS ? round_up(V, 64) : 0;
   size_t off = 0;
   auto take = [&](size_t bytes, size_t align) {
     off = (off + align - 1) / align * align;
@@ -111,10 +114,13 @@ bool make_layout(int64_t T, int32_t Hd, int64_t V, int32_t which, Layout* L, int
   L->Hc = take(2 * cr * static_cast<size_t>(Hd), 1024);
   // H_c transposed (rows [Hd x rows], or k-blocks [rows / 64][Hd][64] when a
   // row would exceed kMaxTransposedRowBytes): the K-major B operand of the dW GEMM
-  L->HcT = which == GRPO_WS_LOSS ? take(2 * cr * static_cast<size_t>(Hd), 1024) : off;
-  L->dz = which == GRPO_WS_LOSS ? take(2 * cr * static_cast<size_t>(L->vchunk), 1024) : off;
+  L->HcT = loss ? take(2 * cr * static_cast<size_t>(Hd), 1024) : off;
+  L->dz = loss ? take(2 * cr * static_cast<size_t>(L->vchunk), 1024) : off;
   // dH over the compacted rows, accumulated across vocabulary chunks
-  L->dhc = which == GRPO_WS_LOSS ? take(4 * cr * static_cast<size_t>(Hd), 1024) : off;
+  L->dhc = loss ? take(4 * cr * static_cast<size_t>(Hd), 1024) : off;
+  // the fp32 logits [rows x ldz] of the forward, kept for the backward (last,
+  // so that every other region sits where the plain loss layout has it)
+  L->z = take(4 * cr * static_cast<size_t>(L->ldz), 1024);
   L->total = (off + 1023) / 1024 * 1024;
   return true;
 }
@@ -139,6 +145,23 @@ bool fit_layout(int64_t T, int32_t Hd, int64_t V, int32_t which, size_t ws_bytes
     lo = 1;
   }
   return make_layout(T, Hd, V, which, L, lo * kRowAlign);
+}
+
+// The layout of a loss call with a workspace of ws_bytes.  The logits are
+// kept from the forward to the backward (a) when the workspace holds them at
+// the row capacity the plain loss layout gives (fit_layout), or (b) when
+// ws_bytes is exactly a kept-logits size (grpo_workspace_bytes(_rows) with
+// GRPO_WS_LOSS_LOGITS), and not also exactly a plain one: a workspace sized
+// for max_valid rows with the logits is larger than the plain layout needs
+// for more rows, so its size, not the largest plain capacity, says what it
+// was made for.  Any other size keeps the plain layout's capacity.
+bool fit_loss_layout(int64_t T, int32_t Hd, int64_t V, size_t ws_bytes, Layout* L) {
+  if (!fit_layout(T, Hd, V, GRPO_WS_LOSS, ws_bytes, L)) return false;
+  Layout kept;
+  if (fit_layout(T, Hd, V, GRPO_WS_LOSS_LOGITS, ws_bytes, &kept) &&
+      (kept.rows >= L->rows || (kept.total == ws_bytes && L->total != ws_bytes)))
+    *L = kept;
+  return true;
 }
 
 // ---------------------------------------------------------------- driver entry points
@@ -230,7 +253,8 @@ bool device_info(DeviceInfo* out) {
         cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
       return false;
     if (major != 10 || minor != 3) return false;
-    if (!prepare_kernels<kEpiLse, false, false>(&pairs) || !prepare_kernels<kEpiDz, false, false>(&pairs) ||
+    if (!prepare_kernels<kEpiLse, false, false>(&pairs) || !prepare_kernels<kEpiLseZ, false, false>(&pairs) ||
+        !prepare_kernels<kEpiDz, false, false>(&pairs) ||
         !prepare_kernels<kEpiF32, false, true>(&pairs) || !prepare_kernels<kEpiF32, true, false>(&pairs) ||
         !prepare_kernels<kEpiF32, true, false, true>(&pairs) || !prepare_kernels<kEpiAdam, true, false, true>(&pairs) ||
         !prepare_kernels<kEpiAdam, true, false>(&pairs) || !prepare_kernels<kEpiSample, false, false>(&pairs))
@@ -451,7 +475,7 @@ cudaError_t launch_gemm_cfg(const Operand& A, const Operand* B, const GemmArgs& 
         !out_map(&tb[2], &D[2], true) || !out_map(&tb[3], &D[3], false))
       return cudaErrorInvalidValue;
   } else if (EpiShape<E>::kTmaOut) {
-    if (!out_map(&td, D, E == kEpiF32)) return cudaErrorInvalidValue;
+    if (!out_map(&td, D, EpiShape<E>::kOutF32)) return cudaErrorInvalidValue;
   } else {
     td = ta;  // not read
   }
@@ -524,6 +548,7 @@ cudaError_t run_compaction(const uint16_t* H, const int32_t* targets, const uint
 
 // Forward GEMM with the log-softmax epilogue over all V columns of each of
 // the n_heads LM heads (one launch; the heads share the gathered hidden states).
+// With a layout that keeps the logits (one head), they are stored as well.
 cudaError_t run_lse(const uint16_t* const* W, int n_heads, int32_t Hd, int64_t V, void* ws, const Layout& Ly,
                     const DeviceInfo& di, cudaStream_t s) {
   GemmArgs a{};
@@ -557,6 +582,12 @@ cudaError_t run_lse(const uint16_t* const* W, int n_heads, int32_t Hd, int64_t V
   for (int h = 0; h < n_heads; ++h)
     B[h] = Operand{W[h], static_cast<uint64_t>(V), static_cast<uint64_t>(Hd), static_cast<uint64_t>(Hd)};
   TraceScope trace(GRPO_K_LSE_GEMM, V * n_heads, s);
+  if (Ly.ldz > 0) {
+    if (n_heads != 1) return cudaErrorInvalidValue;
+    const OutMat Z{at<float>(ws, Ly.z), static_cast<uint64_t>(Ly.rows), static_cast<uint64_t>(V),
+                   static_cast<uint64_t>(Ly.ldz)};
+    return launch_gemm<kEpiLseZ, false, false>(A, B, a, Ly.rows, di, s, &Z);
+  }
   return launch_gemm<kEpiLse, false, false>(A, B, a, Ly.rows, di, s);
 }
 
@@ -605,6 +636,13 @@ size_t grpo_workspace_bytes_rows(int64_t T, int64_t max_valid, int32_t Hd, int64
 size_t grpo_workspace_bytes(int64_t T, int32_t Hd, int64_t V, int32_t which) {
   Layout L;
   return make_layout(T, Hd, V, which, &L) ? L.total : 0;
+}
+
+int32_t grpo_loss_plan(int64_t T, int32_t Hd, int64_t V, size_t ws_bytes, int64_t* rows) {
+  Layout L;
+  if (!fit_loss_layout(T, Hd, V, ws_bytes, &L)) return -1;
+  if (rows) *rows = L.rows;
+  return L.ldz > 0 ? 1 : 0;
 }
 
 grpo_status grpo_group_advantages(const float* rewards, int64_t n_resp, int32_t G, float eps,
@@ -871,7 +909,7 @@ grpo_status loss_impl(const uint16_t* H, const uint16_t* W, const int32_t* targe
     return GRPO_ERR_INVALID_ARG;
   if (!aligned(W, 16) || !aligned(H, 16) || !aligned(dH, 16) || !aligned(dW, 16))
     return GRPO_ERR_INVALID_ARG;
-  if (!ws || !aligned(ws, 256) || !fit_layout(T, Hd, V, GRPO_WS_LOSS, ws_bytes, &Ly))
+  if (!ws || !aligned(ws, 256) || !fit_loss_layout(T, Hd, V, ws_bytes, &Ly))
     return GRPO_ERR_WORKSPACE;
   if (chunk_events) {
     const int64_t chunks = (V + Ly.vchunk - 1) / Ly.vchunk;
@@ -939,7 +977,14 @@ grpo_status loss_impl(const uint16_t* H, const uint16_t* W, const int32_t* targe
   const OutMat outDh{dHc, tp, hd, hd};
   for (int64_t c0 = 0; c0 < V && e == cudaSuccess; c0 += vc) {
     const int64_t width = std::min<int64_t>(vc, V - c0);
-    {  // dZ chunk = g (onehot - softmax) from recomputed logits
+    if (Ly.ldz > 0) {  // dZ chunk = g (onehot - softmax) from the logits the forward kept
+      TraceScope trace(GRPO_K_DZ_LOGITS, width, s);
+      const int blocks = static_cast<int>(std::min<int64_t>(Ly.rows, int64_t(sms) * 8));
+      dz_from_logits_kernel<<<blocks, 256, 0, s>>>(at<float>(ws, Ly.z), Ly.ldz, at<float>(ws, Ly.lse_c),
+                                                   at<float>(ws, Ly.g_c), at<int>(ws, Ly.yc), n_valid, Ly.rows,
+                                                   c0, static_cast<int>(width), static_cast<int>(vc), dz);
+      e = cudaGetLastError();
+    } else {  // dZ chunk = g (onehot - softmax) from recomputed logits
       GemmArgs a{};
       a.n_valid = n_valid;
       a.m_dyn = 1;

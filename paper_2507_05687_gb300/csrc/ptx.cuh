@@ -420,4 +420,16 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
   return r;
 }
 
+// One element of dZ = g (onehot(y) - softmax(z)), the gradient of the loss
+// through the log-softmax (Eq. 1 differentiated through log pi_theta):
+// z the logit, lse2 the row's log-sum-exp in log2 units, g = dloss/dlogp of
+// the row, target whether this column is the row's token.  Written with
+// explicitly rounded operations (nothing left for the compiler to contract)
+// so that every kernel that forms dZ gets the same bits from the same z.
+__device__ __forceinline__ float dz_value(float z, float lse2, float g, bool target) {
+  const float kLog2e = 1.4426950408889634f;
+  const float d = __fmul_rn(-g, fast_exp2(__fmaf_rn(z, kLog2e, -lse2)));
+  return target ? __fadd_rn(d, g) : d;
+}
+
 }  // namespace grpo

@@ -5,6 +5,7 @@ import ctypes
 import os
 import re
 
+import numpy as np
 import pytest
 
 import paper_2507_05687_gb300 as grpo
@@ -64,7 +65,7 @@ FAKE = 0x10000  # never dereferenced: every call below is rejected on the host
 
 def test_workspace_sized_for_fewer_rows(lib):
     f, g = grpo.workspace_bytes, grpo.workspace_bytes_rows
-    for which in (0, 1, 2, 3):
+    for which in (0, 1, 2, 3, 4):
         full = f(32768, 4096, 155136, which)
         assert g(32768, 32768, 4096, 155136, which) == full == g(32768, 10**9, 4096, 155136, which)
         sizes = [g(32768, n, 4096, 155136, which) for n in (1, 256, 257, 5000, 20000)]
@@ -72,6 +73,37 @@ def test_workspace_sized_for_fewer_rows(lib):
         assert g(32768, -1, 4096, 155136, which) == 0
     # a ragged batch: 1M padded rows, 168k unmasked
     assert g(1 << 20, 168251, 4096, 155136, 1) < 0.2 * f(1 << 20, 4096, 155136, 1)
+
+
+def test_loss_plan_keeps_logits_only_without_losing_capacity(lib):
+    """grpo_loss_plan: a GRPO_WS_LOSS_LOGITS workspace is the plain loss one plus
+    the fp32 logits [rows x V]; the loss calls keep the logits exactly when the
+    workspace holds them at the row capacity the plain layout gives."""
+    f, g, plan = grpo.workspace_bytes, grpo.workspace_bytes_rows, grpo.loss_plan
+    T, Hd, V = 32768, 4096, 155136
+    kept, plain = f(T, Hd, V, grpo.GRPO_WS_LOSS_LOGITS), f(T, Hd, V, grpo.GRPO_WS_LOSS)
+    assert kept - plain == 4 * T * V
+    assert plan(T, Hd, V, kept) == (1, T) and plan(T, Hd, V, kept + 5000) == (1, T)
+    assert plan(T, Hd, V, kept - 1) == (0, T) and plan(T, Hd, V, plain) == (0, T)
+    assert plan(T, Hd, V, plain - 1) == (0, T - 256)
+    rng = np.random.default_rng(7)
+    # exactly a kept-logits size: the capacity it was sized for, logits kept
+    for mv in (1, 256, 5000, 19572, 32768):
+        assert plan(T, Hd, V, g(T, mv, Hd, V, grpo.GRPO_WS_LOSS_LOGITS)) == (1, (mv + 255) // 256 * 256)
+        assert plan(T, Hd, V, g(T, mv, Hd, V, grpo.GRPO_WS_LOSS_LOGITS) + 1024)[0] == (mv == 32768)
+    # any other size: the plain layout's capacity, logits kept only at that capacity
+    for ws in rng.integers(g(T, 1, Hd, V, 1), kept + 1, size=200):
+        k, rows = plan(T, Hd, V, int(ws))
+        assert rows % 256 == 0 and g(T, rows, Hd, V, 1) <= ws and (rows == T or g(T, rows + 1, Hd, V, 1) > ws)
+        assert k == (g(T, rows, Hd, V, grpo.GRPO_WS_LOSS_LOGITS) <= ws)
+    # odd vocabulary: logits rows padded to 64 columns
+    assert f(100, 64, 1001, 4) - f(100, 64, 1001, 1) == 4 * 256 * 1024
+    rows = ctypes.c_int64(-5)
+    assert lib.grpo_loss_plan(T, Hd, V, g(T, 1, Hd, V, 1) - 1, ctypes.byref(rows)) == -1 and rows.value == -5
+    for bad in ((-1, Hd, V), (T, 60, V), (T, Hd, 0)):
+        assert lib.grpo_loss_plan(*bad, kept, None) == -1
+    with pytest.raises(grpo.GrpoError):
+        plan(T, Hd, V, 1000)
 
 
 def test_host_rejections(lib):

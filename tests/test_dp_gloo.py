@@ -136,3 +136,42 @@ def test_failed_rank_makes_the_other_raise_not_hang():
     res = _run(0, fail_rank=1)
     assert res[1][1] == "error" and "planted failure" in res[1][2]
     assert res[0][1] == "error"  # the collective timed out or saw the peer leave
+
+
+def _bench_worker(rank, world, port, q):
+    import sys
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    sys.path.insert(0, root)
+    import torch.distributed as dist
+    try:
+        import bench
+        dist.init_process_group("gloo", init_method=f"tcp://127.0.0.1:{port}", rank=rank, world_size=world,
+                                timeout=datetime.timedelta(seconds=20))
+        dt, n = bench.across_ranks(torch, torch.device("cpu"), dist, 0.25 + 0.5 * rank, 1000 + 7 * rank)
+        q.put((rank, "ok", dt, n))
+    except Exception:  # reported to the parent, never swallowed
+        q.put((rank, "error", traceback.format_exc(), None))
+    finally:
+        if dist.is_initialized():
+            dist.destroy_process_group()
+
+
+def test_bench_end_to_end_numbers_combine_slowest_rank_and_all_tokens():
+    """The end-to-end figure across ranks is every rank's tokens over the
+    slowest rank's time, the same rule as the device-timed value."""
+    import bench
+    assert bench.across_ranks(torch, torch.device("cpu"), None, 0.5, 10) == (0.5, 10)
+    ctx = mp.get_context("spawn")
+    q = ctx.Queue()
+    port = _free_port()
+    procs = [ctx.Process(target=_bench_worker, args=(r, 2, port, q)) for r in range(2)]
+    for p in procs:
+        p.start()
+    res = dict((item[0], item) for item in (q.get(timeout=120) for _ in procs))
+    for p in procs:
+        p.join(timeout=60)
+        if p.is_alive():
+            p.kill()
+    for r in range(2):
+        assert res[r][1] == "ok", res[r][2]
+        assert res[r][2] == pytest.approx(0.75) and res[r][3] == 2007

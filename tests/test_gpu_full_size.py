@@ -124,7 +124,9 @@ def test_fwd_bwd_full_size(name):
     adv = oracle.group_advantages(r, w.G, float(np.float32(w.adv_eps)))
 
     H, W = dev_tensor(Hb, torch.bfloat16), dev_tensor(Wb, torch.bfloat16)
-    ws = grpo.workspace(w.T, w.Hd, w.V, grpo.GRPO_WS_LOSS, DEV, max_valid=idx.size)  # as bench.py sizes it
+    # as bench.py sizes it: the unmasked rows, the logits kept from the forward for the backward
+    ws = grpo.workspace(w.T, w.Hd, w.V, grpo.GRPO_WS_LOSS_LOGITS, DEV, max_valid=idx.size)
+    assert grpo.loss_plan(w.T, w.Hd, w.V, ws.numel()) == (1, (idx.size + 255) // 256 * 256)
     adv_d = grpo.group_advantages(dev_tensor(r, torch.float32), w.G, w.adv_eps)
     assert np.array_equal(adv_d.cpu().numpy().view(np.uint32), adv.view(np.uint32))
     loss, dH, dW = grpo.loss_fwd_bwd(H, W, dev_tensor(y, torch.int32), dev_tensor(m, torch.uint8),
@@ -161,6 +163,18 @@ def test_fwd_bwd_full_size(name):
     colsum = dW.double().sum(0)
     colabs = dW.double().abs().sum(0)
     assert (colsum.norm() / colabs.norm()).item() <= 1e-2
+
+    if name == "fwdbwd_8b":
+        # the backward that recomputes the logits gives the same bits
+        del ws
+        ws0 = grpo.workspace(w.T, w.Hd, w.V, grpo.GRPO_WS_LOSS, DEV, max_valid=idx.size)
+        assert grpo.loss_plan(w.T, w.Hd, w.V, ws0.numel())[0] == 0
+        again = grpo.loss_fwd_bwd(H, W, dev_tensor(y, torch.int32), dev_tensor(m, torch.uint8),
+                                  dev_tensor(old, torch.float32), dev_tensor(ref, torch.float32), adv_d,
+                                  w.n_resp, w.L, w.clip_eps, w.beta, 0, ws=ws0)
+        assert grpo.check_device_status(ws0) == grpo.GRPO_OK
+        for a, b in zip((loss, dH, dW), again):
+            assert torch.equal(a, b)
 
 
 def test_sampling_full_size():

@@ -22,7 +22,8 @@ build_mod.build()
 DEV = torch.device("cuda", 0)
 
 
-def test_loss_step_replays_from_a_graph(monkeypatch):
+@pytest.mark.parametrize("kind", ["plain", "kept_logits"])
+def test_loss_step_replays_from_a_graph(kind, monkeypatch):
     monkeypatch.setenv("GRPO_VOCAB_CHUNK", "768")
     w = wl.Workload("g", 2, 4, 60, 128, 2100, "uniform", 1, 60, rewards="mix", seed=wl.SEED_BASE + 950)
     Hb, Wb, y, m, r = wl.gen_hidden(w), wl.gen_weight(w), wl.gen_targets(w), wl.gen_mask(w), wl.gen_rewards(w)
@@ -33,7 +34,8 @@ def test_loss_step_replays_from_a_graph(monkeypatch):
     H, W = dev_tensor(Hb, torch.bfloat16), dev_tensor(Wb, torch.bfloat16)
     yd, md = dev_tensor(y, torch.int32), dev_tensor(m, torch.uint8)
     oldd, refd, rd = dev_tensor(old, torch.float32), dev_tensor(ref, torch.float32), dev_tensor(r, torch.float32)
-    ws = grpo.workspace(w.T, w.Hd, w.V, grpo.GRPO_WS_LOSS, DEV)
+    ws = grpo.workspace(w.T, w.Hd, w.V, grpo.GRPO_WS_LOSS if kind == "plain" else grpo.GRPO_WS_LOSS_LOGITS, DEV)
+    assert grpo.loss_plan(w.T, w.Hd, w.V, ws.numel())[0] == (kind == "kept_logits")
     adv = torch.empty(w.n_resp, dtype=torch.float32, device=DEV)
     out = (torch.empty(1, device=DEV), torch.empty(w.T, w.Hd, device=DEV), torch.empty(w.V, w.Hd, device=DEV))
 

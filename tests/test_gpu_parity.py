@@ -41,9 +41,10 @@ def _dev(c):
                 adv=dev_tensor(c["adv"], torch.float32), r=dev_tensor(c["r"], torch.float32))
 
 
-def _check_fwd_bwd(c, agg_mode=0):
+def _check_fwd_bwd(c, agg_mode=0, kind=grpo.GRPO_WS_LOSS):
     w, d = c["w"], _dev(c)
-    ws = grpo.workspace(w.T, w.Hd, w.V, grpo.GRPO_WS_LOSS, DEV)
+    ws = grpo.workspace(w.T, w.Hd, w.V, kind, DEV)
+    assert grpo.loss_plan(w.T, w.Hd, w.V, ws.numel())[0] == (kind == grpo.GRPO_WS_LOSS_LOGITS)
     loss, dH, dW = grpo.loss_fwd_bwd(d["H"], d["W"], d["y"], d["m"], d["old"], d["ref"], d["adv"],
                                      w.n_resp, w.L, w.clip_eps, w.beta, agg_mode, ws=ws)
     assert grpo.check_device_status(ws) == grpo.GRPO_OK
@@ -224,6 +225,62 @@ def test_clamped_kl(agg_mode):
                           w.n_resp, w.L, w.clip_eps, beta, agg_mode)
     for x, y in zip(a, b):
         assert torch.equal(x, y)
+
+
+KEPT_SHAPES = [
+    # (n_prompts, G, L, Hd, V, vocabulary chunk or None, tile pair)
+    (1, 4, 64, 256, 4096, None, "1"),          # the tiny workload's shape
+    (2, 4, 90, 320, 1800, "512", "1"),         # several chunks, a tail chunk of 264 columns
+    (3, 4, 60, 192, 1001, "256", "1"),         # odd vocabulary: a tail of 233 columns (not a multiple of 8)
+    (3, 4, 60, 192, 2100, "768", "0"),         # 128 x 256 single-CTA tiles
+    (2, 3, 200, 128, 777, None, "1"),          # rows past one 256-row tile, one chunk narrower than a tile
+]
+
+
+@pytest.mark.parametrize("agg_mode", [0, 1])
+@pytest.mark.parametrize("shape", KEPT_SHAPES)
+def test_kept_logits_match_oracle_and_recompute(shape, agg_mode, monkeypatch):
+    """A GRPO_WS_LOSS_LOGITS workspace: the forward stores the fp32 logits and
+    the backward forms dZ from them.  The results meet the oracle bar and equal
+    those of the backward that recomputes the logits, bit for bit."""
+    P, G, L, Hd, V, chunk, pair = shape
+    if chunk:
+        monkeypatch.setenv("GRPO_VOCAB_CHUNK", chunk)
+    monkeypatch.setenv("GRPO_CTA_PAIR", pair)
+    w = wl.Workload("t", P, G, L, Hd, V, "uniform", 1, L, rewards="mix", seed=wl.SEED_BASE + 5300 + V + Hd)
+    c = _case(w, agg_mode)
+    kept = _check_fwd_bwd(c, agg_mode, kind=grpo.GRPO_WS_LOSS_LOGITS)
+    plain = _check_fwd_bwd(c, agg_mode, kind=grpo.GRPO_WS_LOSS)
+    for a, b in zip(kept, plain):
+        assert torch.equal(a, b)
+
+
+def test_kept_logits_lean_workspace_and_capacity(monkeypatch):
+    """A kept-logits workspace sized for the unmasked rows works like the plain
+    lean one (same bits); a batch with more unmasked rows than it holds reports
+    GRPO_ERR_CAPACITY instead of writing past the logits."""
+    monkeypatch.setenv("GRPO_VOCAB_CHUNK", "512")
+    w = wl.Workload("t", 2, 4, 160, 192, 1500, "uniform", 1, 40, rewards="mix", seed=wl.SEED_BASE + 5400)
+    c = _case(w)
+    nv = int(c["m"].sum())
+    assert nv <= 256 < w.T
+    d = _dev(c)
+    res = []
+    for kind in (grpo.GRPO_WS_LOSS_LOGITS, grpo.GRPO_WS_LOSS):
+        ws = grpo.workspace(w.T, w.Hd, w.V, kind, DEV, max_valid=nv)
+        assert grpo.loss_plan(w.T, w.Hd, w.V, ws.numel()) == (int(kind == grpo.GRPO_WS_LOSS_LOGITS), 256)
+        res.append(grpo.loss_fwd_bwd(d["H"], d["W"], d["y"], d["m"], d["old"], d["ref"], d["adv"],
+                                     w.n_resp, w.L, w.clip_eps, w.beta, 0, ws=ws))
+        assert grpo.check_device_status(ws) == grpo.GRPO_OK
+    for a, b in zip(*res):
+        assert torch.equal(a, b)
+    assert rel_fro(res[0][2].double().cpu().numpy(), c["want"]["dW"]) <= GRAD_RTOL
+    # every row unmasked: 1280 rows against a capacity of 256
+    ws = grpo.workspace(w.T, w.Hd, w.V, grpo.GRPO_WS_LOSS_LOGITS, DEV, max_valid=nv)
+    grpo.loss_fwd_bwd(d["H"], d["W"], d["y"], torch.ones_like(d["m"]), d["old"], d["ref"], d["adv"], w.n_resp,
+                      w.L, w.clip_eps, w.beta, 0, ws=ws)
+    assert grpo.check_device_status(ws) == grpo.GRPO_ERR_CAPACITY
+    _check_fwd_bwd(c, kind=grpo.GRPO_WS_LOSS_LOGITS)    # a full workspace on the same context
 
 
 def test_fwd_bwd_is_deterministic():
