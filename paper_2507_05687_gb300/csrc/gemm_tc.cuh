@@ -272,8 +272,10 @@ struct OutStage {
 // rows in the 64-byte swizzle, 128-byte rows in the 128-byte one: the 16-byte
 // chunk index is XORed with bits 7.. of the offset, which also puts the writes
 // of any 8 consecutive lanes on distinct bank groups), then lane 0 issues a
-// TMA store, or an element-wise add at L2 when `reduce`.
-template <int kWords>
+// TMA store, or an element-wise add at L2 when `reduce`.  kEvictFirst: the
+// stored lines are the first L2 evicts (an output that is not read again
+// while it could still be in L2 should not push out the operand tiles).
+template <int kWords, bool kEvictFirst = false>
 __device__ __forceinline__ void out_block(OutStage& o, const uint32_t* words, int x, int y, bool reduce) {
   constexpr int kRowBytes = kWords * 4;
   const uint32_t buf = o.smem + static_cast<uint32_t>(o.count & 1) * (32 * kRowBytes);
@@ -290,6 +292,7 @@ __device__ __forceinline__ void out_block(OutStage& o, const uint32_t* words, in
   __syncwarp();
   if (o.lane == 0) {
     if (reduce) tma_reduce_add_2d(o.map, buf, x, y);
+    else if (kEvictFirst) tma_store_2d_hint(o.map, buf, x, y, l2_policy(kHintEvictFirst));
     else tma_store_2d(o.map, buf, x, y);
     bulk_commit();
   }
@@ -377,12 +380,13 @@ __device__ __forceinline__ bool epi_tile(EpiRow& e, const GemmArgs& a, uint32_t 
     const int cb = col0 + c * 32;
     if (kEpi == kEpiLse || kEpi == kEpiLseZ) {
       // kEpiLseZ: the raw logits first (blocks wholly past M or N skipped, the
-      // tensor map clips the rest)
+      // tensor map clips the rest); they are read again only by the backward's
+      // dZ pass, long after they have left L2
       if (kEpi == kEpiLseZ && row0 < m_rows && cb < a.N) {
         uint32_t bits[32];
 #pragma unroll
         for (int j = 0; j < 32; ++j) bits[j] = __float_as_uint(v[j]);
-        out_block<32>(os, bits, cb, row0, false);
+        out_block<32, true>(os, bits, cb, row0, false);
       }
       if (cb + 32 > a.N) {
 #pragma unroll

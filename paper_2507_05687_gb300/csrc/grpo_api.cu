@@ -49,6 +49,17 @@ int64_t vocab_chunk(int64_t V) {
   return std::min<int64_t>(c, round_up(V, 256));
 }
 
+// Vocabulary tiles per forward work unit before any narrowing for small
+// batches: kLseTilesPerUnit, or GRPO_LSE_TILES (4, 8, 16 or 32; read where
+// the layout is made, so a workspace is sized and used with the same value).
+int lse_tiles_per_unit() {
+  if (const char* e = std::getenv("GRPO_LSE_TILES")) {
+    const int v = std::atoi(e);
+    if (v == 4 || v == 8 || v == 16 || v == 32) return v;
+  }
+  return kLseTilesPerUnit;
+}
+
 // Workspace layout (byte offsets); every region is 256-byte aligned, the
 // bf16 matrices 1024-byte aligned.  Regions indexed by token position hold
 // T_pad rows; regions indexed by compacted (unmasked) row hold `rows`, the
@@ -73,7 +84,7 @@ bool make_layout(int64_t T, int32_t Hd, int64_t V, int32_t which, Layout* L, int
   L->T_pad = round_up(std::max<int64_t>(T, 1), kRowAlign);
   const int64_t vtiles = (V + kTileN - 1) / kTileN;
   // partial (max, sum) entries per row: one per vocabulary split and column half
-  L->lse_tiles = kLseTilesPerUnit;
+  L->lse_tiles = lse_tiles_per_unit();
   const int64_t m_tiles = (std::max<int64_t>(T, 1) + 2 * kRowsCta - 1) / (2 * kRowsCta);
   while (L->lse_tiles > 4 && m_tiles * ((vtiles + L->lse_tiles - 1) / L->lse_tiles) < kNominalPairs)
     L->lse_tiles /= 2;
@@ -318,16 +329,21 @@ bool use_pairs() {
 // groups (each W tile read by that many CTAs at once) while the group's A
 // tiles (38 MB on GB300) stay in L2; measured DRAM reads per launch at
 // 19,572 tokens x 155,136: 62.7 GB with 8 M tiles, 34.8 GB with pairs / 2,
-// 26.7 GB with pairs / 4.  The backward GEMMs measured best at 8.
-// GRPO_GROUP_M="a,b,c,d" overrides the defaults.
+// 26.7 GB with pairs / 4.  The backward GEMMs measured best at 8.  The
+// forward that also stores the logits (which = 4) measured best at 8 M tiles
+// as well: 47.5 against 47.8 ms per step at 19,572 tokens, and 123 against
+// 133 ms for the forward of 160,089 tokens, whose logits (99 GB) stream
+// through L2 beside the operand tiles.
+// GRPO_GROUP_M="a,b,c,d[,e]" overrides the defaults.
 int group_m(int which, const DeviceInfo& di) {
   const int workers = use_pairs() && di.pairs > 0 ? di.pairs : di.sms;
   const int quarter = std::max(1, workers / 4);
-  int g[4] = {quarter, 8, 8, 8};
+  int g[5] = {quarter, 8, 8, 8, 8};
   if (const char* e = std::getenv("GRPO_GROUP_M")) {
-    int v[4];
-    if (std::sscanf(e, "%d,%d,%d,%d", &v[0], &v[1], &v[2], &v[3]) == 4)
-      for (int i = 0; i < 4; ++i) g[i] = v[i] > 0 ? v[i] : g[i];
+    int v[5];
+    const int n = std::sscanf(e, "%d,%d,%d,%d,%d", &v[0], &v[1], &v[2], &v[3], &v[4]);
+    if (n >= 4)
+      for (int i = 0; i < n; ++i) g[i] = v[i] > 0 ? v[i] : g[i];
   }
   return g[which];
 }
@@ -559,7 +575,7 @@ cudaError_t run_lse(const uint16_t* const* W, int n_heads, int32_t Hd, int64_t V
   a.K = Hd;
   a.n_per_unit = Ly.lse_tiles;
   a.n_heads = n_heads;
-  a.group_m = group_m(0, di);
+  a.group_m = group_m(Ly.ldz > 0 ? 4 : 0, di);
   // Fault-injection test hook (failure-detection tests): GRPO_TEST_DROP_KBLOCK=k
   // makes CTA 0 skip the copies of its k-th k-block (1-based) so its pipeline
   // wait runs out after 0.2 s and the call reports GRPO_ERR_TIMEOUT.
