@@ -6,6 +6,7 @@
 
 #include <stdint.h>
 
+#include "dz_rows.cuh"
 #include "ptx.cuh"
 
 namespace grpo {
@@ -459,54 +460,14 @@ __global__ void dh_rows_kernel(const int* __restrict__ rank_of, int64_t T, int H
   }
 }
 
-// dZ chunk from the logits the forward GEMM stored (kEpiLseZ): columns
-// c0 .. c0 + width of z [rows x ldz] (fp32) -> dz [rows x vc] (bf16), by the
-// same dz_value as the kEpiDz epilogue, so from the same logits the same bits.
-// What that epilogue's tiles write as 0 is written as 0 here too: rows from
-// N_valid up to the next 256-row tile edge and columns from width up to the
-// next 256-column edge (within vc), which the dH and dW GEMMs read against
-// zero operands.  One block per row at a time (the row's lse, g and target
-// read once), 8 consecutive columns per thread: two 16-byte streaming loads
-// of logits (read once) and one 16-byte store.
+// dZ chunk from the logits the forward GEMM stored (kEpiLseZ): dz_rows with
+// one block per row at a time.
 __global__ void dz_from_logits_kernel(const float* __restrict__ z, int64_t ldz, const float* __restrict__ lse,
                                       const float* __restrict__ gcoef, const int* __restrict__ yc,
                                       const int* __restrict__ n_valid, int64_t rows_cap, int64_t c0, int width,
                                       int vc, uint16_t* __restrict__ dz) {
-  const float kLog2e = 1.4426950408889634f;
-  const int nv = *n_valid;
-  const int64_t rows = min(rows_cap, (static_cast<int64_t>(nv) + 255) / 256 * 256);
-  const int cols = min(vc, (width + 255) / 256 * 256);  // a multiple of 8, as vc is
-  for (int64_t r = blockIdx.x; r < rows; r += gridDim.x) {
-    uint16_t* out = dz + r * vc;
-    if (r >= nv) {
-      for (int c = threadIdx.x * 8; c < cols; c += blockDim.x * 8)
-        *reinterpret_cast<uint4*>(out + c) = make_uint4(0u, 0u, 0u, 0u);
-      continue;
-    }
-    const float lse2 = lse[r] * kLog2e;
-    const float g = gcoef[r];
-    const int64_t ty = yc[r] - c0;  // the target's column within the chunk
-    const float* src = z + r * ldz + c0;
-    for (int c = threadIdx.x * 8; c < cols; c += blockDim.x * 8) {
-      float v[8];
-      if (c + 8 <= width) {
-        const float4 a = __ldcs(reinterpret_cast<const float4*>(src + c));
-        const float4 b = __ldcs(reinterpret_cast<const float4*>(src + c) + 1);
-        v[0] = a.x, v[1] = a.y, v[2] = a.z, v[3] = a.w, v[4] = b.x, v[5] = b.y, v[6] = b.z, v[7] = b.w;
-      } else {
-#pragma unroll
-        for (int j = 0; j < 8; ++j) v[j] = c + j < width ? src[c + j] : 0.f;
-      }
-      uint32_t w[4];
-#pragma unroll
-      for (int j = 0; j < 8; j += 2) {
-        const float d0 = c + j < width ? dz_value(v[j], lse2, g, c + j == ty) : 0.f;
-        const float d1 = c + j + 1 < width ? dz_value(v[j + 1], lse2, g, c + j + 1 == ty) : 0.f;
-        w[j / 2] = pack_bf16x2(d0, d1);
-      }
-      *reinterpret_cast<uint4*>(out + c) = make_uint4(w[0], w[1], w[2], w[3]);
-    }
-  }
+  dz_rows(z, ldz, lse, gcoef, yc, *n_valid, rows_cap, c0, width, vc, dz, blockIdx.x, gridDim.x, threadIdx.x,
+          blockDim.x);
 }
 
 }  // namespace grpo
