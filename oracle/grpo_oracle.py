@@ -28,6 +28,15 @@ What it computes, in the paper's notation (Section 3.3):
       dZ_{t,v} = g_t (1[v = y_t] - p_{t,v}),  dH = dZ W,  dW = dZ^T H.
   At the kink of min() (rho A == clip(rho) A) the unclipped branch is taken.
 
+* the rollout draw that produces o_{i,t} ~ pi_theta_old (the sampling step
+  before Eq. 1, Section 3.3): Gumbel-max over softmax(z_t / temperature) with
+  Philox4x32-10 noise, optionally restricted to the nucleus (top-p) of that
+  distribution (Holtzman et al., "The Curious Case of Neural Text
+  Degeneration", 2020): the smallest set of the most probable tokens whose
+  mass reaches top_p, every token tied with its least probable member
+  included.  Gumbel-max over a subset draws from the distribution
+  renormalised on that subset.
+
 Rows with mask 0 have logp = 0, weight 0, and zero dH rows.
 Every floating value is float64; bf16 inputs are widened exactly.
 """
@@ -369,3 +378,72 @@ def sample_tokens(H, W, mask, temperature: float, seed: int, offset: int, rows=N
         logp[rr] = zbest - (run_max + np.log(run_sum))
         gap[rr] = best - second
     return tokens, logp, gap
+
+
+def nucleus(y, top_p: float):
+    """Nucleus (top-p) set of softmax(y) for one row of tempered logits y: sort
+    the tokens by probability, take the shortest prefix whose cumulative mass
+    reaches top_p, and keep every token whose logit is at least that of the
+    prefix's last token (so tokens tied with it are kept too).  top_p >= 1
+    keeps the whole vocabulary.  Returns (bool mask, threshold logit, the
+    set's probability mass)."""
+    y = np.asarray(y, dtype=np.float64)
+    if top_p >= 1.0:
+        return np.ones(y.size, dtype=bool), -np.inf, 1.0
+    mx = y.max()
+    p = np.exp(y - (mx + np.log(np.exp(y - mx).sum())))
+    order = np.argsort(-y, kind="stable")
+    cum = np.cumsum(p[order])
+    k = min(int(np.searchsorted(cum, top_p, side="left")), y.size - 1)
+    thr = y[order[k]]
+    keep = y >= thr
+    return keep, thr, float(p[keep].sum())
+
+
+def sample_tokens_top_p(H, W, mask, temperature: float, top_p: float, seed: int, offset: int, rows=None,
+                        band_mass: float = 1e-5, band_logit: float = 1e-3):
+    """Gumbel-max sampling restricted to the nucleus: y_t = argmax over v in
+    nucleus(z_t / temperature, top_p) of (z_{t,v} / temperature + G[t, v]), the
+    lowest v on ties, with the noise of gumbel_noise.  Returns, for every row
+    (masked rows: -1, 0, inf, (inf, inf)): tokens, the log-prob of the sampled
+    token under the untruncated softmax(z / temperature), the gap between the
+    best and second-best perturbed score inside the nucleus, and the band of
+    logits [lo, hi] whose membership could change if the cumulative masses
+    moved by band_mass or the logits by band_logit (lower-precision
+    arithmetic near the nucleus boundary)."""
+    Hf = np.asarray(H)
+    Wf = as_f64(W)
+    T, V = Hf.shape[0], Wf.shape[0]
+    m = np.asarray(mask) != 0
+    idx = np.flatnonzero(m) if rows is None else np.asarray(rows, dtype=np.int64)
+    idx = idx[m[idx]]
+    tokens = np.full(T, -1, dtype=np.int64)
+    logp = np.zeros(T)
+    gap = np.full(T, np.inf)
+    band = np.full((T, 2), np.inf)
+    inv_t = 1.0 / temperature
+    for r0 in range(0, idx.size, 32):
+        rr = idx[r0:r0 + 32]
+        Z = (as_f64(Hf[rr]) @ Wf.T) * inv_t
+        G = gumbel_noise(seed, offset, rr, V)
+        for i, t in enumerate(rr):
+            y = Z[i]
+            keep, _, _ = nucleus(y, top_p)
+            S = np.where(keep, y + G[i], -np.inf)
+            j = int(np.argmax(S))
+            S[j] = -np.inf
+            gap[t] = (y[j] + G[i, j]) - S.max() if keep.sum() > 1 else np.inf
+            mx = y.max()
+            lse = mx + np.log(np.exp(y - mx).sum())
+            tokens[t] = j
+            logp[t] = y[j] - lse
+            if top_p >= 1.0:
+                band[t] = (-np.inf, -np.inf)
+            else:
+                order = np.argsort(-y, kind="stable")
+                cum = np.cumsum(np.exp(y[order] - lse))
+                k_lo = min(int(np.searchsorted(cum, top_p - band_mass, side="left")), V - 1)
+                k_hi = min(int(np.searchsorted(cum, top_p + band_mass, side="left")), V - 1)
+                band[t] = (y[order[k_hi]] - band_logit, y[order[k_lo]] + band_logit)
+    return tokens, logp, gap, band
+

@@ -421,6 +421,63 @@ def test_sampling_counter_layout():
     assert not np.array_equal(g, oracle.gumbel_noise(98, 5, [3, 4], 9))
 
 
+def _nucleus_by_threshold_search(y, top_p):
+    """The nucleus as the highest logit threshold whose upper set reaches
+    top_p, searched over the row's distinct logit values with explicit sums."""
+    p = [math.exp(v) for v in y]
+    total = math.fsum(p)
+    for thr in sorted(set(y), reverse=True):
+        if math.fsum(pv for pv, v in zip(p, y) if v >= thr) / total >= top_p:
+            return np.array([v >= thr for v in y])
+    return np.ones(len(y), dtype=bool)
+
+
+def test_nucleus_matches_threshold_search():
+    """Random rows with many ties (logits on a half-integer grid): the nucleus
+    equals the threshold search, keeps whole tie groups, and drops below top_p
+    without its lowest tie group."""
+    rng = np.random.default_rng(31)
+    for _ in range(400):
+        V = int(rng.integers(1, 13))
+        y = (rng.integers(-4, 5, V) / 2.0).tolist()
+        top_p = float(rng.choice([rng.uniform(0.01, 0.99), 0.5, 0.9, 1.0]))
+        keep, thr, mass = oracle.nucleus(np.array(y), top_p)
+        want = _nucleus_by_threshold_search(y, top_p)
+        np.testing.assert_array_equal(keep, want)
+        if top_p < 1.0:
+            p = scipy.special.softmax(np.array(y))
+            assert mass >= top_p - 1e-12
+            assert p[np.array(y) > thr].sum() < top_p
+
+
+def test_top_p_draws_follow_the_truncated_softmax():
+    """Many rows with the same logits: inside the nucleus the sampled tokens'
+    frequencies follow the softmax renormalised on it, outside they never
+    occur; top_p = 1 is the plain sampler, a tiny top_p the greedy one."""
+    from scipy.stats import chisquare
+    V, T = 6, 30000
+    W = np.array([[1.0, 0, 0], [0.5, 0, 0], [0, 1, 0], [0, 0, 1], [-1.0, 0, 0], [0.2, 0.2, 0.2]])
+    H = np.tile(np.array([[0.9, -0.4, 0.3]]), (T, 1))
+    z = W @ H[0]
+    ones = np.ones(T, np.uint8)
+    for tau, top_p in ((1.0, 0.6), (0.5, 0.8), (2.0, 0.5)):
+        p = scipy.special.softmax(z / tau)
+        keep = oracle.nucleus(z / tau, top_p)[0]
+        assert 1 < keep.sum() < V
+        tok, logp, _, _ = oracle.sample_tokens_top_p(H, W, ones, tau, top_p, seed=1234, offset=7)
+        counts = np.bincount(tok, minlength=V)
+        assert counts[~keep].sum() == 0
+        q = p[keep] / p[keep].sum()
+        assert chisquare(counts[keep], q * T).pvalue > 1e-4
+        np.testing.assert_allclose(logp, np.log(p)[tok], rtol=0, atol=1e-12)
+    t1, l1, _, _ = oracle.sample_tokens_top_p(H[:2000], W, ones[:2000], 0.7, 1.0, seed=9, offset=3)
+    t2, l2, _ = oracle.sample_tokens(H[:2000], W, ones[:2000], 0.7, seed=9, offset=3)
+    np.testing.assert_array_equal(t1, t2)
+    np.testing.assert_allclose(l1, l2, rtol=0, atol=1e-12)
+    tok, _, _, _ = oracle.sample_tokens_top_p(H[:50], W, ones[:50], 1.0, 1e-9, seed=5, offset=0)
+    assert np.all(tok == np.argmax(z))
+
+
 # ---------------------------------------------------------------------------
 # planted mistakes: each must trip one of the pins above
 # ---------------------------------------------------------------------------
@@ -493,3 +550,37 @@ def test_planted_gumbel_sign_is_caught(monkeypatch):
     monkeypatch.setattr(go, "gumbel_noise", lambda *a, **k: -real(*a, **k))
     with pytest.raises(AssertionError):
         test_gumbel_max_samples_follow_the_softmax()
+
+
+def test_planted_nucleus_that_splits_ties_is_caught(monkeypatch):
+    def bad(y, top_p):
+        # the shortest prefix in stable order, ties with its last token cut off
+        y = np.asarray(y, dtype=np.float64)
+        if top_p >= 1.0:
+            return np.ones(y.size, dtype=bool), -np.inf, 1.0
+        p = scipy.special.softmax(y)
+        order = np.argsort(-y, kind="stable")
+        k = min(int(np.searchsorted(np.cumsum(p[order]), top_p, side="left")), y.size - 1)
+        keep = np.zeros(y.size, dtype=bool)
+        keep[order[:k + 1]] = True
+        return keep, y[order[k]], float(p[keep].sum())
+    monkeypatch.setattr(oracle, "nucleus", bad)
+    with pytest.raises(AssertionError):
+        test_nucleus_matches_threshold_search()
+
+
+def test_planted_nucleus_one_token_too_many_is_caught(monkeypatch):
+    real = go.nucleus
+
+    def bad(y, top_p):
+        keep, thr, mass = real(y, top_p)
+        if top_p < 1.0 and not keep.all():
+            y = np.asarray(y, dtype=np.float64)
+            nxt = y[~keep].max()
+            keep = y >= nxt
+            thr = nxt
+        return keep, thr, mass
+    monkeypatch.setattr(oracle, "nucleus", bad)
+    with pytest.raises(AssertionError):
+        test_nucleus_matches_threshold_search()
+
