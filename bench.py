@@ -39,7 +39,7 @@ KERNEL_SOURCES = ["paper_2507_05687_gb300/csrc/gemm_tc.cuh", "paper_2507_05687_g
                   "paper_2507_05687_gb300/csrc/grpo_api.cu", "paper_2507_05687_gb300/csrc/small_kernels.cuh",
                   "paper_2507_05687_gb300/csrc/dz_rows.cuh"]
 KIND_NAMES = ["advantages", "compact", "lse_gemm", "logp_merge", "loss", "dz_gemm", "dh_gemm", "dw_gemm",
-              "dh_rows", "adamw", "sample_gemm", "transpose", "dz_logits"]
+              "dh_rows", "adamw", "sample_gemm", "transpose", "dz_logits", "top_p"]
 KERNELS_PER_SCOPE = {1: 4, 4: 2}  # compaction scope = 4 kernels, loss scope = 2 kernels; others 1
 
 
@@ -58,6 +58,9 @@ def parse():
                         "workspace) or recompute them in the backward with a second logits GEMM (GRPO_WS_LOSS)")
     p.add_argument("--sample", action="store_true",
                    help="time the rollout draw (grpo_sample_tokens) over the workload's rows instead")
+    p.add_argument("--top-p", type=float, default=1.0,
+                   help="with --sample and a value below 1: the nucleus draw (grpo_sample_tokens_top_p), the "
+                        "forward storing the logits and one selection pass per row")
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--cpu-sample-tokens", type=int, default=1024,
@@ -211,6 +214,15 @@ def roofline(trace, n_valid_total_per_rank, Hd, steps, peak_tf, peak_kind, workl
         traffic = bytes_per_launch * avg_cols / cols_ref
     common = {"kernel": KIND_NAMES[dom], "traffic": traffic, "launches_per_step": len(recs) // max(1, steps),
               "avg_launch_ms": round(sum(secs) / len(secs) * 1e3, 4), "time_share": shares}
+    if 13 in by and hbm_gbs:
+        # nucleus selection + draw: the stored logits are read once from HBM per row
+        # (the later passes over the row mostly hit L2): N_valid x V fp32 per launch
+        tr13 = by[13]
+        pb = 4.0 * n_valid_total_per_rank * (sum(c for c, _ in tr13) / len(tr13))
+        ps = sum(ms for _, ms in tr13) / len(tr13) / 1e3
+        common["top_p_hbm"] = {"achieved": round(pb / ps / 1e9, 1), "peak": hbm_gbs, "unit": "GB/s",
+                               "frac": round(pb / ps / 1e9 / hbm_gbs, 4), "bytes_per_launch": pb,
+                               "avg_launch_ms": round(ps * 1e3, 4)}
     if 12 in by and hbm_gbs:
         # dZ from the kept logits, HBM-bound: per launch it reads N_valid x cols
         # fp32 logits and writes N_valid x cols bf16 dZ (algorithmic bytes)
@@ -351,13 +363,18 @@ def main():
     from paper_2507_05687_gb300 import dp
 
     if sampling:
-        ws = grpo.workspace(w.T, w.Hd, w.V, grpo.GRPO_WS_SAMPLE, dev, max_valid=n_valid)
+        top_p = args.top_p < 1.0
+        ws = grpo.workspace(w.T, w.Hd, w.V, grpo.GRPO_WS_SAMPLE_TOP_P if top_p else grpo.GRPO_WS_SAMPLE, dev,
+                            max_valid=n_valid)
         tok_out = (torch.empty(w.T, dtype=torch.int32, device=dev), torch.empty(w.T, dtype=torch.float32, device=dev))
         draw = [0]
 
         def step():
             draw[0] += 1  # a new offset per step: a fresh draw
-            grpo.sample_tokens(H, W, m, 1.0, seed=w.seed, offset=draw[0], ws=ws, out=tok_out)
+            if top_p:
+                grpo.sample_tokens_top_p(H, W, m, 1.0, args.top_p, seed=w.seed, offset=draw[0], ws=ws, out=tok_out)
+            else:
+                grpo.sample_tokens(H, W, m, 1.0, seed=w.seed, offset=draw[0], ws=ws, out=tok_out)
     elif scoring:
         heads = [W, to_dev(wl.gen_weight(w, "old", inp["W"]), torch.bfloat16),
                  to_dev(wl.gen_weight(w, "ref", inp["W"]), torch.bfloat16)]
@@ -453,7 +470,8 @@ def main():
     value = tot_valid / (ms / 1e3)
 
     burst, sustained, hbm, peak_src = peaks()
-    rkey = w.name + ("+sample" if sampling else "") + ("" if args.adamw == "none" else "+adamw_" + args.adamw) + \
+    rkey = w.name + ("+sample" if sampling else "") + ("+top_p" if sampling and args.top_p < 1.0 else "") + \
+        ("" if args.adamw == "none" else "+adamw_" + args.adamw) + \
         ("+recompute" if args.logits == "recompute" and not (sampling or scoring) else "")
     rf = roofline(trace, n_valid, w.Hd, args.steps, sustained, f"bf16 sustained, {peak_src}", rkey, hbm)
     if sampling:
@@ -498,7 +516,8 @@ def main():
                        "old_ref_logp": inp["old_src"], "adamw": args.adamw,
                        "logits": None if sampling or scoring else
                        ("kept from the forward" if args.logits == "keep" else "recomputed in the backward"),
-                       "step": "sample" if sampling else ("score3" if scoring else "fwdbwd")},
+                       "step": "sample" if sampling else ("score3" if scoring else "fwdbwd"),
+                       "top_p": args.top_p if sampling else None},
             "step_gemm_tflops_executed": round(step_exec / (ms / 1e3) / 1e12, 1),
             "step_frac_executed": round(step_exec / (ms / 1e3) / 1e12 / burst, 4),
             "step_frac_6x": round(step_model / (ms / 1e3) / 1e12 / burst, 4),

@@ -63,7 +63,8 @@ enum {
   GRPO_WS_LOSS = 1,
   GRPO_WS_LOGPROBS_HEADS = 2,
   GRPO_WS_SAMPLE = 3,
-  GRPO_WS_LOSS_LOGITS = 4
+  GRPO_WS_LOSS_LOGITS = 4,
+  GRPO_WS_SAMPLE_TOP_P = 5
 };
 
 /* Most LM heads grpo_token_logprobs_heads sweeps in one call. */
@@ -138,6 +139,33 @@ grpo_status grpo_token_logprobs_heads(const uint16_t* H, const uint16_t* const* 
 grpo_status grpo_sample_tokens(const uint16_t* H, const uint16_t* W, const uint8_t* mask, int64_t T, int32_t Hd,
                                int64_t V, float temperature, uint64_t seed, uint64_t offset, int32_t* tokens_out,
                                float* logp_out, void* ws, size_t ws_bytes, void* stream);
+
+/*
+ * grpo_sample_tokens restricted to the nucleus (top-p truncation; the rollout
+ * draw before Eq. 1, Section 3.3; the paper names no sampling parameters, this
+ * is the common nucleus rule of Holtzman et al., 2020): with y = z_t /
+ * temperature and p = softmax(y), the nucleus is the shortest set of the most
+ * probable tokens whose mass reaches top_p together with every token tied with
+ * its least probable member, and
+ *   o_t = argmax over v in the nucleus of  y_v + G_{t,v}   (lowest v on a tie)
+ * with G exactly as grpo_sample_tokens defines it, which draws from p
+ * renormalised on the nucleus; top_p = 1 draws the same tokens as
+ * grpo_sample_tokens.  The forward GEMM stores the fp32 logits of the unmasked
+ * rows in the workspace (4 * V bytes per row) and one pass per row finds the
+ * threshold (mass in 2^-40 fixed point, so the result does not depend on the
+ * order of the sums) and the argmax.
+ *   top_p       in (0, 1]
+ *   logp_out    [T] fp32 device, log softmax(y) at the sampled token (the
+ *               untruncated distribution; subtract log of the nucleus mass for
+ *               the truncated one)
+ *   ws          at least grpo_workspace_bytes(T, Hd, V, GRPO_WS_SAMPLE_TOP_P)
+ *               bytes (or grpo_workspace_bytes_rows for fewer unmasked rows)
+ * Other arguments, outputs and limits as grpo_sample_tokens.
+ */
+grpo_status grpo_sample_tokens_top_p(const uint16_t* H, const uint16_t* W, const uint8_t* mask, int64_t T,
+                                     int32_t Hd, int64_t V, float temperature, float top_p, uint64_t seed,
+                                     uint64_t offset, int32_t* tokens_out, float* logp_out, void* ws, size_t ws_bytes,
+                                     void* stream);
 
 /*
  * The noise grpo_sample_tokens adds, written out for checking the generator
@@ -325,9 +353,10 @@ grpo_status grpo_token_logprobs_noalloc(const uint16_t* H, const uint16_t* W, co
 
 /*
  * Bytes of workspace the call `which` (GRPO_WS_LOGPROBS, GRPO_WS_LOSS,
- * GRPO_WS_LOGPROBS_HEADS, GRPO_WS_SAMPLE or GRPO_WS_LOSS_LOGITS) needs for T
- * tokens, hidden size Hd and vocabulary V.  Returns 0 for arguments the calls
- * would reject.  Sized for the worst case N_valid = T.
+ * GRPO_WS_LOGPROBS_HEADS, GRPO_WS_SAMPLE, GRPO_WS_LOSS_LOGITS or
+ * GRPO_WS_SAMPLE_TOP_P) needs for T tokens, hidden size Hd and vocabulary V.
+ * Returns 0 for arguments the calls would reject.  Sized for the worst case
+ * N_valid = T.
  */
 size_t grpo_workspace_bytes(int64_t T, int32_t Hd, int64_t V, int32_t which);
 
@@ -395,7 +424,8 @@ enum {
   GRPO_K_ADAMW = 9,       /* standalone AdamW step (grpo_adamw_step) */
   GRPO_K_SAMPLE_GEMM = 10, /* logits GEMM + log-sum-exp + Gumbel-max draw */
   GRPO_K_TRANSPOSE = 11,  /* K-major (transposed) copy of the gathered hidden states for dW */
-  GRPO_K_DZ_LOGITS = 12   /* kept logits -> dZ chunk (bf16), element-wise */
+  GRPO_K_DZ_LOGITS = 12,  /* kept logits -> dZ chunk (bf16), element-wise */
+  GRPO_K_TOP_P = 13       /* nucleus threshold + Gumbel-max over the kept logits (per row) */
 };
 
 /*

@@ -33,6 +33,7 @@ GRPO_WS_LOSS = 1
 GRPO_WS_LOGPROBS_HEADS = 2
 GRPO_WS_SAMPLE = 3
 GRPO_WS_LOSS_LOGITS = 4
+GRPO_WS_SAMPLE_TOP_P = 5
 GRPO_MAX_HEADS = 4
 
 # name -> (restype, argtypes); mirrors include/grpo.h
@@ -61,6 +62,8 @@ SIGNATURES = {
                                                ctypes.c_size_t, _P]),
     "grpo_sample_tokens": (ctypes.c_int, [_P, _P, _P, _I64, _I32, _I64, _F, ctypes.c_uint64, ctypes.c_uint64, _P, _P,
                                           _P, ctypes.c_size_t, _P]),
+    "grpo_sample_tokens_top_p": (ctypes.c_int, [_P, _P, _P, _I64, _I32, _I64, _F, _F, ctypes.c_uint64,
+                                                ctypes.c_uint64, _P, _P, _P, ctypes.c_size_t, _P]),
     "grpo_gumbel_noise": (ctypes.c_int, [ctypes.c_uint64, ctypes.c_uint64, _I64, _I64, _I64, _P, _P]),
     "grpo_adamw_step": (ctypes.c_int, [_P, _P, _P, _P, _P, _I64, _F, _F, _F, _F, _F, _I64, _P]),
     "grpo_token_logprobs_noalloc": (ctypes.c_int, [_P, _P, _P, _P, _I64, _I32, _I64, _P, _P]),
@@ -288,6 +291,33 @@ def sample_tokens(H: torch.Tensor, W: torch.Tensor, mask: torch.Tensor, temperat
     _check(load().grpo_sample_tokens(_ptr(H), _ptr(W), _ptr(mask), T, Hd, V, float(temperature),
                                      int(seed) & (2 ** 64 - 1), int(offset) & (2 ** 64 - 1), _ptr(tok), _ptr(logp),
                                      _ptr(ws), ws.numel(), _stream(dev)), "grpo_sample_tokens")
+    return _to_host(tok, logp) if host else (tok, logp)
+
+
+def sample_tokens_top_p(H: torch.Tensor, W: torch.Tensor, mask: torch.Tensor, temperature: float = 1.0,
+                        top_p: float = 1.0, seed: int = 0, offset: int = 0, ws: Optional[torch.Tensor] = None,
+                        out=None):
+    """grpo_sample_tokens_top_p: the draw of sample_tokens restricted to the
+    nucleus of softmax(H W^T / temperature) (the most probable tokens whose mass
+    reaches top_p); returns (tokens int32 [T] (-1 masked), logp fp32 [T] under
+    the untruncated distribution)."""
+    dev, host = _target_device(H, W)
+    H = _on_device(H, dev, torch.bfloat16, "H")
+    W = _on_device(W, dev, torch.bfloat16, "W")
+    mask = _on_device(mask.view(torch.uint8) if mask.dtype == torch.bool else mask, dev, torch.uint8, "mask")
+    T, Hd = H.shape
+    V = W.shape[0]
+    _shape(W, (V, Hd), "W")
+    _shape(mask, (T,), "mask")
+    ws = workspace(T, Hd, V, GRPO_WS_SAMPLE_TOP_P, dev) if ws is None else _workspace(ws, dev)
+    if out is None:
+        out = (torch.empty(T, dtype=torch.int32, device=dev), torch.empty(T, dtype=torch.float32, device=dev))
+    tok = _output(out[0], (T,), torch.int32, dev, "out[0]")
+    logp = _output(out[1], (T,), torch.float32, dev, "out[1]")
+    _check(load().grpo_sample_tokens_top_p(_ptr(H), _ptr(W), _ptr(mask), T, Hd, V, float(temperature),
+                                           float(top_p), int(seed) & (2 ** 64 - 1), int(offset) & (2 ** 64 - 1),
+                                           _ptr(tok), _ptr(logp), _ptr(ws), ws.numel(), _stream(dev)),
+           "grpo_sample_tokens_top_p")
     return _to_host(tok, logp) if host else (tok, logp)
 
 

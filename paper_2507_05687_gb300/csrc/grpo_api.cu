@@ -16,6 +16,7 @@
 #include "../../include/grpo.h"
 #include "gemm_tc.cuh"
 #include "small_kernels.cuh"
+#include "top_p.cuh"
 
 using namespace grpo;
 
@@ -77,7 +78,7 @@ bool make_layout(int64_t T, int32_t Hd, int64_t V, int32_t which, Layout* L, int
   if (T < 0 || T >= (int64_t(1) << 31) || Hd <= 0 || Hd % 64 != 0 || V <= 0 ||
       V >= (int64_t(1) << 31) ||
       (which != GRPO_WS_LOGPROBS && which != GRPO_WS_LOSS && which != GRPO_WS_LOGPROBS_HEADS &&
-       which != GRPO_WS_SAMPLE && which != GRPO_WS_LOSS_LOGITS))
+       which != GRPO_WS_SAMPLE && which != GRPO_WS_LOSS_LOGITS && which != GRPO_WS_SAMPLE_TOP_P))
     return false;
   const bool loss = which == GRPO_WS_LOSS || which == GRPO_WS_LOSS_LOGITS;
   const size_t heads = which == GRPO_WS_LOGPROBS_HEADS ? kMaxHeads : 1;
@@ -94,7 +95,7 @@ bool make_layout(int64_t T, int32_t Hd, int64_t V, int32_t which, Layout* L, int
   L->nblk_scan = (std::max<int64_t>(T, 1) + kScanChunk - 1) / kScanChunk;
   L->nblk_loss = (L->rows + kLossThreads - 1) / kLossThreads;
   L->vchunk = loss ? vocab_chunk(V) : 0;
-  L->ldz = which == GRPO_WS_LOSS_LOGITS ? round_up(V, 64) : 0;
+  L->ldz = which == GRPO_WS_LOSS_LOGITS || which == GRPO_WS_SAMPLE_TOP_P ? round_up(V, 64) : 0;
   size_t off = 0;
   auto take = [&](size_t bytes, size_t align) {
     off = (off + align - 1) / align * align;
@@ -797,6 +798,42 @@ grpo_status grpo_sample_tokens(const uint16_t* H, const uint16_t* W, const uint8
                                                at<int>(ws, Ly.best_c), at<float>(ws, Ly.best_z),
                                                static_cast<int>(Ly.nsplit), Ly.rows, tokens_out, logp_out,
                                                at<unsigned>(ws, Ly.status));
+    e = cudaGetLastError();
+  }
+  return from_cuda(e);
+}
+
+grpo_status grpo_sample_tokens_top_p(const uint16_t* H, const uint16_t* W, const uint8_t* mask, int64_t T,
+                                     int32_t Hd, int64_t V, float temperature, float top_p, uint64_t seed,
+                                     uint64_t offset, int32_t* tokens_out, float* logp_out, void* ws, size_t ws_bytes,
+                                     void* stream) {
+  Layout Ly;
+  if (!make_layout(T, Hd, V, GRPO_WS_SAMPLE_TOP_P, &Ly)) return GRPO_ERR_INVALID_ARG;
+  if (!W || !aligned(W, 16)) return GRPO_ERR_INVALID_ARG;
+  if (T > 0 && (!H || !mask || !tokens_out || !logp_out)) return GRPO_ERR_INVALID_ARG;
+  if (H && !aligned(H, 16)) return GRPO_ERR_INVALID_ARG;
+  if (!(temperature > 0.f) || !(temperature < INFINITY) || !(top_p > 0.f) || !(top_p <= 1.f))
+    return GRPO_ERR_INVALID_ARG;
+  if (!ws || !aligned(ws, 256) || !fit_layout(T, Hd, V, GRPO_WS_SAMPLE_TOP_P, ws_bytes, &Ly))
+    return GRPO_ERR_WORKSPACE;
+  if (T == 0) return GRPO_OK;
+  DeviceInfo di;
+  if (!device_info(&di)) return GRPO_ERR_UNSUPPORTED;
+  if (!get_encode()) return GRPO_ERR_CUDA;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  // the logits of every unmasked row, stored by the forward GEMM
+  cudaError_t e = run_compaction(H, nullptr, mask, T, Hd, V, ws, Ly, di.sms, s);
+  if (e == cudaSuccess) e = run_lse(&W, 1, Hd, V, ws, Ly, di, s);
+  if (e == cudaSuccess) {
+    TraceScope trace(GRPO_K_TOP_P, V, s);
+    const int fb = static_cast<int>(std::min<int64_t>((T + 255) / 256, int64_t(di.sms) * 16));
+    top_p_fill_kernel<<<fb, 256, 0, s>>>(mask, at<int>(ws, Ly.rank_of), T, tokens_out, logp_out);
+    const int rb = static_cast<int>(std::min<int64_t>(Ly.rows, int64_t(di.sms) * 4));
+    top_p_kernel<<<rb, kTopPThreads, 0, s>>>(
+        at<float>(ws, Ly.z), Ly.ldz, static_cast<int>(V), at<int>(ws, Ly.n_valid), at<int>(ws, Ly.cidx),
+        1.f / temperature, top_p, static_cast<uint32_t>(seed), static_cast<uint32_t>(seed >> 32),
+        static_cast<uint32_t>(offset), static_cast<uint32_t>(offset >> 32), tokens_out, logp_out,
+        at<unsigned>(ws, Ly.status));
     e = cudaGetLastError();
   }
   return from_cuda(e);

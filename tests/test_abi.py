@@ -65,7 +65,7 @@ FAKE = 0x10000  # never dereferenced: every call below is rejected on the host
 
 def test_workspace_sized_for_fewer_rows(lib):
     f, g = grpo.workspace_bytes, grpo.workspace_bytes_rows
-    for which in (0, 1, 2, 3, 4):
+    for which in (0, 1, 2, 3, 4, 5):
         full = f(32768, 4096, 155136, which)
         assert g(32768, 32768, 4096, 155136, which) == full == g(32768, 10**9, 4096, 155136, which)
         sizes = [g(32768, n, 4096, 155136, which) for n in (1, 256, 257, 5000, 20000)]
@@ -145,6 +145,16 @@ def test_host_rejections(lib):
     assert L.grpo_gumbel_noise(1, 2, 0, 4, 4, None, None) == grpo.GRPO_ERR_INVALID_ARG
     assert L.grpo_gumbel_noise(1, 2, 0, 4, 4, FAKE + 2, None) == grpo.GRPO_ERR_INVALID_ARG
     assert L.grpo_gumbel_noise(1, 2, 2**32, 0, 4, None, None) == grpo.GRPO_OK
+    wst = grpo.workspace_bytes(100, 64, 1000, grpo.GRPO_WS_SAMPLE_TOP_P)
+    assert wst > grpo.workspace_bytes(100, 64, 1000, grpo.GRPO_WS_LOGPROBS) + 4 * 256 * 1024 - 1
+    targs = [FAKE, FAKE, FAKE, 100, 64, 1000, 1.0, 0.9, 1, 2, FAKE, FAKE, FAKE, wst, None]
+    for i, v in ((7, 0.0), (7, -0.5), (7, 1.01), (7, float("nan")), (6, 0.0), (6, float("inf")), (4, 60)):
+        bad = list(targs); bad[i] = v
+        assert L.grpo_sample_tokens_top_p(*bad) == grpo.GRPO_ERR_INVALID_ARG, (i, v)
+    bad = list(targs); bad[13] = wst - 1024 * 257   # fewer than 256 rows of logits fit
+    assert L.grpo_sample_tokens_top_p(*bad) == grpo.GRPO_ERR_WORKSPACE
+    bad = list(targs); bad[3] = 0                 # no rows: nothing to do
+    assert L.grpo_sample_tokens_top_p(*bad) == grpo.GRPO_OK
     eargs = largs[:14] + [0.0] + largs[14:17] + [None, 0] + largs[17:]
     assert L.grpo_loss_fwd_bwd_events(*eargs) == grpo.GRPO_ERR_INVALID_ARG          # no event array
     few = (ctypes.c_void_p * 1)(FAKE)
