@@ -36,6 +36,8 @@
 //            running log-sum-exp of z / temperature and the running argmax of
 //            z / temperature + Gumbel noise (Philox4x32-10, counter = (v / 4, t,
 //            offset), key = seed); the logits never leave the SM.
+//   kEpiSampleZ the same, and the fp32 logits z themselves are stored (as
+//            kEpiLseZ does), for the nucleus (top-p) selection that follows.
 //   kEpiAdam dW = dZ^T H consumed in place by an AdamW step on the matching
 //            LM-head rows (fp32 master, both moments, bf16 weights out), so
 //            dW itself is never stored; the weights and moments move through
@@ -71,7 +73,7 @@ struct TileCfg {
   static constexpr int kStageBytes = kABytes + kBBytes;
 };
 
-enum { kEpiLse = 0, kEpiDz = 1, kEpiF32 = 2, kEpiAdam = 3, kEpiSample = 4, kEpiLseZ = 5 };
+enum { kEpiLse = 0, kEpiDz = 1, kEpiF32 = 2, kEpiAdam = 3, kEpiSample = 4, kEpiLseZ = 5, kEpiSampleZ = 6 };
 
 // Epilogue warps per CTA: 4 = one per TMEM lane quarter (each thread walks its
 // row's 256 columns); 8 = two per quarter, each taking half the columns.  The
@@ -80,19 +82,20 @@ enum { kEpiLse = 0, kEpiDz = 1, kEpiF32 = 2, kEpiAdam = 3, kEpiSample = 4, kEpiL
 // of the same batch went from 15.7 to 16.7 ms per step.
 template <int kEpi>
 struct EpiShape {
-  static constexpr int kWarps = kEpi == kEpiSample ? 8 : 4;
+  static constexpr int kWarps = kEpi == kEpiSample || kEpi == kEpiSampleZ ? 8 : 4;
   static constexpr int kHalves = kWarps / 4;    // column halves of a tile, one per warp of a quarter
   static constexpr int kThreads = 64 + 32 * kWarps;
-  static constexpr bool kTmaOut = kEpi == kEpiDz || kEpi == kEpiF32 || kEpi == kEpiAdam || kEpi == kEpiLseZ;
+  static constexpr bool kTmaOut =
+      kEpi == kEpiDz || kEpi == kEpiF32 || kEpi == kEpiAdam || kEpi == kEpiLseZ || kEpi == kEpiSampleZ;
   // element type of the output tensor map: fp32 (128-byte rows of 32, 128-byte
   // swizzle) or bf16 (kEpiDz: 64-byte rows, 64-byte swizzle)
-  static constexpr bool kOutF32 = kEpi == kEpiF32 || kEpi == kEpiLseZ || kEpi == kEpiAdam;
+  static constexpr bool kOutF32 = kEpi == kEpiF32 || kEpi == kEpiLseZ || kEpi == kEpiAdam || kEpi == kEpiSampleZ;
   // one warp's 32 x 32 block in shared memory: bf16 dZ / fp32 output or
   // logits, two per warp; kEpiAdam: fp32 weights, first and second moments (4 KB each) and the
   // bf16 weights (2 KB), one per warp (the dW K-loop is long enough to hide it)
   static constexpr int kBlockBytes =
       kEpi == kEpiDz                        ? 32 * 32 * 2
-      : kEpi == kEpiF32 || kEpi == kEpiLseZ ? 32 * 32 * 4
+      : kEpi == kEpiF32 || kEpi == kEpiLseZ || kEpi == kEpiSampleZ ? 32 * 32 * 4
       : kEpi == kEpiAdam                    ? 3 * 4096 + 2048
                                             : 0;
   static constexpr int kBlocks = kEpi == kEpiAdam ? 1 : 2;
@@ -100,10 +103,11 @@ struct EpiShape {
 };
 
 // Operand-ring depth: 6 stages of 32 KB (pair) / 4 of 48 KB (single), one
-// fewer for kEpiAdam (6 / 3), whose staging blocks take the room.
+// fewer for kEpiAdam and kEpiSampleZ (5 / 3), whose staging blocks take the
+// room (kEpiSampleZ: 8 warps x 2 blocks of 4 KB).
 template <int kPair, int kEpi>
 __host__ __device__ constexpr int ring_stages() {
-  return kEpi == kEpiAdam ? (kPair == 2 ? 5 : 3) : (kPair == 2 ? 6 : 4);
+  return kEpi == kEpiAdam || kEpi == kEpiSampleZ ? (kPair == 2 ? 5 : 3) : (kPair == 2 ? 6 : 4);
 }
 
 // Dynamic shared memory of one CTA: the operand ring, the output staging
@@ -227,7 +231,7 @@ __device__ __forceinline__ void epi_begin(EpiRow& e, const GemmArgs& a, int r, i
   e.best_s = -INFINITY;
   e.best_z = -INFINITY;
   e.best_c = -1;
-  if (kEpi == kEpiSample) {
+  if (kEpi == kEpiSample || kEpi == kEpiSampleZ) {
     if (e.rv) e.orow = a.row_map[r];
   } else if (kEpi == kEpiLse || kEpi == kEpiLseZ) {
     e.y = e.rv ? a.yc[r] : -1;
@@ -412,7 +416,15 @@ __device__ __forceinline__ bool epi_tile(EpiRow& e, const GemmArgs& a, uint32_t 
         e.run_s = e.run_s * fast_exp2(e.run_m - nm) + acc;
         e.run_m = nm;
       }
-    } else if (kEpi == kEpiSample) {
+    } else if (kEpi == kEpiSample || kEpi == kEpiSampleZ) {
+      // kEpiSampleZ: the raw logits first (as kEpiLseZ, evict-first), read
+      // again by the nucleus selection after this GEMM
+      if (kEpi == kEpiSampleZ && row0 < m_rows && cb < a.N) {
+        uint32_t bits[32];
+#pragma unroll
+        for (int j = 0; j < 32; ++j) bits[j] = __float_as_uint(v[j]);
+        out_block<32, true>(os, bits, cb, row0, false);
+      }
       // scaled logits (cols >= N: -inf) -> running LSE and running argmax of z + noise
 #pragma unroll
       for (int j = 0; j < 32; ++j) v[j] = (cb + j < a.N) ? v[j] * a.inv_temp : -INFINITY;
@@ -478,7 +490,7 @@ __device__ __forceinline__ bool epi_tile(EpiRow& e, const GemmArgs& a, uint32_t 
 template <int kEpi>
 __device__ __forceinline__ void epi_end(const EpiRow& e, const GemmArgs& a, int un, int head, int half) {
   const long entry = static_cast<long>(un) * EpiShape<kEpi>::kHalves + half;  // split entry of this column half
-  if (kEpi == kEpiSample && e.rv) {
+  if ((kEpi == kEpiSample || kEpi == kEpiSampleZ) && e.rv) {
     const long at = entry * a.ldp + e.r;
     a.part_m[at] = e.run_m;
     a.part_s[at] = e.run_s;

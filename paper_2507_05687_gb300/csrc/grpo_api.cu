@@ -71,7 +71,7 @@ struct Layout {
   int64_t ldz;    // leading dimension (fp32 elements) of the stored logits; 0: not stored
   int lse_tiles;  // vocabulary tiles (of 256) per forward work unit
   size_t status, n_valid, counts, offsets, cidx, rank_of, yc, zy, part_m, part_s, lse_c, g_c,
-      block_loss, resp_len, best_s, best_c, best_z, Hc, HcT, dz, dhc, z, total;
+      block_loss, resp_len, best_s, best_c, best_z, Hc, HcT, dz, dhc, z, slow_rows, slow_tgt, n_slow, total;
 };
 
 bool make_layout(int64_t T, int32_t Hd, int64_t V, int32_t which, Layout* L, int64_t rows_cap = -1) {
@@ -90,7 +90,8 @@ bool make_layout(int64_t T, int32_t Hd, int64_t V, int32_t which, Layout* L, int
   while (L->lse_tiles > 4 && m_tiles * ((vtiles + L->lse_tiles - 1) / L->lse_tiles) < kNominalPairs)
     L->lse_tiles /= 2;
   L->nsplit = (vtiles + L->lse_tiles - 1) / L->lse_tiles *
-              (which == GRPO_WS_SAMPLE ? EpiShape<kEpiSample>::kHalves : EpiShape<kEpiLse>::kHalves);
+              (which == GRPO_WS_SAMPLE || which == GRPO_WS_SAMPLE_TOP_P ? EpiShape<kEpiSample>::kHalves
+                                                                         : EpiShape<kEpiLse>::kHalves);
   L->rows = rows_cap < 0 ? L->T_pad : std::min(L->T_pad, round_up(std::max<int64_t>(rows_cap, 1), kRowAlign));
   L->nblk_scan = (std::max<int64_t>(T, 1) + kScanChunk - 1) / kScanChunk;
   L->nblk_loss = (L->rows + kLossThreads - 1) / kLossThreads;
@@ -119,7 +120,7 @@ bool make_layout(int64_t T, int32_t Hd, int64_t V, int32_t which, Layout* L, int
   L->g_c = take(4 * cr, 256);
   L->block_loss = take(8 * L->nblk_loss, 256);
   L->resp_len = take(4 * tp, 256);
-  const size_t best = which == GRPO_WS_SAMPLE ? 4 * cr * L->nsplit : 0;
+  const size_t best = which == GRPO_WS_SAMPLE || which == GRPO_WS_SAMPLE_TOP_P ? 4 * cr * L->nsplit : 0;
   L->best_s = take(best, 256);
   L->best_c = take(best, 256);
   L->best_z = take(best, 256);
@@ -133,6 +134,11 @@ bool make_layout(int64_t T, int32_t Hd, int64_t V, int32_t which, Layout* L, int
   // the fp32 logits [rows x ldz] of the forward, kept for the backward (last,
   // so that every other region sits where the plain loss layout has it)
   L->z = take(4 * cr * static_cast<size_t>(L->ldz), 1024);
+  // the nucleus draw: the rows whose plain winner falls outside, their targets, their count
+  const bool top_p = which == GRPO_WS_SAMPLE_TOP_P;
+  L->slow_rows = take(top_p ? 4 * cr : 0, 256);
+  L->slow_tgt = take(top_p ? 8 * cr : 0, 256);
+  L->n_slow = take(top_p ? 4 : 0, 256);
   L->total = (off + 1023) / 1024 * 1024;
   return true;
 }
@@ -227,9 +233,16 @@ bool encode_blk(CUtensorMap* map, const void* base, uint64_t rows, uint64_t k, u
 
 struct DeviceInfo {
   int sms = 0;
-  int pairs = 0;  // CTA pairs of the pair kernels that can be resident at once
+  int pairs = 0;        // CTA pairs of the pair kernels that can be resident at once
+  int top_p_clusters = 0;  // clusters of the nucleus selection kernel resident at once
   bool ok = false;
 };
+
+// Every variant's dynamic shared memory fits the 227 KB a CTA may opt into.
+static_assert(smem_bytes<2, kEpiSampleZ>() <= 232448 && smem_bytes<1, kEpiSampleZ>() <= 232448 &&
+                  smem_bytes<2, kEpiAdam>() <= 232448 && smem_bytes<2, kEpiF32>() <= 232448 &&
+                  smem_bytes<1, kEpiF32>() <= 232448,
+              "shared memory budget");
 
 template <int E, bool A, bool B, bool BLK = false>
 bool prepare_kernels(int* pairs) {
@@ -269,10 +282,23 @@ bool device_info(DeviceInfo* out) {
         !prepare_kernels<kEpiDz, false, false>(&pairs) ||
         !prepare_kernels<kEpiF32, false, true>(&pairs) || !prepare_kernels<kEpiF32, true, false>(&pairs) ||
         !prepare_kernels<kEpiF32, true, false, true>(&pairs) || !prepare_kernels<kEpiAdam, true, false, true>(&pairs) ||
-        !prepare_kernels<kEpiAdam, true, false>(&pairs) || !prepare_kernels<kEpiSample, false, false>(&pairs))
+        !prepare_kernels<kEpiAdam, true, false>(&pairs) || !prepare_kernels<kEpiSample, false, false>(&pairs) ||
+        !prepare_kernels<kEpiSampleZ, false, false>(&pairs))
       return false;
+    // the nucleus selection walks its rows in a loop over a fixed set of
+    // clusters: launch no more than can be resident together (a cluster must
+    // fit in one GPC, so this is below SMs x CTAs per SM / cluster size)
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(kTopPCtas * 1024, 1, 1);
+    cfg.blockDim = dim3(kTopPThreads, 1, 1);
+    int tpc = 0;
+    if (cudaOccupancyMaxActiveClusters(&tpc, top_p_kernel, &cfg) != cudaSuccess) {
+      cudaGetLastError();
+      tpc = 0;
+    }
     cache[dev].sms = sms;
     cache[dev].pairs = std::max(pairs, 0);
+    cache[dev].top_p_clusters = std::max(tpc, 1);
     cache[dev].ok = true;
   }
   *out = cache[dev];
@@ -821,20 +847,81 @@ grpo_status grpo_sample_tokens_top_p(const uint16_t* H, const uint16_t* W, const
   if (!device_info(&di)) return GRPO_ERR_UNSUPPORTED;
   if (!get_encode()) return GRPO_ERR_CUDA;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
-  // the logits of every unmasked row, stored by the forward GEMM
+  // the sampling GEMM (running LSE and the plain Gumbel-max winner per split),
+  // storing the logits of every unmasked row for the nucleus selection
   cudaError_t e = run_compaction(H, nullptr, mask, T, Hd, V, ws, Ly, di.sms, s);
-  if (e == cudaSuccess) e = run_lse(&W, 1, Hd, V, ws, Ly, di, s);
+  if (e == cudaSuccess) {
+    GemmArgs a{};
+    a.n_valid = at<int>(ws, Ly.n_valid);
+    a.m_dyn = 1;
+    a.N = static_cast<int>(V);
+    a.K = Hd;
+    a.n_per_unit = Ly.lse_tiles;
+    a.n_heads = 1;
+    a.group_m = group_m(4, di);
+    l2_hints(0, &a.a_hint, &a.b_hint);
+    a.status = at<unsigned>(ws, Ly.status);
+    a.row_map = at<int>(ws, Ly.cidx);
+    a.part_m = at<float>(ws, Ly.part_m);
+    a.part_s = at<float>(ws, Ly.part_s);
+    a.best_s = at<float>(ws, Ly.best_s);
+    a.best_c = at<int>(ws, Ly.best_c);
+    a.best_z = at<float>(ws, Ly.best_z);
+    a.ldp = Ly.rows;
+    a.inv_temp = 1.f / temperature;
+    a.seed_lo = static_cast<uint32_t>(seed);
+    a.seed_hi = static_cast<uint32_t>(seed >> 32);
+    a.off_lo = static_cast<uint32_t>(offset);
+    a.off_hi = static_cast<uint32_t>(offset >> 32);
+    const Operand A{at<uint16_t>(ws, Ly.Hc), static_cast<uint64_t>(Ly.rows), static_cast<uint64_t>(Hd),
+                    static_cast<uint64_t>(Hd)};
+    const Operand B{W, static_cast<uint64_t>(V), static_cast<uint64_t>(Hd), static_cast<uint64_t>(Hd)};
+    const OutMat Z{at<float>(ws, Ly.z), static_cast<uint64_t>(Ly.rows), static_cast<uint64_t>(V),
+                   static_cast<uint64_t>(Ly.ldz)};
+    TraceScope trace(GRPO_K_SAMPLE_GEMM, V, s);
+    e = launch_gemm<kEpiSampleZ, false, false>(A, B, a, Ly.rows, di, s, &Z);
+  }
   if (e == cudaSuccess) {
     TraceScope trace(GRPO_K_TOP_P, V, s);
     const int fb = static_cast<int>(std::min<int64_t>((T + 255) / 256, int64_t(di.sms) * 16));
     top_p_fill_kernel<<<fb, 256, 0, s>>>(mask, at<int>(ws, Ly.rank_of), T, tokens_out, logp_out);
-    const int rb = static_cast<int>(std::min<int64_t>(Ly.rows, int64_t(di.sms) * 4));
-    top_p_kernel<<<rb, kTopPThreads, 0, s>>>(
-        at<float>(ws, Ly.z), Ly.ldz, static_cast<int>(V), at<int>(ws, Ly.n_valid), at<int>(ws, Ly.cidx),
-        1.f / temperature, top_p, static_cast<uint32_t>(seed), static_cast<uint32_t>(seed >> 32),
-        static_cast<uint32_t>(offset), static_cast<uint32_t>(offset >> 32), tokens_out, logp_out,
-        at<unsigned>(ws, Ly.status));
+    // the plain draw of every unmasked row, and per row what the selection needs
+    // (workspace arrays the sampling path leaves unused: LSE, the winner's y,
+    // the row maximum)
+    float* lse_r = at<float>(ws, Ly.lse_c);
+    float* y0_r = at<float>(ws, Ly.g_c);
+    float* hi_r = at<float>(ws, Ly.zy);
+    const int pb = static_cast<int>(std::min<int64_t>((Ly.rows + 7) / 8, int64_t(di.sms) * 8));
+    top_p_prep_kernel<<<pb, 256, 0, s>>>(at<int>(ws, Ly.n_valid), at<int>(ws, Ly.cidx), at<float>(ws, Ly.part_m),
+                                         at<float>(ws, Ly.part_s), at<float>(ws, Ly.best_s),
+                                         at<int>(ws, Ly.best_c), at<float>(ws, Ly.best_z),
+                                         static_cast<int>(Ly.nsplit), Ly.rows, lse_r, y0_r, hi_r, tokens_out,
+                                         logp_out, at<unsigned>(ws, Ly.status));
     e = cudaGetLastError();
+    if (e == cudaSuccess && top_p < 1.f) {
+      unsigned* n_slow = at<unsigned>(ws, Ly.n_slow);
+      e = cudaMemsetAsync(n_slow, 0, 4, s);
+      // is the winner in the nucleus?  one CTA per row, rows in turn; four CTAs
+      // per SM (58 registers x 256 threads), all resident
+      const int fb2 = static_cast<int>(std::min<int64_t>(Ly.rows, int64_t(di.sms) * 4));
+      if (e == cudaSuccess)
+        top_p_fast_kernel<<<fb2, kTopPThreads, 0, s>>>(at<float>(ws, Ly.z), Ly.ldz, static_cast<int>(V),
+                                                       at<int>(ws, Ly.n_valid), lse_r, y0_r, 1.f / temperature,
+                                                       top_p, at<int>(ws, Ly.slow_rows),
+                                                       at<unsigned long long>(ws, Ly.slow_tgt), n_slow);
+      // the rows whose winner falls outside: clusters of kTopPCtas CTAs, one row
+      // per cluster at a time, as many clusters as can be resident together
+      const int64_t clusters = std::max<int64_t>(1, std::min<int64_t>(Ly.rows, di.top_p_clusters));
+      const int rb = static_cast<int>(clusters * kTopPCtas);
+      if (e == cudaSuccess)
+        top_p_kernel<<<rb, kTopPThreads, 0, s>>>(
+            at<float>(ws, Ly.z), Ly.ldz, static_cast<int>(V), reinterpret_cast<const int*>(n_slow),
+            at<int>(ws, Ly.slow_rows), at<unsigned long long>(ws, Ly.slow_tgt), at<int>(ws, Ly.cidx), lse_r, y0_r,
+            hi_r, 1.f / temperature, static_cast<uint32_t>(seed), static_cast<uint32_t>(seed >> 32),
+            static_cast<uint32_t>(offset), static_cast<uint32_t>(offset >> 32), tokens_out, logp_out,
+            at<unsigned>(ws, Ly.status));
+      if (e == cudaSuccess) e = cudaGetLastError();
+    }
   }
   return from_cuda(e);
 }

@@ -208,8 +208,8 @@ __device__ __forceinline__ float merge_lse(const float* __restrict__ pm, const f
                                            int nsplit, long ldp, int r) {
   float m = -INFINITY;
   for (int j = 0; j < nsplit; ++j) m = fmaxf(m, pm[j * ldp + r]);
-  float s = 0.f;
-  for (int j = 0; j < nsplit; ++j) s += ps[j * ldp + r] * fast_exp2(pm[j * ldp + r] - m);
+  float s = 0.f;  // explicitly rounded, so that other merges of the same splits can match it bit for bit
+  for (int j = 0; j < nsplit; ++j) s = __fadd_rn(s, __fmul_rn(ps[j * ldp + r], fast_exp2(pm[j * ldp + r] - m)));
   return (m + __log2f(s)) * 0.6931471805599453f;
 }
 
