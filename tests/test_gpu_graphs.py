@@ -62,21 +62,32 @@ def test_loss_step_replays_from_a_graph(kind, monkeypatch):
             assert torch.equal(a, b)
 
 
-def test_decode_step_draw_replays_from_a_graph():
+@pytest.mark.parametrize("top_p", [None, 0.9])
+def test_decode_step_draw_replays_from_a_graph(top_p):
+    """A decode-step draw, plain or nucleus (its list of rows whose winner falls
+    outside is rebuilt on the device every replay), captured and replayed."""
     w = wl.DECODE_WORKLOADS["decode256_8b"].with_(V=32768)
     Hb, Wb, m = wl.gen_hidden(w), wl.gen_weight(w), wl.gen_mask(w)
     H, W, md = dev_tensor(Hb, torch.bfloat16), dev_tensor(Wb, torch.bfloat16), dev_tensor(m, torch.uint8)
-    ws = grpo.workspace(w.T, w.Hd, w.V, grpo.GRPO_WS_SAMPLE, DEV)
+    ws = grpo.workspace(w.T, w.Hd, w.V, grpo.GRPO_WS_SAMPLE if top_p is None else grpo.GRPO_WS_SAMPLE_TOP_P, DEV)
     out = (torch.empty(w.T, dtype=torch.int32, device=DEV), torch.empty(w.T, device=DEV))
-    eager = grpo.sample_tokens(H, W, md, 1.0, seed=11, offset=3, ws=ws, out=out)
-    eager = [t.clone() for t in eager]
+
+    def draw():
+        if top_p is None:
+            return grpo.sample_tokens(H, W, md, 1.0, seed=11, offset=3, ws=ws, out=out)
+        return grpo.sample_tokens_top_p(H, W, md, 1.0, top_p, seed=11, offset=3, ws=ws, out=out)
+
+    eager = [t.clone() for t in draw()]
     g = torch.cuda.CUDAGraph()
     with torch.cuda.graph(g):
-        grpo.sample_tokens(H, W, md, 1.0, seed=11, offset=3, ws=ws, out=out)
-    out[0].fill_(-7)
-    g.replay()
-    torch.cuda.synchronize()
-    assert torch.equal(out[0], eager[0]) and torch.equal(out[1], eager[1])
+        draw()
+    for _ in range(2):
+        out[0].fill_(-7)
+        out[1].fill_(float("nan"))
+        g.replay()
+        torch.cuda.synchronize()
+        assert grpo.check_device_status(ws) == grpo.GRPO_OK
+        assert torch.equal(out[0], eager[0]) and torch.equal(out[1], eager[1])
 
 
 def test_calls_on_two_streams_with_their_own_workspaces():
