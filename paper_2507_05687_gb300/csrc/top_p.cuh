@@ -153,21 +153,30 @@ template <int kUnroll, int kShare = kTopPCtas, typename F>
 __device__ __forceinline__ void top_p_walk(const float* zr, int V, float inv_temp, int rank, F f) {
   constexpr int kStride = kShare * kTopPThreads;
   const int groups = (V + 3) / 4;
-  for (int g0 = rank * kTopPThreads + threadIdx.x; g0 < groups; g0 += kUnroll * kStride) {
+  const float4* zq = reinterpret_cast<const float4*>(zr);
+  int g0 = rank * kTopPThreads + threadIdx.x;
+  // whole rounds: kUnroll unconditional loads in flight, then their logits
+  for (; g0 + (kUnroll - 1) * kStride < groups - 1; g0 += kUnroll * kStride) {
     float4 q[kUnroll];
 #pragma unroll
-    for (int u = 0; u < kUnroll; ++u) {
-      const int g = g0 + u * kStride;
-      q[u] = g < groups ? __ldcg(reinterpret_cast<const float4*>(zr) + g) : make_float4(0.f, 0.f, 0.f, 0.f);
-    }
+    for (int u = 0; u < kUnroll; ++u) q[u] = __ldcg(zq + g0 + u * kStride);
 #pragma unroll
     for (int u = 0; u < kUnroll; ++u) {
-      const int v = 4 * (g0 + u * kStride);
-      const float zz[4] = {q[u].x, q[u].y, q[u].z, q[u].w};
-#pragma unroll
-      for (int k = 0; k < 4; ++k)
-        if (v + k < V) f(v + k, zz[k] * inv_temp);
+      const int v = 4 * (g0 + u * kStride);  // every group here lies below the last, so v + 3 < V
+      f(v, q[u].x * inv_temp);
+      f(v + 1, q[u].y * inv_temp);
+      f(v + 2, q[u].z * inv_temp);
+      f(v + 3, q[u].w * inv_temp);
     }
+  }
+  // the rest, one group at a time (the last group may be partial)
+  for (; g0 < groups; g0 += kStride) {
+    const float4 q = __ldcg(zq + g0);
+    const int v = 4 * g0;
+    const float zz[4] = {q.x, q.y, q.z, q.w};
+#pragma unroll
+    for (int k = 0; k < 4; ++k)
+      if (v + k < V) f(v + k, zz[k] * inv_temp);
   }
 }
 
