@@ -13,9 +13,10 @@
 //      do not depend on the order of the atomics), over 2048 buckets of
 //      1/64 nat below the row maximum; the bucket where the mass counted from
 //      the top reaches top_p holds the threshold;
-//   2. that bucket's logits gathered in shared memory: the threshold y* is the
-//      largest candidate y with (mass above the bucket) + (candidate mass >= y)
-//      >= target; a bucket with more than kTopPCand logits is histogrammed
+//   2. that bucket's logits gathered in shared memory and sorted: the threshold
+//      y* is the first y (largest first) at which the mass above the bucket
+//      plus the running mass reaches the target; a bucket with more than
+//      kTopPCand logits is histogrammed
 //      again over its own range first (one whose logits are all equal is taken
 //      whole: ties stay together);
 //   3. the argmax over y >= y* of y + G with the GEMM's noise (Philox4x32-10
@@ -180,6 +181,73 @@ __device__ __forceinline__ void top_p_walk(const float* zr, int V, float inv_tem
   }
 }
 
+// The threshold among the nc gathered candidates (host CTA, every thread; the
+// result in every thread): the candidates sorted by y, largest first (bitonic
+// sort, padded to a power of two with -inf), their masses summed in that order
+// (fixed-order block scan); y* is the y at the first position where the mass
+// above the bucket plus the running sum reaches the target.  Equal logits sit
+// next to each other, so y*'s whole tie group counts toward the target.
+// -inf if no position does (the nucleus is then the whole vocabulary).
+__device__ __forceinline__ float top_p_resolve(TopPShared& sh, int nc) {
+  const int tid = threadIdx.x;
+  int n = 1;
+  while (n < nc) n <<= 1;  // <= kTopPCand
+  for (int i = nc + tid; i < n; i += kTopPThreads) {
+    sh.cy[i] = -INFINITY;
+    sh.cq[i] = 0ull;
+  }
+  __syncthreads();
+  for (int k = 2; k <= n; k <<= 1) {
+    for (int j = k >> 1; j > 0; j >>= 1) {
+      for (int i = tid; i < n; i += kTopPThreads) {
+        const int l = i ^ j;
+        if (l > i) {
+          const float a = sh.cy[i], b = sh.cy[l];
+          if ((i & k) == 0 ? a < b : a > b) {  // descending runs where bit k is clear
+            sh.cy[i] = b;
+            sh.cy[l] = a;
+            const unsigned long long t = sh.cq[i];
+            sh.cq[i] = sh.cq[l];
+            sh.cq[l] = t;
+          }
+        }
+      }
+      __syncthreads();
+    }
+  }
+  // running sums: thread tid owns positions [tid * per, (tid + 1) * per)
+  const int per = (n + kTopPThreads - 1) / kTopPThreads;
+  const int b0 = tid * per;
+  unsigned long long own = 0ull;
+  for (int i = b0; i < b0 + per && i < n; ++i) own += sh.cq[i];
+  unsigned long long inc = own;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const unsigned long long v = __shfl_up_sync(0xffffffffu, inc, o);
+    if ((tid & 31) >= o) inc += v;
+  }
+  if ((tid & 31) == 31) sh.ra[tid >> 5] = inc;
+  __syncthreads();
+  unsigned long long acc = inc - own;
+  for (int w = 0; w < (tid >> 5); ++w) acc += sh.ra[w];
+  const unsigned long long need = sh.target - sh.cum_before;
+  int first = n;
+  for (int i = b0; i < b0 + per && i < n; ++i) {
+    acc += sh.cq[i];
+    if (acc >= need) {
+      first = i;
+      break;
+    }
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) first = min(first, __shfl_xor_sync(0xffffffffu, first, o));
+  __syncthreads();
+  if ((tid & 31) == 0) sh.ri[tid >> 5] = first;
+  __syncthreads();
+  for (int w = 0; w < kTopPWarps; ++w) first = min(first, sh.ri[w]);
+  return first < n ? sh.cy[first] : -INFINITY;
+}
+
 // The better of two perturbed scores (the lower token on a tie; -1 loses).
 __device__ __forceinline__ bool top_p_better(float s, int v, float s0, int v0) {
   return s > s0 || (s == s0 && v >= 0 && (v0 < 0 || v < v0));
@@ -331,15 +399,7 @@ __global__ void __cluster_dims__(kTopPCtas, 1, 1) __launch_bounds__(kTopPThreads
       if (host) {
         const int nc = static_cast<int>(min(sh.ncand, static_cast<unsigned>(kTopPCand)));
         if (sh.ncand <= static_cast<unsigned>(kTopPCand)) {
-          // the threshold: the largest candidate y whose upper set (with all above the bucket) reaches the target
-          float best = -INFINITY;
-          for (int i = tid; i < nc; i += kTopPThreads) {
-            const float yi = sh.cy[i];
-            unsigned long long above = 0ull;
-            for (int j = 0; j < nc; ++j) above += sh.cy[j] >= yi ? sh.cq[j] : 0ull;
-            if (sh.cum_before + above >= sh.target) best = fmaxf(best, yi);
-          }
-          best = top_p_block_max(sh, best);
+          const float best = top_p_resolve(sh, nc);
           if (tid == 0) {
             sh.ystar = best;
             sh.mode = 2;
