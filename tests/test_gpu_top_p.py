@@ -36,20 +36,21 @@ def _draw(Hb, Wb, m, tau, top_p, seed, offset, ws=None):
     return tok.cpu().numpy(), lp.cpu().numpy()
 
 
-def _compare(Hb, Wb, m, tau, top_p, seed, offset, tok, logp, band_mass=1e-5, band_logit=1e-4):
-    want, want_lp, gap, band = oracle.sample_tokens_top_p(Hb, Wb, m, tau, top_p, seed, offset,
+def _compare(Hb, Wb, m, tau, top_p, seed, offset, tok, logp, band_mass=1e-5, band_logit=1e-4, rows=None):
+    want, want_lp, gap, band = oracle.sample_tokens_top_p(Hb, Wb, m, tau, top_p, seed, offset, rows=rows,
                                                            band_mass=band_mass, band_logit=band_logit)
-    idx = wl.valid_index(m)
+    idx = wl.valid_index(m) if rows is None else np.asarray(rows)
     assert np.all(tok[m == 0] == -1) and np.all(logp[m == 0] == 0.0)
     same = tok[idx] == want[idx]
     assert same.mean() >= 0.9, same.mean()
     Wf = oracle.as_f64(Wb)
     for t in idx:
-        y = (oracle.as_f64(Hb[t]) @ Wf.T) / tau
+        h = oracle.as_f64(Hb[t])
+        y_got, y_want = (h @ Wf[tok[t]]) / tau, (h @ Wf[want[t]]) / tau
         lo, hi = band[t]
-        assert y[tok[t]] >= lo, (t, y[tok[t]], lo)         # never outside the nucleus and its band
+        assert y_got >= lo, (t, y_got, lo)         # never outside the nucleus and its band
         if tok[t] != want[t]:
-            in_band = lo <= y[tok[t]] <= hi or lo <= y[want[t]] <= hi
+            in_band = lo <= y_got <= hi or lo <= y_want <= hi
             assert gap[t] <= TIE or in_band, (t, tok[t], want[t], gap[t])
     ok = idx[same]
     assert np.abs(logp[ok] - want_lp[ok]).max() <= LOGP_ATOL
@@ -184,3 +185,15 @@ def test_top_p_lean_workspace_capacity_and_arguments():
             grpo.sample_tokens_top_p(H, W, md, 1.0, bad)
     empty = grpo.sample_tokens_top_p(H[:0], W, md[:0], 1.0, 0.9)
     assert empty[0].numel() == 0
+
+
+@pytest.mark.parametrize("top_p,n_rows", [(0.9, 256), (0.5, 128)])
+def test_top_p_decode_step_full_vocabulary(top_p, n_rows):
+    """A decode step of the 8B head (256 rows x 155,136 tokens, Hd 4096)
+    against the oracle (on n_rows of the rows): the shape the nucleus draw
+    serves in rollout generation, with about (1 - top_p) of the rows through
+    the cluster kernel's histogram path."""
+    w = wl.DECODE_WORKLOADS["decode256_8b"]
+    Hb, Wb, m = wl.gen_hidden(w), wl.gen_weight(w), wl.gen_mask(w)
+    tok, lp = _draw(Hb, Wb, m, 1.0, top_p, 20250705, 9)
+    _compare(Hb, Wb, m, 1.0, top_p, 20250705, 9, tok, lp, rows=wl.valid_index(m)[:n_rows])
