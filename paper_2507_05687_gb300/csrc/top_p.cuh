@@ -580,16 +580,55 @@ __global__ void __launch_bounds__(kTopPThreads)
                       const float* __restrict__ lse_r, const float* __restrict__ y0_r, float inv_temp, float top_p,
                       int* __restrict__ slow_rows, unsigned long long* __restrict__ slow_target,
                       unsigned* __restrict__ n_slow) {
+  constexpr int kUnroll = 8;
   __shared__ unsigned long long ra[kTopPWarps];
+  __shared__ float wbuf[kTopPWarps][32 * 4 * kUnroll];  // one warp's logits above the winner in a round
   const int tid = threadIdx.x;
+  const int lane = tid & 31;
+  float* buf = wbuf[tid >> 5];
   const int nv = *n_valid;
+  const int groups = (V + 3) / 4;
   for (int r = blockIdx.x; r < nv; r += gridDim.x) {
     const float* zr = z + static_cast<int64_t>(r) * ldz;
+    const float4* zq = reinterpret_cast<const float4*>(zr);
     const float lse = lse_r[r], y0 = y0_r[r];
     unsigned long long above = 0ull;
-    top_p_walk<8, 1>(zr, V, inv_temp, 0, [&](int, float y) {
-      if (y > y0) above += top_p_mass(y, lse);  // most logits lie below the winner: a compare only
-    });
+    // whole rounds: most logits lie below the winner, so each warp gathers the
+    // ones above it (ballot + prefix count) and computes their masses with all
+    // lanes busy instead of a few lanes at a time
+    // (the test uses the warp's last lane, so that every lane of a warp runs the
+    // same rounds: the ballots need the whole warp)
+    int g0 = tid;
+    for (; g0 - lane + 31 + (kUnroll - 1) * kTopPThreads < groups - 1; g0 += kUnroll * kTopPThreads) {
+      float4 q[kUnroll];
+#pragma unroll
+      for (int u = 0; u < kUnroll; ++u) q[u] = __ldcg(zq + g0 + u * kTopPThreads);
+      int cnt = 0;
+#pragma unroll
+      for (int u = 0; u < kUnroll; ++u) {
+        const float yy[4] = {q[u].x * inv_temp, q[u].y * inv_temp, q[u].z * inv_temp, q[u].w * inv_temp};
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+          const bool a = yy[k] > y0;
+          const unsigned bal = __ballot_sync(0xffffffffu, a);
+          if (a) buf[cnt + __popc(bal & ((1u << lane) - 1u))] = yy[k];
+          cnt += __popc(bal);
+        }
+      }
+      __syncwarp();
+      for (int i = lane; i < cnt; i += 32) above += top_p_mass(buf[i], lse);
+      __syncwarp();
+    }
+    // the rest, one group at a time (the last group may be partial)
+    for (; g0 < groups; g0 += kTopPThreads) {
+      const float4 q = __ldcg(zq + g0);
+      const float zz[4] = {q.x, q.y, q.z, q.w};
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        const float y = zz[k] * inv_temp;
+        if (4 * g0 + k < V && y > y0) above += top_p_mass(y, lse);
+      }
+    }
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) above += __shfl_xor_sync(0xffffffffu, above, o);
     if ((tid & 31) == 0) ra[tid >> 5] = above;
