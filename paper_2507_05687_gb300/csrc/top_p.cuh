@@ -52,6 +52,7 @@ constexpr int kTopPBuckets = 2048;
 constexpr int kTopPCand = 1024;    // candidates resolved exactly in shared memory
 constexpr int kTopPLevels = 6;     // histogram levels before the candidates fit
 constexpr int kTopPWarps = kTopPThreads / 32;
+static_assert(kTopPBuckets == kTopPCtas * kTopPThreads, "one histogram bucket per thread of the cluster in the merge");
 
 // Shared memory of one CTA.  The fields marked "host" are used in CTA 0 of
 // the cluster only (the other CTAs write into and read from CTA 0's copy).
@@ -298,17 +299,20 @@ __global__ void __cluster_dims__(kTopPCtas, 1, 1) __launch_bounds__(kTopPThreads
         }
       });
       cluster_sync();
-      if (host) {  // merge the histograms in rank order, find the bucket that holds the threshold
-        for (int b = tid; b < kTopPBuckets; b += kTopPThreads) {
-          unsigned long long part[kTopPCtas];
+      {  // merge the histograms: CTA k sums buckets [k * kTopPThreads, (k + 1) * kTopPThreads) over
+         // the cluster in rank order and leaves the sums in CTA 0's histogram (disjoint slices, so no
+         // CTA reads a bucket another one writes)
+        const int b = rank * kTopPThreads + tid;
+        unsigned long long part[kTopPCtas];
 #pragma unroll
-          for (int k = 1; k < kTopPCtas; ++k) part[k] = ld_shared_cluster_u64(mapa_shared(smem_addr(&sh.hist[b]), k));
-          unsigned long long m = sh.hist[b];
+        for (int k = 0; k < kTopPCtas; ++k) part[k] = ld_shared_cluster_u64(mapa_shared(smem_addr(&sh.hist[b]), k));
+        unsigned long long m = 0ull;
 #pragma unroll
-          for (int k = 1; k < kTopPCtas; ++k) m += part[k];
-          sh.hist[b] = m;
-        }
-        __syncthreads();
+        for (int k = 0; k < kTopPCtas; ++k) m += part[k];
+        st_shared_cluster_u64(at0(&sh.hist[b]), m);
+      }
+      cluster_sync();
+      if (host) {  // find the bucket that holds the threshold
         // the first bucket where the mass from the top reaches the target: each
         // thread sums a range of buckets, thread 0 walks the range sums and then
         // the buckets of the one range that crosses
