@@ -63,19 +63,18 @@ struct TopPShared {
   float ly[kTopPCand];                     // this CTA's candidates before they go to the host
   unsigned long long lq[kTopPCand];
   unsigned long long scan[kTopPThreads];   // host: per-thread bucket-range sums of the scan
-  unsigned long long slot_a[kTopPCtas], slot_b[kTopPCtas];  // host: one partial per CTA
-  uint32_t slot_f[kTopPCtas], slot_g[kTopPCtas], slot_i[kTopPCtas];
+  uint32_t slot_f[kTopPCtas], slot_g[kTopPCtas], slot_i[kTopPCtas];  // host: one partial per CTA
   float lvl_hi[kTopPLevels];
   float lvl_scale[kTopPLevels];
   int lvl_b[kTopPLevels];
-  unsigned long long ra[kTopPWarps], rb[kTopPWarps];
+  unsigned long long ra[kTopPWarps];
   float rf[kTopPWarps], rg[kTopPWarps];
   int ri[kTopPWarps];
   unsigned long long cum_before, target;   // host, copied to every CTA
   unsigned ncand;                          // host
   unsigned lcand, lbase;                   // this CTA's candidate count and its offset at the host
   float lse, y0, ystar;
-  int tok0, nlvl;
+  int nlvl;
   int mode;  // 0 histogram, 1 resolve the gathered candidates, 2 threshold known
 };
 
@@ -123,27 +122,6 @@ __device__ __forceinline__ float top_p_block_max(TopPShared& sh, float v) {
   float r = sh.rf[0];
   for (int i = 1; i < kTopPWarps; ++i) r = fmaxf(r, sh.rf[i]);
   return r;
-}
-
-// Block-wide sums of two 64-bit values in a fixed order (every thread gets them).
-__device__ __forceinline__ void top_p_block_sum2(TopPShared& sh, unsigned long long& a, unsigned long long& b) {
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) {
-    a += __shfl_xor_sync(0xffffffffu, a, o);
-    b += __shfl_xor_sync(0xffffffffu, b, o);
-  }
-  __syncthreads();
-  if ((threadIdx.x & 31) == 0) {
-    sh.ra[threadIdx.x >> 5] = a;
-    sh.rb[threadIdx.x >> 5] = b;
-  }
-  __syncthreads();
-  a = 0ull;
-  b = 0ull;
-  for (int i = 0; i < kTopPWarps; ++i) {
-    a += sh.ra[i];
-    b += sh.rb[i];
-  }
 }
 
 // Walks this CTA's share of the row (kShare CTAs share it; rank is this
