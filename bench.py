@@ -92,7 +92,7 @@ def make_inputs(w: wl.Workload):
     y, m, r = wl.gen_targets(w), wl.gen_mask(w), wl.gen_rewards(w)
     old = np.zeros(w.T, np.float32)
     ref = np.zeros(w.T, np.float32)
-    src = None
+    src = lse_gold = None
     g = GOLDEN.get(w.name)
     path = os.path.join(ROOT, "tests", "golden", f"{g}.npz") if g else None
     if path and os.path.exists(path) and w.seed == wl.ALL_WORKLOADS[w.name].seed:
@@ -101,8 +101,32 @@ def make_inputs(w: wl.Workload):
         if int(d["n_valid"]) == idx.size:
             old[idx] = d["old_logp"]
             ref[idx] = d["ref_logp"]
+            lse_gold = d["lse_policy"]
             src = "float64 oracle on the perturbed heads (tests/golden)"
-    return dict(H=Hb, W=Wb, y=y, m=m, r=r, old=old, ref=ref, old_src=src)
+    return dict(H=Hb, W=Wb, y=y, m=m, r=r, old=old, ref=ref, old_src=src, lse_gold=lse_gold)
+
+
+def parity_logp(inp, grpo, H, W, y, m):
+    """The library's log-probs of this batch against the float64 oracle's, on every
+    valid token: the oracle's log-sum-exp stored in tests/golden, minus nothing
+    but the target logit recomputed here in float64 (one dot product per token).
+    None when no stored values exist for the batch."""
+    lse = inp.get("lse_gold")
+    if lse is None:
+        return None
+    idx = wl.valid_index(inp["m"])
+    got = grpo.token_logprobs(H, W, y, m).cpu().numpy()[idx].astype(np.float64)
+
+    def widen(bits):
+        return (bits.astype(np.uint32) << np.uint32(16)).view(np.float32).astype(np.float64)
+
+    err = np.empty(idx.size)
+    for a in range(0, idx.size, 8192):
+        rows = idx[a:a + 8192]
+        zy = np.einsum("ij,ij->i", widen(inp["H"][rows]), widen(inp["W"][inp["y"][rows]]))
+        err[a:a + rows.size] = np.abs(got[a:a + rows.size] - (zy - lse[a:a + rows.size]))
+    return {"logp_max_abs_err": float(err.max()), "logp_mean_abs_err": float(err.mean()), "tokens": int(idx.size),
+            "bar": 2e-3, "reference": "float64 oracle (log-sum-exp stored in tests/golden, target logit in float64)"}
 
 
 def fill_old_ref_on_gpu(w, inp, grpo, torch, dev):
@@ -494,6 +518,8 @@ def main():
             if world == 1:
                 e2e_offload = measure_e2e_offload(grpo, torch, dev, w, inp, steps=min(args.steps, 5), ws=ws)
 
+    parity = parity_logp(inp, grpo, H, W, y, m) if rank == 0 and not sampling else None
+
     cpu = None
     if not args.no_cpu_baseline and rank == 0 and world == 1 and not sampling:
         ntok, dt = (cpu_oracle_scoring_sample if scoring else cpu_oracle_sample)(w, inp, args.cpu_sample_tokens)
@@ -522,6 +548,7 @@ def main():
             "step_frac_executed": round(step_exec / (ms / 1e3) / 1e12 / burst, 4),
             "step_frac_6x": round(step_model / (ms / 1e3) / 1e12 / burst, 4),
             "roofline": rf, "clocks": clocks, "gpu_launches": launches, "e2e": e2e, "cpu_baseline": cpu,
+            "parity": parity,
         }
         if e2e_offload is not None:
             line["e2e_offload"] = e2e_offload
