@@ -71,7 +71,8 @@ struct Layout {
   int64_t ldz;    // leading dimension (fp32 elements) of the stored logits; 0: not stored
   int lse_tiles;  // vocabulary tiles (of 256) per forward work unit
   size_t status, n_valid, counts, offsets, cidx, rank_of, yc, zy, part_m, part_s, lse_c, g_c,
-      block_loss, resp_len, best_s, best_c, best_z, Hc, HcT, dz, dhc, z, slow_rows, slow_tgt, n_slow, total;
+      block_loss, resp_len, best_s, best_c, best_z, Hc, HcT, dz, dhc, z, slow_rows, slow_tgt, n_slow, row_above,
+      row_done, total;
 };
 
 bool make_layout(int64_t T, int32_t Hd, int64_t V, int32_t which, Layout* L, int64_t rows_cap = -1) {
@@ -139,6 +140,8 @@ bool make_layout(int64_t T, int32_t Hd, int64_t V, int32_t which, Layout* L, int
   L->slow_rows = take(top_p ? 4 * cr : 0, 256);
   L->slow_tgt = take(top_p ? 8 * cr : 0, 256);
   L->n_slow = take(top_p ? 4 : 0, 256);
+  L->row_above = take(top_p ? 8 * cr : 0, 256);
+  L->row_done = take(top_p ? 4 * cr : 0, 256);
   L->total = (off + 1023) / 1024 * 1024;
   return true;
 }
@@ -895,20 +898,26 @@ grpo_status grpo_sample_tokens_top_p(const uint16_t* H, const uint16_t* W, const
     top_p_prep_kernel<<<pb, 256, 0, s>>>(at<int>(ws, Ly.n_valid), at<int>(ws, Ly.cidx), at<float>(ws, Ly.part_m),
                                          at<float>(ws, Ly.part_s), at<float>(ws, Ly.best_s),
                                          at<int>(ws, Ly.best_c), at<float>(ws, Ly.best_z),
-                                         static_cast<int>(Ly.nsplit), Ly.rows, lse_r, y0_r, hi_r, tokens_out,
-                                         logp_out, at<unsigned>(ws, Ly.status));
+                                         static_cast<int>(Ly.nsplit), Ly.rows, lse_r, y0_r, hi_r,
+                                         at<unsigned long long>(ws, Ly.row_above), at<unsigned>(ws, Ly.row_done),
+                                         tokens_out, logp_out, at<unsigned>(ws, Ly.status));
     e = cudaGetLastError();
     if (e == cudaSuccess && top_p < 1.f) {
       unsigned* n_slow = at<unsigned>(ws, Ly.n_slow);
       e = cudaMemsetAsync(n_slow, 0, 4, s);
-      // is the winner in the nucleus?  one CTA per row, rows in turn; four CTAs
-      // per SM (58 registers x 256 threads), all resident
-      const int fb2 = static_cast<int>(std::min<int64_t>(Ly.rows, int64_t(di.sms) * 4));
+      // is the winner in the nucleus?  four CTAs per SM, all resident; a row is
+      // cut into slices (one CTA each, up to 8) until there are about two
+      // pieces of work per CTA (the row count is the capacity here: the
+      // unmasked count is only known on the device)
+      const int64_t slots = int64_t(di.sms) * 4;
+      const int slices = static_cast<int>(
+          std::max<int64_t>(1, std::min<int64_t>(8, (2 * slots + Ly.rows - 1) / std::max<int64_t>(1, Ly.rows))));
+      const int fb2 = static_cast<int>(std::min<int64_t>(Ly.rows * slices, slots));
       if (e == cudaSuccess)
-        top_p_fast_kernel<<<fb2, kTopPThreads, 0, s>>>(at<float>(ws, Ly.z), Ly.ldz, static_cast<int>(V),
-                                                       at<int>(ws, Ly.n_valid), lse_r, y0_r, 1.f / temperature,
-                                                       top_p, at<int>(ws, Ly.slow_rows),
-                                                       at<unsigned long long>(ws, Ly.slow_tgt), n_slow);
+        top_p_fast_kernel<<<fb2, kTopPThreads, 0, s>>>(
+            at<float>(ws, Ly.z), Ly.ldz, static_cast<int>(V), at<int>(ws, Ly.n_valid), slices, lse_r, y0_r,
+            1.f / temperature, top_p, at<unsigned long long>(ws, Ly.row_above), at<unsigned>(ws, Ly.row_done),
+            at<int>(ws, Ly.slow_rows), at<unsigned long long>(ws, Ly.slow_tgt), n_slow);
       // the rows whose winner falls outside: clusters of kTopPCtas CTAs, one row
       // per cluster at a time, as many clusters as can be resident together
       const int64_t clusters = std::max<int64_t>(1, std::min<int64_t>(Ly.rows, di.top_p_clusters));

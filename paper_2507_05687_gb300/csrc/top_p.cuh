@@ -494,7 +494,7 @@ __global__ void __cluster_dims__(kTopPCtas, 1, 1) __launch_bounds__(kTopPThreads
 // Per unmasked row, the plain draw from the sampling GEMM's splits: written
 // to the outputs (the nucleus selection replaces it only where the winner
 // falls outside the nucleus), and the row's LSE, winner's y and maximum y kept
-// for the selection.  One warp per row reads the splits in parallel; the LSE
+// for the selection (whose per-row accumulators it clears).  One warp per row reads the splits in parallel; the LSE
 // sum runs in split order with merge_lse's rounding, and the winner is the best
 // score with the lowest split on a tie, as sample_merge_kernel takes them, so
 // the draw is the plain sampler's bit for bit.
@@ -502,8 +502,9 @@ __global__ void top_p_prep_kernel(const int* __restrict__ n_valid, const int* __
                                   const float* __restrict__ pm, const float* __restrict__ ps,
                                   const float* __restrict__ bs, const int* __restrict__ bc,
                                   const float* __restrict__ bz, int nsplit, long ldp, float* __restrict__ lse_r,
-                                  float* __restrict__ y0_r, float* __restrict__ hi_r, int32_t* __restrict__ tokens,
-                                  float* __restrict__ logp, unsigned* status) {
+                                  float* __restrict__ y0_r, float* __restrict__ hi_r,
+                                  unsigned long long* __restrict__ row_above, unsigned* __restrict__ row_done,
+                                  int32_t* __restrict__ tokens, float* __restrict__ logp, unsigned* status) {
   const float kLn2 = 0.69314718055994531f;
   const int lane = threadIdx.x & 31;
   const int nv = *n_valid;
@@ -545,6 +546,8 @@ __global__ void top_p_prep_kernel(const int* __restrict__ n_valid, const int* __
       lse_r[r] = lse;
       y0_r[r] = y0;
       hi_r[r] = m * kLn2;
+      row_above[r] = 0ull;  // the fast pass's per-row accumulators
+      row_done[r] = 0u;
       const int t = cidx[r];
       tokens[t] = tok;
       logp[t] = y0 - lse;
@@ -552,14 +555,20 @@ __global__ void top_p_prep_kernel(const int* __restrict__ n_valid, const int* __
   }
 }
 
-// Is each row's plain winner in its nucleus?  One CTA per row, many rows in
-// flight per SM: the mass strictly above the winner
-// (2^-40 fixed point, fixed-order sums), the target top_p_target.  The winner
-// is in exactly when the mass above it is below the target; a row whose winner
-// is outside goes to the list top_p_kernel works through, with its target.
+// Is each row's plain winner in its nucleus?  The mass strictly above the
+// winner (2^-40 fixed point, exact integer sums), against the target
+// top_p_target: the winner is in exactly when that mass is below the target;
+// a row whose winner is outside goes to the list top_p_kernel works through,
+// with its target.  A row is cut into `slices` interleaved slices, one CTA
+// each (more than one for batches with too few rows to fill the GPU): each
+// adds its slice's mass into the row's accumulator with a device-wide atomic,
+// fences, and counts itself done; the CTA that completes the count makes the
+// decision (nothing waits for anything).  row_above / row_done start at 0
+// (top_p_prep_kernel clears them).
 __global__ void __launch_bounds__(kTopPThreads)
     top_p_fast_kernel(const float* __restrict__ z, int64_t ldz, int V, const int* __restrict__ n_valid,
-                      const float* __restrict__ lse_r, const float* __restrict__ y0_r, float inv_temp, float top_p,
+                      int slices, const float* __restrict__ lse_r, const float* __restrict__ y0_r, float inv_temp,
+                      float top_p, unsigned long long* __restrict__ row_above, unsigned* __restrict__ row_done,
                       int* __restrict__ slow_rows, unsigned long long* __restrict__ slow_target,
                       unsigned* __restrict__ n_slow) {
   constexpr int kUnroll = 8;
@@ -570,9 +579,12 @@ __global__ void __launch_bounds__(kTopPThreads)
   float* buf = wbuf[tid >> 5];
   const int nv = *n_valid;
   const int groups = (V + 3) / 4;
-  for (int r = blockIdx.x; r < nv; r += gridDim.x) {
-    const float* zr = z + static_cast<int64_t>(r) * ldz;
-    const float4* zq = reinterpret_cast<const float4*>(zr);
+  const int stride = slices * kTopPThreads;
+  const int64_t items = static_cast<int64_t>(nv) * slices;
+  for (int64_t it = blockIdx.x; it < items; it += gridDim.x) {
+    const int r = static_cast<int>(it / slices);
+    const int sl = static_cast<int>(it - static_cast<int64_t>(r) * slices);
+    const float4* zq = reinterpret_cast<const float4*>(z + static_cast<int64_t>(r) * ldz);
     const float lse = lse_r[r], y0 = y0_r[r];
     unsigned long long above = 0ull;
     // whole rounds: most logits lie below the winner, so each warp gathers the
@@ -580,11 +592,11 @@ __global__ void __launch_bounds__(kTopPThreads)
     // lanes busy instead of a few lanes at a time
     // (the test uses the warp's last lane, so that every lane of a warp runs the
     // same rounds: the ballots need the whole warp)
-    int g0 = tid;
-    for (; g0 - lane + 31 + (kUnroll - 1) * kTopPThreads < groups - 1; g0 += kUnroll * kTopPThreads) {
+    int g0 = sl * kTopPThreads + tid;
+    for (; g0 - lane + 31 + (kUnroll - 1) * stride < groups - 1; g0 += kUnroll * stride) {
       float4 q[kUnroll];
 #pragma unroll
-      for (int u = 0; u < kUnroll; ++u) q[u] = __ldcg(zq + g0 + u * kTopPThreads);
+      for (int u = 0; u < kUnroll; ++u) q[u] = __ldcg(zq + g0 + u * stride);
       int cnt = 0;
 #pragma unroll
       for (int u = 0; u < kUnroll; ++u) {
@@ -602,7 +614,7 @@ __global__ void __launch_bounds__(kTopPThreads)
       __syncwarp();
     }
     // the rest, one group at a time (the last group may be partial)
-    for (; g0 < groups; g0 += kTopPThreads) {
+    for (; g0 < groups; g0 += stride) {
       const float4 q = __ldcg(zq + g0);
       const float zz[4] = {q.x, q.y, q.z, q.w};
 #pragma unroll
@@ -618,8 +630,18 @@ __global__ void __launch_bounds__(kTopPThreads)
     if (tid == 0) {
       above = 0ull;
       for (int w = 0; w < kTopPWarps; ++w) above += ra[w];
+      bool decide = true;
+      if (slices > 1) {
+        atomicAdd(&row_above[r], above);
+        __threadfence();
+        decide = atomicAdd(&row_done[r], 1u) == static_cast<unsigned>(slices - 1);
+        if (decide) {
+          __threadfence();
+          above = atomicAdd(&row_above[r], 0ull);  // every slice's mass (each fenced before counting itself)
+        }
+      }
       const unsigned long long target = top_p_target(top_p);
-      if (above >= target) {
+      if (decide && above >= target) {
         const unsigned k = atomicAdd(n_slow, 1u);
         slow_rows[k] = r;
         slow_target[k] = target;
