@@ -197,3 +197,15 @@ def test_top_p_decode_step_full_vocabulary(top_p, n_rows):
     Hb, Wb, m = wl.gen_hidden(w), wl.gen_weight(w), wl.gen_mask(w)
     tok, lp = _draw(Hb, Wb, m, 1.0, top_p, 20250705, 9)
     _compare(Hb, Wb, m, 1.0, top_p, 20250705, 9, tok, lp, rows=wl.valid_index(m)[:n_rows])
+
+
+@pytest.mark.parametrize("V", [1, 2, 3, 5])
+def test_top_p_tiny_vocabularies(V):
+    """Vocabularies below and just above one 4-logit group: the walks' tails
+    alone (and, at V = 1, a nucleus that is the single token)."""
+    w = wl.Workload("p", 2, 4, 30, 64, V, "uniform", 1, 30, seed=wl.SEED_BASE + 3100 + V, w_std=0.5)
+    Hb, Wb, m = wl.gen_hidden(w), wl.gen_weight(w), wl.gen_mask(w)
+    for top_p in (0.5, 0.9):
+        tok, lp = _draw(Hb, Wb, m, 1.0, top_p, 12, 3)
+        assert np.all(tok[m != 0] >= 0) and np.all(tok[m != 0] < V)
+        _compare(Hb, Wb, m, 1.0, top_p, 12, 3, tok, lp)
