@@ -283,6 +283,46 @@ def test_kept_logits_lean_workspace_and_capacity(monkeypatch):
     _check_fwd_bwd(c, kind=grpo.GRPO_WS_LOSS_LOGITS)    # a full workspace on the same context
 
 
+def test_entry_points_agree_across_workspaces(monkeypatch):
+    """Every loss entry point (global normaliser, KL cap, per-chunk events,
+    dW streamed to pinned host memory, fused AdamW) gives the same bits with a
+    kept-logits workspace as with the plain one that recomputes the logits."""
+    monkeypatch.setenv("GRPO_VOCAB_CHUNK", "512")
+    w = wl.Workload("t", 2, 4, 70, 192, 1700, "uniform", 1, 70, rewards="mix", seed=wl.SEED_BASE + 5500)
+    c = _case(w)
+    d = _dev(c)
+    nv = float(c["m"].sum())
+    args = (d["H"], d["W"], d["y"], d["m"], d["old"], d["ref"], d["adv"], w.n_resp, w.L, w.clip_eps, w.beta, 0)
+    n_chunks = -(-w.V // grpo.vocab_chunk_cols(w.V))
+    assert n_chunks == 4
+
+    def run(kind):
+        ws = grpo.workspace(w.T, w.Hd, w.V, kind, DEV)
+        out = [grpo.loss_fwd_bwd(*args, ws=ws, norm=2.5 * nv),
+               grpo.loss_fwd_bwd(*args, ws=ws, kl_clamp=0.05)]
+        events = [torch.cuda.Event() for _ in range(n_chunks)]
+        out.append(grpo.loss_fwd_bwd(*args, ws=ws, chunk_events=events))
+        host = (torch.empty(1).pin_memory(), torch.empty(w.T, w.Hd).pin_memory(),
+                torch.empty(w.V, w.Hd).pin_memory())
+        out.append(grpo.loss_fwd_bwd(*args, ws=ws, out=host))
+        rng = np.random.default_rng(3)
+        master = dev_tensor(oracle.widen_bf16(c["W"]).astype(np.float32), torch.float32)
+        ea = torch.zeros_like(master)
+        eas = dev_tensor((1e-4 * rng.random(master.shape)).astype(np.float32), torch.float32)
+        W_out = torch.empty_like(d["W"])
+        lo, dH = grpo.loss_fwd_bwd_adamw(*args[:9], master, ea, eas, 1, lr=1e-3, W_out=W_out, ws=ws)
+        out.append((lo, dH, master, ea, eas, W_out))
+        torch.cuda.synchronize()
+        assert grpo.check_device_status(ws) == grpo.GRPO_OK
+        return out
+
+    kept, plain = run(grpo.GRPO_WS_LOSS_LOGITS), run(grpo.GRPO_WS_LOSS)
+    for a, b in zip(kept, plain):
+        for x, y in zip(a, b):
+            assert torch.equal(x.cpu(), y.cpu())
+    assert not torch.equal(kept[0][0], kept[1][0])      # the cap and the normaliser change the loss
+
+
 def test_fwd_bwd_is_deterministic():
     c = _case(wl.Workload("t", 1, 4, 70, 256, 2000, "uniform", 5, 70, seed=wl.SEED_BASE + 600))
     a = _check_fwd_bwd(c)
