@@ -7,36 +7,37 @@
 //
 // The sampling GEMM (kEpiSampleZ) has already produced, per row, the log-sum-
 // exp of y = z / temperature, the row maximum and the plain Gumbel-max winner
-// over the whole vocabulary, and stored the fp32 logits z.  For a row whose
-// plain winner falls outside the nucleus (see below):
-//   1. a histogram of the probability mass, in 2^-40 fixed point (so the sums
-//      do not depend on the order of the atomics), over 2048 buckets of
-//      1/64 nat below the row maximum; the bucket where the mass counted from
-//      the top reaches top_p holds the threshold;
-//   2. that bucket's logits gathered in shared memory and sorted: the threshold
-//      y* is the first y (largest first) at which the mass above the bucket
-//      plus the running mass reaches the target; a bucket with more than
-//      kTopPCand logits is histogrammed
-//      again over its own range first (one whose logits are all equal is taken
-//      whole: ties stay together);
-//   3. the argmax over y >= y* of y + G with the GEMM's noise (Philox4x32-10
-//      word v mod 4 of counter (v div 4, t, offset), key seed) and fp32
-//      operations, the lowest v on ties.
-// Before any of that, a pass with one CTA per row (top_p_fast_kernel) decides
-// whether the plain winner w0 (the GEMM's argmax over the whole vocabulary,
-// already written to the outputs by top_p_prep_kernel) is in the nucleus: it
-// is exactly when the mass of the logits strictly above y_w0 is below the
-// target (then y_w0 >= y*; otherwise the tokens above it already reach the
-// target and y* > y_w0).  A winner inside is the nucleus winner too, its
-// perturbed score beating every token; that is the case for about a fraction
-// top_p of the rows.  Only the others go through steps 1-3 (top_p_kernel), and
-// top_p = 1 needs neither kernel.
+// w0 over the whole vocabulary, and stored the fp32 logits z.
 //
-// A row of the remaining list is shared by a cluster of kTopPCtas CTAs
-// (distributed shared memory): each walks an interleaved eighth of the row, and
-// CTA 0 of the cluster holds the merged histogram, candidates and decisions,
-// which the others read back after a cluster barrier.
-// Every reduction has a fixed order, so a row's draw is deterministic.
+// A pass with one CTA per row (top_p_fast_kernel) first decides whether w0 is
+// in the nucleus: it is exactly when the mass of the logits strictly above
+// y_w0 is below the target (then y_w0 >= y*; otherwise the tokens above it
+// already reach the target and y* > y_w0).  A winner inside is the nucleus
+// winner too, its perturbed score beating every token; that is the case for
+// about a fraction top_p of the rows, and top_p = 1 needs no selection at all.
+// Masses are probabilities in 2^-40 fixed point, so no sum depends on the
+// order of the atomics that form it.
+//
+// The other rows form a list, and a cluster of kTopPCtas CTAs takes one row
+// at a time (distributed shared memory; each CTA walks an interleaved eighth
+// of the row).  Since y* > y_w0, only logits above y_w0 matter:
+//   1. a histogram of their mass over 2048 buckets spanning [y_w0, max y]
+//      (at most 1/64 nat each); the bucket where the mass counted from the top
+//      reaches the target holds y*;
+//   2. a second walk gathers that bucket's logits as candidates (every CTA
+//      receives all of them) and, on the way, keeps the best perturbed score
+//      y + G over the logits above the bucket, which are all in the nucleus
+//      (G: the GEMM's noise, Philox4x32-10 word v mod 4 of counter
+//      (v div 4, t, offset), key seed, fp32 operations, the lowest v on ties);
+//      a bucket with more than kTopPCand logits is histogrammed again over its
+//      own range first (one whose logits are all equal is taken whole: ties
+//      stay together);
+//   3. y* is the largest candidate y whose mass together with that of the
+//      candidates above it reaches what the target still needs (an exact rank
+//      count, the candidates split over the cluster), and the draw is the best
+//      of the score from step 2 and the scores of the candidates >= y*.
+// Every reduction has a fixed order or is exact, so a row's draw is
+// deterministic.
 #pragma once
 
 #include <stdint.h>
@@ -57,25 +58,31 @@ static_assert(kTopPBuckets == kTopPCtas * kTopPThreads, "one histogram bucket pe
 // Shared memory of one CTA.  The fields marked "host" are used in CTA 0 of
 // the cluster only (the other CTAs write into and read from CTA 0's copy).
 struct TopPShared {
-  unsigned long long hist[kTopPBuckets];   // this CTA's histogram; host: then the merged one
-  float cy[kTopPCand];                     // host: the gathered candidates
+  union {
+    unsigned long long hist[kTopPBuckets];  // histogram pass: this CTA's histogram; host: then the merged one
+    struct {                                // gather pass: this CTA's candidates before they are broadcast
+      float y[kTopPCand];
+      int v[kTopPCand];
+    } loc;
+  };
+  float cy[kTopPCand];                      // the cluster's candidates: every CTA holds all of them
   unsigned long long cq[kTopPCand];
-  float ly[kTopPCand];                     // this CTA's candidates before they go to the host
-  unsigned long long lq[kTopPCand];
-  unsigned long long scan[kTopPThreads];   // host: per-thread bucket-range sums of the scan
-  uint32_t slot_f[kTopPCtas], slot_g[kTopPCtas], slot_i[kTopPCtas];  // host: one partial per CTA
+  int cv[kTopPCand];
+  unsigned long long scan[kTopPThreads];    // host: per-thread bucket-range sums of the scan
+  // host, one value per CTA: the range of its candidates, its part of the threshold search, its best draw
+  uint32_t slot_lo[kTopPCtas], slot_hi[kTopPCtas], slot_r[kTopPCtas], slot_f[kTopPCtas], slot_g[kTopPCtas],
+      slot_i[kTopPCtas];
   float lvl_hi[kTopPLevels];
   float lvl_scale[kTopPLevels];
   int lvl_b[kTopPLevels];
   unsigned long long ra[kTopPWarps];
   float rf[kTopPWarps], rg[kTopPWarps];
   int ri[kTopPWarps];
-  unsigned long long cum_before, target;   // host, copied to every CTA
-  unsigned ncand;                          // host
-  unsigned lcand, lbase;                   // this CTA's candidate count and its offset at the host
-  float lse, y0, ystar;
-  int nlvl;
-  int mode;  // 0 histogram, 1 resolve the gathered candidates, 2 threshold known
+  unsigned long long cum_before;            // host, copied to every CTA
+  unsigned ncand;                           // host: the reservation counter; every CTA: the cluster's count
+  unsigned lcand, lbase;                    // this CTA's candidate count and its offset in the cluster's list
+  float ystar;
+  int full;                                 // the threshold is known but the candidates did not all fit
 };
 
 // Probability of tempered logit y in 2^-40 units, truncated toward zero: the
@@ -90,6 +97,18 @@ __device__ __forceinline__ unsigned long long top_p_mass(float y, float lse) {
   return e >= 0 ? m << e : m >> (-e);
 }
 
+// Adds q to a 64-bit histogram bucket with 32-bit shared atomics: q's low word
+// into the bucket's low word, then its high word plus the carry out of that
+// add (the old low word plus q's low word wrapped) into the high word.  The
+// bucket ends as the exact sum whatever the order of the adds.
+__device__ __forceinline__ void top_p_hist_add(unsigned long long* h, unsigned long long q) {
+  unsigned* w = reinterpret_cast<unsigned*>(h);  // little-endian: w[0] is the low word
+  const unsigned lo = static_cast<unsigned>(q);
+  const unsigned old = atomicAdd(w, lo);
+  const unsigned hi = static_cast<unsigned>(q >> 32) + (old + lo < old ? 1u : 0u);
+  if (hi) atomicAdd(w + 1, hi);
+}
+
 __device__ __forceinline__ int top_p_bucket(float y, float hi, float scale) {
   return static_cast<int>(fminf(fmaxf((hi - y) * scale, 0.f), static_cast<float>(kTopPBuckets - 1)));
 }
@@ -99,6 +118,17 @@ __device__ __forceinline__ bool top_p_in(const TopPShared& sh, float y, int n) {
   for (int l = 0; l < n; ++l)
     if (top_p_bucket(y, sh.lvl_hi[l], sh.lvl_scale[l]) != sh.lvl_b[l]) return false;
   return true;
+}
+
+// Where y lies against the chosen buckets of the first n levels: 2 in all of
+// them (a candidate), 1 above one of them (above the threshold, which lies in
+// the chosen bucket; the bucket index never increases with y), 0 below.
+__device__ __forceinline__ int top_p_class(const TopPShared& sh, float y, int n) {
+  for (int l = 0; l < n; ++l) {
+    const int b = top_p_bucket(y, sh.lvl_hi[l], sh.lvl_scale[l]);
+    if (b != sh.lvl_b[l]) return b < sh.lvl_b[l] ? 1 : 0;
+  }
+  return 2;
 }
 
 // The mass the nucleus must reach, in the units of top_p_mass: top_p of the
@@ -124,112 +154,59 @@ __device__ __forceinline__ float top_p_block_max(TopPShared& sh, float v) {
   return r;
 }
 
-// Walks this CTA's share of the row (kShare CTAs share it; rank is this
-// CTA's place among them): groups of four logits (16-byte loads; the row's
-// leading dimension is a multiple of 64, so a group never leaves the row's
-// storage) g = rank * kTopPThreads + tid + k * kShare * kTopPThreads, kUnroll
-// groups per thread in flight; f(v, y) for every v < V.
-template <int kUnroll, int kShare = kTopPCtas, typename F>
-__device__ __forceinline__ void top_p_walk(const float* zr, int V, float inv_temp, int rank, F f) {
-  constexpr int kStride = kShare * kTopPThreads;
+// Walks this CTA's share of the row: groups of four logits (16-byte loads; the
+// row's leading dimension is a multiple of 64, so a group never leaves the
+// row's storage) g = rank * kTopPThreads + tid + k * kTopPCtas * kTopPThreads,
+// up to kUnroll groups per thread loaded together (the last round predicated),
+// then f(g, q) for each.  Lanes of a partial last group past V are the
+// caller's to skip.
+template <int kUnroll, typename F>
+__device__ __forceinline__ void top_p_groups(const float* zr, int V, int rank, F f) {
+  constexpr int kStride = kTopPCtas * kTopPThreads;
   const int groups = (V + 3) / 4;
   const float4* zq = reinterpret_cast<const float4*>(zr);
-  int g0 = rank * kTopPThreads + threadIdx.x;
-  // whole rounds: kUnroll unconditional loads in flight, then their logits
-  for (; g0 + (kUnroll - 1) * kStride < groups - 1; g0 += kUnroll * kStride) {
+  for (int g0 = rank * kTopPThreads + static_cast<int>(threadIdx.x); g0 < groups; g0 += kUnroll * kStride) {
     float4 q[kUnroll];
 #pragma unroll
-    for (int u = 0; u < kUnroll; ++u) q[u] = __ldcg(zq + g0 + u * kStride);
+    for (int u = 0; u < kUnroll; ++u) {
+      const int g = g0 + u * kStride;
+      q[u] = g < groups ? __ldcg(zq + g) : make_float4(0.f, 0.f, 0.f, 0.f);
+    }
 #pragma unroll
     for (int u = 0; u < kUnroll; ++u) {
-      const int v = 4 * (g0 + u * kStride);  // every group here lies below the last, so v + 3 < V
-      f(v, q[u].x * inv_temp);
-      f(v + 1, q[u].y * inv_temp);
-      f(v + 2, q[u].z * inv_temp);
-      f(v + 3, q[u].w * inv_temp);
+      const int g = g0 + u * kStride;
+      if (g < groups) f(g, q[u]);
     }
   }
-  // the rest, one group at a time (the last group may be partial)
-  for (; g0 < groups; g0 += kStride) {
-    const float4 q = __ldcg(zq + g0);
-    const int v = 4 * g0;
-    const float zz[4] = {q.x, q.y, q.z, q.w};
-#pragma unroll
-    for (int k = 0; k < 4; ++k)
-      if (v + k < V) f(v + k, zz[k] * inv_temp);
-  }
-}
-
-// The threshold among the nc gathered candidates (host CTA, every thread; the
-// result in every thread): the candidates sorted by y, largest first (bitonic
-// sort, padded to a power of two with -inf), their masses summed in that order
-// (fixed-order block scan); y* is the y at the first position where the mass
-// above the bucket plus the running sum reaches the target.  Equal logits sit
-// next to each other, so y*'s whole tie group counts toward the target.
-// -inf if no position does (the nucleus is then the whole vocabulary).
-__device__ __forceinline__ float top_p_resolve(TopPShared& sh, int nc) {
-  const int tid = threadIdx.x;
-  int n = 1;
-  while (n < nc) n <<= 1;  // <= kTopPCand
-  for (int i = nc + tid; i < n; i += kTopPThreads) {
-    sh.cy[i] = -INFINITY;
-    sh.cq[i] = 0ull;
-  }
-  __syncthreads();
-  for (int k = 2; k <= n; k <<= 1) {
-    for (int j = k >> 1; j > 0; j >>= 1) {
-      for (int i = tid; i < n; i += kTopPThreads) {
-        const int l = i ^ j;
-        if (l > i) {
-          const float a = sh.cy[i], b = sh.cy[l];
-          if ((i & k) == 0 ? a < b : a > b) {  // descending runs where bit k is clear
-            sh.cy[i] = b;
-            sh.cy[l] = a;
-            const unsigned long long t = sh.cq[i];
-            sh.cq[i] = sh.cq[l];
-            sh.cq[l] = t;
-          }
-        }
-      }
-      __syncthreads();
-    }
-  }
-  // running sums: thread tid owns positions [tid * per, (tid + 1) * per)
-  const int per = (n + kTopPThreads - 1) / kTopPThreads;
-  const int b0 = tid * per;
-  unsigned long long own = 0ull;
-  for (int i = b0; i < b0 + per && i < n; ++i) own += sh.cq[i];
-  unsigned long long inc = own;
-#pragma unroll
-  for (int o = 1; o < 32; o <<= 1) {
-    const unsigned long long v = __shfl_up_sync(0xffffffffu, inc, o);
-    if ((tid & 31) >= o) inc += v;
-  }
-  if ((tid & 31) == 31) sh.ra[tid >> 5] = inc;
-  __syncthreads();
-  unsigned long long acc = inc - own;
-  for (int w = 0; w < (tid >> 5); ++w) acc += sh.ra[w];
-  const unsigned long long need = sh.target - sh.cum_before;
-  int first = n;
-  for (int i = b0; i < b0 + per && i < n; ++i) {
-    acc += sh.cq[i];
-    if (acc >= need) {
-      first = i;
-      break;
-    }
-  }
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) first = min(first, __shfl_xor_sync(0xffffffffu, first, o));
-  __syncthreads();
-  if ((tid & 31) == 0) sh.ri[tid >> 5] = first;
-  __syncthreads();
-  for (int w = 0; w < kTopPWarps; ++w) first = min(first, sh.ri[w]);
-  return first < n ? sh.cy[first] : -INFINITY;
 }
 
 // The better of two perturbed scores (the lower token on a tie; -1 loses).
 __device__ __forceinline__ bool top_p_better(float s, int v, float s0, int v0) {
   return s > s0 || (s == s0 && v >= 0 && (v0 < 0 || v < v0));
+}
+
+// This CTA's part of the threshold search over the nc gathered candidates:
+// y* is the largest candidate y whose mass M(y) = sum of q_j over the
+// candidates with y_j >= y reaches `need` (the first position, largest y
+// first, where the running sum reaches need: the running sum at the end of
+// y's group of equal logits is M(y), and it grows down the list).  The CTA
+// takes the candidates [rank * per, (rank + 1) * per), tpi threads each
+// (a power of two, so a candidate's threads share a warp); returns the
+// largest qualifying y of its candidates in every thread, -inf if none.
+__device__ __forceinline__ float top_p_rank_slice(TopPShared& sh, int nc, int rank, unsigned long long need) {
+  const int per = (nc + kTopPCtas - 1) / kTopPCtas;  // <= kTopPCand / kTopPCtas = 128
+  int tpi = 32;
+  while (tpi > 1 && per * tpi > kTopPThreads) tpi >>= 1;
+  const int k = static_cast<int>(threadIdx.x) / tpi;
+  const int i = rank * per + k;
+  const bool act = k < per && i < nc;
+  const float yi = act ? sh.cy[i] : INFINITY;
+  unsigned long long m = 0ull;
+  if (act)
+    for (int j = static_cast<int>(threadIdx.x) & (tpi - 1); j < nc; j += tpi)
+      if (sh.cy[j] >= yi) m += sh.cq[j];
+  for (int o = tpi >> 1; o > 0; o >>= 1) m += __shfl_xor_sync(0xffffffffu, m, o);
+  return top_p_block_max(sh, act && m >= need ? yi : -INFINITY);
 }
 
 __global__ void __cluster_dims__(kTopPCtas, 1, 1) __launch_bounds__(kTopPThreads, 4)
@@ -244,38 +221,47 @@ __global__ void __cluster_dims__(kTopPCtas, 1, 1) __launch_bounds__(kTopPThreads
   const int rank = static_cast<int>(cluster_ctarank());
   const bool host = rank == 0;
   const int ns = *n_slow;
-  // CTA 0's copy of a field
-  auto at0 = [&](const void* p) { return mapa_shared(smem_addr(p), 0); };
+  // CTA k's copy of a field
+  auto atk = [&](const void* p, int k) { return mapa_shared(smem_addr(p), static_cast<uint32_t>(k)); };
   for (int si = blockIdx.x / kTopPCtas; si < ns; si += gridDim.x / kTopPCtas) {
     const int r = slow_rows[si];
     const float* zr = z + static_cast<int64_t>(r) * ldz;
     const int t = cidx[r];
+    const float lse = lse_r[r], y0 = y0_r[r];
+    const unsigned long long target = slow_target[si];
     if (tid == 0) {
-      sh.lse = lse_r[r];
-      sh.y0 = y0_r[r];
-      sh.target = slow_target[si];
-      sh.lvl_hi[0] = hi_r[r];  // the row maximum of y (to rounding): the top of the first level
-    }
-    if (tid == 0) {
-      sh.nlvl = 0;
+      // the first level spans the logits above the plain winner (y* > y0: the
+      // mass above y0 reaches the target), at most 1/64 nat a bucket
+      const float hi = hi_r[r];  // the row maximum of y (to rounding)
+      sh.lvl_hi[0] = hi;
+      sh.lvl_scale[0] = hi > y0 ? fminf(fmaxf(64.f, static_cast<float>(kTopPBuckets - 1) / (hi - y0)), 1e30f) : 64.f;
       sh.cum_before = 0ull;
-      sh.ystar = -INFINITY;
-      sh.mode = 0;
-      sh.lvl_scale[0] = 64.f;
+      sh.full = 0;
     }
-    __syncthreads();
-    const float lse = sh.lse;
-    while (sh.mode == 0) {
-      const int L = sh.nlvl;
+    // Each level: histogram the mass of the logits above y0 that lie in the
+    // chosen buckets of the levels before; pick the bucket where the mass from
+    // the top reaches the target; gather that bucket's logits as candidates
+    // and, on the way, draw over the logits above it (all in the nucleus).
+    float bs = -INFINITY, by = 0.f;  // this thread's best perturbed score, its token and logit
+    int bv = -1;
+    int L = 0;
+    for (;;) {
+      __syncthreads();
       for (int b = tid; b < kTopPBuckets; b += kTopPThreads) sh.hist[b] = 0ull;
       __syncthreads();
-      const float hi = sh.lvl_hi[L], scale = sh.lvl_scale[L];
-      top_p_walk<4>(zr, V, inv_temp, rank, [&](int, float y) {
-        if (top_p_in(sh, y, L)) {
-          const unsigned long long q = top_p_mass(y, lse);
-          if (q) atomicAdd(&sh.hist[top_p_bucket(y, hi, scale)], q);  // far-tail logits add nothing
-        }
-      });
+      {
+        const float hi = sh.lvl_hi[L], scale = sh.lvl_scale[L];
+        top_p_groups<8>(zr, V, rank, [&](int g, float4 q) {
+          const float yy[4] = {q.x * inv_temp, q.y * inv_temp, q.z * inv_temp, q.w * inv_temp};
+#pragma unroll
+          for (int k = 0; k < 4; ++k) {
+            if (4 * g + k < V && yy[k] > y0 && top_p_in(sh, yy[k], L)) {
+              const unsigned long long m = top_p_mass(yy[k], lse);
+              if (m) top_p_hist_add(&sh.hist[top_p_bucket(yy[k], hi, scale)], m);  // far tail adds nothing
+            }
+          }
+        });
+      }
       cluster_sync();
       {  // merge the histograms: CTA k sums buckets [k * kTopPThreads, (k + 1) * kTopPThreads) over
          // the cluster in rank order and leaves the sums in CTA 0's histogram (disjoint slices, so no
@@ -283,11 +269,11 @@ __global__ void __cluster_dims__(kTopPCtas, 1, 1) __launch_bounds__(kTopPThreads
         const int b = rank * kTopPThreads + tid;
         unsigned long long part[kTopPCtas];
 #pragma unroll
-        for (int k = 0; k < kTopPCtas; ++k) part[k] = ld_shared_cluster_u64(mapa_shared(smem_addr(&sh.hist[b]), k));
+        for (int k = 0; k < kTopPCtas; ++k) part[k] = ld_shared_cluster_u64(atk(&sh.hist[b], k));
         unsigned long long m = 0ull;
 #pragma unroll
         for (int k = 0; k < kTopPCtas; ++k) m += part[k];
-        st_shared_cluster_u64(at0(&sh.hist[b]), m);
+        st_shared_cluster_u64(atk(&sh.hist[b], 0), m);
       }
       cluster_sync();
       if (host) {  // find the bucket that holds the threshold
@@ -313,7 +299,7 @@ __global__ void __cluster_dims__(kTopPCtas, 1, 1) __launch_bounds__(kTopPThreads
             const unsigned long long n = __shfl_up_sync(0xffffffffu, inc, o);
             if (tid >= o) inc += n;
           }
-          const unsigned cross = __ballot_sync(0xffffffffu, sh.cum_before + inc >= sh.target);
+          const unsigned cross = __ballot_sync(0xffffffffu, sh.cum_before + inc >= target);
           const int ln = cross ? __ffs(cross) - 1 : 31;
           const unsigned long long before = __shfl_sync(0xffffffffu, inc - own, ln);
           sh.ra[0] = before;
@@ -325,12 +311,12 @@ __global__ void __cluster_dims__(kTopPCtas, 1, 1) __launch_bounds__(kTopPThreads
           unsigned long long acc = sh.cum_before + sh.ra[0];
           int seg = sh.ri[0] * kSeg;
           for (; seg < (sh.ri[0] + 1) * kSeg - 1; ++seg) {
-            if (acc + sh.scan[seg] >= sh.target) break;
+            if (acc + sh.scan[seg] >= target) break;
             acc += sh.scan[seg];
           }
           int b = seg * kPer;
           for (; b < (seg + 1) * kPer - 1; ++b) {
-            if (acc + sh.hist[b] >= sh.target) break;
+            if (acc + sh.hist[b] >= target) break;
             acc += sh.hist[b];
           }
           sh.cum_before = acc;
@@ -340,89 +326,131 @@ __global__ void __cluster_dims__(kTopPCtas, 1, 1) __launch_bounds__(kTopPThreads
       }
       cluster_sync();
       if (tid == 0) {
-        sh.lvl_b[L] = static_cast<int>(ld_shared_cluster(at0(&sh.lvl_b[L])));
-        sh.cum_before = ld_shared_cluster_u64(at0(&sh.cum_before));
-        sh.nlvl = L + 1;
+        if (!host) {
+          sh.lvl_b[L] = static_cast<int>(ld_shared_cluster(atk(&sh.lvl_b[L], 0)));
+          sh.cum_before = ld_shared_cluster_u64(atk(&sh.cum_before, 0));
+        }
+        sh.lcand = 0u;
       }
       __syncthreads();
-      // gather the bucket's logits (and their range, in case they do not fit):
-      // into this CTA's buffer first, then one reservation at the host and a copy
-      if (tid == 0) sh.lcand = 0u;
-      __syncthreads();
+      // gather the bucket's logits (and their range, in case they do not fit)
+      // into this CTA's list; draw over the logits above the bucket (Gumbel-max
+      // with the GEMM's noise: Philox4x32-10 word v mod 4 of counter
+      // (v div 4, t, offset), fp32 operations; along a thread's walk v grows, so
+      // a strict > keeps the lowest v of equal scores)
       float lo = INFINITY, hi2 = -INFINITY;
-      top_p_walk<4>(zr, V, inv_temp, rank, [&](int, float y) {
-        if (top_p_in(sh, y, L + 1)) {
-          lo = fminf(lo, y);
-          hi2 = fmaxf(hi2, y);
-          const unsigned i = atomicAdd(&sh.lcand, 1u);
-          if (i < static_cast<unsigned>(kTopPCand)) {
-            sh.ly[i] = y;
-            sh.lq[i] = top_p_mass(y, lse);
+      bs = -INFINITY;
+      bv = -1;
+      by = 0.f;
+      top_p_groups<4>(zr, V, rank, [&](int g, float4 q) {
+        const float yy[4] = {q.x * inv_temp, q.y * inv_temp, q.z * inv_temp, q.w * inv_temp};
+        int cls[4];
+        bool above = false;
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+          cls[k] = 4 * g + k < V && yy[k] > y0 ? top_p_class(sh, yy[k], L + 1) : 0;
+          above |= cls[k] == 1;
+        }
+        if (above) {
+          const uint4 w = philox4x32_10(make_uint4(static_cast<uint32_t>(g), static_cast<uint32_t>(t), off_lo, off_hi),
+                                        seed_lo, seed_hi);
+          const uint32_t ws[4] = {w.x, w.y, w.z, w.w};
+#pragma unroll
+          for (int k = 0; k < 4; ++k) {
+            if (cls[k] == 1) {
+              const float sc = yy[k] + gumbel_of(ws[k]);
+              if (sc > bs) {
+                bs = sc;
+                bv = 4 * g + k;
+                by = yy[k];
+              }
+            }
+          }
+        }
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+          if (cls[k] == 2) {
+            lo = fminf(lo, yy[k]);
+            hi2 = fmaxf(hi2, yy[k]);
+            const unsigned i = atomicAdd(&sh.lcand, 1u);
+            if (i < static_cast<unsigned>(kTopPCand)) {
+              sh.loc.y[i] = yy[k];
+              sh.loc.v[i] = 4 * g + k;
+            }
           }
         }
       });
       lo = -top_p_block_max(sh, -lo);
       hi2 = top_p_block_max(sh, hi2);
       if (tid == 0) {
-        st_shared_cluster(at0(&sh.slot_f[rank]), __float_as_uint(lo));
-        st_shared_cluster(at0(&sh.slot_g[rank]), __float_as_uint(hi2));
-        sh.lbase = atom_add_shared_cluster(at0(&sh.ncand), sh.lcand);
+        st_shared_cluster(atk(&sh.slot_lo[rank], 0), __float_as_uint(lo));
+        st_shared_cluster(atk(&sh.slot_hi[rank], 0), __float_as_uint(hi2));
+        sh.lbase = atom_add_shared_cluster(atk(&sh.ncand, 0), sh.lcand);
       }
       __syncthreads();
-      {
+      {  // this CTA's candidates into every CTA's list, at the offset it reserved
         const unsigned n = min(sh.lcand, static_cast<unsigned>(kTopPCand));
         const unsigned base = sh.lbase;
         for (unsigned i = tid; i < n && base + i < static_cast<unsigned>(kTopPCand); i += kTopPThreads) {
-          st_shared_cluster(at0(&sh.cy[base + i]), __float_as_uint(sh.ly[i]));
-          st_shared_cluster_u64(at0(&sh.cq[base + i]), sh.lq[i]);
+          const float y = sh.loc.y[i];
+          const unsigned long long m = top_p_mass(y, lse);
+          const int v = sh.loc.v[i];
+#pragma unroll
+          for (int k = 0; k < kTopPCtas; ++k) {
+            st_shared_cluster(atk(&sh.cy[base + i], k), __float_as_uint(y));
+            st_shared_cluster_u64(atk(&sh.cq[base + i], k), m);
+            st_shared_cluster(atk(&sh.cv[base + i], k), static_cast<uint32_t>(v));
+          }
         }
       }
       cluster_sync();
-      if (host) {
-        const int nc = static_cast<int>(min(sh.ncand, static_cast<unsigned>(kTopPCand)));
-        if (sh.ncand <= static_cast<unsigned>(kTopPCand)) {
-          const float best = top_p_resolve(sh, nc);
-          if (tid == 0) {
-            sh.ystar = best;
-            sh.mode = 2;
-          }
-        } else if (tid == 0) {
+      if (tid == 0) {
+        if (!host) sh.ncand = ld_shared_cluster(atk(&sh.ncand, 0));
+        if (sh.ncand > static_cast<unsigned>(kTopPCand)) {
+          // too many to resolve here: every CTA reads the bucket's range and
+          // decides alike whether to histogram it once more
           float l = INFINITY, h = -INFINITY;
           for (int k = 0; k < kTopPCtas; ++k) {
-            l = fminf(l, __uint_as_float(sh.slot_f[k]));
-            h = fmaxf(h, __uint_as_float(sh.slot_g[k]));
+            l = fminf(l, __uint_as_float(ld_shared_cluster(atk(&sh.slot_lo[k], 0))));
+            h = fmaxf(h, __uint_as_float(ld_shared_cluster(atk(&sh.slot_hi[k], 0))));
           }
           if (!(h > l) || L + 1 >= kTopPLevels) {
             sh.ystar = l;  // all equal (or out of levels: the whole bucket)
-            sh.mode = 2;
-            if (h > l) atomicOr(status, kDevNonFinite);
+            sh.full = 1;
+            if (host && h > l) atomicOr(status, kDevNonFinite);
           } else {
             sh.lvl_hi[L + 1] = h;
             sh.lvl_scale[L + 1] = static_cast<float>(kTopPBuckets - 1) / (h - l);
           }
         }
       }
-      cluster_sync();
-      if (tid == 0) {
-        sh.mode = static_cast<int>(ld_shared_cluster(at0(&sh.mode)));
-        sh.ystar = __uint_as_float(ld_shared_cluster(at0(&sh.ystar)));
-        sh.lvl_hi[L + 1 < kTopPLevels ? L + 1 : L] =
-            __uint_as_float(ld_shared_cluster(at0(&sh.lvl_hi[L + 1 < kTopPLevels ? L + 1 : L])));
-        sh.lvl_scale[L + 1 < kTopPLevels ? L + 1 : L] =
-            __uint_as_float(ld_shared_cluster(at0(&sh.lvl_scale[L + 1 < kTopPLevels ? L + 1 : L])));
-      }
       __syncthreads();
+      const int nc = static_cast<int>(sh.ncand);
+      if (nc <= kTopPCand) {
+        const float c = top_p_rank_slice(sh, nc, rank, target - sh.cum_before);
+        if (tid == 0) st_shared_cluster(atk(&sh.slot_r[rank], 0), __float_as_uint(c));
+        cluster_sync();
+        if (tid == 0) {
+          float ys = -INFINITY;
+          for (int k = 0; k < kTopPCtas; ++k) ys = fmaxf(ys, __uint_as_float(ld_shared_cluster(atk(&sh.slot_r[k], 0))));
+          sh.ystar = ys;
+          sh.full = ys == -INFINITY;  // no crossing (the masses fell short): the whole vocabulary
+        }
+        __syncthreads();
+        break;
+      }
+      if (sh.full) break;
+      ++L;
     }
     const float ystar = sh.ystar;
-    {  // the plain winner is outside the nucleus: the argmax over it
-      // Gumbel-max over y >= y*, the lowest v on ties
-      float bs = -INFINITY, by = 0.f;
-      int bv = -1;
-      const int groups = (V + 3) / 4;
-      for (int g = rank * kTopPThreads + tid; g < groups; g += kTopPCtas * kTopPThreads) {
-        const float4 q = __ldcg(reinterpret_cast<const float4*>(zr) + g);
+    if (sh.full) {
+      // the candidates are not all at hand: Gumbel-max over every y >= y*
+      bs = -INFINITY;
+      bv = -1;
+      by = 0.f;
+      top_p_groups<4>(zr, V, rank, [&](int g, float4 q) {
         const float yy[4] = {q.x * inv_temp, q.y * inv_temp, q.z * inv_temp, q.w * inv_temp};
-        if (!(yy[0] >= ystar || yy[1] >= ystar || yy[2] >= ystar || yy[3] >= ystar)) continue;
+        if (!(yy[0] >= ystar || yy[1] >= ystar || yy[2] >= ystar || yy[3] >= ystar)) return;
         const uint4 w = philox4x32_10(make_uint4(static_cast<uint32_t>(g), static_cast<uint32_t>(t), off_lo, off_hi),
                                       seed_lo, seed_hi);
         const uint32_t ws[4] = {w.x, w.y, w.z, w.w};
@@ -430,64 +458,85 @@ __global__ void __cluster_dims__(kTopPCtas, 1, 1) __launch_bounds__(kTopPThreads
         for (int k = 0; k < 4; ++k) {
           const int v = 4 * g + k;
           if (v < V && yy[k] >= ystar) {
-            const float sc2 = yy[k] + gumbel_of(ws[k]);
-            if (sc2 > bs) {
-              bs = sc2;
+            const float sc = yy[k] + gumbel_of(ws[k]);
+            if (sc > bs) {
+              bs = sc;
               bv = v;
               by = yy[k];
             }
           }
         }
+      });
+    } else {
+      // the candidates at or above y*, this CTA's share of them
+      const int nc = static_cast<int>(sh.ncand);
+      for (int i = rank + kTopPCtas * tid; i < nc; i += kTopPCtas * kTopPThreads) {
+        const float y = sh.cy[i];
+        if (y >= ystar) {
+          const int v = sh.cv[i];
+          const uint4 w = philox4x32_10(
+              make_uint4(static_cast<uint32_t>(v >> 2), static_cast<uint32_t>(t), off_lo, off_hi), seed_lo, seed_hi);
+          const uint32_t ws[4] = {w.x, w.y, w.z, w.w};
+          const float sc = y + gumbel_of(ws[v & 3]);
+          if (top_p_better(sc, v, bs, bv)) {
+            bs = sc;
+            bv = v;
+            by = y;
+          }
+        }
       }
+    }
 #pragma unroll
-      for (int o = 16; o > 0; o >>= 1) {
-        const float os = __shfl_xor_sync(0xffffffffu, bs, o);
-        const int ov = __shfl_xor_sync(0xffffffffu, bv, o);
-        const float oy = __shfl_xor_sync(0xffffffffu, by, o);
+    for (int o = 16; o > 0; o >>= 1) {
+      const float os = __shfl_xor_sync(0xffffffffu, bs, o);
+      const int ov = __shfl_xor_sync(0xffffffffu, bv, o);
+      const float oy = __shfl_xor_sync(0xffffffffu, by, o);
+      if (top_p_better(os, ov, bs, bv)) {
+        bs = os;
+        bv = ov;
+        by = oy;
+      }
+    }
+    __syncthreads();
+    if ((tid & 31) == 0) {
+      sh.rf[tid >> 5] = bs;
+      sh.ri[tid >> 5] = bv;
+      sh.rg[tid >> 5] = by;
+    }
+    __syncthreads();
+    if (tid == 0) {
+      for (int i = 1; i < kTopPWarps; ++i)
+        if (top_p_better(sh.rf[i], sh.ri[i], bs, bv)) {
+          bs = sh.rf[i];
+          bv = sh.ri[i];
+          by = sh.rg[i];
+        }
+      st_shared_cluster(atk(&sh.slot_f[rank], 0), __float_as_uint(bs));
+      st_shared_cluster(atk(&sh.slot_g[rank], 0), __float_as_uint(by));
+      st_shared_cluster(atk(&sh.slot_i[rank], 0), static_cast<uint32_t>(bv));
+    }
+    cluster_sync();
+    if (host && tid == 0) {
+      bs = -INFINITY;
+      bv = -1;
+      by = 0.f;
+      for (int k = 0; k < kTopPCtas; ++k) {
+        const float os = __uint_as_float(sh.slot_f[k]);
+        const int ov = static_cast<int>(sh.slot_i[k]);
         if (top_p_better(os, ov, bs, bv)) {
           bs = os;
           bv = ov;
-          by = oy;
+          by = __uint_as_float(sh.slot_g[k]);
         }
       }
-      __syncthreads();
-      if ((tid & 31) == 0) {
-        sh.rf[tid >> 5] = bs;
-        sh.ri[tid >> 5] = bv;
-        sh.rg[tid >> 5] = by;
-      }
-      __syncthreads();
-      if (tid == 0) {
-        for (int i = 1; i < kTopPWarps; ++i)
-          if (top_p_better(sh.rf[i], sh.ri[i], bs, bv)) {
-            bs = sh.rf[i];
-            bv = sh.ri[i];
-            by = sh.rg[i];
-          }
-        st_shared_cluster(at0(&sh.slot_f[rank]), __float_as_uint(bs));
-        st_shared_cluster(at0(&sh.slot_g[rank]), __float_as_uint(by));
-        st_shared_cluster(at0(&sh.slot_i[rank]), static_cast<uint32_t>(bv));
-      }
-      cluster_sync();
-      if (host && tid == 0) {
-        bs = -INFINITY;
-        bv = -1;
-        by = 0.f;
-        for (int k = 0; k < kTopPCtas; ++k) {
-          const float os = __uint_as_float(sh.slot_f[k]);
-          const int ov = static_cast<int>(sh.slot_i[k]);
-          if (top_p_better(os, ov, bs, bv)) {
-            bs = os;
-            bv = ov;
-            by = __uint_as_float(sh.slot_g[k]);
-          }
-        }
-        if (!isfinite(lse) || bv < 0) atomicOr(status, kDevNonFinite);
-        tokens[t] = bv;
-        logp[t] = by - lse;
-      }
+      if (!isfinite(lse) || bv < 0) atomicOr(status, kDevNonFinite);
+      tokens[t] = bv;
+      logp[t] = by - lse;
     }
-    cluster_sync();  // the host's slots are free again before the next row
+    // No barrier before the next row: the host's slots are written again only
+    // after the next row's third cluster barrier, which the host reaches after
+    // reading them here; nothing else of another CTA is touched after the one
+    // above.
   }
 }
 
