@@ -1,6 +1,11 @@
 """Host logic of bench.py on CPU: the roofline of the dominant kernel from a
 launch trace, the HBM figures of the element-wise passes, and the lookup of
 stored DRAM traffic.  (The device-timed run itself needs a GPU.)"""
+import json
+import os
+import subprocess
+import sys
+
 import pytest
 
 import bench
@@ -66,3 +71,26 @@ def test_stored_traffic_is_scaled_to_the_launch_and_keyed_by_source():
     rf = bench.roofline(tr, N, HD, 1, 1724.3, "x", "fwdbwd_8b", 6678.5)
     assert rf["traffic"] == pytest.approx(bytes_ref * (V / 10) / cols_ref, rel=1e-9)
     assert bench.stored_traffic("fwdbwd_8b", "no_such_kernel") is None
+
+
+def test_reference_arm_prints_one_contract_line():
+    """bench.py --impl reference: the float64 oracle on the host cores prints
+    one JSON line with the contract's keys on rank 0; another rank prints
+    nothing and exits 0."""
+    cmd = [sys.executable, os.path.join(bench.ROOT, "bench.py"), "--impl", "reference", "--workload", "tiny_fwdbwd",
+           "--steps", "2", "--warmup", "1", "--cpu-sample-tokens", "64"]
+    env = {k: v for k, v in os.environ.items() if k not in ("RANK", "WORLD_SIZE", "LOCAL_RANK")}
+    out = subprocess.run(cmd, capture_output=True, text=True, timeout=300, cwd=bench.ROOT, env=env)
+    assert out.returncode == 0, out.stderr
+    lines = [ln for ln in out.stdout.splitlines() if ln.startswith("{")]
+    assert len(lines) == 1
+    d = json.loads(lines[0])
+    assert d["impl"] == "reference" and d["metric"] == bench.METRIC and d["unit"] == "tokens/s"
+    assert d["value"] > 0 and d["steps"] == 2 and d["warmup"] == 1 and d["higher_is_better"] is True
+    assert d["dtype"] == "f64" and d["config"]["workload"] == "tiny_fwdbwd"
+    cb = d["cpu_baseline"]
+    assert cb["kind"] == "oracle" and cb["value"] == d["value"] and cb["cores"] >= 1 and cb["sample"]
+    assert d["e2e"] == {"value": d["value"], "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}
+    out = subprocess.run(cmd, capture_output=True, text=True, timeout=300, cwd=bench.ROOT, env=dict(env, RANK="1"))
+    assert out.returncode == 0, out.stderr
+    assert not [ln for ln in out.stdout.splitlines() if ln.startswith("{")]
