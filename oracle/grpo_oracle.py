@@ -120,6 +120,20 @@ def token_logprobs(H, W, targets, mask, vocab_chunk: int = 8192, row_chunk: int 
     return logp, lse
 
 
+def target_logits(H, W, targets, rows, row_chunk: int = 16384) -> np.ndarray:
+    """z_{t, y_t} = H_t . W_{y_t} in float64 for the listed rows: the logit of
+    the sampled token, from which logp_t = z_{t, y_t} - LSE_t (Eq. 1's
+    pi_theta at o_{i,t}) once the row's log-sum-exp is known."""
+    rows = np.asarray(rows, dtype=np.int64)
+    y = np.asarray(targets, dtype=np.int64)
+    Hs, Ws = np.asarray(H), np.asarray(W)
+    out = np.empty(rows.size)
+    for a in range(0, rows.size, row_chunk):
+        r = rows[a:a + row_chunk]
+        out[a:a + r.size] = np.einsum("ij,ij->i", as_f64(Hs[r]), as_f64(Ws[y[r]]))
+    return out
+
+
 # ---------------------------------------------------------------------------
 # Eq. 1: per-token terms, weights, loss and its derivative in logp
 # ---------------------------------------------------------------------------

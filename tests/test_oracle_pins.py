@@ -9,6 +9,7 @@ import json
 import math
 import os
 import statistics
+import struct
 
 import numpy as np
 import pytest
@@ -108,6 +109,29 @@ def test_logprobs_match_bruteforce_and_scipy():
     np.testing.assert_allclose(logp[m], ls[m], rtol=0, atol=1e-12)
     np.testing.assert_allclose(lse[m], scipy.special.logsumexp(Z, axis=1)[m], rtol=0, atol=1e-12)
     assert np.all(logp[~m] == 0) and np.all(lse[~m] == 0)
+
+
+def test_target_logits_match_explicit_sums_and_logp_plus_lse():
+    """z_{t,y_t} against dot products written out in pure Python (bf16 inputs
+    widened bit by bit), and logp_t = z_{t,y_t} - LSE_t against brute force."""
+    rng = np.random.default_rng(17)
+    T, Hd, V = 9, 7, 13
+    Hb = rng.integers(0, 1 << 16, (T, Hd), dtype=np.uint16) & np.uint16(0xBFFF)   # finite bf16 bit patterns
+    Wb = rng.integers(0, 1 << 16, (V, Hd), dtype=np.uint16) & np.uint16(0xBFFF)
+    y = rng.integers(0, V, T)
+    rows = np.array([0, 3, 4, 8])
+
+    def bits(b):
+        return struct.unpack("<f", struct.pack("<I", int(b) << 16))[0]
+    want = [math.fsum(bits(Hb[t, k]) * bits(Wb[y[t], k]) for k in range(Hd)) for t in rows]
+    np.testing.assert_allclose(oracle.target_logits(Hb, Wb, y, rows), want, rtol=1e-13, atol=0)
+    c = _rand_case(3, T_resp=2, G=2, L=4, Hd=5, V=9, scale=1.2)
+    m = c["mask"] != 0
+    logp, lse = oracle.token_logprobs(c["H"], c["W"], c["y"], c["mask"])
+    idx = np.flatnonzero(m)
+    bf = np.array(brute.logprobs(c["H"].tolist(), c["W"].tolist(), c["y"].tolist(), c["mask"].tolist()))
+    np.testing.assert_allclose(oracle.target_logits(c["H"], c["W"], c["y"], idx) - lse[idx], bf[idx],
+                               rtol=0, atol=1e-12)
 
 
 def test_logprobs_chunking_invariant_and_large_logits():
@@ -478,6 +502,54 @@ def test_top_p_draws_follow_the_truncated_softmax():
     assert np.all(tok == np.argmax(z))
 
 
+def _nucleus_threshold_by_search(y, mass):
+    """The nucleus threshold for a target mass: the highest distinct logit
+    whose upper set carries at least `mass` of softmax(y) (explicit sums);
+    the lowest logit when no threshold reaches it."""
+    p = [math.exp(v) for v in y]
+    total = math.fsum(p)
+    for thr in sorted(set(y), reverse=True):
+        if math.fsum(pv for pv, v in zip(p, y) if v >= thr) / total >= mass:
+            return thr
+    return min(y)
+
+
+def test_top_p_band_brackets_the_nucleus_threshold():
+    """The band sample_tokens_top_p returns for a row is [thr(top_p + band_mass)
+    - band_logit, thr(top_p - band_mass) + band_logit], with thr(.) the
+    nucleus threshold at that mass found by the explicit threshold search: so
+    it contains the nucleus threshold at top_p itself, and is no wider than the
+    mass and logit margins make it.  Rows with continuous logits and rows with
+    many ties."""
+    rng = np.random.default_rng(41)
+    checked = 0
+    for case in range(60):
+        V, Hd = int(rng.integers(2, 40)), 4
+        W = rng.normal(0, 1.0, (V, Hd))
+        if case % 3 == 0:
+            W = np.round(W * 2) / 2    # ties between vocabulary rows
+        H = rng.normal(0, 1.0, (3, Hd))
+        tau = float(rng.choice([0.7, 1.0, 1.5]))
+        top_p = float(rng.uniform(0.05, 0.98))
+        band_mass = float(rng.choice([1e-5, 1e-3, 0.05]))
+        band_logit = float(rng.choice([0.0, 1e-4, 1e-2]))
+        _, _, _, band = oracle.sample_tokens_top_p(H, W, np.ones(3, np.uint8), tau, top_p, seed=3, offset=case,
+                                                   band_mass=band_mass, band_logit=band_logit)
+        for t in range(3):
+            y = ((W @ H[t]) / tau).tolist()
+            lo = _nucleus_threshold_by_search(y, top_p + band_mass) - band_logit
+            hi = _nucleus_threshold_by_search(y, top_p - band_mass) + band_logit
+            assert band[t, 0] == pytest.approx(lo, rel=0, abs=1e-12), (case, t)
+            assert band[t, 1] == pytest.approx(hi, rel=0, abs=1e-12), (case, t)
+            thr = _nucleus_threshold_by_search(y, top_p)
+            assert lo <= thr <= hi
+            checked += 1
+    assert checked == 180
+    # top_p = 1 keeps everything: no band
+    _, _, _, band = oracle.sample_tokens_top_p(np.ones((2, 3)), np.eye(3), np.ones(2, np.uint8), 1.0, 1.0, 1, 0)
+    assert np.all(band == -np.inf)
+
+
 # ---------------------------------------------------------------------------
 # planted mistakes: each must trip one of the pins above
 # ---------------------------------------------------------------------------
@@ -584,3 +656,25 @@ def test_planted_nucleus_one_token_too_many_is_caught(monkeypatch):
     with pytest.raises(AssertionError):
         test_nucleus_matches_threshold_search()
 
+
+def test_planted_widened_top_p_band_is_caught(monkeypatch):
+    """A band ten times wider than its margins would excuse GPU/oracle
+    disagreements it should not: the band pin must catch it."""
+    real = go.sample_tokens_top_p
+
+    def wide(*a, band_mass=1e-5, band_logit=1e-3, **kw):
+        return real(*a, band_mass=10 * band_mass, band_logit=10 * band_logit, **kw)
+    monkeypatch.setattr(oracle, "sample_tokens_top_p", wide)
+    with pytest.raises(AssertionError):
+        test_top_p_band_brackets_the_nucleus_threshold()
+
+
+def test_planted_swapped_top_p_band_ends_are_caught(monkeypatch):
+    """Band ends taken from the wrong side of top_p (the mass margins swapped)."""
+    real = go.sample_tokens_top_p
+
+    def swapped(*a, band_mass=1e-5, **kw):
+        return real(*a, band_mass=-band_mass, **kw)
+    monkeypatch.setattr(oracle, "sample_tokens_top_p", swapped)
+    with pytest.raises(AssertionError):
+        test_top_p_band_brackets_the_nucleus_threshold()

@@ -1,4 +1,4 @@
-"""Property-based pins of the float64 oracle (random small shapes and values).
+"""Property pins of the float64 oracle over seeded random small shapes and values.
 
 Each property follows from Eq. 1 / Eq. 2 of Section 3.3 or from the algebra of
 the softmax, independently of how the oracle computes it:
@@ -20,11 +20,26 @@ import pytest
 import oracle
 from oracle import brute
 
-hyp = pytest.importorskip("hypothesis")
-st = pytest.importorskip("hypothesis.strategies")
-given, settings = hyp.given, hyp.settings
+EXAMPLES = 30
 
-SETTINGS = dict(max_examples=30, deadline=None, derandomize=True)
+
+def _examples(draw_seed, /, **space):
+    """EXAMPLES parameter sets drawn with a fixed seed: each key of `space` is an
+    inclusive integer range (lo, hi) or a list of values to choose from."""
+    rng = np.random.default_rng(draw_seed)
+    out = []
+    for _ in range(EXAMPLES):
+        ex = {}
+        for k, v in space.items():
+            ex[k] = int(rng.integers(v[0], v[1] + 1)) if isinstance(v, tuple) else v[int(rng.integers(len(v)))]
+        out.append(ex)
+    return out
+
+
+def _cases(draw_seed, /, **space):
+    exs = _examples(draw_seed, **space)
+    names = list(space)
+    return pytest.mark.parametrize(",".join(names), [tuple(e[n] for n in names) for e in exs])
 
 
 def _case(seed, n_groups, G, L, Hd, V, ragged=True):
@@ -40,9 +55,7 @@ def _case(seed, n_groups, G, L, Hd, V, ragged=True):
     return rng, H, W, y, m, r, n_resp
 
 
-@settings(**SETTINGS)
-@given(seed=st.integers(0, 10**6), n_groups=st.integers(1, 5), G=st.integers(2, 16),
-       shift=st.sampled_from([-3.0, -0.5, 0.25, 2.0]))
+@_cases(101, seed=(0, 10**6), n_groups=(1, 5), G=(2, 16), shift=[-3.0, -0.5, 0.25, 2.0])
 def test_advantages_shift_invariant_and_zero_mean(seed, n_groups, G, shift):
     rng = np.random.default_rng(seed)
     r = rng.choice([0.0, 0.5, 1.0], n_groups * G)  # dyadic: the shifted sums stay exact
@@ -52,8 +65,7 @@ def test_advantages_shift_invariant_and_zero_mean(seed, n_groups, G, shift):
     assert np.all(np.abs(a.reshape(n_groups, G).sum(1)) <= 1e-5 * G)
 
 
-@settings(**SETTINGS)
-@given(seed=st.integers(0, 10**6), T=st.integers(1, 6), Hd=st.integers(1, 6), V=st.integers(2, 12))
+@_cases(102, seed=(0, 10**6), T=(1, 6), Hd=(1, 6), V=(2, 12))
 def test_logprobs_form_a_distribution_and_match_brute_force(seed, T, Hd, V):
     rng = np.random.default_rng(seed)
     H, W = rng.normal(0, 1.5, (T, Hd)), rng.normal(0, 1.5, (V, Hd))
@@ -67,9 +79,7 @@ def test_logprobs_form_a_distribution_and_match_brute_force(seed, T, Hd, V):
                                rtol=1e-12, atol=1e-12)
 
 
-@settings(**SETTINGS)
-@given(seed=st.integers(0, 10**6), n_groups=st.integers(1, 3), G=st.integers(2, 4), L=st.integers(1, 5),
-       Hd=st.integers(1, 6), V=st.integers(2, 10))
+@_cases(103, seed=(0, 10**6), n_groups=(1, 3), G=(2, 4), L=(1, 5), Hd=(1, 6), V=(2, 10))
 def test_dH_closed_form_and_vocabulary_relabelling(seed, n_groups, G, L, Hd, V):
     rng, H, W, y, m, r, n_resp = _case(seed, n_groups, G, L, Hd, V)
     logp, _ = oracle.token_logprobs(H, W, y, m)
@@ -92,8 +102,7 @@ def test_dH_closed_form_and_vocabulary_relabelling(seed, n_groups, G, L, Hd, V):
     np.testing.assert_allclose(out2["dW"], out["dW"][perm], rtol=1e-10, atol=1e-14)
 
 
-@settings(**SETTINGS)
-@given(seed=st.integers(0, 10**6), n_groups=st.integers(1, 3), G=st.integers(2, 4), L=st.integers(1, 5))
+@_cases(104, seed=(0, 10**6), n_groups=(1, 3), G=(2, 4), L=(1, 5))
 def test_aggregations_agree_for_equal_lengths(seed, n_groups, G, L):
     rng, H, W, y, m, r, n_resp = _case(seed, n_groups, G, L, 3, 5, ragged=False)
     logp, _ = oracle.token_logprobs(H, W, y, m)
