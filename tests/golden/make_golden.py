@@ -1,6 +1,7 @@
 """Write the float64 oracle's log-probs for the 8B-shaped workloads.
 
     python tests/golden/make_golden.py [batch8b] [long_8b] [ragged_8b]
+    python tests/golden/make_golden.py loss [batch8b] [long_8b] [ragged_8b]
 
 Calls only oracle/ and the seeded generators of workloads.py.  For each batch
 it stores, in compacted order (unmasked rows by increasing position):
@@ -13,7 +14,9 @@ it stores, in compacted order (unmasked rows by increasing position):
 
 old_logp / ref_logp are inputs of the loss (they come from earlier forward
 passes of the old and reference policies); lse_policy is an expected value.
-A full run takes about an hour of float64 BLAS on 8 cores.
+A full run takes about an hour of float64 BLAS on 8 cores.  The `loss` mode
+reads those files back and writes <batch>_loss.json, the oracle's loss of
+each batch (see make_loss), in a minute or two.
 """
 from __future__ import annotations
 
@@ -67,6 +70,44 @@ def make(batch: str) -> str:
     return path
 
 
+def make_loss(batch: str) -> str:
+    """<batch>_loss.json: the oracle's loss of the batch in both aggregations
+    (Eq. 1 as a masked token-mean, agg_mode 0, and as printed, agg_mode 1) and
+    the size of the terms it sums (sum_t |w_t l_t|), from the log-sum-exps
+    and old / reference log-probs stored in <batch>.npz, the advantages of
+    the batch's rewards (Eq. 2) and the float64 target logits."""
+    import json
+    w = wl.WORKLOADS[BATCHES[batch]]
+    d = np.load(os.path.join(HERE, f"{batch}.npz"))
+    H, W, y, mask = wl.gen_hidden(w), wl.gen_weight(w, "policy"), wl.gen_targets(w), wl.gen_mask(w)
+    ck = checksums(w, H, W, y, mask)
+    for k in ("ck_h", "ck_w", "ck_y", "n_valid"):
+        assert ck[k] == d[k], k
+    idx = wl.valid_index(mask)
+    logp = np.zeros(w.T)
+    logp[idx] = oracle.target_logits(H, W, y, idx) - d["lse_policy"]
+    old = np.zeros(w.T, np.float32)
+    ref = np.zeros(w.T, np.float32)
+    old[idx], ref[idx] = d["old_logp"], d["ref_logp"]
+    adv = oracle.group_advantages(wl.gen_rewards(w), w.G, float(np.float32(w.adv_eps)))
+    out = {"workload": w.name, "n_valid": int(idx.size), "clip_eps": w.clip_eps, "beta": w.beta}
+    for agg in (0, 1):
+        loss, _, tt = oracle.grpo_loss(logp, old, ref, adv, mask, w.n_resp, w.L, w.clip_eps, w.beta, agg)
+        out[f"loss_agg{agg}"] = loss
+        out[f"sum_abs_terms_agg{agg}"] = float(np.sum(np.abs(tt["w"] * tt["ell"])))
+    path = os.path.join(HERE, f"{batch}_loss.json")
+    with open(path, "w") as f:
+        json.dump(out, f, indent=1)
+        f.write("\n")
+    print(f"[{batch}] wrote {path}", flush=True)
+    return path
+
+
 if __name__ == "__main__":
-    for b in (sys.argv[1:] or list(BATCHES)):
-        make(b)
+    args = sys.argv[1:]
+    if args[:1] == ["loss"]:
+        for b in (args[1:] or list(BATCHES)):
+            make_loss(b)
+    else:
+        for b in (args or list(BATCHES)):
+            make(b)
