@@ -53,9 +53,14 @@ def parse():
     p.add_argument("--adamw", choices=["none", "fused", "separate"], default="none",
                    help="fwd+bwd workloads: add the AdamW step of the LM head, fused into the dW GEMM "
                         "or as a separate pass over the stored dW")
-    p.add_argument("--logits", choices=["keep", "recompute"], default="keep",
-                   help="fwd+bwd workloads: keep the forward's fp32 logits for the backward (a GRPO_WS_LOSS_LOGITS "
-                        "workspace) or recompute them in the backward with a second logits GEMM (GRPO_WS_LOSS)")
+    p.add_argument("--logits", choices=["keep", "recompute"], default="recompute",
+                   help="fwd+bwd workloads: recompute the logits chunk by chunk in the backward with a second "
+                        "logits GEMM, nothing of [tokens x vocabulary] size stored (GRPO_WS_LOSS, the default), "
+                        "or keep the forward's fp32 logits for the backward (an exact GRPO_WS_LOSS_LOGITS workspace)")
+    p.add_argument("--no-kept-compare", action="store_true",
+                   help="skip the extra timing of the kept-logits backward reported beside the recomputing one")
+    p.add_argument("--e2e-steps", type=int, default=20,
+                   help="steps of the end-to-end measurement (per-step wall clock, median reported)")
     p.add_argument("--sample", action="store_true",
                    help="time the rollout draw (grpo_sample_tokens) over the workload's rows instead")
     p.add_argument("--top-p", type=float, default=1.0,
@@ -103,7 +108,29 @@ def make_inputs(w: wl.Workload):
             ref[idx] = d["ref_logp"]
             lse_gold = d["lse_policy"]
             src = "float64 oracle on the perturbed heads (tests/golden)"
-    return dict(H=Hb, W=Wb, y=y, m=m, r=r, old=old, ref=ref, old_src=src, lse_gold=lse_gold)
+    loss_gold = None
+    lpath = os.path.join(ROOT, "tests", "golden", f"{g}_loss.json") if g else None
+    if src is not None and lpath and os.path.exists(lpath):
+        with open(lpath) as f:
+            loss_gold = json.load(f)
+        if loss_gold.get("workload") != w.name:
+            loss_gold = None
+    return dict(H=Hb, W=Wb, y=y, m=m, r=r, old=old, ref=ref, old_src=src, lse_gold=lse_gold, loss_gold=loss_gold)
+
+
+def parity_loss(inp, loss_gpu: float, agg_mode: int = 0):
+    """The library's loss of this batch against the float64 oracle's, stored by
+    tests/golden/make_golden.py: the plain relative error and the error over
+    max(|loss|, sum_t |w_t l_t|) (the advantages of a group sum to zero, so
+    the loss can sit near 0 while its terms do not).  None without stored values."""
+    gold = inp.get("loss_gold")
+    if gold is None:
+        return None
+    want = gold[f"loss_agg{agg_mode}"]
+    scale = max(abs(want), gold[f"sum_abs_terms_agg{agg_mode}"])
+    d = abs(loss_gpu - want)
+    return {"loss": loss_gpu, "loss_oracle": want, "loss_rel": d / abs(want) if want else None,
+            "loss_rel_terms": d / scale, "loss_bar": 1e-3}
 
 
 def parity_logp(inp, grpo, H, W, y, m):
@@ -203,22 +230,36 @@ def kernel_hash() -> str:
     return h.hexdigest()[:16]
 
 
-def stored_traffic(workload: str, kind_name: str):
-    """DRAM bytes per launch from the committed ncu summary, if it was taken on
-    the current kernel source and this workload (profiles/traffic.txt:
-    '<hash> <workload> <kind> <bytes/launch> <cols>')."""
-    path = os.path.join(ROOT, "profiles", "traffic.txt")
+TRAFFIC_PATH = os.path.join(ROOT, "profiles", "traffic.txt")
+
+
+def stored_traffic(variant: str, kind_name: str, Hd: int, V: int, n_valid: int, path: str = TRAFFIC_PATH):
+    """DRAM bytes per launch of one kernel class, from a committed small-case ncu
+    capture (profiles/traffic.txt lines '<hash> <variant> <capture workload>
+    <capture rows> <kind> <bytes/launch> <cols/launch>'), scaled to n_valid
+    rows: the capture runs the same kernel on the same hidden size and
+    vocabulary over fewer rows, and each launch's operand panels, re-reads
+    and outputs grow with its row tiles.  Only lines taken on the current
+    kernel sources count.  Returns (bytes per launch at n_valid rows and the
+    capture's columns, the capture's columns per launch, what was captured)
+    or None."""
     if not os.path.exists(path):
         return None
     kh = kernel_hash()
     for line in open(path):
         f = line.split()
-        if len(f) >= 5 and f[0] == kh and f[1] == workload and f[2] == kind_name:
-            return float(f[3]), int(f[4])
+        if line.startswith("#") or len(f) < 7 or f[0] != kh or f[1] != variant or f[4] != kind_name:
+            continue
+        cw = wl.ALL_WORKLOADS.get(f[2])
+        if cw is None or cw.Hd != Hd or cw.V != V:
+            continue
+        n_cap, b, cols = int(f[3]), float(f[5]), int(f[6])
+        return b * n_valid / n_cap, cols, f"ncu on {f[2]} ({n_cap} unmasked rows), scaled by rows to {n_valid}"
     return None
 
 
-def roofline(trace, n_valid_total_per_rank, Hd, steps, peak_tf, peak_kind, workload_key, hbm_gbs=None):
+def roofline(trace, n_valid_total_per_rank, Hd, steps, peak_tf, peak_kind, variant, hbm_gbs=None, V=None,
+             traffic_path=TRAFFIC_PATH):
     by = {}
     for kind, cols, ms in trace:
         by.setdefault(kind, []).append((cols, ms))
@@ -230,13 +271,15 @@ def roofline(trace, n_valid_total_per_rank, Hd, steps, peak_tf, peak_kind, workl
     achieved = (sum(flops) / len(flops)) / (sum(secs) / len(secs)) / 1e12
     total_ms = sum(ms for v in by.values() for _, ms in v)
     shares = {KIND_NAMES[k]: round(sum(ms for _, ms in v) / total_ms, 4) for k, v in sorted(by.items())}
-    tr = stored_traffic(workload_key, KIND_NAMES[dom])
-    traffic = None
     avg_cols = sum(c for c, _ in recs) / len(recs)
+    tr = None if V is None else stored_traffic(variant, KIND_NAMES[dom], Hd, V, n_valid_total_per_rank,
+                                               traffic_path)
+    traffic = traffic_src = None
     if tr is not None:
-        bytes_per_launch, cols_ref = tr
+        bytes_per_launch, cols_ref, traffic_src = tr
         traffic = bytes_per_launch * avg_cols / cols_ref
-    common = {"kernel": KIND_NAMES[dom], "traffic": traffic, "launches_per_step": len(recs) // max(1, steps),
+    common = {"kernel": KIND_NAMES[dom], "traffic": traffic, "traffic_from": traffic_src,
+              "launches_per_step": len(recs) // max(1, steps),
               "avg_launch_ms": round(sum(secs) / len(secs) * 1e3, 4), "time_share": shares}
     if 13 in by and hbm_gbs:
         # nucleus selection + draw: the stored logits are read once from HBM per row
@@ -253,7 +296,8 @@ def roofline(trace, n_valid_total_per_rank, Hd, steps, peak_tf, peak_kind, workl
         zr = by[12]
         zb = sum(6.0 * n_valid_total_per_rank * c for c, _ in zr) / len(zr)
         zs = sum(ms for _, ms in zr) / len(zr) / 1e3
-        ztr = stored_traffic(workload_key, "dz_logits")
+        ztr = None if V is None else stored_traffic(variant, "dz_logits", Hd, V, n_valid_total_per_rank,
+                                                    traffic_path)
         common["dz_logits_hbm"] = {
             "achieved": round(zb / zs / 1e9, 1), "peak": hbm_gbs, "unit": "GB/s",
             "frac": round(zb / zs / 1e9 / hbm_gbs, 4), "bytes_per_launch": zb, "avg_launch_ms": round(zs * 1e3, 4),
@@ -483,6 +527,7 @@ def main():
     if st != grpo.GRPO_OK:
         raise SystemExit(f"device status after timing: {grpo.status_string(st)}")
 
+    loss_timed = None if sampling or scoring or args.adamw != "none" else float(out[0].item())
     tot_valid = n_valid
     if dist is not None:
         t = torch.tensor([ms], device=dev)
@@ -494,10 +539,8 @@ def main():
     value = tot_valid / (ms / 1e3)
 
     burst, sustained, hbm, peak_src = peaks()
-    rkey = w.name + ("+sample" if sampling else "") + ("+top_p" if sampling and args.top_p < 1.0 else "") + \
-        ("" if args.adamw == "none" else "+adamw_" + args.adamw) + \
-        ("+recompute" if args.logits == "recompute" and not (sampling or scoring) else "")
-    rf = roofline(trace, n_valid, w.Hd, args.steps, sustained, f"bf16 sustained, {peak_src}", rkey, hbm)
+    rf = roofline(trace, n_valid, w.Hd, args.steps, sustained, f"bf16 sustained, {peak_src}",
+                  path_variant(args, sampling, scoring), hbm, V=w.V)
     if sampling:
         step_exec = step_model = 2.0 * n_valid * w.Hd * w.V
     elif scoring:
@@ -511,14 +554,25 @@ def main():
     e2e = e2e_offload = None
     if not args.no_e2e and not sampling:
         if scoring:
-            e2e = measure_e2e_scoring(grpo, torch, dev, w, inp, heads, steps=min(args.steps, 5), dist=dist)
+            e2e = measure_e2e_scoring(grpo, torch, dev, w, inp, heads, steps=args.e2e_steps, dist=dist)
         else:
             # the step's own workspace: a second one of the same size may not fit beside it
-            e2e = measure_e2e(grpo, torch, dev, w, inp, steps=min(args.steps, 5), dist=dist, ws=ws)
+            e2e = measure_e2e(grpo, torch, dev, w, inp, steps=args.e2e_steps, dist=dist, ws=ws)
             if world == 1:
-                e2e_offload = measure_e2e_offload(grpo, torch, dev, w, inp, steps=min(args.steps, 5), ws=ws)
+                e2e_offload = measure_e2e_offload(grpo, torch, dev, w, inp, steps=args.e2e_steps, ws=ws)
 
-    parity = parity_logp(inp, grpo, H, W, y, m) if rank == 0 and not sampling else None
+    kept = None
+    if not (args.no_kept_compare or sampling or scoring) and args.logits == "recompute" and args.adamw == "none" \
+            and world == 1:
+        kept = measure_kept_logits(grpo, torch, dev, w, (H, W, y, m, old, ref, r), n_valid,
+                                   steps=min(args.steps, 10), out=out)
+
+    parity = None
+    if rank == 0 and not sampling:
+        parity = parity_logp(inp, grpo, H, W, y, m) or {}
+        if loss_timed is not None and world == 1:
+            parity.update(parity_loss(inp, loss_timed) or {})
+        parity = parity or None
 
     cpu = None
     if not args.no_cpu_baseline and rank == 0 and world == 1 and not sampling:
@@ -552,9 +606,77 @@ def main():
         }
         if e2e_offload is not None:
             line["e2e_offload"] = e2e_offload
+        if kept is not None:
+            line["kept_logits_ms_per_step"] = kept.get("ms_per_step")
+            line["kept_logits"] = kept
         print(json.dumps(line), flush=True)
     if dist is not None:
         dist.destroy_process_group()
+
+
+def path_variant(args, sampling: bool, scoring: bool) -> str:
+    """Which code path a run times (the key of its traffic lines)."""
+    if sampling:
+        return "sample" + ("+top_p" if args.top_p < 1.0 else "")
+    if scoring:
+        return "score3"
+    return "fwdbwd" + ("+kept" if args.logits == "keep" else "") + \
+        ("" if args.adamw == "none" else "+adamw_" + args.adamw)
+
+
+def measure_kept_logits(grpo, torch, dev, w, tensors, n_valid: int, steps: int, out):
+    """The same step with the opt-in backward that keeps the forward's fp32
+    logits (an exact GRPO_WS_LOSS_LOGITS workspace for the unmasked rows):
+    timed like the main step, reported beside it.  None (with the reason) when
+    that workspace does not fit in the free device memory."""
+    H, W, y, m, old, ref, r = tensors
+    need = grpo.workspace_bytes_rows(w.T, n_valid, w.Hd, w.V, grpo.GRPO_WS_LOSS_LOGITS)
+    torch.cuda.empty_cache()
+    free = torch.cuda.mem_get_info(dev)[0]
+    if need > free - (2 << 30):
+        return {"ms_per_step": None, "skipped": f"workspace of {need / 1e9:.1f} GB does not fit ({free / 1e9:.1f} GB free)"}
+    ws = grpo.workspace(w.T, w.Hd, w.V, grpo.GRPO_WS_LOSS_LOGITS, dev, max_valid=n_valid)
+    if grpo.loss_plan(w.T, w.Hd, w.V, ws.numel())[0] != 1:
+        raise SystemExit("the kept-logits workspace does not keep the logits")
+    adv = torch.empty(w.n_resp, dtype=torch.float32, device=dev)
+
+    def step():
+        grpo.group_advantages(r, w.G, w.adv_eps, out=adv)
+        grpo.loss_fwd_bwd(H, W, y, m, old, ref, adv, w.n_resp, w.L, w.clip_eps, w.beta, 0, ws=ws, out=out)
+
+    for _ in range(3):
+        step()
+    if grpo.check_device_status(ws) != grpo.GRPO_OK:
+        raise SystemExit("device status after the kept-logits warm-up is not OK")
+    stream = torch.cuda.current_stream(dev)
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize(dev)
+    ev0.record(stream)
+    for _ in range(steps):
+        step()
+    ev1.record(stream)
+    torch.cuda.synchronize(dev)
+    ms = ev0.elapsed_time(ev1) / steps
+    st = grpo.check_device_status(ws)
+    del ws
+    torch.cuda.empty_cache()
+    if st != grpo.GRPO_OK:
+        raise SystemExit("device status after the kept-logits steps is not OK")
+    return {"ms_per_step": round(ms, 3), "value": round(n_valid / (ms / 1e3), 1), "unit": "tokens/s",
+            "steps": steps, "workspace_bytes": int(need),
+            "what": "opt-in variant: the forward stores the fp32 logits [rows x V] in the workspace and the "
+                    "backward forms dZ from them by an HBM pass instead of the recomputing GEMM"}
+
+
+def timed_steps(one, steps: int):
+    """(median, mean) wall-clock seconds of `steps` calls of one(), each of which
+    returns only once its results are on the host."""
+    ts = []
+    for _ in range(max(1, steps)):
+        t0 = time.perf_counter()
+        one()
+        ts.append(time.perf_counter() - t0)
+    return statistics.median(ts), sum(ts) / len(ts)
 
 
 def across_ranks(torch, dev, dist, dt: float, n_tok: int):
@@ -591,12 +713,11 @@ def measure_e2e_scoring(grpo, torch, dev, w, inp, heads, steps: int, dist=None):
     one()
     if dist is not None:
         dist.barrier()
-    t0 = time.perf_counter()
-    for _ in range(steps):
-        one()
-    dt, n_tok = across_ranks(torch, dev, dist, (time.perf_counter() - t0) / steps, n_valid)
+    med, mean = timed_steps(one, steps)
+    dt, n_tok = across_ranks(torch, dev, dist, med, n_valid)
     return {"value": round(n_tok / dt, 1), "unit": "tokens/s", "ms_per_step": round(dt * 1e3, 2),
-            "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h), "steps": steps,
+            "ms_mean": round(mean * 1e3, 2), "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
+            "steps": steps, "statistic": "median of per-step wall-clock times",
             "what": "H, targets, mask copied from pinned host memory each step; the policy / old / reference "
                     "heads resident on the device; the log-probs read back"}
 
@@ -638,12 +759,11 @@ def measure_e2e(grpo, torch, dev, w, inp, steps: int, dist=None, ws=None):
     torch.cuda.synchronize(dev)
     if dist is not None:
         dist.barrier()
-    t0 = time.perf_counter()
-    for _ in range(steps):
-        one()
-    dt, n_tok = across_ranks(torch, dev, dist, (time.perf_counter() - t0) / steps, n_valid)
+    med, mean = timed_steps(one, steps)
+    dt, n_tok = across_ranks(torch, dev, dist, med, n_valid)
     return {"value": round(n_tok / dt, 1), "unit": "tokens/s", "ms_per_step": round(dt * 1e3, 2),
-            "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h), "steps": steps,
+            "ms_mean": round(mean * 1e3, 2), "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
+            "steps": steps, "statistic": "median of per-step wall-clock times",
             "what": "H, targets, mask, old/ref log-probs, rewards copied from pinned host memory each step; W "
                     "resident on the device; the loss read back; dH, dW left on the device"}
 
@@ -675,13 +795,10 @@ def measure_e2e_offload(grpo, torch, dev, w, inp, steps: int, ws=None):
 
     one()
     torch.cuda.synchronize(dev)
-    t0 = time.perf_counter()
-    for _ in range(steps):
-        loss, dH, dW = one()   # returns pinned host tensors once they have landed
-    dt = (time.perf_counter() - t0) / steps
-    n_valid = int(inp["m"].sum())
-    return {"value": round(n_valid / dt, 1), "unit": "tokens/s", "ms_per_step": round(dt * 1e3, 2),
-            "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h), "steps": steps,
+    med, mean = timed_steps(one, steps)   # one() returns pinned host tensors once they have landed
+    return {"value": round(n_valid / med, 1), "unit": "tokens/s", "ms_per_step": round(med * 1e3, 2),
+            "ms_mean": round(mean * 1e3, 2), "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
+            "steps": steps, "statistic": "median of per-step wall-clock times",
             "what": "batch and W copied from pinned host memory each step; loss, dH, dW copied back"}
 
 

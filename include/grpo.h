@@ -53,10 +53,14 @@ typedef enum {
 
 /*
  * Which call a workspace is sized for (grpo_workspace_bytes `which`).
- * GRPO_WS_LOSS_LOGITS sizes a loss workspace that also keeps the fp32 logits
- * of the forward ([rows x V], 4 bytes each: 12.2 GB for 19,572 unmasked rows
- * at V 155136) so that the backward forms dZ from them with an HBM-bound
- * pass instead of recomputing the logits GEMM; see grpo_loss_plan.
+ * GRPO_WS_LOSS sizes the loss workspace of the default backward, which
+ * recomputes each vocabulary chunk of the logits with a second GEMM: nothing
+ * of [tokens x vocabulary] size is ever stored.  GRPO_WS_LOSS_LOGITS is an
+ * opt-in: a loss workspace that also keeps the fp32 logits of the forward
+ * ([rows x V], 4 bytes each: 12.2 GB for 19,572 unmasked rows at V 155136) so
+ * that the backward forms dZ from them with an HBM-bound pass instead of
+ * recomputing the logits GEMM.  A loss call keeps the logits only when its
+ * ws_bytes is exactly such a size; see grpo_loss_plan.
  */
 enum {
   GRPO_WS_LOGPROBS = 0,
@@ -193,10 +197,12 @@ grpo_status grpo_gumbel_noise(uint64_t seed, uint64_t offset, int64_t row0, int6
  *   loss_out             device pointer to one fp32
  *   dH                   [T x Hd] fp32 device; padding rows get 0
  *   dW                   [V x Hd] fp32 device
- *   ws                   at least grpo_workspace_bytes(T, Hd, V, GRPO_WS_LOSS) bytes;
- *                        with grpo_workspace_bytes(T, Hd, V, GRPO_WS_LOSS_LOGITS)
- *                        the logits are kept from the forward for the backward
- *                        (faster; bit-identical results, see grpo_loss_plan)
+ *   ws                   at least grpo_workspace_bytes(T, Hd, V, GRPO_WS_LOSS) bytes:
+ *                        the backward recomputes the logits chunk by chunk and
+ *                        never stores them.  Opt-in: exactly
+ *                        grpo_workspace_bytes(T, Hd, V, GRPO_WS_LOSS_LOGITS)
+ *                        bytes keep the fp32 logits from the forward for the
+ *                        backward (bit-identical results, see grpo_loss_plan)
  * Requires n_resp >= 1, L >= 1, clip_eps >= 0, agg_mode in {0, 1}, dH and dW
  * 16-byte aligned, and the limits of grpo_token_logprobs.
  */
@@ -337,19 +343,32 @@ grpo_status grpo_adamw_step(float* W_master, float* exp_avg, float* exp_avg_sq, 
  *   - Returns GRPO_ERR_WORKSPACE if grpo_workspace_bytes(T, Hd, V,
  *     GRPO_WS_LOGPROBS) exceeds 64 MiB (7,680 tokens at Hd 4096,
  *     V 155136), GRPO_ERR_INVALID_ARG for arguments grpo_token_logprobs rejects.
- *   - The first call on a device looks up the array's device address (with
- *     that device current); make that first call before any stream capture.
+ *   - Every call looks up the array's device address in the current device's
+ *     context (so a context made after cudaDeviceReset gets its own).  The
+ *     first call on a device also loads the library's device code there; make
+ *     that first call before any stream capture.
  *   - Every call uses the same array and leaves its contents behind; each call
  *     clears what it needs cleared.  Calls whose work can overlap on the GPU
  *     (different streams, or different host threads) race on the array and
  *     give wrong results: serialise them.
- *   - Device-side problems (a target outside [0, V)) give 0 for the affected
- *     rows as in grpo_token_logprobs, but there is no workspace to pass to
- *     grpo_check_device_status.
+ *   - Device-side problems (a target outside [0, V), a non-finite log-sum-exp)
+ *     give 0 for the affected rows as in grpo_token_logprobs and set the
+ *     array's device status word: read it with grpo_noalloc_check_status.
  */
 grpo_status grpo_token_logprobs_noalloc(const uint16_t* H, const uint16_t* W, const int32_t* targets,
                                         const uint8_t* mask, int64_t T, int32_t Hd, int64_t V,
                                         float* logp_out, void* stream);
+
+/*
+ * grpo_check_device_status for the fixed array of grpo_token_logprobs_noalloc
+ * (the paper has no counterpart): synchronises `stream`, then reports the
+ * device status word the last no-alloc call on the current device left
+ * behind, as GRPO_OK, GRPO_ERR_DEVICE_CHECK, GRPO_ERR_TIMEOUT or
+ * GRPO_ERR_CAPACITY (GRPO_ERR_CUDA if the array cannot be reached).  Allocates
+ * nothing.  The word is cleared at the start of every no-alloc call, and a
+ * no-alloc call still running on another stream may change it.
+ */
+grpo_status grpo_noalloc_check_status(void* stream);
 
 /*
  * Bytes of workspace the call `which` (GRPO_WS_LOGPROBS, GRPO_WS_LOSS,
@@ -384,13 +403,12 @@ size_t grpo_workspace_bytes_rows(int64_t T, int64_t max_valid, int32_t Hd, int64
  * logits for the backward, 0 when the backward recomputes them with a second
  * logits GEMM, -1 for arguments or a workspace the calls would reject; *rows
  * (if not null) gets the row capacity (unmasked rows the call can hold).
- * The logits are kept when the workspace holds them at the row capacity the
- * plain loss layout gives (so a plain workspace never loses capacity to
- * them), or when ws_bytes is exactly what grpo_workspace_bytes or
- * grpo_workspace_bytes_rows returns for GRPO_WS_LOSS_LOGITS, in which case the
- * capacity is the one it was sized for (max_valid rounded up to 256 rows).
- * A workspace of another size (e.g. rounded up) that does not hold the logits
- * at the plain capacity runs the recomputing backward.
+ * The logits are kept only when ws_bytes is exactly what grpo_workspace_bytes
+ * or grpo_workspace_bytes_rows returns for GRPO_WS_LOSS_LOGITS (and not also
+ * exactly the plain layout's size); the row capacity is then the one it was
+ * sized for (max_valid rounded up to 256 rows).  Any other size, however
+ * large, runs the recomputing backward with the largest plain capacity that
+ * fits, so a caller who never asks for the logits never gets them stored.
  * Both ways give bit-identical loss, dH and dW: the two GEMMs accumulate the
  * same logits in the same order, and both form dZ with the same arithmetic.
  */

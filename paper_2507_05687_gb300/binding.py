@@ -67,6 +67,7 @@ SIGNATURES = {
     "grpo_gumbel_noise": (ctypes.c_int, [ctypes.c_uint64, ctypes.c_uint64, _I64, _I64, _I64, _P, _P]),
     "grpo_adamw_step": (ctypes.c_int, [_P, _P, _P, _P, _P, _I64, _F, _F, _F, _F, _F, _I64, _P]),
     "grpo_token_logprobs_noalloc": (ctypes.c_int, [_P, _P, _P, _P, _I64, _I32, _I64, _P, _P]),
+    "grpo_noalloc_check_status": (ctypes.c_int, [_P]),
     "grpo_workspace_bytes": (ctypes.c_size_t, [_I64, _I32, _I64, _I32]),
     "grpo_workspace_bytes_rows": (ctypes.c_size_t, [_I64, _I64, _I32, _I64, _I32]),
     "grpo_loss_plan": (ctypes.c_int32, [_I64, _I32, _I64, ctypes.c_size_t, _P]),
@@ -191,17 +192,15 @@ def loss_plan(T: int, Hd: int, V: int, ws_bytes: int) -> Tuple[int, int]:
     return kept, int(rows.value)
 
 
-def loss_workspace(T: int, Hd: int, V: int, device=None, max_valid: Optional[int] = None) -> torch.Tensor:
-    """A workspace for the loss calls: one that keeps the logits from the
-    forward for the backward (GRPO_WS_LOSS_LOGITS) when that fits in half of
-    the device's free memory, else the plain one (GRPO_WS_LOSS).  Both give
-    the same results; the first skips the backward's logits GEMM."""
-    dev = torch.device(device or "cuda")
-    kept = workspace_bytes(T, Hd, V, GRPO_WS_LOSS_LOGITS) if max_valid is None else \
-        workspace_bytes_rows(T, max_valid, Hd, V, GRPO_WS_LOSS_LOGITS)
-    free = torch.cuda.mem_get_info(dev)[0] if dev.type == "cuda" else 0
-    which = GRPO_WS_LOSS_LOGITS if 0 < kept <= free // 2 else GRPO_WS_LOSS
-    return workspace(T, Hd, V, which, dev, max_valid=max_valid)
+def loss_workspace(T: int, Hd: int, V: int, device=None, max_valid: Optional[int] = None,
+                   keep_logits: bool = False) -> torch.Tensor:
+    """A workspace for the loss calls.  By default the plain one
+    (GRPO_WS_LOSS): the backward recomputes the logits chunk by chunk and no
+    [tokens x vocabulary] buffer exists.  keep_logits=True sizes it exactly
+    for GRPO_WS_LOSS_LOGITS instead: the forward stores the fp32 logits and the
+    backward reads them back (same results, bit for bit)."""
+    which = GRPO_WS_LOSS_LOGITS if keep_logits else GRPO_WS_LOSS
+    return workspace(T, Hd, V, which, device or "cuda", max_valid=max_valid)
 
 
 def workspace(T: int, Hd: int, V: int, which: int, device=None, max_valid: Optional[int] = None) -> torch.Tensor:

@@ -168,19 +168,19 @@ bool fit_layout(int64_t T, int32_t Hd, int64_t V, int32_t which, size_t ws_bytes
   return make_layout(T, Hd, V, which, L, lo * kRowAlign);
 }
 
-// The layout of a loss call with a workspace of ws_bytes.  The logits are
-// kept from the forward to the backward (a) when the workspace holds them at
-// the row capacity the plain loss layout gives (fit_layout), or (b) when
-// ws_bytes is exactly a kept-logits size (grpo_workspace_bytes(_rows) with
-// GRPO_WS_LOSS_LOGITS), and not also exactly a plain one: a workspace sized
-// for max_valid rows with the logits is larger than the plain layout needs
-// for more rows, so its size, not the largest plain capacity, says what it
-// was made for.  Any other size keeps the plain layout's capacity.
+// The layout of a loss call with a workspace of ws_bytes.  By default the
+// backward recomputes each vocabulary chunk of the logits and nothing of
+// [tokens x vocabulary] size is stored.  The logits are kept from the forward
+// to the backward only when ws_bytes is exactly a kept-logits size
+// (grpo_workspace_bytes(_rows) with GRPO_WS_LOSS_LOGITS) and not also exactly
+// the plain layout's size: the caller asked for that layout by its size.  A
+// larger workspace of any other size keeps the plain layout, however much
+// room it has.
 bool fit_loss_layout(int64_t T, int32_t Hd, int64_t V, size_t ws_bytes, Layout* L) {
   if (!fit_layout(T, Hd, V, GRPO_WS_LOSS, ws_bytes, L)) return false;
   Layout kept;
-  if (fit_layout(T, Hd, V, GRPO_WS_LOSS_LOGITS, ws_bytes, &kept) &&
-      (kept.rows >= L->rows || (kept.total == ws_bytes && L->total != ws_bytes)))
+  if (fit_layout(T, Hd, V, GRPO_WS_LOSS_LOGITS, ws_bytes, &kept) && kept.total == ws_bytes &&
+      L->total != ws_bytes)
     *L = kept;
   return true;
 }
@@ -1319,20 +1319,16 @@ namespace {
 constexpr size_t kStaticScratchBytes = size_t(64) << 20;  // 64 MiB on every device that loads the library
 static __device__ __align__(256) unsigned char g_static_scratch[kStaticScratchBytes];
 
-// Device address of g_static_scratch on the current device, looked up once per
-// device.  The host-side symbol is only a stand-in, never a device address.
+// Device address of g_static_scratch in the current device's context.  The
+// host-side symbol is only a stand-in, never a device address.  Looked up on
+// every call (a table lookup in the runtime once the module is loaded), so a
+// context made after cudaDeviceReset gets its own address, never a stale one;
+// the first call on a device loads the module and should come before any
+// stream capture.
 void* static_scratch() {
-  static std::mutex mu;
-  static void* addr[64] = {};
-  int dev = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return nullptr;
-  std::lock_guard<std::mutex> lk(mu);
-  if (!addr[dev]) {
-    void* p = nullptr;
-    if (cudaGetSymbolAddress(&p, g_static_scratch) != cudaSuccess) return nullptr;
-    addr[dev] = p;
-  }
-  return addr[dev];
+  void* p = nullptr;
+  if (cudaGetSymbolAddress(&p, g_static_scratch) != cudaSuccess) return nullptr;
+  return p;
 }
 
 }  // namespace
@@ -1347,4 +1343,10 @@ extern "C" grpo_status grpo_token_logprobs_noalloc(const uint16_t* H, const uint
   void* ws = static_scratch();
   if (!ws) return GRPO_ERR_CUDA;
   return grpo_token_logprobs(H, W, targets, mask, T, Hd, V, logp_out, ws, kStaticScratchBytes, stream);
+}
+
+extern "C" grpo_status grpo_noalloc_check_status(void* stream) {
+  void* ws = static_scratch();
+  if (!ws) return GRPO_ERR_CUDA;
+  return grpo_check_device_status(ws, stream);
 }

@@ -7,15 +7,18 @@ reach the library from a language binding that has no device allocator.  For
 them the library keeps a fixed 64 MiB scratch array in its own device memory.
 
 This file checks, through the C ABI, that the workspace-free call gives the
-same log-probs as grpo_token_logprobs with a caller workspace (within the
-tolerance of the other parity tests), on two calls in a row of different
-sizes, so state the first call leaves in the shared array cannot leak into the
-second; and that sizes beyond the array are refused.  It is named so pytest
-collects it last.
+same log-probs as grpo_token_logprobs with a caller workspace, bit for bit
+(the same kernels on the same inputs), and the float64 oracle's within the
+log-prob tolerance, on two calls in a row of different sizes, so that state
+the first call leaves in the shared array cannot leak into the second; that a
+bad target in a no-alloc call is reported by grpo_noalloc_check_status and
+cleared by the next call; and that sizes beyond the array are refused.  It is
+named so pytest collects it last.
 """
 import numpy as np
 import pytest
 
+import oracle
 import workloads as wl
 from tests._util import LOGP_ATOL, dev_tensor
 
@@ -33,9 +36,8 @@ DEV = torch.device("cuda", 0)
 STATIC_BYTES = 64 << 20
 
 
-def _inputs(w):
-    return (dev_tensor(wl.gen_hidden(w), torch.bfloat16), dev_tensor(wl.gen_weight(w), torch.bfloat16),
-            dev_tensor(wl.gen_targets(w), torch.int32), dev_tensor(wl.gen_mask(w), torch.uint8))
+def _host(w):
+    return wl.gen_hidden(w), wl.gen_weight(w), wl.gen_targets(w), wl.gen_mask(w)
 
 
 def _noalloc(H, W, y, m):
@@ -49,23 +51,53 @@ def _noalloc(H, W, y, m):
     return out
 
 
-def test_noalloc_matches_workspace_call_twice_in_a_row():
-    cases = [
-        # a larger batch first, then a smaller one with a vocabulary tail, so the
-        # second call runs on an array holding the first call's leftovers
-        wl.Workload("na1", 2, 4, 300, 512, 9000, "uniform", 1, 300, seed=wl.SEED_BASE + 4242),
-        wl.Workload("na2", 1, 3, 77, 256, 1000, "uniform", 1, 77, seed=wl.SEED_BASE + 4343),
-    ]
-    for w in cases:
+def _status():
+    return grpo.load().grpo_noalloc_check_status(torch.cuda.current_stream(DEV).cuda_stream)
+
+
+CASES = [
+    # a larger batch first, then a smaller one with a vocabulary tail, so the
+    # second call runs on an array holding the first call's leftovers
+    wl.Workload("na1", 2, 4, 300, 512, 9000, "uniform", 1, 300, seed=wl.SEED_BASE + 4242),
+    wl.Workload("na2", 1, 3, 77, 256, 1000, "uniform", 1, 77, seed=wl.SEED_BASE + 4343),
+]
+
+
+def test_noalloc_matches_workspace_call_and_oracle_twice_in_a_row():
+    for w in CASES:
         assert grpo.workspace_bytes(w.T, w.Hd, w.V, grpo.GRPO_WS_LOGPROBS) <= STATIC_BYTES
-        H, W, y, m = _inputs(w)
+        Hb, Wb, yb, mb = _host(w)
+        H, W = dev_tensor(Hb, torch.bfloat16), dev_tensor(Wb, torch.bfloat16)
+        y, m = dev_tensor(yb, torch.int32), dev_tensor(mb, torch.uint8)
         want = grpo.token_logprobs(H, W, y, m)
         got = _noalloc(H, W, y, m)
-        torch.cuda.synchronize()
+        assert _status() == grpo.GRPO_OK
         g, e = got.cpu().numpy(), want.cpu().numpy()
-        assert np.isfinite(g).all()
-        assert np.all(g[m.cpu().numpy() == 0] == 0.0)
-        assert np.abs(g - e).max() <= LOGP_ATOL
+        assert np.array_equal(g.view(np.uint32), e.view(np.uint32))
+        assert np.all(g[mb == 0] == 0.0)
+        ref, _ = oracle.token_logprobs(Hb, Wb, yb, mb)
+        assert np.abs(g.astype(np.float64) - ref).max() <= LOGP_ATOL
+
+
+def test_noalloc_reports_a_bad_target_and_clears_it():
+    w = CASES[1]
+    Hb, Wb, yb, mb = _host(w)
+    bad = yb.copy()
+    t_bad = int(wl.valid_index(mb)[3])
+    bad[t_bad] = w.V + 5    # outside [0, V) on an unmasked row
+    H, W = dev_tensor(Hb, torch.bfloat16), dev_tensor(Wb, torch.bfloat16)
+    m = dev_tensor(mb, torch.uint8)
+    got = _noalloc(H, W, dev_tensor(bad, torch.int32), m).cpu().numpy()
+    assert _status() == grpo.GRPO_ERR_DEVICE_CHECK
+    assert got[t_bad] == 0.0
+    # the other rows are those of a good call
+    ref, _ = oracle.token_logprobs(Hb, Wb, yb, mb)
+    keep = np.ones(w.T, bool)
+    keep[t_bad] = False
+    assert np.abs(got[keep].astype(np.float64) - ref[keep]).max() <= LOGP_ATOL
+    # the next call starts with a clear word
+    _noalloc(H, W, dev_tensor(yb, torch.int32), m)
+    assert _status() == grpo.GRPO_OK
 
 
 def test_noalloc_refuses_sizes_beyond_its_array():

@@ -100,6 +100,11 @@ WORKLOADS = {
 PROFILE_WORKLOADS = {
     "fwdbwd_small": Workload("fwdbwd_small", 2, 8, 512, 4096, 32768, "uniform", 128, 512,
                              rewards="mix", seed=SEED_BASE + 6),
+    # the bench's hidden size, vocabulary, vocabulary chunks and lengths over a
+    # quarter of its prompts (about 5k unmasked rows, about 5 GB on the device):
+    # DRAM-counter captures of single GEMM launches, scaled to the bench by rows
+    "fwdbwd_mid": Workload("fwdbwd_mid", 2, 8, 512, 4096, 155136, "uniform", 128, 512,
+                           rewards="mix", seed=SEED_BASE + 8),
 }
 # One decode step of rollout generation: every active sequence samples its next
 # token, so the LM-head GEMM sees a few hundred to a few thousand rows (here
