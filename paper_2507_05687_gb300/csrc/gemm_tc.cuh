@@ -126,7 +126,7 @@ struct GemmArgs {
   int b_off_n, b_off_k; // coordinate offsets into B's tensor map
   int n_per_unit;       // consecutive N tiles one CTA (pair) walks as one work unit
   int n_heads;          // B matrices (LM heads) swept against the same A, 1..kMaxHeads
-  int group_m;          // raster: M tiles per group sharing the same N sweep
+  int group_m;          // raster: at most this many M tiles per group sharing the same N sweep
   int a_hint, b_hint;   // L2 eviction policy of A / B loads (kHint*)
   unsigned* status;     // device status word
   unsigned long long wait_ns;  // bound of every pipeline wait (0: kWaitLimitNs)
@@ -170,6 +170,7 @@ struct GemmArgs {
 
 struct TileSched {
   int m_tiles, n_tiles, units_head, units_n, total, k_blocks, m_rows;
+  int group;  // M tiles per raster group (balanced, at most GemmArgs::group_m)
 };
 
 __device__ __forceinline__ TileSched make_sched(const GemmArgs& a, int tile_m) {
@@ -183,18 +184,22 @@ __device__ __forceinline__ TileSched make_sched(const GemmArgs& a, int tile_m) {
   s.units_n = s.units_head * max(1, a.n_heads);
   s.total = s.m_tiles * s.units_n;
   s.k_blocks = (K + kBK - 1) / kBK;
+  // as few groups as group_m allows, of near-equal height: a last group of a
+  // few M tiles would stream all of B again for a sliver of the work
+  const int gmax = max(1, a.group_m);
+  const int ngroups = max(1, (s.m_tiles + gmax - 1) / gmax);
+  s.group = max(1, (s.m_tiles + ngroups - 1) / ngroups);
   return s;
 }
 
-// Work unit u -> (m tile, n unit).  Groups of group_m consecutive M tiles
+// Work unit u -> (m tile, n unit).  Groups of s.group consecutive M tiles
 // sweep the N units together, so the CTAs running at the same time share B
 // tiles (and A tiles) in L2.
-__device__ __forceinline__ void unit_coords(const GemmArgs& a, const TileSched& s, int u, int& mt,
-                                            int& un) {
-  const int per_group = a.group_m * s.units_n;
+__device__ __forceinline__ void unit_coords(const GemmArgs&, const TileSched& s, int u, int& mt, int& un) {
+  const int per_group = s.group * s.units_n;
   const int g = u / per_group;
-  const int first = g * a.group_m;
-  const int gm = min(a.group_m, s.m_tiles - first);
+  const int first = g * s.group;
+  const int gm = min(s.group, s.m_tiles - first);
   const int w = u - g * per_group;
   mt = first + w % gm;
   un = w / gm;
@@ -323,6 +328,12 @@ __device__ __forceinline__ bool adam_block(OutStage& o, const float* g, int x, i
     }
   }
   const bool got = mbar_wait(o.ld_bar, o.ld_phase, o.abort, o.wlim);
+  if (!got && o.lane == 0) {
+    // the wait gave up: let the block's loads land before the buffer can be
+    // released (they complete on ld_bar unless they were never issued)
+    volatile int never = 0;
+    if (!mbar_wait(o.ld_bar, o.ld_phase, &never, kDrainNs)) __nanosleep(kDrainPauseNs);
+  }
   o.ld_phase ^= 1u;
   if (!__all_sync(0xffffffffu, got)) return false;
   const uint32_t row = static_cast<uint32_t>(o.lane * 128);
@@ -654,6 +665,25 @@ __device__ __forceinline__ void gemm_body(const CUtensorMap* tmA, const CUtensor
       for (int s = 0; s < kStages; ++s)
         if (uses[s] > 0)
           mbar_wait(smem_addr(&empty_bar[s]), static_cast<uint32_t>(uses[s] - 1) & 1u, abort_flag, wlim);
+      // After an abort those waits give up at once, and a stage may still
+      // have copies in flight.  The issuing CTA's full barrier of a stage
+      // counts every byte both CTAs of the pair loaded into it, so a bounded
+      // wait on the phase of each stage's last fill returns once they have
+      // landed (the teardown's cluster barrier then holds the peer until this
+      // drain ends).  Where that phase cannot complete (a copy that was never
+      // issued), and on the peer, whose copies only the issuing CTA's
+      // barriers count, a fixed pause stands in for the wait.
+      if (*abort_flag) {
+        bool drained = issuer;
+        if (issuer) {
+          volatile int never = 0;
+          for (int s = 0; s < kStages; ++s)
+            if (uses[s] > 0 && !mbar_wait(smem_addr(&full_bar[s]), static_cast<uint32_t>(uses[s] - 1) & 1u, &never,
+                                          kDrainNs))
+              drained = false;
+        }
+        if (!drained) __nanosleep(kDrainPauseNs);
+      }
     }
   } else if (warp == 1) {
     // ------------------------------------------------------------ MMA issuer
@@ -790,9 +820,7 @@ __device__ __forceinline__ void gemm_body(const CUtensorMap* tmA, const CUtensor
     if (ES::kTmaOut && lane == 0) bulk_wait_all();
   }
 
-  // After a timeout, give copies that may still be in flight time to land
-  // before the shared memory they target is released.
-  if (*abort_flag) __nanosleep(200000);
+  // (after a timeout the producer has drained the copies it issued: above)
   tc_fence_before();
   if (kPair == 2) cluster_sync(); else __syncthreads();
   if (warp == 1) {

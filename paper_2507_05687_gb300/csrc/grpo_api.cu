@@ -238,6 +238,7 @@ struct DeviceInfo {
   int sms = 0;
   int pairs = 0;        // CTA pairs of the pair kernels that can be resident at once
   int top_p_clusters = 0;  // clusters of the nucleus selection kernel resident at once
+  int fast_ctas = 0;       // CTAs of the nucleus fast pass resident at once (all SMs)
   bool ok = false;
 };
 
@@ -302,6 +303,15 @@ bool device_info(DeviceInfo* out) {
     cache[dev].sms = sms;
     cache[dev].pairs = std::max(pairs, 0);
     cache[dev].top_p_clusters = std::max(tpc, 1);
+    // the nucleus fast pass streams the stored logits through a shared-memory
+    // ring (kFastSmem bytes); its grid is what can be resident at once
+    int per_sm = 0;
+    if (cudaFuncSetAttribute(top_p_fast_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kFastSmem) !=
+            cudaSuccess ||
+        cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, top_p_fast_kernel, kTopPThreads, kFastSmem) !=
+            cudaSuccess)
+      return false;
+    cache[dev].fast_ctas = std::max(1, per_sm) * sms;
     cache[dev].ok = true;
   }
   *out = cache[dev];
@@ -352,23 +362,22 @@ bool use_pairs() {
   return !(e && e[0] == '0');
 }
 
-// Raster group height (M tiles per group) of each GEMM: LSE, dZ, dH, dW.
-// The forward GEMM re-reads A (the gathered hidden states) for every one of
-// its ~600 vocabulary tiles: a group of a quarter as many M tiles as there
-// are CTAs (pairs) makes every round of the persistent grid cover whole
-// groups (each W tile read by that many CTAs at once) while the group's A
-// tiles (38 MB on GB300) stay in L2; measured DRAM reads per launch at
-// 19,572 tokens x 155,136: 62.7 GB with 8 M tiles, 34.8 GB with pairs / 2,
-// 26.7 GB with pairs / 4.  The backward GEMMs measured best at 8.  The
-// forward that also stores the logits (which = 4) measured best at 8 M tiles
-// as well: 47.5 against 47.8 ms per step at 19,572 tokens, and 123 against
-// 133 ms for the forward of 160,089 tokens, whose logits (99 GB) stream
-// through L2 beside the operand tiles.
+// Largest raster group (M tiles per group) of each GEMM: LSE, dZ, dH, dW,
+// and the forward that stores the logits (4).  The kernel splits the M tiles
+// into as few groups of near-equal height as this allows.  The forward GEMM
+// re-reads A (the gathered hidden states) for every one of its ~600
+// vocabulary tiles, while the CTAs working on one group share each W tile
+// in L2: up to 24 M tiles (48 MB of A) per group.  Measured on 5,390 rows x
+// 155,136 (22 M tiles): 6.57 GB of DRAM reads per forward launch with groups
+// of 19 + 3 tiles, 4.02 GB with all 22 in one group, 11.5 GB with two of 11;
+// at 19,572 rows the step time moved by less than run-to-run noise (59.6-61
+// ms) between groups of 16, 19, 20 and 26.  The backward GEMMs measured best
+// at 8; so did the forward that also stores the logits (47.5 against 47.8 ms
+// per step at 19,572 tokens, 123 against 133 ms for the forward of 160,089
+// tokens, whose logits stream through L2 beside the operand tiles).
 // GRPO_GROUP_M="a,b,c,d[,e]" overrides the defaults.
-int group_m(int which, const DeviceInfo& di) {
-  const int workers = use_pairs() && di.pairs > 0 ? di.pairs : di.sms;
-  const int quarter = std::max(1, workers / 4);
-  int g[5] = {quarter, 8, 8, 8, 8};
+int group_m(int which, const DeviceInfo&) {
+  int g[5] = {24, 8, 8, 8, 8};
   if (const char* e = std::getenv("GRPO_GROUP_M")) {
     int v[5];
     const int n = std::sscanf(e, "%d,%d,%d,%d,%d", &v[0], &v[1], &v[2], &v[3], &v[4]);
@@ -905,19 +914,20 @@ grpo_status grpo_sample_tokens_top_p(const uint16_t* H, const uint16_t* W, const
     if (e == cudaSuccess && top_p < 1.f) {
       unsigned* n_slow = at<unsigned>(ws, Ly.n_slow);
       e = cudaMemsetAsync(n_slow, 0, 4, s);
-      // is the winner in the nucleus?  four CTAs per SM, all resident; a row is
-      // cut into slices (one CTA each, up to 8) until there are about two
-      // pieces of work per CTA (the row count is the capacity here: the
-      // unmasked count is only known on the device)
-      const int64_t slots = int64_t(di.sms) * 4;
-      const int slices = static_cast<int>(
-          std::max<int64_t>(1, std::min<int64_t>(8, (2 * slots + Ly.rows - 1) / std::max<int64_t>(1, Ly.rows))));
-      const int fb2 = static_cast<int>(std::min<int64_t>(Ly.rows * slices, slots));
+      // is the winner in the nucleus?  every CTA that can be resident, each
+      // over one contiguous range of the rows' logit chunks (the unmasked row
+      // count is only known on the device; CTAs past the work return at once)
+      // test hook: GRPO_TEST_TOP_P_LIST_ALL=1 lists every row (a margin above
+      // any mass), so the selection's exact confirmation decides each one
+      unsigned long long margin = top_p_margin(V);
+      if (const char* h = std::getenv("GRPO_TEST_TOP_P_LIST_ALL"))
+        if (h[0] == '1') margin = 1ull << 42;
       if (e == cudaSuccess)
-        top_p_fast_kernel<<<fb2, kTopPThreads, 0, s>>>(
-            at<float>(ws, Ly.z), Ly.ldz, static_cast<int>(V), at<int>(ws, Ly.n_valid), slices, lse_r, y0_r,
+        top_p_fast_kernel<<<di.fast_ctas, kTopPThreads, kFastSmem, s>>>(
+            at<float>(ws, Ly.z), Ly.ldz, static_cast<int>(V), at<int>(ws, Ly.n_valid), lse_r, y0_r,
             1.f / temperature, top_p, at<unsigned long long>(ws, Ly.row_above), at<unsigned>(ws, Ly.row_done),
-            at<int>(ws, Ly.slow_rows), at<unsigned long long>(ws, Ly.slow_tgt), n_slow);
+            at<int>(ws, Ly.slow_rows), at<unsigned long long>(ws, Ly.slow_tgt), n_slow, margin,
+            at<unsigned>(ws, Ly.status));
       // the rows whose winner falls outside: clusters of kTopPCtas CTAs, one row
       // per cluster at a time, as many clusters as can be resident together
       const int64_t clusters = std::max<int64_t>(1, std::min<int64_t>(Ly.rows, di.top_p_clusters));

@@ -19,6 +19,12 @@ enum : unsigned {
 // A wait longer than this is treated as a hang: the kernel records kDevTimeout
 // and unwinds instead of spinning forever.  Real waits are microseconds.
 constexpr unsigned long long kWaitLimitNs = 2000000000ull;  // 2 s
+// After a wait gave up, how long the kernel waits for copies it already
+// issued to land before it releases the shared memory they target.
+constexpr unsigned long long kDrainNs = 20000000ull;  // 20 ms
+// The fixed pause that stands in for that wait where no barrier can show it
+// (a copy counted on a barrier whose phase can no longer complete).
+constexpr unsigned kDrainPauseNs = 200000u;  // 200 us
 
 __device__ __forceinline__ uint32_t smem_addr(const void* p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));
@@ -119,6 +125,15 @@ __device__ __forceinline__ void tma_store_2d(const CUtensorMap* map, uint32_t sr
   asm volatile("cp.async.bulk.tensor.2d.global.shared::cta.tile.bulk_group [%0, {%2, %3}], [%1];" ::"l"(
                    reinterpret_cast<uint64_t>(map)),
                "r"(src), "r"(c0), "r"(c1)
+               : "memory");
+}
+
+// Untiled bulk copy of `bytes` (a multiple of 16; both addresses 16-byte
+// aligned) from global memory into this CTA's shared memory, completing on
+// mbarrier `bar` (which must expect the bytes).
+__device__ __forceinline__ void bulk_load_1d(uint32_t dst, const void* src, uint32_t bytes, uint32_t bar) {
+  asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(dst),
+               "l"(src), "r"(bytes), "r"(bar)
                : "memory");
 }
 

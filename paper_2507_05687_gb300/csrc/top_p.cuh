@@ -9,18 +9,21 @@
 // exp of y = z / temperature, the row maximum and the plain Gumbel-max winner
 // w0 over the whole vocabulary, and stored the fp32 logits z.
 //
-// A pass with one CTA per row (top_p_fast_kernel) first decides whether w0 is
-// in the nucleus: it is exactly when the mass of the logits strictly above
+// w0 is in the nucleus exactly when the mass of the logits strictly above
 // y_w0 is below the target (then y_w0 >= y*; otherwise the tokens above it
 // already reach the target and y* > y_w0).  A winner inside is the nucleus
 // winner too, its perturbed score beating every token; that is the case for
 // about a fraction top_p of the rows, and top_p = 1 needs no selection at all.
 // Masses are probabilities in 2^-40 fixed point, so no sum depends on the
-// order of the atomics that form it.
+// order of the atomics that form it.  A streaming pass over every row's
+// logits (top_p_fast_kernel) lists the rows whose winner may lie outside,
+// from fp32 sums within a proven margin of the exact mass.
 //
-// The other rows form a list, and a cluster of kTopPCtas CTAs takes one row
-// at a time (distributed shared memory; each CTA walks an interleaved eighth
-// of the row).  Since y* > y_w0, only logits above y_w0 matter:
+// A cluster of kTopPCtas CTAs takes one listed row at a time (distributed
+// shared memory; each CTA walks an interleaved eighth of the row).  Only the
+// logits above y_w0 matter; the first level's histogram of their exact masses
+// confirms the row (a row whose total falls short keeps its plain draw), and
+// then y* > y_w0:
 //   1. a histogram of their mass over 2048 buckets spanning [y_w0, max y]
 //      (at most 1/64 nat each); the bucket where the mass counted from the top
 //      reaches the target holds y*;
@@ -83,6 +86,7 @@ struct TopPShared {
   unsigned lcand, lbase;                    // this CTA's candidate count and its offset in the cluster's list
   float ystar;
   int full;                                 // the threshold is known but the candidates did not all fit
+  int skip;                                 // the row's exact mass above its winner is below the target
 };
 
 // Probability of tempered logit y in 2^-40 units, truncated toward zero: the
@@ -304,6 +308,9 @@ __global__ void __cluster_dims__(kTopPCtas, 1, 1) __launch_bounds__(kTopPThreads
           const unsigned long long before = __shfl_sync(0xffffffffu, inc - own, ln);
           sh.ra[0] = before;
           sh.ri[0] = ln;
+          // level 0 holds every logit above the winner: when even their exact
+          // mass falls short of the target, the winner is in the nucleus
+          if (tid == 0) sh.skip = L == 0 && !cross;
         }
         __syncthreads();
         if (tid == 0) {
@@ -327,12 +334,22 @@ __global__ void __cluster_dims__(kTopPCtas, 1, 1) __launch_bounds__(kTopPThreads
       cluster_sync();
       if (tid == 0) {
         if (!host) {
+          sh.skip = static_cast<int>(ld_shared_cluster(atk(&sh.skip, 0)));
           sh.lvl_b[L] = static_cast<int>(ld_shared_cluster(atk(&sh.lvl_b[L], 0)));
           sh.cum_before = ld_shared_cluster_u64(atk(&sh.cum_before, 0));
         }
         sh.lcand = 0u;
       }
       __syncthreads();
+      // A skipped row ends here, after one more cluster barrier: the other
+      // CTAs have just read the host's fields above, and the host must not
+      // move on (or, after its last row, exit, releasing the shared memory
+      // they read) before they have.  In a row that goes on, the host waits at
+      // the next cluster barrier below before it writes any of them again.
+      if (sh.skip) {
+        cluster_sync();
+        break;
+      }
       // gather the bucket's logits (and their range, in case they do not fit)
       // into this CTA's list; draw over the logits above the bucket (Gumbel-max
       // with the GEMM's noise: Philox4x32-10 word v mod 4 of counter
@@ -442,6 +459,7 @@ __global__ void __cluster_dims__(kTopPCtas, 1, 1) __launch_bounds__(kTopPThreads
       if (sh.full) break;
       ++L;
     }
+    if (sh.skip) continue;  // the plain draw (already written) stands
     const float ystar = sh.ystar;
     if (sh.full) {
       // the candidates are not all at hand: Gumbel-max over every y >= y*
@@ -604,100 +622,186 @@ __global__ void top_p_prep_kernel(const int* __restrict__ n_valid, const int* __
   }
 }
 
-// Is each row's plain winner in its nucleus?  The mass strictly above the
-// winner (2^-40 fixed point, exact integer sums), against the target
-// top_p_target: the winner is in exactly when that mass is below the target;
-// a row whose winner is outside goes to the list top_p_kernel works through,
-// with its target.  A row is cut into `slices` interleaved slices, one CTA
-// each (more than one for batches with too few rows to fill the GPU): each
-// adds its slice's mass into the row's accumulator with a device-wide atomic,
-// fences, and counts itself done; the CTA that completes the count makes the
-// decision (nothing waits for anything).  row_above / row_done start at 0
-// (top_p_prep_kernel clears them).
-__global__ void __launch_bounds__(kTopPThreads)
+// Which rows' plain winner may lie outside its nucleus?  The winner is in
+// exactly when the mass strictly above it, in the 2^-40 fixed point of
+// top_p_mass, is below top_p_target.  This pass only sorts the rows: it sums
+// the same per-logit values p_v 2^40 in fp32 over each thread's 32 logits of a
+// chunk and adds those sums, truncated, as integers.  Against the exact
+// fixed-point mass E that approximation A is off by at most 31 u A' (the fp32
+// sums of 32 positive terms, u = 2^-24, A' <= 2^41) plus one unit per logit
+// and per sum, so |A - E| < 2^23 + 2 V = top_p_margin(V): a row with A plus
+// that margin below the target certainly keeps its winner, and every other row goes to the list
+// top_p_kernel works through, which confirms it with the exact mass first
+// (the total of its level-0 histogram) and leaves a row whose exact mass
+// falls short with its plain draw.
+//
+// The stored logits stream through shared memory.  Each row is cut into
+// chunks of kFastChunk logits, the chunks of all rows are numbered row by
+// row, and each CTA takes one contiguous range of them (so the grid stays
+// busy whatever the number of rows).  One thread keeps kFastStages chunks in
+// flight with bulk copies that complete on a per-stage mbarrier, while all
+// threads work through the oldest (each thread 32 logits of a chunk, 16-byte
+// shared loads).  When the CTA leaves a row it adds its sum for the row into
+// the row's accumulator (integer device atomics, so the order does not
+// matter), fences, and
+// adds the number of chunks it covered to the row's count; the CTA that
+// completes the count decides (nothing waits for anything).  row_above /
+// row_done start at 0 (top_p_prep_kernel clears them).  Every wait is
+// bounded: on expiry the CTA sets kDevTimeout, lets the copies it issued
+// land (bounded again) and returns.
+constexpr int kFastChunk = 8192;   // logits per stage (32 KB)
+
+// The bound on |A - E| above for a vocabulary of V.
+inline unsigned long long top_p_margin(int64_t V) { return (1ull << 23) + 2ull * static_cast<unsigned long long>(V); }
+constexpr int kFastStages = 3;
+constexpr int kFastSmem = kFastStages * kFastChunk * 4 + kFastStages * 8;
+static_assert(kFastChunk % (kTopPWarps * 128) == 0, "whole float4 rounds per warp");
+
+__global__ void __launch_bounds__(kTopPThreads, 2)
     top_p_fast_kernel(const float* __restrict__ z, int64_t ldz, int V, const int* __restrict__ n_valid,
-                      int slices, const float* __restrict__ lse_r, const float* __restrict__ y0_r, float inv_temp,
+                      const float* __restrict__ lse_r, const float* __restrict__ y0_r, float inv_temp,
                       float top_p, unsigned long long* __restrict__ row_above, unsigned* __restrict__ row_done,
                       int* __restrict__ slow_rows, unsigned long long* __restrict__ slow_target,
-                      unsigned* __restrict__ n_slow) {
-  constexpr int kUnroll = 8;
+                      unsigned* __restrict__ n_slow, unsigned long long margin, unsigned* status) {
+  constexpr int kSeg = kFastChunk / kTopPWarps;  // logits of a chunk one warp reads
+  constexpr int kPer = kSeg / 128;               // float4 per lane
+  extern __shared__ __align__(128) unsigned char fast_smem[];
+  float* ring = reinterpret_cast<float*>(fast_smem);
+  uint64_t* full = reinterpret_cast<uint64_t*>(fast_smem + kFastStages * kFastChunk * 4);
   __shared__ unsigned long long ra[kTopPWarps];
-  __shared__ float wbuf[kTopPWarps][32 * 4 * kUnroll];  // one warp's logits above the winner in a round
+  __shared__ int never;  // the waits here have no abort flag: never set
   const int tid = threadIdx.x;
   const int lane = tid & 31;
-  float* buf = wbuf[tid >> 5];
+  const int warp = tid >> 5;
   const int nv = *n_valid;
-  const int groups = (V + 3) / 4;
-  const int stride = slices * kTopPThreads;
-  const int64_t items = static_cast<int64_t>(nv) * slices;
-  for (int64_t it = blockIdx.x; it < items; it += gridDim.x) {
-    const int r = static_cast<int>(it / slices);
-    const int sl = static_cast<int>(it - static_cast<int64_t>(r) * slices);
-    const float4* zq = reinterpret_cast<const float4*>(z + static_cast<int64_t>(r) * ldz);
-    const float lse = lse_r[r], y0 = y0_r[r];
-    unsigned long long above = 0ull;
-    // whole rounds: most logits lie below the winner, so each warp gathers the
-    // ones above it (ballot + prefix count) and computes their masses with all
-    // lanes busy instead of a few lanes at a time
-    // (the test uses the warp's last lane, so that every lane of a warp runs the
-    // same rounds: the ballots need the whole warp)
-    int g0 = sl * kTopPThreads + tid;
-    for (; g0 - lane + 31 + (kUnroll - 1) * stride < groups - 1; g0 += kUnroll * stride) {
-      float4 q[kUnroll];
-#pragma unroll
-      for (int u = 0; u < kUnroll; ++u) q[u] = __ldcg(zq + g0 + u * stride);
-      int cnt = 0;
-#pragma unroll
-      for (int u = 0; u < kUnroll; ++u) {
-        const float yy[4] = {q[u].x * inv_temp, q[u].y * inv_temp, q[u].z * inv_temp, q[u].w * inv_temp};
-#pragma unroll
-        for (int k = 0; k < 4; ++k) {
-          const bool a = yy[k] > y0;
-          const unsigned bal = __ballot_sync(0xffffffffu, a);
-          if (a) buf[cnt + __popc(bal & ((1u << lane) - 1u))] = yy[k];
-          cnt += __popc(bal);
-        }
-      }
-      __syncwarp();
-      for (int i = lane; i < cnt; i += 32) above += top_p_mass(buf[i], lse);
-      __syncwarp();
-    }
-    // the rest, one group at a time (the last group may be partial)
-    for (; g0 < groups; g0 += stride) {
-      const float4 q = __ldcg(zq + g0);
-      const float zz[4] = {q.x, q.y, q.z, q.w};
-#pragma unroll
-      for (int k = 0; k < 4; ++k) {
-        const float y = zz[k] * inv_temp;
-        if (4 * g0 + k < V && y > y0) above += top_p_mass(y, lse);
-      }
-    }
+  const int cpr = (V + kFastChunk - 1) / kFastChunk;  // chunks per row
+  const int64_t items = static_cast<int64_t>(nv) * cpr;
+  const int64_t per = (items + gridDim.x - 1) / gridDim.x;
+  const int64_t i0 = static_cast<int64_t>(blockIdx.x) * per;
+  const int64_t i1 = min(items, i0 + per);
+  if (i0 >= i1) return;
+  if (tid == 0) {
+    for (int s = 0; s < kFastStages; ++s) mbar_init(smem_addr(&full[s]), 1);
+    never = 0;
+    fence_mbar_init();
+  }
+  __syncthreads();
+  const unsigned long long target = top_p_target(top_p);
+  // thread 0: the copy of chunk `it` into stage s (whole 16-byte groups: the
+  // row's storage, ldz >= V rounded up to 64, covers the last partial group,
+  // whose extra lanes are skipped below)
+  auto issue = [&](int64_t it, int s) {
+    const int64_t r = it / cpr;
+    const int c0 = static_cast<int>(it - r * cpr) * kFastChunk;
+    const uint32_t bytes = static_cast<uint32_t>((min(kFastChunk, V - c0) + 3) & ~3) * 4u;
+    const uint32_t bar = smem_addr(&full[s]);
+    mbar_arrive_expect_tx(bar, bytes);
+    bulk_load_1d(smem_addr(ring + s * kFastChunk), z + r * ldz + c0, bytes, bar);
+  };
+  if (tid == 0)
+    for (int s = 0; s < kFastStages && i0 + s < i1; ++s) issue(i0 + s, s);
+
+  int64_t row = i0 / cpr;
+  unsigned long long above = 0ull;
+  unsigned covered = 0;
+  // this CTA's mass of `row` and its chunk count into the row's accumulators
+  auto flush = [&]() {
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) above += __shfl_xor_sync(0xffffffffu, above, o);
-    if ((tid & 31) == 0) ra[tid >> 5] = above;
+    if (lane == 0) ra[warp] = above;
     __syncthreads();
     if (tid == 0) {
-      above = 0ull;
-      for (int w = 0; w < kTopPWarps; ++w) above += ra[w];
-      bool decide = true;
-      if (slices > 1) {
-        atomicAdd(&row_above[r], above);
+      unsigned long long m = 0ull;
+      for (int w = 0; w < kTopPWarps; ++w) m += ra[w];
+      atomicAdd(&row_above[row], m);
+      __threadfence();
+      if (atomicAdd(&row_done[row], covered) + covered == static_cast<unsigned>(cpr)) {
         __threadfence();
-        decide = atomicAdd(&row_done[r], 1u) == static_cast<unsigned>(slices - 1);
-        if (decide) {
-          __threadfence();
-          above = atomicAdd(&row_above[r], 0ull);  // every slice's mass (each fenced before counting itself)
+        const unsigned long long total = atomicAdd(&row_above[row], 0ull);  // every CTA's sum, each fenced first
+        if (total + margin >= target) {
+          const unsigned k = atomicAdd(n_slow, 1u);
+          slow_rows[k] = static_cast<int>(row);
+          slow_target[k] = target;
         }
-      }
-      const unsigned long long target = top_p_target(top_p);
-      if (decide && above >= target) {
-        const unsigned k = atomicAdd(n_slow, 1u);
-        slow_rows[k] = r;
-        slow_target[k] = target;
       }
     }
     __syncthreads();
+    above = 0ull;
+    covered = 0;
+  };
+
+  int64_t it = i0;
+  bool ok = true;
+  for (; it < i1; ++it) {
+    const int k = static_cast<int>(it - i0);
+    const int s = k % kFastStages;
+    const int64_t r = it / cpr;
+    if (r != row) {  // uniform across the CTA
+      flush();
+      row = r;
+    }
+    const bool got = mbar_wait(smem_addr(&full[s]), static_cast<uint32_t>(k / kFastStages) & 1u, &never);
+    if (!__syncthreads_and(got)) {
+      ok = false;
+      break;
+    }
+    const int c0 = static_cast<int>(it - r * cpr) * kFastChunk;
+    const int n = min(kFastChunk, V - c0);  // logits of this chunk inside the row
+    const float y0 = y0_r[r], lse = lse_r[r];
+    const float* seg = ring + s * kFastChunk + warp * kSeg;
+    float4 q[kPer];
+#pragma unroll
+    for (int j = 0; j < kPer; ++j) q[j] = reinterpret_cast<const float4*>(seg)[lane + 32 * j];
+    // p_v 2^40 exactly as top_p_mass forms it, summed over the logits above the winner
+    const float kLog2e = 1.4426950408889634f;
+    float acc = 0.f;
+    if (n == kFastChunk) {
+#pragma unroll
+      for (int j = 0; j < kPer; ++j) {
+        const float zz[4] = {q[j].x, q[j].y, q[j].z, q[j].w};
+#pragma unroll
+        for (int kk = 0; kk < 4; ++kk) {
+          const float y = zz[kk] * inv_temp;
+          const float f = fast_exp2((y - lse) * kLog2e) * 1099511627776.0f;
+          acc += y > y0 ? f : 0.f;
+        }
+      }
+    } else {  // the row's last, partial chunk
+#pragma unroll
+      for (int j = 0; j < kPer; ++j) {
+        const float zz[4] = {q[j].x, q[j].y, q[j].z, q[j].w};
+        const int e0 = warp * kSeg + 4 * (lane + 32 * j);
+#pragma unroll
+        for (int kk = 0; kk < 4; ++kk) {
+          const float y = zz[kk] * inv_temp;
+          const float f = fast_exp2((y - lse) * kLog2e) * 1099511627776.0f;
+          acc += e0 + kk < n && y > y0 ? f : 0.f;
+        }
+      }
+    }
+    above += __float2ull_rz(acc);
+    ++covered;
+    __syncthreads();  // every warp is done with stage s
+    if (tid == 0 && it + kFastStages < i1) issue(it + kFastStages, s);
   }
+  if (ok) {
+    flush();
+    return;
+  }
+  // a copy did not arrive in time: report it, let the copies issued for the
+  // chunks not yet consumed land (bounded), and give up on the rest
+  if (tid == 0) {
+    atomicOr(status, kDevTimeout);
+    bool drained = true;
+    for (int64_t j = it; j < i1 && j < it + kFastStages; ++j) {
+      const int kj = static_cast<int>(j - i0);
+      if (!mbar_wait(smem_addr(&full[kj % kFastStages]), static_cast<uint32_t>(kj / kFastStages) & 1u, &never,
+                     kDrainNs))
+        drained = false;
+    }
+    if (!drained) __nanosleep(kDrainPauseNs);
+  }
+  __syncthreads();
 }
 
 // Masked rows (and rows past the workspace's row capacity) of a top-p draw: token -1, log-prob 0.

@@ -213,3 +213,24 @@ def test_top_p_tiny_vocabularies(V):
         tok, lp = _draw(Hb, Wb, m, 1.0, top_p, 12, 3)
         assert np.all(tok[m != 0] >= 0) and np.all(tok[m != 0] < V)
         _compare(Hb, Wb, m, 1.0, top_p, 12, 3, tok, lp)
+
+
+@pytest.mark.parametrize("top_p", [0.3, 0.9])
+def test_every_row_listed_gives_the_same_draws(monkeypatch, top_p):
+    """The streaming pass lists only rows whose winner may lie outside the
+    nucleus (from fp32 sums within a bound of the exact mass); the selection
+    confirms each listed row with the exact mass and leaves a row whose mass
+    above the winner falls short with its plain draw.  With every row listed
+    (a test hook), that confirmation decides all of them: the draws and
+    log-probs are the same bits as with the bound, on a flat and a peaked
+    distribution and a decode step of the full vocabulary."""
+    cases = [wl.Workload("p", 2, 3, 90, 192, 5000, "uniform", 1, 90, seed=wl.SEED_BASE + 3300, w_std=0.08),
+             wl.Workload("p", 2, 3, 90, 192, 4097, "uniform", 1, 90, seed=wl.SEED_BASE + 3301, w_std=0.5),
+             wl.DECODE_WORKLOADS["decode256_8b"]]
+    for w in cases:
+        Hb, Wb, m = wl.gen_hidden(w), wl.gen_weight(w), wl.gen_mask(w)
+        want = _draw(Hb, Wb, m, 1.0, top_p, 77, 5)
+        monkeypatch.setenv("GRPO_TEST_TOP_P_LIST_ALL", "1")
+        got = _draw(Hb, Wb, m, 1.0, top_p, 77, 5)
+        monkeypatch.delenv("GRPO_TEST_TOP_P_LIST_ALL")
+        assert np.array_equal(got[0], want[0]) and np.array_equal(got[1], want[1])
