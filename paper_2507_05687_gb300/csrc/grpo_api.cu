@@ -936,7 +936,9 @@ grpo_status grpo_sample_tokens_top_p(const uint16_t* H, const uint16_t* W, const
         top_p_kernel<<<rb, kTopPThreads, 0, s>>>(
             at<float>(ws, Ly.z), Ly.ldz, static_cast<int>(V), reinterpret_cast<const int*>(n_slow),
             at<int>(ws, Ly.slow_rows), at<unsigned long long>(ws, Ly.slow_tgt), at<int>(ws, Ly.cidx), lse_r, y0_r,
-            hi_r, 1.f / temperature, static_cast<uint32_t>(seed), static_cast<uint32_t>(seed >> 32),
+            hi_r, at<float>(ws, Ly.best_s), at<int>(ws, Ly.best_c), at<float>(ws, Ly.best_z),
+            static_cast<int>(Ly.nsplit), Ly.rows, Ly.lse_tiles, 1.f / temperature, static_cast<uint32_t>(seed),
+            static_cast<uint32_t>(seed >> 32),
             static_cast<uint32_t>(offset), static_cast<uint32_t>(offset >> 32), tokens_out, logp_out,
             at<unsigned>(ws, Ly.status));
       if (e == cudaSuccess) e = cudaGetLastError();

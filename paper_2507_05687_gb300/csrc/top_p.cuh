@@ -28,23 +28,25 @@
 //      (at most 1/64 nat each); the bucket where the mass counted from the top
 //      reaches the target holds y*;
 //   2. a second walk gathers that bucket's logits as candidates (every CTA
-//      receives all of them) and, on the way, keeps the best perturbed score
-//      y + G over the logits above the bucket, which are all in the nucleus
-//      (G: the GEMM's noise, Philox4x32-10 word v mod 4 of counter
-//      (v div 4, t, offset), key seed, fp32 operations, the lowest v on ties);
-//      a bucket with more than kTopPCand logits is histogrammed again over its
-//      own range first (one whose logits are all equal is taken whole: ties
-//      stay together);
+//      receives all of them); a bucket with more than kTopPCand logits is
+//      histogrammed again over its own range first (one whose logits are all
+//      equal is taken whole: ties stay together);
 //   3. y* is the largest candidate y whose mass together with that of the
 //      candidates above it reaches what the target still needs (an exact rank
-//      count, the candidates split over the cluster), and the draw is the best
-//      of the score from step 2 and the scores of the candidates >= y*.
+//      count, the candidates split over the cluster);
+//   4. the draw is the best perturbed score y + G over y >= y* (G: the GEMM's
+//      noise, Philox4x32-10 word v mod 4 of counter (v div 4, t, offset), key
+//      seed, fp32 operations, the lowest v on ties).  The sampling GEMM kept
+//      each split entry's best score over all its tokens; an entry whose
+//      winner has y >= y* contributes it as it is, and only the other entries
+//      (about 1 - top_p of them where the distribution is flat) are walked.
 // Every reduction has a fixed order or is exact, so a row's draw is
 // deterministic.
 #pragma once
 
 #include <stdint.h>
 
+#include "gemm_tc.cuh"
 #include "ptx.cuh"
 #include "small_kernels.cuh"
 
@@ -56,6 +58,8 @@ constexpr int kTopPBuckets = 2048;
 constexpr int kTopPCand = 1024;    // candidates resolved exactly in shared memory
 constexpr int kTopPLevels = 6;     // histogram levels before the candidates fit
 constexpr int kTopPWarps = kTopPThreads / 32;
+// column halves of a tile in the sampling GEMM's split entries (one per epilogue warp of a lane quarter)
+constexpr int kSampleHalves = EpiShape<kEpiSample>::kHalves;
 static_assert(kTopPBuckets == kTopPCtas * kTopPThreads, "one histogram bucket per thread of the cluster in the merge");
 
 // Shared memory of one CTA.  The fields marked "host" are used in CTA 0 of
@@ -65,12 +69,10 @@ struct TopPShared {
     unsigned long long hist[kTopPBuckets];  // histogram pass: this CTA's histogram; host: then the merged one
     struct {                                // gather pass: this CTA's candidates before they are broadcast
       float y[kTopPCand];
-      int v[kTopPCand];
     } loc;
   };
   float cy[kTopPCand];                      // the cluster's candidates: every CTA holds all of them
   unsigned long long cq[kTopPCand];
-  int cv[kTopPCand];
   unsigned long long scan[kTopPThreads];    // host: per-thread bucket-range sums of the scan
   // host, one value per CTA: the range of its candidates, its part of the threshold search, its best draw
   uint32_t slot_lo[kTopPCtas], slot_hi[kTopPCtas], slot_r[kTopPCtas], slot_f[kTopPCtas], slot_g[kTopPCtas],
@@ -217,9 +219,10 @@ __global__ void __cluster_dims__(kTopPCtas, 1, 1) __launch_bounds__(kTopPThreads
     top_p_kernel(const float* __restrict__ z, int64_t ldz, int V, const int* __restrict__ n_slow,
                  const int* __restrict__ slow_rows, const unsigned long long* __restrict__ slow_target,
                  const int* __restrict__ cidx, const float* __restrict__ lse_r, const float* __restrict__ y0_r,
-                 const float* __restrict__ hi_r, float inv_temp, uint32_t seed_lo, uint32_t seed_hi,
-                 uint32_t off_lo, uint32_t off_hi, int32_t* __restrict__ tokens, float* __restrict__ logp,
-                 unsigned* status) {
+                 const float* __restrict__ hi_r, const float* __restrict__ best_s, const int* __restrict__ best_c,
+                 const float* __restrict__ best_z, int nsplit, long ldp, int unit_tiles, float inv_temp,
+                 uint32_t seed_lo, uint32_t seed_hi, uint32_t off_lo, uint32_t off_hi, int32_t* __restrict__ tokens,
+                 float* __restrict__ logp, unsigned* status) {
   __shared__ TopPShared sh;
   const int tid = threadIdx.x;
   const int rank = static_cast<int>(cluster_ctarank());
@@ -246,8 +249,8 @@ __global__ void __cluster_dims__(kTopPCtas, 1, 1) __launch_bounds__(kTopPThreads
     // chosen buckets of the levels before; pick the bucket where the mass from
     // the top reaches the target; gather that bucket's logits as candidates
     // and, on the way, draw over the logits above it (all in the nucleus).
-    float bs = -INFINITY, by = 0.f;  // this thread's best perturbed score, its token and logit
-    int bv = -1;
+    float bs, by;  // this thread's best perturbed score, its token and logit (the draw below)
+    int bv;
     int L = 0;
     for (;;) {
       __syncthreads();
@@ -351,49 +354,17 @@ __global__ void __cluster_dims__(kTopPCtas, 1, 1) __launch_bounds__(kTopPThreads
         break;
       }
       // gather the bucket's logits (and their range, in case they do not fit)
-      // into this CTA's list; draw over the logits above the bucket (Gumbel-max
-      // with the GEMM's noise: Philox4x32-10 word v mod 4 of counter
-      // (v div 4, t, offset), fp32 operations; along a thread's walk v grows, so
-      // a strict > keeps the lowest v of equal scores)
+      // into this CTA's list
       float lo = INFINITY, hi2 = -INFINITY;
-      bs = -INFINITY;
-      bv = -1;
-      by = 0.f;
       top_p_groups<4>(zr, V, rank, [&](int g, float4 q) {
         const float yy[4] = {q.x * inv_temp, q.y * inv_temp, q.z * inv_temp, q.w * inv_temp};
-        int cls[4];
-        bool above = false;
 #pragma unroll
         for (int k = 0; k < 4; ++k) {
-          cls[k] = 4 * g + k < V && yy[k] > y0 ? top_p_class(sh, yy[k], L + 1) : 0;
-          above |= cls[k] == 1;
-        }
-        if (above) {
-          const uint4 w = philox4x32_10(make_uint4(static_cast<uint32_t>(g), static_cast<uint32_t>(t), off_lo, off_hi),
-                                        seed_lo, seed_hi);
-          const uint32_t ws[4] = {w.x, w.y, w.z, w.w};
-#pragma unroll
-          for (int k = 0; k < 4; ++k) {
-            if (cls[k] == 1) {
-              const float sc = yy[k] + gumbel_of(ws[k]);
-              if (sc > bs) {
-                bs = sc;
-                bv = 4 * g + k;
-                by = yy[k];
-              }
-            }
-          }
-        }
-#pragma unroll
-        for (int k = 0; k < 4; ++k) {
-          if (cls[k] == 2) {
+          if (4 * g + k < V && yy[k] > y0 && top_p_in(sh, yy[k], L + 1)) {
             lo = fminf(lo, yy[k]);
             hi2 = fmaxf(hi2, yy[k]);
             const unsigned i = atomicAdd(&sh.lcand, 1u);
-            if (i < static_cast<unsigned>(kTopPCand)) {
-              sh.loc.y[i] = yy[k];
-              sh.loc.v[i] = 4 * g + k;
-            }
+            if (i < static_cast<unsigned>(kTopPCand)) sh.loc.y[i] = yy[k];
           }
         }
       });
@@ -411,12 +382,10 @@ __global__ void __cluster_dims__(kTopPCtas, 1, 1) __launch_bounds__(kTopPThreads
         for (unsigned i = tid; i < n && base + i < static_cast<unsigned>(kTopPCand); i += kTopPThreads) {
           const float y = sh.loc.y[i];
           const unsigned long long m = top_p_mass(y, lse);
-          const int v = sh.loc.v[i];
 #pragma unroll
           for (int k = 0; k < kTopPCtas; ++k) {
             st_shared_cluster(atk(&sh.cy[base + i], k), __float_as_uint(y));
             st_shared_cluster_u64(atk(&sh.cq[base + i], k), m);
-            st_shared_cluster(atk(&sh.cv[base + i], k), static_cast<uint32_t>(v));
           }
         }
       }
@@ -460,46 +429,50 @@ __global__ void __cluster_dims__(kTopPCtas, 1, 1) __launch_bounds__(kTopPThreads
       ++L;
     }
     if (sh.skip) continue;  // the plain draw (already written) stands
+    // The draw: the best perturbed score over the logits y >= y*, the lowest
+    // token on ties.  The sampling GEMM kept, for every split entry (a
+    // vocabulary unit of unit_tiles tiles, one column half of each tile), its
+    // best score over all of the entry's tokens.  Where that winner lies in
+    // the nucleus it is the entry's best over its nucleus tokens too; only the
+    // other entries are walked, with the GEMM's noise (Philox4x32-10 word v
+    // mod 4 of counter (v div 4, t, offset), fp32 operations).
     const float ystar = sh.ystar;
-    if (sh.full) {
-      // the candidates are not all at hand: Gumbel-max over every y >= y*
-      bs = -INFINITY;
-      bv = -1;
-      by = 0.f;
-      top_p_groups<4>(zr, V, rank, [&](int g, float4 q) {
+    bs = -INFINITY;
+    bv = -1;
+    by = 0.f;
+    for (int e = rank; e < nsplit; e += kTopPCtas) {
+      const long at = static_cast<long>(e) * ldp + r;
+      const float bz = best_z[at];
+      if (bz >= ystar) {
+        if (tid == 0 && top_p_better(best_s[at], best_c[at], bs, bv)) {
+          bs = best_s[at];
+          bv = best_c[at];
+          by = bz;
+        }
+        continue;
+      }
+      const int c0 = (e / kSampleHalves) * unit_tiles * kTileN + (e % kSampleHalves) * (kTileN / kSampleHalves);
+      constexpr int kGroupsPerTile = kTileN / kSampleHalves / 4;  // 4-token groups of one tile's column half
+      for (int gi = tid; gi < unit_tiles * kGroupsPerTile; gi += kTopPThreads) {
+        const int v0 = c0 + (gi / kGroupsPerTile) * kTileN + 4 * (gi % kGroupsPerTile);
+        if (v0 >= V) continue;
+        const float4 q = __ldcg(reinterpret_cast<const float4*>(zr + v0));
         const float yy[4] = {q.x * inv_temp, q.y * inv_temp, q.z * inv_temp, q.w * inv_temp};
-        if (!(yy[0] >= ystar || yy[1] >= ystar || yy[2] >= ystar || yy[3] >= ystar)) return;
-        const uint4 w = philox4x32_10(make_uint4(static_cast<uint32_t>(g), static_cast<uint32_t>(t), off_lo, off_hi),
+        if (!(yy[0] >= ystar || yy[1] >= ystar || yy[2] >= ystar || yy[3] >= ystar)) continue;
+        const uint4 w = philox4x32_10(make_uint4(static_cast<uint32_t>(v0 >> 2), static_cast<uint32_t>(t), off_lo,
+                                                 off_hi),
                                       seed_lo, seed_hi);
         const uint32_t ws[4] = {w.x, w.y, w.z, w.w};
 #pragma unroll
         for (int k = 0; k < 4; ++k) {
-          const int v = 4 * g + k;
+          const int v = v0 + k;
           if (v < V && yy[k] >= ystar) {
             const float sc = yy[k] + gumbel_of(ws[k]);
-            if (sc > bs) {
+            if (top_p_better(sc, v, bs, bv)) {
               bs = sc;
               bv = v;
               by = yy[k];
             }
-          }
-        }
-      });
-    } else {
-      // the candidates at or above y*, this CTA's share of them
-      const int nc = static_cast<int>(sh.ncand);
-      for (int i = rank + kTopPCtas * tid; i < nc; i += kTopPCtas * kTopPThreads) {
-        const float y = sh.cy[i];
-        if (y >= ystar) {
-          const int v = sh.cv[i];
-          const uint4 w = philox4x32_10(
-              make_uint4(static_cast<uint32_t>(v >> 2), static_cast<uint32_t>(t), off_lo, off_hi), seed_lo, seed_hi);
-          const uint32_t ws[4] = {w.x, w.y, w.z, w.w};
-          const float sc = y + gumbel_of(ws[v & 3]);
-          if (top_p_better(sc, v, bs, bv)) {
-            bs = sc;
-            bv = v;
-            by = y;
           }
         }
       }
