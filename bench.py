@@ -34,10 +34,11 @@ import workloads as wl  # noqa: E402
 
 METRIC = "response tokens/s for GRPO logprob+loss fwd+bwd; % of dense bf16 peak"
 GOLDEN = {"fwdbwd_8b": "batch8b", "logprob3_8b": "batch8b", "long_8b": "long_8b", "ragged_8b": "ragged_8b"}
-# the GEMM kernels and the launch parameters (raster, cache hints) that set their DRAM traffic
+# the GEMM kernels, their launch parameters (raster, cache hints, chunk width)
+# and the kept-logits dZ pass: what sets the DRAM traffic of the kernels the
+# roofline reports
 KERNEL_SOURCES = ["paper_2507_05687_gb300/csrc/gemm_tc.cuh", "paper_2507_05687_gb300/csrc/ptx.cuh",
-                  "paper_2507_05687_gb300/csrc/grpo_api.cu", "paper_2507_05687_gb300/csrc/small_kernels.cuh",
-                  "paper_2507_05687_gb300/csrc/dz_rows.cuh"]
+                  "paper_2507_05687_gb300/csrc/gemm_launch.cuh", "paper_2507_05687_gb300/csrc/dz_rows.cuh"]
 KIND_NAMES = ["advantages", "compact", "lse_gemm", "logp_merge", "loss", "dz_gemm", "dh_gemm", "dw_gemm",
               "dh_rows", "adamw", "sample_gemm", "transpose", "dz_logits", "top_p"]
 KERNELS_PER_SCOPE = {1: 4, 4: 2}  # compaction scope = 4 kernels, loss scope = 2 kernels; others 1
