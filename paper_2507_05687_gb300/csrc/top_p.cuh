@@ -92,15 +92,13 @@ struct TopPShared {
 };
 
 // Probability of tempered logit y in 2^-40 units, truncated toward zero: the
-// float p * 2^40 (< 2^41) turned into an integer from its fields (significand
-// shifted by the exponent), which is exact and cheaper than a 64-bit convert.
+// float p * 2^40 converted exactly (one truncating conversion; measured a
+// little faster in the selection than building the integer from the float's
+// fields).  A value that is not finite or not below 2^41 gives 0.
 __device__ __forceinline__ unsigned long long top_p_mass(float y, float lse) {
   const float kLog2e = 1.4426950408889634f;
-  const uint32_t b = __float_as_uint(fast_exp2((y - lse) * kLog2e) * 1099511627776.0f);
-  const int e = static_cast<int>((b >> 23) & 0xFFu) - 150;  // value = significand * 2^e
-  const unsigned long long m = static_cast<unsigned long long>((b & 0x7FFFFFu) | 0x800000u);
-  if (e <= -24 || e > 40 || (b >> 31)) return 0ull;  // below 1, not finite, or negative
-  return e >= 0 ? m << e : m >> (-e);
+  const float f = fast_exp2((y - lse) * kLog2e) * 1099511627776.0f;
+  return f < 2199023255552.0f ? __float2ull_rz(f) : 0ull;
 }
 
 // Adds q to a 64-bit histogram bucket with 32-bit shared atomics: q's low word
