@@ -125,5 +125,24 @@ inline int group_m(int which) {
   return g[which];
 }
 
+// Raster along N for GEMM `which` (LSE, dZ, dH, dW): when > 0, groups of at
+// most this many N units keep their B tiles in L2 while the group sweeps
+// every M tile (group_m is then unused).  The dZ GEMM's B is a W chunk (134 MB
+// at 16,384 columns) and its A the gathered hidden states (160 MB at 19,572
+// rows): grouped by 8 M tiles it reads the W chunk once per group (10 times
+// per launch at 77 M tiles), grouped by 16 N tiles (32 MB of W) it reads W
+// once and A once per group (4 times).  dH and dW would read their larger A
+// (the dZ chunk) that many times instead, so they keep the M groups.
+// GRPO_GROUP_N="a,b,c,d" overrides (0: group along M).
+inline int group_n(int which) {
+  int g[4] = {0, 16, 0, 0};
+  if (const char* e = std::getenv("GRPO_GROUP_N")) {
+    int v[4];
+    if (std::sscanf(e, "%d,%d,%d,%d", &v[0], &v[1], &v[2], &v[3]) == 4)
+      for (int i = 0; i < 4; ++i) g[i] = v[i] >= 0 ? v[i] : g[i];
+  }
+  return g[which];
+}
+
 }  // namespace launch
 }  // namespace grpo

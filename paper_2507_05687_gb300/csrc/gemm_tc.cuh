@@ -127,6 +127,8 @@ struct GemmArgs {
   int n_per_unit;       // consecutive N tiles one CTA (pair) walks as one work unit
   int n_heads;          // B matrices (LM heads) swept against the same A, 1..kMaxHeads
   int group_m;          // raster: at most this many M tiles per group sharing the same N sweep
+  int group_n;          // raster along N instead (when > 0): at most this many N units per group,
+                        // their B tiles shared while the group sweeps every M tile
   int a_hint, b_hint;   // L2 eviction policy of A / B loads (kHint*)
   unsigned* status;     // device status word
   unsigned long long wait_ns;  // bound of every pipeline wait (0: kWaitLimitNs)
@@ -170,7 +172,7 @@ struct GemmArgs {
 
 struct TileSched {
   int m_tiles, n_tiles, units_head, units_n, total, k_blocks, m_rows;
-  int group;  // M tiles per raster group (balanced, at most GemmArgs::group_m)
+  int group;  // M tiles (or, with GemmArgs::group_n, N units) per raster group, balanced
 };
 
 __device__ __forceinline__ TileSched make_sched(const GemmArgs& a, int tile_m) {
@@ -184,18 +186,29 @@ __device__ __forceinline__ TileSched make_sched(const GemmArgs& a, int tile_m) {
   s.units_n = s.units_head * max(1, a.n_heads);
   s.total = s.m_tiles * s.units_n;
   s.k_blocks = (K + kBK - 1) / kBK;
-  // as few groups as group_m allows, of near-equal height: a last group of a
-  // few M tiles would stream all of B again for a sliver of the work
-  const int gmax = max(1, a.group_m);
-  const int ngroups = max(1, (s.m_tiles + gmax - 1) / gmax);
-  s.group = max(1, (s.m_tiles + ngroups - 1) / ngroups);
+  // as few groups as group_m (group_n) allows, of near-equal height: a last
+  // group of a few M tiles would stream all of B again for a sliver of the work
+  const int along = a.group_n > 0 ? s.units_n : s.m_tiles;
+  const int gmax = max(1, a.group_n > 0 ? a.group_n : a.group_m);
+  const int ngroups = max(1, (along + gmax - 1) / gmax);
+  s.group = max(1, (along + ngroups - 1) / ngroups);
   return s;
 }
 
 // Work unit u -> (m tile, n unit).  Groups of s.group consecutive M tiles
 // sweep the N units together, so the CTAs running at the same time share B
 // tiles (and A tiles) in L2.
-__device__ __forceinline__ void unit_coords(const GemmArgs&, const TileSched& s, int u, int& mt, int& un) {
+__device__ __forceinline__ void unit_coords(const GemmArgs& a, const TileSched& s, int u, int& mt, int& un) {
+  if (a.group_n > 0) {  // groups of s.group N units sweep every M tile
+    const int per_group = s.group * s.m_tiles;
+    const int g = u / per_group;
+    const int first = g * s.group;
+    const int gn = min(s.group, s.units_n - first);
+    const int w = u - g * per_group;
+    un = first + w % gn;
+    mt = w / gn;
+    return;
+  }
   const int per_group = s.group * s.units_n;
   const int g = u / per_group;
   const int first = g * s.group;

@@ -1049,6 +1049,7 @@ grpo_status loss_impl(const uint16_t* H, const uint16_t* W, const int32_t* targe
       a.b_off_n = static_cast<int>(c0);
       a.n_per_unit = units_n(0);
       a.group_m = group_m(1);
+      a.group_n = group_n(1);
       l2_hints(1, &a.a_hint, &a.b_hint);
       a.status = status;
       a.yc = at<int>(ws, Ly.yc);
