@@ -621,12 +621,12 @@ __global__ void top_p_prep_kernel(const int* __restrict__ n_valid, const int* __
 // bounded: on expiry the CTA sets kDevTimeout, lets the copies it issued
 // land (bounded again) and returns.
 constexpr int kFastChunk = 8192;   // logits per stage (32 KB)
-
-// The bound on |A - E| above for a vocabulary of V.
-inline unsigned long long top_p_margin(int64_t V) { return (1ull << 23) + 2ull * static_cast<unsigned long long>(V); }
 constexpr int kFastStages = 3;
 constexpr int kFastSmem = kFastStages * kFastChunk * 4 + kFastStages * 8;
 static_assert(kFastChunk % (kTopPWarps * 128) == 0, "whole float4 rounds per warp");
+
+// The bound on |A - E| above for a vocabulary of V, in units of 2^-40.
+inline unsigned long long top_p_margin(int64_t V) { return (1ull << 23) + 2ull * static_cast<unsigned long long>(V); }
 
 __global__ void __launch_bounds__(kTopPThreads, 2)
     top_p_fast_kernel(const float* __restrict__ z, int64_t ldz, int V, const int* __restrict__ n_valid,
