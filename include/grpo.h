@@ -155,9 +155,12 @@ grpo_status grpo_sample_tokens(const uint16_t* H, const uint16_t* W, const uint8
  * with G exactly as grpo_sample_tokens defines it, which draws from p
  * renormalised on the nucleus; top_p = 1 draws the same tokens as
  * grpo_sample_tokens.  The forward GEMM stores the fp32 logits of the unmasked
- * rows in the workspace (4 * V bytes per row) and one pass per row finds the
- * threshold (mass in 2^-40 fixed point, so the result does not depend on the
- * order of the sums) and the argmax.
+ * rows in the workspace (4 * V bytes per row) and keeps each vocabulary
+ * split's best perturbed score; a streaming pass lists the rows whose plain
+ * winner may fall outside the nucleus, and only those are resolved exactly:
+ * the threshold from masses in 2^-40 fixed point (so the result does not
+ * depend on the order of the sums), then the argmax over the nucleus from the
+ * splits' winners, walking only the splits whose winner falls outside.
  *   top_p       in (0, 1]
  *   logp_out    [T] fp32 device, log softmax(y) at the sampled token (the
  *               untruncated distribution; subtract log of the nucleus mass for
