@@ -19,8 +19,8 @@
 // logits (top_p_fast_kernel) lists the rows whose winner may lie outside,
 // from fp32 sums within a proven margin of the exact mass.
 //
-// A cluster of kTopPCtas CTAs takes one listed row at a time (distributed
-// shared memory; each CTA walks an interleaved eighth of the row).  Only the
+// A cluster of 2, 4 or 8 CTAs takes one listed row at a time (distributed
+// shared memory; each CTA walks an interleaved share of the row).  Only the
 // logits above y_w0 matter; the first level's histogram of their exact masses
 // confirms the row (a row whose total falls short keeps its plain draw), and
 // then y* > y_w0:
@@ -46,6 +46,8 @@
 
 #include <stdint.h>
 
+#include <cstdlib>
+
 #include "gemm_tc.cuh"
 #include "ptx.cuh"
 #include "small_kernels.cuh"
@@ -53,14 +55,14 @@
 namespace grpo {
 
 constexpr int kTopPThreads = 256;
-constexpr int kTopPCtas = 8;       // CTAs of a cluster sharing one row
+constexpr int kTopPCtas = 8;       // most CTAs of a cluster sharing one row (clusters of 2, 4 or 8)
 constexpr int kTopPBuckets = 2048;
 constexpr int kTopPCand = 1024;    // candidates resolved exactly in shared memory
 constexpr int kTopPLevels = 6;     // histogram levels before the candidates fit
 constexpr int kTopPWarps = kTopPThreads / 32;
 // column halves of a tile in the sampling GEMM's split entries (one per epilogue warp of a lane quarter)
 constexpr int kSampleHalves = EpiShape<kEpiSample>::kHalves;
-static_assert(kTopPBuckets == kTopPCtas * kTopPThreads, "one histogram bucket per thread of the cluster in the merge");
+static_assert(kTopPBuckets % (kTopPCtas * kTopPThreads) == 0, "whole histogram buckets per thread in the merge");
 
 // Shared memory of one CTA.  The fields marked "host" are used in CTA 0 of
 // the cluster only (the other CTAs write into and read from CTA 0's copy).
@@ -70,6 +72,10 @@ struct TopPShared {
     struct {                                // gather pass: this CTA's candidates before they are broadcast
       float y[kTopPCand];
     } loc;
+    struct {                                // the draw: this CTA's entries whose winner lies outside the nucleus
+      int e[kTopPThreads];
+      unsigned n;
+    } out;
   };
   float cy[kTopPCand];                      // the cluster's candidates: every CTA holds all of them
   unsigned long long cq[kTopPCand];
@@ -92,13 +98,18 @@ struct TopPShared {
 };
 
 // Probability of tempered logit y in 2^-40 units, truncated toward zero: the
-// float p * 2^40 converted exactly (one truncating conversion; measured a
-// little faster in the selection than building the integer from the float's
-// fields).  A value that is not finite or not below 2^41 gives 0.
+// float f = p * 2^40 converted exactly.  A value that is not finite or not
+// below 2^41 gives 0.  The conversion is a 32-bit one: below 2^32 f truncates
+// directly; from 2^32 on f is a multiple of its ulp (at least 2^9), so f 2^-9
+// is an integer below 2^32 and converts exactly, then shifts back.  (A
+// 64-bit conversion per logit measured a third of the histogram walk.)
 __device__ __forceinline__ unsigned long long top_p_mass(float y, float lse) {
   const float kLog2e = 1.4426950408889634f;
   const float f = fast_exp2((y - lse) * kLog2e) * 1099511627776.0f;
-  return f < 2199023255552.0f ? __float2ull_rz(f) : 0ull;
+  if (!(f < 2199023255552.0f)) return 0ull;
+  const bool big = f >= 4294967296.0f;
+  const unsigned v = __float2uint_rz(big ? f * 0.001953125f : f);
+  return static_cast<unsigned long long>(v) << (big ? 9 : 0);
 }
 
 // Adds q to a 64-bit histogram bucket with 32-bit shared atomics: q's low word
@@ -117,22 +128,15 @@ __device__ __forceinline__ int top_p_bucket(float y, float hi, float scale) {
   return static_cast<int>(fminf(fmaxf((hi - y) * scale, 0.f), static_cast<float>(kTopPBuckets - 1)));
 }
 
-// True when y lies in the chosen bucket of every one of the first n levels.
-__device__ __forceinline__ bool top_p_in(const TopPShared& sh, float y, int n) {
-  for (int l = 0; l < n; ++l)
+// True when y lies in the chosen bucket of every one of the first n levels;
+// the first level's range and bucket come in registers (hi0, scale0, b0), the
+// walks' common case, the deeper ones from shared memory.
+__device__ __forceinline__ bool top_p_in(const TopPShared& sh, float hi0, float scale0, int b0, float y, int n) {
+  if (n == 0) return true;
+  if (top_p_bucket(y, hi0, scale0) != b0) return false;
+  for (int l = 1; l < n; ++l)
     if (top_p_bucket(y, sh.lvl_hi[l], sh.lvl_scale[l]) != sh.lvl_b[l]) return false;
   return true;
-}
-
-// Where y lies against the chosen buckets of the first n levels: 2 in all of
-// them (a candidate), 1 above one of them (above the threshold, which lies in
-// the chosen bucket; the bucket index never increases with y), 0 below.
-__device__ __forceinline__ int top_p_class(const TopPShared& sh, float y, int n) {
-  for (int l = 0; l < n; ++l) {
-    const int b = top_p_bucket(y, sh.lvl_hi[l], sh.lvl_scale[l]);
-    if (b != sh.lvl_b[l]) return b < sh.lvl_b[l] ? 1 : 0;
-  }
-  return 2;
 }
 
 // The mass the nucleus must reach, in the units of top_p_mass: top_p of the
@@ -158,15 +162,15 @@ __device__ __forceinline__ float top_p_block_max(TopPShared& sh, float v) {
   return r;
 }
 
-// Walks this CTA's share of the row: groups of four logits (16-byte loads; the
-// row's leading dimension is a multiple of 64, so a group never leaves the
-// row's storage) g = rank * kTopPThreads + tid + k * kTopPCtas * kTopPThreads,
-// up to kUnroll groups per thread loaded together (the last round predicated),
-// then f(g, q) for each.  Lanes of a partial last group past V are the
-// caller's to skip.
-template <int kUnroll, typename F>
+// Walks this CTA's share of the row in a cluster of kC CTAs: groups of four
+// logits (16-byte loads; the row's leading dimension is a multiple of 64, so a
+// group never leaves the row's storage) g = rank * kTopPThreads + tid + k * kC
+// * kTopPThreads, up to kUnroll groups per thread loaded together (the last
+// round predicated), then f(g, q) for each.  Lanes of a partial last group
+// past V are the caller's to skip.
+template <int kC, int kUnroll, typename F>
 __device__ __forceinline__ void top_p_groups(const float* zr, int V, int rank, F f) {
-  constexpr int kStride = kTopPCtas * kTopPThreads;
+  constexpr int kStride = kC * kTopPThreads;
   const int groups = (V + 3) / 4;
   const float4* zq = reinterpret_cast<const float4*>(zr);
   for (int g0 = rank * kTopPThreads + static_cast<int>(threadIdx.x); g0 < groups; g0 += kUnroll * kStride) {
@@ -194,26 +198,35 @@ __device__ __forceinline__ bool top_p_better(float s, int v, float s0, int v0) {
 // candidates with y_j >= y reaches `need` (the first position, largest y
 // first, where the running sum reaches need: the running sum at the end of
 // y's group of equal logits is M(y), and it grows down the list).  The CTA
-// takes the candidates [rank * per, (rank + 1) * per), tpi threads each
-// (a power of two, so a candidate's threads share a warp); returns the
-// largest qualifying y of its candidates in every thread, -inf if none.
+// takes the candidates [rank * per, (rank + 1) * per) of a cluster of kC,
+// tpi threads each (a power of two, so a candidate's threads share a warp;
+// one thread each, in rounds, when there are more candidates than threads);
+// returns the largest qualifying y of its candidates in every thread, -inf if
+// none.
+template <int kC>
 __device__ __forceinline__ float top_p_rank_slice(TopPShared& sh, int nc, int rank, unsigned long long need) {
-  const int per = (nc + kTopPCtas - 1) / kTopPCtas;  // <= kTopPCand / kTopPCtas = 128
+  const int per = (nc + kC - 1) / kC;  // <= kTopPCand / kC
   int tpi = 32;
   while (tpi > 1 && per * tpi > kTopPThreads) tpi >>= 1;
-  const int k = static_cast<int>(threadIdx.x) / tpi;
-  const int i = rank * per + k;
-  const bool act = k < per && i < nc;
-  const float yi = act ? sh.cy[i] : INFINITY;
-  unsigned long long m = 0ull;
-  if (act)
-    for (int j = static_cast<int>(threadIdx.x) & (tpi - 1); j < nc; j += tpi)
-      if (sh.cy[j] >= yi) m += sh.cq[j];
-  for (int o = tpi >> 1; o > 0; o >>= 1) m += __shfl_xor_sync(0xffffffffu, m, o);
-  return top_p_block_max(sh, act && m >= need ? yi : -INFINITY);
+  const int step = kTopPThreads / tpi;  // candidates per round
+  float best = -INFINITY;
+  for (int k0 = 0; k0 < per; k0 += step) {  // the same rounds in every thread
+    const int k = k0 + static_cast<int>(threadIdx.x) / tpi;
+    const int i = rank * per + k;
+    const bool act = k < per && i < nc;
+    const float yi = act ? sh.cy[i] : INFINITY;
+    unsigned long long m = 0ull;
+    if (act)
+      for (int j = static_cast<int>(threadIdx.x) & (tpi - 1); j < nc; j += tpi)
+        if (sh.cy[j] >= yi) m += sh.cq[j];
+    for (int o = tpi >> 1; o > 0; o >>= 1) m += __shfl_xor_sync(0xffffffffu, m, o);
+    if (act && m >= need) best = fmaxf(best, yi);
+  }
+  return top_p_block_max(sh, best);
 }
 
-__global__ void __cluster_dims__(kTopPCtas, 1, 1) __launch_bounds__(kTopPThreads, 4)
+template <int kC>
+__global__ void __cluster_dims__(kC, 1, 1) __launch_bounds__(kTopPThreads, 4)
     top_p_kernel(const float* __restrict__ z, int64_t ldz, int V, const int* __restrict__ n_slow,
                  const int* __restrict__ slow_rows, const unsigned long long* __restrict__ slow_target,
                  const int* __restrict__ cidx, const float* __restrict__ lse_r, const float* __restrict__ y0_r,
@@ -228,7 +241,7 @@ __global__ void __cluster_dims__(kTopPCtas, 1, 1) __launch_bounds__(kTopPThreads
   const int ns = *n_slow;
   // CTA k's copy of a field
   auto atk = [&](const void* p, int k) { return mapa_shared(smem_addr(p), static_cast<uint32_t>(k)); };
-  for (int si = blockIdx.x / kTopPCtas; si < ns; si += gridDim.x / kTopPCtas) {
+  for (int si = blockIdx.x / kC; si < ns; si += gridDim.x / kC) {
     const int r = slow_rows[si];
     const float* zr = z + static_cast<int64_t>(r) * ldz;
     const int t = cidx[r];
@@ -256,11 +269,13 @@ __global__ void __cluster_dims__(kTopPCtas, 1, 1) __launch_bounds__(kTopPThreads
       __syncthreads();
       {
         const float hi = sh.lvl_hi[L], scale = sh.lvl_scale[L];
-        top_p_groups<8>(zr, V, rank, [&](int g, float4 q) {
+        const float hi0 = sh.lvl_hi[0], scale0 = sh.lvl_scale[0];
+        const int b0 = L > 0 ? sh.lvl_b[0] : 0;
+        top_p_groups<kC, 8>(zr, V, rank, [&](int g, float4 q) {
           const float yy[4] = {q.x * inv_temp, q.y * inv_temp, q.z * inv_temp, q.w * inv_temp};
 #pragma unroll
           for (int k = 0; k < 4; ++k) {
-            if (4 * g + k < V && yy[k] > y0 && top_p_in(sh, yy[k], L)) {
+            if (4 * g + k < V && yy[k] > y0 && top_p_in(sh, hi0, scale0, b0, yy[k], L)) {
               const unsigned long long m = top_p_mass(yy[k], lse);
               if (m) top_p_hist_add(&sh.hist[top_p_bucket(yy[k], hi, scale)], m);  // far tail adds nothing
             }
@@ -268,17 +283,21 @@ __global__ void __cluster_dims__(kTopPCtas, 1, 1) __launch_bounds__(kTopPThreads
         });
       }
       cluster_sync();
-      {  // merge the histograms: CTA k sums buckets [k * kTopPThreads, (k + 1) * kTopPThreads) over
-         // the cluster in rank order and leaves the sums in CTA 0's histogram (disjoint slices, so no
+      {  // merge the histograms: CTA k sums its slice of kMerge * kTopPThreads buckets over the
+         // cluster in rank order and leaves the sums in CTA 0's histogram (disjoint slices, so no
          // CTA reads a bucket another one writes)
-        const int b = rank * kTopPThreads + tid;
-        unsigned long long part[kTopPCtas];
+        constexpr int kMerge = kTopPBuckets / (kC * kTopPThreads);
 #pragma unroll
-        for (int k = 0; k < kTopPCtas; ++k) part[k] = ld_shared_cluster_u64(atk(&sh.hist[b], k));
-        unsigned long long m = 0ull;
+        for (int j = 0; j < kMerge; ++j) {
+          const int b = (rank * kMerge + j) * kTopPThreads + tid;
+          unsigned long long part[kC];
 #pragma unroll
-        for (int k = 0; k < kTopPCtas; ++k) m += part[k];
-        st_shared_cluster_u64(atk(&sh.hist[b], 0), m);
+          for (int k = 0; k < kC; ++k) part[k] = ld_shared_cluster_u64(atk(&sh.hist[b], k));
+          unsigned long long m = 0ull;
+#pragma unroll
+          for (int k = 0; k < kC; ++k) m += part[k];
+          st_shared_cluster_u64(atk(&sh.hist[b], 0), m);
+        }
       }
       cluster_sync();
       if (host) {  // find the bucket that holds the threshold
@@ -354,11 +373,13 @@ __global__ void __cluster_dims__(kTopPCtas, 1, 1) __launch_bounds__(kTopPThreads
       // gather the bucket's logits (and their range, in case they do not fit)
       // into this CTA's list
       float lo = INFINITY, hi2 = -INFINITY;
-      top_p_groups<4>(zr, V, rank, [&](int g, float4 q) {
+      const float hi0 = sh.lvl_hi[0], scale0 = sh.lvl_scale[0];
+      const int b0 = sh.lvl_b[0];
+      top_p_groups<kC, 8>(zr, V, rank, [&](int g, float4 q) {
         const float yy[4] = {q.x * inv_temp, q.y * inv_temp, q.z * inv_temp, q.w * inv_temp};
 #pragma unroll
         for (int k = 0; k < 4; ++k) {
-          if (4 * g + k < V && yy[k] > y0 && top_p_in(sh, yy[k], L + 1)) {
+          if (4 * g + k < V && yy[k] > y0 && top_p_in(sh, hi0, scale0, b0, yy[k], L + 1)) {
             lo = fminf(lo, yy[k]);
             hi2 = fmaxf(hi2, yy[k]);
             const unsigned i = atomicAdd(&sh.lcand, 1u);
@@ -381,7 +402,7 @@ __global__ void __cluster_dims__(kTopPCtas, 1, 1) __launch_bounds__(kTopPThreads
           const float y = sh.loc.y[i];
           const unsigned long long m = top_p_mass(y, lse);
 #pragma unroll
-          for (int k = 0; k < kTopPCtas; ++k) {
+          for (int k = 0; k < kC; ++k) {
             st_shared_cluster(atk(&sh.cy[base + i], k), __float_as_uint(y));
             st_shared_cluster_u64(atk(&sh.cq[base + i], k), m);
           }
@@ -394,7 +415,7 @@ __global__ void __cluster_dims__(kTopPCtas, 1, 1) __launch_bounds__(kTopPThreads
           // too many to resolve here: every CTA reads the bucket's range and
           // decides alike whether to histogram it once more
           float l = INFINITY, h = -INFINITY;
-          for (int k = 0; k < kTopPCtas; ++k) {
+          for (int k = 0; k < kC; ++k) {
             l = fminf(l, __uint_as_float(ld_shared_cluster(atk(&sh.slot_lo[k], 0))));
             h = fmaxf(h, __uint_as_float(ld_shared_cluster(atk(&sh.slot_hi[k], 0))));
           }
@@ -411,12 +432,12 @@ __global__ void __cluster_dims__(kTopPCtas, 1, 1) __launch_bounds__(kTopPThreads
       __syncthreads();
       const int nc = static_cast<int>(sh.ncand);
       if (nc <= kTopPCand) {
-        const float c = top_p_rank_slice(sh, nc, rank, target - sh.cum_before);
+        const float c = top_p_rank_slice<kC>(sh, nc, rank, target - sh.cum_before);
         if (tid == 0) st_shared_cluster(atk(&sh.slot_r[rank], 0), __float_as_uint(c));
         cluster_sync();
         if (tid == 0) {
           float ys = -INFINITY;
-          for (int k = 0; k < kTopPCtas; ++k) ys = fmaxf(ys, __uint_as_float(ld_shared_cluster(atk(&sh.slot_r[k], 0))));
+          for (int k = 0; k < kC; ++k) ys = fmaxf(ys, __uint_as_float(ld_shared_cluster(atk(&sh.slot_r[k], 0))));
           sh.ystar = ys;
           sh.full = ys == -INFINITY;  // no crossing (the masses fell short): the whole vocabulary
         }
@@ -438,38 +459,68 @@ __global__ void __cluster_dims__(kTopPCtas, 1, 1) __launch_bounds__(kTopPThreads
     bs = -INFINITY;
     bv = -1;
     by = 0.f;
-    for (int e = rank; e < nsplit; e += kTopPCtas) {
-      const long at = static_cast<long>(e) * ldp + r;
-      const float bz = best_z[at];
-      if (bz >= ystar) {
-        if (tid == 0 && top_p_better(best_s[at], best_c[at], bs, bv)) {
-          bs = best_s[at];
-          bv = best_c[at];
-          by = bz;
+    // This CTA's entries are e = rank + kC j.  Each thread classifies
+    // one of them (the loads of all entries in flight together); the entries
+    // whose winner lies outside are then walked as one list of 4-token groups.
+    constexpr int kGroupsPerTile = kTileN / kSampleHalves / 4;  // 4-token groups of one tile's column half
+    const int per_entry = unit_tiles * kGroupsPerTile;
+    const int nj = nsplit > rank ? (nsplit - rank + kC - 1) / kC : 0;
+    for (int base = 0; base < nj; base += kTopPThreads) {
+      __syncthreads();  // the previous batch's list has been walked
+      if (tid == 0) sh.out.n = 0u;
+      __syncthreads();
+      if (base + tid < nj) {
+        const int e = rank + kC * (base + tid);
+        const long at = static_cast<long>(e) * ldp + r;
+        const float bz = best_z[at];
+        if (bz >= ystar) {
+          const float s0 = best_s[at];
+          const int c = best_c[at];
+          if (top_p_better(s0, c, bs, bv)) {
+            bs = s0;
+            bv = c;
+            by = bz;
+          }
+        } else {
+          sh.out.e[atomicAdd(&sh.out.n, 1u)] = e;
         }
-        continue;
       }
-      const int c0 = (e / kSampleHalves) * unit_tiles * kTileN + (e % kSampleHalves) * (kTileN / kSampleHalves);
-      constexpr int kGroupsPerTile = kTileN / kSampleHalves / 4;  // 4-token groups of one tile's column half
-      for (int gi = tid; gi < unit_tiles * kGroupsPerTile; gi += kTopPThreads) {
-        const int v0 = c0 + (gi / kGroupsPerTile) * kTileN + 4 * (gi % kGroupsPerTile);
-        if (v0 >= V) continue;
-        const float4 q = __ldcg(reinterpret_cast<const float4*>(zr + v0));
-        const float yy[4] = {q.x * inv_temp, q.y * inv_temp, q.z * inv_temp, q.w * inv_temp};
-        if (!(yy[0] >= ystar || yy[1] >= ystar || yy[2] >= ystar || yy[3] >= ystar)) continue;
-        const uint4 w = philox4x32_10(make_uint4(static_cast<uint32_t>(v0 >> 2), static_cast<uint32_t>(t), off_lo,
-                                                 off_hi),
-                                      seed_lo, seed_hi);
-        const uint32_t ws[4] = {w.x, w.y, w.z, w.w};
+      __syncthreads();
+      const int total = static_cast<int>(sh.out.n) * per_entry;
+      constexpr int kU = 4;  // groups per thread loaded together
+      for (int g0 = tid; g0 < total; g0 += kU * kTopPThreads) {
+        float4 q[kU];
+        int v0[kU];
 #pragma unroll
-        for (int k = 0; k < 4; ++k) {
-          const int v = v0 + k;
-          if (v < V && yy[k] >= ystar) {
-            const float sc = yy[k] + gumbel_of(ws[k]);
-            if (top_p_better(sc, v, bs, bv)) {
-              bs = sc;
-              bv = v;
-              by = yy[k];
+        for (int u = 0; u < kU; ++u) {
+          const int gi = g0 + u * kTopPThreads;
+          v0[u] = V;
+          if (gi < total) {
+            const int e = sh.out.e[gi / per_entry];
+            const int gl = gi - (gi / per_entry) * per_entry;
+            v0[u] = (e / kSampleHalves) * unit_tiles * kTileN + (e % kSampleHalves) * (kTileN / kSampleHalves) +
+                    (gl / kGroupsPerTile) * kTileN + 4 * (gl % kGroupsPerTile);
+          }
+          q[u] = v0[u] < V ? __ldcg(reinterpret_cast<const float4*>(zr + v0[u])) : make_float4(0.f, 0.f, 0.f, 0.f);
+        }
+#pragma unroll
+        for (int u = 0; u < kU; ++u) {
+          if (v0[u] >= V) continue;
+          const float yy[4] = {q[u].x * inv_temp, q[u].y * inv_temp, q[u].z * inv_temp, q[u].w * inv_temp};
+          if (!(yy[0] >= ystar || yy[1] >= ystar || yy[2] >= ystar || yy[3] >= ystar)) continue;
+          const uint4 w = philox4x32_10(
+              make_uint4(static_cast<uint32_t>(v0[u] >> 2), static_cast<uint32_t>(t), off_lo, off_hi), seed_lo, seed_hi);
+          const uint32_t ws[4] = {w.x, w.y, w.z, w.w};
+#pragma unroll
+          for (int k = 0; k < 4; ++k) {
+            const int v = v0[u] + k;
+            if (v < V && yy[k] >= ystar) {
+              const float sc = yy[k] + gumbel_of(ws[k]);
+              if (top_p_better(sc, v, bs, bv)) {
+                bs = sc;
+                bv = v;
+                by = yy[k];
+              }
             }
           }
         }
@@ -509,7 +560,7 @@ __global__ void __cluster_dims__(kTopPCtas, 1, 1) __launch_bounds__(kTopPThreads
       bs = -INFINITY;
       bv = -1;
       by = 0.f;
-      for (int k = 0; k < kTopPCtas; ++k) {
+      for (int k = 0; k < kC; ++k) {
         const float os = __uint_as_float(sh.slot_f[k]);
         const int ov = static_cast<int>(sh.slot_i[k]);
         if (top_p_better(os, ov, bs, bv)) {
@@ -627,6 +678,29 @@ static_assert(kFastChunk % (kTopPWarps * 128) == 0, "whole float4 rounds per war
 
 // The bound on |A - E| above for a vocabulary of V, in units of 2^-40.
 inline unsigned long long top_p_margin(int64_t V) { return (1ull << 23) + 2ull * static_cast<unsigned long long>(V); }
+
+// log2 of the cluster size of the selection (1, 2 or 3: clusters of 2, 4 or
+// 8 CTAs) for a draw over up to `rows` rows.  About a fraction 1 - top_p of
+// the rows are listed (the winner falls outside its nucleus that often).  A
+// cluster takes one listed row at a time, so few listed rows want large
+// clusters (each row done sooner, while about 74 clusters of 8 fit on a
+// GB300) and many want small ones (fewer cluster barriers per logit).
+// Measured draws over V = 155,136 (the listed-row estimate in brackets):
+// 256 rows at top_p 0.9 [33] 0.37 / 0.39 / 0.43 ms with clusters of 8 / 4 /
+// 2, at 0.5 [166] 0.43 / 0.42 / 0.46; 2048 rows at 0.9 [266] 1.96-2.06 /
+// 1.96-2.10 / 2.03-2.11, at 0.5 [1331] 2.59 / 2.48 / 2.46; 19,572 of 32,768
+// rows at 0.5 [21299] 24.7-24.9 / 24.3-24.7 / 23.4-24.1 ms.  GRPO_TOP_P_CLUSTER=2|4|8
+// overrides the choice.
+inline int top_p_cluster_log2(int64_t rows, float top_p) {
+  if (const char* e = std::getenv("GRPO_TOP_P_CLUSTER")) {
+    const int c = std::atoi(e);
+    if (c == 2) return 1;
+    if (c == 4) return 2;
+    if (c == 8) return 3;
+  }
+  const double listed = static_cast<double>(rows) * (1.0 - static_cast<double>(top_p)) * 1.3;
+  return listed <= 100.0 ? 3 : listed <= 400.0 ? 2 : 1;
+}
 
 __global__ void __launch_bounds__(kTopPThreads, 2)
     top_p_fast_kernel(const float* __restrict__ z, int64_t ldz, int V, const int* __restrict__ n_valid,

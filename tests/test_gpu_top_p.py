@@ -234,3 +234,30 @@ def test_every_row_listed_gives_the_same_draws(monkeypatch, top_p):
         got = _draw(Hb, Wb, m, 1.0, top_p, 77, 5)
         monkeypatch.delenv("GRPO_TEST_TOP_P_LIST_ALL")
         assert np.array_equal(got[0], want[0]) and np.array_equal(got[1], want[1])
+
+
+@pytest.mark.parametrize("top_p", [0.9, 0.5])
+def test_cluster_size_gives_the_same_draws(monkeypatch, top_p):
+    """The selection takes each listed row in a cluster of 8, 4 or 2 CTAs
+    (chosen by the expected number of listed rows); the histogram merge, the
+    candidate split of the threshold search and the draw's entry split all
+    change with the size, and every reduction in them is exact or has a total
+    order, so the draws and log-probs are the same bits for every size, here
+    with every row listed too (both levels of the selection run on every
+    row) and on a crowded vocabulary that needs a second histogram level."""
+    cases = [wl.Workload("p", 2, 3, 90, 192, 5000, "uniform", 1, 90, seed=wl.SEED_BASE + 3310, w_std=0.08),
+             wl.Workload("p", 2, 3, 90, 192, 4097, "uniform", 1, 90, seed=wl.SEED_BASE + 3311, w_std=0.5),
+             wl.Workload("p", 1, 2, 40, 64, 50000, "uniform", 1, 40, seed=wl.SEED_BASE + 2900, w_std=0.018),
+             wl.DECODE_WORKLOADS["decode256_8b"]]
+    for w in cases:
+        Hb, Wb, m = wl.gen_hidden(w), wl.gen_weight(w), wl.gen_mask(w)
+        for list_all in ("0", "1"):
+            monkeypatch.setenv("GRPO_TEST_TOP_P_LIST_ALL", list_all)
+            got = {}
+            for c in ("8", "4", "2"):
+                monkeypatch.setenv("GRPO_TOP_P_CLUSTER", c)
+                got[c] = _draw(Hb, Wb, m, 1.0, top_p, 91, 3)
+            for c in ("4", "2"):
+                assert np.array_equal(got[c][0], got["8"][0]) and np.array_equal(got[c][1], got["8"][1]), (w.V, c)
+    monkeypatch.delenv("GRPO_TOP_P_CLUSTER")
+    monkeypatch.delenv("GRPO_TEST_TOP_P_LIST_ALL")
