@@ -11,7 +11,7 @@ shaped like an 8B policy's rollout (workloads.py).  Prints one JSON line.
 
 value: response (unmasked) tokens per second over all ranks, inputs resident
 in HBM; e2e: the same through the public API with pinned host buffers, the
-host<->device copies inside the timed region.
+host<->device transfers inside the timed region.
 """
 from __future__ import annotations
 
@@ -701,7 +701,8 @@ def measure_e2e_scoring(grpo, torch, dev, w, inp, heads, steps: int, dist=None):
         return torch.from_numpy(np.ascontiguousarray(a)).view(dt).pin_memory()
 
     hH, hy, hm = pin(inp["H"], torch.bfloat16), pin(inp["y"], torch.int32), pin(inp["m"], torch.uint8)
-    h2d = sum(t.numel() * t.element_size() for t in [hH, hy, hm])
+    # H stays in page-locked host memory: the row gather reads the unmasked rows over the host link
+    h2d = n_valid * w.Hd * 2 + sum(t.numel() * t.element_size() for t in [hy, hm])
     d2h = len(heads) * w.T * 4
     hout = torch.empty(len(heads), w.T, dtype=torch.float32).pin_memory()
     ws = grpo.workspace(w.T, w.Hd, w.V, grpo.GRPO_WS_LOGPROBS_HEADS, dev, max_valid=n_valid)
@@ -719,8 +720,9 @@ def measure_e2e_scoring(grpo, torch, dev, w, inp, heads, steps: int, dist=None):
     return {"value": round(n_tok / dt, 1), "unit": "tokens/s", "ms_per_step": round(dt * 1e3, 2),
             "ms_mean": round(mean * 1e3, 2), "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
             "steps": steps, "statistic": "median of per-step wall-clock times",
-            "what": "H, targets, mask copied from pinned host memory each step; the policy / old / reference "
-                    "heads resident on the device; the log-probs read back"}
+            "what": "H read from pinned host memory by the row gather each step (the unmasked rows cross the "
+                    "host link), targets and mask copied; the policy / old / reference heads resident on the "
+                    "device; the log-probs read back"}
 
 
 def measure_e2e(grpo, torch, dev, w, inp, steps: int, dist=None, ws=None):
@@ -739,7 +741,8 @@ def measure_e2e(grpo, torch, dev, w, inp, steps: int, dist=None, ws=None):
     Wd = torch.from_numpy(np.ascontiguousarray(inp["W"])).view(torch.bfloat16).to(dev)
     hH, hy, hm = pin(inp["H"], torch.bfloat16), pin(inp["y"], torch.int32), pin(inp["m"], torch.uint8)
     hold, href, hr = pin(inp["old"], torch.float32), pin(inp["ref"], torch.float32), pin(inp["r"], torch.float32)
-    h2d = sum(t.numel() * t.element_size() for t in (hH, hy, hm, hold, href, hr))
+    # H stays in page-locked host memory: the row gather reads the unmasked rows over the host link
+    h2d = n_valid * w.Hd * 2 + sum(t.numel() * t.element_size() for t in (hy, hm, hold, href, hr))
     d2h = 4
     out = (torch.empty(1, dtype=torch.float32, device=dev), torch.empty(w.T, w.Hd, dtype=torch.float32, device=dev),
            torch.empty(w.V, w.Hd, dtype=torch.float32, device=dev))
@@ -765,8 +768,9 @@ def measure_e2e(grpo, torch, dev, w, inp, steps: int, dist=None, ws=None):
     return {"value": round(n_tok / dt, 1), "unit": "tokens/s", "ms_per_step": round(dt * 1e3, 2),
             "ms_mean": round(mean * 1e3, 2), "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
             "steps": steps, "statistic": "median of per-step wall-clock times",
-            "what": "H, targets, mask, old/ref log-probs, rewards copied from pinned host memory each step; W "
-                    "resident on the device; the loss read back; dH, dW left on the device"}
+            "what": "H read from pinned host memory by the row gather each step (the unmasked rows cross the "
+                    "host link); targets, mask, old/ref log-probs, rewards copied; W resident on the device; the "
+                    "loss read back; dH, dW left on the device"}
 
 
 def measure_e2e_offload(grpo, torch, dev, w, inp, steps: int, ws=None):
@@ -781,7 +785,8 @@ def measure_e2e_offload(grpo, torch, dev, w, inp, steps: int, ws=None):
     hH, hW = pin(inp["H"], torch.bfloat16), pin(inp["W"], torch.bfloat16)
     hy, hm = pin(inp["y"], torch.int32), pin(inp["m"], torch.uint8)
     hold, href, hr = pin(inp["old"], torch.float32), pin(inp["ref"], torch.float32), pin(inp["r"], torch.float32)
-    h2d = sum(t.numel() * t.element_size() for t in (hH, hW, hy, hm, hold, href, hr))
+    # H stays in page-locked host memory (the row gather reads the unmasked rows); W is copied
+    h2d = n_valid * w.Hd * 2 + sum(t.numel() * t.element_size() for t in (hW, hy, hm, hold, href, hr))
     d2h = 4 + w.T * w.Hd * 4 + w.V * w.Hd * 4
 
     # the caller's own buffers, allocated once: pinned host outputs and a device workspace
@@ -800,7 +805,8 @@ def measure_e2e_offload(grpo, torch, dev, w, inp, steps: int, ws=None):
     return {"value": round(n_valid / med, 1), "unit": "tokens/s", "ms_per_step": round(med * 1e3, 2),
             "ms_mean": round(mean * 1e3, 2), "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
             "steps": steps, "statistic": "median of per-step wall-clock times",
-            "what": "batch and W copied from pinned host memory each step; loss, dH, dW copied back"}
+            "what": "H read from pinned host memory by the row gather (the unmasked rows cross the host link); "
+                    "the rest of the batch and W copied each step; loss, dH, dW copied back"}
 
 
 if __name__ == "__main__":

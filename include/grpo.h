@@ -12,6 +12,13 @@
  * - Every array pointer is a DEVICE pointer owned by the caller; the library
  *   never frees or keeps it.  bf16 arrays are passed as their 16-bit patterns
  *   (uint16_t).  All matrices are row-major and densely packed.
+ * - One exception: the hidden states H may also be page-locked host memory
+ *   registered with CUDA (cudaHostAlloc, cudaMallocHost, cudaHostRegister).
+ *   The row gather then reads the unmasked rows over the host link (the
+ *   masked rows never cross it) instead of the caller copying every row to
+ *   the device first.  As with an asynchronous copy, H must stay unchanged
+ *   and allocated until the call's work on the stream has completed.
+ *   Pageable host memory is GRPO_ERR_INVALID_ARG.
  * - `stream` is a cudaStream_t (NULL = legacy default stream).  Work is
  *   enqueued on it; no entry point synchronises the stream except
  *   grpo_check_device_status.  Nothing is allocated: scratch space comes from
@@ -96,7 +103,8 @@ grpo_status grpo_group_advantages(const float* rewards, int64_t n_resp, int32_t 
  * Per-token log-probability of the sampled token, the pi_theta(o_{i,t} | q, o_{i,<t})
  * of Eq. 1 (Section 3.3):  logp_t = z_{t,y_t} - log sum_v exp(z_{t,v}),  z_t = H_t W^T.
  * The [T x V] logits are never written to memory.
- *   H        [T x Hd] bf16 device, final hidden states (16-byte aligned)
+ *   H        [T x Hd] bf16 device (or page-locked host, see above), final hidden
+ *            states (16-byte aligned)
  *   W        [V x Hd] bf16 device, LM-head weight (16-byte aligned)
  *   targets  [T] int32 device, sampled token ids, must lie in [0, V) where mask != 0
  *   mask     [T] uint8 device, 0 = padding row

@@ -131,6 +131,32 @@ def _on_device(t: torch.Tensor, dev: torch.device, dtype: torch.dtype, name: str
     return t.contiguous()
 
 
+def _hidden(H: torch.Tensor, dev: torch.device) -> torch.Tensor:
+    """H for the C call: left in page-locked host memory when it is there (the
+    library's row gather then reads only the unmasked rows over the host link),
+    else on `dev` (copied when it is elsewhere)."""
+    if H.dtype != torch.bfloat16:
+        raise TypeError(f"H: expected {torch.bfloat16}, got {H.dtype}")
+    if not H.is_cuda and H.is_contiguous() and H.is_pinned():
+        return H
+    return _on_device(H, dev, torch.bfloat16, "H")
+
+
+# Host tensors the device reads during a call (a page-locked H): each stays
+# referenced until an event recorded after the call's work has completed, so
+# that it cannot be freed or reused while the row gather still reads it.
+_in_flight = []
+
+
+def _keep_until_done(t: torch.Tensor, dev: torch.device) -> None:
+    while _in_flight and _in_flight[0][0].query():
+        _in_flight.pop(0)
+    if not t.is_cuda:
+        ev = torch.cuda.Event()
+        ev.record(torch.cuda.current_stream(dev))
+        _in_flight.append((ev, t))
+
+
 def _shape(t: torch.Tensor, shape, name: str) -> None:
     """The C ABI sees only pointers and sizes: a tensor of the wrong shape would
     be read or written past its end, so every shape is checked here."""
@@ -227,7 +253,7 @@ def token_logprobs(H: torch.Tensor, W: torch.Tensor, targets: torch.Tensor, mask
                    ws: Optional[torch.Tensor] = None, out: Optional[torch.Tensor] = None) -> torch.Tensor:
     """grpo_token_logprobs: log softmax(H W^T) at the sampled tokens; padding rows give 0."""
     dev, host = _target_device(H, W)
-    H = _on_device(H, dev, torch.bfloat16, "H")
+    H = _hidden(H, dev)
     W = _on_device(W, dev, torch.bfloat16, "W")
     targets = _on_device(targets, dev, torch.int32, "targets")
     mask = _on_device(mask.view(torch.uint8) if mask.dtype == torch.bool else mask, dev, torch.uint8, "mask")
@@ -241,6 +267,7 @@ def token_logprobs(H: torch.Tensor, W: torch.Tensor, targets: torch.Tensor, mask
         torch.empty(T, dtype=torch.float32, device=dev)
     _check(load().grpo_token_logprobs(_ptr(H), _ptr(W), _ptr(targets), _ptr(mask), T, Hd, V, _ptr(logp),
                                       _ptr(ws), ws.numel(), _stream(dev)), "grpo_token_logprobs")
+    _keep_until_done(H, dev)
     return _to_host(logp) if host else logp
 
 
@@ -250,7 +277,7 @@ def token_logprobs_heads(H: torch.Tensor, W_heads, targets: torch.Tensor, mask: 
     old, reference ...); returns [n_heads, T] fp32, 0 on padding rows."""
     W_heads = list(W_heads)
     dev, host = _target_device(H, *W_heads)
-    H = _on_device(H, dev, torch.bfloat16, "H")
+    H = _hidden(H, dev)
     W_heads = [_on_device(w, dev, torch.bfloat16, f"W_heads[{i}]") for i, w in enumerate(W_heads)]
     targets = _on_device(targets, dev, torch.int32, "targets")
     mask = _on_device(mask.view(torch.uint8) if mask.dtype == torch.bool else mask, dev, torch.uint8, "mask")
@@ -267,6 +294,7 @@ def token_logprobs_heads(H: torch.Tensor, W_heads, targets: torch.Tensor, mask: 
     _check(load().grpo_token_logprobs_heads(_ptr(H), ptrs, len(W_heads), _ptr(targets), _ptr(mask), T, Hd, V,
                                             _ptr(logp), _ptr(ws), ws.numel(), _stream(dev)),
            "grpo_token_logprobs_heads")
+    _keep_until_done(H, dev)
     return _to_host(logp) if host else logp
 
 
@@ -275,7 +303,7 @@ def sample_tokens(H: torch.Tensor, W: torch.Tensor, mask: torch.Tensor, temperat
     """grpo_sample_tokens: Gumbel-max draw from softmax(H W^T / temperature) at
     the unmasked rows; returns (tokens int32 [T] (-1 masked), logp fp32 [T])."""
     dev, host = _target_device(H, W)
-    H = _on_device(H, dev, torch.bfloat16, "H")
+    H = _hidden(H, dev)
     W = _on_device(W, dev, torch.bfloat16, "W")
     mask = _on_device(mask.view(torch.uint8) if mask.dtype == torch.bool else mask, dev, torch.uint8, "mask")
     T, Hd = H.shape
@@ -290,6 +318,7 @@ def sample_tokens(H: torch.Tensor, W: torch.Tensor, mask: torch.Tensor, temperat
     _check(load().grpo_sample_tokens(_ptr(H), _ptr(W), _ptr(mask), T, Hd, V, float(temperature),
                                      int(seed) & (2 ** 64 - 1), int(offset) & (2 ** 64 - 1), _ptr(tok), _ptr(logp),
                                      _ptr(ws), ws.numel(), _stream(dev)), "grpo_sample_tokens")
+    _keep_until_done(H, dev)
     return _to_host(tok, logp) if host else (tok, logp)
 
 
@@ -301,7 +330,7 @@ def sample_tokens_top_p(H: torch.Tensor, W: torch.Tensor, mask: torch.Tensor, te
     reaches top_p); returns (tokens int32 [T] (-1 masked), logp fp32 [T] under
     the untruncated distribution)."""
     dev, host = _target_device(H, W)
-    H = _on_device(H, dev, torch.bfloat16, "H")
+    H = _hidden(H, dev)
     W = _on_device(W, dev, torch.bfloat16, "W")
     mask = _on_device(mask.view(torch.uint8) if mask.dtype == torch.bool else mask, dev, torch.uint8, "mask")
     T, Hd = H.shape
@@ -317,6 +346,7 @@ def sample_tokens_top_p(H: torch.Tensor, W: torch.Tensor, mask: torch.Tensor, te
                                            float(top_p), int(seed) & (2 ** 64 - 1), int(offset) & (2 ** 64 - 1),
                                            _ptr(tok), _ptr(logp), _ptr(ws), ws.numel(), _stream(dev)),
            "grpo_sample_tokens_top_p")
+    _keep_until_done(H, dev)
     return _to_host(tok, logp) if host else (tok, logp)
 
 
@@ -334,7 +364,7 @@ def loss_fwd_bwd(H: torch.Tensor, W: torch.Tensor, targets: torch.Tensor, mask: 
     `out` may be device tensors (written in place) or host tensors, preferably
     pinned (the results are copied there before the call returns)."""
     dev, host = _target_device(H, W)
-    H = _on_device(H, dev, torch.bfloat16, "H")
+    H = _hidden(H, dev)
     W = _on_device(W, dev, torch.bfloat16, "W")
     targets = _on_device(targets, dev, torch.int32, "targets")
     mask = _on_device(mask.view(torch.uint8) if mask.dtype == torch.bool else mask, dev, torch.uint8, "mask")
@@ -374,6 +404,7 @@ def loss_fwd_bwd(H: torch.Tensor, W: torch.Tensor, targets: torch.Tensor, mask: 
         _check(lib.grpo_loss_fwd_bwd_to_host(*common, float(norm), _ptr(loss), _ptr(dH), _ptr(dW),
                                              _ptr(host_out[2]), _ptr(ws), ws.numel(), _stream(dev)),
                "grpo_loss_fwd_bwd_to_host")
+        _keep_until_done(H, dev)
         lh, dHh = _to_host(loss, dH, dst=host_out[:2])
         return lh, dHh, host_out[2]
     if chunk_events is not None:
@@ -394,6 +425,7 @@ def loss_fwd_bwd(H: torch.Tensor, W: torch.Tensor, targets: torch.Tensor, mask: 
         _check(lib.grpo_loss_fwd_bwd_norm(*common, float(norm), *tail), "grpo_loss_fwd_bwd_norm")
     else:
         _check(lib.grpo_loss_fwd_bwd(*common, *tail), "grpo_loss_fwd_bwd")
+    _keep_until_done(H, dev)
     if host or host_out is not None:
         return _to_host(loss, dH, dW, dst=host_out)
     return loss, dH, dW

@@ -477,6 +477,22 @@ T* at(void* ws, size_t off) {
 }
 
 
+// The pointer the row gather reads H through: H itself for device (or
+// managed) memory; for page-locked host memory registered with CUDA its
+// device-side address, so the gather reads the unmasked rows over the host
+// link and the masked ones never cross it; nullptr for memory the device
+// cannot read (pageable host memory).
+const uint16_t* hidden_view(const uint16_t* H) {
+  cudaPointerAttributes pa{};
+  if (cudaPointerGetAttributes(&pa, H) != cudaSuccess) {
+    cudaGetLastError();
+    return nullptr;
+  }
+  if (pa.type == cudaMemoryTypeHost) return static_cast<const uint16_t*>(pa.devicePointer);
+  if (pa.type == cudaMemoryTypeUnregistered) return nullptr;
+  return H;
+}
+
 // Compaction of unmasked rows + gather of their hidden states and targets.
 cudaError_t run_compaction(const uint16_t* H, const int32_t* targets, const uint8_t* mask, int64_t T,
                            int32_t Hd, int64_t V, void* ws, const Layout& Ly, int sms,
@@ -632,6 +648,7 @@ grpo_status grpo_token_logprobs(const uint16_t* H, const uint16_t* W, const int3
   DeviceInfo di;
   if (!device_info(&di)) return GRPO_ERR_UNSUPPORTED;
   if (!get_encode()) return GRPO_ERR_CUDA;
+  if (!(H = hidden_view(H))) return GRPO_ERR_INVALID_ARG;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   cudaError_t e = run_compaction(H, targets, mask, T, Hd, V, ws, Ly, di.sms, s);
   if (e == cudaSuccess) e = run_lse(&W, 1, Hd, V, ws, Ly, di, s);
@@ -663,6 +680,7 @@ grpo_status grpo_token_logprobs_heads(const uint16_t* H, const uint16_t* const* 
   DeviceInfo di;
   if (!device_info(&di)) return GRPO_ERR_UNSUPPORTED;
   if (!get_encode()) return GRPO_ERR_CUDA;
+  if (!(H = hidden_view(H))) return GRPO_ERR_INVALID_ARG;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   cudaError_t e = run_compaction(H, targets, mask, T, Hd, V, ws, Ly, di.sms, s);
   if (e == cudaSuccess) e = run_lse(W_heads, n_heads, Hd, V, ws, Ly, di, s);
@@ -697,6 +715,7 @@ grpo_status grpo_sample_tokens(const uint16_t* H, const uint16_t* W, const uint8
   DeviceInfo di;
   if (!device_info(&di)) return GRPO_ERR_UNSUPPORTED;
   if (!get_encode()) return GRPO_ERR_CUDA;
+  if (!(H = hidden_view(H))) return GRPO_ERR_INVALID_ARG;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   cudaError_t e = run_compaction(H, nullptr, mask, T, Hd, V, ws, Ly, di.sms, s);
   if (e == cudaSuccess) {
@@ -758,6 +777,7 @@ grpo_status grpo_sample_tokens_top_p(const uint16_t* H, const uint16_t* W, const
   DeviceInfo di;
   if (!device_info(&di)) return GRPO_ERR_UNSUPPORTED;
   if (!get_encode()) return GRPO_ERR_CUDA;
+  if (!(H = hidden_view(H))) return GRPO_ERR_INVALID_ARG;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   // the sampling GEMM (running LSE and the plain Gumbel-max winner per split),
   // storing the logits of every unmasked row for the nucleus selection
@@ -987,6 +1007,7 @@ grpo_status loss_impl(const uint16_t* H, const uint16_t* W, const int32_t* targe
   DeviceInfo di;
   if (!device_info(&di)) return GRPO_ERR_UNSUPPORTED;
   if (!get_encode()) return GRPO_ERR_CUDA;
+  if (!(H = hidden_view(H))) return GRPO_ERR_INVALID_ARG;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   const int sms = di.sms;
   int* n_valid = at<int>(ws, Ly.n_valid);
