@@ -149,12 +149,14 @@ _in_flight = []
 
 
 def _keep_until_done(t: torch.Tensor, dev: torch.device) -> None:
-    while _in_flight and _in_flight[0][0].query():
-        _in_flight.pop(0)
-    if not t.is_cuda:
-        ev = torch.cuda.Event()
-        ev.record(torch.cuda.current_stream(dev))
-        _in_flight.append((ev, t))
+    if t.is_cuda:
+        return
+    if not torch.cuda.is_current_stream_capturing():  # no event queries inside a graph capture
+        while _in_flight and _in_flight[0][0].query():
+            _in_flight.pop(0)
+    ev = torch.cuda.Event()
+    ev.record(torch.cuda.current_stream(dev))
+    _in_flight.append((ev, t))
 
 
 def _shape(t: torch.Tensor, shape, name: str) -> None:
