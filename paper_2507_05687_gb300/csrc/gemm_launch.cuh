@@ -94,6 +94,38 @@ inline bool hct_blocks(int64_t T_pad) {
   return T_pad * 2 > kMaxTransposedRowBytes;
 }
 
+// Pace gate of the forward and sampling GEMMs (GemmArgs::gate): how many
+// vocabulary tiles a CTA may run ahead of the slowest CTAs of the grid, and
+// how many CTAs (per 64) may lag further; GRPO_GATE="slack[,lag]" overrides
+// them (slack 0: no gate).
+constexpr int kGateSlack = 2;
+constexpr int kGateLagPer64 = 0;
+constexpr int kGateSlots = 1024;  // CTAs a workspace's gate array holds
+
+// Whether GEMM `which` (LSE and sampling forwards, dZ, dH, dW) takes the pace
+// gate; GRPO_GATE_GEMMS="l,z,h,w" (1 or 0 each) overrides the defaults.
+inline bool gate_on(int which) {
+  int g[4] = {1, 0, 0, 0};
+  if (const char* e = std::getenv("GRPO_GATE_GEMMS")) {
+    int v[4];
+    if (std::sscanf(e, "%d,%d,%d,%d", &v[0], &v[1], &v[2], &v[3]) == 4)
+      for (int i = 0; i < 4; ++i) g[i] = v[i] != 0;
+  }
+  return g[which] != 0;
+}
+
+inline void gate_params(int grid, int* slack, int* lag) {
+  int s = kGateSlack, l = kGateLagPer64;
+  if (const char* e = std::getenv("GRPO_GATE")) {
+    int a = -1, b = -1;
+    const int n = std::sscanf(e, "%d,%d", &a, &b);
+    if (n >= 1 && a >= 0) s = a;
+    if (n == 2 && b >= 0 && b <= 64) l = b;
+  }
+  *slack = s;
+  *lag = grid * l / 64;
+}
+
 // 2-CTA (cta_group::2) tiles unless GRPO_CTA_PAIR=0.
 inline bool use_pairs() {
   const char* e = std::getenv("GRPO_CTA_PAIR");

@@ -50,6 +50,8 @@
 // MN-major.
 #pragma once
 
+#include <climits>
+
 #include <cuda.h>
 #include <stdint.h>
 
@@ -136,6 +138,10 @@ struct GemmArgs {
                         // k-block number drop_kblock1 - 1 (0: never), so a wait runs out
   int drop_adam1;       // the same for kEpiAdam: CTA 0's epilogue warp 0 skips the loads of
                         // its weight block number drop_adam1 - 1 (0: never)
+  int* gate;            // [gridDim.x] tiles each CTA has begun, zeroed before the launch
+                        // (nullptr: no gate); see gate_wait
+  int gate_slack;       // tiles a CTA may run ahead of the slowest ones
+  int gate_lag;         // CTAs allowed to lag further behind
 
   // kEpiLse
   const int* yc;        // [M] target of each compacted row (-1: none)
@@ -216,6 +222,40 @@ __device__ __forceinline__ void unit_coords(const GemmArgs& a, const TileSched& 
   const int w = u - g * per_group;
   mt = first + w % gm;
   un = w / gm;
+}
+
+// The pace gate of the persistent grid.  The CTAs sweeping one raster group
+// read each B tile at about the same time only while they stay in step; left
+// alone they drift apart by up to a work unit (the CTAs of a column start
+// their units in different rounds), the B tiles between a column's first and
+// last reader outgrow L2, and B is read from DRAM several times (measured: a
+// W tile's readers spread over a median 13 tiles and the forward reading
+// 24 GB for 5 GB of raster groups at 19,572 rows).  Each CTA publishes the
+// number of tiles it has begun; before its k-th tile the producer warp waits
+// until all CTAs but `lag` have begun tile k - slack.  The wait is a pace hint, not a
+// dependency: it gives up after kGateNs and the CTA goes on, so it can delay a
+// CTA but never stop one (a CTA that has issued all its loads publishes
+// INT_MAX).
+constexpr unsigned long long kGateNs = 200000ull;  // 200 us
+
+__device__ __forceinline__ void gate_wait(int* gate, int slack, int lag, int k, int lane) {
+  volatile int* g = gate;
+  if (lane == 0) g[blockIdx.x] = k;
+  if (k <= slack) return;
+  const int need = k - slack;
+  const int n = static_cast<int>(gridDim.x);
+  unsigned long long t0 = 0;
+  for (;;) {
+    int behind = 0;  // CTAs that have not begun tile `need` yet
+    for (int i = lane; i < n; i += 32) behind += g[i] < need;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) behind += __shfl_xor_sync(0xffffffffu, behind, o);
+    if (behind <= lag) return;
+    const unsigned long long now = global_timer_ns();
+    if (t0 == 0) t0 = now;
+    else if (now - t0 > kGateNs) return;
+    __nanosleep(256);
+  }
 }
 
 // ---------------------------------------------------------------- epilogue
@@ -607,7 +647,8 @@ __device__ __forceinline__ void gemm_body(const CUtensorMap* tmA, const CUtensor
 
   if (warp == 0) {
     // ------------------------------------------------------------ producer
-    if (lane == 0) {
+    // Lane 0 issues the copies; the whole warp takes the pace gate between tiles.
+    {
       const uint64_t pol_a = l2_policy(args.a_hint);
       const uint64_t pol_b = l2_policy(args.b_hint);
       int stage = 0;
@@ -617,6 +658,7 @@ __device__ __forceinline__ void gemm_body(const CUtensorMap* tmA, const CUtensor
       for (int s = 0; s < kStages; ++s) uses[s] = 0;
       bool ok = true;
       int kblock_count = 0;  // k-blocks this CTA has staged (fault-injection hook)
+      int tiles_begun = 0;
       for (int u = unit0; u < sch.total && ok; u += unit_stride) {
         int mt, un;
         unit_coords(args, sch, u, mt, un);
@@ -624,7 +666,9 @@ __device__ __forceinline__ void gemm_body(const CUtensorMap* tmA, const CUtensor
         const int nt0 = (un - head * sch.units_head) * args.n_per_unit;
         const int nt1 = min(sch.n_tiles, nt0 + args.n_per_unit);
         for (int nt = nt0; nt < nt1 && ok; ++nt) {
-          for (int kb = 0; kb < KB; ++kb) {
+          if (args.gate) gate_wait(args.gate, args.gate_slack, args.gate_lag, tiles_begun, lane);
+          ++tiles_begun;
+          for (int kb = 0; kb < KB && lane == 0; ++kb) {
             if (!mbar_wait(smem_addr(&empty_bar[stage]), phase ^ 1u, abort_flag, wlim)) {
               ok = false;
               break;
@@ -670,12 +714,17 @@ __device__ __forceinline__ void gemm_body(const CUtensorMap* tmA, const CUtensor
               phase ^= 1u;
             }
           }
+          ok = __shfl_sync(0xffffffffu, ok, 0);
         }
       }
-      if (!ok) raise_abort();
+      if (args.gate && lane == 0) {  // every copy issued: nobody waits for this CTA any more
+        volatile int* g = args.gate;
+        g[blockIdx.x] = INT_MAX;
+      }
+      if (lane == 0 && !ok) raise_abort();
       // Every stage this CTA filled must have been consumed (so its copies
       // have landed) before the CTA can exit.
-      for (int s = 0; s < kStages; ++s)
+      for (int s = 0; s < kStages && lane == 0; ++s)
         if (uses[s] > 0)
           mbar_wait(smem_addr(&empty_bar[s]), static_cast<uint32_t>(uses[s] - 1) & 1u, abort_flag, wlim);
       // After an abort those waits give up at once, and a stage may still
@@ -686,7 +735,7 @@ __device__ __forceinline__ void gemm_body(const CUtensorMap* tmA, const CUtensor
       // drain ends).  Where that phase cannot complete (a copy that was never
       // issued), and on the peer, whose copies only the issuing CTA's
       // barriers count, a fixed pause stands in for the wait.
-      if (*abort_flag) {
+      if (lane == 0 && *abort_flag) {
         bool drained = issuer;
         if (issuer) {
           volatile int never = 0;

@@ -35,7 +35,7 @@ struct Layout {
   int64_t T_pad, rows, nsplit, nblk_scan, nblk_loss, vchunk;
   int64_t ldz;    // leading dimension (fp32 elements) of the stored logits; 0: not stored
   int lse_tiles;  // vocabulary tiles (of 256) per forward work unit
-  size_t status, n_valid, counts, offsets, cidx, rank_of, yc, zy, part_m, part_s, lse_c, g_c,
+  size_t status, n_valid, gate, counts, offsets, cidx, rank_of, yc, zy, part_m, part_s, lse_c, g_c,
       block_loss, resp_len, best_s, best_c, best_z, Hc, HcT, dz, dhc, z, slow_rows, slow_tgt, n_slow, row_above,
       row_done, total;
 };
@@ -74,6 +74,7 @@ bool make_layout(int64_t T, int32_t Hd, int64_t V, int32_t which, Layout* L, int
   const size_t cr = static_cast<size_t>(L->rows);   // compacted rows
   L->status = take(4, 256);
   L->n_valid = take(4, 4);
+  L->gate = take(4 * kGateSlots, 256);  // the forward GEMM's pace gate, one counter per CTA
   L->counts = take(4 * L->nblk_scan, 256);
   L->offsets = take(4 * L->nblk_scan, 256);
   L->cidx = take(4 * cr, 256);
@@ -440,14 +441,24 @@ cudaError_t launch_gemm_cfg(const Operand& A, const Operand* B, const GemmArgs& 
   const unsigned grid = static_cast<unsigned>(
       kPair == 2 ? 2 * std::max<int64_t>(1, std::min<int64_t>(di.pairs, units))
                  : std::max<int64_t>(1, std::min<int64_t>(di.sms, units)));
+  GemmArgs ag = a;
+  if (ag.gate) {
+    gate_params(static_cast<int>(grid), &ag.gate_slack, &ag.gate_lag);
+    if (ag.gate_slack <= 0 || grid > static_cast<unsigned>(kGateSlots)) {
+      ag.gate = nullptr;
+    } else {
+      const cudaError_t e = cudaMemsetAsync(ag.gate, 0, grid * sizeof(int), s);
+      if (e != cudaSuccess) return e;
+    }
+  }
   auto go = [&](auto blk_tag) {
     constexpr bool BLK = decltype(blk_tag)::value;
     if (kPair == 2)
       gemm_tc_pair_kernel<E, AMN, BMN, BLK><<<grid, EpiShape<E>::kThreads, smem_bytes<2, E>(), s>>>(
-          ta, tb[0], tb[1], tb[2], tb[3], td, a);
+          ta, tb[0], tb[1], tb[2], tb[3], td, ag);
     else
       gemm_tc_kernel<E, AMN, BMN, BLK><<<grid, EpiShape<E>::kThreads, smem_bytes<1, E>(), s>>>(
-          ta, tb[0], tb[1], tb[2], tb[3], td, a);
+          ta, tb[0], tb[1], tb[2], tb[3], td, ag);
   };
   if constexpr (kBlkOk) {
     if (blk) go(std::true_type{});
@@ -531,6 +542,7 @@ cudaError_t run_lse(const uint16_t* const* W, int n_heads, int32_t Hd, int64_t V
   a.n_per_unit = Ly.lse_tiles;
   a.n_heads = n_heads;
   a.group_m = group_m(Ly.ldz > 0 ? 4 : 0);
+  if (gate_on(0)) a.gate = at<int>(ws, Ly.gate);
   // Fault-injection test hook (failure-detection tests): GRPO_TEST_DROP_KBLOCK=k
   // makes CTA 0 skip the copies of its k-th k-block (1-based) so its pipeline
   // wait runs out after 0.2 s and the call reports GRPO_ERR_TIMEOUT.
@@ -727,6 +739,7 @@ grpo_status grpo_sample_tokens(const uint16_t* H, const uint16_t* W, const uint8
     a.n_per_unit = Ly.lse_tiles;
     a.n_heads = 1;
     a.group_m = group_m(0);
+    if (gate_on(0)) a.gate = at<int>(ws, Ly.gate);
     l2_hints(0, &a.a_hint, &a.b_hint);
     a.status = at<unsigned>(ws, Ly.status);
     a.row_map = at<int>(ws, Ly.cidx);
@@ -791,6 +804,7 @@ grpo_status grpo_sample_tokens_top_p(const uint16_t* H, const uint16_t* W, const
     a.n_per_unit = Ly.lse_tiles;
     a.n_heads = 1;
     a.group_m = group_m(4);
+    if (gate_on(0)) a.gate = at<int>(ws, Ly.gate);
     l2_hints(0, &a.a_hint, &a.b_hint);
     a.status = at<unsigned>(ws, Ly.status);
     a.row_map = at<int>(ws, Ly.cidx);
@@ -1082,6 +1096,7 @@ grpo_status loss_impl(const uint16_t* H, const uint16_t* W, const int32_t* targe
       a.n_per_unit = units_n(0);
       a.group_m = group_m(1);
       a.group_n = group_n(1);
+      if (gate_on(1)) a.gate = at<int>(ws, Ly.gate);
       l2_hints(1, &a.a_hint, &a.b_hint);
       a.status = status;
       a.yc = at<int>(ws, Ly.yc);
@@ -1100,6 +1115,7 @@ grpo_status loss_impl(const uint16_t* H, const uint16_t* W, const int32_t* targe
       h.b_off_k = static_cast<int>(c0);
       h.n_per_unit = units_n(1);
       h.group_m = group_m(2);
+      if (gate_on(2)) h.gate = at<int>(ws, Ly.gate);
       l2_hints(2, &h.a_hint, &h.b_hint);
       h.status = status;
       h.accumulate = c0 > 0;
@@ -1115,6 +1131,7 @@ grpo_status loss_impl(const uint16_t* H, const uint16_t* W, const int32_t* targe
       w.k_dyn = 1;
       w.n_per_unit = units_n(2);
       w.group_m = group_m(3);
+      if (gate_on(3)) w.gate = at<int>(ws, Ly.gate);
       l2_hints(3, &w.a_hint, &w.b_hint);
       w.status = status;
       w.accumulate = 0;
