@@ -535,3 +535,28 @@ def test_binding_rejects_mismatched_shapes():
         grpo.sample_tokens(d["H"], d["W"], d["m"][:-1])
     # and the well-formed call still works
     grpo.loss_fwd_bwd(*args)
+
+
+def test_paced_forward_gives_the_same_bits(monkeypatch):
+    """The forward and sampling GEMMs pace their persistent grid (a bounded
+    wait between tiles, for batches of at least 4096 rows); the pace changes
+    only when a CTA issues its copies, so the log-probs, the loss and its
+    gradients, and a draw are the same bits with the gate off, at its default
+    and at its tightest, and match the oracle."""
+    w = wl.Workload("t", 4, 4, 512, 128, 4096, "uniform", 200, 512, seed=wl.SEED_BASE + 1650)
+    c = _case(w)
+    assert int(c["m"].sum()) >= 4096 and w.T >= 4096
+    d = _dev(c)
+    got = {}
+    for gate in ("0", "2", "1", None):
+        if gate is None:
+            monkeypatch.delenv("GRPO_GATE", raising=False)
+        else:
+            monkeypatch.setenv("GRPO_GATE", gate)
+        lp = grpo.token_logprobs(d["H"], d["W"], d["y"], d["m"])
+        loss, dH, dW = _check_fwd_bwd(c)
+        tok, tlp = grpo.sample_tokens(d["H"], d["W"], d["m"], 1.0, seed=3, offset=1)
+        got[gate] = (lp, loss, dH, dW, tok, tlp)
+    for gate in ("2", "1", None):
+        for x, y in zip(got[gate], got["0"]):
+            assert torch.equal(x, y), gate
