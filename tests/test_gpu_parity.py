@@ -547,16 +547,19 @@ def test_paced_forward_gives_the_same_bits(monkeypatch):
     c = _case(w)
     assert int(c["m"].sum()) >= 4096 and w.T >= 4096
     d = _dev(c)
-    got = {}
-    for gate in ("0", "2", "1", None):
-        if gate is None:
-            monkeypatch.delenv("GRPO_GATE", raising=False)
-        else:
-            monkeypatch.setenv("GRPO_GATE", gate)
-        lp = grpo.token_logprobs(d["H"], d["W"], d["y"], d["m"])
-        loss, dH, dW = _check_fwd_bwd(c)
-        tok, tlp = grpo.sample_tokens(d["H"], d["W"], d["m"], 1.0, seed=3, offset=1)
-        got[gate] = (lp, loss, dH, dW, tok, tlp)
-    for gate in ("2", "1", None):
-        for x, y in zip(got[gate], got["0"]):
-            assert torch.equal(x, y), gate
+    for pair in ("1", "0"):  # 2-CTA and single-CTA tiles (the gate counts CTAs either way)
+        monkeypatch.setenv("GRPO_CTA_PAIR", pair)
+        got = {}
+        for gate in ("0", "2", "1", None):
+            if gate is None:
+                monkeypatch.delenv("GRPO_GATE", raising=False)
+            else:
+                monkeypatch.setenv("GRPO_GATE", gate)
+            lp = grpo.token_logprobs(d["H"], d["W"], d["y"], d["m"])
+            loss, dH, dW = _check_fwd_bwd(c)
+            tok, tlp = grpo.sample_tokens(d["H"], d["W"], d["m"], 1.0, seed=3, offset=1)
+            got[gate] = (lp, loss, dH, dW, tok, tlp)
+        for gate in ("2", "1", None):
+            for x, y in zip(got[gate], got["0"]):
+                assert torch.equal(x, y), (pair, gate)
+    monkeypatch.delenv("GRPO_CTA_PAIR")
