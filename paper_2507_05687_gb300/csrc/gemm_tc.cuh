@@ -232,30 +232,52 @@ __device__ __forceinline__ void unit_coords(const GemmArgs& a, const TileSched& 
 // W tile's readers spread over a median 13 tiles and the forward reading
 // 24 GB for 5 GB of raster groups at 19,572 rows).  Each CTA publishes the
 // number of tiles it has begun; before its k-th tile the producer warp waits
-// until all CTAs but `lag` have begun tile k - slack.  The wait is a pace hint, not a
-// dependency: it gives up after kGateNs and the CTA goes on, so it can delay a
-// CTA but never stop one (a CTA that has issued all its loads publishes
+// until all CTAs but `lag` have begun tile k - slack.  The counters it tests
+// were loaded when the previous tile began (so their latency hides behind that
+// tile's copies, and a CTA in step goes on at once); only when those stale
+// values fall short does it poll afresh.  The wait is a pace hint, not a
+// dependency: it gives up after kGateNs and the CTA goes on, so it can delay
+// a CTA but never stop one (a CTA that has issued all its loads publishes
 // INT_MAX).
 constexpr unsigned long long kGateNs = 200000ull;  // 200 us
+constexpr int kGateMaxCtas = 160;                   // counters a lane prefetches: 5 x 32
+static_assert(kGateMaxCtas % 32 == 0, "whole counters per lane");
 
-__device__ __forceinline__ void gate_wait(int* gate, int slack, int lag, int k, int lane) {
-  volatile int* g = gate;
-  if (lane == 0) g[blockIdx.x] = k;
-  if (k <= slack) return;
-  const int need = k - slack;
-  const int n = static_cast<int>(gridDim.x);
-  unsigned long long t0 = 0;
-  for (;;) {
-    int behind = 0;  // CTAs that have not begun tile `need` yet
-    for (int i = lane; i < n; i += 32) behind += g[i] < need;
+struct GatePrefetch {
+  int v[kGateMaxCtas / 32];  // counters i = lane + 32 j, as loaded when the previous tile began
+};
+
+__device__ __forceinline__ int gate_behind(const GatePrefetch& p, int need, int n, int lane) {
+  int behind = 0;
 #pragma unroll
-    for (int o = 16; o > 0; o >>= 1) behind += __shfl_xor_sync(0xffffffffu, behind, o);
-    if (behind <= lag) return;
-    const unsigned long long now = global_timer_ns();
-    if (t0 == 0) t0 = now;
-    else if (now - t0 > kGateNs) return;
-    __nanosleep(256);
+  for (int j = 0; j < kGateMaxCtas / 32; ++j) behind += lane + 32 * j < n && p.v[j] < need;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) behind += __shfl_xor_sync(0xffffffffu, behind, o);
+  return behind;
+}
+
+__device__ __forceinline__ void gate_load(GatePrefetch& p, const volatile int* g, int n, int lane) {
+#pragma unroll
+  for (int j = 0; j < kGateMaxCtas / 32; ++j) p.v[j] = lane + 32 * j < n ? g[lane + 32 * j] : INT_MAX;
+}
+
+__device__ __forceinline__ void gate_wait(int* gate, int slack, int lag, int k, int lane, GatePrefetch& pre) {
+  volatile int* g = gate;
+  const int n = static_cast<int>(gridDim.x);
+  if (lane == 0) g[blockIdx.x] = k;
+  if (k > slack) {
+    const int need = k - slack;
+    if (gate_behind(pre, need, n, lane) > lag) {  // the stale counters fall short: poll
+      const unsigned long long t0 = global_timer_ns();
+      for (;;) {
+        gate_load(pre, g, n, lane);
+        if (gate_behind(pre, need, n, lane) <= lag) break;
+        if (global_timer_ns() - t0 > kGateNs) break;
+        __nanosleep(64);
+      }
+    }
   }
+  gate_load(pre, g, n, lane);  // for the next tile: consumed when it begins
 }
 
 // ---------------------------------------------------------------- epilogue
@@ -659,6 +681,9 @@ __device__ __forceinline__ void gemm_body(const CUtensorMap* tmA, const CUtensor
       bool ok = true;
       int kblock_count = 0;  // k-blocks this CTA has staged (fault-injection hook)
       int tiles_begun = 0;
+      GatePrefetch gate_pre;
+#pragma unroll
+      for (int j = 0; j < kGateMaxCtas / 32; ++j) gate_pre.v[j] = 0;
       for (int u = unit0; u < sch.total && ok; u += unit_stride) {
         int mt, un;
         unit_coords(args, sch, u, mt, un);
@@ -666,7 +691,7 @@ __device__ __forceinline__ void gemm_body(const CUtensorMap* tmA, const CUtensor
         const int nt0 = (un - head * sch.units_head) * args.n_per_unit;
         const int nt1 = min(sch.n_tiles, nt0 + args.n_per_unit);
         for (int nt = nt0; nt < nt1 && ok; ++nt) {
-          if (args.gate) gate_wait(args.gate, args.gate_slack, args.gate_lag, tiles_begun, lane);
+          if (args.gate) gate_wait(args.gate, args.gate_slack, args.gate_lag, tiles_begun, lane, gate_pre);
           ++tiles_begun;
           for (int kb = 0; kb < KB && lane == 0; ++kb) {
             if (!mbar_wait(smem_addr(&empty_bar[stage]), phase ^ 1u, abort_flag, wlim)) {

@@ -444,7 +444,7 @@ cudaError_t launch_gemm_cfg(const Operand& A, const Operand* B, const GemmArgs& 
   GemmArgs ag = a;
   if (ag.gate) {
     gate_params(static_cast<int>(grid), &ag.gate_slack, &ag.gate_lag);
-    if (ag.gate_slack <= 0 || grid > static_cast<unsigned>(kGateSlots) || max_m_rows < kGateMinRows) {
+    if (ag.gate_slack <= 0 || grid > static_cast<unsigned>(kGateMaxCtas) || max_m_rows < kGateMinRows) {
       ag.gate = nullptr;
     } else {
       const cudaError_t e = cudaMemsetAsync(ag.gate, 0, grid * sizeof(int), s);
