@@ -98,7 +98,7 @@ inline bool hct_blocks(int64_t T_pad) {
 // vocabulary tiles a CTA may run ahead of the slowest CTAs of the grid, and
 // how many CTAs (per 64) may lag further; GRPO_GATE="slack[,lag]" overrides
 // them (slack 0: no gate).
-constexpr int kGateSlack = 2;
+constexpr int kGateSlack = 1;  // tested against counters a tile old: about 2 tiles of spread
 constexpr int kGateLagPer64 = 0;
 constexpr int kGateSlots = 1024;  // CTAs a workspace's gate array holds
 // Batches of fewer rows take no gate: a decode step's forward reads W about

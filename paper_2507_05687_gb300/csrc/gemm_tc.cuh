@@ -232,7 +232,7 @@ __device__ __forceinline__ void unit_coords(const GemmArgs& a, const TileSched& 
 // W tile's readers spread over a median 13 tiles and the forward reading
 // 24 GB for 5 GB of raster groups at 19,572 rows).  Each CTA publishes the
 // number of tiles it has begun; before its k-th tile the producer warp waits
-// until all CTAs but `lag` have begun tile k - slack.  The counters it tests
+// until all CTAs but `lag` had begun tile k - slack.  The counters it tests
 // were loaded when the previous tile began (so their latency hides behind that
 // tile's copies, and a CTA in step goes on at once); only when those stale
 // values fall short does it poll afresh.  The wait is a pace hint, not a
