@@ -68,7 +68,7 @@ static_assert(kTopPBuckets % (kTopPCtas * kTopPThreads) == 0, "whole histogram b
 // the cluster only (the other CTAs write into and read from CTA 0's copy).
 struct TopPShared {
   union {
-    unsigned long long hist[kTopPBuckets];  // histogram pass: this CTA's histogram; host: then the merged one
+    unsigned long long hist[kTopPBuckets];  // histogram pass: this CTA's histogram; then its slice merged
     struct {                                // gather pass: this CTA's candidates before they are broadcast
       float y[kTopPCand];
     } loc;
@@ -79,8 +79,9 @@ struct TopPShared {
   };
   float cy[kTopPCand];                      // the cluster's candidates: every CTA holds all of them
   unsigned long long cq[kTopPCand];
-  unsigned long long scan[kTopPThreads];    // host: per-thread bucket-range sums of the scan
-  // host, one value per CTA: the range of its candidates, its part of the threshold search, its best draw
+  unsigned long long tot[kTopPCtas];        // every CTA: the merged mass of each CTA's histogram slice
+  // one value per CTA: host only, the range of its candidates and its best draw; every CTA, its
+  // part of the threshold search
   uint32_t slot_lo[kTopPCtas], slot_hi[kTopPCtas], slot_r[kTopPCtas], slot_f[kTopPCtas], slot_g[kTopPCtas],
       slot_i[kTopPCtas];
   float lvl_hi[kTopPLevels];
@@ -89,12 +90,12 @@ struct TopPShared {
   unsigned long long ra[kTopPWarps];
   float rf[kTopPWarps], rg[kTopPWarps];
   int ri[kTopPWarps];
-  unsigned long long cum_before;            // host, copied to every CTA
+  unsigned long long cum_before;            // every CTA: the mass above the chosen buckets
+  unsigned long long cum_next;              // every CTA: cum_before of the next level, from the CTA that found it
   unsigned ncand;                           // host: the reservation counter; every CTA: the cluster's count
   unsigned lcand, lbase;                    // this CTA's candidate count and its offset in the cluster's list
   float ystar;
   int full;                                 // the threshold is known but the candidates did not all fit
-  int skip;                                 // the row's exact mass above its winner is below the target
 };
 
 // Probability of tempered logit y in 2^-40 units, truncated toward zero: the
@@ -263,6 +264,7 @@ __global__ void __cluster_dims__(kC, 1, 1) __launch_bounds__(kTopPThreads, 4)
     float bs, by;  // this thread's best perturbed score, its token and logit (the draw below)
     int bv;
     int L = 0;
+    bool skip_row = false;  // the row keeps its plain draw
     for (;;) {
       __syncthreads();
       for (int b = tid; b < kTopPBuckets; b += kTopPThreads) sh.hist[b] = 0ull;
@@ -284,9 +286,10 @@ __global__ void __cluster_dims__(kC, 1, 1) __launch_bounds__(kTopPThreads, 4)
       }
       cluster_sync();
       {  // merge the histograms: CTA k sums its slice of kMerge * kTopPThreads buckets over the
-         // cluster in rank order and leaves the sums in CTA 0's histogram (disjoint slices, so no
-         // CTA reads a bucket another one writes)
+         // cluster in rank order into its own histogram (only CTA k reads the buckets of slice k,
+         // so no CTA reads a bucket another one writes) and sends the slice's total to every CTA
         constexpr int kMerge = kTopPBuckets / (kC * kTopPThreads);
+        unsigned long long t = 0ull;
 #pragma unroll
         for (int j = 0; j < kMerge; ++j) {
           const int b = (rank * kMerge + j) * kTopPThreads + tid;
@@ -296,80 +299,103 @@ __global__ void __cluster_dims__(kC, 1, 1) __launch_bounds__(kTopPThreads, 4)
           unsigned long long m = 0ull;
 #pragma unroll
           for (int k = 0; k < kC; ++k) m += part[k];
-          st_shared_cluster_u64(atk(&sh.hist[b], 0), m);
+          sh.hist[b] = m;
+          t += m;
         }
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) t += __shfl_xor_sync(0xffffffffu, t, o);
+        if ((tid & 31) == 0) sh.ra[tid >> 5] = t;
+        __syncthreads();
+        if (tid < kC) {
+          unsigned long long sum = 0ull;
+          for (int w = 0; w < kTopPWarps; ++w) sum += sh.ra[w];
+          st_shared_cluster_u64(atk(&sh.tot[rank], tid), sum);
+        }
+        if (host && tid == 0) sh.ncand = 0u;  // nobody reserves candidates before the next barrier
       }
       cluster_sync();
-      if (host) {  // find the bucket that holds the threshold
-        // the first bucket where the mass from the top reaches the target: each
-        // thread sums a range of buckets, thread 0 walks the range sums and then
-        // the buckets of the one range that crosses
-        constexpr int kPer = kTopPBuckets / kTopPThreads;
-        unsigned long long part = 0ull;
-#pragma unroll
-        for (int i = 0; i < kPer; ++i) part += sh.hist[tid * kPer + i];
-        sh.scan[tid] = part;
-        __syncthreads();
-        if (tid < 32) {
-          // warp 0: lane l owns segments [l * kSeg, (l + 1) * kSeg); an inclusive
-          // scan of the lane sums finds the lane whose segments cross
-          constexpr int kSeg = kTopPThreads / 32;
-          unsigned long long own = 0ull;
-#pragma unroll
-          for (int i = 0; i < kSeg; ++i) own += sh.scan[tid * kSeg + i];
-          unsigned long long inc = own;
+      // The slice that holds the threshold: the first where the mass from the top
+      // reaches the target.  Every CTA decides alike from the same totals.
+      int cs = -1;
+      unsigned long long before = sh.cum_before;
+      for (int k = 0; k < kC; ++k) {
+        if (before + sh.tot[k] >= target) {
+          cs = k;
+          break;
+        }
+        before += sh.tot[k];
+      }
+      // level 0 holds every logit above the winner: when even their exact mass
+      // falls short of the target, the winner is in the nucleus (no CTA touches
+      // another's shared memory after the barrier above in this row)
+      if (L == 0 && cs < 0) {
+        skip_row = true;
+        break;
+      }
+      if (cs < 0) {  // (the masses fell short at a deeper level) the last bucket, as a scan would end
+        cs = kC - 1;
+        before -= sh.tot[kC - 1];
+      }
+      if (rank == cs) {  // the bucket within this slice, by block scans of kTopPThreads buckets at a time
+        constexpr int kMerge = kTopPBuckets / (kC * kTopPThreads);
+        const int lane = tid & 31, warp = tid >> 5;
+        unsigned long long acc = before;
+        int found = -1;
+        unsigned long long found_cum = 0ull;
+        for (int j = 0; j < kMerge && found < 0; ++j) {
+          const int b = (rank * kMerge + j) * kTopPThreads + tid;
+          const unsigned long long v = sh.hist[b];
+          unsigned long long inc = v;
 #pragma unroll
           for (int o = 1; o < 32; o <<= 1) {
             const unsigned long long n = __shfl_up_sync(0xffffffffu, inc, o);
-            if (tid >= o) inc += n;
+            if (lane >= o) inc += n;
           }
-          const unsigned cross = __ballot_sync(0xffffffffu, sh.cum_before + inc >= target);
-          const int ln = cross ? __ffs(cross) - 1 : 31;
-          const unsigned long long before = __shfl_sync(0xffffffffu, inc - own, ln);
-          sh.ra[0] = before;
-          sh.ri[0] = ln;
-          // level 0 holds every logit above the winner: when even their exact
-          // mass falls short of the target, the winner is in the nucleus
-          if (tid == 0) sh.skip = L == 0 && !cross;
+          __syncthreads();  // sh.ra / sh.ri of the previous round read
+          if (lane == 31) sh.ra[warp] = inc;
+          __syncthreads();
+          unsigned long long pre = 0ull, all = 0ull;
+          for (int w = 0; w < kTopPWarps; ++w) {
+            if (w < warp) pre += sh.ra[w];
+            all += sh.ra[w];
+          }
+          inc += pre;
+          const unsigned hit = __ballot_sync(0xffffffffu, acc + inc >= target);
+          __syncthreads();  // every warp has read sh.ra
+          if (lane == 0) sh.ri[warp] = hit ? __ffs(hit) - 1 : 32;
+          __syncthreads();
+          int first = kTopPThreads;
+          for (int w = 0; w < kTopPWarps; ++w)
+            if (sh.ri[w] < 32) {
+              first = w * 32 + sh.ri[w];
+              break;
+            }
+          if (first < kTopPThreads) {
+            found = (rank * kMerge + j) * kTopPThreads + first;
+            if (tid == first) found_cum = acc + inc - v;  // the mass above the bucket
+          } else {
+            acc += all;
+          }
         }
-        __syncthreads();
-        if (tid == 0) {
-          constexpr int kSeg = kTopPThreads / 32;
-          unsigned long long acc = sh.cum_before + sh.ra[0];
-          int seg = sh.ri[0] * kSeg;
-          for (; seg < (sh.ri[0] + 1) * kSeg - 1; ++seg) {
-            if (acc + sh.scan[seg] >= target) break;
-            acc += sh.scan[seg];
+        if (found < 0) {  // no crossing in the last slice: its last bucket (only at a deeper level)
+          found = (rank * kMerge + kMerge - 1) * kTopPThreads + kTopPThreads - 1;
+          if (tid == kTopPThreads - 1) found_cum = acc - sh.hist[found];
+        }
+        // the thread that holds the bucket sends it and the mass above it to every CTA
+        const int holder = found - (found / kTopPThreads) * kTopPThreads;
+        if (tid == holder) {
+          for (int k = 0; k < kC; ++k) {
+            st_shared_cluster(atk(&sh.lvl_b[L], k), static_cast<uint32_t>(found));
+            st_shared_cluster_u64(atk(&sh.cum_next, k), found_cum);
           }
-          int b = seg * kPer;
-          for (; b < (seg + 1) * kPer - 1; ++b) {
-            if (acc + sh.hist[b] >= target) break;
-            acc += sh.hist[b];
-          }
-          sh.cum_before = acc;
-          sh.lvl_b[L] = b;
-          sh.ncand = 0u;
         }
       }
       cluster_sync();
       if (tid == 0) {
-        if (!host) {
-          sh.skip = static_cast<int>(ld_shared_cluster(atk(&sh.skip, 0)));
-          sh.lvl_b[L] = static_cast<int>(ld_shared_cluster(atk(&sh.lvl_b[L], 0)));
-          sh.cum_before = ld_shared_cluster_u64(atk(&sh.cum_before, 0));
-        }
+        sh.cum_before = sh.cum_next;
         sh.lcand = 0u;
       }
       __syncthreads();
-      // A skipped row ends here, after one more cluster barrier: the other
-      // CTAs have just read the host's fields above, and the host must not
-      // move on (or, after its last row, exit, releasing the shared memory
-      // they read) before they have.  In a row that goes on, the host waits at
-      // the next cluster barrier below before it writes any of them again.
-      if (sh.skip) {
-        cluster_sync();
-        break;
-      }
       // gather the bucket's logits (and their range, in case they do not fit)
       // into this CTA's list
       float lo = INFINITY, hi2 = -INFINITY;
@@ -433,11 +459,11 @@ __global__ void __cluster_dims__(kC, 1, 1) __launch_bounds__(kTopPThreads, 4)
       const int nc = static_cast<int>(sh.ncand);
       if (nc <= kTopPCand) {
         const float c = top_p_rank_slice<kC>(sh, nc, rank, target - sh.cum_before);
-        if (tid == 0) st_shared_cluster(atk(&sh.slot_r[rank], 0), __float_as_uint(c));
+        if (tid < kC) st_shared_cluster(atk(&sh.slot_r[rank], tid), __float_as_uint(c));  // to every CTA
         cluster_sync();
         if (tid == 0) {
           float ys = -INFINITY;
-          for (int k = 0; k < kC; ++k) ys = fmaxf(ys, __uint_as_float(ld_shared_cluster(atk(&sh.slot_r[k], 0))));
+          for (int k = 0; k < kC; ++k) ys = fmaxf(ys, __uint_as_float(sh.slot_r[k]));
           sh.ystar = ys;
           sh.full = ys == -INFINITY;  // no crossing (the masses fell short): the whole vocabulary
         }
@@ -447,7 +473,7 @@ __global__ void __cluster_dims__(kC, 1, 1) __launch_bounds__(kTopPThreads, 4)
       if (sh.full) break;
       ++L;
     }
-    if (sh.skip) continue;  // the plain draw (already written) stands
+    if (skip_row) continue;  // the plain draw (already written) stands
     // The draw: the best perturbed score over the logits y >= y*, the lowest
     // token on ties.  The sampling GEMM kept, for every split entry (a
     // vocabulary unit of unit_tiles tiles, one column half of each tile), its
