@@ -239,7 +239,10 @@ __device__ __forceinline__ void unit_coords(const GemmArgs& a, const TileSched& 
 // dependency: it gives up after kGateNs and the CTA goes on, so it can delay
 // a CTA but never stop one (a CTA that has issued all its loads publishes
 // INT_MAX).
-constexpr unsigned long long kGateNs = 200000ull;  // 200 us
+// A CTA never waits longer than a couple of tiles' time (about 20 us each at
+// the 8B shape): in step the waits are far shorter, and a CTA that cannot
+// start (its SM held by other work) should not hold the grid back for long.
+constexpr unsigned long long kGateNs = 50000ull;  // 50 us
 constexpr int kGateMaxCtas = 160;                   // counters a lane prefetches: 5 x 32
 static_assert(kGateMaxCtas % 32 == 0, "whole counters per lane");
 
