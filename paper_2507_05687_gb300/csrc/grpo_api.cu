@@ -665,7 +665,7 @@ grpo_status grpo_token_logprobs(const uint16_t* H, const uint16_t* W, const int3
   cudaError_t e = run_compaction(H, targets, mask, T, Hd, V, ws, Ly, di.sms, s);
   if (e == cudaSuccess) e = run_lse(&W, 1, Hd, V, ws, Ly, di, s);
   if (e == cudaSuccess) {
-    const int blocks = static_cast<int>(std::min<int64_t>((T + 255) / 256, di.sms * 16));
+    const int blocks = static_cast<int>(std::min<int64_t>((T + 7) / 8, di.sms * 16));  // a warp per row
     TraceScope trace(GRPO_K_LOGP_MERGE, 0, s);
     logp_merge_kernel<<<blocks, 256, 0, s>>>(mask, at<int>(ws, Ly.rank_of), T, at<float>(ws, Ly.part_m),
                                              at<float>(ws, Ly.part_s), static_cast<int>(Ly.nsplit),
@@ -697,7 +697,7 @@ grpo_status grpo_token_logprobs_heads(const uint16_t* H, const uint16_t* const* 
   cudaError_t e = run_compaction(H, targets, mask, T, Hd, V, ws, Ly, di.sms, s);
   if (e == cudaSuccess) e = run_lse(W_heads, n_heads, Hd, V, ws, Ly, di, s);
   if (e == cudaSuccess) {
-    const int blocks = static_cast<int>(std::min<int64_t>((T + 255) / 256, di.sms * 16));
+    const int blocks = static_cast<int>(std::min<int64_t>((T + 7) / 8, di.sms * 16));  // a warp per row
     TraceScope trace(GRPO_K_LOGP_MERGE, 0, s);
     for (int h = 0; h < n_heads && e == cudaSuccess; ++h) {
       const size_t head_parts = static_cast<size_t>(h) * Ly.nsplit * Ly.rows;
@@ -761,7 +761,7 @@ grpo_status grpo_sample_tokens(const uint16_t* H, const uint16_t* W, const uint8
     e = launch_gemm<kEpiSample, false, false>(A, B, a, Ly.rows, di, s);
   }
   if (e == cudaSuccess) {
-    const int blocks = static_cast<int>(std::min<int64_t>((T + 255) / 256, di.sms * 16));
+    const int blocks = static_cast<int>(std::min<int64_t>((T + 7) / 8, di.sms * 16));  // a warp per row
     TraceScope trace(GRPO_K_LOGP_MERGE, 0, s);
     sample_merge_kernel<<<blocks, 256, 0, s>>>(mask, at<int>(ws, Ly.rank_of), T, at<float>(ws, Ly.part_m),
                                                at<float>(ws, Ly.part_s), at<float>(ws, Ly.best_s),

@@ -213,22 +213,45 @@ __device__ __forceinline__ float merge_lse(const float* __restrict__ pm, const f
   return (m + __log2f(s)) * 0.6931471805599453f;
 }
 
-// logp_out[t] for every row (0 on padding and on rows with a bad target).
+// merge_lse by one warp, the same value in every lane, bit for bit: the max
+// in any order, the terms formed in parallel and summed in split order (each
+// lane's term added in turn through a shuffle), so that a row's splits are
+// read at once instead of one after another (a decode step has few rows and
+// up to ~300 splits each).
+__device__ __forceinline__ float merge_lse_warp(const float* __restrict__ pm, const float* __restrict__ ps,
+                                                int nsplit, long ldp, int r, int lane) {
+  float m = -INFINITY;
+  for (int j = lane; j < nsplit; j += 32) m = fmaxf(m, pm[j * ldp + r]);
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
+  float s = 0.f;
+  for (int j0 = 0; j0 < nsplit; j0 += 32) {
+    const int j = j0 + lane;
+    const float term = j < nsplit ? __fmul_rn(ps[j * ldp + r], fast_exp2(pm[j * ldp + r] - m)) : 0.f;
+    const int n = min(32, nsplit - j0);
+    for (int k = 0; k < n; ++k) s = __fadd_rn(s, __shfl_sync(0xffffffffu, term, k));
+  }
+  return (m + __log2f(s)) * 0.6931471805599453f;
+}
+
+// logp_out[t] for every row (0 on padding and on rows with a bad target); one
+// warp per row.
 __global__ void logp_merge_kernel(const uint8_t* __restrict__ mask, const int* __restrict__ rank_of,
                                   int64_t T, const float* __restrict__ pm, const float* __restrict__ ps,
                                   int nsplit, long ldp, const float* __restrict__ zy,
                                   const int* __restrict__ yc, float* __restrict__ logp_out,
                                   unsigned* status) {
-  for (int64_t t = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; t < T;
-       t += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+  const int lane = threadIdx.x & 31;
+  const int64_t warps = (static_cast<int64_t>(gridDim.x) * blockDim.x) >> 5;
+  for (int64_t t = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5; t < T; t += warps) {
     float out = 0.f;
     const int r = mask[t] ? rank_of[t] : -1;
     if (r >= 0) {
-      const float lse = merge_lse(pm, ps, nsplit, ldp, r);
-      if (!isfinite(lse)) atomicOr(status, kDevNonFinite);
+      const float lse = merge_lse_warp(pm, ps, nsplit, ldp, r, lane);
+      if (lane == 0 && !isfinite(lse)) atomicOr(status, kDevNonFinite);
       out = yc[r] >= 0 ? zy[r] - lse : 0.f;
     }
-    logp_out[t] = out;
+    if (lane == 0) logp_out[t] = out;
   }
 }
 
@@ -260,27 +283,42 @@ __global__ void sample_merge_kernel(const uint8_t* __restrict__ mask, const int*
                                     const float* __restrict__ bs, const int* __restrict__ bc,
                                     const float* __restrict__ bz, int nsplit, long ldp,
                                     int32_t* __restrict__ tokens, float* __restrict__ logp, unsigned* status) {
-  for (int64_t t = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; t < T;
-       t += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+  // one warp per row: the best score over the splits (the lowest split on a tie), then the LSE
+  const int lane = threadIdx.x & 31;
+  const int64_t warps = (static_cast<int64_t>(gridDim.x) * blockDim.x) >> 5;
+  for (int64_t t = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5; t < T; t += warps) {
     int tok = -1;
     float lp = 0.f;
     const int r = mask[t] ? rank_of[t] : -1;
     if (r >= 0) {
-      float best = -INFINITY, z = 0.f;
-      for (int j = 0; j < nsplit; ++j) {
+      float best = -INFINITY;
+      int jb = nsplit;
+      for (int j = lane; j < nsplit; j += 32) {
         const float sc = bs[j * ldp + r];
-        if (sc > best) {
+        if (sc > best) {  // a lane's splits in increasing order: its lowest on a tie
           best = sc;
-          tok = bc[j * ldp + r];
-          z = bz[j * ldp + r];
+          jb = j;
         }
       }
-      const float lse = merge_lse(pm, ps, nsplit, ldp, r);
-      if (!isfinite(lse) || tok < 0) atomicOr(status, kDevNonFinite);
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) {
+        const float ob = __shfl_xor_sync(0xffffffffu, best, o);
+        const int oj = __shfl_xor_sync(0xffffffffu, jb, o);
+        if (ob > best || (ob == best && oj < jb)) {
+          best = ob;
+          jb = oj;
+        }
+      }
+      const float z = jb < nsplit ? bz[jb * ldp + r] : 0.f;
+      tok = jb < nsplit ? bc[jb * ldp + r] : -1;
+      const float lse = merge_lse_warp(pm, ps, nsplit, ldp, r, lane);
+      if (lane == 0 && (!isfinite(lse) || tok < 0)) atomicOr(status, kDevNonFinite);
       lp = z - lse;
     }
-    tokens[t] = tok;
-    logp[t] = lp;
+    if (lane == 0) {
+      tokens[t] = tok;
+      logp[t] = lp;
+    }
   }
 }
 
