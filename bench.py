@@ -41,7 +41,10 @@ KERNEL_SOURCES = ["paper_2507_05687_gb300/csrc/gemm_tc.cuh", "paper_2507_05687_g
                   "paper_2507_05687_gb300/csrc/gemm_launch.cuh", "paper_2507_05687_gb300/csrc/dz_rows.cuh"]
 KIND_NAMES = ["advantages", "compact", "lse_gemm", "logp_merge", "loss", "dz_gemm", "dh_gemm", "dw_gemm",
               "dh_rows", "adamw", "sample_gemm", "transpose", "dz_logits", "top_p"]
-KERNELS_PER_SCOPE = {1: 4, 4: 2}  # compaction scope = 4 kernels, loss scope = 2 kernels; others 1
+# kernels per traced scope: compaction 4 (2 for batches of at most 4096 rows, whose mask
+# count, scan and scatter run as one block), loss 2; others 1
+KERNELS_PER_SCOPE = {1: 4, 4: 2}
+SMALL_COMPACTION_ROWS = 4096
 
 
 def parse():
@@ -523,7 +526,10 @@ def main():
     kms = (ctypes.c_float * nrec)()
     lib.grpo_trace_read(kinds, cols, kms, nrec)
     trace = [(kinds[i], cols[i], kms[i]) for i in range(nrec)]
-    launches = sum(KERNELS_PER_SCOPE.get(k, 1) for k, _, _ in trace)
+    per_scope = dict(KERNELS_PER_SCOPE)
+    if w.T <= SMALL_COMPACTION_ROWS:
+        per_scope[1] = 2
+    launches = sum(per_scope.get(k, 1) for k, _, _ in trace)
     st = grpo.check_device_status(ws)
     if st != grpo.GRPO_OK:
         raise SystemExit(f"device status after timing: {grpo.status_string(st)}")

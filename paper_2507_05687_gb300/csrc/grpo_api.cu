@@ -513,7 +513,10 @@ cudaError_t run_compaction(const uint16_t* H, const int32_t* targets, const uint
   cudaError_t e = cudaMemsetAsync(status, 0, 8, s);  // status word and n_valid
   if (e != cudaSuccess) return e;
   TraceScope trace(GRPO_K_COMPACT, 0, s);
-  if (T > 0) {
+  if (T > 0 && T <= kScanChunk) {  // one block does all three steps
+    mask_compact_small_kernel<<<1, kScanThreads, 0, s>>>(mask, T, static_cast<int>(Ly.rows), n_valid,
+                                                         at<int>(ws, Ly.cidx), at<int>(ws, Ly.rank_of), status);
+  } else if (T > 0) {
     const int nb = static_cast<int>(Ly.nblk_scan);
     mask_count_kernel<<<nb, kScanThreads, 0, s>>>(mask, T, at<int>(ws, Ly.counts));
     count_scan_kernel<<<1, 1024, 0, s>>>(at<int>(ws, Ly.counts), nb, at<int>(ws, Ly.offsets), n_valid,

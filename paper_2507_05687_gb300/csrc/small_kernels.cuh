@@ -13,6 +13,7 @@ namespace grpo {
 
 constexpr int kScanChunk = 4096;   // tokens per block in the compaction kernels
 constexpr int kScanThreads = 256;  // 16 tokens per thread
+static_assert(kScanChunk == kScanThreads * 16, "one chunk per block of the compaction kernels");
 
 // ------------------------------------------------------------------ Eq. 2
 
@@ -150,6 +151,43 @@ __global__ void mask_scatter_kernel(const uint8_t* __restrict__ mask, int64_t T,
         rank_of[t] = -1;
       }
     }
+  }
+}
+
+// The three kernels above in one block, for batches of at most kScanChunk
+// rows (a decode step): the same cidx, rank_of, n_valid and capacity status,
+// with two launches fewer.
+__global__ void mask_compact_small_kernel(const uint8_t* __restrict__ mask, int64_t T, int cap,
+                                          int* __restrict__ n_valid, int* __restrict__ cidx,
+                                          int* __restrict__ rank_of, unsigned* status) {
+  __shared__ int sh[32];
+  const int64_t base = static_cast<int64_t>(threadIdx.x) * 16;
+  uint32_t bits = 0;
+  int c = 0;
+#pragma unroll
+  for (int j = 0; j < 16; ++j) {
+    const bool m = base + j < T && mask[base + j] != 0;
+    bits |= (m ? 1u : 0u) << j;
+    c += m ? 1 : 0;
+  }
+  int total;
+  int pos = block_exclusive_scan(c, sh, &total);
+#pragma unroll
+  for (int j = 0; j < 16; ++j) {
+    const int64_t t = base + j;
+    if (t < T) {
+      if (bits & (1u << j)) {
+        if (pos < cap) cidx[pos] = static_cast<int>(t);
+        rank_of[t] = pos < cap ? pos : -1;
+        ++pos;
+      } else {
+        rank_of[t] = -1;
+      }
+    }
+  }
+  if (threadIdx.x == 0) {
+    *n_valid = min(total, cap);
+    if (total > cap) atomicOr(status, kDevCapacity);
   }
 }
 
