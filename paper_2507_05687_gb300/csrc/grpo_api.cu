@@ -203,7 +203,7 @@ bool encode_blk(CUtensorMap* map, const void* base, uint64_t rows, uint64_t k, u
 struct DeviceInfo {
   int sms = 0;
   int pairs = 0;        // CTA pairs of the pair kernels that can be resident at once
-  int top_p_clusters[3] = {0, 0, 0};  // clusters of 2, 4, 8 CTAs of the nucleus selection resident at once
+  int top_p_clusters[4] = {0, 0, 0, 0};  // clusters of 2, 4, 8, 16 CTAs of the nucleus selection resident at once
   int fast_ctas = 0;       // CTAs of the nucleus fast pass resident at once (all SMs)
   bool ok = false;
 };
@@ -259,21 +259,34 @@ bool device_info(DeviceInfo* out) {
     // clusters: launch no more than can be resident together (a cluster must
     // fit in one GPC, so this is below SMs x CTAs per SM / cluster size)
     auto resident_clusters = [](auto kernel, int cluster) {
+      if (cluster > 8 &&
+          cudaFuncSetAttribute(kernel, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) != cudaSuccess) {
+        cudaGetLastError();
+        return 0;
+      }
+      cudaLaunchAttribute attr[1];
+      attr[0].id = cudaLaunchAttributeClusterDimension;
+      attr[0].val.clusterDim.x = cluster;
+      attr[0].val.clusterDim.y = 1;
+      attr[0].val.clusterDim.z = 1;
       cudaLaunchConfig_t cfg = {};
       cfg.gridDim = dim3(cluster * 1024, 1, 1);
       cfg.blockDim = dim3(kTopPThreads, 1, 1);
+      cfg.attrs = attr;
+      cfg.numAttrs = 1;
       int n = 0;
       if (cudaOccupancyMaxActiveClusters(&n, kernel, &cfg) != cudaSuccess) {
         cudaGetLastError();
         n = 0;
       }
-      return std::max(n, 1);
+      return n;
     };
     cache[dev].sms = sms;
     cache[dev].pairs = std::max(pairs, 0);
     cache[dev].top_p_clusters[0] = resident_clusters(top_p_kernel<2>, 2);
     cache[dev].top_p_clusters[1] = resident_clusters(top_p_kernel<4>, 4);
     cache[dev].top_p_clusters[2] = resident_clusters(top_p_kernel<8>, 8);
+    cache[dev].top_p_clusters[3] = resident_clusters(top_p_kernel<16>, 16);  // 0: not available
     // the nucleus fast pass streams the stored logits through a shared-memory
     // ring (kFastSmem bytes); its grid is what can be resident at once
     int per_sm = 0;
@@ -867,22 +880,39 @@ grpo_status grpo_sample_tokens_top_p(const uint16_t* H, const uint16_t* W, const
             at<unsigned>(ws, Ly.status));
       // the rows whose winner falls outside: clusters of 2, 4 or 8 CTAs, one
       // row per cluster at a time, as many clusters as can be resident together
-      const int lg = top_p_cluster_log2(Ly.rows, top_p);
+      int lg = top_p_cluster_log2(Ly.rows, top_p);
+      while (lg > 1 && di.top_p_clusters[lg - 1] <= 0) --lg;  // a size this device cannot place
       const int64_t clusters = std::max<int64_t>(1, std::min<int64_t>(Ly.rows, di.top_p_clusters[lg - 1]));
       const int rb = static_cast<int>(clusters << lg);
       auto select = [&](auto kernel) {
-        kernel<<<rb, kTopPThreads, 0, s>>>(
-            at<float>(ws, Ly.z), Ly.ldz, static_cast<int>(V), reinterpret_cast<const int*>(n_slow),
-            at<int>(ws, Ly.slow_rows), at<unsigned long long>(ws, Ly.slow_tgt), at<int>(ws, Ly.cidx), lse_r, y0_r,
-            hi_r, at<float>(ws, Ly.best_s), at<int>(ws, Ly.best_c), at<float>(ws, Ly.best_z),
-            static_cast<int>(Ly.nsplit), Ly.rows, Ly.lse_tiles, 1.f / temperature, static_cast<uint32_t>(seed),
+        cudaLaunchAttribute attr[1];
+        attr[0].id = cudaLaunchAttributeClusterDimension;
+        attr[0].val.clusterDim.x = 1u << lg;
+        attr[0].val.clusterDim.y = 1;
+        attr[0].val.clusterDim.z = 1;
+        cudaLaunchConfig_t cfg = {};
+        cfg.gridDim = dim3(static_cast<unsigned>(rb), 1, 1);
+        cfg.blockDim = dim3(kTopPThreads, 1, 1);
+        cfg.stream = s;
+        cfg.attrs = attr;
+        cfg.numAttrs = 1;
+        return cudaLaunchKernelEx(
+            &cfg, kernel, at<float>(ws, Ly.z), Ly.ldz, static_cast<int>(V), reinterpret_cast<const int*>(n_slow),
+            static_cast<const int*>(at<int>(ws, Ly.slow_rows)),
+            static_cast<const unsigned long long*>(at<unsigned long long>(ws, Ly.slow_tgt)),
+            static_cast<const int*>(at<int>(ws, Ly.cidx)), static_cast<const float*>(lse_r),
+            static_cast<const float*>(y0_r), static_cast<const float*>(hi_r),
+            static_cast<const float*>(at<float>(ws, Ly.best_s)), static_cast<const int*>(at<int>(ws, Ly.best_c)),
+            static_cast<const float*>(at<float>(ws, Ly.best_z)), static_cast<int>(Ly.nsplit),
+            static_cast<long>(Ly.rows), Ly.lse_tiles, 1.f / temperature, static_cast<uint32_t>(seed),
             static_cast<uint32_t>(seed >> 32), static_cast<uint32_t>(offset), static_cast<uint32_t>(offset >> 32),
             tokens_out, logp_out, at<unsigned>(ws, Ly.status));
       };
       if (e == cudaSuccess) {
-        if (lg == 1) select(top_p_kernel<2>);
-        else if (lg == 2) select(top_p_kernel<4>);
-        else select(top_p_kernel<8>);
+        if (lg == 1) e = select(top_p_kernel<2>);
+        else if (lg == 2) e = select(top_p_kernel<4>);
+        else if (lg == 3) e = select(top_p_kernel<8>);
+        else e = select(top_p_kernel<16>);
       }
       if (e == cudaSuccess) e = cudaGetLastError();
     }

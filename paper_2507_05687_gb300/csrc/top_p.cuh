@@ -55,14 +55,14 @@
 namespace grpo {
 
 constexpr int kTopPThreads = 256;
-constexpr int kTopPCtas = 8;       // most CTAs of a cluster sharing one row (clusters of 2, 4 or 8)
+constexpr int kTopPCtas = 16;      // most CTAs of a cluster sharing one row (clusters of 2, 4, 8 or 16)
 constexpr int kTopPBuckets = 2048;
 constexpr int kTopPCand = 1024;    // candidates resolved exactly in shared memory
 constexpr int kTopPLevels = 6;     // histogram levels before the candidates fit
 constexpr int kTopPWarps = kTopPThreads / 32;
 // column halves of a tile in the sampling GEMM's split entries (one per epilogue warp of a lane quarter)
 constexpr int kSampleHalves = EpiShape<kEpiSample>::kHalves;
-static_assert(kTopPBuckets % (kTopPCtas * kTopPThreads) == 0, "whole histogram buckets per thread in the merge");
+static_assert(kTopPBuckets % kTopPCtas == 0, "whole histogram slices per CTA in the merge");
 
 // Shared memory of one CTA.  The fields marked "host" are used in CTA 0 of
 // the cluster only (the other CTAs write into and read from CTA 0's copy).
@@ -226,8 +226,10 @@ __device__ __forceinline__ float top_p_rank_slice(TopPShared& sh, int nc, int ra
   return top_p_block_max(sh, best);
 }
 
+// Launched in clusters of kC CTAs (the launch sets the cluster shape; 16 is a
+// non-portable size the launch enables).
 template <int kC>
-__global__ void __cluster_dims__(kC, 1, 1) __launch_bounds__(kTopPThreads, 4)
+__global__ void __launch_bounds__(kTopPThreads, 4)
     top_p_kernel(const float* __restrict__ z, int64_t ldz, int V, const int* __restrict__ n_slow,
                  const int* __restrict__ slow_rows, const unsigned long long* __restrict__ slow_target,
                  const int* __restrict__ cidx, const float* __restrict__ lse_r, const float* __restrict__ y0_r,
@@ -285,14 +287,14 @@ __global__ void __cluster_dims__(kC, 1, 1) __launch_bounds__(kTopPThreads, 4)
         });
       }
       cluster_sync();
-      {  // merge the histograms: CTA k sums its slice of kMerge * kTopPThreads buckets over the
-         // cluster in rank order into its own histogram (only CTA k reads the buckets of slice k,
-         // so no CTA reads a bucket another one writes) and sends the slice's total to every CTA
-        constexpr int kMerge = kTopPBuckets / (kC * kTopPThreads);
+      {  // merge the histograms: CTA k sums its slice of kSlice buckets over the cluster in rank
+         // order into its own histogram (only CTA k reads the buckets of slice k, so no CTA reads
+         // a bucket another one writes) and sends the slice's total to every CTA
+        constexpr int kSlice = kTopPBuckets / kC;
         unsigned long long t = 0ull;
 #pragma unroll
-        for (int j = 0; j < kMerge; ++j) {
-          const int b = (rank * kMerge + j) * kTopPThreads + tid;
+        for (int p = tid; p < kSlice; p += kTopPThreads) {
+          const int b = rank * kSlice + p;
           unsigned long long part[kC];
 #pragma unroll
           for (int k = 0; k < kC; ++k) part[k] = ld_shared_cluster_u64(atk(&sh.hist[b], k));
@@ -337,14 +339,16 @@ __global__ void __cluster_dims__(kC, 1, 1) __launch_bounds__(kTopPThreads, 4)
         before -= sh.tot[kC - 1];
       }
       if (rank == cs) {  // the bucket within this slice, by block scans of kTopPThreads buckets at a time
-        constexpr int kMerge = kTopPBuckets / (kC * kTopPThreads);
+        constexpr int kSlice = kTopPBuckets / kC;
         const int lane = tid & 31, warp = tid >> 5;
         unsigned long long acc = before;
         int found = -1;
         unsigned long long found_cum = 0ull;
-        for (int j = 0; j < kMerge && found < 0; ++j) {
-          const int b = (rank * kMerge + j) * kTopPThreads + tid;
-          const unsigned long long v = sh.hist[b];
+        for (int p0 = 0; p0 < kSlice && found < 0; p0 += kTopPThreads) {
+          // positions past the slice (a slice shorter than the block) add nothing, so the
+          // first crossing, if the round has one, is inside the slice
+          const int b = rank * kSlice + p0 + tid;
+          const unsigned long long v = p0 + tid < kSlice ? sh.hist[b] : 0ull;
           unsigned long long inc = v;
 #pragma unroll
           for (int o = 1; o < 32; o <<= 1) {
@@ -371,18 +375,20 @@ __global__ void __cluster_dims__(kC, 1, 1) __launch_bounds__(kTopPThreads, 4)
               break;
             }
           if (first < kTopPThreads) {
-            found = (rank * kMerge + j) * kTopPThreads + first;
+            found = rank * kSlice + p0 + first;
             if (tid == first) found_cum = acc + inc - v;  // the mass above the bucket
           } else {
             acc += all;
           }
         }
+        // the thread that holds the bucket (its position in its round) sends it and the mass
+        // above it to every CTA
+        const int holder_of_last = (kSlice - 1) % kTopPThreads;
         if (found < 0) {  // no crossing in the last slice: its last bucket (only at a deeper level)
-          found = (rank * kMerge + kMerge - 1) * kTopPThreads + kTopPThreads - 1;
-          if (tid == kTopPThreads - 1) found_cum = acc - sh.hist[found];
+          found = rank * kSlice + kSlice - 1;
+          if (tid == holder_of_last) found_cum = acc - sh.hist[found];
         }
-        // the thread that holds the bucket sends it and the mass above it to every CTA
-        const int holder = found - (found / kTopPThreads) * kTopPThreads;
+        const int holder = (found - rank * kSlice) % kTopPThreads;
         if (tid == holder) {
           for (int k = 0; k < kC; ++k) {
             st_shared_cluster(atk(&sh.lvl_b[L], k), static_cast<uint32_t>(found));
@@ -705,8 +711,8 @@ static_assert(kFastChunk % (kTopPWarps * 128) == 0, "whole float4 rounds per war
 // The bound on |A - E| above for a vocabulary of V, in units of 2^-40.
 inline unsigned long long top_p_margin(int64_t V) { return (1ull << 23) + 2ull * static_cast<unsigned long long>(V); }
 
-// log2 of the cluster size of the selection (1, 2 or 3: clusters of 2, 4 or
-// 8 CTAs) for a draw over up to `rows` rows.  About a fraction 1 - top_p of
+// log2 of the cluster size of the selection (1 to 4: clusters of 2, 4, 8 or
+// 16 CTAs) for a draw over up to `rows` rows.  About a fraction 1 - top_p of
 // the rows are listed (the winner falls outside its nucleus that often).  A
 // cluster takes one listed row at a time, so few listed rows want large
 // clusters (each row done sooner, while about 74 clusters of 8 fit on a
@@ -716,16 +722,18 @@ inline unsigned long long top_p_margin(int64_t V) { return (1ull << 23) + 2ull *
 // 2, at 0.5 [166] 0.43 / 0.42 / 0.46; 2048 rows at 0.9 [266] 1.96-2.06 /
 // 1.96-2.10 / 2.03-2.11, at 0.5 [1331] 2.59 / 2.48 / 2.46; 19,572 of 32,768
 // rows at 0.5 [21299] 24.7-24.9 / 24.3-24.7 / 23.4-24.1 ms.  GRPO_TOP_P_CLUSTER=2|4|8
-// overrides the choice.
+// overrides the choice (16: one round of rows for a decode step's few
+// listed rows, each walked by twice as many CTAs).
 inline int top_p_cluster_log2(int64_t rows, float top_p) {
   if (const char* e = std::getenv("GRPO_TOP_P_CLUSTER")) {
     const int c = std::atoi(e);
     if (c == 2) return 1;
     if (c == 4) return 2;
     if (c == 8) return 3;
+    if (c == 16) return 4;
   }
   const double listed = static_cast<double>(rows) * (1.0 - static_cast<double>(top_p)) * 1.3;
-  return listed <= 100.0 ? 3 : listed <= 400.0 ? 2 : 1;
+  return listed <= 36.0 ? 4 : listed <= 100.0 ? 3 : listed <= 400.0 ? 2 : 1;
 }
 
 __global__ void __launch_bounds__(kTopPThreads, 2)

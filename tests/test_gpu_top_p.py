@@ -238,7 +238,7 @@ def test_every_row_listed_gives_the_same_draws(monkeypatch, top_p):
 
 @pytest.mark.parametrize("top_p", [0.9, 0.5])
 def test_cluster_size_gives_the_same_draws(monkeypatch, top_p):
-    """The selection takes each listed row in a cluster of 8, 4 or 2 CTAs
+    """The selection takes each listed row in a cluster of 16, 8, 4 or 2 CTAs
     (chosen by the expected number of listed rows); the histogram merge, the
     candidate split of the threshold search and the draw's entry split all
     change with the size, and every reduction in them is exact or has a total
@@ -254,10 +254,10 @@ def test_cluster_size_gives_the_same_draws(monkeypatch, top_p):
         for list_all in ("0", "1"):
             monkeypatch.setenv("GRPO_TEST_TOP_P_LIST_ALL", list_all)
             got = {}
-            for c in ("8", "4", "2"):
+            for c in ("8", "16", "4", "2"):
                 monkeypatch.setenv("GRPO_TOP_P_CLUSTER", c)
                 got[c] = _draw(Hb, Wb, m, 1.0, top_p, 91, 3)
-            for c in ("4", "2"):
+            for c in ("16", "4", "2"):
                 assert np.array_equal(got[c][0], got["8"][0]) and np.array_equal(got[c][1], got["8"][1]), (w.V, c)
     monkeypatch.delenv("GRPO_TOP_P_CLUSTER")
     monkeypatch.delenv("GRPO_TEST_TOP_P_LIST_ALL")
