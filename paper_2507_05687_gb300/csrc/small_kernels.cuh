@@ -242,33 +242,53 @@ __global__ void resp_len_kernel(const uint8_t* __restrict__ mask, int64_t n_resp
 // ------------------------------------------------------------------ merge + loss
 
 // log-sum-exp of row r from the per-split partials (log2 units inside).
+// The log-sum-exp of a row from its splits' running (max, sum) pairs:
+// m = the largest max, s = the sum over splits j of ps_j 2^(pm_j - m), in one
+// fixed order that a thread and a warp reach alike: 32 partial sums (partial l
+// over the splits j = l, l + 32, ... in increasing j), then a butterfly over
+// the partials (l + l^16 for l < 16, then l + l^8 for l < 8, ...).  Every
+// merge of the same splits (log-probs, loss, sampling, the nucleus draw) gets
+// the same bits.
+__device__ __forceinline__ float split_term(const float* __restrict__ pm, const float* __restrict__ ps, long at,
+                                            float m) {
+  return __fmul_rn(ps[at], fast_exp2(pm[at] - m));
+}
+
 __device__ __forceinline__ float merge_lse(const float* __restrict__ pm, const float* __restrict__ ps,
                                            int nsplit, long ldp, int r) {
   float m = -INFINITY;
   for (int j = 0; j < nsplit; ++j) m = fmaxf(m, pm[j * ldp + r]);
-  float s = 0.f;  // explicitly rounded, so that other merges of the same splits can match it bit for bit
-  for (int j = 0; j < nsplit; ++j) s = __fadd_rn(s, __fmul_rn(ps[j * ldp + r], fast_exp2(pm[j * ldp + r] - m)));
-  return (m + __log2f(s)) * 0.6931471805599453f;
+  float p[32];
+#pragma unroll
+  for (int l = 0; l < 32; ++l) p[l] = 0.f;
+  for (int j0 = 0; j0 < nsplit; j0 += 32) {
+#pragma unroll
+    for (int l = 0; l < 32; ++l)
+      if (j0 + l < nsplit) p[l] = __fadd_rn(p[l], split_term(pm, ps, (j0 + l) * ldp + r, m));
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+#pragma unroll
+    for (int l = 0; l < o; ++l) p[l] = __fadd_rn(p[l], p[l + o]);
+  }
+  return (m + __log2f(p[0])) * 0.6931471805599453f;
 }
 
-// merge_lse by one warp, the same value in every lane, bit for bit: the max
-// in any order, the terms formed in parallel and summed in split order (each
-// lane's term added in turn through a shuffle), so that a row's splits are
-// read at once instead of one after another (a decode step has few rows and
-// up to ~300 splits each).
+// merge_lse by one warp, the same value in every lane, bit for bit (lane l
+// holds partial l; the butterfly runs over shuffles), with a row's splits read
+// at once instead of one after another (a decode step has few rows and up to
+// ~300 splits each).  Also returns the row's max m.
 __device__ __forceinline__ float merge_lse_warp(const float* __restrict__ pm, const float* __restrict__ ps,
-                                                int nsplit, long ldp, int r, int lane) {
+                                                int nsplit, long ldp, int r, int lane, float* m_out = nullptr) {
   float m = -INFINITY;
   for (int j = lane; j < nsplit; j += 32) m = fmaxf(m, pm[j * ldp + r]);
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
   float s = 0.f;
-  for (int j0 = 0; j0 < nsplit; j0 += 32) {
-    const int j = j0 + lane;
-    const float term = j < nsplit ? __fmul_rn(ps[j * ldp + r], fast_exp2(pm[j * ldp + r] - m)) : 0.f;
-    const int n = min(32, nsplit - j0);
-    for (int k = 0; k < n; ++k) s = __fadd_rn(s, __shfl_sync(0xffffffffu, term, k));
-  }
+  for (int j = lane; j < nsplit; j += 32) s = __fadd_rn(s, split_term(pm, ps, j * ldp + r, m));
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) s = __fadd_rn(s, __shfl_xor_sync(0xffffffffu, s, o));
+  if (m_out) *m_out = m;
   return (m + __log2f(s)) * 0.6931471805599453f;
 }
 

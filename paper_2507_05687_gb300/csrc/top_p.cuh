@@ -616,7 +616,7 @@ __global__ void __launch_bounds__(kTopPThreads, 4)
 // to the outputs (the nucleus selection replaces it only where the winner
 // falls outside the nucleus), and the row's LSE, winner's y and maximum y kept
 // for the selection (whose per-row accumulators it clears).  One warp per row reads the splits in parallel; the LSE
-// sum runs in split order with merge_lse's rounding, and the winner is the best
+// is merge_lse's (merge_lse_warp), and the winner is the best
 // score with the lowest split on a tie, as sample_merge_kernel takes them, so
 // the draw is the plain sampler's bit for bit.
 __global__ void top_p_prep_kernel(const int* __restrict__ n_valid, const int* __restrict__ cidx,
@@ -632,10 +632,9 @@ __global__ void top_p_prep_kernel(const int* __restrict__ n_valid, const int* __
   const int warps = static_cast<int>((static_cast<int64_t>(gridDim.x) * blockDim.x) >> 5);
   for (int r = static_cast<int>((static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5); r < nv;
        r += warps) {
-    float m = -INFINITY, best = -INFINITY;
+    float best = -INFINITY;
     int jb = nsplit;
     for (int j = lane; j < nsplit; j += 32) {
-      m = fmaxf(m, pm[j * ldp + r]);
       const float sc = bs[j * ldp + r];
       if (sc > best) {
         best = sc;
@@ -644,7 +643,6 @@ __global__ void top_p_prep_kernel(const int* __restrict__ n_valid, const int* __
     }
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) {
-      m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
       const float ob = __shfl_xor_sync(0xffffffffu, best, o);
       const int oj = __shfl_xor_sync(0xffffffffu, jb, o);
       if (ob > best || (ob == best && oj < jb)) {
@@ -652,15 +650,9 @@ __global__ void top_p_prep_kernel(const int* __restrict__ n_valid, const int* __
         jb = oj;
       }
     }
-    float s = 0.f;
-    for (int j0 = 0; j0 < nsplit; j0 += 32) {
-      const int j = j0 + lane;
-      const float term = j < nsplit ? __fmul_rn(ps[j * ldp + r], fast_exp2(pm[j * ldp + r] - m)) : 0.f;
-      const int n = min(32, nsplit - j0);
-      for (int k = 0; k < n; ++k) s = __fadd_rn(s, __shfl_sync(0xffffffffu, term, k));
-    }
+    float m;
+    const float lse = merge_lse_warp(pm, ps, nsplit, ldp, r, lane, &m);
     if (lane == 0) {
-      const float lse = (m + __log2f(s)) * kLn2;
       const int tok = jb < nsplit ? bc[jb * ldp + r] : -1;
       const float y0 = jb < nsplit ? bz[jb * ldp + r] : 0.f;
       if (!isfinite(lse) || tok < 0) atomicOr(status, kDevNonFinite);
