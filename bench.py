@@ -558,13 +558,15 @@ def main():
         step_exec = (6.0 if args.logits == "keep" else 8.0) * n_valid * w.Hd * w.V
         step_model = 6.0 * n_valid * w.Hd * w.V
 
-    e2e = e2e_offload = None
+    e2e = e2e_offload = e2e_staged = None
     if not args.no_e2e and not sampling:
         if scoring:
             e2e = measure_e2e_scoring(grpo, torch, dev, w, inp, heads, steps=args.e2e_steps, dist=dist)
         else:
             # the step's own workspace: a second one of the same size may not fit beside it
             e2e = measure_e2e(grpo, torch, dev, w, inp, steps=args.e2e_steps, dist=dist, ws=ws)
+            if dist is None:
+                e2e_staged = measure_e2e_staged(grpo, torch, dev, w, inp, steps=args.e2e_steps, ws=ws)
             if world == 1:
                 e2e_offload = measure_e2e_offload(grpo, torch, dev, w, inp, steps=args.e2e_steps, ws=ws)
 
@@ -613,6 +615,8 @@ def main():
         }
         if e2e_offload is not None:
             line["e2e_offload"] = e2e_offload
+        if e2e_staged is not None:
+            line["e2e_staged"] = e2e_staged
         if kept is not None:
             line["kept_logits_ms_per_step"] = kept.get("ms_per_step")
             line["kept_logits"] = kept
@@ -777,6 +781,48 @@ def measure_e2e(grpo, torch, dev, w, inp, steps: int, dist=None, ws=None):
             "what": "H read from pinned host memory by the row gather each step (the unmasked rows cross the "
                     "host link); targets, mask, old/ref log-probs, rewards copied; W resident on the device; the "
                     "loss read back; dH, dW left on the device"}
+
+
+def measure_e2e_staged(grpo, torch, dev, w, inp, steps: int, ws=None):
+    """The training step of measure_e2e fed through staging.BatchStager: each
+    step's whole batch (every row of H, targets, mask, old / ref log-probs,
+    rewards) is copied from pinned host memory into a device slot on a copy
+    stream while the previous step computes; the step waits for its batch's
+    copies, runs on the device tensors and reads the loss back."""
+    from paper_2507_05687_gb300.staging import BatchStager
+    n_valid = int(inp["m"].sum())
+
+    def pin(a, dt):
+        return torch.from_numpy(np.ascontiguousarray(a)).view(dt).pin_memory()
+
+    Wd = torch.from_numpy(np.ascontiguousarray(inp["W"])).view(torch.bfloat16).to(dev)
+    batch = (pin(inp["H"], torch.bfloat16), pin(inp["y"], torch.int32), pin(inp["m"], torch.uint8),
+             pin(inp["old"], torch.float32), pin(inp["ref"], torch.float32), pin(inp["r"], torch.float32))
+    h2d = sum(t.numel() * t.element_size() for t in batch)
+    out = (torch.empty(1, dtype=torch.float32, device=dev), torch.empty(w.T, w.Hd, dtype=torch.float32, device=dev),
+           torch.empty(w.V, w.Hd, dtype=torch.float32, device=dev))
+    if ws is None:
+        ws = grpo.loss_workspace(w.T, w.Hd, w.V, dev, max_valid=n_valid)
+    stager = BatchStager(dev)
+    stager.submit(batch)
+
+    def one():
+        H, y, m, old, ref, r = stager.get()
+        stager.submit(batch)  # the next step's batch (the same synthetic arrays), copied while this one runs
+        adv = grpo.group_advantages(r, w.G, w.adv_eps)
+        loss, _, _ = grpo.loss_fwd_bwd(H, Wd, y, m, old, ref, adv, w.n_resp, w.L, w.clip_eps, w.beta, ws=ws, out=out)
+        stager.release()
+        return loss.item()
+
+    one()
+    torch.cuda.synchronize(dev)
+    med, mean = timed_steps(one, steps)
+    return {"value": round(n_valid / med, 1), "unit": "tokens/s", "ms_per_step": round(med * 1e3, 2),
+            "ms_mean": round(mean * 1e3, 2), "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": 4,
+            "steps": steps, "statistic": "median of per-step wall-clock times",
+            "what": "the whole batch copied from pinned host memory each step on a copy stream while the previous "
+                    "step computes (staging.BatchStager, two device slots); the step waits for its copies; W "
+                    "resident; the loss read back"}
 
 
 def measure_e2e_offload(grpo, torch, dev, w, inp, steps: int, ws=None):
