@@ -512,7 +512,12 @@ const uint16_t* hidden_view(const uint16_t* H) {
     cudaGetLastError();
     return nullptr;
   }
-  if (pa.type == cudaMemoryTypeHost) return static_cast<const uint16_t*>(pa.devicePointer);
+  if (pa.type == cudaMemoryTypeHost) {
+    if (!pa.devicePointer) return nullptr;
+    // the device address of H itself, whether the attributes describe H or its allocation's start
+    const ptrdiff_t off = pa.hostPointer ? reinterpret_cast<const char*>(H) - static_cast<const char*>(pa.hostPointer) : 0;
+    return reinterpret_cast<const uint16_t*>(static_cast<const char*>(pa.devicePointer) + off);
+  }
   if (pa.type == cudaMemoryTypeUnregistered) return nullptr;
   return H;
 }

@@ -60,6 +60,19 @@ def test_host_hidden_states_give_the_same_bits():
     assert torch.equal(la, lb) and torch.equal(dHa, dHb) and torch.equal(dWa, dWb)
 
 
+def test_host_hidden_states_inside_a_larger_pinned_allocation():
+    """H as a view at an offset into a larger pinned buffer (the library maps the
+    address of H itself, not the allocation's start)."""
+    w = W_SMALL
+    Hb, Wb, y, m, r, Hp = _inputs(w)
+    big = torch.empty(w.T + 48, w.Hd, dtype=torch.bfloat16).pin_memory()
+    big[48:] = Hp
+    Hv = big[48:]
+    assert Hv.is_pinned() and Hv.is_contiguous() and Hv.data_ptr() != big.data_ptr()
+    Wd, yd, md = dev_tensor(Wb, torch.bfloat16), dev_tensor(y, torch.int32), dev_tensor(m, torch.uint8)
+    assert torch.equal(grpo.token_logprobs(Hv, Wd, yd, md), grpo.token_logprobs(Hp, Wd, yd, md))
+
+
 def test_pageable_host_hidden_states_are_copied_by_the_binding():
     """The binding copies pageable H to the device (the C ABI cannot read it)."""
     w = W_SMALL
