@@ -338,61 +338,58 @@ __global__ void __launch_bounds__(kTopPThreads, 4)
         cs = kC - 1;
         before -= sh.tot[kC - 1];
       }
-      if (rank == cs) {  // the bucket within this slice, by block scans of kTopPThreads buckets at a time
+      if (rank == cs) {  // the bucket within this slice: one block scan over per-thread runs of buckets
         constexpr int kSlice = kTopPBuckets / kC;
+        constexpr int kPer = (kSlice + kTopPThreads - 1) / kTopPThreads;  // consecutive buckets a thread sums
         const int lane = tid & 31, warp = tid >> 5;
-        unsigned long long acc = before;
-        int found = -1;
-        unsigned long long found_cum = 0ull;
-        for (int p0 = 0; p0 < kSlice && found < 0; p0 += kTopPThreads) {
-          // positions past the slice (a slice shorter than the block) add nothing, so the
-          // first crossing, if the round has one, is inside the slice
-          const int b = rank * kSlice + p0 + tid;
-          const unsigned long long v = p0 + tid < kSlice ? sh.hist[b] : 0ull;
-          unsigned long long inc = v;
+        const int p0 = tid * kPer;  // this thread's first position in the slice
+        unsigned long long own = 0ull;
 #pragma unroll
-          for (int o = 1; o < 32; o <<= 1) {
-            const unsigned long long n = __shfl_up_sync(0xffffffffu, inc, o);
-            if (lane >= o) inc += n;
-          }
-          __syncthreads();  // sh.ra / sh.ri of the previous round read
-          if (lane == 31) sh.ra[warp] = inc;
-          __syncthreads();
-          unsigned long long pre = 0ull, all = 0ull;
-          for (int w = 0; w < kTopPWarps; ++w) {
-            if (w < warp) pre += sh.ra[w];
-            all += sh.ra[w];
-          }
-          inc += pre;
-          const unsigned hit = __ballot_sync(0xffffffffu, acc + inc >= target);
-          __syncthreads();  // every warp has read sh.ra
-          if (lane == 0) sh.ri[warp] = hit ? __ffs(hit) - 1 : 32;
-          __syncthreads();
-          int first = kTopPThreads;
-          for (int w = 0; w < kTopPWarps; ++w)
-            if (sh.ri[w] < 32) {
-              first = w * 32 + sh.ri[w];
-              break;
-            }
-          if (first < kTopPThreads) {
-            found = rank * kSlice + p0 + first;
-            if (tid == first) found_cum = acc + inc - v;  // the mass above the bucket
-          } else {
-            acc += all;
-          }
+        for (int i = 0; i < kPer; ++i)
+          if (p0 + i < kSlice) own += sh.hist[rank * kSlice + p0 + i];
+        unsigned long long inc = own;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+          const unsigned long long n = __shfl_up_sync(0xffffffffu, inc, o);
+          if (lane >= o) inc += n;
         }
-        // the thread that holds the bucket (its position in its round) sends it and the mass
-        // above it to every CTA
-        const int holder_of_last = (kSlice - 1) % kTopPThreads;
-        if (found < 0) {  // no crossing in the last slice: its last bucket (only at a deeper level)
-          found = rank * kSlice + kSlice - 1;
-          if (tid == holder_of_last) found_cum = acc - sh.hist[found];
+        if (lane == 31) sh.ra[warp] = inc;
+        __syncthreads();
+        unsigned long long pre = 0ull, all = 0ull;
+        for (int w = 0; w < kTopPWarps; ++w) {
+          if (w < warp) pre += sh.ra[w];
+          all += sh.ra[w];
         }
-        const int holder = (found - rank * kSlice) % kTopPThreads;
-        if (tid == holder) {
+        inc += pre;
+        // the first thread whose runs reach the target holds the crossing (its runs
+        // are consecutive, so it walks them alone)
+        const unsigned hit = __ballot_sync(0xffffffffu, before + inc >= target);
+        if (lane == 0) sh.ri[warp] = hit ? __ffs(hit) - 1 : 32;
+        __syncthreads();
+        int first = kTopPThreads;
+        for (int w = 0; w < kTopPWarps; ++w)
+          if (sh.ri[w] < 32) {
+            first = w * 32 + sh.ri[w];
+            break;
+          }
+        if (tid == first) {
+          unsigned long long a = before + inc - own;  // the mass above this thread's runs
+          int b = rank * kSlice + p0;
+          for (int i = 0; i < kPer - 1 && p0 + i < kSlice - 1; ++i, ++b) {
+            if (a + sh.hist[b] >= target) break;
+            a += sh.hist[b];
+          }
           for (int k = 0; k < kC; ++k) {
-            st_shared_cluster(atk(&sh.lvl_b[L], k), static_cast<uint32_t>(found));
-            st_shared_cluster_u64(atk(&sh.cum_next, k), found_cum);
+            st_shared_cluster(atk(&sh.lvl_b[L], k), static_cast<uint32_t>(b));
+            st_shared_cluster_u64(atk(&sh.cum_next, k), a);
+          }
+        } else if (first == kTopPThreads && tid == 0) {
+          // no crossing in the last slice (only at a deeper level): its last bucket
+          const int b = rank * kSlice + kSlice - 1;
+          const unsigned long long a = before + all - sh.hist[b];
+          for (int k = 0; k < kC; ++k) {
+            st_shared_cluster(atk(&sh.lvl_b[L], k), static_cast<uint32_t>(b));
+            st_shared_cluster_u64(atk(&sh.cum_next, k), a);
           }
         }
       }
